@@ -1,0 +1,164 @@
+"""CPU oracle for region-conditional sparse retrieval (test infrastructure).
+
+TEST INFRASTRUCTURE ONLY: the tests, ``__graft_entry__.smoke()`` and the
+benchmark's CPU-baseline leg call this module; the product path never does.
+It shares no code with the CUDA library.  The arithmetic lives in
+``rcsr_oracle.c`` (fp64, plain loops, one OpenMP thread per region); this
+file only compiles it with gcc and marshals numpy arrays.
+
+Functions and what they follow:
+
+* ``region_topk``  -- Def. B.2 MIPS(q_{r_i}, D; k_r) / Eq. rcsr top-k':
+  exact per-region top-k by (score desc, id asc).
+* ``merge``        -- §3.3 / Def. B.2 / Alg. 1 Dedup of the union of the
+  per-region lists, keeping each id's max score, cut to the first K.
+* ``retrieve``     -- both steps (the CPU baseline).
+* ``score_matrix`` -- every s(r, i) in fp64 (brute force on tiny inputs).
+"""
+from __future__ import annotations
+
+import ctypes
+import os
+import subprocess
+
+import numpy as np
+
+_HERE = os.path.dirname(os.path.abspath(__file__))
+_SRC = os.path.join(_HERE, "rcsr_oracle.c")
+_OUT = os.path.join(_HERE, "_build", "libskip_oracle.so")
+_lib = None
+
+
+def build(force: bool = False) -> str:
+    """Compile the oracle with gcc (OpenMP) into oracle/_build/."""
+    if not force and os.path.exists(_OUT) and os.path.getmtime(_OUT) >= os.path.getmtime(_SRC):
+        return _OUT
+    os.makedirs(os.path.dirname(_OUT), exist_ok=True)
+    tmp = _OUT + ".tmp.%d" % os.getpid()
+    cmd = ["gcc", "-O2", "-std=c11", "-fopenmp", "-fPIC", "-shared", "-Wall", "-Wextra",
+           _SRC, "-o", tmp, "-lm"]
+    subprocess.run(cmd, check=True)
+    os.replace(tmp, _OUT)
+    return _OUT
+
+
+def _load():
+    global _lib
+    if _lib is not None:
+        return _lib
+    lib = ctypes.CDLL(build())
+    P = ctypes.c_void_p
+    i64, i32 = ctypes.c_int64, ctypes.c_int
+    lib.skip_oracle_region_topk.argtypes = [P, P, P, i64, i32, P, i64, i32, P, P, i32]
+    lib.skip_oracle_merge.argtypes = [P, P, i32, i32, P, i32, i32, P, P]
+    lib.skip_oracle_retrieve.argtypes = [P, P, P, i64, i32, P, P, i32, i64, i32, i32, P, P, P, P, i32]
+    lib.skip_oracle_score_matrix.argtypes = [P, P, P, i64, i32, P, i64, P]
+    lib.skip_oracle_bf16_value.argtypes = [ctypes.c_uint16]
+    lib.skip_oracle_bf16_value.restype = ctypes.c_double
+    lib.skip_oracle_e4m3_value.argtypes = [ctypes.c_uint8]
+    lib.skip_oracle_e4m3_value.restype = ctypes.c_double
+    for f in ("skip_oracle_region_topk", "skip_oracle_merge", "skip_oracle_retrieve",
+              "skip_oracle_score_matrix", "skip_oracle_threads"):
+        getattr(lib, f).restype = ctypes.c_int
+    _lib = lib
+    return lib
+
+
+def _ptr(a):
+    return None if a is None else a.ctypes.data_as(ctypes.c_void_p)
+
+
+def _corpus_args(corpus, row_scale):
+    """corpus: uint16 [N, d] (bf16 bits) or uint8 [N, d] (e4m3 bytes)."""
+    corpus = np.ascontiguousarray(corpus)
+    if corpus.dtype == np.uint16:
+        return corpus, None, None
+    if corpus.dtype == np.uint8:
+        if row_scale is None:
+            raise ValueError("e4m3 corpus needs row_scale")
+        return None, corpus, np.ascontiguousarray(row_scale, dtype=np.float32)
+    raise TypeError("corpus must be uint16 (bf16 bits) or uint8 (e4m3)")
+
+
+def threads() -> int:
+    return int(_load().skip_oracle_threads())
+
+
+def bf16_value(bits: int) -> float:
+    return float(_load().skip_oracle_bf16_value(int(bits)))
+
+
+def e4m3_value(byte: int) -> float:
+    return float(_load().skip_oracle_e4m3_value(int(byte)))
+
+
+def region_topk(corpus, regions, kk, row_scale=None, nthreads=0):
+    """Exact top-kk per region: (ids int64 [R, kk], scores float64 [R, kk])."""
+    lib = _load()
+    cb, ce, sc = _corpus_args(corpus, row_scale)
+    c = cb if cb is not None else ce
+    regions = np.ascontiguousarray(regions, dtype=np.uint16)
+    N, d = c.shape
+    R = regions.shape[0]
+    ids = np.empty((R, kk), dtype=np.int64)
+    sco = np.empty((R, kk), dtype=np.float64)
+    rc = lib.skip_oracle_region_topk(_ptr(cb), _ptr(ce), _ptr(sc), N, d, _ptr(regions), R, kk,
+                                     _ptr(ids), _ptr(sco), int(nthreads))
+    if rc:
+        raise RuntimeError("oracle region_topk failed (%d)" % rc)
+    return ids, sco
+
+
+def merge(reg_ids, reg_scores, k, offsets, K):
+    """Union + dedup (max score) + top-K per question: (ids [Q, K], scores [Q, K])."""
+    lib = _load()
+    reg_ids = np.ascontiguousarray(reg_ids, dtype=np.int64)
+    reg_scores = np.ascontiguousarray(reg_scores, dtype=np.float64)
+    offsets = np.ascontiguousarray(offsets, dtype=np.int32)
+    Q = offsets.shape[0] - 1
+    ld = reg_ids.shape[1] if reg_ids.ndim == 2 else k
+    out_ids = np.empty((Q, K), dtype=np.int64)
+    out_sc = np.empty((Q, K), dtype=np.float64)
+    rc = lib.skip_oracle_merge(_ptr(reg_ids), _ptr(reg_scores), ld, k, _ptr(offsets), Q, K,
+                               _ptr(out_ids), _ptr(out_sc))
+    if rc:
+        raise RuntimeError("oracle merge failed (%d)" % rc)
+    return out_ids, out_sc
+
+
+def retrieve(corpus, regions, offsets, k, K, row_scale=None, nthreads=0):
+    """Whole path: (reg_ids [R,k], reg_scores [R,k], out_ids [Q,K], out_scores [Q,K])."""
+    lib = _load()
+    cb, ce, sc = _corpus_args(corpus, row_scale)
+    c = cb if cb is not None else ce
+    regions = np.ascontiguousarray(regions, dtype=np.uint16)
+    offsets = np.ascontiguousarray(offsets, dtype=np.int32)
+    N, d = c.shape
+    R = regions.shape[0]
+    Q = offsets.shape[0] - 1
+    reg_ids = np.empty((R, k), dtype=np.int64)
+    reg_sc = np.empty((R, k), dtype=np.float64)
+    out_ids = np.empty((Q, K), dtype=np.int64)
+    out_sc = np.empty((Q, K), dtype=np.float64)
+    rc = lib.skip_oracle_retrieve(_ptr(cb), _ptr(ce), _ptr(sc), N, d, _ptr(regions), _ptr(offsets),
+                                  Q, R, k, K, _ptr(reg_ids), _ptr(reg_sc), _ptr(out_ids),
+                                  _ptr(out_sc), int(nthreads))
+    if rc:
+        raise RuntimeError("oracle retrieve failed (%d)" % rc)
+    return reg_ids, reg_sc, out_ids, out_sc
+
+
+def score_matrix(corpus, regions, row_scale=None):
+    """Every s(r, i) in fp64: [R, N]."""
+    lib = _load()
+    cb, ce, sc = _corpus_args(corpus, row_scale)
+    c = cb if cb is not None else ce
+    regions = np.ascontiguousarray(regions, dtype=np.uint16)
+    N, d = c.shape
+    R = regions.shape[0]
+    out = np.empty((R, N), dtype=np.float64)
+    rc = lib.skip_oracle_score_matrix(_ptr(cb), _ptr(ce), _ptr(sc), N, d, _ptr(regions), R,
+                                      _ptr(out))
+    if rc:
+        raise RuntimeError("oracle score_matrix failed (%d)" % rc)
+    return out

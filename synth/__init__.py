@@ -1,0 +1,226 @@
+"""Seeded synthetic inputs for region-conditional sparse retrieval (RCSR).
+
+This module is shared by the CUDA path's tests and benchmark and by the CPU
+oracle.  It only draws and quantises inputs: it holds no scoring, selection,
+merging or deduplication arithmetic.
+
+What the inputs stand in for (paper §4.1 "Knowledge corpora"/"Implementation",
+App. I.1 "Retrieval index", App. I.4 hyperparameter table): a passage corpus
+of 1.7M-109M entries with 768-dimensional index vectors (Wikipedia 6.5M,
+WikiData 8.2M, the ViQuAE KB 1.7M, Wikipedia 21M + Wikidata 88M), and per
+question up to 8 (main text) or more region query embeddings q_{r_i}
+(App. B.2, Eq. rcsr_query).  None of those corpora or trained encoders exist
+here, so rows and queries are drawn from the distributions below.
+
+Recipe (one per workload, seeds fixed per workload):
+
+* corpus seed = workload index, region seed = 1000 + workload index;
+* ``gaussian`` rows: x ~ N(0, I_d), then x / ||x||;
+* ``clustered`` rows: centres c ~ N(0, I_d) normalised; each row draws a
+  centre uniformly and sets x = normalise(c + sigma * N(0, I_d)) with
+  sigma = 0.3 / sqrt(d) per coordinate (noise norm ~0.3, cos(x, c) ~ 0.96);
+* regions of gaussian workloads: N(0, I_d) normalised;
+* regions of clustered workloads: each question picks 1..4 "entity" centres
+  uniformly from the corpus centres, each of its regions picks one of them
+  and applies the same noise model;
+* bf16 = round-to-nearest-even of the fp32 value (``torch.bfloat16``);
+* e4m3 = OCP float8_e4m3fn of x / scale_i, round-to-nearest-even, with
+  scale_i = max_j |x_ij| / 448 (1.0 for an all-zero row);
+* ragged region counts are U{lo..hi} per question from the region seed.
+
+Generation is chunked (``CHUNK`` rows per draw, each chunk with its own
+derived seed) so that multi-GB corpora can be drawn straight into device
+memory.  The same seed gives the same bytes on the same device type and
+PyTorch build; CPU- and CUDA-drawn inputs differ from each other.
+"""
+from __future__ import annotations
+
+import dataclasses
+import math
+from typing import Optional
+
+import torch
+
+CHUNK = 1 << 20  # rows per generator draw
+
+
+@dataclasses.dataclass(frozen=True)
+class WorkloadSpec:
+    name: str
+    index: int          # workload index: corpus seed, region seed = 1000 + index
+    N: int              # corpus rows
+    d: int              # embedding dimension
+    dtype: str          # "bf16" or "e4m3"
+    Q: int              # questions
+    regions: tuple      # (lo, hi) regions per question, inclusive
+    k_region: int       # per-region top-k' (paper: k', k_r)
+    K: int              # merged top-K per question
+    corpus: str         # "gaussian" or "clustered"
+    centres: int = 0    # cluster count for clustered corpora
+
+    @property
+    def fixed_regions(self) -> bool:
+        return self.regions[0] == self.regions[1]
+
+
+# The five workloads the method is measured on: a tiny exact check, a 1M
+# clustered corpus, a 10M throughput batch, a 6M fp8 latency batch and a 20M
+# ragged pruned batch.
+WORKLOADS = {
+    "tiny_100k": WorkloadSpec("tiny_100k", 0, 100_000, 768, "bf16", 4, (8, 8), 10, 20, "gaussian"),
+    "clustered_1m": WorkloadSpec("clustered_1m", 1, 1_000_000, 768, "bf16", 64, (16, 16), 20, 50,
+                                 "clustered", 1024),
+    "throughput_10m": WorkloadSpec("throughput_10m", 2, 10_000_000, 768, "bf16", 256, (16, 16), 20, 50,
+                                   "clustered", 1024),
+    "latency_fp8_6m": WorkloadSpec("latency_fp8_6m", 3, 6_000_000, 1024, "e4m3", 1, (32, 32), 10, 100,
+                                   "gaussian"),
+    "ragged_20m": WorkloadSpec("ragged_20m", 4, 20_000_000, 512, "bf16", 1024, (1, 32), 100, 100,
+                               "clustered", 4096),
+}
+
+
+@dataclasses.dataclass
+class Workload:
+    spec: WorkloadSpec
+    corpus: torch.Tensor            # [N, d] bfloat16, or uint8 holding e4m3 bytes
+    row_scale: Optional[torch.Tensor]  # [N] float32 for e4m3, else None
+    regions: torch.Tensor           # [R_total, d] bfloat16
+    offsets: torch.Tensor           # [Q + 1] int32, offsets[0] = 0
+    centres: Optional[torch.Tensor] = None  # [C, d] float32 (clustered only)
+
+    @property
+    def R_total(self) -> int:
+        return int(self.regions.shape[0])
+
+
+def _gen(seed: int, device) -> torch.Generator:
+    g = torch.Generator(device=device)
+    g.manual_seed(int(seed))
+    return g
+
+
+def _normalise(x: torch.Tensor) -> torch.Tensor:
+    n = torch.linalg.vector_norm(x, dim=1, keepdim=True)
+    return x / torch.where(n > 0, n, torch.ones_like(n))
+
+
+def draw_centres(spec_or_seed, C: int, d: int, device="cpu") -> torch.Tensor:
+    seed = spec_or_seed.index if isinstance(spec_or_seed, WorkloadSpec) else int(spec_or_seed)
+    g = _gen(seed * 7919 + 17, device)
+    return _normalise(torch.randn(C, d, generator=g, device=device, dtype=torch.float32))
+
+
+def corpus_rows_fp32(seed: int, n0: int, n: int, d: int, kind: str,
+                     centres: Optional[torch.Tensor], device="cpu") -> torch.Tensor:
+    """fp32 unit rows [n0, n0 + n) of a corpus; n0 must be a multiple of CHUNK
+    unless the whole draw lies in one chunk."""
+    out = torch.empty(n, d, dtype=torch.float32, device=device)
+    done = 0
+    while done < n:
+        row = n0 + done
+        chunk = row // CHUNK
+        off = row - chunk * CHUNK
+        take = min(n - done, CHUNK - off)
+        g = _gen(seed * 1_000_003 + chunk, device)
+        if kind == "gaussian":
+            x = torch.randn(off + take, d, generator=g, device=device, dtype=torch.float32)[off:]
+        elif kind == "clustered":
+            C = centres.shape[0]
+            a = torch.randint(0, C, (off + take,), generator=g, device=device)[off:]
+            z = torch.randn(off + take, d, generator=g, device=device, dtype=torch.float32)[off:]
+            x = centres[a] + (0.3 / math.sqrt(d)) * z
+        else:
+            raise ValueError(kind)
+        out[done:done + take] = _normalise(x)
+        done += take
+    return out
+
+
+def quantise_e4m3(x: torch.Tensor):
+    """Per-row scaled OCP e4m3: returns (uint8 bytes [n, d], float32 scale [n])."""
+    amax = x.abs().amax(dim=1)
+    scale = torch.where(amax > 0, amax / 448.0, torch.ones_like(amax)).to(torch.float32)
+    q = (x / scale[:, None]).clamp(-448.0, 448.0).to(torch.float8_e4m3fn)
+    return q.view(torch.uint8), scale
+
+
+def make_corpus(spec: WorkloadSpec, device="cpu", N: Optional[int] = None):
+    """Corpus of the workload (optionally only its first N rows).
+    Returns (corpus, row_scale, centres)."""
+    N = spec.N if N is None else N
+    centres = draw_centres(spec, spec.centres, spec.d, device) if spec.corpus == "clustered" else None
+    if spec.dtype == "bf16":
+        corpus = torch.empty(N, spec.d, dtype=torch.bfloat16, device=device)
+        scale = None
+    else:
+        corpus = torch.empty(N, spec.d, dtype=torch.uint8, device=device)
+        scale = torch.empty(N, dtype=torch.float32, device=device)
+    for n0 in range(0, N, CHUNK):
+        n = min(CHUNK, N - n0)
+        x = corpus_rows_fp32(spec.index, n0, n, spec.d, spec.corpus, centres, device)
+        if spec.dtype == "bf16":
+            corpus[n0:n0 + n] = x.to(torch.bfloat16)
+        else:
+            q, s = quantise_e4m3(x)
+            corpus[n0:n0 + n] = q
+            scale[n0:n0 + n] = s
+        del x
+    return corpus, scale, centres
+
+
+def region_counts(spec: WorkloadSpec, Q: Optional[int] = None) -> torch.Tensor:
+    Q = spec.Q if Q is None else Q
+    lo, hi = spec.regions
+    if lo == hi:
+        return torch.full((Q,), lo, dtype=torch.int64)
+    g = _gen(1000 + spec.index, "cpu")
+    return torch.randint(lo, hi + 1, (Q,), generator=g)
+
+
+def offsets_from_counts(counts) -> torch.Tensor:
+    counts = torch.as_tensor(counts, dtype=torch.int64)
+    off = torch.zeros(counts.numel() + 1, dtype=torch.int64)
+    off[1:] = torch.cumsum(counts, 0)
+    return off.to(torch.int32)
+
+
+def make_regions(spec: WorkloadSpec, centres: Optional[torch.Tensor], device="cpu",
+                 Q: Optional[int] = None):
+    """Region query batch (bf16 [R_total, d]) and offsets (int32 [Q+1], on CPU)."""
+    counts = region_counts(spec, Q)
+    offsets = offsets_from_counts(counts)
+    R = int(offsets[-1])
+    g = _gen(1000 + spec.index + 1_000_003, "cpu")
+    if spec.corpus == "gaussian":
+        x = _normalise(torch.randn(R, spec.d, generator=g, dtype=torch.float32))
+    else:
+        C = centres.shape[0]
+        cen = centres.to("cpu")
+        rows = []
+        for q in range(counts.numel()):
+            ne = int(torch.randint(1, 5, (1,), generator=g))
+            ent = torch.randint(0, C, (ne,), generator=g)
+            pick = ent[torch.randint(0, ne, (int(counts[q]),), generator=g)]
+            z = torch.randn(int(counts[q]), spec.d, generator=g, dtype=torch.float32)
+            rows.append(cen[pick] + (0.3 / math.sqrt(spec.d)) * z)
+        x = _normalise(torch.cat(rows, 0)) if rows else torch.empty(0, spec.d)
+    return x.to(torch.bfloat16).to(device), offsets
+
+
+def make_workload(name_or_spec, device="cpu", N: Optional[int] = None,
+                  Q: Optional[int] = None) -> Workload:
+    spec = WORKLOADS[name_or_spec] if isinstance(name_or_spec, str) else name_or_spec
+    corpus, scale, centres = make_corpus(spec, device, N)
+    regions, offsets = make_regions(spec, centres, device, Q)
+    return Workload(spec, corpus, scale, regions, offsets, centres)
+
+
+def random_bf16(n: int, d: int, seed: int, device="cpu") -> torch.Tensor:
+    """Unit-norm Gaussian rows as bf16 (small test inputs)."""
+    g = _gen(seed, device)
+    return _normalise(torch.randn(n, d, generator=g, device=device)).to(torch.bfloat16)
+
+
+def bf16_bits(t: torch.Tensor):
+    """uint16 numpy view of a bf16 tensor (host)."""
+    return t.detach().to("cpu").contiguous().view(torch.int16).numpy().view("uint16")
