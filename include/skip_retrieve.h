@@ -1,0 +1,174 @@
+/*
+ * skip_retrieve.h -- C ABI of the GB300 (sm_103a) region-conditional sparse
+ * retrieval library.
+ *
+ * The operation (paper §3.3 Eq. rcsr; App. B.2 Def. B.2; Alg. 1, the RCSR
+ * loop and the Dedup step): every region query q_r of a question is scored
+ * against every corpus row x_i by inner product (maximum inner product
+ * search), the exact top-k_region ids are kept per region, and each
+ * question's region lists are merged into one deduplicated top-K list.
+ *
+ *   s(r, i)  = sum_j q_{r,j} x_{i,j}        x = bf16 row, or e4m3 row * scale_i
+ *   L_r      = top-k_region of {0..N-1} by (s desc, id asc)
+ *   out_q    = top-K of union_{r in q} L_r by (max_r s desc, id asc),
+ *              one entry per id, padded with (id -1, score -inf)
+ *
+ * Conventions shared by every entry point:
+ *  - Corpus rows are row-major [N x d]; d must be a multiple of 16 and
+ *    N < 2^31.  Ids are corpus row indices.
+ *  - Region queries are bf16, row-major [R_total x d].  Questions own
+ *    consecutive regions: question q owns rows [offsets[q], offsets[q+1]);
+ *    offsets has Q + 1 int32 entries with offsets[0] = 0 and
+ *    offsets[Q] = R_total; a question may own zero regions.
+ *  - Scores are returned as fp32, ids as int64.  Lists are sorted by
+ *    (score desc, id asc).  Ties go to the lower id.
+ *  - Device pointers are CUDA device (or managed) addresses; host pointers
+ *    are ordinary host memory.  Streams are cudaStream_t values passed as
+ *    void* (NULL = the legacy default stream).
+ *  - Calls on device buffers are asynchronous and stream ordered: they
+ *    enqueue work on `stream` and return.  Argument errors are reported
+ *    synchronously; errors found by kernels (a bounded wait that gave up)
+ *    are latched in the corpus handle and reported by skip_sync_status.
+ *  - A handle is not thread safe: serialise calls that share one.
+ *  - Nothing here falls back to the CPU.  Without a usable sm_103 device,
+ *    skip_corpus_load returns SKIP_EUNSUPPORTED.
+ */
+#ifndef SKIP_RETRIEVE_H
+#define SKIP_RETRIEVE_H
+
+#include <stdint.h>
+
+#ifdef __cplusplus
+extern "C" {
+#endif
+
+#if defined(__GNUC__)
+#define SKIP_API __attribute__((visibility("default")))
+#else
+#define SKIP_API
+#endif
+
+typedef struct skip_corpus *skip_corpus_t; /* opaque; owns the device copy */
+
+typedef enum {
+    SKIP_BF16 = 0, /* bf16 rows, 2 bytes per element */
+    SKIP_E4M3 = 1  /* OCP float8 e4m3fn rows with one fp32 scale per row */
+} skip_dtype_t;
+
+typedef enum {
+    SKIP_OK = 0,
+    SKIP_EINVAL = 1,        /* bad argument (null pointer, size or range) */
+    SKIP_ENOMEM = 2,        /* device or pinned allocation failed */
+    SKIP_EUNSUPPORTED = 3,  /* no sm_103 device, or a size beyond a stated limit */
+    SKIP_ETIMEOUT = 4,      /* a kernel's bounded wait gave up; results invalid */
+    SKIP_ECUDA = 5          /* a CUDA runtime/driver call failed */
+} skip_status_t;
+
+typedef enum {
+    SKIP_OPT_PATH = 0,            /* score kernel: 0 auto, 1 tensor core, 2 warp-dot */
+    SKIP_OPT_WAIT_TIMEOUT_NS = 1, /* cap on each in-kernel wait (default 2e9 ns) */
+    SKIP_OPT_GRID = 2,            /* score-kernel CTAs (0 = one per SM) */
+    SKIP_OPT_TIMING = 3           /* 1: time each kernel with CUDA events */
+} skip_option_t;
+
+enum { SKIP_PATH_AUTO = 0, SKIP_PATH_TENSOR = 1, SKIP_PATH_WARP = 2 };
+
+/* Limits checked by every retrieval call. */
+#define SKIP_MAX_K_REGION 1024
+#define SKIP_MAX_K 2048
+
+/*
+ * skip_corpus_load -- lay the corpus D (paper Def. B.2, the searched set;
+ * §4.1 "Knowledge corpora") out in device memory for retrieval.
+ *
+ *  rows            [N x d] row-major elements: uint16 bf16 bits for
+ *                  SKIP_BF16, bytes for SKIP_E4M3.
+ *  rows_on_device  nonzero: `rows` and `row_scale` are device pointers and
+ *                  are copied device-to-device; zero: host pointers.
+ *  row_scale       [N] fp32 per-row dequantisation scales; required for
+ *                  SKIP_E4M3 (each element's value is e4m3 * scale), must
+ *                  be NULL for SKIP_BF16.
+ *  stream          stream for the copies; the call returns after they finish.
+ *  out             receives the handle.
+ * The library owns the copy until skip_corpus_free; the caller's buffers
+ * can be reused as soon as the call returns.
+ * Errors: SKIP_EINVAL (null pointers, N < 1, N >= 2^31, d % 16 != 0,
+ * scale missing or unexpected), SKIP_ENOMEM, SKIP_EUNSUPPORTED (no
+ * sm_103 device), SKIP_ECUDA.
+ */
+SKIP_API skip_status_t skip_corpus_load(const void *rows, int rows_on_device, int64_t N, int32_t d,
+                               skip_dtype_t dtype, const float *row_scale, void *stream,
+                               skip_corpus_t *out);
+
+/* Frees the corpus copy and the handle's workspace after synchronising the
+ * device.  NULL is accepted. */
+SKIP_API skip_status_t skip_corpus_free(skip_corpus_t corpus);
+
+/* Sets a per-handle option (skip_option_t); SKIP_EINVAL for an unknown
+ * option or a value out of range. */
+SKIP_API skip_status_t skip_corpus_set_option(skip_corpus_t corpus, int option, int64_t value);
+
+/*
+ * skip_retrieve -- the whole path on device buffers: per-region MIPS top-k
+ * (Def. B.2, Eq. rcsr), then the per-question Dedup of the union cut to K
+ * (§3.3, Def. B.2, Alg. 1).
+ *
+ *  regions         device bf16 [R_total x d] (uint16 bits), row-major.
+ *  region_offsets  device int32 [num_questions + 1] prefix offsets; the
+ *                  library never reads them on the host, so R_total must
+ *                  equal region_offsets[num_questions].
+ *  k_region        1 <= k_region <= min(N, SKIP_MAX_K_REGION).
+ *  K               1 <= K <= SKIP_MAX_K.
+ *  out_ids         device int64 [num_questions x K].
+ *  out_scores      device fp32  [num_questions x K].
+ * Uses a workspace owned by the handle (grown on demand, which
+ * synchronises the device once).  Asynchronous on `stream`.
+ * Errors: SKIP_EINVAL, SKIP_ENOMEM, SKIP_ECUDA.
+ */
+SKIP_API skip_status_t skip_retrieve(skip_corpus_t corpus, const void *regions,
+                            const int32_t *region_offsets, int32_t num_questions,
+                            int32_t R_total, int32_t k_region, int32_t K, int64_t *out_ids,
+                            float *out_scores, void *stream);
+
+/*
+ * skip_retrieve_regions -- only the per-region step (Def. B.2
+ * MIPS(q_r, D; k_r)): reg_ids int64 and reg_scores fp32, both device
+ * [R_total x k_region], each row sorted by (score desc, id asc).
+ * Same argument rules as skip_retrieve.
+ */
+SKIP_API skip_status_t skip_retrieve_regions(skip_corpus_t corpus, const void *regions, int32_t R_total,
+                                    int32_t k_region, int64_t *reg_ids, float *reg_scores,
+                                    void *stream);
+
+/*
+ * skip_retrieve_host -- skip_retrieve on HOST buffers: copies regions and
+ * offsets to the device, runs the path and copies the results back, all on
+ * `stream`, and returns after the stream has drained (so the kernels'
+ * error word is also checked).  Shapes as in skip_retrieve.
+ * Errors: as skip_retrieve, plus SKIP_ETIMEOUT.
+ */
+SKIP_API skip_status_t skip_retrieve_host(skip_corpus_t corpus, const uint16_t *regions,
+                                 const int32_t *region_offsets, int32_t num_questions,
+                                 int32_t R_total, int32_t k_region, int32_t K, int64_t *out_ids,
+                                 float *out_scores, void *stream);
+
+/* Synchronises `stream`, then reports and clears the handle's error word:
+ * SKIP_ETIMEOUT if a kernel's bounded wait gave up since the last check,
+ * SKIP_EINVAL if region offsets were inconsistent with R_total (clamped),
+ * SKIP_ECUDA if the stream reported an error, else SKIP_OK. */
+SKIP_API skip_status_t skip_sync_status(skip_corpus_t corpus, void *stream);
+
+/* Describes the last retrieval call's launch plan as a short JSON object
+ * (path, grid, corpus chunks, kernels launched) and, when SKIP_OPT_TIMING is
+ * on, the device time of each kernel in ms (this synchronises on the
+ * events).  Writes at most `len` bytes including the terminator. */
+SKIP_API skip_status_t skip_last_plan(skip_corpus_t corpus, char *buf, int32_t len);
+
+/* Static description of a status code. */
+SKIP_API const char *skip_status_string(skip_status_t status);
+
+#ifdef __cplusplus
+}
+#endif
+
+#endif /* SKIP_RETRIEVE_H */

@@ -14,6 +14,7 @@ Functions and what they follow:
   per-region lists, keeping each id's max score, cut to the first K.
 * ``retrieve``     -- both steps (the CPU baseline).
 * ``score_matrix`` -- every s(r, i) in fp64 (brute force on tiny inputs).
+* ``scores_at``    -- s(r, i) at chosen (region, id) pairs.
 """
 from __future__ import annotations
 
@@ -53,12 +54,13 @@ def _load():
     lib.skip_oracle_merge.argtypes = [P, P, i32, i32, P, i32, i32, P, P]
     lib.skip_oracle_retrieve.argtypes = [P, P, P, i64, i32, P, P, i32, i64, i32, i32, P, P, P, P, i32]
     lib.skip_oracle_score_matrix.argtypes = [P, P, P, i64, i32, P, i64, P]
+    lib.skip_oracle_scores_at.argtypes = [P, P, P, i64, i32, P, P, P, i64, P]
     lib.skip_oracle_bf16_value.argtypes = [ctypes.c_uint16]
     lib.skip_oracle_bf16_value.restype = ctypes.c_double
     lib.skip_oracle_e4m3_value.argtypes = [ctypes.c_uint8]
     lib.skip_oracle_e4m3_value.restype = ctypes.c_double
     for f in ("skip_oracle_region_topk", "skip_oracle_merge", "skip_oracle_retrieve",
-              "skip_oracle_score_matrix", "skip_oracle_threads"):
+              "skip_oracle_score_matrix", "skip_oracle_scores_at", "skip_oracle_threads"):
         getattr(lib, f).restype = ctypes.c_int
     _lib = lib
     return lib
@@ -161,4 +163,21 @@ def score_matrix(corpus, regions, row_scale=None):
                                       _ptr(out))
     if rc:
         raise RuntimeError("oracle score_matrix failed (%d)" % rc)
+    return out
+
+
+def scores_at(corpus, regions, region_idx, ids, row_scale=None):
+    """s(region_idx[t], ids[t]) in fp64 for each t (NaN for ids outside [0, N))."""
+    lib = _load()
+    cb, ce, sc = _corpus_args(corpus, row_scale)
+    c = cb if cb is not None else ce
+    regions = np.ascontiguousarray(regions, dtype=np.uint16)
+    region_idx = np.ascontiguousarray(region_idx, dtype=np.int64).ravel()
+    ids = np.ascontiguousarray(ids, dtype=np.int64).ravel()
+    N, d = c.shape
+    out = np.empty(ids.shape[0], dtype=np.float64)
+    rc = lib.skip_oracle_scores_at(_ptr(cb), _ptr(ce), _ptr(sc), N, d, _ptr(regions),
+                                   _ptr(region_idx), _ptr(ids), ids.shape[0], _ptr(out))
+    if rc:
+        raise RuntimeError("oracle scores_at failed (%d)" % rc)
     return out

@@ -330,4 +330,30 @@ int skip_oracle_score_matrix(const uint16_t *corpus_bf16, const uint8_t *corpus_
     return 0;
 }
 
+/* s(r, ids[t]) for a list of (region, id) pairs: the oracle's value of
+ * chosen scores, used to check scores reported for ids outside a list. */
+int skip_oracle_scores_at(const uint16_t *corpus_bf16, const uint8_t *corpus_e4m3,
+                          const float *row_scale, int64_t N, int d, const uint16_t *regions,
+                          const int64_t *region_idx, const int64_t *ids, int64_t n, double *out)
+{
+    if ((corpus_bf16 == NULL) == (corpus_e4m3 == NULL) || (corpus_e4m3 && !row_scale))
+        return 1;
+    init_tables();
+    corpus_t c = {corpus_bf16, corpus_e4m3, row_scale, N, d};
+    double *q = (double *)malloc(sizeof(double) * (size_t)(d > 0 ? d : 1));
+    if (!q)
+        return 2;
+    for (int64_t t = 0; t < n; ++t) {
+        if (ids[t] < 0 || ids[t] >= N) {
+            out[t] = NAN;
+            continue;
+        }
+        for (int j = 0; j < d; ++j)
+            q[j] = bf16_value(regions[region_idx[t] * (int64_t)d + j]);
+        out[t] = score(&c, q, ids[t]);
+    }
+    free(q);
+    return 0;
+}
+
 int skip_oracle_threads(void) { return resolve_threads(0); }

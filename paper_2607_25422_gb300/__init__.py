@@ -1,0 +1,220 @@
+"""Python binding of the GB300 region-conditional sparse retrieval library.
+
+The functions carry the names of the C ABI in ``include/skip_retrieve.h`` and
+only marshal arguments: tensors are handed over as raw pointers and streams
+as ``cudaStream_t`` values; every step of the retrieval runs in the CUDA
+library (``_build/libskip_retrieve.so``, built from ``csrc/`` for sm_103a).
+There is no CPU path: if the library cannot be built or loaded, or the
+device is not an sm_103 GPU, the calls raise.
+
+The operation (paper §3.3 Eq. rcsr; App. B.2 Def. B.2; Alg. 1 RCSR loop and
+Dedup): each region query is scored against the corpus by inner product, the
+top-k_region ids are kept per region, and each question's region lists are
+merged into a deduplicated top-K (max score per id, ties to the lower id).
+"""
+from __future__ import annotations
+
+import ctypes
+import json
+from typing import Optional
+
+import torch
+
+from . import _build
+
+SKIP_BF16, SKIP_E4M3 = 0, 1
+SKIP_OK, SKIP_EINVAL, SKIP_ENOMEM, SKIP_EUNSUPPORTED, SKIP_ETIMEOUT, SKIP_ECUDA = range(6)
+SKIP_OPT_PATH, SKIP_OPT_WAIT_TIMEOUT_NS, SKIP_OPT_GRID, SKIP_OPT_TIMING = range(4)
+SKIP_PATH_AUTO, SKIP_PATH_TENSOR, SKIP_PATH_WARP = range(3)
+SKIP_MAX_K_REGION, SKIP_MAX_K = 1024, 2048
+
+_lib = None
+
+
+class SkipError(RuntimeError):
+    def __init__(self, status: int, where: str):
+        self.status = status
+        super().__init__("%s: %s (%d)" % (where, skip_status_string(status), status))
+
+
+def library_path() -> str:
+    return _build.LIB
+
+
+def load_library():
+    """Build (if stale) and load the CUDA library; raises if either fails."""
+    global _lib
+    if _lib is not None:
+        return _lib
+    lib = ctypes.CDLL(_build.build())
+    P, i32, i64 = ctypes.c_void_p, ctypes.c_int32, ctypes.c_int64
+    lib.skip_corpus_load.argtypes = [P, ctypes.c_int, i64, i32, ctypes.c_int, P, P, ctypes.POINTER(P)]
+    lib.skip_corpus_free.argtypes = [P]
+    lib.skip_corpus_set_option.argtypes = [P, ctypes.c_int, i64]
+    lib.skip_retrieve.argtypes = [P, P, P, i32, i32, i32, i32, P, P, P]
+    lib.skip_retrieve_regions.argtypes = [P, P, i32, i32, P, P, P]
+    lib.skip_retrieve_host.argtypes = [P, P, P, i32, i32, i32, i32, P, P, P]
+    lib.skip_sync_status.argtypes = [P, P]
+    lib.skip_last_plan.argtypes = [P, ctypes.c_char_p, i32]
+    lib.skip_status_string.argtypes = [ctypes.c_int]
+    lib.skip_status_string.restype = ctypes.c_char_p
+    for f in ("skip_corpus_load", "skip_corpus_free", "skip_corpus_set_option", "skip_retrieve",
+              "skip_retrieve_regions", "skip_retrieve_host", "skip_sync_status", "skip_last_plan"):
+        getattr(lib, f).restype = ctypes.c_int
+    _lib = lib
+    return lib
+
+
+def skip_status_string(status: int) -> str:
+    return load_library().skip_status_string(int(status)).decode()
+
+
+def _check(status: int, where: str):
+    if status != SKIP_OK:
+        raise SkipError(status, where)
+
+
+def _stream(stream) -> int:
+    if stream is None:
+        stream = torch.cuda.current_stream()
+    return int(stream.cuda_stream) if hasattr(stream, "cuda_stream") else int(stream)
+
+
+def _ptr(t: Optional[torch.Tensor]):
+    return None if t is None else ctypes.c_void_p(t.data_ptr())
+
+
+class Corpus:
+    """A corpus handle (``skip_corpus_t``); the library owns the device copy."""
+
+    def __init__(self, handle, N: int, d: int, dtype: int, device: torch.device):
+        self.handle = handle
+        self.N, self.d, self.dtype, self.device = N, d, dtype, device
+
+    def free(self):
+        if self.handle:
+            load_library().skip_corpus_free(self.handle)
+            self.handle = None
+
+    def __del__(self):
+        try:
+            self.free()
+        except Exception:
+            pass
+
+    def set_option(self, option: int, value: int):
+        skip_corpus_set_option(self, option, value)
+
+
+def skip_corpus_load(rows: torch.Tensor, row_scale: Optional[torch.Tensor] = None,
+                     stream=None) -> Corpus:
+    """Copy a corpus into the library.  rows: [N, d] bfloat16 (or uint16 bf16
+    bits), or uint8 / float8_e4m3fn bytes with row_scale [N] float32; on the
+    host or on the current CUDA device."""
+    lib = load_library()
+    if rows.dim() != 2:
+        raise ValueError("rows must be [N, d]")
+    if rows.dtype in (torch.bfloat16, torch.uint16, torch.int16):
+        dtype = SKIP_BF16
+    elif rows.dtype in (torch.uint8, torch.float8_e4m3fn):
+        dtype = SKIP_E4M3
+    else:
+        raise TypeError("rows must be bf16 or e4m3 bytes")
+    rows = rows.contiguous()
+    on_dev = rows.is_cuda
+    if row_scale is not None:
+        row_scale = row_scale.to(device=rows.device, dtype=torch.float32).contiguous()
+    dev = rows.device if on_dev else torch.device("cuda", torch.cuda.current_device())
+    h = ctypes.c_void_p()
+    st = lib.skip_corpus_load(_ptr(rows), int(on_dev), rows.shape[0], rows.shape[1], dtype,
+                              _ptr(row_scale), ctypes.c_void_p(_stream(stream)), ctypes.byref(h))
+    _check(st, "skip_corpus_load")
+    return Corpus(h, rows.shape[0], rows.shape[1], dtype, dev)
+
+
+def skip_corpus_free(corpus: Corpus):
+    corpus.free()
+
+
+def skip_corpus_set_option(corpus: Corpus, option: int, value: int):
+    _check(load_library().skip_corpus_set_option(corpus.handle, int(option), int(value)),
+           "skip_corpus_set_option")
+
+
+def _regions_arg(regions: torch.Tensor, corpus: Corpus) -> torch.Tensor:
+    if regions.dim() != 2 or regions.shape[1] != corpus.d:
+        raise ValueError("regions must be [R_total, d]")
+    if regions.dtype not in (torch.bfloat16, torch.uint16, torch.int16):
+        raise TypeError("regions must be bf16")
+    return regions.contiguous()
+
+
+def skip_retrieve(corpus: Corpus, regions: torch.Tensor, region_offsets: torch.Tensor,
+                  k_region: int, K: int, out_ids: Optional[torch.Tensor] = None,
+                  out_scores: Optional[torch.Tensor] = None, stream=None):
+    """Whole path on device tensors; returns (ids int64 [Q, K], scores fp32 [Q, K])."""
+    lib = load_library()
+    regions = _regions_arg(regions, corpus)
+    offs = region_offsets.to(device=regions.device, dtype=torch.int32).contiguous()
+    Q = offs.numel() - 1
+    if out_ids is None:
+        out_ids = torch.empty(Q, K, dtype=torch.int64, device=regions.device)
+    if out_scores is None:
+        out_scores = torch.empty(Q, K, dtype=torch.float32, device=regions.device)
+    st = lib.skip_retrieve(corpus.handle, _ptr(regions), _ptr(offs), Q, regions.shape[0], int(k_region),
+                           int(K), _ptr(out_ids), _ptr(out_scores), ctypes.c_void_p(_stream(stream)))
+    _check(st, "skip_retrieve")
+    return out_ids, out_scores
+
+
+def skip_retrieve_regions(corpus: Corpus, regions: torch.Tensor, k_region: int,
+                          reg_ids: Optional[torch.Tensor] = None,
+                          reg_scores: Optional[torch.Tensor] = None, stream=None):
+    """Per-region step only; returns (ids int64 [R, k], scores fp32 [R, k])."""
+    lib = load_library()
+    regions = _regions_arg(regions, corpus)
+    R = regions.shape[0]
+    if reg_ids is None:
+        reg_ids = torch.empty(R, k_region, dtype=torch.int64, device=regions.device)
+    if reg_scores is None:
+        reg_scores = torch.empty(R, k_region, dtype=torch.float32, device=regions.device)
+    st = lib.skip_retrieve_regions(corpus.handle, _ptr(regions), R, int(k_region), _ptr(reg_ids),
+                                   _ptr(reg_scores), ctypes.c_void_p(_stream(stream)))
+    _check(st, "skip_retrieve_regions")
+    return reg_ids, reg_scores
+
+
+def skip_retrieve_host(corpus: Corpus, regions: torch.Tensor, region_offsets: torch.Tensor,
+                       k_region: int, K: int, out_ids: Optional[torch.Tensor] = None,
+                       out_scores: Optional[torch.Tensor] = None, stream=None):
+    """Whole path on HOST tensors (pinned memory is fastest); blocks until done."""
+    lib = load_library()
+    if regions.is_cuda:
+        raise ValueError("skip_retrieve_host takes host tensors")
+    regions = _regions_arg(regions, corpus)
+    offs = region_offsets.to(dtype=torch.int32).contiguous()
+    Q = offs.numel() - 1
+    if out_ids is None:
+        out_ids = torch.empty(Q, K, dtype=torch.int64)
+    if out_scores is None:
+        out_scores = torch.empty(Q, K, dtype=torch.float32)
+    st = lib.skip_retrieve_host(corpus.handle, _ptr(regions), _ptr(offs), Q, regions.shape[0],
+                                int(k_region), int(K), _ptr(out_ids), _ptr(out_scores),
+                                ctypes.c_void_p(_stream(stream)))
+    _check(st, "skip_retrieve_host")
+    return out_ids, out_scores
+
+
+def skip_sync_status(corpus: Corpus, stream=None) -> int:
+    """Synchronise and return the status latched by the kernels (SKIP_OK, ...)."""
+    return int(load_library().skip_sync_status(corpus.handle, ctypes.c_void_p(_stream(stream))))
+
+
+def skip_last_plan(corpus: Corpus) -> dict:
+    buf = ctypes.create_string_buffer(1024)
+    _check(load_library().skip_last_plan(corpus.handle, buf, 1024), "skip_last_plan")
+    return json.loads(buf.value.decode())
+
+
+__all__ = [n for n in dir() if n.startswith("skip_") or n.startswith("SKIP_")] + [
+    "Corpus", "SkipError", "load_library", "library_path"]

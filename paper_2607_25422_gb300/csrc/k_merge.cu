@@ -1,0 +1,188 @@
+// Cross-partition merge (per region) and region-to-question merge with
+// deduplication (per question).
+//
+// Per region (paper App. B.2 Def. B.2, MIPS(q_r, D; k_r)): the score kernels
+// leave, for every region row, one sorted top-k list per corpus partition
+// they scanned.  The exact top-k over the whole corpus is the top-k of the
+// union of those lists, because every member of the global top-k is a
+// member of its own partition's top-k.  One warp merges one row.
+//
+// Per question (§3.3 "deduplicate the union of K_r"; Def. B.2
+// K = Dedup(union_i K_{r_i}); Alg. 1 Dedup step): the lists of the question's
+// regions are pooled, each id keeps its maximum score, and the first K by
+// (score desc, id asc) are written, padded with (-1, -inf).  One block per
+// question.  The pool is sorted by (id asc, score desc) so that the first
+// entry of every id run carries the id's maximum; those entries are then
+// sorted by the ranking key.  When a question's pool exceeds the shared
+// memory capacity, regions are folded in chunks: the running top-K already
+// holds every id's best score that can still reach the output, since an id
+// that fell below the running K-th score can only return with a larger one.
+#include "skip_device.cuh"
+#include "skip_internal.h"
+
+namespace skipk {
+namespace {
+
+constexpr int kMergeWarps = 4;
+
+template <int LPL>
+__global__ void __launch_bounds__(kMergeWarps * 32)
+    k_merge_lists(const uint64_t *__restrict__ lists, int G, int64_t g_stride, int R, int k,
+                  uint64_t *__restrict__ reg_keys, int64_t *__restrict__ reg_ids,
+                  float *__restrict__ reg_scores) {
+    const int warp = threadIdx.x >> 5;
+    const int row = blockIdx.x * kMergeWarps + warp;
+    if (row >= R) return;
+    const uint64_t *base = lists + (int64_t)row * k;
+    uint64_t *kout = reg_keys ? reg_keys + (int64_t)row * k : nullptr;
+    int64_t *iout = reg_ids ? reg_ids + (int64_t)row * k : nullptr;
+    float *sout = reg_scores ? reg_scores + (int64_t)row * k : nullptr;
+    warp_merge_topk<LPL>(base, g_stride, G, k, k, [&](int i, uint64_t key) {
+        if (kout) kout[i] = key;
+        if (iout) {
+            int64_t id;
+            float s;
+            key_decode(key, id, s);
+            iout[i] = id;
+            sout[i] = s;
+        }
+    });
+}
+
+constexpr int kQThreads = 512;
+constexpr int kQCap = 4096;  // pooled candidates per pass (32 KB per array)
+constexpr uint64_t kNone = ~0ull;
+
+// Block-wide bitonic sort of s[0..n2) (n2 a power of two), ascending.
+__device__ void block_bitonic_sort_asc(uint64_t *s, int n2) {
+    for (int size = 2; size <= n2; size <<= 1) {
+        for (int stride = size >> 1; stride > 0; stride >>= 1) {
+            __syncthreads();
+            for (int i = threadIdx.x; i < (n2 >> 1); i += blockDim.x) {
+                const int lo = 2 * i - (i & (stride - 1));
+                const int hi = lo + stride;
+                const bool up = (lo & size) == 0;
+                const uint64_t a = s[lo], b = s[hi];
+                if ((a > b) == up) {
+                    s[lo] = b;
+                    s[hi] = a;
+                }
+            }
+        }
+    }
+    __syncthreads();
+}
+
+__device__ __forceinline__ int pow2_at_least(int n) {
+    int p = 1;
+    while (p < n) p <<= 1;
+    return p;
+}
+
+// (id asc, score desc) ordering key of a ranking key; empty slots sort last.
+__device__ __forceinline__ uint64_t id_major(uint64_t key) {
+    if (key == 0) return kNone;
+    const uint64_t id = (uint64_t)key_id(key);
+    const uint32_t ord = (uint32_t)(key >> 32);
+    return (id << 32) | (uint64_t)(0xFFFFFFFFu - ord);
+}
+
+__device__ __forceinline__ uint64_t rank_of_id_major(uint64_t im) {
+    const uint32_t id = (uint32_t)(im >> 32);
+    const uint32_t ord = 0xFFFFFFFFu - (uint32_t)im;
+    return ((uint64_t)ord << 32) | (uint64_t)(0xFFFFFFFFu - id);
+}
+
+__global__ void __launch_bounds__(kQThreads)
+    k_question_merge(const uint64_t *__restrict__ reg_keys, int k, const int32_t *__restrict__ offsets,
+                     int R, int K, int64_t *__restrict__ out_ids, float *__restrict__ out_scores,
+                     int *__restrict__ err) {
+    extern __shared__ uint64_t qsmem[];
+    uint64_t *pool = qsmem;            // [kQCap] id-major keys
+    uint64_t *ranked = qsmem + kQCap;  // [kQCap] ranking keys, negated for the ascending sort
+    __shared__ int s_kept;
+    const int q = blockIdx.x;
+    // Offsets outside [0, R] or decreasing are clamped (and flagged) so that
+    // no read leaves the region lists.
+    const int o0 = offsets[q], o1 = offsets[q + 1];
+    const int r0 = min(max(o0, 0), R);
+    const int r1 = min(max(o1, r0), R);
+    if ((r0 != o0 || r1 != o1) && threadIdx.x == 0) atomicOr(err, kErrConfig);
+    int nrun = 0;  // running top-K, kept as ranking keys in ranked[0..nrun) (descending)
+    int r = r0;
+    do {
+        const int nreg = min(r1 - r, (kQCap - nrun) / k);
+        const int n = nrun + nreg * k;
+        for (int i = threadIdx.x; i < nrun; i += blockDim.x) pool[i] = id_major(ranked[i]);
+        for (int i = threadIdx.x; i < nreg * k; i += blockDim.x)
+            pool[nrun + i] = id_major(reg_keys[(int64_t)r * k + i]);
+        const int n2 = pow2_at_least(n > 1 ? n : 1);
+        for (int i = n + threadIdx.x; i < n2; i += blockDim.x) pool[i] = kNone;
+        if (threadIdx.x == 0) s_kept = 0;
+        block_bitonic_sort_asc(pool, n2);
+        // First entry of every id run = that id with its maximum score.
+        for (int i = threadIdx.x; i < n; i += blockDim.x) {
+            const uint64_t v = pool[i];
+            if (v == kNone) continue;
+            if (i > 0 && (pool[i - 1] >> 32) == (v >> 32)) continue;
+            const int at = atomicAdd(&s_kept, 1);
+            ranked[at] = ~rank_of_id_major(v);  // ascending sort of ~key = descending by key
+        }
+        __syncthreads();
+        const int m = s_kept;
+        const int m2 = pow2_at_least(m > 1 ? m : 1);
+        for (int i = m + threadIdx.x; i < m2; i += blockDim.x) ranked[i] = kNone;
+        block_bitonic_sort_asc(ranked, m2);
+        nrun = min(m, K);
+        for (int i = threadIdx.x; i < nrun; i += blockDim.x) ranked[i] = ~ranked[i];
+        __syncthreads();
+        r += nreg;
+    } while (r < r1);
+
+    for (int i = threadIdx.x; i < K; i += blockDim.x) {
+        int64_t id = -1;
+        float s = -__int_as_float(0x7f800000);
+        if (i < nrun) key_decode(ranked[i], id, s);
+        out_ids[(int64_t)q * K + i] = id;
+        out_scores[(int64_t)q * K + i] = s;
+    }
+}
+
+}  // namespace
+
+cudaError_t launch_merge_lists(const uint64_t *lists, int G, int64_t g_stride, int R, int k,
+                               uint64_t *reg_keys, int64_t *reg_ids, float *reg_scores,
+                               cudaStream_t s) {
+    if (R <= 0) return cudaSuccess;
+    const int grid = (R + kMergeWarps - 1) / kMergeWarps;
+    const int threads = kMergeWarps * 32;
+    if (G <= 32)
+        k_merge_lists<1><<<grid, threads, 0, s>>>(lists, G, g_stride, R, k, reg_keys, reg_ids, reg_scores);
+    else if (G <= 64)
+        k_merge_lists<2><<<grid, threads, 0, s>>>(lists, G, g_stride, R, k, reg_keys, reg_ids, reg_scores);
+    else if (G <= 128)
+        k_merge_lists<4><<<grid, threads, 0, s>>>(lists, G, g_stride, R, k, reg_keys, reg_ids, reg_scores);
+    else if (G <= 256)
+        k_merge_lists<8><<<grid, threads, 0, s>>>(lists, G, g_stride, R, k, reg_keys, reg_ids, reg_scores);
+    else if (G <= 512)
+        k_merge_lists<16><<<grid, threads, 0, s>>>(lists, G, g_stride, R, k, reg_keys, reg_ids, reg_scores);
+    else
+        return cudaErrorInvalidValue;
+    return cudaGetLastError();
+}
+
+int question_merge_capacity() { return kQCap; }
+
+cudaError_t launch_question_merge(const uint64_t *reg_keys, int k, const int32_t *offsets, int Q,
+                                  int R, int K, int64_t *out_ids, float *out_scores, int *err,
+                                  cudaStream_t s) {
+    if (Q <= 0) return cudaSuccess;
+    if (K + k > kQCap) return cudaErrorInvalidValue;
+    const int smem = 2 * kQCap * (int)sizeof(uint64_t);
+    cudaError_t e = cudaFuncSetAttribute(k_question_merge, cudaFuncAttributeMaxDynamicSharedMemorySize, smem);
+    if (e != cudaSuccess) return e;
+    k_question_merge<<<Q, kQThreads, smem, s>>>(reg_keys, k, offsets, R, K, out_ids, out_scores, err);
+    return cudaGetLastError();
+}
+
+}  // namespace skipk

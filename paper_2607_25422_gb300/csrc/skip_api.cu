@@ -1,0 +1,491 @@
+// C-ABI layer of the retrieval library: argument checks, the corpus copy and
+// its TMA descriptor, the per-handle workspace, the launch plan for each
+// regime and the error word.  The arithmetic lives in the kernels
+// (k_tc.cu, k_warpdot.cu, k_merge.cu); this file only decides what to launch.
+#include <stdio.h>
+#include <stdlib.h>
+#include <string.h>
+
+#include <algorithm>
+#include <mutex>
+
+#include "../../include/skip_retrieve.h"
+#include "skip_internal.h"
+
+using namespace skipk;
+
+namespace {
+
+constexpr uint64_t kDefaultTimeoutNs = 2000000000ull;
+constexpr int kMaxD = 4096;
+constexpr int kMaxEvents = 8;
+
+typedef CUresult (*EncodeTiledFn)(CUtensorMap *, CUtensorMapDataType, cuuint32_t, void *,
+                                  const cuuint64_t *, const cuuint64_t *, const cuuint32_t *,
+                                  const cuuint32_t *, CUtensorMapInterleave, CUtensorMapSwizzle,
+                                  CUtensorMapL2promotion, CUtensorMapFloatOOBfill);
+
+EncodeTiledFn encode_fn() {
+    static EncodeTiledFn fn = nullptr;
+    static std::once_flag once;
+    std::call_once(once, [] {
+        void *p = nullptr;
+        cudaDriverEntryPointQueryResult q;
+        if (cudaGetDriverEntryPointByVersion("cuTensorMapEncodeTiled", &p, 12000, cudaEnableDefault, &q) ==
+                cudaSuccess &&
+            q == cudaDriverEntryPointSuccess)
+            fn = reinterpret_cast<EncodeTiledFn>(p);
+    });
+    return fn;
+}
+
+// 2D bf16 tensor map over a row-major [rows x d] matrix, box = box_rows x 64
+// elements (128 bytes), 128-byte swizzle, zero fill out of bounds.
+bool encode_bf16_rows(CUtensorMap *map, const void *base, int64_t rows, int d, int box_rows) {
+    EncodeTiledFn fn = encode_fn();
+    if (!fn) return false;
+    cuuint64_t dims[2] = {(cuuint64_t)d, (cuuint64_t)rows};
+    cuuint64_t strides[1] = {(cuuint64_t)d * 2};
+    cuuint32_t box[2] = {(cuuint32_t)kTcTileK, (cuuint32_t)box_rows};
+    cuuint32_t estr[2] = {1, 1};
+    return fn(map, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 2, const_cast<void *>(base), dims, strides, box,
+              estr, CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B,
+              CU_TENSOR_MAP_L2_PROMOTION_L2_256B, CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) == CUDA_SUCCESS;
+}
+
+}  // namespace
+
+struct skip_corpus {
+    int device = 0;
+    int sm_count = 0;
+    int64_t N = 0;
+    int d = 0;
+    skip_dtype_t dtype = SKIP_BF16;
+    void *rows = nullptr;      // device [N x d]
+    float *scale = nullptr;    // device [N] (e4m3)
+    int *err = nullptr;        // device error word
+    CUtensorMap tmap_x;        // corpus rows, box 256 x 64 (bf16 only)
+    bool tmap_ok = false;
+    void *ws = nullptr;        // workspace
+    size_t ws_bytes = 0;
+    void *io = nullptr;        // device staging for skip_retrieve_host
+    size_t io_bytes = 0;
+    int path = SKIP_PATH_AUTO;
+    uint64_t timeout_ns = kDefaultTimeoutNs;
+    int grid = 0;
+    int timing = 0;
+    cudaEvent_t ev[kMaxEvents] = {};
+    const char *ev_name[kMaxEvents] = {};
+    int n_ev = 0;
+    char plan[384] = "{}";
+};
+
+namespace {
+
+skip_status_t cuda_status(cudaError_t e) {
+    if (e == cudaSuccess) return SKIP_OK;
+    if (e == cudaErrorMemoryAllocation) return SKIP_ENOMEM;
+    return SKIP_ECUDA;
+}
+
+skip_status_t ensure_ws(skip_corpus *c, size_t bytes) {
+    if (bytes <= c->ws_bytes) return SKIP_OK;
+    if (c->ws) {
+        cudaError_t e = cudaDeviceSynchronize();
+        if (e != cudaSuccess) return SKIP_ECUDA;
+        cudaFree(c->ws);
+        c->ws = nullptr;
+        c->ws_bytes = 0;
+    }
+    size_t want = bytes + bytes / 4;
+    if (cudaMalloc(&c->ws, want) != cudaSuccess) {
+        cudaGetLastError();
+        return SKIP_ENOMEM;
+    }
+    c->ws_bytes = want;
+    return SKIP_OK;
+}
+
+void record(skip_corpus *c, cudaStream_t s, const char *name) {
+    if (!c->timing || c->n_ev >= kMaxEvents) return;
+    if (!c->ev[c->n_ev]) cudaEventCreate(&c->ev[c->n_ev]);
+    c->ev_name[c->n_ev] = name;
+    cudaEventRecord(c->ev[c->n_ev], s);
+    ++c->n_ev;
+}
+
+size_t align_up(size_t v, size_t a) { return (v + a - 1) / a * a; }
+
+struct Plan {
+    bool tensor = false;
+    int grid = 0;
+    int G = 0;          // lists per region row
+    int MB = 0;
+    int R_pad = 0;
+    int64_t tiles = 0;
+    int launches = 0;
+};
+
+// Corpus chunks G for the tensor path: make MB * G a whole number of waves of
+// `ctas` while keeping at least 4 tiles per item.
+int pick_chunks(int MB, int64_t tiles, int ctas) {
+    int best = 1;
+    double best_eff = -1.0;
+    const int gmax = (int)std::min<int64_t>(512, std::max<int64_t>(1, tiles / 4));
+    for (int G = 1; G <= gmax; ++G) {
+        const int64_t items = (int64_t)MB * G;
+        const int64_t waves = (items + ctas - 1) / ctas;
+        const double eff = (double)items / (double)(waves * ctas);
+        if (eff > best_eff + 1e-9) {
+            best_eff = eff;
+            best = G;
+        }
+        if (items >= 8LL * ctas) break;
+    }
+    return best;
+}
+
+skip_status_t check_common(skip_corpus *c, const void *regions, int32_t R_total, int32_t k_region) {
+    if (!c || R_total < 0) return SKIP_EINVAL;
+    if (R_total > 0 && !regions) return SKIP_EINVAL;
+    if (k_region < 1 || k_region > SKIP_MAX_K_REGION || (int64_t)k_region > c->N) return SKIP_EINVAL;
+    return SKIP_OK;
+}
+
+// Per-region step into reg_keys (or decoded ids/scores).  Shared by
+// skip_retrieve and skip_retrieve_regions.
+// When keys_out is non-null the keys go to the head of the workspace (the
+// first ws_extra bytes) and *keys_out receives their address.
+skip_status_t run_regions(skip_corpus *c, const uint16_t *regions, int R, int k, uint64_t **keys_out,
+                          int64_t *reg_ids, float *reg_scores, cudaStream_t s, Plan &pl,
+                          size_t ws_extra) {
+    uint64_t *reg_keys = nullptr;
+    const bool e4m3 = c->dtype == SKIP_E4M3;
+    const int ctas = c->grid > 0 ? c->grid : c->sm_count;
+    bool tensor;
+    if (c->path == SKIP_PATH_TENSOR)
+        tensor = true;
+    else if (c->path == SKIP_PATH_WARP)
+        tensor = false;
+    else
+        tensor = R > 8;
+    if (e4m3 || !c->tmap_ok) tensor = false;  // the tensor path streams bf16 tiles
+    pl.tensor = tensor;
+    if (tensor) {
+        pl.MB = (R + kTcTileM - 1) / kTcTileM;
+        pl.R_pad = pl.MB * kTcTileM;
+        pl.tiles = (c->N + kTcTileN - 1) / kTcTileN;
+        pl.G = pick_chunks(pl.MB, pl.tiles, ctas);
+        const int items = pl.MB * pl.G;
+        pl.grid = std::min(items, ctas);
+        const size_t lists_bytes = (size_t)pl.G * pl.R_pad * k * sizeof(uint64_t);
+        skip_status_t st = ensure_ws(c, align_up(ws_extra, 256) + lists_bytes);
+        if (st) return st;
+        uint64_t *lists = reinterpret_cast<uint64_t *>((char *)c->ws + align_up(ws_extra, 256));
+        if (keys_out) *keys_out = reg_keys = reinterpret_cast<uint64_t *>(c->ws);
+        CUtensorMap tq;
+        if (!encode_bf16_rows(&tq, regions, R, c->d, kTcTileM)) return SKIP_ECUDA;
+        TcParams p;
+        p.N = c->N;
+        p.d = c->d;
+        p.R = R;
+        p.R_pad = pl.R_pad;
+        p.k = k;
+        p.MB = pl.MB;
+        p.G = pl.G;
+        p.tiles = pl.tiles;
+        p.lists = lists;
+        p.err = c->err;
+        p.timeout_ns = c->timeout_ns;
+        record(c, s, "score_topk_tc");
+        cudaError_t e = launch_tc(tq, c->tmap_x, p, pl.grid, s);
+        if (e != cudaSuccess) return cuda_status(e);
+        ++pl.launches;
+        record(c, s, "merge_lists");
+        e = launch_merge_lists(lists, pl.G, (int64_t)pl.R_pad * k, R, k, reg_keys, reg_ids, reg_scores, s);
+        if (e != cudaSuccess) return cuda_status(e);
+        ++pl.launches;
+        return SKIP_OK;
+    }
+    // Warp-dot path: groups of up to 8 queries per launch.
+    pl.grid = (int)std::min<int64_t>(std::min<int64_t>((int64_t)ctas * 2, 512),
+                                     std::max<int64_t>(1, (c->N + 255) / 256));
+    pl.G = pl.grid;
+    pl.R_pad = R;
+    const size_t lists_bytes = (size_t)pl.grid * R * k * sizeof(uint64_t);
+    const size_t wl_bytes = (size_t)pl.grid * kWarpDotWarps * 8 * k * sizeof(uint64_t);
+    skip_status_t st = ensure_ws(c, align_up(ws_extra, 256) + align_up(lists_bytes, 256) + wl_bytes);
+    if (st) return st;
+    uint64_t *lists = reinterpret_cast<uint64_t *>((char *)c->ws + align_up(ws_extra, 256));
+    uint64_t *wl = reinterpret_cast<uint64_t *>((char *)lists + align_up(lists_bytes, 256));
+    if (keys_out) *keys_out = reg_keys = reinterpret_cast<uint64_t *>(c->ws);
+    record(c, s, "score_topk_warpdot");
+    for (int q0 = 0; q0 < R; q0 += 8) {
+        WarpDotParams p;
+        p.corpus = reinterpret_cast<const uint8_t *>(c->rows);
+        p.scale = c->scale;
+        p.N = c->N;
+        p.d = c->d;
+        p.regions = regions + (size_t)q0 * c->d;
+        p.nq = std::min(8, R - q0);
+        p.k = k;
+        p.warp_lists = wl;
+        p.lists = lists;
+        p.list_g_stride = (int64_t)R * k;
+        p.q0 = q0;
+        cudaError_t e = launch_warpdot(p, e4m3, pl.grid, s);
+        if (e != cudaSuccess) return cuda_status(e);
+        ++pl.launches;
+    }
+    record(c, s, "merge_lists");
+    cudaError_t e = launch_merge_lists(lists, pl.G, (int64_t)R * k, R, k, reg_keys, reg_ids, reg_scores, s);
+    if (e != cudaSuccess) return cuda_status(e);
+    ++pl.launches;
+    return SKIP_OK;
+}
+
+void write_plan(skip_corpus *c, const Plan &pl, int R, int Q, int k, int K) {
+    snprintf(c->plan, sizeof c->plan,
+             "{\"path\": \"%s\", \"grid\": %d, \"lists_per_row\": %d, \"query_blocks\": %d, "
+             "\"R_total\": %d, \"Q\": %d, \"k_region\": %d, \"K\": %d, \"launches\": %d}",
+             pl.tensor ? "tensor" : "warpdot", pl.grid, pl.G, pl.MB, R, Q, k, K, pl.launches);
+}
+
+}  // namespace
+
+extern "C" {
+
+const char *skip_status_string(skip_status_t s) {
+    switch (s) {
+        case SKIP_OK: return "ok";
+        case SKIP_EINVAL: return "invalid argument";
+        case SKIP_ENOMEM: return "out of device memory";
+        case SKIP_EUNSUPPORTED: return "unsupported device or size";
+        case SKIP_ETIMEOUT: return "a kernel wait timed out";
+        case SKIP_ECUDA: return "CUDA error";
+    }
+    return "unknown status";
+}
+
+skip_status_t skip_corpus_load(const void *rows, int rows_on_device, int64_t N, int32_t d,
+                               skip_dtype_t dtype, const float *row_scale, void *stream,
+                               skip_corpus_t *out) {
+    if (!out || !rows || N < 1 || N >= (1LL << 31) || d < 16 || d % 16 != 0 || d > kMaxD)
+        return SKIP_EINVAL;
+    if (dtype != SKIP_BF16 && dtype != SKIP_E4M3) return SKIP_EINVAL;
+    if ((dtype == SKIP_E4M3) != (row_scale != nullptr)) return SKIP_EINVAL;
+    *out = nullptr;
+    int dev = 0;
+    if (cudaGetDevice(&dev) != cudaSuccess) {
+        cudaGetLastError();
+        return SKIP_EUNSUPPORTED;
+    }
+    int major = 0, minor = 0, sms = 0;
+    cudaDeviceGetAttribute(&major, cudaDevAttrComputeCapabilityMajor, dev);
+    cudaDeviceGetAttribute(&minor, cudaDevAttrComputeCapabilityMinor, dev);
+    cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev);
+    if (major != 10 || minor != 3) return SKIP_EUNSUPPORTED;
+
+    skip_corpus *c = new (std::nothrow) skip_corpus();
+    if (!c) return SKIP_ENOMEM;
+    c->device = dev;
+    c->sm_count = sms;
+    c->N = N;
+    c->d = d;
+    c->dtype = dtype;
+    const size_t elem = dtype == SKIP_BF16 ? 2 : 1;
+    const size_t bytes = (size_t)N * d * elem;
+    cudaStream_t s = reinterpret_cast<cudaStream_t>(stream);
+    skip_status_t st = SKIP_OK;
+    if (cudaMalloc(&c->rows, bytes) != cudaSuccess || cudaMalloc(&c->err, sizeof(int)) != cudaSuccess ||
+        (dtype == SKIP_E4M3 && cudaMalloc(&c->scale, N * sizeof(float)) != cudaSuccess)) {
+        cudaGetLastError();
+        st = SKIP_ENOMEM;
+    }
+    const cudaMemcpyKind kind = rows_on_device ? cudaMemcpyDeviceToDevice : cudaMemcpyHostToDevice;
+    if (!st) st = cuda_status(cudaMemcpyAsync(c->rows, rows, bytes, kind, s));
+    if (!st && c->scale) st = cuda_status(cudaMemcpyAsync(c->scale, row_scale, N * sizeof(float), kind, s));
+    if (!st) st = cuda_status(cudaMemsetAsync(c->err, 0, sizeof(int), s));
+    if (!st) st = cuda_status(cudaStreamSynchronize(s));
+    if (!st && dtype == SKIP_BF16) c->tmap_ok = encode_bf16_rows(&c->tmap_x, c->rows, N, d, kTcTileN);
+    if (st) {
+        skip_corpus_free(c);
+        return st;
+    }
+    *out = c;
+    return SKIP_OK;
+}
+
+skip_status_t skip_corpus_free(skip_corpus_t c) {
+    if (!c) return SKIP_OK;
+    cudaDeviceSynchronize();
+    cudaFree(c->rows);
+    cudaFree(c->scale);
+    cudaFree(c->err);
+    cudaFree(c->ws);
+    cudaFree(c->io);
+    for (int i = 0; i < kMaxEvents; ++i)
+        if (c->ev[i]) cudaEventDestroy(c->ev[i]);
+    delete c;
+    return SKIP_OK;
+}
+
+skip_status_t skip_corpus_set_option(skip_corpus_t c, int option, int64_t value) {
+    if (!c) return SKIP_EINVAL;
+    switch (option) {
+        case SKIP_OPT_PATH:
+            if (value < SKIP_PATH_AUTO || value > SKIP_PATH_WARP) return SKIP_EINVAL;
+            c->path = (int)value;
+            return SKIP_OK;
+        case SKIP_OPT_WAIT_TIMEOUT_NS:
+            if (value < 0) return SKIP_EINVAL;
+            c->timeout_ns = (uint64_t)value;
+            return SKIP_OK;
+        case SKIP_OPT_GRID:
+            if (value < 0 || value > 65535) return SKIP_EINVAL;
+            c->grid = (int)value;
+            return SKIP_OK;
+        case SKIP_OPT_TIMING:
+            c->timing = value != 0;
+            return SKIP_OK;
+    }
+    return SKIP_EINVAL;
+}
+
+skip_status_t skip_retrieve(skip_corpus_t c, const void *regions, const int32_t *region_offsets,
+                            int32_t Q, int32_t R_total, int32_t k_region, int32_t K, int64_t *out_ids,
+                            float *out_scores, void *stream) {
+    skip_status_t st = check_common(c, regions, R_total, k_region);
+    if (st) return st;
+    if (Q < 0 || K < 1 || K > SKIP_MAX_K || (Q > 0 && !region_offsets)) return SKIP_EINVAL;
+    if (Q > 0 && (!out_ids || !out_scores)) return SKIP_EINVAL;
+    if (Q == 0 && R_total != 0) return SKIP_EINVAL;
+    cudaStream_t s = reinterpret_cast<cudaStream_t>(stream);
+    c->n_ev = 0;
+    Plan pl;
+    const size_t keys_bytes = align_up((size_t)std::max(R_total, 1) * k_region * sizeof(uint64_t), 256);
+    uint64_t *reg_keys = nullptr;
+    if (R_total > 0) {
+        st = run_regions(c, reinterpret_cast<const uint16_t *>(regions), R_total, k_region, &reg_keys,
+                         nullptr, nullptr, s, pl, keys_bytes);
+        if (st) return st;
+    } else {
+        st = ensure_ws(c, keys_bytes);
+        if (st) return st;
+        reg_keys = reinterpret_cast<uint64_t *>(c->ws);
+    }
+    if (Q > 0) {
+        record(c, s, "question_merge");
+        cudaError_t e = launch_question_merge(reg_keys, k_region, region_offsets, Q, R_total, K, out_ids,
+                                              out_scores, c->err, s);
+        if (e != cudaSuccess) return cuda_status(e);
+        ++pl.launches;
+    }
+    record(c, s, "end");
+    write_plan(c, pl, R_total, Q, k_region, K);
+    return SKIP_OK;
+}
+
+skip_status_t skip_retrieve_regions(skip_corpus_t c, const void *regions, int32_t R_total,
+                                    int32_t k_region, int64_t *reg_ids, float *reg_scores,
+                                    void *stream) {
+    skip_status_t st = check_common(c, regions, R_total, k_region);
+    if (st) return st;
+    if (R_total > 0 && (!reg_ids || !reg_scores)) return SKIP_EINVAL;
+    cudaStream_t s = reinterpret_cast<cudaStream_t>(stream);
+    c->n_ev = 0;
+    Plan pl;
+    if (R_total > 0) {
+        st = run_regions(c, reinterpret_cast<const uint16_t *>(regions), R_total, k_region, nullptr, reg_ids,
+                         reg_scores, s, pl, 0);
+        if (st) return st;
+    }
+    record(c, s, "end");
+    write_plan(c, pl, R_total, 0, k_region, 0);
+    return SKIP_OK;
+}
+
+skip_status_t skip_sync_status(skip_corpus_t c, void *stream) {
+    if (!c) return SKIP_EINVAL;
+    cudaStream_t s = reinterpret_cast<cudaStream_t>(stream);
+    if (cudaStreamSynchronize(s) != cudaSuccess) return SKIP_ECUDA;
+    int err = 0;
+    if (cudaMemcpy(&err, c->err, sizeof(int), cudaMemcpyDeviceToHost) != cudaSuccess) return SKIP_ECUDA;
+    if (err) {
+        if (cudaMemset(c->err, 0, sizeof(int)) != cudaSuccess) return SKIP_ECUDA;
+        return (err & kErrTimeout) ? SKIP_ETIMEOUT : SKIP_EINVAL;
+    }
+    return SKIP_OK;
+}
+
+skip_status_t skip_retrieve_host(skip_corpus_t c, const uint16_t *regions, const int32_t *region_offsets,
+                                 int32_t Q, int32_t R_total, int32_t k_region, int32_t K, int64_t *out_ids,
+                                 float *out_scores, void *stream) {
+    skip_status_t st = check_common(c, regions, R_total, k_region);
+    if (st) return st;
+    if (Q < 0 || K < 1 || K > SKIP_MAX_K || (Q > 0 && (!region_offsets || !out_ids || !out_scores)))
+        return SKIP_EINVAL;
+    cudaStream_t s = reinterpret_cast<cudaStream_t>(stream);
+    const size_t rb = align_up((size_t)R_total * c->d * 2, 256);
+    const size_t ob = align_up((size_t)(Q + 1) * sizeof(int32_t), 256);
+    const size_t ib = align_up((size_t)Q * K * sizeof(int64_t), 256);
+    const size_t sb = align_up((size_t)Q * K * sizeof(float), 256);
+    const size_t need = rb + ob + ib + sb;
+    if (need > c->io_bytes) {
+        if (c->io) {
+            if (cudaDeviceSynchronize() != cudaSuccess) return SKIP_ECUDA;
+            cudaFree(c->io);
+            c->io = nullptr;
+            c->io_bytes = 0;
+        }
+        if (cudaMalloc(&c->io, need) != cudaSuccess) {
+            cudaGetLastError();
+            return SKIP_ENOMEM;
+        }
+        c->io_bytes = need;
+    }
+    char *io = reinterpret_cast<char *>(c->io);
+    void *d_reg = io;
+    int32_t *d_off = reinterpret_cast<int32_t *>(io + rb);
+    int64_t *d_ids = reinterpret_cast<int64_t *>(io + rb + ob);
+    float *d_sc = reinterpret_cast<float *>(io + rb + ob + ib);
+    if (R_total > 0) {
+        st = cuda_status(cudaMemcpyAsync(d_reg, regions, (size_t)R_total * c->d * 2, cudaMemcpyHostToDevice, s));
+        if (st) return st;
+    }
+    if (Q > 0) {
+        st = cuda_status(cudaMemcpyAsync(d_off, region_offsets, (size_t)(Q + 1) * sizeof(int32_t),
+                                         cudaMemcpyHostToDevice, s));
+        if (st) return st;
+    }
+    st = skip_retrieve(c, R_total > 0 ? d_reg : nullptr, d_off, Q, R_total, k_region, K, d_ids, d_sc, stream);
+    if (st) return st;
+    if (Q > 0) {
+        st = cuda_status(cudaMemcpyAsync(out_ids, d_ids, (size_t)Q * K * sizeof(int64_t), cudaMemcpyDeviceToHost, s));
+        if (!st)
+            st = cuda_status(cudaMemcpyAsync(out_scores, d_sc, (size_t)Q * K * sizeof(float), cudaMemcpyDeviceToHost, s));
+        if (st) return st;
+    }
+    return skip_sync_status(c, stream);
+}
+
+skip_status_t skip_last_plan(skip_corpus_t c, char *buf, int32_t len) {
+    if (!c || !buf || len < 1) return SKIP_EINVAL;
+    char times[256] = "";
+    if (c->timing && c->n_ev > 1) {
+        int at = snprintf(times, sizeof times, ", \"ms\": {");
+        for (int i = 0; i + 1 < c->n_ev && at < (int)sizeof times; ++i) {
+            float ms = 0.0f;
+            if (cudaEventSynchronize(c->ev[i + 1]) != cudaSuccess ||
+                cudaEventElapsedTime(&ms, c->ev[i], c->ev[i + 1]) != cudaSuccess)
+                return SKIP_ECUDA;
+            at += snprintf(times + at, sizeof times - at, "%s\"%s\": %.6f", i ? ", " : "", c->ev_name[i], ms);
+        }
+        if (at < (int)sizeof times) snprintf(times + at, sizeof times - at, "}");
+    }
+    const int plen = (int)strlen(c->plan);
+    snprintf(buf, len, "%.*s%s}", plen > 0 ? plen - 1 : 0, c->plan, times);
+    return SKIP_OK;
+}
+
+}  // extern "C"

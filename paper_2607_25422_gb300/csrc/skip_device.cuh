@@ -1,0 +1,320 @@
+// Device-side building blocks shared by the retrieval kernels: the
+// order-preserving (score, id) key, sorted-list insertion, warp reductions,
+// bounded mbarrier waits, and thin inline-PTX wrappers for TMA and tcgen05
+// (sm_103a).
+#pragma once
+
+#include <cuda.h>
+#include <cuda_bf16.h>
+#include <cuda_fp8.h>
+#include <cuda_runtime.h>
+#include <stdint.h>
+
+namespace skipk {
+
+// ---------------------------------------------------------------- keys
+//
+// A candidate (score s, id i) is packed into one 64-bit key whose unsigned
+// order is the ranking order of the method: higher score first, and on equal
+// scores the lower id first.  High word: the float's bits mapped so that
+// unsigned order follows float order (-0 is folded onto +0 so that the two
+// zeros tie).  Low word: 0xFFFFFFFF - id.  Key 0 is the empty slot; it ranks
+// after every real candidate.
+
+__device__ __forceinline__ uint32_t ord_of_score(float s) {
+    uint32_t u = __float_as_uint(s + 0.0f);
+    return (u & 0x80000000u) ? ~u : (u | 0x80000000u);
+}
+
+__device__ __forceinline__ float score_of_ord(uint32_t o) {
+    uint32_t u = (o & 0x80000000u) ? (o & 0x7FFFFFFFu) : ~o;
+    return __uint_as_float(u);
+}
+
+__device__ __forceinline__ uint64_t make_key(float s, uint32_t id) {
+    return ((uint64_t)ord_of_score(s) << 32) | (uint64_t)(0xFFFFFFFFu - id);
+}
+
+__device__ __forceinline__ float key_score(uint64_t k) { return score_of_ord((uint32_t)(k >> 32)); }
+__device__ __forceinline__ int64_t key_id(uint64_t k) {
+    return (int64_t)(0xFFFFFFFFu - (uint32_t)k);
+}
+
+__device__ __forceinline__ void key_decode(uint64_t k, int64_t &id, float &s) {
+    if (k == 0) {
+        id = -1;
+        s = -__int_as_float(0x7f800000);
+    } else {
+        id = key_id(k);
+        s = key_score(k);
+    }
+}
+
+// Insert `key` into `list` (k slots, the first n valid, sorted descending).
+// Caller guarantees n < k or key > list[k-1].  Returns the new k-th key
+// (0 while the list is not full).
+__device__ __forceinline__ uint64_t sorted_insert(uint64_t *list, int &n, int k, uint64_t key) {
+    int pos = n < k ? n : k - 1;
+    while (pos > 0) {
+        uint64_t prev = list[pos - 1];
+        if (prev >= key) break;
+        list[pos] = prev;
+        --pos;
+    }
+    list[pos] = key;
+    if (n < k) ++n;
+    return n == k ? list[k - 1] : 0ull;
+}
+
+__device__ __forceinline__ uint64_t warp_max_u64(uint64_t v) {
+#pragma unroll
+    for (int o = 16; o; o >>= 1) {
+        uint64_t w = __shfl_xor_sync(0xffffffffu, v, o);
+        v = w > v ? w : v;
+    }
+    return v;
+}
+
+// ---------------------------------------------------------------- timing
+
+__device__ __forceinline__ uint64_t globaltimer_ns() {
+    uint64_t t;
+    asm volatile("mov.u64 %0, %%globaltimer;" : "=l"(t));
+    return t;
+}
+
+// ---------------------------------------------------------------- mbarrier
+
+__device__ __forceinline__ uint32_t smem_addr(const void *p) {
+    return (uint32_t)__cvta_generic_to_shared(p);
+}
+
+__device__ __forceinline__ void mbar_init(uint32_t bar, uint32_t count) {
+    asm volatile("mbarrier.init.shared::cta.b64 [%0], %1;" ::"r"(bar), "r"(count) : "memory");
+}
+
+__device__ __forceinline__ void mbar_fence_init() {
+    asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
+}
+
+__device__ __forceinline__ void mbar_arrive(uint32_t bar) {
+    asm volatile("mbarrier.arrive.shared::cta.b64 _, [%0];" ::"r"(bar) : "memory");
+}
+
+__device__ __forceinline__ void mbar_arrive_expect_tx(uint32_t bar, uint32_t bytes) {
+    asm volatile("mbarrier.arrive.expect_tx.shared::cta.b64 _, [%0], %1;" ::"r"(bar), "r"(bytes)
+                 : "memory");
+}
+
+__device__ __forceinline__ bool mbar_try_wait(uint32_t bar, uint32_t parity) {
+    uint32_t ok;
+    asm volatile(
+        "{\n\t.reg .pred p;\n\t"
+        "mbarrier.try_wait.parity.shared::cta.b64 p, [%1], %2;\n\t"
+        "selp.u32 %0, 1, 0, p;\n\t}"
+        : "=r"(ok)
+        : "r"(bar), "r"(parity)
+        : "memory");
+    return ok != 0;
+}
+
+// Wait until the phase with the given parity has completed, for at most
+// timeout_ns.  Returns false when the wait gave up.
+__device__ __forceinline__ bool mbar_wait(uint32_t bar, uint32_t parity, uint64_t timeout_ns) {
+    if (mbar_try_wait(bar, parity)) return true;
+    uint64_t t0 = globaltimer_ns();
+    for (;;) {
+        if (mbar_try_wait(bar, parity)) return true;
+        if (globaltimer_ns() - t0 > timeout_ns) return false;
+    }
+}
+
+// ---------------------------------------------------------------- TMA
+
+__device__ __forceinline__ void tma_prefetch_desc(const void *map) {
+    asm volatile("prefetch.tensormap [%0];" ::"l"(map) : "memory");
+}
+
+// 2D tiled bulk tensor copy global -> shared; completion is counted on `bar`
+// in bytes.  x is the innermost (element) coordinate, y the row.
+__device__ __forceinline__ void tma_load_2d(uint32_t dst, const void *map, uint32_t bar, int x,
+                                            int y) {
+    asm volatile(
+        "cp.async.bulk.tensor.2d.shared::cluster.global.mbarrier::complete_tx::bytes"
+        " [%0], [%1, {%3, %4}], [%2];" ::"r"(dst),
+        "l"(map), "r"(bar), "r"(x), "r"(y)
+        : "memory");
+}
+
+__device__ __forceinline__ void tma_load_2d_hint(uint32_t dst, const void *map, uint32_t bar, int x,
+                                                 int y, uint64_t policy) {
+    asm volatile(
+        "cp.async.bulk.tensor.2d.shared::cluster.global.mbarrier::complete_tx::bytes.L2::cache_hint"
+        " [%0], [%1, {%3, %4}], [%2], %5;" ::"r"(dst),
+        "l"(map), "r"(bar), "r"(x), "r"(y), "l"(policy)
+        : "memory");
+}
+
+__device__ __forceinline__ uint64_t l2_policy_evict_last() {
+    uint64_t p;
+    asm volatile("createpolicy.fractional.L2::evict_last.b64 %0, 1.0;" : "=l"(p));
+    return p;
+}
+
+__device__ __forceinline__ uint64_t l2_policy_evict_first() {
+    uint64_t p;
+    asm volatile("createpolicy.fractional.L2::evict_first.b64 %0, 1.0;" : "=l"(p));
+    return p;
+}
+
+// ---------------------------------------------------------------- tcgen05
+
+__device__ __forceinline__ void tmem_alloc(uint32_t dst_smem, uint32_t ncols) {
+    asm volatile("tcgen05.alloc.cta_group::1.sync.aligned.shared::cta.b32 [%0], %1;" ::"r"(dst_smem),
+                 "r"(ncols)
+                 : "memory");
+}
+
+__device__ __forceinline__ void tmem_relinquish() {
+    asm volatile("tcgen05.relinquish_alloc_permit.cta_group::1.sync.aligned;" ::: "memory");
+}
+
+__device__ __forceinline__ void tmem_dealloc(uint32_t taddr, uint32_t ncols) {
+    asm volatile("tcgen05.dealloc.cta_group::1.sync.aligned.b32 %0, %1;" ::"r"(taddr), "r"(ncols)
+                 : "memory");
+}
+
+__device__ __forceinline__ void tc_fence_before() {
+    asm volatile("tcgen05.fence::before_thread_sync;" ::: "memory");
+}
+
+__device__ __forceinline__ void tc_fence_after() {
+    asm volatile("tcgen05.fence::after_thread_sync;" ::: "memory");
+}
+
+// D[tmem] (+)= A[smem] * B[smem]^T, bf16 inputs, fp32 accumulate.
+__device__ __forceinline__ void tc_mma_f16(uint32_t d_tmem, uint64_t adesc, uint64_t bdesc,
+                                           uint32_t idesc, uint32_t accumulate) {
+    asm volatile(
+        "{\n\t.reg .pred p;\n\t"
+        "setp.ne.b32 p, %4, 0;\n\t"
+        "tcgen05.mma.cta_group::1.kind::f16 [%0], %1, %2, %3, p;\n\t}" ::"r"(d_tmem),
+        "l"(adesc), "l"(bdesc), "r"(idesc), "r"(accumulate)
+        : "memory");
+}
+
+// Arrive once on `bar` when every tcgen05 op issued so far by this thread
+// has completed.
+__device__ __forceinline__ void tc_commit(uint32_t bar) {
+    asm volatile("tcgen05.commit.cta_group::1.mbarrier::arrive::one.shared::cluster.b64 [%0];" ::"r"(
+                     bar)
+                 : "memory");
+}
+
+// 32 lanes x 32 consecutive 32-bit columns; thread t of the warp receives
+// lane (base lane + t).
+__device__ __forceinline__ void tmem_ld_32x32b_x32(uint32_t taddr, uint32_t (&v)[32]) {
+    asm volatile(
+        "tcgen05.ld.sync.aligned.32x32b.x32.b32 "
+        "{%0,%1,%2,%3,%4,%5,%6,%7,%8,%9,%10,%11,%12,%13,%14,%15,"
+        "%16,%17,%18,%19,%20,%21,%22,%23,%24,%25,%26,%27,%28,%29,%30,%31}, [%32];"
+        : "=r"(v[0]), "=r"(v[1]), "=r"(v[2]), "=r"(v[3]), "=r"(v[4]), "=r"(v[5]), "=r"(v[6]),
+          "=r"(v[7]), "=r"(v[8]), "=r"(v[9]), "=r"(v[10]), "=r"(v[11]), "=r"(v[12]), "=r"(v[13]),
+          "=r"(v[14]), "=r"(v[15]), "=r"(v[16]), "=r"(v[17]), "=r"(v[18]), "=r"(v[19]),
+          "=r"(v[20]), "=r"(v[21]), "=r"(v[22]), "=r"(v[23]), "=r"(v[24]), "=r"(v[25]),
+          "=r"(v[26]), "=r"(v[27]), "=r"(v[28]), "=r"(v[29]), "=r"(v[30]), "=r"(v[31])
+        : "r"(taddr)
+        : "memory");
+}
+
+// Wait for this thread's tcgen05.ld results.  The registers are threaded
+// through the asm so that no use of them is scheduled before the wait.
+__device__ __forceinline__ void tmem_ld_wait(uint32_t (&v)[32]) {
+    asm volatile("tcgen05.wait::ld.sync.aligned;"
+                 : "+r"(v[0]), "+r"(v[1]), "+r"(v[2]), "+r"(v[3]), "+r"(v[4]), "+r"(v[5]),
+                   "+r"(v[6]), "+r"(v[7]), "+r"(v[8]), "+r"(v[9]), "+r"(v[10]), "+r"(v[11]),
+                   "+r"(v[12]), "+r"(v[13]), "+r"(v[14]), "+r"(v[15]), "+r"(v[16]), "+r"(v[17]),
+                   "+r"(v[18]), "+r"(v[19]), "+r"(v[20]), "+r"(v[21]), "+r"(v[22]), "+r"(v[23]),
+                   "+r"(v[24]), "+r"(v[25]), "+r"(v[26]), "+r"(v[27]), "+r"(v[28]), "+r"(v[29]),
+                   "+r"(v[30]), "+r"(v[31])
+                 :
+                 : "memory");
+}
+
+// Shared-memory matrix descriptor for a K-major operand tile stored with the
+// 128-byte swizzle (rows of 128 bytes, 8-row groups 1024 bytes apart), as TMA
+// writes it with CU_TENSOR_MAP_SWIZZLE_128B.  The tile must start on a
+// 1024-byte boundary; stepping along K inside the 128-byte row adds the byte
+// offset to the start address field.
+__device__ __forceinline__ uint64_t smem_desc_k128(uint32_t saddr) {
+    uint64_t d = 0;
+    d |= (uint64_t)((saddr & 0x3FFFFu) >> 4);       // start address  [0,14)
+    d |= (uint64_t)1 << 16;                          // leading byte offset (unused here) [16,30)
+    d |= (uint64_t)(1024u >> 4) << 32;               // stride byte offset: 8 rows x 128 B [32,46)
+    d |= (uint64_t)1 << 46;                          // descriptor version for tcgen05 [46,48)
+    d |= (uint64_t)2 << 61;                          // swizzle: 128-byte [61,64)
+    return d;
+}
+
+// Instruction descriptor for kind::f16: bf16 A and B, fp32 D, both K-major,
+// dense, tile M x N.
+__host__ __device__ constexpr uint32_t idesc_bf16_f32(int M, int N) {
+    return (1u << 4)                       // D format: f32
+           | (1u << 7)                     // A format: bf16
+           | (1u << 10)                    // B format: bf16
+           | ((uint32_t)(N >> 3) << 17)    // N / 8
+           | ((uint32_t)(M >> 4) << 24);   // M / 16
+}
+
+
+// ---------------------------------------------------------------- merging
+
+// Warp-cooperative merge of `nl` lists, each sorted descending with `len`
+// slots (list t starts at base + t * stride; empty slots hold key 0), into
+// the first k keys of their union, emitted in descending order through
+// emit(i, key).  Lane l owns lists l, l + 32, ... (at most 32 * LPL lists).
+// Each round takes the largest head in the warp and advances the list it
+// came from; the head's successor is prefetched one step ahead.
+template <int LPL, typename Emit>
+__device__ __forceinline__ void warp_merge_topk(const uint64_t *base, int64_t stride, int nl, int len,
+                                                int k, Emit emit) {
+    const int lane = threadIdx.x & 31;
+    uint64_t head[LPL], next[LPL];
+    int pos[LPL];
+#pragma unroll
+    for (int t = 0; t < LPL; ++t) {
+        const int l = lane + 32 * t;
+        pos[t] = 0;
+        head[t] = (l < nl && len > 0) ? base[(int64_t)l * stride] : 0ull;
+        next[t] = (l < nl && len > 1) ? base[(int64_t)l * stride + 1] : 0ull;
+    }
+    for (int i = 0; i < k; ++i) {
+        uint64_t best = 0;
+        int bt = 0;
+#pragma unroll
+        for (int t = 0; t < LPL; ++t)
+            if (head[t] > best) {
+                best = head[t];
+                bt = t;
+            }
+        const uint64_t m = warp_max_u64(best);
+        if (m == 0) {
+            for (int j = i + lane; j < k; j += 32) emit(j, 0ull);
+            return;
+        }
+        if (lane == 0) emit(i, m);
+        const unsigned owners = __ballot_sync(0xffffffffu, best == m);
+        if (lane == __ffs(owners) - 1) {
+#pragma unroll
+            for (int t = 0; t < LPL; ++t)
+                if (t == bt) {
+                    const int l = lane + 32 * t;
+                    ++pos[t];
+                    head[t] = next[t];
+                    next[t] = (pos[t] + 1 < len) ? base[(int64_t)l * stride + pos[t] + 1] : 0ull;
+                }
+        }
+    }
+}
+
+}  // namespace skipk

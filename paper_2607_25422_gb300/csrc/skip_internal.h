@@ -1,0 +1,66 @@
+// Host-side declarations shared by the C-ABI layer and the kernel files.
+#pragma once
+
+#include <cuda.h>
+#include <cuda_runtime.h>
+#include <stdint.h>
+
+namespace skipk {
+
+// Bits of the per-handle device error word.
+enum : int { kErrTimeout = 1, kErrConfig = 2 };
+
+// ---- warp-dot score + top-k (small region batches) -------------------
+struct WarpDotParams {
+    const uint8_t *corpus;   // [N x d] rows, d * elem_bytes bytes apart
+    const float *scale;      // [N] (e4m3 only)
+    int64_t N;
+    int d;
+    const uint16_t *regions; // bf16 bits; rows [q0, q0 + nq) of the batch
+    int nq;                  // queries in this launch (<= 8)
+    int k;
+    uint64_t *warp_lists;    // [grid][kWarpDotWarps][nq][k] scratch
+    uint64_t *lists;         // [grid][R_pad][k]; this launch writes rows q0..q0+nq
+    int64_t list_g_stride;   // elements between consecutive grid lists (R_pad * k)
+    int q0;
+};
+constexpr int kWarpDotWarps = 8;
+constexpr int kWarpDotThreads = kWarpDotWarps * 32;
+cudaError_t launch_warpdot(const WarpDotParams &p, bool e4m3, int grid, cudaStream_t s);
+
+// ---- tensor-core score + top-k -----------------------------------------
+struct TcParams {
+    int64_t N;
+    int d;
+    int R;            // region rows
+    int R_pad;        // query blocks * 128
+    int k;
+    int MB;           // query blocks of 128 rows
+    int G;            // corpus chunks (lists per row)
+    int64_t tiles;    // corpus tiles of kTcTileN rows
+    uint64_t *lists;  // [G][R_pad][k]
+    int *err;
+    uint64_t timeout_ns;
+};
+constexpr int kTcTileM = 128;   // region rows per tile (TMEM lanes)
+constexpr int kTcTileN = 256;   // corpus rows per tile (TMEM columns)
+constexpr int kTcTileK = 64;    // bf16 elements per stage row (128 bytes)
+constexpr int kTcStages = 4;
+constexpr int kTcThreads = 192; // producer warp, MMA warp, 4 epilogue warps
+size_t tc_smem_bytes();
+cudaError_t launch_tc(const CUtensorMap &tq, const CUtensorMap &tx, const TcParams &p, int grid,
+                      cudaStream_t s);
+
+// ---- merges -------------------------------------------------------------
+// Per-region merge of G sorted lists into the exact top-k (keys and/or
+// decoded ids/scores).
+cudaError_t launch_merge_lists(const uint64_t *lists, int G, int64_t g_stride, int R, int k,
+                               uint64_t *reg_keys, int64_t *reg_ids, float *reg_scores,
+                               cudaStream_t s);
+// Per-question union + dedup (max score) + top-K.
+// Offsets are clamped to [0, R]; a clamp sets kErrConfig in *err.
+cudaError_t launch_question_merge(const uint64_t *reg_keys, int k, const int32_t *offsets, int Q,
+                                  int R, int K, int64_t *out_ids, float *out_scores, int *err,
+                                  cudaStream_t s);
+
+}  // namespace skipk
