@@ -1,0 +1,397 @@
+#!/usr/bin/env python
+"""Throughput of region-conditional sparse retrieval on GB300.
+
+A step is one call of the whole path (per-region MIPS top-k over the corpus,
+cross-partition merge, per-question dedup and top-K; paper §3.3 Eq. rcsr,
+App. B.2 Def. B.2, Alg. 1) on one batch of questions whose region embeddings
+and corpus are already resident in HBM.  The default workload is the 1M-row
+clustered corpus (N = 1,000,000 x d = 768 bf16, 64 questions x 16 regions,
+k_region = 20, K = 50).  The corpus (1.54 GB) is larger than L2 (129 MB), so
+every step streams it from HBM without an explicit flush.
+
+Printed as one JSON line: questions/s (``value``), corpus GB/s, region rows/s,
+TFLOP/s, the roofline of the dominant kernel (CUDA events on the launching
+stream, recorded by the library around each kernel), clocks sampled during the
+timed region, the end-to-end rate through the host-buffer entry point
+(host->device copies and result read-back inside the timed region), and the
+CPU oracle timed on a bounded sample of the same workload.
+
+Multi-GPU (torchrun): each rank holds a replica of the corpus and serves its
+own batch of questions (weak scaling); ranks exchange nothing on the data
+path, only the barrier and the max of the timings.
+
+``--impl reference`` times the CPU oracle instead (rank 0 only), one question
+per step over a prefix of the corpus, scaled to full-corpus questions/s.
+"""
+from __future__ import annotations
+
+import argparse
+import hashlib
+import json
+import os
+import statistics
+import subprocess
+import sys
+import time
+
+import numpy as np
+import torch
+
+ROOT = os.path.dirname(os.path.abspath(__file__))
+sys.path.insert(0, ROOT)
+
+import synth  # noqa: E402
+
+METRIC = "retrieval queries/s and corpus GB/s (1 GB300) as fraction of roofline"
+SCORE_KERNELS = ("score_topk_tc", "score_topk_warpdot")
+KERNEL_SOURCES = {
+    "score_topk_tc": ["paper_2607_25422_gb300/csrc/k_tc.cu", "paper_2607_25422_gb300/csrc/skip_device.cuh"],
+    "score_topk_warpdot": ["paper_2607_25422_gb300/csrc/k_warpdot.cu",
+                           "paper_2607_25422_gb300/csrc/skip_device.cuh"],
+}
+
+
+def load_peaks():
+    p = os.path.join(ROOT, "MEASURED_PEAKS.json")
+    if os.path.exists(p):
+        with open(p) as f:
+            m = json.load(f)
+        return {"hbm_gbs": m["hbm_gbs"], "bf16_tflops": m["bf16_tflops"],
+                "bf16_tflops_sustained": m.get("bf16_tflops_sustained"), "source": "measured"}
+    return {"hbm_gbs": 6800.0, "bf16_tflops": 1900.0, "bf16_tflops_sustained": 1700.0, "source": "fallback"}
+
+
+def source_sha(kernel):
+    h = hashlib.sha256()
+    for rel in KERNEL_SOURCES.get(kernel, []):
+        with open(os.path.join(ROOT, rel), "rb") as f:
+            h.update(f.read())
+    return h.hexdigest()[:16]
+
+
+def profiled_traffic(kernel, workload):
+    """DRAM bytes per launch from a committed ncu summary, if it was taken
+    on the kernel as it is now."""
+    p = os.path.join(ROOT, "profiles", "%s_%s.json" % (kernel, workload))
+    if not os.path.exists(p):
+        return None
+    with open(p) as f:
+        s = json.load(f)
+    if s.get("source_sha") != source_sha(kernel):
+        return None
+    return s.get("dram_bytes_per_launch")
+
+
+class ClockSampler:
+    """nvidia-smi clocks and throttle reasons sampled every 100 ms."""
+
+    FIELDS = ("index,clocks.sm,clocks.max.sm,power.draw,clocks_event_reasons.active,"
+              "clocks_event_reasons.hw_slowdown,clocks_event_reasons.hw_thermal_slowdown,"
+              "clocks_event_reasons.sw_thermal_slowdown,clocks_event_reasons.sw_power_cap")
+
+    def __init__(self, index):
+        self.index = index
+        self.proc = None
+
+    def start(self):
+        try:
+            self.proc = subprocess.Popen(
+                ["nvidia-smi", "-i", str(self.index), "--query-gpu=" + self.FIELDS,
+                 "--format=csv,noheader,nounits", "-lms", "100"],
+                stdout=subprocess.PIPE, stderr=subprocess.DEVNULL, text=True)
+        except OSError:
+            self.proc = None
+
+    def stop(self):
+        if self.proc is None:
+            return {"samples": 0}
+        self.proc.terminate()
+        try:
+            out, _ = self.proc.communicate(timeout=5)
+        except subprocess.TimeoutExpired:
+            self.proc.kill()
+            out, _ = self.proc.communicate()
+        sm, mx, reasons = [], [], set()
+        names = ("hw_slowdown", "hw_thermal_slowdown", "sw_thermal_slowdown", "sw_power_cap")
+        for line in out.strip().splitlines():
+            f = [x.strip() for x in line.split(",")]
+            if len(f) < 9:
+                continue
+            try:
+                sm.append(float(f[1]))
+                mx.append(float(f[2]))
+            except ValueError:
+                continue
+            for n, v in zip(names, f[5:9]):
+                if v.lower().startswith("active"):
+                    reasons.add(n)
+        if not sm:
+            return {"samples": 0}
+        return {"sm_mhz": statistics.median(sm), "sm_max_mhz": max(mx), "reasons": sorted(reasons),
+                "samples": len(sm)}
+
+
+def dist_setup():
+    world = int(os.environ.get("WORLD_SIZE", "1"))
+    rank = int(os.environ.get("RANK", "0"))
+    local = int(os.environ.get("LOCAL_RANK", "0"))
+    if world > 1:
+        import torch.distributed as dist
+        torch.cuda.set_device(local)
+        dist.init_process_group("nccl", device_id=torch.device("cuda", local))
+    else:
+        torch.cuda.set_device(0)
+    return world, rank, local
+
+
+def barrier(world):
+    if world > 1:
+        import torch.distributed as dist
+        dist.barrier()
+
+
+def max_over_ranks(x, world):
+    if world == 1:
+        return x
+    import torch.distributed as dist
+    t = torch.tensor([x], dtype=torch.float64, device="cuda")
+    dist.all_reduce(t, op=dist.ReduceOp.MAX)
+    return float(t.item())
+
+
+def workload_config(spec, R_total, world):
+    lo, hi = spec.regions
+    return {
+        "workload": spec.name, "N": spec.N, "d": spec.d, "corpus_dtype": spec.dtype,
+        "questions_per_gpu": spec.Q, "regions_per_question": lo if lo == hi else "U{%d..%d}" % (lo, hi),
+        "R_total_per_gpu": R_total, "k_region": spec.k_region, "K": spec.K, "corpus": spec.corpus,
+        "l2": "inputs larger than L2 (corpus %.2f GB > 129 MB), no flush" % (
+            spec.N * spec.d * (2 if spec.dtype == "bf16" else 1) / 1e9),
+        "parallelism": "replicas: corpus copy per GPU, question batches sharded across %d rank(s)" % world,
+    }
+
+
+def make_inputs(spec, rank, world, device):
+    corpus, scale, centres = synth.make_corpus(spec, device=device)
+    regions_all, offsets_all = synth.make_regions(spec, centres, "cpu", Q=spec.Q * world)
+    r0, r1 = int(offsets_all[rank * spec.Q]), int(offsets_all[(rank + 1) * spec.Q])
+    regions = regions_all[r0:r1].contiguous()
+    offsets = (offsets_all[rank * spec.Q:(rank + 1) * spec.Q + 1] - r0).to(torch.int32)
+    return corpus, scale, regions, offsets
+
+
+def host_corpus(corpus, scale):
+    if corpus.dtype == torch.bfloat16:
+        return synth.bf16_bits(corpus), None
+    return corpus.cpu().numpy(), scale.cpu().numpy()
+
+
+def cpu_baseline(spec, corpus_np, scale_np, regions, offsets, questions):
+    import oracle
+    nthreads = len(os.sched_getaffinity(0))
+    q = min(questions, offsets.numel() - 1)
+    r1 = int(offsets[q])
+    reg = synth.bf16_bits(regions[:r1])
+    off = offsets[:q + 1].numpy()
+    oracle.build()
+    t0 = time.perf_counter()
+    oracle.retrieve(corpus_np, reg, off, spec.k_region, spec.K, row_scale=scale_np, nthreads=nthreads)
+    dt = time.perf_counter() - t0
+    return {"value": q / dt, "unit": "queries/s", "cores": nthreads, "kind": "oracle",
+            "sample": "first %d questions (%d regions) over the full %d-row corpus, fp64, %d OpenMP threads, "
+                      "%.1f s" % (q, r1, spec.N, nthreads, dt)}
+
+
+def run_reference(args, spec):
+    """The CPU oracle as the reference arm: one question per step over the
+    first n_s corpus rows, scaled by N / n_s to full-corpus questions/s."""
+    import oracle
+    world = int(os.environ.get("WORLD_SIZE", "1"))
+    rank = int(os.environ.get("RANK", "0"))
+    if rank != 0:
+        return
+    oracle.build()
+    nthreads = len(os.sched_getaffinity(0))
+    corpus, scale, centres = synth.make_corpus(spec, device="cpu", N=min(spec.N, 1 << 18))
+    regions, offsets = synth.make_regions(spec, centres, "cpu")
+    cnp, snp = host_corpus(corpus, scale)
+    q_regions = [synth.bf16_bits(regions[int(offsets[q]):int(offsets[q + 1])]) for q in range(spec.Q)]
+
+    def step(i, n_s):
+        reg = q_regions[i % spec.Q]
+        off = np.array([0, reg.shape[0]], np.int32)
+        oracle.retrieve(cnp[:n_s], reg, off, spec.k_region, spec.K,
+                        row_scale=None if snp is None else snp[:n_s], nthreads=nthreads)
+
+    n_s = cnp.shape[0]
+    t0 = time.perf_counter()
+    step(0, n_s)
+    t_one = time.perf_counter() - t0
+    budget = 120.0
+    n_s = int(max(4096, min(n_s, n_s * budget / max(1e-9, t_one * (args.steps + args.warmup)))))
+    for i in range(args.warmup):
+        step(i, n_s)
+    t0 = time.perf_counter()
+    for i in range(args.steps):
+        step(i, n_s)
+    dt = time.perf_counter() - t0
+    value = args.steps * (n_s / spec.N) / dt
+    sample = ("one question per step (%s regions) over the first %d of %d corpus rows, fp64, %d OpenMP "
+              "threads; scaled by N / %d" % (spec.regions[0], n_s, spec.N, nthreads, n_s))
+    line = {"impl": "reference", "metric": METRIC, "value": value, "unit": "queries/s", "n_gpus": world,
+            "steps": args.steps, "warmup": args.warmup, "ms_per_step": 1e3 * dt / args.steps,
+            "higher_is_better": True, "scaling": "weak", "vs_baseline": None, "dtype": "f64",
+            "data": "synthetic", "config": workload_config(spec, int(offsets[-1]), 1),
+            "cpu_baseline": {"value": value, "unit": "queries/s", "cores": nthreads, "kind": "oracle",
+                             "sample": sample},
+            "e2e": {"value": value, "unit": "queries/s", "h2d_bytes_per_step": 0, "d2h_bytes_per_step": 0}}
+    print(json.dumps(line), flush=True)
+
+
+def main():
+    ap = argparse.ArgumentParser()
+    ap.add_argument("--gpus", type=int, default=1)
+    ap.add_argument("--steps", type=int, default=300)
+    ap.add_argument("--warmup", type=int, default=5)
+    ap.add_argument("--impl", default="native", choices=["native", "reference"])
+    ap.add_argument("--workload", default="clustered_1m", choices=sorted(synth.WORKLOADS))
+    ap.add_argument("--cpu-questions", type=int, default=8, help="questions in the oracle sample")
+    ap.add_argument("--no-cpu-baseline", action="store_true")
+    ap.add_argument("--path", default="auto", choices=["auto", "tensor", "warp"])
+    ap.add_argument("--cluster", type=int, default=0, choices=[0, 1, 2, 4, 8],
+                    help="tensor-path CTAs per cluster (0 = library's choice)")
+    args = ap.parse_args()
+    if args.warmup < 3:
+        raise SystemExit("at least 3 warm-up steps")
+    spec = synth.WORKLOADS[args.workload]
+    if args.impl == "reference":
+        run_reference(args, spec)
+        return
+
+    import paper_2607_25422_gb300 as skip
+
+    world, rank, local = dist_setup()
+    dev = torch.device("cuda", torch.cuda.current_device())
+    corpus, scale, regions, offsets = make_inputs(spec, rank, world, dev)
+    R = regions.shape[0]
+    Q = offsets.numel() - 1
+    c = skip.skip_corpus_load(corpus, row_scale=scale)
+    keep_host = rank == 0 and world == 1 and not args.no_cpu_baseline
+    corpus_np, scale_np = host_corpus(corpus, scale) if keep_host else (None, None)
+    del corpus
+    torch.cuda.empty_cache()
+    c.set_option(skip.SKIP_OPT_PATH, {"auto": 0, "tensor": 1, "warp": 2}[args.path])
+    c.set_option(skip.SKIP_OPT_CLUSTER, args.cluster)
+    reg_d = regions.to(dev)
+    off_d = offsets.to(dev)
+    out_ids = torch.empty(Q, spec.K, dtype=torch.int64, device=dev)
+    out_sc = torch.empty(Q, spec.K, dtype=torch.float32, device=dev)
+    stream = torch.cuda.current_stream()
+
+    def step():
+        skip.skip_retrieve(c, reg_d, off_d, spec.k_region, spec.K, out_ids, out_sc, stream)
+
+    for _ in range(args.warmup):
+        step()
+    st = skip.skip_sync_status(c)
+    if st != skip.SKIP_OK:
+        raise SystemExit("warm-up kernel status: %s" % skip.skip_status_string(st))
+    plan = skip.skip_last_plan(c)
+
+    # ---- timed region (device-resident inputs)
+    c.set_option(skip.SKIP_OPT_TIMING, 1)
+    skip.skip_timing_report(c)
+    sampler = ClockSampler(torch.cuda.current_device())
+    barrier(world)
+    torch.cuda.synchronize()
+    sampler.start()
+    time.sleep(0.3)
+    e0 = torch.cuda.Event(enable_timing=True)
+    e1 = torch.cuda.Event(enable_timing=True)
+    e0.record(stream)
+    for _ in range(args.steps):
+        step()
+    e1.record(stream)
+    torch.cuda.synchronize()
+    clocks = sampler.stop()
+    barrier(world)
+    ms_local = e0.elapsed_time(e1)
+    kernels = skip.skip_timing_report(c)
+    c.set_option(skip.SKIP_OPT_TIMING, 0)
+    st = skip.skip_sync_status(c)
+    if st != skip.SKIP_OK:
+        raise SystemExit("timed kernel status: %s" % skip.skip_status_string(st))
+    ms = max_over_ranks(ms_local, world)
+
+    # ---- end to end through the host-buffer entry point
+    reg_h = regions.pin_memory()
+    off_h = offsets.pin_memory()
+    ids_h = torch.empty(Q, spec.K, dtype=torch.int64).pin_memory()
+    sc_h = torch.empty(Q, spec.K, dtype=torch.float32).pin_memory()
+    for _ in range(3):
+        skip.skip_retrieve_host(c, reg_h, off_h, spec.k_region, spec.K, ids_h, sc_h, stream)
+    barrier(world)
+    torch.cuda.synchronize()
+    t0 = time.perf_counter()
+    for _ in range(args.steps):
+        skip.skip_retrieve_host(c, reg_h, off_h, spec.k_region, spec.K, ids_h, sc_h, stream)
+    torch.cuda.synchronize()
+    e2e_s = max_over_ranks(time.perf_counter() - t0, world)
+    h2d = R * spec.d * 2 + (Q + 1) * 4
+    d2h = Q * spec.K * (8 + 4)
+
+    # ---- derived figures
+    total_q = Q * world * args.steps
+    secs = ms / 1e3
+    elem = 2 if spec.dtype == "bf16" else 1
+    corpus_bytes = spec.N * (spec.d * elem + (4 if spec.dtype == "e4m3" else 0))
+    flops = 2.0 * R * spec.N * spec.d
+    peaks = load_peaks()
+    kname = next((k for k in SCORE_KERNELS if k in kernels), None)
+    kinfo = kernels.get(kname, {"launches": 0, "ms": float("nan")})
+    k_ms = kinfo["ms"] / max(1, kinfo["launches"])
+    t_hbm = corpus_bytes / (peaks["hbm_gbs"] * 1e9)
+    t_tc = flops / (peaks["bf16_tflops"] * 1e12)
+    if t_tc >= t_hbm:
+        achieved = flops / (k_ms / 1e3) / 1e12
+        roof = {"bound": "tensor", "achieved": achieved, "peak": peaks["bf16_tflops"], "unit": "TFLOP/s",
+                "frac": achieved / peaks["bf16_tflops"]}
+        if peaks.get("bf16_tflops_sustained"):
+            roof["frac_of_sustained"] = achieved / peaks["bf16_tflops_sustained"]
+    else:
+        achieved = corpus_bytes / (k_ms / 1e3) / 1e9
+        roof = {"bound": "hbm", "achieved": achieved, "peak": peaks["hbm_gbs"], "unit": "GB/s",
+                "frac": achieved / peaks["hbm_gbs"]}
+    traffic = profiled_traffic(kname, spec.name) if kname else None
+    roof.update({"traffic": traffic, "kernel": kname, "kernel_ms": k_ms, "peak_source": peaks["source"] +
+                 " (MEASURED_PEAKS.json burst)" if peaks["source"] == "measured" else "fallback",
+                 "algorithmic_flops_per_launch": flops, "algorithmic_bytes_per_launch": corpus_bytes,
+                 "step_roofline_frac": max(t_hbm, t_tc) / (secs / args.steps)})
+    line = {
+        "metric": METRIC, "value": total_q / secs, "unit": "queries/s", "n_gpus": world,
+        "steps": args.steps, "warmup": args.warmup, "ms_per_step": ms / args.steps,
+        "higher_is_better": True, "scaling": "weak", "vs_baseline": None, "dtype": "bf16",
+        "data": "synthetic", "config": workload_config(spec, R, world),
+        "corpus_gbs": corpus_bytes * world * args.steps / secs / 1e9,
+        "region_rows_per_s": R * world * args.steps / secs,
+        "tflops": flops * world * args.steps / secs / 1e12,
+        "roofline": roof,
+        "clocks": clocks,
+        "e2e": {"value": total_q / e2e_s, "unit": "queries/s", "h2d_bytes_per_step": h2d,
+                "d2h_bytes_per_step": d2h, "entry_point": "skip_retrieve_host (pinned host buffers)"},
+        "gpu_launches": int(sum(v["launches"] for v in kernels.values())),
+        "kernels": kernels,
+        "plan": plan,
+    }
+    if keep_host:
+        line["cpu_baseline"] = cpu_baseline(spec, corpus_np, scale_np, regions, offsets, args.cpu_questions)
+    c.free()
+    if rank == 0:
+        print(json.dumps(line), flush=True)
+    if world > 1:
+        import torch.distributed as dist
+        dist.destroy_process_group()
+
+
+if __name__ == "__main__":
+    main()

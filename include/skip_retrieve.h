@@ -68,7 +68,8 @@ typedef enum {
     SKIP_OPT_PATH = 0,            /* score kernel: 0 auto, 1 tensor core, 2 warp-dot */
     SKIP_OPT_WAIT_TIMEOUT_NS = 1, /* cap on each in-kernel wait (default 2e9 ns) */
     SKIP_OPT_GRID = 2,            /* score-kernel CTAs (0 = one per SM) */
-    SKIP_OPT_TIMING = 3           /* 1: time each kernel with CUDA events */
+    SKIP_OPT_TIMING = 3,          /* 1: time each kernel with CUDA events */
+    SKIP_OPT_CLUSTER = 4          /* tensor path CTAs per cluster: 0 pick, 1, 2, 4 or 8 */
 } skip_option_t;
 
 enum { SKIP_PATH_AUTO = 0, SKIP_PATH_TENSOR = 1, SKIP_PATH_WARP = 2 };
@@ -163,6 +164,14 @@ SKIP_API skip_status_t skip_sync_status(skip_corpus_t corpus, void *stream);
  * on, the device time of each kernel in ms (this synchronises on the
  * events).  Writes at most `len` bytes including the terminator. */
 SKIP_API skip_status_t skip_last_plan(skip_corpus_t corpus, char *buf, int32_t len);
+
+/* Infrastructure (no counterpart in the paper): with SKIP_OPT_TIMING on,
+ * every retrieval call records CUDA events on its stream around each kernel
+ * it launches.  This call waits for the last event, writes a JSON object
+ * {"<kernel>": {"launches": n, "ms": total device time}, ...} accumulated
+ * over all calls since the previous report, and clears the record.
+ * SKIP_EINVAL if `len` is too small. */
+SKIP_API skip_status_t skip_timing_report(skip_corpus_t corpus, char *buf, int32_t len);
 
 /* Static description of a status code. */
 SKIP_API const char *skip_status_string(skip_status_t status);

@@ -24,7 +24,7 @@ from . import _build
 
 SKIP_BF16, SKIP_E4M3 = 0, 1
 SKIP_OK, SKIP_EINVAL, SKIP_ENOMEM, SKIP_EUNSUPPORTED, SKIP_ETIMEOUT, SKIP_ECUDA = range(6)
-SKIP_OPT_PATH, SKIP_OPT_WAIT_TIMEOUT_NS, SKIP_OPT_GRID, SKIP_OPT_TIMING = range(4)
+SKIP_OPT_PATH, SKIP_OPT_WAIT_TIMEOUT_NS, SKIP_OPT_GRID, SKIP_OPT_TIMING, SKIP_OPT_CLUSTER = range(5)
 SKIP_PATH_AUTO, SKIP_PATH_TENSOR, SKIP_PATH_WARP = range(3)
 SKIP_MAX_K_REGION, SKIP_MAX_K = 1024, 2048
 
@@ -56,10 +56,12 @@ def load_library():
     lib.skip_retrieve_host.argtypes = [P, P, P, i32, i32, i32, i32, P, P, P]
     lib.skip_sync_status.argtypes = [P, P]
     lib.skip_last_plan.argtypes = [P, ctypes.c_char_p, i32]
+    lib.skip_timing_report.argtypes = [P, ctypes.c_char_p, i32]
     lib.skip_status_string.argtypes = [ctypes.c_int]
     lib.skip_status_string.restype = ctypes.c_char_p
     for f in ("skip_corpus_load", "skip_corpus_free", "skip_corpus_set_option", "skip_retrieve",
-              "skip_retrieve_regions", "skip_retrieve_host", "skip_sync_status", "skip_last_plan"):
+              "skip_retrieve_regions", "skip_retrieve_host", "skip_sync_status", "skip_last_plan",
+              "skip_timing_report"):
         getattr(lib, f).restype = ctypes.c_int
     _lib = lib
     return lib
@@ -213,6 +215,14 @@ def skip_sync_status(corpus: Corpus, stream=None) -> int:
 def skip_last_plan(corpus: Corpus) -> dict:
     buf = ctypes.create_string_buffer(1024)
     _check(load_library().skip_last_plan(corpus.handle, buf, 1024), "skip_last_plan")
+    return json.loads(buf.value.decode())
+
+
+def skip_timing_report(corpus: Corpus) -> dict:
+    """Per-kernel launches and device ms accumulated since the last report
+    (needs SKIP_OPT_TIMING = 1); clears the record."""
+    buf = ctypes.create_string_buffer(1 << 16)
+    _check(load_library().skip_timing_report(corpus.handle, buf, 1 << 16), "skip_timing_report")
     return json.loads(buf.value.decode())
 
 

@@ -14,14 +14,21 @@
 // compare per chunk.  Corpus rows of a tile are visited in increasing id
 // order, so "beats" is a strict score comparison and ties keep the lower id.
 //
-// Work: items (query block, corpus chunk); a persistent CTA walks items
-// blockIdx.x, blockIdx.x + gridDim.x, ...  Items are numbered chunk-major, so
-// the CTAs running at the same time read the same corpus chunk and every
-// corpus tile comes from HBM about once and is re-read by the other query
-// blocks from L2.  Each item leaves one sorted list per region row; the merge
-// kernel combines the chunks.
+// Work: a cluster of CL CTAs (CL = 1, 2, 4 or 8) holds CL query blocks and
+// walks items (query group, corpus chunk) in lock step; CTA r of the cluster
+// loads rows [r * 256 / CL, (r + 1) * 256 / CL) of each corpus tile and
+// multicasts them to all CL CTAs, so a corpus tile leaves L2 once per
+// cluster instead of once per query block, and a stage is refilled only when
+// every CTA's MMAs have released it (the MMA commit is multicast too).
+// Persistent clusters walk items cid, cid + #clusters, ...; items are
+// numbered chunk-major so that the clusters of the other query groups read
+// the same chunk at the same time and find it in L2.  Each item leaves one
+// sorted list per region row; the merge kernel combines the chunks.
 //
-// Warp roles (192 threads): warp 0 issues TMA loads into a 4-stage
+// Per-row lists live in shared memory ([slot][row], k slots) when they fit
+// next to a pipeline of at least two stages, else in global memory.
+//
+// Warp roles (192 threads): warp 0 issues TMA loads into a 2..4-stage
 // shared-memory ring; warp 1 owns TMEM (two 256-column fp32 accumulators)
 // and issues tcgen05.mma from one thread; warps 2..5 are the epilogue, warp w
 // reading TMEM lanes 32 * (w % 4) .. + 31.  Every wait is bounded; a wait
@@ -40,10 +47,11 @@ constexpr int kStageBytes = kABytes + kBBytes;
 constexpr uint32_t kTmemCols = 512;                 // two 256-column accumulators
 constexpr uint64_t kDrainTimeoutNs = 1000000000ull;  // 1 s for copies/MMAs in flight
 constexpr uint32_t kIdesc = idesc_bf16_f32(kTcTileM, kTcTileN);
+constexpr int kMaxStages = 4;
 
 struct __align__(8) TcShared {
-    uint64_t full[kTcStages];   // stage loaded (TMA transaction bytes)
-    uint64_t empty[kTcStages];  // stage consumed (tcgen05.commit)
+    uint64_t full[kMaxStages];   // stage loaded (TMA transaction bytes)
+    uint64_t empty[kMaxStages];  // stage consumed (tcgen05.commit)
     uint64_t tfull[2];          // accumulator ready (tcgen05.commit)
     uint64_t tempty[2];         // accumulator drained (4 epilogue warps)
     uint64_t drain;             // MMA completion at exit
@@ -56,17 +64,42 @@ struct Item {
     int64_t t0, t1;
 };
 
-__device__ __forceinline__ Item item_of(const TcParams &p, int u) {
+__device__ __forceinline__ Item item_of(const TcParams &p, int v, int rank) {
     Item it;
-    it.g = u / p.MB;
-    it.mb = u - it.g * p.MB;
+    it.g = v / p.QG;
+    it.mb = (v - it.g * p.QG) * p.CL + rank;
     it.t0 = (int64_t)it.g * p.tiles / p.G;
     it.t1 = (int64_t)(it.g + 1) * p.tiles / p.G;
     return it;
 }
 
-__device__ __noinline__ uint64_t insert_key(uint64_t *list, int nfill, int k, uint64_t key) {
-    return sorted_insert(list, nfill, k, key);
+// Insert key into a row list (slot t at L[t * ls], n valid, descending);
+// the caller has checked that key beats the k-th entry.  Returns the new n.
+__device__ __forceinline__ int list_insert(uint64_t *L, int ls, int n, int k, uint64_t key) {
+    int pos = n < k ? n : k - 1;
+    while (pos > 0) {
+        const uint64_t prev = L[(pos - 1) * ls];
+        if (prev >= key) break;
+        L[pos * ls] = prev;
+        --pos;
+    }
+    L[pos * ls] = key;
+    return n < k ? n + 1 : n;
+}
+
+// v[j] for a run-time j without indexing the register array (5 levels of
+// selects), so that v stays in registers.
+__device__ __forceinline__ uint32_t select32(const uint32_t (&v)[32], int j) {
+    uint32_t a[16];
+#pragma unroll
+    for (int i = 0; i < 16; ++i) a[i] = (j & 16) ? v[i + 16] : v[i];
+#pragma unroll
+    for (int i = 0; i < 8; ++i) a[i] = (j & 8) ? a[i + 8] : a[i];
+#pragma unroll
+    for (int i = 0; i < 4; ++i) a[i] = (j & 4) ? a[i + 4] : a[i];
+#pragma unroll
+    for (int i = 0; i < 2; ++i) a[i] = (j & 2) ? a[i + 2] : a[i];
+    return (j & 1) ? a[1] : a[0];
 }
 
 __device__ __forceinline__ float fmax32(const uint32_t (&v)[32]) {
@@ -85,17 +118,26 @@ __global__ void __launch_bounds__(kTcThreads, 1)
                     const TcParams p) {
     extern __shared__ uint8_t smem_raw[];
     uint8_t *smem = reinterpret_cast<uint8_t *>(((uintptr_t)smem_raw + 1023) & ~(uintptr_t)1023);
+    const int S = p.stages;
     uint8_t *sA = smem;
-    uint8_t *sB = smem + kTcStages * kABytes;
-    TcShared *sh = reinterpret_cast<TcShared *>(smem + kTcStages * kStageBytes);
+    uint8_t *sB = smem + S * kABytes;
+    uint64_t *slists = reinterpret_cast<uint64_t *>(smem + S * kStageBytes);
+    const size_t list_bytes = p.list_in_smem ? (size_t)kTcTileM * p.k * 8 : 0;
+    TcShared *sh = reinterpret_cast<TcShared *>(smem + S * kStageBytes + list_bytes);
     const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
-    const int items = p.MB * p.G;
+    const int items = p.QG * p.G;
     const int KB = (p.d + kTcTileK - 1) / kTcTileK;
+    const int CL = p.CL;
+    const int rank = CL > 1 ? (int)cluster_rank() : 0;
+    const int cid = CL > 1 ? (int)cluster_index() : (int)blockIdx.x;
+    const int ncl = CL > 1 ? (int)cluster_count() : (int)gridDim.x;
+    const uint16_t mask = (uint16_t)((1u << CL) - 1u);
+    const int slice_rows = kTcTileN / CL;
 
     if (threadIdx.x == 0) {
-        for (int s = 0; s < kTcStages; ++s) {
+        for (int s = 0; s < S; ++s) {
             mbar_init(smem_addr(&sh->full[s]), 1);
-            mbar_init(smem_addr(&sh->empty[s]), 1);
+            mbar_init(smem_addr(&sh->empty[s]), CL);
         }
         for (int b = 0; b < 2; ++b) {
             mbar_init(smem_addr(&sh->tfull[b]), 1);
@@ -115,6 +157,8 @@ __global__ void __launch_bounds__(kTcThreads, 1)
     tc_fence_before();
     __syncthreads();
     tc_fence_after();
+    // Every CTA's barriers are initialised before any multicast targets them.
+    if (CL > 1) cluster_sync_all();
     const uint32_t tmem = sh->tmem_base;
 
     if (warp == 0) {
@@ -124,8 +168,8 @@ __global__ void __launch_bounds__(kTcThreads, 1)
             uint32_t ph = 0;
             int64_t issued = 0;
             bool ok = true;
-            for (int u = blockIdx.x; u < items && ok; u += gridDim.x) {
-                const Item it = item_of(p, u);
+            for (int v = cid; v < items && ok; v += ncl) {
+                const Item it = item_of(p, v, rank);
                 for (int64_t t = it.t0; t < it.t1 && ok; ++t) {
                     for (int kb = 0; kb < KB; ++kb) {
                         if (!mbar_wait(smem_addr(&sh->empty[s]), ph ^ 1u, p.timeout_ns)) {
@@ -135,9 +179,13 @@ __global__ void __launch_bounds__(kTcThreads, 1)
                         const uint32_t fb = smem_addr(&sh->full[s]);
                         mbar_arrive_expect_tx(fb, kStageBytes);
                         tma_load_2d(smem_addr(sA + s * kABytes), &tq, fb, kb * kTcTileK, it.mb * kTcTileM);
-                        tma_load_2d(smem_addr(sB + s * kBBytes), &tx, fb, kb * kTcTileK, (int)(t * kTcTileN));
+                        if (CL == 1)
+                            tma_load_2d(smem_addr(sB + s * kBBytes), &tx, fb, kb * kTcTileK, (int)(t * kTcTileN));
+                        else
+                            tma_load_2d_mc(smem_addr(sB + s * kBBytes + rank * slice_rows * 128), &tx, fb,
+                                           kb * kTcTileK, (int)(t * kTcTileN) + rank * slice_rows, mask);
                         ++issued;
-                        if (++s == kTcStages) {
+                        if (++s == S) {
                             s = 0;
                             ph ^= 1u;
                         }
@@ -146,8 +194,8 @@ __global__ void __launch_bounds__(kTcThreads, 1)
             }
             if (!ok) atomicOr(p.err, kErrTimeout);
             // Copies in flight: wait for the last load issued on every stage.
-            for (int st = 0; st < kTcStages; ++st) {
-                const int64_t uses = issued / kTcStages + (st < issued % kTcStages ? 1 : 0);
+            for (int st = 0; st < S; ++st) {
+                const int64_t uses = issued / S + (st < issued % S ? 1 : 0);
                 if (uses == 0) continue;
                 if (!mbar_wait(smem_addr(&sh->full[st]), (uint32_t)((uses - 1) & 1), kDrainTimeoutNs))
                     atomicOr(p.err, kErrTimeout);
@@ -160,8 +208,8 @@ __global__ void __launch_bounds__(kTcThreads, 1)
             uint32_t ph = 0;
             uint32_t lt = 0;
             bool ok = true;
-            for (int u = blockIdx.x; u < items && ok; u += gridDim.x) {
-                const Item it = item_of(p, u);
+            for (int v = cid; v < items && ok; v += ncl) {
+                const Item it = item_of(p, v, rank);
                 for (int64_t t = it.t0; t < it.t1 && ok; ++t, ++lt) {
                     const uint32_t buf = lt & 1u, use = lt >> 1;
                     if (!mbar_wait(smem_addr(&sh->tempty[buf]), (use & 1u) ^ 1u, p.timeout_ns)) {
@@ -182,8 +230,11 @@ __global__ void __launch_bounds__(kTcThreads, 1)
                         for (int kk = 0; kk < kTcTileK / 16; ++kk)
                             tc_mma_f16(dt, ad + (uint64_t)(kk * 2), bd + (uint64_t)(kk * 2), kIdesc,
                                        (kb | kk) != 0);
-                        tc_commit(smem_addr(&sh->empty[s]));
-                        if (++s == kTcStages) {
+                        if (CL == 1)
+                            tc_commit(smem_addr(&sh->empty[s]));
+                        else
+                            tc_commit_mc(smem_addr(&sh->empty[s]), mask);
+                        if (++s == S) {
                             s = 0;
                             ph ^= 1u;
                         }
@@ -205,13 +256,34 @@ __global__ void __launch_bounds__(kTcThreads, 1)
         const float kNegInf = -__int_as_float(0x7f800000);
         uint32_t lt = 0;
         bool ok = true;
-        for (int u = blockIdx.x; u < items && ok; u += gridDim.x) {
-            const Item it = item_of(p, u);
+        for (int v = cid; v < items && ok; v += ncl) {
+            const Item it = item_of(p, v, rank);
             const int row = it.mb * kTcTileM + rib;
-            const bool row_valid = row < p.R;
-            uint64_t *list = p.lists + ((int64_t)it.g * p.R_pad + row) * p.k;
+            const bool row_valid = it.mb < p.MB && row < p.R;
+            uint64_t *glist = p.lists + ((int64_t)it.g * p.R_pad + row) * p.k;
+            uint64_t *L = p.list_in_smem ? slists + rib : glist;
+            const int ls = p.list_in_smem ? kTcTileM : 1;
             int nfill = 0;
             float thr = kNegInf;
+            // Common case: no score of the 32 beats the threshold (a max and
+            // a compare).  Otherwise a branch-free bit mask of the survivors
+            // is walked in increasing column (= id) order, so that lanes
+            // without survivors idle for a few instructions only.
+            auto scan32 = [&](uint32_t (&v)[32], uint32_t id0) {
+                if (!row_valid || !(fmax32(v) > thr)) return;
+                uint32_t m = 0;
+#pragma unroll
+                for (int j = 0; j < 32; ++j) m |= (__uint_as_float(v[j]) > thr ? 1u : 0u) << j;
+                while (m) {
+                    const int j = __ffs(m) - 1;
+                    m &= m - 1;
+                    const float sj = __uint_as_float(select32(v, j));
+                    if (sj > thr) {
+                        nfill = list_insert(L, ls, nfill, p.k, make_key(sj, id0 + j));
+                        if (nfill == p.k) thr = key_score(L[(p.k - 1) * ls]);
+                    }
+                }
+            };
             for (int64_t t = it.t0; t < it.t1; ++t, ++lt) {
                 const uint32_t buf = lt & 1u, use = lt >> 1;
                 if (!mbar_wait(smem_addr(&sh->tfull[buf]), use & 1u, p.timeout_ns)) {
@@ -222,40 +294,42 @@ __global__ void __launch_bounds__(kTcThreads, 1)
                 const int64_t n0 = t * kTcTileN;
                 const bool tail = n0 + kTcTileN > p.N;
 #pragma unroll 1
-                for (int c = 0; c < kTcTileN / 32; ++c) {
-                    uint32_t v[32];
-                    tmem_ld_32x32b_x32(tmem + lane_addr + buf * kTcTileN + c * 32, v);
-                    tmem_ld_wait(v);
-                    const uint32_t id0 = (uint32_t)(n0 + c * 32);
+                for (int c = 0; c < kTcTileN / 64; ++c) {
+                    uint32_t v0[32], v1[32];
+                    const uint32_t taddr = tmem + lane_addr + buf * kTcTileN + c * 64;
+                    tmem_ld_32x32b_x32(taddr, v0);
+                    tmem_ld_32x32b_x32(taddr + 32, v1);
+                    tmem_ld_wait(v0);
+                    regs_after_wait(v1);
+                    const uint32_t id0 = (uint32_t)(n0 + c * 64);
                     if (tail) {
 #pragma unroll
-                        for (int j = 0; j < 32; ++j)
-                            if ((int64_t)id0 + j >= p.N) v[j] = 0xFF800000u;
-                    }
-                    if (row_valid && fmax32(v) > thr) {
-#pragma unroll
                         for (int j = 0; j < 32; ++j) {
-                            const float sj = __uint_as_float(v[j]);
-                            if (sj > thr) {
-                                const uint64_t kth = insert_key(list, nfill, p.k, make_key(sj, id0 + j));
-                                if (nfill < p.k) ++nfill;
-                                thr = kth ? key_score(kth) : kNegInf;
-                            }
+                            if ((int64_t)id0 + j >= p.N) v0[j] = 0xFF800000u;
+                            if ((int64_t)id0 + 32 + j >= p.N) v1[j] = 0xFF800000u;
                         }
                     }
+                    if (c == kTcTileN / 64 - 1) {
+                        // Last read of this accumulator: hand it back before scanning.
+                        tc_fence_before();
+                        __syncwarp();
+                        if (lane == 0) mbar_arrive(smem_addr(&sh->tempty[buf]));
+                    }
+                    scan32(v0, id0);
+                    scan32(v1, id0 + 32);
                 }
-                tc_fence_before();
-                __syncwarp();
-                if (lane == 0) mbar_arrive(smem_addr(&sh->tempty[buf]));
             }
-            if (row_valid)
-                for (int t = nfill; t < p.k; ++t) list[t] = 0ull;
+            if (row_valid) {
+                for (int t = 0; t < p.k; ++t) glist[t] = t < nfill ? L[t * ls] : 0ull;
+            }
         }
         if (!ok && lane == 0) atomicOr(p.err, kErrTimeout);
     }
 
     tc_fence_before();
     __syncthreads();
+    // No peer may still multicast into, or arrive on, this CTA when it exits.
+    if (CL > 1) cluster_sync_all();
     tc_fence_after();
     if (warp == 1) {
         __syncwarp();
@@ -265,16 +339,63 @@ __global__ void __launch_bounds__(kTcThreads, 1)
 
 }  // namespace
 
-size_t tc_smem_bytes() { return 1024 + (size_t)kTcStages * kStageBytes + sizeof(TcShared); }
+size_t tc_smem_bytes(int stages, int k, bool list_in_smem) {
+    return 1024 + (size_t)stages * kStageBytes + (list_in_smem ? (size_t)kTcTileM * k * 8 : 0) +
+           sizeof(TcShared);
+}
+
+void tc_pick_layout(int k, int max_smem, int *stages, bool *list_in_smem) {
+    for (int st = kMaxStages; st >= 2; --st)
+        if (tc_smem_bytes(st, k, true) <= (size_t)max_smem) {
+            *stages = st;
+            *list_in_smem = true;
+            return;
+        }
+    *stages = kMaxStages;
+    *list_in_smem = false;
+}
+
+static cudaLaunchConfig_t tc_config(int grid, int CL, size_t smem, cudaStream_t s, cudaLaunchAttribute *attr) {
+    cudaLaunchConfig_t cfg = {};
+    cfg.gridDim = dim3(grid, 1, 1);
+    cfg.blockDim = dim3(kTcThreads, 1, 1);
+    cfg.dynamicSmemBytes = smem;
+    cfg.stream = s;
+    attr[0].id = cudaLaunchAttributeClusterDimension;
+    attr[0].val.clusterDim.x = CL;
+    attr[0].val.clusterDim.y = 1;
+    attr[0].val.clusterDim.z = 1;
+    cfg.attrs = attr;
+    cfg.numAttrs = 1;
+    return cfg;
+}
+
+int tc_max_clusters(int CL, int stages, int k, bool list_in_smem) {
+    const size_t smem = tc_smem_bytes(stages, k, list_in_smem);
+    if (cudaFuncSetAttribute(k_tc_score_topk, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem) !=
+        cudaSuccess) {
+        cudaGetLastError();
+        return 0;
+    }
+    cudaLaunchAttribute attr[1];
+    cudaLaunchConfig_t cfg = tc_config(CL * 64, CL, smem, 0, attr);
+    int n = 0;
+    if (cudaOccupancyMaxActiveClusters(&n, k_tc_score_topk, &cfg) != cudaSuccess) {
+        cudaGetLastError();
+        return 0;
+    }
+    return n;
+}
 
 cudaError_t launch_tc(const CUtensorMap &tq, const CUtensorMap &tx, const TcParams &p, int grid,
                       cudaStream_t s) {
-    const size_t smem = tc_smem_bytes();
+    const size_t smem = tc_smem_bytes(p.stages, p.k, p.list_in_smem != 0);
     cudaError_t e = cudaFuncSetAttribute(k_tc_score_topk, cudaFuncAttributeMaxDynamicSharedMemorySize,
                                          (int)smem);
     if (e != cudaSuccess) return e;
-    k_tc_score_topk<<<grid, kTcThreads, smem, s>>>(tq, tx, p);
-    return cudaGetLastError();
+    cudaLaunchAttribute attr[1];
+    cudaLaunchConfig_t cfg = tc_config(grid, p.CL, smem, s, attr);
+    return cudaLaunchKernelEx(&cfg, k_tc_score_topk, tq, tx, p);
 }
 
 }  // namespace skipk

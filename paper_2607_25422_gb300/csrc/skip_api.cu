@@ -7,7 +7,10 @@
 #include <string.h>
 
 #include <algorithm>
+#include <map>
 #include <mutex>
+#include <string>
+#include <vector>
 
 #include "../../include/skip_retrieve.h"
 #include "skip_internal.h"
@@ -18,7 +21,7 @@ namespace {
 
 constexpr uint64_t kDefaultTimeoutNs = 2000000000ull;
 constexpr int kMaxD = 4096;
-constexpr int kMaxEvents = 8;
+constexpr size_t kMaxEvents = 1 << 20;
 
 typedef CUresult (*EncodeTiledFn)(CUtensorMap *, CUtensorMapDataType, cuuint32_t, void *,
                                   const cuuint64_t *, const cuuint64_t *, const cuuint32_t *,
@@ -58,6 +61,7 @@ bool encode_bf16_rows(CUtensorMap *map, const void *base, int64_t rows, int d, i
 struct skip_corpus {
     int device = 0;
     int sm_count = 0;
+    int max_smem = 0;          // opt-in shared memory per block
     int64_t N = 0;
     int d = 0;
     skip_dtype_t dtype = SKIP_BF16;
@@ -73,10 +77,16 @@ struct skip_corpus {
     int path = SKIP_PATH_AUTO;
     uint64_t timeout_ns = kDefaultTimeoutNs;
     int grid = 0;
+    int cluster = 0;           // 0 = pick; else CTAs per cluster
+    std::map<int, int> cluster_cache;  // resident clusters per (size, stages, list place)
     int timing = 0;
-    cudaEvent_t ev[kMaxEvents] = {};
-    const char *ev_name[kMaxEvents] = {};
-    int n_ev = 0;
+    // Timing: events recorded on the launching stream before each kernel and
+    // after the last one, kept across calls until skip_timing_report.
+    std::vector<cudaEvent_t> ev_pool;
+    std::vector<const char *> ev_name;
+    std::vector<int> ev_call;
+    size_t ev_used = 0;
+    int call_id = 0;
     char plan[384] = "{}";
 };
 
@@ -107,11 +117,18 @@ skip_status_t ensure_ws(skip_corpus *c, size_t bytes) {
 }
 
 void record(skip_corpus *c, cudaStream_t s, const char *name) {
-    if (!c->timing || c->n_ev >= kMaxEvents) return;
-    if (!c->ev[c->n_ev]) cudaEventCreate(&c->ev[c->n_ev]);
-    c->ev_name[c->n_ev] = name;
-    cudaEventRecord(c->ev[c->n_ev], s);
-    ++c->n_ev;
+    if (!c->timing || c->ev_used >= kMaxEvents) return;
+    if (c->ev_used == c->ev_pool.size()) {
+        cudaEvent_t e;
+        if (cudaEventCreate(&e) != cudaSuccess) return;
+        c->ev_pool.push_back(e);
+        c->ev_name.push_back(nullptr);
+        c->ev_call.push_back(0);
+    }
+    c->ev_name[c->ev_used] = name;
+    c->ev_call[c->ev_used] = c->call_id;
+    cudaEventRecord(c->ev_pool[c->ev_used], s);
+    ++c->ev_used;
 }
 
 size_t align_up(size_t v, size_t a) { return (v + a - 1) / a * a; }
@@ -124,6 +141,9 @@ struct Plan {
     int R_pad = 0;
     int64_t tiles = 0;
     int launches = 0;
+    int stages = 0;
+    bool list_in_smem = false;
+    int CL = 1;
 };
 
 // Corpus chunks G for the tensor path: make MB * G a whole number of waves of
@@ -173,18 +193,54 @@ skip_status_t run_regions(skip_corpus *c, const uint16_t *regions, int R, int k,
     pl.tensor = tensor;
     if (tensor) {
         pl.MB = (R + kTcTileM - 1) / kTcTileM;
-        pl.R_pad = pl.MB * kTcTileM;
         pl.tiles = (c->N + kTcTileN - 1) / kTcTileN;
-        pl.G = pick_chunks(pl.MB, pl.tiles, ctas);
-        const int items = pl.MB * pl.G;
-        pl.grid = std::min(items, ctas);
+        bool in_smem = false;
+        int stages = 0;
+        tc_pick_layout(k, c->max_smem, &stages, &in_smem);
+        // Cluster size: the CTAs of a cluster share each corpus tile (one L2
+        // read, multicast).  Take the largest size that keeps at least 90%
+        // of the SMs the best size keeps busy, unless set by option.
+        int cl_best = 1, ncl_best = 0;
+        {
+            int used[4] = {0, 0, 0, 0}, ncls[4] = {0, 0, 0, 0};
+            int best_used = 0;
+            for (int i = 0; i < 4; ++i) {
+                const int CL = 1 << i;
+                if (c->cluster && CL != c->cluster) continue;
+                if (!c->cluster && CL > 1 && CL > pl.MB) break;
+                const int key = CL * 100 + stages * 10 + (in_smem ? 1 : 0);
+                auto hit = c->cluster_cache.find(key);
+                if (hit == c->cluster_cache.end())
+                    hit = c->cluster_cache.emplace(key, tc_max_clusters(CL, stages, k, in_smem)).first;
+                ncls[i] = hit->second;
+                const int QG = (pl.MB + CL - 1) / CL;
+                const double eff = (double)pl.MB / (double)(QG * CL);
+                used[i] = (int)(std::min(ncls[i] * CL, ctas) * eff);
+                best_used = std::max(best_used, used[i]);
+            }
+            for (int i = 3; i >= 0; --i)
+                if (used[i] > 0 && used[i] * 10 >= best_used * 9) {
+                    cl_best = 1 << i;
+                    ncl_best = ncls[i];
+                    break;
+                }
+            if (ncl_best == 0) return SKIP_ECUDA;
+        }
+        pl.CL = cl_best;
+        const int QG = (pl.MB + cl_best - 1) / cl_best;
+        const int ncl = std::max(1, std::min(ncl_best, ctas / cl_best));
+        pl.R_pad = QG * cl_best * kTcTileM;
+        pl.G = pick_chunks(QG, pl.tiles, ncl);
+        const int items = QG * pl.G;
+        pl.grid = std::min(items, ncl) * cl_best;
         const size_t lists_bytes = (size_t)pl.G * pl.R_pad * k * sizeof(uint64_t);
         skip_status_t st = ensure_ws(c, align_up(ws_extra, 256) + lists_bytes);
         if (st) return st;
         uint64_t *lists = reinterpret_cast<uint64_t *>((char *)c->ws + align_up(ws_extra, 256));
         if (keys_out) *keys_out = reg_keys = reinterpret_cast<uint64_t *>(c->ws);
-        CUtensorMap tq;
+        CUtensorMap tq, tx;
         if (!encode_bf16_rows(&tq, regions, R, c->d, kTcTileM)) return SKIP_ECUDA;
+        if (!encode_bf16_rows(&tx, c->rows, c->N, c->d, kTcTileN / cl_best)) return SKIP_ECUDA;
         TcParams p;
         p.N = c->N;
         p.d = c->d;
@@ -192,13 +248,19 @@ skip_status_t run_regions(skip_corpus *c, const uint16_t *regions, int R, int k,
         p.R_pad = pl.R_pad;
         p.k = k;
         p.MB = pl.MB;
+        p.CL = pl.CL;
+        p.QG = QG;
         p.G = pl.G;
         p.tiles = pl.tiles;
         p.lists = lists;
         p.err = c->err;
         p.timeout_ns = c->timeout_ns;
+        p.stages = stages;
+        p.list_in_smem = in_smem;
+        pl.stages = p.stages;
+        pl.list_in_smem = in_smem;
         record(c, s, "score_topk_tc");
-        cudaError_t e = launch_tc(tq, c->tmap_x, p, pl.grid, s);
+        cudaError_t e = launch_tc(tq, tx, p, pl.grid, s);
         if (e != cudaSuccess) return cuda_status(e);
         ++pl.launches;
         record(c, s, "merge_lists");
@@ -247,8 +309,10 @@ skip_status_t run_regions(skip_corpus *c, const uint16_t *regions, int R, int k,
 void write_plan(skip_corpus *c, const Plan &pl, int R, int Q, int k, int K) {
     snprintf(c->plan, sizeof c->plan,
              "{\"path\": \"%s\", \"grid\": %d, \"lists_per_row\": %d, \"query_blocks\": %d, "
-             "\"R_total\": %d, \"Q\": %d, \"k_region\": %d, \"K\": %d, \"launches\": %d}",
-             pl.tensor ? "tensor" : "warpdot", pl.grid, pl.G, pl.MB, R, Q, k, K, pl.launches);
+             "\"R_total\": %d, \"Q\": %d, \"k_region\": %d, \"K\": %d, \"launches\": %d, "
+             "\"stages\": %d, \"cluster\": %d, \"lists\": \"%s\"}",
+             pl.tensor ? "tensor" : "warpdot", pl.grid, pl.G, pl.MB, R, Q, k, K, pl.launches, pl.stages, pl.CL,
+             pl.tensor ? (pl.list_in_smem ? "shared" : "global") : "global");
 }
 
 }  // namespace
@@ -284,12 +348,15 @@ skip_status_t skip_corpus_load(const void *rows, int rows_on_device, int64_t N, 
     cudaDeviceGetAttribute(&major, cudaDevAttrComputeCapabilityMajor, dev);
     cudaDeviceGetAttribute(&minor, cudaDevAttrComputeCapabilityMinor, dev);
     cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev);
+    int max_smem = 0;
+    cudaDeviceGetAttribute(&max_smem, cudaDevAttrMaxSharedMemoryPerBlockOptin, dev);
     if (major != 10 || minor != 3) return SKIP_EUNSUPPORTED;
 
     skip_corpus *c = new (std::nothrow) skip_corpus();
     if (!c) return SKIP_ENOMEM;
     c->device = dev;
     c->sm_count = sms;
+    c->max_smem = max_smem;
     c->N = N;
     c->d = d;
     c->dtype = dtype;
@@ -324,8 +391,7 @@ skip_status_t skip_corpus_free(skip_corpus_t c) {
     cudaFree(c->err);
     cudaFree(c->ws);
     cudaFree(c->io);
-    for (int i = 0; i < kMaxEvents; ++i)
-        if (c->ev[i]) cudaEventDestroy(c->ev[i]);
+    for (cudaEvent_t e : c->ev_pool) cudaEventDestroy(e);
     delete c;
     return SKIP_OK;
 }
@@ -348,6 +414,10 @@ skip_status_t skip_corpus_set_option(skip_corpus_t c, int option, int64_t value)
         case SKIP_OPT_TIMING:
             c->timing = value != 0;
             return SKIP_OK;
+        case SKIP_OPT_CLUSTER:
+            if (value != 0 && value != 1 && value != 2 && value != 4 && value != 8) return SKIP_EINVAL;
+            c->cluster = (int)value;
+            return SKIP_OK;
     }
     return SKIP_EINVAL;
 }
@@ -361,7 +431,7 @@ skip_status_t skip_retrieve(skip_corpus_t c, const void *regions, const int32_t 
     if (Q > 0 && (!out_ids || !out_scores)) return SKIP_EINVAL;
     if (Q == 0 && R_total != 0) return SKIP_EINVAL;
     cudaStream_t s = reinterpret_cast<cudaStream_t>(stream);
-    c->n_ev = 0;
+    ++c->call_id;
     Plan pl;
     const size_t keys_bytes = align_up((size_t)std::max(R_total, 1) * k_region * sizeof(uint64_t), 256);
     uint64_t *reg_keys = nullptr;
@@ -393,7 +463,7 @@ skip_status_t skip_retrieve_regions(skip_corpus_t c, const void *regions, int32_
     if (st) return st;
     if (R_total > 0 && (!reg_ids || !reg_scores)) return SKIP_EINVAL;
     cudaStream_t s = reinterpret_cast<cudaStream_t>(stream);
-    c->n_ev = 0;
+    ++c->call_id;
     Plan pl;
     if (R_total > 0) {
         st = run_regions(c, reinterpret_cast<const uint16_t *>(regions), R_total, k_region, nullptr, reg_ids,
@@ -471,20 +541,52 @@ skip_status_t skip_retrieve_host(skip_corpus_t c, const uint16_t *regions, const
 
 skip_status_t skip_last_plan(skip_corpus_t c, char *buf, int32_t len) {
     if (!c || !buf || len < 1) return SKIP_EINVAL;
-    char times[256] = "";
-    if (c->timing && c->n_ev > 1) {
-        int at = snprintf(times, sizeof times, ", \"ms\": {");
-        for (int i = 0; i + 1 < c->n_ev && at < (int)sizeof times; ++i) {
+    std::string times;
+    if (c->timing && c->ev_used > 1) {
+        bool first = true;
+        for (size_t i = 0; i + 1 < c->ev_used; ++i) {
+            if (c->ev_call[i] != c->call_id || c->ev_call[i + 1] != c->call_id) continue;
             float ms = 0.0f;
-            if (cudaEventSynchronize(c->ev[i + 1]) != cudaSuccess ||
-                cudaEventElapsedTime(&ms, c->ev[i], c->ev[i + 1]) != cudaSuccess)
+            if (cudaEventSynchronize(c->ev_pool[i + 1]) != cudaSuccess ||
+                cudaEventElapsedTime(&ms, c->ev_pool[i], c->ev_pool[i + 1]) != cudaSuccess)
                 return SKIP_ECUDA;
-            at += snprintf(times + at, sizeof times - at, "%s\"%s\": %.6f", i ? ", " : "", c->ev_name[i], ms);
+            char item[96];
+            snprintf(item, sizeof item, "%s\"%s\": %.6f", first ? "" : ", ", c->ev_name[i], ms);
+            times += item;
+            first = false;
         }
-        if (at < (int)sizeof times) snprintf(times + at, sizeof times - at, "}");
+        times = ", \"ms\": {" + times + "}";
     }
     const int plen = (int)strlen(c->plan);
-    snprintf(buf, len, "%.*s%s}", plen > 0 ? plen - 1 : 0, c->plan, times);
+    snprintf(buf, len, "%.*s%s}", plen > 0 ? plen - 1 : 0, c->plan, times.c_str());
+    return SKIP_OK;
+}
+
+skip_status_t skip_timing_report(skip_corpus_t c, char *buf, int32_t len) {
+    if (!c || !buf || len < 1) return SKIP_EINVAL;
+    std::map<std::string, std::pair<int64_t, double>> acc;
+    if (c->ev_used > 0 && cudaEventSynchronize(c->ev_pool[c->ev_used - 1]) != cudaSuccess) return SKIP_ECUDA;
+    for (size_t i = 0; i + 1 < c->ev_used; ++i) {
+        if (c->ev_call[i] != c->ev_call[i + 1]) continue;
+        float ms = 0.0f;
+        if (cudaEventElapsedTime(&ms, c->ev_pool[i], c->ev_pool[i + 1]) != cudaSuccess) return SKIP_ECUDA;
+        auto &a = acc[c->ev_name[i]];
+        a.first += 1;
+        a.second += ms;
+    }
+    c->ev_used = 0;
+    std::string out = "{";
+    bool first = true;
+    for (auto &kv : acc) {
+        char item[160];
+        snprintf(item, sizeof item, "%s\"%s\": {\"launches\": %lld, \"ms\": %.6f}", first ? "" : ", ",
+                 kv.first.c_str(), (long long)kv.second.first, kv.second.second);
+        out += item;
+        first = false;
+    }
+    out += "}";
+    if ((int)out.size() + 1 > len) return SKIP_EINVAL;
+    memcpy(buf, out.c_str(), out.size() + 1);
     return SKIP_OK;
 }
 

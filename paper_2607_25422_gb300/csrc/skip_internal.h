@@ -33,21 +33,28 @@ struct TcParams {
     int64_t N;
     int d;
     int R;            // region rows
-    int R_pad;        // query blocks * 128
+    int R_pad;        // padded query blocks * 128
     int k;
-    int MB;           // query blocks of 128 rows
+    int MB;           // query blocks of 128 rows holding region rows
+    int CL;           // CTAs per cluster (1, 2, 4, 8), one query block each
+    int QG;           // query groups: ceil(MB / CL)
     int G;            // corpus chunks (lists per row)
     int64_t tiles;    // corpus tiles of kTcTileN rows
     uint64_t *lists;  // [G][R_pad][k]
     int *err;
     uint64_t timeout_ns;
+    int stages;       // pipeline depth (2..4)
+    int list_in_smem; // per-row lists in shared memory (else global)
 };
 constexpr int kTcTileM = 128;   // region rows per tile (TMEM lanes)
 constexpr int kTcTileN = 256;   // corpus rows per tile (TMEM columns)
 constexpr int kTcTileK = 64;    // bf16 elements per stage row (128 bytes)
-constexpr int kTcStages = 4;
 constexpr int kTcThreads = 192; // producer warp, MMA warp, 4 epilogue warps
-size_t tc_smem_bytes();
+size_t tc_smem_bytes(int stages, int k, bool list_in_smem);
+// Deepest pipeline that fits next to shared-memory lists, else global lists.
+void tc_pick_layout(int k, int max_smem, int *stages, bool *list_in_smem);
+// Clusters of CL CTAs that can be resident at once with this layout.
+int tc_max_clusters(int CL, int stages, int k, bool list_in_smem);
 cudaError_t launch_tc(const CUtensorMap &tq, const CUtensorMap &tx, const TcParams &p, int grid,
                       cudaStream_t s);
 

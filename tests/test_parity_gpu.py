@@ -24,11 +24,12 @@ def _bits(t):
     return synth.bf16_bits(t)
 
 
-def run_gpu(corpus, regions, offsets, k, K, path, scale=None):
+def run_gpu(corpus, regions, offsets, k, K, path, scale=None, cluster=0):
     dev = torch.device("cuda")
     c = skip.skip_corpus_load(corpus.to(dev), row_scale=None if scale is None else scale.to(dev))
     try:
         c.set_option(skip.SKIP_OPT_PATH, path)
+        c.set_option(skip.SKIP_OPT_CLUSTER, cluster)
         reg = regions.to(dev)
         rid, rsc = skip.skip_retrieve_regions(c, reg, k)
         oid, osc = skip.skip_retrieve(c, reg, torch.as_tensor(offsets).to(dev), k, K)
@@ -120,6 +121,21 @@ def test_random_bf16(case, path):
     cn, rn = _bits(ct), _bits(rt)
     truth = oracle_truth(cn, rn, offsets, k, K)
     gpu = run_gpu(ct, rt, offsets, k, K, PATHS[path])
+    assert_parity(cn, rn, offsets, k, K, gpu, truth)
+
+
+@pytest.mark.parametrize("cluster", [1, 2, 4, 8])
+def test_cluster_sizes(cluster):
+    """Every cluster size of the tensor path, with query blocks that do not
+    fill the last cluster and a ragged corpus tail."""
+    N, d, R, Q, k, K = 40000, 256, 700, 30, 16, 40
+    ct = synth.random_bf16(N, d, seed=77)
+    rt = synth.random_bf16(R, d, seed=78)
+    offsets = ragged_offsets(Q, R, seed=79)
+    cn, rn = _bits(ct), _bits(rt)
+    truth = oracle_truth(cn, rn, offsets, k, K)
+    gpu = run_gpu(ct, rt, offsets, k, K, skip.SKIP_PATH_TENSOR, cluster=cluster)
+    assert gpu[4]["cluster"] == cluster
     assert_parity(cn, rn, offsets, k, K, gpu, truth)
 
 
