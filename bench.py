@@ -259,7 +259,9 @@ def main():
     ap.add_argument("--no-cpu-baseline", action="store_true")
     ap.add_argument("--path", default="auto", choices=["auto", "tensor", "warp"])
     ap.add_argument("--cluster", type=int, default=0, choices=[0, 1, 2, 4, 8],
-                    help="tensor-path CTAs per cluster (0 = library's choice)")
+                    help="single-CTA tensor path CTAs per cluster (0 = library's choice)")
+    ap.add_argument("--mma", default="auto", choices=["auto", "single", "pair"],
+                    help="tensor-path MMA shape (auto = library's choice)")
     args = ap.parse_args()
     if args.warmup < 3:
         raise SystemExit("at least 3 warm-up steps")
@@ -282,6 +284,7 @@ def main():
     torch.cuda.empty_cache()
     c.set_option(skip.SKIP_OPT_PATH, {"auto": 0, "tensor": 1, "warp": 2}[args.path])
     c.set_option(skip.SKIP_OPT_CLUSTER, args.cluster)
+    c.set_option(skip.SKIP_OPT_MMA, {"auto": 0, "single": 1, "pair": 2}[args.mma])
     reg_d = regions.to(dev)
     off_d = offsets.to(dev)
     out_ids = torch.empty(Q, spec.K, dtype=torch.int64, device=dev)

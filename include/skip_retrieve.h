@@ -69,7 +69,8 @@ typedef enum {
     SKIP_OPT_WAIT_TIMEOUT_NS = 1, /* cap on each in-kernel wait (default 2e9 ns) */
     SKIP_OPT_GRID = 2,            /* score-kernel CTAs (0 = one per SM) */
     SKIP_OPT_TIMING = 3,          /* 1: time each kernel with CUDA events */
-    SKIP_OPT_CLUSTER = 4          /* tensor path CTAs per cluster: 0 pick, 1, 2, 4 or 8 */
+    SKIP_OPT_CLUSTER = 4,         /* single-CTA tensor path CTAs per cluster: 0 pick, 1, 2, 4, 8 */
+    SKIP_OPT_MMA = 5              /* tensor path MMA: 0 pick, 1 single CTA, 2 CTA pair */
 } skip_option_t;
 
 enum { SKIP_PATH_AUTO = 0, SKIP_PATH_TENSOR = 1, SKIP_PATH_WARP = 2 };

@@ -7,54 +7,79 @@
 // them to HBM: the epilogue reads each accumulator tile out of tensor memory
 // and keeps, per region row, a sorted top-k list and its k-th score.
 //
-// Tile: A = 128 region rows (TMEM lanes), B = 256 corpus rows (TMEM
+// Tile: 128 region rows per CTA (TMEM lanes) x 256 corpus rows (TMEM
 // columns), K streamed in 64-element (128-byte) slices.  One thread of the
 // epilogue owns one region row, so its threshold lives in a register and the
 // common case -- no score of a 32-column chunk beats it -- costs a max and a
 // compare per chunk.  Corpus rows of a tile are visited in increasing id
 // order, so "beats" is a strict score comparison and ties keep the lower id.
 //
-// Work: a cluster of CL CTAs (CL = 1, 2, 4 or 8) holds CL query blocks and
-// walks items (query group, corpus chunk) in lock step; CTA r of the cluster
-// loads rows [r * 256 / CL, (r + 1) * 256 / CL) of each corpus tile and
-// multicasts them to all CL CTAs, so a corpus tile leaves L2 once per
-// cluster instead of once per query block, and a stage is refilled only when
-// every CTA's MMAs have released it (the MMA commit is multicast too).
-// Persistent clusters walk items cid, cid + #clusters, ...; items are
-// numbered chunk-major so that the clusters of the other query groups read
-// the same chunk at the same time and find it in L2.  Each item leaves one
-// sorted list per region row; the merge kernel combines the chunks.
+// Two MMA shapes:
+//  * single CTA (cta_group::1, M = 128): the CTA stages its 128 region rows
+//    and the whole 256-row corpus tile; a cluster of CL CTAs (1, 2, 4, 8)
+//    with CL query blocks shares each corpus tile -- CTA r loads rows
+//    [r * 256 / CL, (r + 1) * 256 / CL) and multicasts them to all CL CTAs,
+//    and the MMA commits that release a stage are multicast too;
+//  * CTA pair (cta_group::2, M = 256): a cluster of two CTAs on two SMs
+//    computes 256 region rows (two query blocks) against a 256-row corpus
+//    tile, each CTA staging its own 128 region rows and half of the corpus
+//    tile (32 KB per 64-wide slice instead of 48 KB), which buys a deeper
+//    pipeline for the same shared memory.  One thread of the even CTA
+//    issues the MMAs; both CTAs' copies complete on the even CTA's barrier,
+//    its commits are multicast to both CTAs, and both CTAs' epilogues hand
+//    the accumulator back to it.
+//
+// Work: persistent clusters walk items (query group, corpus chunk)
+// cid, cid + #clusters, ...; items are numbered chunk-major so that the
+// clusters of the other query groups read the same chunk at the same time
+// and find it in L2.  Each item leaves one sorted list per region row; the
+// merge kernel combines the chunks.
+//
+// The k-th best score of any chunk of a row bounds the row's global top-k
+// from below, so the chunks of a row share one threshold: each CTA publishes
+// its chunk's k-th score with an atomic max on the order-preserving integer
+// and re-reads the row's best once per tile; a score is kept only if it
+// beats its own chunk's k-th score and is not below the shared one (equal
+// scores from another chunk may still win on id).
 //
 // Per-row lists live in shared memory ([slot][row], k slots) when they fit
 // next to a pipeline of at least two stages, else in global memory.
 //
-// Warp roles (192 threads): warp 0 issues TMA loads into a 2..4-stage
-// shared-memory ring; warp 1 owns TMEM (two 256-column fp32 accumulators)
-// and issues tcgen05.mma from one thread; warps 2..5 are the epilogue, warp w
-// reading TMEM lanes 32 * (w % 4) .. + 31.  Every wait is bounded; a wait
-// that gives up sets the error word, the other roles then give up too, and
-// before exit the producer waits for its copies in flight and the MMA thread
-// for its MMAs, so that TMEM is freed by its owner with nothing outstanding.
+// Warp roles (192 threads): warp 0 issues TMA loads into the shared-memory
+// ring; warp 1 owns TMEM (two 256-column fp32 accumulators) and issues
+// tcgen05.mma from one thread; warps 2..5 are the epilogue, warp w reading
+// TMEM lanes 32 * (w % 4) .. + 31.  Every wait is bounded; a wait that gives
+// up sets the error word, the other roles then give up too, and before exit
+// the producer waits for its copies in flight and the MMA thread for its
+// MMAs, and the cluster synchronises, so that TMEM is freed with nothing
+// outstanding.
 #include "skip_device.cuh"
 #include "skip_internal.h"
 
 namespace skipk {
 namespace {
 
-constexpr int kABytes = kTcTileM * kTcTileK * 2;  // 16 KB
-constexpr int kBBytes = kTcTileN * kTcTileK * 2;  // 32 KB
-constexpr int kStageBytes = kABytes + kBBytes;
-constexpr uint32_t kTmemCols = 512;                 // two 256-column accumulators
+constexpr int kABytes = kTcTileM * kTcTileK * 2;  // 16 KB: 128 region rows x 64
+constexpr int kBFull = kTcTileN * kTcTileK * 2;   // 32 KB: 256 corpus rows x 64
+constexpr uint32_t kTmemCols = 512;               // two 256-column accumulators
 constexpr uint64_t kDrainTimeoutNs = 1000000000ull;  // 1 s for copies/MMAs in flight
-constexpr uint32_t kIdesc = idesc_bf16_f32(kTcTileM, kTcTileN);
-constexpr int kMaxStages = 4;
+constexpr int kMaxStages = 8;
+
+template <bool PAIR>
+struct Geom {
+    static constexpr int kBBytes = PAIR ? kBFull / 2 : kBFull;  // corpus rows staged by one CTA
+    static constexpr int kStageBytes = kABytes + kBBytes;       // per CTA and stage
+    static constexpr uint32_t kTxBytes = PAIR ? 2 * kStageBytes : kStageBytes;  // on the MMA CTA's barrier
+    static constexpr uint32_t kIdesc = idesc_bf16_f32(PAIR ? 2 * kTcTileM : kTcTileM, kTcTileN);
+    static constexpr int kMaxSt = PAIR ? 6 : 4;
+};
 
 struct __align__(8) TcShared {
     uint64_t full[kMaxStages];   // stage loaded (TMA transaction bytes)
     uint64_t empty[kMaxStages];  // stage consumed (tcgen05.commit)
-    uint64_t tfull[2];          // accumulator ready (tcgen05.commit)
-    uint64_t tempty[2];         // accumulator drained (4 epilogue warps)
-    uint64_t drain;             // MMA completion at exit
+    uint64_t tfull[2];           // accumulator ready (tcgen05.commit)
+    uint64_t tempty[2];          // accumulator drained (epilogue warps)
+    uint64_t drain;              // MMA completion at exit
     uint32_t tmem_base;
 };
 
@@ -113,17 +138,19 @@ __device__ __forceinline__ float fmax32(const uint32_t (&v)[32]) {
     return m[0];
 }
 
+template <bool PAIR>
 __global__ void __launch_bounds__(kTcThreads, 1)
     k_tc_score_topk(const __grid_constant__ CUtensorMap tq, const __grid_constant__ CUtensorMap tx,
                     const TcParams p) {
+    using Gm = Geom<PAIR>;
     extern __shared__ uint8_t smem_raw[];
     uint8_t *smem = reinterpret_cast<uint8_t *>(((uintptr_t)smem_raw + 1023) & ~(uintptr_t)1023);
     const int S = p.stages;
     uint8_t *sA = smem;
     uint8_t *sB = smem + S * kABytes;
-    uint64_t *slists = reinterpret_cast<uint64_t *>(smem + S * kStageBytes);
+    uint64_t *slists = reinterpret_cast<uint64_t *>(smem + S * Gm::kStageBytes);
     const size_t list_bytes = p.list_in_smem ? (size_t)kTcTileM * p.k * 8 : 0;
-    TcShared *sh = reinterpret_cast<TcShared *>(smem + S * kStageBytes + list_bytes);
+    TcShared *sh = reinterpret_cast<TcShared *>(smem + S * Gm::kStageBytes + list_bytes);
     const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
     const int items = p.QG * p.G;
     const int KB = (p.d + kTcTileK - 1) / kTcTileK;
@@ -133,15 +160,16 @@ __global__ void __launch_bounds__(kTcThreads, 1)
     const int ncl = CL > 1 ? (int)cluster_count() : (int)gridDim.x;
     const uint16_t mask = (uint16_t)((1u << CL) - 1u);
     const int slice_rows = kTcTileN / CL;
+    const bool mma_cta = !PAIR || rank == 0;
 
     if (threadIdx.x == 0) {
         for (int s = 0; s < S; ++s) {
             mbar_init(smem_addr(&sh->full[s]), 1);
-            mbar_init(smem_addr(&sh->empty[s]), CL);
+            mbar_init(smem_addr(&sh->empty[s]), PAIR ? 1 : CL);
         }
         for (int b = 0; b < 2; ++b) {
             mbar_init(smem_addr(&sh->tfull[b]), 1);
-            mbar_init(smem_addr(&sh->tempty[b]), 4);
+            mbar_init(smem_addr(&sh->tempty[b]), PAIR ? 8 : 4);
         }
         mbar_init(smem_addr(&sh->drain), 1);
         mbar_fence_init();
@@ -151,13 +179,18 @@ __global__ void __launch_bounds__(kTcThreads, 1)
         tma_prefetch_desc(&tx);
     }
     if (warp == 1) {
-        tmem_alloc(smem_addr(&sh->tmem_base), kTmemCols);
-        tmem_relinquish();
+        if constexpr (PAIR) {
+            tmem_alloc_pair(smem_addr(&sh->tmem_base), kTmemCols);
+            tmem_relinquish_pair();
+        } else {
+            tmem_alloc(smem_addr(&sh->tmem_base), kTmemCols);
+            tmem_relinquish();
+        }
     }
     tc_fence_before();
     __syncthreads();
     tc_fence_after();
-    // Every CTA's barriers are initialised before any multicast targets them.
+    // Every CTA's barriers are initialised before any peer copy or arrive.
     if (CL > 1) cluster_sync_all();
     const uint32_t tmem = sh->tmem_base;
 
@@ -177,13 +210,22 @@ __global__ void __launch_bounds__(kTcThreads, 1)
                             break;
                         }
                         const uint32_t fb = smem_addr(&sh->full[s]);
-                        mbar_arrive_expect_tx(fb, kStageBytes);
-                        tma_load_2d(smem_addr(sA + s * kABytes), &tq, fb, kb * kTcTileK, it.mb * kTcTileM);
-                        if (CL == 1)
-                            tma_load_2d(smem_addr(sB + s * kBBytes), &tx, fb, kb * kTcTileK, (int)(t * kTcTileN));
-                        else
-                            tma_load_2d_mc(smem_addr(sB + s * kBBytes + rank * slice_rows * 128), &tx, fb,
-                                           kb * kTcTileK, (int)(t * kTcTileN) + rank * slice_rows, mask);
+                        if (mma_cta) mbar_arrive_expect_tx(fb, Gm::kTxBytes);
+                        const int x = kb * kTcTileK;
+                        if constexpr (PAIR) {
+                            // Both CTAs' copies complete on the MMA CTA's barrier.
+                            const uint32_t fl = mapa_shared(fb, 0);
+                            tma_load_2d_pair(smem_addr(sA + s * kABytes), &tq, fl, x, it.mb * kTcTileM);
+                            tma_load_2d_pair(smem_addr(sB + s * Gm::kBBytes), &tx, fl, x,
+                                             (int)(t * kTcTileN) + rank * (kTcTileN / 2));
+                        } else {
+                            tma_load_2d(smem_addr(sA + s * kABytes), &tq, fb, x, it.mb * kTcTileM);
+                            if (CL == 1)
+                                tma_load_2d(smem_addr(sB + s * Gm::kBBytes), &tx, fb, x, (int)(t * kTcTileN));
+                            else
+                                tma_load_2d_mc(smem_addr(sB + s * Gm::kBBytes + rank * slice_rows * 128), &tx, fb,
+                                               x, (int)(t * kTcTileN) + rank * slice_rows, mask);
+                        }
                         ++issued;
                         if (++s == S) {
                             s = 0;
@@ -194,16 +236,19 @@ __global__ void __launch_bounds__(kTcThreads, 1)
             }
             if (!ok) atomicOr(p.err, kErrTimeout);
             // Copies in flight: wait for the last load issued on every stage.
-            for (int st = 0; st < S; ++st) {
-                const int64_t uses = issued / S + (st < issued % S ? 1 : 0);
-                if (uses == 0) continue;
-                if (!mbar_wait(smem_addr(&sh->full[st]), (uint32_t)((uses - 1) & 1), kDrainTimeoutNs))
-                    atomicOr(p.err, kErrTimeout);
+            // (In a pair both CTAs' copies complete on the MMA CTA's barrier.)
+            if (mma_cta) {
+                for (int st = 0; st < S; ++st) {
+                    const int64_t uses = issued / S + (st < issued % S ? 1 : 0);
+                    if (uses == 0) continue;
+                    if (!mbar_wait(smem_addr(&sh->full[st]), (uint32_t)((uses - 1) & 1), kDrainTimeoutNs))
+                        atomicOr(p.err, kErrTimeout);
+                }
             }
         }
     } else if (warp == 1) {
         // ------------------------------------------------ MMA issuer
-        if (lane == 0) {
+        if (lane == 0 && mma_cta) {
             int s = 0;
             uint32_t ph = 0;
             uint32_t lt = 0;
@@ -225,12 +270,19 @@ __global__ void __launch_bounds__(kTcThreads, 1)
                         }
                         tc_fence_after();
                         const uint64_t ad = smem_desc_k128(smem_addr(sA + s * kABytes));
-                        const uint64_t bd = smem_desc_k128(smem_addr(sB + s * kBBytes));
+                        const uint64_t bd = smem_desc_k128(smem_addr(sB + s * Gm::kBBytes));
 #pragma unroll
-                        for (int kk = 0; kk < kTcTileK / 16; ++kk)
-                            tc_mma_f16(dt, ad + (uint64_t)(kk * 2), bd + (uint64_t)(kk * 2), kIdesc,
-                                       (kb | kk) != 0);
-                        if (CL == 1)
+                        for (int kk = 0; kk < kTcTileK / 16; ++kk) {
+                            if constexpr (PAIR)
+                                tc_mma_f16_pair(dt, ad + (uint64_t)(kk * 2), bd + (uint64_t)(kk * 2), Gm::kIdesc,
+                                                (kb | kk) != 0);
+                            else
+                                tc_mma_f16(dt, ad + (uint64_t)(kk * 2), bd + (uint64_t)(kk * 2), Gm::kIdesc,
+                                           (kb | kk) != 0);
+                        }
+                        if constexpr (PAIR)
+                            tc_commit_pair_mc(smem_addr(&sh->empty[s]), 3);
+                        else if (CL == 1)
                             tc_commit(smem_addr(&sh->empty[s]));
                         else
                             tc_commit_mc(smem_addr(&sh->empty[s]), mask);
@@ -240,12 +292,21 @@ __global__ void __launch_bounds__(kTcThreads, 1)
                         }
                     }
                     if (!ok) break;
-                    tc_commit(smem_addr(&sh->tfull[buf]));
+                    if constexpr (PAIR)
+                        tc_commit_pair_mc(smem_addr(&sh->tfull[buf]), 3);
+                    else
+                        tc_commit(smem_addr(&sh->tfull[buf]));
                 }
             }
             if (!ok) atomicOr(p.err, kErrTimeout);
             // MMAs in flight: a commit arrives once all earlier ones are done.
-            tc_commit(smem_addr(&sh->drain));
+            if constexpr (PAIR)
+                tc_commit_pair_mc(smem_addr(&sh->drain), 3);
+            else
+                tc_commit(smem_addr(&sh->drain));
+            if (!mbar_wait(smem_addr(&sh->drain), 0, kDrainTimeoutNs)) atomicOr(p.err, kErrTimeout);
+        } else if (lane == 0 && PAIR) {
+            // The other CTA of the pair: its TMEM is written by the MMA CTA.
             if (!mbar_wait(smem_addr(&sh->drain), 0, kDrainTimeoutNs)) atomicOr(p.err, kErrTimeout);
         }
     } else {
@@ -264,20 +325,28 @@ __global__ void __launch_bounds__(kTcThreads, 1)
             uint64_t *L = p.list_in_smem ? slists + rib : glist;
             const int ls = p.list_in_smem ? kTcTileM : 1;
             int nfill = 0;
-            float thr = kNegInf;
+            float thr = kNegInf;   // this chunk's k-th score (strict: later ids lose ties)
+            float gthr = kNegInf;  // best k-th score any chunk of this row has found
+            uint32_t published = 0;
+            uint32_t *tau = p.tau + row;
             // Common case: no score of the 32 beats the threshold (a max and
             // a compare).  Otherwise a branch-free bit mask of the survivors
             // is walked in increasing column (= id) order, so that lanes
             // without survivors idle for a few instructions only.
-            auto scan32 = [&](uint32_t (&v)[32], uint32_t id0) {
-                if (!row_valid || !(fmax32(v) > thr)) return;
+            auto scan32 = [&](uint32_t (&vv)[32], uint32_t id0) {
+                if (!row_valid) return;
+                const float mx = fmax32(vv);
+                if (!(mx > thr && mx >= gthr)) return;
                 uint32_t m = 0;
 #pragma unroll
-                for (int j = 0; j < 32; ++j) m |= (__uint_as_float(v[j]) > thr ? 1u : 0u) << j;
+                for (int j = 0; j < 32; ++j) {
+                    const float sj = __uint_as_float(vv[j]);
+                    m |= (sj > thr && sj >= gthr ? 1u : 0u) << j;
+                }
                 while (m) {
                     const int j = __ffs(m) - 1;
                     m &= m - 1;
-                    const float sj = __uint_as_float(select32(v, j));
+                    const float sj = __uint_as_float(select32(vv, j));
                     if (sj > thr) {
                         nfill = list_insert(L, ls, nfill, p.k, make_key(sj, id0 + j));
                         if (nfill == p.k) thr = key_score(L[(p.k - 1) * ls]);
@@ -291,6 +360,16 @@ __global__ void __launch_bounds__(kTcThreads, 1)
                     break;
                 }
                 tc_fence_after();
+                if (row_valid) {
+                    // Publish this chunk's k-th score, then adopt the row's best.
+                    const uint32_t mine = nfill == p.k ? ord_of_score(thr) : 0u;
+                    if (mine > published) {
+                        atomicMax(tau, mine);
+                        published = mine;
+                    }
+                    const uint32_t best = *reinterpret_cast<volatile uint32_t *>(tau);
+                    if (best > published) gthr = score_of_ord(best);
+                }
                 const int64_t n0 = t * kTcTileN;
                 const bool tail = n0 + kTcTileN > p.N;
 #pragma unroll 1
@@ -313,7 +392,13 @@ __global__ void __launch_bounds__(kTcThreads, 1)
                         // Last read of this accumulator: hand it back before scanning.
                         tc_fence_before();
                         __syncwarp();
-                        if (lane == 0) mbar_arrive(smem_addr(&sh->tempty[buf]));
+                        if (lane == 0) {
+                            const uint32_t te = smem_addr(&sh->tempty[buf]);
+                            if (PAIR && rank != 0)
+                                mbar_arrive_cluster(mapa_shared(te, 0));
+                            else
+                                mbar_arrive(te);
+                        }
                     }
                     scan32(v0, id0);
                     scan32(v1, id0 + 32);
@@ -328,34 +413,26 @@ __global__ void __launch_bounds__(kTcThreads, 1)
 
     tc_fence_before();
     __syncthreads();
-    // No peer may still multicast into, or arrive on, this CTA when it exits.
+    // No peer may still copy into, arrive on, or (pair) write the TMEM of
+    // this CTA when it frees TMEM and exits.
     if (CL > 1) cluster_sync_all();
     tc_fence_after();
     if (warp == 1) {
         __syncwarp();
-        tmem_dealloc(tmem, kTmemCols);
+        if constexpr (PAIR)
+            tmem_dealloc_pair(tmem, kTmemCols);
+        else
+            tmem_dealloc(tmem, kTmemCols);
     }
 }
 
-}  // namespace
-
-size_t tc_smem_bytes(int stages, int k, bool list_in_smem) {
-    return 1024 + (size_t)stages * kStageBytes + (list_in_smem ? (size_t)kTcTileM * k * 8 : 0) +
-           sizeof(TcShared);
+template <bool PAIR>
+size_t smem_bytes(int stages, int k, bool list_in_smem) {
+    return 1024 + (size_t)stages * Geom<PAIR>::kStageBytes +
+           (list_in_smem ? (size_t)kTcTileM * k * 8 : 0) + sizeof(TcShared);
 }
 
-void tc_pick_layout(int k, int max_smem, int *stages, bool *list_in_smem) {
-    for (int st = kMaxStages; st >= 2; --st)
-        if (tc_smem_bytes(st, k, true) <= (size_t)max_smem) {
-            *stages = st;
-            *list_in_smem = true;
-            return;
-        }
-    *stages = kMaxStages;
-    *list_in_smem = false;
-}
-
-static cudaLaunchConfig_t tc_config(int grid, int CL, size_t smem, cudaStream_t s, cudaLaunchAttribute *attr) {
+cudaLaunchConfig_t tc_config(int grid, int CL, size_t smem, cudaStream_t s, cudaLaunchAttribute *attr) {
     cudaLaunchConfig_t cfg = {};
     cfg.gridDim = dim3(grid, 1, 1);
     cfg.blockDim = dim3(kTcThreads, 1, 1);
@@ -370,32 +447,51 @@ static cudaLaunchConfig_t tc_config(int grid, int CL, size_t smem, cudaStream_t 
     return cfg;
 }
 
-int tc_max_clusters(int CL, int stages, int k, bool list_in_smem) {
-    const size_t smem = tc_smem_bytes(stages, k, list_in_smem);
-    if (cudaFuncSetAttribute(k_tc_score_topk, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem) !=
-        cudaSuccess) {
+}  // namespace
+
+size_t tc_smem_bytes(bool pair, int stages, int k, bool list_in_smem) {
+    return pair ? smem_bytes<true>(stages, k, list_in_smem) : smem_bytes<false>(stages, k, list_in_smem);
+}
+
+void tc_pick_layout(bool pair, int k, int max_smem, int *stages, bool *list_in_smem) {
+    const int top = pair ? Geom<true>::kMaxSt : Geom<false>::kMaxSt;
+    for (int st = top; st >= 2; --st)
+        if (tc_smem_bytes(pair, st, k, true) <= (size_t)max_smem) {
+            *stages = st;
+            *list_in_smem = true;
+            return;
+        }
+    *stages = 4;
+    *list_in_smem = false;
+}
+
+int tc_max_clusters(bool pair, int CL, int stages, int k, bool list_in_smem) {
+    const size_t smem = tc_smem_bytes(pair, stages, k, list_in_smem);
+    auto kern = pair ? k_tc_score_topk<true> : k_tc_score_topk<false>;
+    if (cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem) != cudaSuccess) {
         cudaGetLastError();
         return 0;
     }
     cudaLaunchAttribute attr[1];
     cudaLaunchConfig_t cfg = tc_config(CL * 64, CL, smem, 0, attr);
     int n = 0;
-    if (cudaOccupancyMaxActiveClusters(&n, k_tc_score_topk, &cfg) != cudaSuccess) {
+    if (cudaOccupancyMaxActiveClusters(&n, kern, &cfg) != cudaSuccess) {
         cudaGetLastError();
         return 0;
     }
     return n;
 }
 
-cudaError_t launch_tc(const CUtensorMap &tq, const CUtensorMap &tx, const TcParams &p, int grid,
+cudaError_t launch_tc(bool pair, const CUtensorMap &tq, const CUtensorMap &tx, const TcParams &p, int grid,
                       cudaStream_t s) {
-    const size_t smem = tc_smem_bytes(p.stages, p.k, p.list_in_smem != 0);
-    cudaError_t e = cudaFuncSetAttribute(k_tc_score_topk, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                                         (int)smem);
+    if (pair && p.CL != 2) return cudaErrorInvalidValue;
+    const size_t smem = tc_smem_bytes(pair, p.stages, p.k, p.list_in_smem != 0);
+    auto kern = pair ? k_tc_score_topk<true> : k_tc_score_topk<false>;
+    cudaError_t e = cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
     if (e != cudaSuccess) return e;
     cudaLaunchAttribute attr[1];
     cudaLaunchConfig_t cfg = tc_config(grid, p.CL, smem, s, attr);
-    return cudaLaunchKernelEx(&cfg, k_tc_score_topk, tq, tx, p);
+    return cudaLaunchKernelEx(&cfg, kern, tq, tx, p);
 }
 
 }  // namespace skipk

@@ -78,6 +78,7 @@ struct skip_corpus {
     uint64_t timeout_ns = kDefaultTimeoutNs;
     int grid = 0;
     int cluster = 0;           // 0 = pick; else CTAs per cluster
+    int mma = 0;               // 0 = pick, 1 = single-CTA MMA, 2 = CTA-pair MMA
     std::map<int, int> cluster_cache;  // resident clusters per (size, stages, list place)
     int timing = 0;
     // Timing: events recorded on the launching stream before each kernel and
@@ -144,6 +145,7 @@ struct Plan {
     int stages = 0;
     bool list_in_smem = false;
     int CL = 1;
+    bool pair = false;
 };
 
 // Corpus chunks G for the tensor path: make MB * G a whole number of waves of
@@ -194,25 +196,36 @@ skip_status_t run_regions(skip_corpus *c, const uint16_t *regions, int R, int k,
     if (tensor) {
         pl.MB = (R + kTcTileM - 1) / kTcTileM;
         pl.tiles = (c->N + kTcTileN - 1) / kTcTileN;
+        // MMA shape: CTA pairs (M = 256) whenever there are two query blocks
+        // to pair, unless set by option.
+        const bool pair = c->mma == 2 || (c->mma == 0 && pl.MB >= 2);
         bool in_smem = false;
         int stages = 0;
-        tc_pick_layout(k, c->max_smem, &stages, &in_smem);
-        // Cluster size: the CTAs of a cluster share each corpus tile (one L2
-        // read, multicast).  Take the largest size that keeps at least 90%
-        // of the SMs the best size keeps busy, unless set by option.
+        tc_pick_layout(pair, k, c->max_smem, &stages, &in_smem);
+        auto max_clusters = [&](int CL) {
+            const int key = (pair ? 10000 : 0) + CL * 100 + stages * 10 + (in_smem ? 1 : 0);
+            auto hit = c->cluster_cache.find(key);
+            if (hit == c->cluster_cache.end())
+                hit = c->cluster_cache.emplace(key, tc_max_clusters(pair, CL, stages, k, in_smem)).first;
+            return hit->second;
+        };
+        // Cluster size (single-CTA MMA): the CTAs of a cluster share each
+        // corpus tile (one L2 read, multicast).  Take the largest size that
+        // keeps at least 90% of the SMs the best size keeps busy, unless set
+        // by option.  A pair is a cluster of two.
         int cl_best = 1, ncl_best = 0;
-        {
+        if (pair) {
+            cl_best = 2;
+            ncl_best = max_clusters(2);
+            if (ncl_best == 0) return SKIP_ECUDA;
+        } else {
             int used[4] = {0, 0, 0, 0}, ncls[4] = {0, 0, 0, 0};
             int best_used = 0;
             for (int i = 0; i < 4; ++i) {
                 const int CL = 1 << i;
                 if (c->cluster && CL != c->cluster) continue;
                 if (!c->cluster && CL > 1 && CL > pl.MB) break;
-                const int key = CL * 100 + stages * 10 + (in_smem ? 1 : 0);
-                auto hit = c->cluster_cache.find(key);
-                if (hit == c->cluster_cache.end())
-                    hit = c->cluster_cache.emplace(key, tc_max_clusters(CL, stages, k, in_smem)).first;
-                ncls[i] = hit->second;
+                ncls[i] = max_clusters(CL);
                 const int QG = (pl.MB + CL - 1) / CL;
                 const double eff = (double)pl.MB / (double)(QG * CL);
                 used[i] = (int)(std::min(ncls[i] * CL, ctas) * eff);
@@ -234,13 +247,17 @@ skip_status_t run_regions(skip_corpus *c, const uint16_t *regions, int R, int k,
         const int items = QG * pl.G;
         pl.grid = std::min(items, ncl) * cl_best;
         const size_t lists_bytes = (size_t)pl.G * pl.R_pad * k * sizeof(uint64_t);
-        skip_status_t st = ensure_ws(c, align_up(ws_extra, 256) + lists_bytes);
+        const size_t tau_bytes = align_up((size_t)pl.R_pad * sizeof(uint32_t), 256);
+        skip_status_t st = ensure_ws(c, align_up(ws_extra, 256) + tau_bytes + lists_bytes);
         if (st) return st;
-        uint64_t *lists = reinterpret_cast<uint64_t *>((char *)c->ws + align_up(ws_extra, 256));
+        uint32_t *tau = reinterpret_cast<uint32_t *>((char *)c->ws + align_up(ws_extra, 256));
+        uint64_t *lists = reinterpret_cast<uint64_t *>((char *)tau + tau_bytes);
         if (keys_out) *keys_out = reg_keys = reinterpret_cast<uint64_t *>(c->ws);
+        if (cudaMemsetAsync(tau, 0, tau_bytes, s) != cudaSuccess) return SKIP_ECUDA;
         CUtensorMap tq, tx;
         if (!encode_bf16_rows(&tq, regions, R, c->d, kTcTileM)) return SKIP_ECUDA;
-        if (!encode_bf16_rows(&tx, c->rows, c->N, c->d, kTcTileN / cl_best)) return SKIP_ECUDA;
+        if (!encode_bf16_rows(&tx, c->rows, c->N, c->d, pair ? kTcTileN / 2 : kTcTileN / cl_best))
+            return SKIP_ECUDA;
         TcParams p;
         p.N = c->N;
         p.d = c->d;
@@ -253,6 +270,7 @@ skip_status_t run_regions(skip_corpus *c, const uint16_t *regions, int R, int k,
         p.G = pl.G;
         p.tiles = pl.tiles;
         p.lists = lists;
+        p.tau = tau;
         p.err = c->err;
         p.timeout_ns = c->timeout_ns;
         p.stages = stages;
@@ -260,7 +278,8 @@ skip_status_t run_regions(skip_corpus *c, const uint16_t *regions, int R, int k,
         pl.stages = p.stages;
         pl.list_in_smem = in_smem;
         record(c, s, "score_topk_tc");
-        cudaError_t e = launch_tc(tq, tx, p, pl.grid, s);
+        pl.pair = pair;
+        cudaError_t e = launch_tc(pair, tq, tx, p, pl.grid, s);
         if (e != cudaSuccess) return cuda_status(e);
         ++pl.launches;
         record(c, s, "merge_lists");
@@ -310,8 +329,9 @@ void write_plan(skip_corpus *c, const Plan &pl, int R, int Q, int k, int K) {
     snprintf(c->plan, sizeof c->plan,
              "{\"path\": \"%s\", \"grid\": %d, \"lists_per_row\": %d, \"query_blocks\": %d, "
              "\"R_total\": %d, \"Q\": %d, \"k_region\": %d, \"K\": %d, \"launches\": %d, "
-             "\"stages\": %d, \"cluster\": %d, \"lists\": \"%s\"}",
+             "\"stages\": %d, \"cluster\": %d, \"mma\": \"%s\", \"lists\": \"%s\"}",
              pl.tensor ? "tensor" : "warpdot", pl.grid, pl.G, pl.MB, R, Q, k, K, pl.launches, pl.stages, pl.CL,
+             pl.pair ? "pair" : "single",
              pl.tensor ? (pl.list_in_smem ? "shared" : "global") : "global");
 }
 
@@ -413,6 +433,10 @@ skip_status_t skip_corpus_set_option(skip_corpus_t c, int option, int64_t value)
             return SKIP_OK;
         case SKIP_OPT_TIMING:
             c->timing = value != 0;
+            return SKIP_OK;
+        case SKIP_OPT_MMA:
+            if (value < 0 || value > 2) return SKIP_EINVAL;
+            c->mma = (int)value;
             return SKIP_OK;
         case SKIP_OPT_CLUSTER:
             if (value != 0 && value != 1 && value != 2 && value != 4 && value != 8) return SKIP_EINVAL;

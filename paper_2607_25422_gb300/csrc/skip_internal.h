@@ -41,6 +41,7 @@ struct TcParams {
     int G;            // corpus chunks (lists per row)
     int64_t tiles;    // corpus tiles of kTcTileN rows
     uint64_t *lists;  // [G][R_pad][k]
+    uint32_t *tau;    // [R_pad] shared per-row threshold (order-preserving ints), zeroed
     int *err;
     uint64_t timeout_ns;
     int stages;       // pipeline depth (2..4)
@@ -50,12 +51,13 @@ constexpr int kTcTileM = 128;   // region rows per tile (TMEM lanes)
 constexpr int kTcTileN = 256;   // corpus rows per tile (TMEM columns)
 constexpr int kTcTileK = 64;    // bf16 elements per stage row (128 bytes)
 constexpr int kTcThreads = 192; // producer warp, MMA warp, 4 epilogue warps
-size_t tc_smem_bytes(int stages, int k, bool list_in_smem);
+// pair: CTA-pair MMA (cta_group::2, clusters of 2); else single-CTA MMA.
+size_t tc_smem_bytes(bool pair, int stages, int k, bool list_in_smem);
 // Deepest pipeline that fits next to shared-memory lists, else global lists.
-void tc_pick_layout(int k, int max_smem, int *stages, bool *list_in_smem);
+void tc_pick_layout(bool pair, int k, int max_smem, int *stages, bool *list_in_smem);
 // Clusters of CL CTAs that can be resident at once with this layout.
-int tc_max_clusters(int CL, int stages, int k, bool list_in_smem);
-cudaError_t launch_tc(const CUtensorMap &tq, const CUtensorMap &tx, const TcParams &p, int grid,
+int tc_max_clusters(bool pair, int CL, int stages, int k, bool list_in_smem);
+cudaError_t launch_tc(bool pair, const CUtensorMap &tq, const CUtensorMap &tx, const TcParams &p, int grid,
                       cudaStream_t s);
 
 // ---- merges -------------------------------------------------------------

@@ -24,12 +24,13 @@ def _bits(t):
     return synth.bf16_bits(t)
 
 
-def run_gpu(corpus, regions, offsets, k, K, path, scale=None, cluster=0):
+def run_gpu(corpus, regions, offsets, k, K, path, scale=None, cluster=0, mma=0):
     dev = torch.device("cuda")
     c = skip.skip_corpus_load(corpus.to(dev), row_scale=None if scale is None else scale.to(dev))
     try:
         c.set_option(skip.SKIP_OPT_PATH, path)
         c.set_option(skip.SKIP_OPT_CLUSTER, cluster)
+        c.set_option(skip.SKIP_OPT_MMA, mma)
         reg = regions.to(dev)
         rid, rsc = skip.skip_retrieve_regions(c, reg, k)
         oid, osc = skip.skip_retrieve(c, reg, torch.as_tensor(offsets).to(dev), k, K)
@@ -126,16 +127,39 @@ def test_random_bf16(case, path):
 
 @pytest.mark.parametrize("cluster", [1, 2, 4, 8])
 def test_cluster_sizes(cluster):
-    """Every cluster size of the tensor path, with query blocks that do not
-    fill the last cluster and a ragged corpus tail."""
+    """Every cluster size of the single-CTA tensor path, with query blocks
+    that do not fill the last cluster and a ragged corpus tail."""
     N, d, R, Q, k, K = 40000, 256, 700, 30, 16, 40
     ct = synth.random_bf16(N, d, seed=77)
     rt = synth.random_bf16(R, d, seed=78)
     offsets = ragged_offsets(Q, R, seed=79)
     cn, rn = _bits(ct), _bits(rt)
     truth = oracle_truth(cn, rn, offsets, k, K)
-    gpu = run_gpu(ct, rt, offsets, k, K, skip.SKIP_PATH_TENSOR, cluster=cluster)
-    assert gpu[4]["cluster"] == cluster
+    gpu = run_gpu(ct, rt, offsets, k, K, skip.SKIP_PATH_TENSOR, cluster=cluster, mma=1)
+    assert gpu[4]["cluster"] == cluster and gpu[4]["mma"] == "single"
+    assert_parity(cn, rn, offsets, k, K, gpu, truth)
+
+
+PAIR_CASES = [
+    # N, d, R, Q, k, K: R spans 1..5 query blocks (odd counts leave a padded CTA)
+    (9000, 128, 100, 6, 10, 20),
+    (33333, 256, 300, 20, 16, 40),
+    (20000, 768, 512, 32, 20, 50),
+    (12000, 512, 620, 40, 100, 100),
+]
+
+
+@pytest.mark.parametrize("case", PAIR_CASES, ids=lambda c: "N%d_d%d_R%d_k%d" % (c[0], c[1], c[2], c[4]))
+def test_pair_mma(case):
+    """The CTA-pair (cta_group::2) tensor path, forced even for one block."""
+    N, d, R, Q, k, K = case
+    ct = synth.random_bf16(N, d, seed=N + 5)
+    rt = synth.random_bf16(R, d, seed=R + 11)
+    offsets = ragged_offsets(Q, R, seed=R)
+    cn, rn = _bits(ct), _bits(rt)
+    truth = oracle_truth(cn, rn, offsets, k, K)
+    gpu = run_gpu(ct, rt, offsets, k, K, skip.SKIP_PATH_TENSOR, mma=2)
+    assert gpu[4]["mma"] == "pair" and gpu[4]["cluster"] == 2
     assert_parity(cn, rn, offsets, k, K, gpu, truth)
 
 
