@@ -42,8 +42,9 @@
 // beats its own chunk's k-th score and is not below the shared one (equal
 // scores from another chunk may still win on id).
 //
-// Per-row lists live in shared memory ([slot][row], k slots) when they fit
-// next to a pipeline of at least two stages, else in global memory.
+// Per-row top-k sets live in shared memory ([slot][row], k slots) when they
+// fit next to a pipeline of at least two stages, else in global memory; a
+// set is unsorted with its smallest key tracked, and sorted at chunk end.
 //
 // Warp roles (192 threads): warp 0 issues TMA loads into the shared-memory
 // ring; warp 1 owns TMEM (two 256-column fp32 accumulators) and issues
@@ -98,18 +99,54 @@ __device__ __forceinline__ Item item_of(const TcParams &p, int v, int rank) {
     return it;
 }
 
-// Insert key into a row list (slot t at L[t * ls], n valid, descending);
-// the caller has checked that key beats the k-th entry.  Returns the new n.
-__device__ __forceinline__ int list_insert(uint64_t *L, int ls, int n, int k, uint64_t key) {
-    int pos = n < k ? n : k - 1;
-    while (pos > 0) {
-        const uint64_t prev = L[(pos - 1) * ls];
-        if (prev >= key) break;
-        L[pos * ls] = prev;
-        --pos;
+// A row's running top-k is an unsorted set of up to k keys (slot t at
+// L[t * ls]) plus the slot of its smallest key.  A key that beats the
+// smallest replaces it and the smallest is found again with k independent
+// loads, which overlap, instead of a shift loop whose loads depend on each
+// other.  The set is sorted once, when the chunk is done.
+struct RowTopK {
+    int n = 0;          // keys held
+    int min_slot = 0;   // slot of the smallest key once n == k
+    uint64_t min_key = 0;
+};
+
+__device__ __forceinline__ void topk_rescan(uint64_t *L, int ls, int k, RowTopK &st) {
+    uint64_t mk = ~0ull;
+    int ms = 0;
+#pragma unroll 4
+    for (int t = 0; t < k; ++t) {
+        const uint64_t x = L[t * ls];
+        if (x < mk) {
+            mk = x;
+            ms = t;
+        }
     }
-    L[pos * ls] = key;
-    return n < k ? n + 1 : n;
+    st.min_key = mk;
+    st.min_slot = ms;
+}
+
+// The caller has checked that key beats the smallest key (or n < k).
+__device__ __forceinline__ void topk_add(uint64_t *L, int ls, int k, RowTopK &st, uint64_t key) {
+    if (st.n < k) {
+        L[st.n * ls] = key;
+        if (++st.n == k) topk_rescan(L, ls, k, st);
+    } else {
+        L[st.min_slot * ls] = key;
+        topk_rescan(L, ls, k, st);
+    }
+}
+
+// Sorts the held keys descending (insertion sort, once per chunk).
+__device__ __forceinline__ void topk_sort(uint64_t *L, int ls, int n) {
+    for (int i = 1; i < n; ++i) {
+        const uint64_t x = L[i * ls];
+        int j = i - 1;
+        while (j >= 0 && L[j * ls] < x) {
+            L[(j + 1) * ls] = L[j * ls];
+            --j;
+        }
+        L[(j + 1) * ls] = x;
+    }
 }
 
 // v[j] for a run-time j without indexing the register array (5 levels of
@@ -324,7 +361,7 @@ __global__ void __launch_bounds__(kTcThreads, 1)
             uint64_t *glist = p.lists + ((int64_t)it.g * p.R_pad + row) * p.k;
             uint64_t *L = p.list_in_smem ? slists + rib : glist;
             const int ls = p.list_in_smem ? kTcTileM : 1;
-            int nfill = 0;
+            RowTopK top;
             float thr = kNegInf;   // this chunk's k-th score (strict: later ids lose ties)
             float gthr = kNegInf;  // best k-th score any chunk of this row has found
             uint32_t published = 0;
@@ -348,8 +385,8 @@ __global__ void __launch_bounds__(kTcThreads, 1)
                     m &= m - 1;
                     const float sj = __uint_as_float(select32(vv, j));
                     if (sj > thr) {
-                        nfill = list_insert(L, ls, nfill, p.k, make_key(sj, id0 + j));
-                        if (nfill == p.k) thr = key_score(L[(p.k - 1) * ls]);
+                        topk_add(L, ls, p.k, top, make_key(sj, id0 + j));
+                        if (top.n == p.k) thr = key_score(top.min_key);
                     }
                 }
             };
@@ -362,7 +399,7 @@ __global__ void __launch_bounds__(kTcThreads, 1)
                 tc_fence_after();
                 if (row_valid) {
                     // Publish this chunk's k-th score, then adopt the row's best.
-                    const uint32_t mine = nfill == p.k ? ord_of_score(thr) : 0u;
+                    const uint32_t mine = top.n == p.k ? ord_of_score(thr) : 0u;
                     if (mine > published) {
                         atomicMax(tau, mine);
                         published = mine;
@@ -405,7 +442,8 @@ __global__ void __launch_bounds__(kTcThreads, 1)
                 }
             }
             if (row_valid) {
-                for (int t = 0; t < p.k; ++t) glist[t] = t < nfill ? L[t * ls] : 0ull;
+                topk_sort(L, ls, top.n);
+                for (int t = 0; t < p.k; ++t) glist[t] = t < top.n ? L[t * ls] : 0ull;
             }
         }
         if (!ok && lane == 0) atomicOr(p.err, kErrTimeout);
