@@ -154,6 +154,36 @@ SKIP_API skip_status_t skip_retrieve_host(skip_corpus_t corpus, const uint16_t *
                                  int32_t R_total, int32_t k_region, int32_t K, int64_t *out_ids,
                                  float *out_scores, void *stream);
 
+/*
+ * skip_retrieve_regions_noalloc -- the per-region step for callers that
+ * cannot allocate device memory.  The paper has no counterpart: this entry
+ * point exists for callers whose device memory is owned by a host framework
+ * (every allocation must come from its pool) and for serving loops that
+ * cannot afford the device-wide synchronisation of cudaMalloc/cudaFree.
+ *
+ * It takes the corpus as device pointers instead of a handle and allocates
+ * nothing: its scratch is one 16 MiB array in the library's device memory,
+ * created once per device that loads the library and kept until the process
+ * exits.  The first call on a device looks that array's address up (make it
+ * before any stream capture).  All calls on a device share the array, so
+ * calls that overlap on the GPU race; calls ordered on one stream do not.
+ *
+ *  corpus_rows     device [N x d] row-major, bf16 bits or e4m3 bytes (dtype);
+ *                  row_scale device [N] fp32 for SKIP_E4M3, NULL for bf16.
+ *  regions         device bf16 [R_total x d].
+ *  reg_ids/scores  device int64 / fp32 [R_total x k_region], each row sorted
+ *                  by (score desc, id asc) -- the same result as
+ *                  skip_retrieve_regions.
+ * Limits as skip_retrieve_regions, plus: the scratch, about
+ * 8 * k_region * (#SMs * R_total + #SMs * 64) bytes, must fit in 16 MiB,
+ * else SKIP_EUNSUPPORTED.  Asynchronous on `stream`.
+ */
+SKIP_API skip_status_t skip_retrieve_regions_noalloc(const void *corpus_rows, int64_t N, int32_t d,
+                                                     skip_dtype_t dtype, const float *row_scale,
+                                                     const void *regions, int32_t R_total,
+                                                     int32_t k_region, int64_t *reg_ids,
+                                                     float *reg_scores, void *stream);
+
 /* Synchronises `stream`, then reports and clears the handle's error word:
  * SKIP_ETIMEOUT if a kernel's bounded wait gave up since the last check,
  * SKIP_EINVAL if region offsets were inconsistent with R_total (clamped),

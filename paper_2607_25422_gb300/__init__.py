@@ -57,11 +57,12 @@ def load_library():
     lib.skip_sync_status.argtypes = [P, P]
     lib.skip_last_plan.argtypes = [P, ctypes.c_char_p, i32]
     lib.skip_timing_report.argtypes = [P, ctypes.c_char_p, i32]
+    lib.skip_retrieve_regions_noalloc.argtypes = [P, i64, i32, ctypes.c_int, P, P, i32, i32, P, P, P]
     lib.skip_status_string.argtypes = [ctypes.c_int]
     lib.skip_status_string.restype = ctypes.c_char_p
     for f in ("skip_corpus_load", "skip_corpus_free", "skip_corpus_set_option", "skip_retrieve",
               "skip_retrieve_regions", "skip_retrieve_host", "skip_sync_status", "skip_last_plan",
-              "skip_timing_report"):
+              "skip_timing_report", "skip_retrieve_regions_noalloc"):
         getattr(lib, f).restype = ctypes.c_int
     _lib = lib
     return lib
@@ -205,6 +206,24 @@ def skip_retrieve_host(corpus: Corpus, regions: torch.Tensor, region_offsets: to
                                 ctypes.c_void_p(_stream(stream)))
     _check(st, "skip_retrieve_host")
     return out_ids, out_scores
+
+
+def skip_retrieve_regions_noalloc(corpus_rows: torch.Tensor, regions: torch.Tensor, k_region: int,
+                                  reg_ids: torch.Tensor, reg_scores: torch.Tensor,
+                                  row_scale: Optional[torch.Tensor] = None, stream=None):
+    """Per-region step on caller-owned device tensors, with no device
+    allocation by the library (its scratch is a fixed array in the library's
+    device memory).  For callers whose device memory must all come from
+    their own pool; the output tensors are theirs to allocate."""
+    lib = load_library()
+    if not (corpus_rows.is_cuda and regions.is_cuda and reg_ids.is_cuda and reg_scores.is_cuda):
+        raise ValueError("skip_retrieve_regions_noalloc takes device tensors")
+    dtype = SKIP_BF16 if corpus_rows.dtype in (torch.bfloat16, torch.uint16, torch.int16) else SKIP_E4M3
+    st = lib.skip_retrieve_regions_noalloc(_ptr(corpus_rows), corpus_rows.shape[0], corpus_rows.shape[1], dtype,
+                                           _ptr(row_scale), _ptr(regions), regions.shape[0], int(k_region),
+                                           _ptr(reg_ids), _ptr(reg_scores), ctypes.c_void_p(_stream(stream)))
+    _check(st, "skip_retrieve_regions_noalloc")
+    return reg_ids, reg_scores
 
 
 def skip_sync_status(corpus: Corpus, stream=None) -> int:
