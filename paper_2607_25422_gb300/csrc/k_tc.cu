@@ -273,14 +273,15 @@ __global__ void __launch_bounds__(kTcThreads, 1)
             }
             if (!ok) atomicOr(p.err, kErrTimeout);
             // Copies in flight: wait for the last load issued on every stage.
-            // (In a pair both CTAs' copies complete on the MMA CTA's barrier.)
-            if (mma_cta) {
-                for (int st = 0; st < S; ++st) {
-                    const int64_t uses = issued / S + (st < issued % S ? 1 : 0);
-                    if (uses == 0) continue;
-                    if (!mbar_wait(smem_addr(&sh->full[st]), (uint32_t)((uses - 1) & 1), kDrainTimeoutNs))
-                        atomicOr(p.err, kErrTimeout);
-                }
+            // In a pair both CTAs' copies complete on the MMA CTA's barrier, so
+            // the other CTA waits instead for the release of its last stages
+            // (which follows their arrival); a release that never comes ends
+            // the wait after the bound, long after any copy has landed.
+            for (int st = 0; st < S; ++st) {
+                const int64_t uses = issued / S + (st < issued % S ? 1 : 0);
+                if (uses == 0) continue;
+                const uint32_t bar = mma_cta ? smem_addr(&sh->full[st]) : smem_addr(&sh->empty[st]);
+                if (!mbar_wait(bar, (uint32_t)((uses - 1) & 1), kDrainTimeoutNs)) atomicOr(p.err, kErrTimeout);
             }
         }
     } else if (warp == 1) {
