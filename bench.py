@@ -43,9 +43,12 @@ sys.path.insert(0, ROOT)
 import synth  # noqa: E402
 
 METRIC = "retrieval queries/s and corpus GB/s (1 GB300) as fraction of roofline"
-SCORE_KERNELS = ("score_topk_tc", "score_topk_warpdot")
+SCORE_KERNELS = ("score_topk_tc", "score_topk_tc_e4m3", "score_topk_warpdot")
 KERNEL_SOURCES = {
-    "score_topk_tc": ["paper_2607_25422_gb300/csrc/k_tc.cu", "paper_2607_25422_gb300/csrc/skip_device.cuh"],
+    "score_topk_tc": ["paper_2607_25422_gb300/csrc/k_tc.cu", "paper_2607_25422_gb300/csrc/tc_common.cuh",
+                      "paper_2607_25422_gb300/csrc/skip_device.cuh"],
+    "score_topk_tc_e4m3": ["paper_2607_25422_gb300/csrc/k_tc_fp8.cu", "paper_2607_25422_gb300/csrc/tc_common.cuh",
+                           "paper_2607_25422_gb300/csrc/skip_device.cuh"],
     "score_topk_warpdot": ["paper_2607_25422_gb300/csrc/k_warpdot.cu",
                            "paper_2607_25422_gb300/csrc/skip_device.cuh"],
 }

@@ -56,6 +56,20 @@ bool encode_bf16_rows(CUtensorMap *map, const void *base, int64_t rows, int d, i
               CU_TENSOR_MAP_L2_PROMOTION_L2_256B, CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) == CUDA_SUCCESS;
 }
 
+// 2D byte tensor map over the e4m3 corpus [rows x d], box 256 rows x 128
+// elements (128 bytes), 128-byte swizzle, zero fill out of bounds.
+bool encode_e4m3_rows(CUtensorMap *map, const void *base, int64_t rows, int d) {
+    EncodeTiledFn fn = encode_fn();
+    if (!fn) return false;
+    cuuint64_t dims[2] = {(cuuint64_t)d, (cuuint64_t)rows};
+    cuuint64_t strides[1] = {(cuuint64_t)d};
+    cuuint32_t box[2] = {128, (cuuint32_t)kTcTileN};
+    cuuint32_t estr[2] = {1, 1};
+    return fn(map, CU_TENSOR_MAP_DATA_TYPE_UINT8, 2, const_cast<void *>(base), dims, strides, box, estr,
+              CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B, CU_TENSOR_MAP_L2_PROMOTION_L2_256B,
+              CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) == CUDA_SUCCESS;
+}
+
 }  // namespace
 
 struct skip_corpus {
@@ -190,9 +204,63 @@ skip_status_t run_regions(skip_corpus *c, const uint16_t *regions, int R, int k,
     else if (c->path == SKIP_PATH_WARP)
         tensor = false;
     else
-        tensor = R > 8;
-    if (e4m3 || !c->tmap_ok) tensor = false;  // the tensor path streams bf16 tiles
+        tensor = e4m3 ? R > 4 : R > 8;
+    if (!e4m3 && !c->tmap_ok) tensor = false;
     pl.tensor = tensor;
+    if (tensor && e4m3) {
+        // e4m3 corpus: single-CTA MMA on bf16-widened corpus tiles.
+        pl.MB = (R + kTcTileM - 1) / kTcTileM;
+        pl.tiles = (c->N + kTcTileN - 1) / kTcTileN;
+        pl.R_pad = pl.MB * kTcTileM;
+        pl.CL = 1;
+        pl.G = pick_chunks(pl.MB, pl.tiles, ctas);
+        const int items = pl.MB * pl.G;
+        pl.grid = std::min(items, ctas);
+        bool in_smem = false;
+        int stages = 0, raw_stages = 0;
+        tc_fp8_pick_layout(k, c->max_smem, &stages, &raw_stages, &in_smem);
+        const size_t lists_bytes = (size_t)pl.G * pl.R_pad * k * sizeof(uint64_t);
+        const size_t tau_bytes = align_up((size_t)pl.R_pad * sizeof(uint32_t), 256);
+        skip_status_t st = ensure_ws(c, align_up(ws_extra, 256) + tau_bytes + lists_bytes);
+        if (st) return st;
+        uint32_t *tau = reinterpret_cast<uint32_t *>((char *)c->ws + align_up(ws_extra, 256));
+        uint64_t *lists = reinterpret_cast<uint64_t *>((char *)tau + tau_bytes);
+        if (keys_out) *keys_out = reg_keys = reinterpret_cast<uint64_t *>(c->ws);
+        if (cudaMemsetAsync(tau, 0, tau_bytes, s) != cudaSuccess) return SKIP_ECUDA;
+        CUtensorMap tq, traw;
+        if (!encode_bf16_rows(&tq, regions, R, c->d, kTcTileM)) return SKIP_ECUDA;
+        if (!encode_e4m3_rows(&traw, c->rows, c->N, c->d)) return SKIP_ECUDA;
+        TcParams p;
+        p.N = c->N;
+        p.d = c->d;
+        p.R = R;
+        p.R_pad = pl.R_pad;
+        p.k = k;
+        p.MB = pl.MB;
+        p.CL = 1;
+        p.QG = pl.MB;
+        p.G = pl.G;
+        p.tiles = pl.tiles;
+        p.lists = lists;
+        p.tau = tau;
+        p.err = c->err;
+        p.timeout_ns = c->timeout_ns;
+        p.stages = stages;
+        p.raw_stages = raw_stages;
+        p.list_in_smem = in_smem;
+        p.scale = c->scale;
+        pl.stages = stages;
+        pl.list_in_smem = in_smem;
+        record(c, s, "score_topk_tc_e4m3");
+        cudaError_t e = launch_tc_fp8(tq, traw, p, pl.grid, s);
+        if (e != cudaSuccess) return cuda_status(e);
+        ++pl.launches;
+        record(c, s, "merge_lists");
+        e = launch_merge_lists(lists, pl.G, (int64_t)pl.R_pad * k, R, k, reg_keys, reg_ids, reg_scores, s);
+        if (e != cudaSuccess) return cuda_status(e);
+        ++pl.launches;
+        return SKIP_OK;
+    }
     if (tensor) {
         pl.MB = (R + kTcTileM - 1) / kTcTileM;
         pl.tiles = (c->N + kTcTileN - 1) / kTcTileN;
@@ -275,6 +343,8 @@ skip_status_t run_regions(skip_corpus *c, const uint16_t *regions, int R, int k,
         p.timeout_ns = c->timeout_ns;
         p.stages = stages;
         p.list_in_smem = in_smem;
+        p.scale = nullptr;
+        p.raw_stages = 0;
         pl.stages = p.stages;
         pl.list_in_smem = in_smem;
         record(c, s, "score_topk_tc");

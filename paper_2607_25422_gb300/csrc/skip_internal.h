@@ -44,8 +44,10 @@ struct TcParams {
     uint32_t *tau;    // [R_pad] shared per-row threshold (order-preserving ints), zeroed
     int *err;
     uint64_t timeout_ns;
-    int stages;       // pipeline depth (2..4)
+    int stages;       // operand pipeline depth
     int list_in_smem; // per-row lists in shared memory (else global)
+    const float *scale;  // [N] row scales (e4m3 corpus only)
+    int raw_stages;      // e4m3 corpus: depth of the raw-slice ring
 };
 constexpr int kTcTileM = 128;   // region rows per tile (TMEM lanes)
 constexpr int kTcTileN = 256;   // corpus rows per tile (TMEM columns)
@@ -59,6 +61,11 @@ void tc_pick_layout(bool pair, int k, int max_smem, int *stages, bool *list_in_s
 int tc_max_clusters(bool pair, int CL, int stages, int k, bool list_in_smem);
 cudaError_t launch_tc(bool pair, const CUtensorMap &tq, const CUtensorMap &tx, const TcParams &p, int grid,
                       cudaStream_t s);
+
+// e4m3 corpus (single-CTA MMA, corpus widened to bf16 in shared memory).
+void tc_fp8_pick_layout(int k, int max_smem, int *stages, int *raw_stages, bool *list_in_smem);
+cudaError_t launch_tc_fp8(const CUtensorMap &tq, const CUtensorMap &traw, const TcParams &p, int grid,
+                          cudaStream_t s);
 
 // ---- merges -------------------------------------------------------------
 // Per-region merge of G sorted lists into the exact top-k (keys and/or

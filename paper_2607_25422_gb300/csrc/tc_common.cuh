@@ -1,0 +1,104 @@
+// Pieces shared by the tensor-core score kernels (bf16 and e4m3 corpora):
+// the work item of a persistent CTA, the per-row top-k set kept by the
+// epilogue, and register helpers for the 32-column chunks it scans.
+#pragma once
+
+#include "skip_device.cuh"
+#include "skip_internal.h"
+
+namespace skipk {
+namespace tc {
+
+struct Item {
+    int mb;
+    int g;
+    int64_t t0, t1;
+};
+
+__device__ __forceinline__ Item item_of(const TcParams &p, int v, int rank) {
+    Item it;
+    it.g = v / p.QG;
+    it.mb = (v - it.g * p.QG) * p.CL + rank;
+    it.t0 = (int64_t)it.g * p.tiles / p.G;
+    it.t1 = (int64_t)(it.g + 1) * p.tiles / p.G;
+    return it;
+}
+
+// A row's running top-k is an unsorted set of up to k keys (slot t at
+// L[t * ls]) plus the slot of its smallest key.  A key that beats the
+// smallest replaces it and the smallest is found again with k independent
+// loads, which overlap, instead of a shift loop whose loads depend on each
+// other.  The set is sorted once, when the chunk is done.
+struct RowTopK {
+    int n = 0;          // keys held
+    int min_slot = 0;   // slot of the smallest key once n == k
+    uint64_t min_key = 0;
+};
+
+__device__ __forceinline__ void topk_rescan(uint64_t *L, int ls, int k, RowTopK &st) {
+    uint64_t mk = ~0ull;
+    int ms = 0;
+#pragma unroll 4
+    for (int t = 0; t < k; ++t) {
+        const uint64_t x = L[t * ls];
+        if (x < mk) {
+            mk = x;
+            ms = t;
+        }
+    }
+    st.min_key = mk;
+    st.min_slot = ms;
+}
+
+// The caller has checked that key beats the smallest key (or n < k).
+__device__ __forceinline__ void topk_add(uint64_t *L, int ls, int k, RowTopK &st, uint64_t key) {
+    if (st.n < k) {
+        L[st.n * ls] = key;
+        if (++st.n == k) topk_rescan(L, ls, k, st);
+    } else {
+        L[st.min_slot * ls] = key;
+        topk_rescan(L, ls, k, st);
+    }
+}
+
+// Sorts the held keys descending (insertion sort, once per chunk).
+__device__ __forceinline__ void topk_sort(uint64_t *L, int ls, int n) {
+    for (int i = 1; i < n; ++i) {
+        const uint64_t x = L[i * ls];
+        int j = i - 1;
+        while (j >= 0 && L[j * ls] < x) {
+            L[(j + 1) * ls] = L[j * ls];
+            --j;
+        }
+        L[(j + 1) * ls] = x;
+    }
+}
+
+// v[j] for a run-time j without indexing the register array (5 levels of
+// selects), so that v stays in registers.
+__device__ __forceinline__ uint32_t select32(const uint32_t (&v)[32], int j) {
+    uint32_t a[16];
+#pragma unroll
+    for (int i = 0; i < 16; ++i) a[i] = (j & 16) ? v[i + 16] : v[i];
+#pragma unroll
+    for (int i = 0; i < 8; ++i) a[i] = (j & 8) ? a[i + 8] : a[i];
+#pragma unroll
+    for (int i = 0; i < 4; ++i) a[i] = (j & 4) ? a[i + 4] : a[i];
+#pragma unroll
+    for (int i = 0; i < 2; ++i) a[i] = (j & 2) ? a[i + 2] : a[i];
+    return (j & 1) ? a[1] : a[0];
+}
+
+__device__ __forceinline__ float fmax32(const uint32_t (&v)[32]) {
+    float m[16];
+#pragma unroll
+    for (int j = 0; j < 16; ++j) m[j] = fmaxf(__uint_as_float(v[j]), __uint_as_float(v[j + 16]));
+#pragma unroll
+    for (int w = 8; w; w >>= 1)
+#pragma unroll
+        for (int j = 0; j < w; ++j) m[j] = fmaxf(m[j], m[j + w]);
+    return m[0];
+}
+
+}  // namespace tc
+}  // namespace skipk

@@ -209,6 +209,24 @@ def test_random_e4m3(case):
     assert_parity(cn, rn, offsets, k, K, gpu, truth, scale_np=sn)
 
 
+@pytest.mark.parametrize("case", [(5000, 1024, 32, 1, 10, 100), (7001, 80, 20, 4, 7, 30),
+                                  (3000, 256, 130, 9, 16, 40), (20000, 512, 40, 5, 50, 60)],
+                         ids=lambda c: "N%d_d%d_R%d_k%d" % (c[0], c[1], c[2], c[4]))
+def test_e4m3_tensor_path(case):
+    """e4m3 corpus on the tensor cores (tiles widened to bf16 in shared
+    memory, row scales applied to the accumulator)."""
+    N, d, R, Q, k, K = case
+    spec = synth.WorkloadSpec("e4m3_tc", 60 + d, N, d, "e4m3", Q, (1, 1), k, K, "gaussian")
+    corpus, scale, _ = synth.make_corpus(spec)
+    rt = synth.random_bf16(R, d, seed=R + 5)
+    offsets = ragged_offsets(Q, R, seed=N)
+    cn, rn, sn = corpus.numpy(), _bits(rt), scale.numpy()
+    truth = oracle_truth(cn, rn, offsets, k, K, scale_np=sn)
+    gpu = run_gpu(corpus, rt, offsets, k, K, skip.SKIP_PATH_TENSOR, scale=scale)
+    assert gpu[4]["path"] == "tensor"
+    assert_parity(cn, rn, offsets, k, K, gpu, truth, scale_np=sn)
+
+
 def test_host_entry_point_matches_device():
     ct = synth.random_bf16(9000, 256, seed=8)
     rt = synth.random_bf16(40, 256, seed=9)
