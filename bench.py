@@ -43,12 +43,18 @@ sys.path.insert(0, ROOT)
 import synth  # noqa: E402
 
 METRIC = "retrieval queries/s and corpus GB/s (1 GB300) as fraction of roofline"
-SCORE_KERNELS = ("score_topk_tc", "score_topk_tc_e4m3", "score_topk_warpdot")
+SCORE_KERNELS = ("score_topk_tc", "score_topk_tc_e4m3", "score_topk_latency", "score_topk_latency_e4m3",
+                 "score_topk_warpdot")
 KERNEL_SOURCES = {
     "score_topk_tc": ["paper_2607_25422_gb300/csrc/k_tc.cu", "paper_2607_25422_gb300/csrc/tc_common.cuh",
                       "paper_2607_25422_gb300/csrc/skip_device.cuh"],
     "score_topk_tc_e4m3": ["paper_2607_25422_gb300/csrc/k_tc_fp8.cu", "paper_2607_25422_gb300/csrc/tc_common.cuh",
                            "paper_2607_25422_gb300/csrc/skip_device.cuh"],
+    "score_topk_latency": ["paper_2607_25422_gb300/csrc/k_latency.cu", "paper_2607_25422_gb300/csrc/tc_common.cuh",
+                           "paper_2607_25422_gb300/csrc/skip_device.cuh"],
+    "score_topk_latency_e4m3": ["paper_2607_25422_gb300/csrc/k_latency.cu",
+                                "paper_2607_25422_gb300/csrc/tc_common.cuh",
+                                "paper_2607_25422_gb300/csrc/skip_device.cuh"],
     "score_topk_warpdot": ["paper_2607_25422_gb300/csrc/k_warpdot.cu",
                            "paper_2607_25422_gb300/csrc/skip_device.cuh"],
 }
@@ -260,7 +266,7 @@ def main():
     ap.add_argument("--workload", default="clustered_1m", choices=sorted(synth.WORKLOADS))
     ap.add_argument("--cpu-questions", type=int, default=8, help="questions in the oracle sample")
     ap.add_argument("--no-cpu-baseline", action="store_true")
-    ap.add_argument("--path", default="auto", choices=["auto", "tensor", "warp"])
+    ap.add_argument("--path", default="auto", choices=["auto", "tensor", "warp", "latency"])
     ap.add_argument("--cluster", type=int, default=0, choices=[0, 1, 2, 4, 8],
                     help="single-CTA tensor path CTAs per cluster (0 = library's choice)")
     ap.add_argument("--mma", default="auto", choices=["auto", "single", "pair"],
@@ -285,7 +291,7 @@ def main():
     corpus_np, scale_np = host_corpus(corpus, scale) if keep_host else (None, None)
     del corpus
     torch.cuda.empty_cache()
-    c.set_option(skip.SKIP_OPT_PATH, {"auto": 0, "tensor": 1, "warp": 2}[args.path])
+    c.set_option(skip.SKIP_OPT_PATH, {"auto": 0, "tensor": 1, "warp": 2, "latency": 3}[args.path])
     c.set_option(skip.SKIP_OPT_CLUSTER, args.cluster)
     c.set_option(skip.SKIP_OPT_MMA, {"auto": 0, "single": 1, "pair": 2}[args.mma])
     reg_d = regions.to(dev)

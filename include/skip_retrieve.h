@@ -65,7 +65,7 @@ typedef enum {
 } skip_status_t;
 
 typedef enum {
-    SKIP_OPT_PATH = 0,            /* score kernel: 0 auto, 1 tensor core, 2 warp-dot */
+    SKIP_OPT_PATH = 0,            /* score kernel: 0 auto, 1 tensor core, 2 warp-dot, 3 small-batch tensor */
     SKIP_OPT_WAIT_TIMEOUT_NS = 1, /* cap on each in-kernel wait (default 2e9 ns) */
     SKIP_OPT_GRID = 2,            /* score-kernel CTAs (0 = one per SM) */
     SKIP_OPT_TIMING = 3,          /* 1: time each kernel with CUDA events */
@@ -73,7 +73,7 @@ typedef enum {
     SKIP_OPT_MMA = 5              /* tensor path MMA: 0 pick, 1 single CTA, 2 CTA pair */
 } skip_option_t;
 
-enum { SKIP_PATH_AUTO = 0, SKIP_PATH_TENSOR = 1, SKIP_PATH_WARP = 2 };
+enum { SKIP_PATH_AUTO = 0, SKIP_PATH_TENSOR = 1, SKIP_PATH_WARP = 2, SKIP_PATH_LATENCY = 3 };
 
 /* Limits checked by every retrieval call. */
 #define SKIP_MAX_K_REGION 1024

@@ -1,0 +1,417 @@
+// Tensor-core score + fused top-k for small region batches (latency mode).
+//
+// Step: per-region MIPS top-k (paper App. B.2 Def. B.2, MIPS(q_r, D; k_r);
+// §3.3 Eq. rcsr) when a batch holds at most 32 region rows -- one question
+// with its regions, the paper's serving case.  Such a scan is bound by
+// streaming the corpus from HBM, so the corpus tile is the streamed MMA
+// operand A (128 corpus rows = 128 TMEM lanes) and the region queries are a
+// small operand B that stays in shared memory for the whole launch: the MMA
+// D = X_tile Q^T leaves, in each TMEM lane, one corpus row's scores against
+// every query.
+//
+// e4m3 corpus: the tensor cores take e4m3 directly (kind::f8f6f4), so the
+// corpus tile is never widened; instead each bf16 query q is split once per
+// call into three e4m3 parts with power-of-two scales,
+//     q ~= s0 a + s1 b + s2 c,   a = e4m3(q / s0), b = e4m3((q - s0 a) / s1), ...
+// each part capturing the previous residual to 4 significant bits, so the
+// remainder is below 2^-12 |q| per element and the score differs from the
+// exact one by less than 2^-12 |q| |x| (unit vectors: 2.5e-4).  Part p of
+// query r is row 32 p + r of B (96 rows); the epilogue combines the three
+// 32-column groups, times the corpus row's scale.  Products of e4m3 values
+// are exact in the fp32 accumulator.
+// bf16 corpus: B is the bf16 queries themselves (kind::f16).
+//
+// Epilogue: lane = corpus row, so for each query the 32 rows of a warp are
+// compared with the query's threshold at once (a ballot); lane q owns the
+// running top-k set of query q for its warp's rows (an unsorted set with its
+// minimum tracked, in shared memory) and inserts the ballot's survivors in
+// increasing row (= id) order.  A per-query threshold shared by all CTAs
+// (atomic max of the sets' k-th scores) prunes the rest.  At the end of a
+// chunk the four warps' sets of each query are merged into the chunk's list.
+//
+// Warps (192 threads): 0 TMA producer, 1 TMEM owner and MMA issuer, 2..5
+// epilogue.  Bounded waits and drains as in the other tensor kernels.
+#include "skip_device.cuh"
+#include "skip_internal.h"
+#include "tc_common.cuh"
+
+namespace skipk {
+namespace {
+
+using namespace tc;
+
+constexpr int kRows = 128;                      // corpus rows per tile
+constexpr int kSlice = 128;                     // bytes of a row per K slice
+constexpr int kAStage = kRows * kSlice;         // 16 KB
+constexpr int kMaxStages = 12;
+constexpr int kThreads = 192;
+constexpr uint32_t kTmemCols = 256;             // two 128-column accumulators
+constexpr uint64_t kDrainTimeoutNs = 1000000000ull;
+
+struct __align__(8) LatShared {
+    uint64_t full[kMaxStages];
+    uint64_t empty[kMaxStages];
+    uint64_t bfull;  // resident query operand loaded
+    uint64_t tfull[2];
+    uint64_t tempty[2];
+    uint64_t drain;
+    uint64_t sorted;  // the 128 epilogue threads have sorted their sets
+    uint64_t merged;  // ... and merged them into the chunk's lists
+    uint32_t tmem_base;
+    float qscale[3][kLatMaxR];
+    float thr[4][32];   // per epilogue warp: each query's set threshold (k-th score)
+    float gthr[4][32];  // ... and the shared threshold it has adopted
+};
+
+template <bool FP8>
+__global__ void __launch_bounds__(kThreads, 1)
+    k_latency_score_topk(const __grid_constant__ CUtensorMap ta, const __grid_constant__ CUtensorMap tb,
+                         const LatParams p) {
+    extern __shared__ uint8_t smem_raw[];
+    uint8_t *smem = reinterpret_cast<uint8_t *>(((uintptr_t)smem_raw + 1023) & ~(uintptr_t)1023);
+    const int S = p.stages;
+    const int KS = p.slices;                 // K slices per corpus row
+    const int bslice = p.Npad * kSlice;      // bytes of one resident B slice
+    uint8_t *sB = smem;
+    uint8_t *sA = sB + KS * bslice;
+    uint64_t *slists = reinterpret_cast<uint64_t *>(sA + S * kAStage);
+    float *strans = reinterpret_cast<float *>(slists + (size_t)4 * p.R * p.k);  // [4][32][33]
+    LatShared *sh = reinterpret_cast<LatShared *>(strans + 4 * 32 * 33);
+    const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+    constexpr int kElemsPerSlice = FP8 ? 128 : 64;
+    constexpr uint32_t kIdescBase = FP8 ? idesc_e4m3_f32(kRows, 16) : idesc_bf16_f32(kRows, 16);
+    const uint32_t idesc = (kIdescBase & ~(0x3Fu << 17)) | ((uint32_t)(p.Npad >> 3) << 17);
+
+    if (threadIdx.x == 0) {
+        for (int s = 0; s < S; ++s) {
+            mbar_init(smem_addr(&sh->full[s]), 1);
+            mbar_init(smem_addr(&sh->empty[s]), 1);
+        }
+        mbar_init(smem_addr(&sh->bfull), 1);
+        for (int b = 0; b < 2; ++b) {
+            mbar_init(smem_addr(&sh->tfull[b]), 1);
+            mbar_init(smem_addr(&sh->tempty[b]), 4);
+        }
+        mbar_init(smem_addr(&sh->drain), 1);
+        mbar_init(smem_addr(&sh->sorted), 128);
+        mbar_init(smem_addr(&sh->merged), 128);
+        mbar_fence_init();
+    }
+    if (FP8)
+        for (int i = threadIdx.x; i < 3 * kLatMaxR; i += blockDim.x) {
+            const int part = i / kLatMaxR, q = i % kLatMaxR;
+            sh->qscale[part][q] = q < p.R ? p.qscale[part * p.R + q] : 0.0f;
+        }
+    if (warp == 0 && lane == 0) {
+        tma_prefetch_desc(&ta);
+        tma_prefetch_desc(&tb);
+    }
+    if (warp == 1) {
+        tmem_alloc(smem_addr(&sh->tmem_base), kTmemCols);
+        tmem_relinquish();
+    }
+    tc_fence_before();
+    __syncthreads();
+    tc_fence_after();
+    const uint32_t tmem = sh->tmem_base;
+    const int items = p.G;
+
+    if (warp == 0) {
+        // ------------------------------------------------ TMA producer
+        if (lane == 0) {
+            const uint32_t bb = smem_addr(&sh->bfull);
+            mbar_arrive_expect_tx(bb, (uint32_t)(KS * bslice));
+            for (int ks = 0; ks < KS; ++ks)
+                tma_load_2d(smem_addr(sB + ks * bslice), &tb, bb, ks * kElemsPerSlice, 0);
+            int s = 0;
+            uint32_t ph = 0;
+            int64_t issued = 0;
+            bool ok = true;
+            for (int v = blockIdx.x; v < items && ok; v += gridDim.x) {
+                const int64_t t0 = (int64_t)v * p.tiles / p.G, t1 = (int64_t)(v + 1) * p.tiles / p.G;
+                for (int64_t t = t0; t < t1 && ok; ++t)
+                    for (int ks = 0; ks < KS; ++ks) {
+                        if (!mbar_wait(smem_addr(&sh->empty[s]), ph ^ 1u, p.timeout_ns)) {
+                            ok = false;
+                            break;
+                        }
+                        const uint32_t fb = smem_addr(&sh->full[s]);
+                        mbar_arrive_expect_tx(fb, kAStage);
+                        tma_load_2d(smem_addr(sA + s * kAStage), &ta, fb, ks * kElemsPerSlice, (int)(t * kRows));
+                        ++issued;
+                        if (++s == S) {
+                            s = 0;
+                            ph ^= 1u;
+                        }
+                    }
+            }
+            if (!ok) atomicOr(p.err, kErrTimeout);
+            for (int st = 0; st < S; ++st) {
+                const int64_t uses = issued / S + (st < issued % S ? 1 : 0);
+                if (uses && !mbar_wait(smem_addr(&sh->full[st]), (uint32_t)((uses - 1) & 1), kDrainTimeoutNs))
+                    atomicOr(p.err, kErrTimeout);
+            }
+            if (!mbar_wait(bb, 0, kDrainTimeoutNs)) atomicOr(p.err, kErrTimeout);
+        }
+    } else if (warp == 1) {
+        // ------------------------------------------------ MMA issuer
+        if (lane == 0) {
+            int s = 0;
+            uint32_t ph = 0, lt = 0;
+            bool ok = mbar_wait(smem_addr(&sh->bfull), 0, p.timeout_ns);
+            for (int v = blockIdx.x; v < items && ok; v += gridDim.x) {
+                const int64_t t0 = (int64_t)v * p.tiles / p.G, t1 = (int64_t)(v + 1) * p.tiles / p.G;
+                for (int64_t t = t0; t < t1 && ok; ++t, ++lt) {
+                    const uint32_t buf = lt & 1u, use = lt >> 1;
+                    if (!mbar_wait(smem_addr(&sh->tempty[buf]), (use & 1u) ^ 1u, p.timeout_ns)) {
+                        ok = false;
+                        break;
+                    }
+                    tc_fence_after();
+                    const uint32_t dt = tmem + buf * 128;
+                    for (int ks = 0; ks < KS; ++ks) {
+                        if (!mbar_wait(smem_addr(&sh->full[s]), ph, p.timeout_ns)) {
+                            ok = false;
+                            break;
+                        }
+                        tc_fence_after();
+                        const uint64_t ad = smem_desc_k128(smem_addr(sA + s * kAStage));
+                        const uint64_t bd = smem_desc_k128(smem_addr(sB + ks * bslice));
+#pragma unroll
+                        for (int kk = 0; kk < 4; ++kk) {
+                            if constexpr (FP8)
+                                tc_mma_f8(dt, ad + (uint64_t)(kk * 2), bd + (uint64_t)(kk * 2), idesc, (ks | kk) != 0);
+                            else
+                                tc_mma_f16(dt, ad + (uint64_t)(kk * 2), bd + (uint64_t)(kk * 2), idesc, (ks | kk) != 0);
+                        }
+                        tc_commit(smem_addr(&sh->empty[s]));
+                        if (++s == S) {
+                            s = 0;
+                            ph ^= 1u;
+                        }
+                    }
+                    if (!ok) break;
+                    tc_commit(smem_addr(&sh->tfull[buf]));
+                }
+            }
+            if (!ok) atomicOr(p.err, kErrTimeout);
+            tc_commit(smem_addr(&sh->drain));
+            if (!mbar_wait(smem_addr(&sh->drain), 0, kDrainTimeoutNs)) atomicOr(p.err, kErrTimeout);
+        }
+    } else {
+        // ------------------------------------------------ epilogue (warps 2..5)
+        const int sub = warp & 3;
+        const uint32_t lane_addr = (uint32_t)(sub * 32) << 16;
+        const float kNegInf = -__int_as_float(0x7f800000);
+        const int R = p.R, k = p.k;
+        uint64_t *Lw = slists + (size_t)sub * R * k;  // this warp's set of query q at Lw + q * k
+        uint32_t lt = 0, chunk = 0;
+        bool ok = true;
+        for (int v = blockIdx.x; v < items && ok; v += gridDim.x) {
+            const int64_t t0 = (int64_t)v * p.tiles / p.G, t1 = (int64_t)(v + 1) * p.tiles / p.G;
+            // Lane q keeps query q's set for this warp's rows of the chunk; its
+            // two thresholds are mirrored in shared memory for the other lanes.
+            RowTopK top;
+            float thr = kNegInf, gthr = kNegInf;
+            uint32_t published = 0;
+            float *thr_w = sh->thr[sub], *gthr_w = sh->gthr[sub];
+            float *Sw = strans + sub * 32 * 33;  // [32 rows][33]: one row's scores per lane
+            thr_w[lane] = kNegInf;
+            gthr_w[lane] = kNegInf;
+            // The shared threshold is read one tile ahead, off the critical path.
+            uint32_t tau_next = lane < R ? *reinterpret_cast<volatile uint32_t *>(p.tau + lane) : 0u;
+            __syncwarp();
+            for (int64_t t = t0; t < t1; ++t, ++lt) {
+                const uint32_t buf = lt & 1u, use = lt >> 1;
+                if (!mbar_wait(smem_addr(&sh->tfull[buf]), use & 1u, p.timeout_ns)) {
+                    ok = false;
+                    break;
+                }
+                tc_fence_after();
+                if (lane < R) {
+                    const uint32_t mine = top.n == k ? ord_of_score(thr) : 0u;
+                    if (mine > published) {
+                        atomicMax(p.tau + lane, mine);
+                        published = mine;
+                    }
+                    if (tau_next > published) gthr = score_of_ord(tau_next);
+                    tau_next = *reinterpret_cast<volatile uint32_t *>(p.tau + lane);
+                    gthr_w[lane] = gthr;
+                }
+                const int64_t rowbase = t * kRows + sub * 32;
+                const int64_t i = rowbase + lane;
+                const bool valid = i < p.N;
+                uint32_t d0[32], d1[32], d2[32];
+                const uint32_t taddr = tmem + lane_addr + buf * 128;
+                tmem_ld_32x32b_x32(taddr, d0);
+                if constexpr (FP8) {
+                    tmem_ld_32x32b_x32(taddr + 32, d1);
+                    tmem_ld_32x32b_x32(taddr + 64, d2);
+                }
+                tmem_ld_wait(d0);
+                if constexpr (FP8) {
+                    regs_after_wait(d1);
+                    regs_after_wait(d2);
+                }
+                tc_fence_before();
+                __syncwarp();
+                if (lane == 0) mbar_arrive(smem_addr(&sh->tempty[buf]));
+                const float cs = FP8 ? (valid ? __ldg(p.corpus_scale + i) : 0.0f) : 1.0f;
+                // All queries' scores of this lane's row, and one ballot per
+                // query against that query's thresholds (branch-free).
+                float sc[kLatMaxR];
+                uint32_t m[kLatMaxR];
+                uint32_t anym = 0;
+#pragma unroll
+                for (int q = 0; q < kLatMaxR; ++q) {
+                    float sq;
+                    if constexpr (FP8)
+                        sq = (sh->qscale[0][q] * __uint_as_float(d0[q]) + sh->qscale[1][q] * __uint_as_float(d1[q]) +
+                              sh->qscale[2][q] * __uint_as_float(d2[q])) * cs;
+                    else
+                        sq = __uint_as_float(d0[q]);
+                    sc[q] = sq;
+                    m[q] = __ballot_sync(0xffffffffu, valid && q < R && sq > thr_w[q] && sq >= gthr_w[q]);
+                    anym |= m[q];
+                }
+                if (anym) {
+                    // Survivors: transpose the warp's 32 x 32 scores through
+                    // shared memory, then lane q inserts query q's survivors
+                    // in increasing row (= id) order, all queries in parallel.
+#pragma unroll
+                    for (int q = 0; q < kLatMaxR; ++q) Sw[lane * 33 + q] = sc[q];
+                    __syncwarp();
+                    uint32_t mine_m = select32(m, lane);
+                    if (lane < R) {
+                        while (mine_m) {
+                            const int l = __ffs(mine_m) - 1;
+                            mine_m &= mine_m - 1;
+                            const float sl = Sw[l * 33 + lane];
+                            if (sl > thr && sl >= gthr) {
+                                topk_add(Lw + (size_t)lane * k, 1, k, top, make_key(sl, (uint32_t)(rowbase + l)));
+                                if (top.n == k) thr = key_score(top.min_key);
+                            }
+                        }
+                        thr_w[lane] = thr;
+                    }
+                    __syncwarp();
+                }
+            }
+            // Chunk done: sort each set, then merge the four warps' sets of
+            // every query into the chunk's list (the two hand-offs between
+            // the epilogue warps are bounded waits, like every other wait).
+            if (lane < R) {
+                topk_sort(Lw + (size_t)lane * k, 1, top.n);
+                for (int t = top.n; t < k; ++t) Lw[(size_t)lane * k + t] = 0ull;
+            }
+            const uint32_t par = (uint32_t)(chunk & 1);
+            mbar_arrive(smem_addr(&sh->sorted));
+            if (!mbar_wait(smem_addr(&sh->sorted), par, p.timeout_ns)) ok = false;
+            for (int q = sub; q < R && ok; q += 4) {
+                uint64_t *out = p.lists + ((int64_t)v * R + q) * k;
+                warp_merge_topk<1>(slists + (size_t)q * k, (int64_t)R * k, 4, k, k,
+                                   [&](int idx, uint64_t key) { out[idx] = key; });
+            }
+            mbar_arrive(smem_addr(&sh->merged));
+            if (!mbar_wait(smem_addr(&sh->merged), par, p.timeout_ns)) ok = false;
+            ++chunk;
+        }
+        if (!ok && lane == 0) atomicOr(p.err, kErrTimeout);
+    }
+
+    tc_fence_before();
+    __syncthreads();
+    tc_fence_after();
+    if (warp == 1) {
+        __syncwarp();
+        tmem_dealloc(tmem, kTmemCols);
+    }
+}
+
+// Splits each bf16 query row into three e4m3 parts with power-of-two scales
+// (rows r, 32 + r, 64 + r of the 96-row operand; the other rows stay zero).
+// One block per query row.
+__global__ void __launch_bounds__(256) k_split_queries(const uint16_t *__restrict__ regions, int R, int d,
+                                                       uint8_t *__restrict__ parts, float *__restrict__ qscale) {
+    __shared__ float red[8];
+    const int r = blockIdx.x;
+    const uint16_t *q = regions + (size_t)r * d;
+    auto block_max = [&](float v) {
+        for (int o = 16; o; o >>= 1) v = fmaxf(v, __shfl_xor_sync(0xffffffffu, v, o));
+        if ((threadIdx.x & 31) == 0) red[threadIdx.x >> 5] = v;
+        __syncthreads();
+        float m = 0.0f;
+        for (int w = 0; w < (int)(blockDim.x >> 5); ++w) m = fmaxf(m, red[w]);
+        __syncthreads();
+        return m;
+    };
+    auto pow2_scale = [](float m) {
+        if (!(m > 0.0f)) return 1.0f;
+        int e;
+        frexpf(m / 448.0f, &e);  // m / 448 = f 2^e, 0.5 <= f < 1
+        return ldexpf(1.0f, e);  // >= m / 448, so |x| / scale <= 448
+    };
+    // Each thread handles elements j = threadIdx.x + 256 t of the row.
+    float m0 = 0.0f;
+    for (int j = threadIdx.x; j < d; j += blockDim.x)
+        m0 = fmaxf(m0, fabsf(__uint_as_float((uint32_t)q[j] << 16)));
+    float res_scale[3];
+    res_scale[0] = pow2_scale(block_max(m0));
+    // Three passes over the row; the residual is recomputed from the parts
+    // already written so that no per-element state has to be kept.
+    for (int part = 0; part < 3; ++part) {
+        const float sc = res_scale[part];
+        float mnext = 0.0f;
+        for (int j = threadIdx.x; j < d; j += blockDim.x) {
+            float x = __uint_as_float((uint32_t)q[j] << 16);
+            for (int pp = 0; pp < part; ++pp) {
+                const __half_raw h = __nv_cvt_fp8_to_halfraw(parts[(size_t)(pp * 32 + r) * d + j], __NV_E4M3);
+                x -= __half2float(__half(h)) * res_scale[pp];
+            }
+            const __nv_fp8_storage_t e = __nv_cvt_float_to_fp8(x / sc, __NV_SATFINITE, __NV_E4M3);
+            parts[(size_t)(part * 32 + r) * d + j] = e;
+            const __half_raw h = __nv_cvt_fp8_to_halfraw(e, __NV_E4M3);
+            mnext = fmaxf(mnext, fabsf(x - __half2float(__half(h)) * sc));
+        }
+        if (part < 2) res_scale[part + 1] = pow2_scale(block_max(mnext));
+        __syncthreads();
+    }
+    if (threadIdx.x < 3) qscale[threadIdx.x * R + r] = res_scale[threadIdx.x];
+}
+
+size_t smem_bytes(int Npad, int slices, int stages, int R, int k) {
+    return 1024 + (size_t)slices * Npad * kSlice + (size_t)stages * kAStage + (size_t)4 * R * k * 8 +
+           (size_t)4 * 32 * 33 * 4 + sizeof(LatShared);
+}
+
+}  // namespace
+
+bool lat_pick_layout(bool fp8, int R, int d, int k, int max_smem, int *Npad, int *slices, int *stages) {
+    if (R < 1 || R > kLatMaxR) return false;
+    *Npad = fp8 ? 96 : (R + 15) / 16 * 16;
+    *slices = fp8 ? (d + 127) / 128 : (d + 63) / 64;
+    for (int st = kMaxStages; st >= 3; --st)
+        if (smem_bytes(*Npad, *slices, st, R, k) <= (size_t)max_smem) {
+            *stages = st;
+            return true;
+        }
+    return false;
+}
+
+cudaError_t launch_split_queries(const uint16_t *regions, int R, int d, uint8_t *parts, float *qscale,
+                                 cudaStream_t s) {
+    k_split_queries<<<R, 256, 0, s>>>(regions, R, d, parts, qscale);
+    return cudaGetLastError();
+}
+
+cudaError_t launch_latency(bool fp8, const CUtensorMap &ta, const CUtensorMap &tb, const LatParams &p, int grid,
+                           cudaStream_t s) {
+    const size_t smem = smem_bytes(p.Npad, p.slices, p.stages, p.R, p.k);
+    auto kern = fp8 ? k_latency_score_topk<true> : k_latency_score_topk<false>;
+    cudaError_t e = cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
+    if (e != cudaSuccess) return e;
+    kern<<<grid, kThreads, smem, s>>>(ta, tb, p);
+    return cudaGetLastError();
+}
+
+}  // namespace skipk

@@ -279,6 +279,8 @@ __global__ void __launch_bounds__(kTcThreads, 1)
             float gthr = kNegInf;  // best k-th score any chunk of this row has found
             uint32_t published = 0;
             uint32_t *tau = p.tau + row;
+            // The shared threshold is read one tile ahead, off the critical path.
+            uint32_t tau_next = row_valid ? *reinterpret_cast<volatile uint32_t *>(tau) : 0u;
             // Common case: no score of the 32 beats the threshold (a max and
             // a compare).  Otherwise a branch-free bit mask of the survivors
             // is walked in increasing column (= id) order, so that lanes
@@ -317,8 +319,8 @@ __global__ void __launch_bounds__(kTcThreads, 1)
                         atomicMax(tau, mine);
                         published = mine;
                     }
-                    const uint32_t best = *reinterpret_cast<volatile uint32_t *>(tau);
-                    if (best > published) gthr = score_of_ord(best);
+                    if (tau_next > published) gthr = score_of_ord(tau_next);
+                    tau_next = *reinterpret_cast<volatile uint32_t *>(tau);
                 }
                 const int64_t n0 = t * kTcTileN;
                 const bool tail = n0 + kTcTileN > p.N;

@@ -346,6 +346,8 @@ __global__ void __launch_bounds__(kThreads, 1)
             float thr = kNegInf, gthr = kNegInf;
             uint32_t published = 0;
             uint32_t *tau = p.tau + row;
+            // The shared threshold is read one tile ahead, off the critical path.
+            uint32_t tau_next = row_valid ? *reinterpret_cast<volatile uint32_t *>(tau) : 0u;
             auto scan32 = [&](uint32_t (&vv)[32], uint32_t id0) {
                 if (!row_valid) return;
                 const float mx = fmax32(vv);
@@ -379,8 +381,8 @@ __global__ void __launch_bounds__(kThreads, 1)
                         atomicMax(tau, mine);
                         published = mine;
                     }
-                    const uint32_t best = *reinterpret_cast<volatile uint32_t *>(tau);
-                    if (best > published) gthr = score_of_ord(best);
+                    if (tau_next > published) gthr = score_of_ord(tau_next);
+                    tau_next = *reinterpret_cast<volatile uint32_t *>(tau);
                 }
                 const int64_t n0 = t * kTcTileN;
 #pragma unroll 1

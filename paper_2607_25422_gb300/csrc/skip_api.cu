@@ -58,12 +58,12 @@ bool encode_bf16_rows(CUtensorMap *map, const void *base, int64_t rows, int d, i
 
 // 2D byte tensor map over the e4m3 corpus [rows x d], box 256 rows x 128
 // elements (128 bytes), 128-byte swizzle, zero fill out of bounds.
-bool encode_e4m3_rows(CUtensorMap *map, const void *base, int64_t rows, int d) {
+bool encode_e4m3_rows(CUtensorMap *map, const void *base, int64_t rows, int d, int box_rows = kTcTileN) {
     EncodeTiledFn fn = encode_fn();
     if (!fn) return false;
     cuuint64_t dims[2] = {(cuuint64_t)d, (cuuint64_t)rows};
     cuuint64_t strides[1] = {(cuuint64_t)d};
-    cuuint32_t box[2] = {128, (cuuint32_t)kTcTileN};
+    cuuint32_t box[2] = {128, (cuuint32_t)box_rows};
     cuuint32_t estr[2] = {1, 1};
     return fn(map, CU_TENSOR_MAP_DATA_TYPE_UINT8, 2, const_cast<void *>(base), dims, strides, box, estr,
               CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B, CU_TENSOR_MAP_L2_PROMOTION_L2_256B,
@@ -160,6 +160,7 @@ struct Plan {
     bool list_in_smem = false;
     int CL = 1;
     bool pair = false;
+    bool latency = false;
 };
 
 // Corpus chunks G for the tensor path: make MB * G a whole number of waves of
@@ -206,6 +207,72 @@ skip_status_t run_regions(skip_corpus *c, const uint16_t *regions, int R, int k,
     else
         tensor = e4m3 ? R > 4 : R > 8;
     if (!e4m3 && !c->tmap_ok) tensor = false;
+    // Small batches: corpus tile as the streamed MMA operand, queries resident.
+    int lat_npad = 0, lat_slices = 0, lat_stages = 0;
+    const bool lat_fits = R <= kLatMaxR && lat_pick_layout(e4m3, R, c->d, k, c->max_smem, &lat_npad, &lat_slices,
+                                                            &lat_stages);
+    if (lat_fits && (c->path == SKIP_PATH_LATENCY || (c->path == SKIP_PATH_AUTO && tensor))) {
+        pl.tensor = true;
+        pl.latency = true;
+        pl.tiles = (c->N + 127) / 128;
+        pl.G = pick_chunks(1, pl.tiles, ctas);
+        pl.grid = std::min(pl.G, ctas);
+        pl.R_pad = R;
+        pl.stages = lat_stages;
+        pl.list_in_smem = true;
+        const size_t tau_bytes = align_up((size_t)R * sizeof(uint32_t), 256);
+        const size_t parts_bytes = e4m3 ? align_up((size_t)96 * c->d, 256) : 0;
+        const size_t qs_bytes = e4m3 ? align_up((size_t)3 * R * sizeof(float), 256) : 0;
+        const size_t lists_bytes = (size_t)pl.G * R * k * sizeof(uint64_t);
+        skip_status_t st =
+            ensure_ws(c, align_up(ws_extra, 256) + tau_bytes + parts_bytes + qs_bytes + lists_bytes);
+        if (st) return st;
+        char *w = (char *)c->ws + align_up(ws_extra, 256);
+        uint32_t *tau = reinterpret_cast<uint32_t *>(w);
+        uint8_t *parts = reinterpret_cast<uint8_t *>(w + tau_bytes);
+        float *qscale = reinterpret_cast<float *>(w + tau_bytes + parts_bytes);
+        uint64_t *lists = reinterpret_cast<uint64_t *>(w + tau_bytes + parts_bytes + qs_bytes);
+        if (keys_out) *keys_out = reg_keys = reinterpret_cast<uint64_t *>(c->ws);
+        if (cudaMemsetAsync(tau, 0, tau_bytes, s) != cudaSuccess) return SKIP_ECUDA;
+        CUtensorMap ta, tb;
+        if (e4m3) {
+            if (cudaMemsetAsync(parts, 0, parts_bytes, s) != cudaSuccess) return SKIP_ECUDA;
+            record(c, s, "split_queries");
+            cudaError_t e = launch_split_queries(regions, R, c->d, parts, qscale, s);
+            if (e != cudaSuccess) return cuda_status(e);
+            ++pl.launches;
+            if (!encode_e4m3_rows(&ta, c->rows, c->N, c->d, 128) || !encode_e4m3_rows(&tb, parts, 96, c->d, 96))
+                return SKIP_ECUDA;
+        } else {
+            if (!encode_bf16_rows(&ta, c->rows, c->N, c->d, 128) || !encode_bf16_rows(&tb, regions, R, c->d, lat_npad))
+                return SKIP_ECUDA;
+        }
+        LatParams p;
+        p.N = c->N;
+        p.d = c->d;
+        p.R = R;
+        p.k = k;
+        p.Npad = lat_npad;
+        p.slices = lat_slices;
+        p.stages = lat_stages;
+        p.tiles = pl.tiles;
+        p.G = pl.G;
+        p.corpus_scale = c->scale;
+        p.qscale = qscale;
+        p.lists = lists;
+        p.tau = tau;
+        p.err = c->err;
+        p.timeout_ns = c->timeout_ns;
+        record(c, s, e4m3 ? "score_topk_latency_e4m3" : "score_topk_latency");
+        cudaError_t e = launch_latency(e4m3, ta, tb, p, pl.grid, s);
+        if (e != cudaSuccess) return cuda_status(e);
+        ++pl.launches;
+        record(c, s, "merge_lists");
+        e = launch_merge_lists(lists, pl.G, (int64_t)R * k, R, k, reg_keys, reg_ids, reg_scores, s);
+        if (e != cudaSuccess) return cuda_status(e);
+        ++pl.launches;
+        return SKIP_OK;
+    }
     pl.tensor = tensor;
     if (tensor && e4m3) {
         // e4m3 corpus: single-CTA MMA on bf16-widened corpus tiles.
@@ -400,7 +467,8 @@ void write_plan(skip_corpus *c, const Plan &pl, int R, int Q, int k, int K) {
              "{\"path\": \"%s\", \"grid\": %d, \"lists_per_row\": %d, \"query_blocks\": %d, "
              "\"R_total\": %d, \"Q\": %d, \"k_region\": %d, \"K\": %d, \"launches\": %d, "
              "\"stages\": %d, \"cluster\": %d, \"mma\": \"%s\", \"lists\": \"%s\"}",
-             pl.tensor ? "tensor" : "warpdot", pl.grid, pl.G, pl.MB, R, Q, k, K, pl.launches, pl.stages, pl.CL,
+             pl.latency ? "latency" : pl.tensor ? "tensor" : "warpdot", pl.grid, pl.G, pl.MB, R, Q, k, K, pl.launches,
+             pl.stages, pl.CL,
              pl.pair ? "pair" : "single",
              pl.tensor ? (pl.list_in_smem ? "shared" : "global") : "global");
 }
@@ -490,7 +558,7 @@ skip_status_t skip_corpus_set_option(skip_corpus_t c, int option, int64_t value)
     if (!c) return SKIP_EINVAL;
     switch (option) {
         case SKIP_OPT_PATH:
-            if (value < SKIP_PATH_AUTO || value > SKIP_PATH_WARP) return SKIP_EINVAL;
+            if (value < SKIP_PATH_AUTO || value > SKIP_PATH_LATENCY) return SKIP_EINVAL;
             c->path = (int)value;
             return SKIP_OK;
         case SKIP_OPT_WAIT_TIMEOUT_NS:

@@ -376,6 +376,27 @@ __device__ __forceinline__ uint64_t smem_desc_k128(uint32_t saddr) {
     return d;
 }
 
+// Instruction descriptor for kind::f8f6f4: e4m3 A and B, fp32 D, both
+// K-major, dense, tile M x N (K = 32 per instruction).
+__host__ __device__ constexpr uint32_t idesc_e4m3_f32(int M, int N) {
+    return (1u << 4)                       // D format: f32
+           | (0u << 7)                     // A format: e4m3
+           | (0u << 10)                    // B format: e4m3
+           | ((uint32_t)(N >> 3) << 17)    // N / 8
+           | ((uint32_t)(M >> 4) << 24);   // M / 16
+}
+
+// D[tmem] (+)= A[smem] * B[smem]^T, e4m3 inputs, fp32 accumulate.
+__device__ __forceinline__ void tc_mma_f8(uint32_t d_tmem, uint64_t adesc, uint64_t bdesc, uint32_t idesc,
+                                          uint32_t accumulate) {
+    asm volatile(
+        "{\n\t.reg .pred p;\n\t"
+        "setp.ne.b32 p, %4, 0;\n\t"
+        "tcgen05.mma.cta_group::1.kind::f8f6f4 [%0], %1, %2, %3, p;\n\t}" ::"r"(d_tmem),
+        "l"(adesc), "l"(bdesc), "r"(idesc), "r"(accumulate)
+        : "memory");
+}
+
 // Instruction descriptor for kind::f16: bf16 A and B, fp32 D, both K-major,
 // dense, tile M x N.
 __host__ __device__ constexpr uint32_t idesc_bf16_f32(int M, int N) {

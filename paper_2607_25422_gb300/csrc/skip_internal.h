@@ -67,6 +67,32 @@ void tc_fp8_pick_layout(int k, int max_smem, int *stages, int *raw_stages, bool 
 cudaError_t launch_tc_fp8(const CUtensorMap &tq, const CUtensorMap &traw, const TcParams &p, int grid,
                           cudaStream_t s);
 
+// ---- small batches on the tensor cores (corpus tile = A, queries = B) ----
+constexpr int kLatMaxR = 32;
+struct LatParams {
+    int64_t N;
+    int d;
+    int R;                    // region rows (<= kLatMaxR)
+    int k;
+    int Npad;                 // MMA N: 96 (e4m3, three query parts) or R rounded up to 16
+    int slices;               // 128-byte K slices per row
+    int stages;               // corpus ring depth
+    int64_t tiles;            // 128-row corpus tiles
+    int G;                    // corpus chunks (lists per query)
+    const float *corpus_scale;  // [N] (e4m3)
+    const float *qscale;        // [3][R] scales of the query parts (e4m3)
+    uint64_t *lists;          // [G][R][k]
+    uint32_t *tau;            // [R] shared thresholds, zeroed
+    int *err;
+    uint64_t timeout_ns;
+};
+bool lat_pick_layout(bool fp8, int R, int d, int k, int max_smem, int *Npad, int *slices, int *stages);
+// e4m3 query parts: parts [96 x d] bytes (zeroed by the caller), qscale [3][R].
+cudaError_t launch_split_queries(const uint16_t *regions, int R, int d, uint8_t *parts, float *qscale,
+                                 cudaStream_t s);
+cudaError_t launch_latency(bool fp8, const CUtensorMap &ta, const CUtensorMap &tb, const LatParams &p, int grid,
+                           cudaStream_t s);
+
 // ---- merges -------------------------------------------------------------
 // Per-region merge of G sorted lists into the exact top-k (keys and/or
 // decoded ids/scores).

@@ -227,6 +227,39 @@ def test_e4m3_tensor_path(case):
     assert_parity(cn, rn, offsets, k, K, gpu, truth, scale_np=sn)
 
 
+LATENCY_CASES = [
+    # dtype, N, d, R, Q, k, K
+    ("bf16", 10000, 64, 1, 1, 5, 5),
+    ("bf16", 30001, 768, 32, 4, 10, 20),
+    ("bf16", 5000, 256, 7, 3, 50, 60),
+    ("bf16", 2000, 128, 20, 5, 64, 80),
+    ("e4m3", 6000, 1024, 32, 1, 10, 100),
+    ("e4m3", 7001, 80, 5, 2, 7, 20),
+    ("e4m3", 20000, 512, 17, 3, 30, 40),
+]
+
+
+@pytest.mark.parametrize("case", LATENCY_CASES, ids=lambda c: "%s_N%d_d%d_R%d_k%d" % (c[0], c[1], c[2], c[3], c[5]))
+def test_small_batch_tensor_path(case):
+    """Small region batches with the corpus tile as the streamed MMA operand
+    (bf16, or e4m3 with the queries split into three e4m3 parts)."""
+    dt, N, d, R, Q, k, K = case
+    if dt == "bf16":
+        corpus, scale = synth.random_bf16(N, d, seed=N + 1), None
+        cn, sn = _bits(corpus), None
+    else:
+        spec = synth.WorkloadSpec("lat_e4m3", 80 + R, N, d, "e4m3", Q, (1, 1), k, K, "gaussian")
+        corpus, scale, _ = synth.make_corpus(spec)
+        cn, sn = corpus.numpy(), scale.numpy()
+    rt = synth.random_bf16(R, d, seed=R + 13)
+    offsets = ragged_offsets(Q, R, seed=N + R)
+    rn = _bits(rt)
+    truth = oracle_truth(cn, rn, offsets, k, K, scale_np=sn)
+    gpu = run_gpu(corpus, rt, offsets, k, K, skip.SKIP_PATH_LATENCY, scale=scale)
+    assert gpu[4]["path"] == "latency"
+    assert_parity(cn, rn, offsets, k, K, gpu, truth, scale_np=sn)
+
+
 def test_host_entry_point_matches_device():
     ct = synth.random_bf16(9000, 256, seed=8)
     rt = synth.random_bf16(40, 256, seed=9)
