@@ -267,6 +267,8 @@ def main():
     ap.add_argument("--cpu-questions", type=int, default=8, help="questions in the oracle sample")
     ap.add_argument("--no-cpu-baseline", action="store_true")
     ap.add_argument("--path", default="auto", choices=["auto", "tensor", "warp", "latency"])
+    ap.add_argument("--rows", type=int, default=0,
+                    help="use only the first ROWS corpus rows (smaller profiling captures; not a bench line)")
     ap.add_argument("--cluster", type=int, default=0, choices=[0, 1, 2, 4, 8],
                     help="single-CTA tensor path CTAs per cluster (0 = library's choice)")
     ap.add_argument("--mma", default="auto", choices=["auto", "single", "pair"],
@@ -275,6 +277,9 @@ def main():
     if args.warmup < 3:
         raise SystemExit("at least 3 warm-up steps")
     spec = synth.WORKLOADS[args.workload]
+    if args.rows:
+        import dataclasses
+        spec = dataclasses.replace(spec, N=min(spec.N, args.rows), name="%s_rows%d" % (spec.name, args.rows))
     if args.impl == "reference":
         run_reference(args, spec)
         return
