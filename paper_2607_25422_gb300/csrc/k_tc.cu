@@ -285,23 +285,26 @@ __global__ void __launch_bounds__(kTcThreads, 1)
             // a compare).  Otherwise a branch-free bit mask of the survivors
             // is walked in increasing column (= id) order, so that lanes
             // without survivors idle for a few instructions only.
+            // One compare per score: s > thr and s >= gthr is s > cthr
+            // (padding columns hold -inf and never pass).
+            float gbelow = kNegInf, cthr = kNegInf;
             auto scan32 = [&](uint32_t (&vv)[32], uint32_t id0) {
                 if (!row_valid) return;
                 const float mx = fmax32(vv);
-                if (!(mx > thr && mx >= gthr)) return;
+                if (!(mx > cthr)) return;
                 uint32_t m = 0;
 #pragma unroll
-                for (int j = 0; j < 32; ++j) {
-                    const float sj = __uint_as_float(vv[j]);
-                    m |= (sj > thr && sj >= gthr ? 1u : 0u) << j;
-                }
+                for (int j = 0; j < 32; ++j) m |= (__uint_as_float(vv[j]) > cthr ? 1u : 0u) << j;
                 while (m) {
                     const int j = __ffs(m) - 1;
                     m &= m - 1;
                     const float sj = __uint_as_float(select32(vv, j));
                     if (sj > thr) {
                         topk_add(L, ls, p.k, top, make_key(sj, id0 + j));
-                        if (top.n == p.k) thr = key_score(top.min_key);
+                        if (top.n == p.k) {
+                            thr = key_score(top.min_key);
+                            cthr = fmaxf(thr, gbelow);
+                        }
                     }
                 }
             };
@@ -319,7 +322,11 @@ __global__ void __launch_bounds__(kTcThreads, 1)
                         atomicMax(tau, mine);
                         published = mine;
                     }
-                    if (tau_next > published) gthr = score_of_ord(tau_next);
+                    if (tau_next > published) {
+                        gthr = score_of_ord(tau_next);
+                        gbelow = float_below(gthr);
+                        cthr = fmaxf(thr, gbelow);
+                    }
                     tau_next = *reinterpret_cast<volatile uint32_t *>(tau);
                 }
                 const int64_t n0 = t * kTcTileN;

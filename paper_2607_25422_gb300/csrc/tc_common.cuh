@@ -36,18 +36,29 @@ struct RowTopK {
 };
 
 __device__ __forceinline__ void topk_rescan(uint64_t *L, int ls, int k, RowTopK &st) {
-    uint64_t mk = ~0ull;
-    int ms = 0;
-#pragma unroll 4
-    for (int t = 0; t < k; ++t) {
-        const uint64_t x = L[t * ls];
-        if (x < mk) {
-            mk = x;
-            ms = t;
-        }
+    // Four independent running minima, combined at the end: the compare
+    // chain is k/4 deep instead of k.  Keys are distinct, so the slot found
+    // does not depend on the order of the compares.
+    uint64_t m0 = ~0ull, m1 = ~0ull, m2 = ~0ull, m3 = ~0ull;
+    int s0 = 0, s1 = 0, s2 = 0, s3 = 0;
+    int t = 0;
+#pragma unroll 2
+    for (; t + 4 <= k; t += 4) {
+        const uint64_t x0 = L[t * ls], x1 = L[(t + 1) * ls], x2 = L[(t + 2) * ls], x3 = L[(t + 3) * ls];
+        if (x0 < m0) { m0 = x0; s0 = t; }
+        if (x1 < m1) { m1 = x1; s1 = t + 1; }
+        if (x2 < m2) { m2 = x2; s2 = t + 2; }
+        if (x3 < m3) { m3 = x3; s3 = t + 3; }
     }
-    st.min_key = mk;
-    st.min_slot = ms;
+    for (; t < k; ++t) {
+        const uint64_t x = L[t * ls];
+        if (x < m0) { m0 = x; s0 = t; }
+    }
+    if (m1 < m0) { m0 = m1; s0 = s1; }
+    if (m3 < m2) { m2 = m3; s2 = s3; }
+    if (m2 < m0) { m0 = m2; s0 = s2; }
+    st.min_key = m0;
+    st.min_slot = s0;
 }
 
 // The caller has checked that key beats the smallest key (or n < k).
@@ -72,6 +83,14 @@ __device__ __forceinline__ void topk_sort(uint64_t *L, int ls, int n) {
         }
         L[(j + 1) * ls] = x;
     }
+}
+
+// The largest float below x (x itself for -inf): "s > below(x)" is "s >= x".
+__device__ __forceinline__ float float_below(float x) {
+    const uint32_t b = __float_as_uint(x);
+    if (b == 0xFF800000u) return x;
+    if ((b & 0x7FFFFFFFu) == 0u) return __uint_as_float(0x80000001u);
+    return __uint_as_float((b & 0x80000000u) ? b + 1u : b - 1u);
 }
 
 // v[j] for a run-time j without indexing the register array (5 levels of

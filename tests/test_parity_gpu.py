@@ -24,13 +24,15 @@ def _bits(t):
     return synth.bf16_bits(t)
 
 
-def run_gpu(corpus, regions, offsets, k, K, path, scale=None, cluster=0, mma=0):
+def run_gpu(corpus, regions, offsets, k, K, path, scale=None, cluster=0, mma=0, options=()):
     dev = torch.device("cuda")
     c = skip.skip_corpus_load(corpus.to(dev), row_scale=None if scale is None else scale.to(dev))
     try:
         c.set_option(skip.SKIP_OPT_PATH, path)
         c.set_option(skip.SKIP_OPT_CLUSTER, cluster)
         c.set_option(skip.SKIP_OPT_MMA, mma)
+        for opt, val in options:
+            c.set_option(opt, val)
         reg = regions.to(dev)
         rid, rsc = skip.skip_retrieve_regions(c, reg, k)
         oid, osc = skip.skip_retrieve(c, reg, torch.as_tensor(offsets).to(dev), k, K)
