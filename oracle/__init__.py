@@ -15,6 +15,11 @@ Functions and what they follow:
 * ``retrieve``     -- both steps (the CPU baseline).
 * ``score_matrix`` -- every s(r, i) in fp64 (brute force on tiny inputs).
 * ``scores_at``    -- s(r, i) at chosen (region, id) pairs.
+* ``skv``          -- App. B.4 Def. B.4 (Eq. skv_score) and the Alg. 1 TopK
+  after it: the passage gate nu_j = sigmoid(h_psi(features)), kept when
+  nu_j >= tau, the best ceil(rho |K|) by (nu desc, id asc)
+  (``skv_oracle.c``).
+* ``bf16_round``   -- a double rounded to bf16 (ties to even), as bits.
 """
 from __future__ import annotations
 
@@ -25,19 +30,20 @@ import subprocess
 import numpy as np
 
 _HERE = os.path.dirname(os.path.abspath(__file__))
-_SRC = os.path.join(_HERE, "rcsr_oracle.c")
+_SRCS = [os.path.join(_HERE, "rcsr_oracle.c"), os.path.join(_HERE, "skv_oracle.c")]
 _OUT = os.path.join(_HERE, "_build", "libskip_oracle.so")
 _lib = None
 
 
 def build(force: bool = False) -> str:
     """Compile the oracle with gcc (OpenMP) into oracle/_build/."""
-    if not force and os.path.exists(_OUT) and os.path.getmtime(_OUT) >= os.path.getmtime(_SRC):
+    if not force and os.path.exists(_OUT) and all(os.path.getmtime(_OUT) >= os.path.getmtime(f)
+                                                   for f in _SRCS):
         return _OUT
     os.makedirs(os.path.dirname(_OUT), exist_ok=True)
     tmp = _OUT + ".tmp.%d" % os.getpid()
     cmd = ["gcc", "-O2", "-std=c11", "-fopenmp", "-fPIC", "-shared", "-Wall", "-Wextra",
-           _SRC, "-o", tmp, "-lm"]
+           *_SRCS, "-o", tmp, "-lm"]
     subprocess.run(cmd, check=True)
     os.replace(tmp, _OUT)
     return _OUT
@@ -59,7 +65,13 @@ def _load():
     lib.skip_oracle_bf16_value.restype = ctypes.c_double
     lib.skip_oracle_e4m3_value.argtypes = [ctypes.c_uint8]
     lib.skip_oracle_e4m3_value.restype = ctypes.c_double
-    for f in ("skip_oracle_region_topk", "skip_oracle_merge", "skip_oracle_retrieve",
+    lib.skip_oracle_skv.argtypes = [P, i64, i32, P, i32, i32, P, P, P, P, P, ctypes.c_float, i32,
+                                    ctypes.c_double, ctypes.c_double, P, P, P, P, P]
+    lib.skip_oracle_skv_count.argtypes = [i32, ctypes.c_double]
+    lib.skip_oracle_bf16_round.argtypes = [ctypes.c_double]
+    lib.skip_oracle_bf16_round.restype = ctypes.c_uint16
+    for f in ("skip_oracle_region_topk", "skip_oracle_merge", "skip_oracle_retrieve", "skip_oracle_skv",
+              "skip_oracle_skv_count",
               "skip_oracle_score_matrix", "skip_oracle_scores_at", "skip_oracle_threads"):
         getattr(lib, f).restype = ctypes.c_int
     _lib = lib
@@ -181,3 +193,48 @@ def scores_at(corpus, regions, region_idx, ids, row_scale=None):
     if rc:
         raise RuntimeError("oracle scores_at failed (%d)" % rc)
     return out
+
+
+def bf16_round(x: float) -> int:
+    """x rounded to bf16 (ties to even); the bit pattern."""
+    return int(_load().skip_oracle_bf16_round(float(x)))
+
+
+def skv_count(n_nonempty: int, rho: float) -> int:
+    """ceil(rho * |K| - 1e-3) clamped to [0, |K|]: how many gated passages are kept."""
+    return int(_load().skip_oracle_skv_count(int(n_nonempty), float(rho)))
+
+
+def skv(corpus, ids, qbar, vbar, w1, b1, w2, b2, tau=0.5, rho=0.6):
+    """SKV gate on candidate lists (Def. B.4 and the Alg. 1 TopK).
+
+    corpus uint16 [N, d] (bf16 bits); ids int64 [Q, K] (-1 = empty slot);
+    qbar, vbar uint16 [Q, d]; w1 uint16 [H, 5d]; b1, w2 float32 [H]; b2 float.
+    Returns a dict: nu_all, bound (float64 [Q, K]), ids (int64 [Q, K]),
+    nu (float64 [Q, K]), count (int32 [Q]).
+    """
+    lib = _load()
+    corpus = np.ascontiguousarray(corpus, dtype=np.uint16)
+    ids = np.ascontiguousarray(ids, dtype=np.int64)
+    qbar = np.ascontiguousarray(qbar, dtype=np.uint16)
+    vbar = np.ascontiguousarray(vbar, dtype=np.uint16)
+    w1 = np.ascontiguousarray(w1, dtype=np.uint16)
+    b1 = np.ascontiguousarray(b1, dtype=np.float32)
+    w2 = np.ascontiguousarray(w2, dtype=np.float32)
+    N, d = corpus.shape
+    Q, K = ids.shape
+    H = w1.shape[0]
+    if w1.shape[1] != 5 * d or qbar.shape != (Q, d) or vbar.shape != (Q, d) or b1.shape != (H,) \
+            or w2.shape != (H,):
+        raise ValueError("skv: inconsistent shapes")
+    nu_all = np.empty((Q, K), np.float64)
+    bound = np.empty((Q, K), np.float64)
+    out_ids = np.empty((Q, K), np.int64)
+    out_nu = np.empty((Q, K), np.float64)
+    count = np.empty(Q, np.int32)
+    rc = lib.skip_oracle_skv(_ptr(corpus), N, d, _ptr(ids), Q, K, _ptr(qbar), _ptr(vbar), _ptr(w1),
+                             _ptr(b1), _ptr(w2), float(b2), H, float(tau), float(rho), _ptr(nu_all),
+                             _ptr(bound), _ptr(out_ids), _ptr(out_nu), _ptr(count))
+    if rc:
+        raise RuntimeError("oracle skv failed (%d)" % rc)
+    return {"nu_all": nu_all, "bound": bound, "ids": out_ids, "nu": out_nu, "count": count}

@@ -224,3 +224,62 @@ def random_bf16(n: int, d: int, seed: int, device="cpu") -> torch.Tensor:
 def bf16_bits(t: torch.Tensor):
     """uint16 numpy view of a bf16 tensor (host)."""
     return t.detach().to("cpu").contiguous().view(torch.int16).numpy().view("uint16")
+
+
+# ---- inputs of the SKV passage gate (App. B.4 Def. B.4) --------------------
+#
+# The gate reads the question embedding qbar, the mean-pooled visual tokens
+# vbar (both d-dimensional here), each candidate passage's embedding (its
+# corpus row) and the two-layer MLP h_psi.  No trained encoder or MLP exists
+# here, so they are drawn:
+#
+# * qbar: normalise(first region query of the question + 0.5 / sqrt(d) * z);
+#   a question with no region draws a Gaussian unit vector; vbar: Gaussian
+#   unit vector; seed 3000 + workload index (or the given seed);
+# * W1 [H x 5d] ~ N(0, 1/5) (the five input blocks are unit-scale vectors, so
+#   pre-activations are ~N(0, 1)), b1 ~ N(0, 0.1^2), w2 ~ N(0, 4/H),
+#   b2 = 0.1; H = 512 (App. I.4, "SKV MLP hidden dim."); W1 stored bf16,
+#   b1 and w2 fp32; seed 4000 + workload index;
+# * standalone candidate lists: per question distinct ids in random order,
+#   the last `empty` slots -1 (seeded).
+
+SKV_HIDDEN = 512
+
+
+def make_skv_mlp(d: int, hidden: int = SKV_HIDDEN, seed: int = 4000, device="cpu"):
+    """(w1 bf16 [H, 5d], b1 fp32 [H], w2 fp32 [H], b2 float)."""
+    g = _gen(seed, "cpu")
+    w1 = (torch.randn(hidden, 5 * d, generator=g) / math.sqrt(5.0)).to(torch.bfloat16)
+    b1 = 0.1 * torch.randn(hidden, generator=g)
+    w2 = (2.0 / math.sqrt(hidden)) * torch.randn(hidden, generator=g)
+    return w1.to(device), b1.to(device), w2.to(device), 0.1
+
+
+def make_skv_queries(regions: torch.Tensor, offsets, seed: int = 3000, device="cpu"):
+    """(qbar bf16 [Q, d], vbar bf16 [Q, d]) for a region batch."""
+    offsets = torch.as_tensor(offsets).to("cpu")
+    Q = offsets.numel() - 1
+    d = regions.shape[1]
+    g = _gen(seed, "cpu")
+    reg = regions.to("cpu").float()
+    z = torch.randn(Q, d, generator=g)
+    lead = _normalise(torch.randn(Q, d, generator=g))
+    for q in range(Q):
+        if int(offsets[q + 1]) > int(offsets[q]):
+            lead[q] = reg[int(offsets[q])]
+    qbar = _normalise(lead + (0.5 / math.sqrt(d)) * z)
+    vbar = _normalise(torch.randn(Q, d, generator=g))
+    return qbar.to(torch.bfloat16).to(device), vbar.to(torch.bfloat16).to(device)
+
+
+def make_candidate_ids(N: int, Q: int, K: int, empty, seed: int) -> torch.Tensor:
+    """int64 [Q, K]: distinct ids per question, the last empty[q] slots -1."""
+    g = _gen(seed, "cpu")
+    out = torch.full((Q, K), -1, dtype=torch.int64)
+    empty = torch.as_tensor(empty).expand(Q) if not torch.is_tensor(empty) or empty.dim() == 0 \
+        else torch.as_tensor(empty)
+    for q in range(Q):
+        n = K - int(empty[q])
+        if n > 0:
+            out[q, :n] = torch.randperm(N, generator=g)[:n]
+    return out

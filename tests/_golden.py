@@ -15,7 +15,8 @@ def read_fixture(name):
         parts = lines[i].split()
         key = parts[0]
         if len(parts) == 2 and key in ("corpus", "regions", "region_ids", "region_scores",
-                                       "merged_ids", "merged_scores"):
+                                       "merged_ids", "merged_scores", "skv_corpus", "w1", "qbar",
+                                       "vbar", "ids", "nu_all", "out_ids", "out_nu"):
             n = int(parts[1])
             rows = [[float(v) for v in lines[i + 1 + t].split()] for t in range(n)]
             out[key] = np.array(rows, dtype=np.float64)
