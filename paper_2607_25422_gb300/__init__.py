@@ -11,6 +11,9 @@ The operation (paper §3.3 Eq. rcsr; App. B.2 Def. B.2; Alg. 1 RCSR loop and
 Dedup): each region query is scored against the corpus by inner product, the
 top-k_region ids are kept per region, and each question's region lists are
 merged into a deduplicated top-K (max score per id, ties to the lower id).
+The SKV passage gate (App. B.4 Def. B.4; ``include/skip_skv.h``) then keeps
+the passages whose verification score nu reaches tau, at most
+ceil(rho |K|) of them.
 """
 from __future__ import annotations
 
@@ -29,6 +32,12 @@ SKIP_PATH_AUTO, SKIP_PATH_TENSOR, SKIP_PATH_WARP, SKIP_PATH_LATENCY = range(4)
 SKIP_MAX_K_REGION, SKIP_MAX_K = 1024, 2048
 
 _lib = None
+
+
+class SkvMlp(ctypes.Structure):
+    """``skip_skv_mlp_t``: the gate MLP h_psi, pointers to device weights."""
+    _fields_ = [("hidden", ctypes.c_int32), ("w1", ctypes.c_void_p), ("b1", ctypes.c_void_p),
+                ("w2", ctypes.c_void_p), ("b2", ctypes.c_float)]
 
 
 class SkipError(RuntimeError):
@@ -58,11 +67,15 @@ def load_library():
     lib.skip_last_plan.argtypes = [P, ctypes.c_char_p, i32]
     lib.skip_timing_report.argtypes = [P, ctypes.c_char_p, i32]
     lib.skip_retrieve_regions_noalloc.argtypes = [P, i64, i32, ctypes.c_int, P, P, i32, i32, P, P, P]
+    lib.skip_skv_gate.argtypes = [P, P, i32, i32, P, P, ctypes.POINTER(SkvMlp), ctypes.c_float,
+                                  ctypes.c_float, P, P, P, P, P]
+    lib.skip_retrieve_skv.argtypes = [P, P, P, i32, i32, i32, i32, P, P, ctypes.POINTER(SkvMlp), ctypes.c_float,
+                                      ctypes.c_float, P, P, P, P, P, P]
     lib.skip_status_string.argtypes = [ctypes.c_int]
     lib.skip_status_string.restype = ctypes.c_char_p
     for f in ("skip_corpus_load", "skip_corpus_free", "skip_corpus_set_option", "skip_retrieve",
               "skip_retrieve_regions", "skip_retrieve_host", "skip_sync_status", "skip_last_plan",
-              "skip_timing_report", "skip_retrieve_regions_noalloc"):
+              "skip_timing_report", "skip_retrieve_regions_noalloc", "skip_skv_gate", "skip_retrieve_skv"):
         getattr(lib, f).restype = ctypes.c_int
     _lib = lib
     return lib
@@ -226,6 +239,64 @@ def skip_retrieve_regions_noalloc(corpus_rows: torch.Tensor, regions: torch.Tens
     return reg_ids, reg_scores
 
 
+def _skv_mlp(w1: torch.Tensor, b1: torch.Tensor, w2: torch.Tensor, b2: float):
+    """Marshal the gate weights (device tensors, kept alive by the caller)."""
+    if w1.dtype not in (torch.bfloat16, torch.uint16, torch.int16) or b1.dtype != torch.float32 \
+            or w2.dtype != torch.float32:
+        raise TypeError("w1 must be bf16 [H, 5d]; b1, w2 float32 [H]")
+    if not (w1.is_contiguous() and b1.is_contiguous() and w2.is_contiguous()):
+        raise ValueError("gate weights must be contiguous")
+    return SkvMlp(w1.shape[0], w1.data_ptr(), b1.data_ptr(), w2.data_ptr(), float(b2))
+
+
+def skip_skv_gate(corpus: Corpus, cand_ids: torch.Tensor, qbar: torch.Tensor, vbar: torch.Tensor,
+                  w1: torch.Tensor, b1: torch.Tensor, w2: torch.Tensor, b2: float, tau_nu: float = 0.5,
+                  rho_r: float = 0.6, with_nu_all: bool = False, stream=None):
+    """SKV gate on candidate lists (device int64 [Q, K], -1 = empty).
+    Returns (ids int64 [Q, K], nu fp32 [Q, K], count int32 [Q]) and, with
+    with_nu_all, nu of every input slot as a fourth tensor."""
+    lib = load_library()
+    cand_ids = cand_ids.to(torch.int64).contiguous()
+    Q, K = cand_ids.shape
+    dev = cand_ids.device
+    qbar, vbar = qbar.contiguous(), vbar.contiguous()
+    mlp = _skv_mlp(w1, b1, w2, b2)
+    out_ids = torch.empty(Q, K, dtype=torch.int64, device=dev)
+    out_nu = torch.empty(Q, K, dtype=torch.float32, device=dev)
+    count = torch.empty(Q, dtype=torch.int32, device=dev)
+    nu_all = torch.empty(Q, K, dtype=torch.float32, device=dev) if with_nu_all else None
+    st = lib.skip_skv_gate(corpus.handle, _ptr(cand_ids), Q, K, _ptr(qbar), _ptr(vbar), ctypes.byref(mlp),
+                           float(tau_nu), float(rho_r), _ptr(out_ids), _ptr(out_nu), _ptr(count), _ptr(nu_all),
+                           ctypes.c_void_p(_stream(stream)))
+    _check(st, "skip_skv_gate")
+    return (out_ids, out_nu, count, nu_all) if with_nu_all else (out_ids, out_nu, count)
+
+
+def skip_retrieve_skv(corpus: Corpus, regions: torch.Tensor, region_offsets: torch.Tensor, k_region: int,
+                      K: int, qbar: torch.Tensor, vbar: torch.Tensor, w1: torch.Tensor, b1: torch.Tensor,
+                      w2: torch.Tensor, b2: float, tau_nu: float = 0.5, rho_r: float = 0.6,
+                      with_merged: bool = False, stream=None):
+    """Retrieval and gate in one call.  Returns (ids, nu, count) and, with
+    with_merged, the merged lists (ids int64 [Q, K], scores fp32 [Q, K])."""
+    lib = load_library()
+    regions = _regions_arg(regions, corpus)
+    offs = region_offsets.to(device=regions.device, dtype=torch.int32).contiguous()
+    Q = offs.numel() - 1
+    dev = regions.device
+    mlp = _skv_mlp(w1, b1, w2, b2)
+    out_ids = torch.empty(Q, K, dtype=torch.int64, device=dev)
+    out_nu = torch.empty(Q, K, dtype=torch.float32, device=dev)
+    count = torch.empty(Q, dtype=torch.int32, device=dev)
+    m_ids = torch.empty(Q, K, dtype=torch.int64, device=dev) if with_merged else None
+    m_sc = torch.empty(Q, K, dtype=torch.float32, device=dev) if with_merged else None
+    st = lib.skip_retrieve_skv(corpus.handle, _ptr(regions), _ptr(offs), Q, regions.shape[0], int(k_region),
+                               int(K), _ptr(qbar.contiguous()), _ptr(vbar.contiguous()), ctypes.byref(mlp),
+                               float(tau_nu), float(rho_r), _ptr(out_ids), _ptr(out_nu), _ptr(count),
+                               _ptr(m_ids), _ptr(m_sc), ctypes.c_void_p(_stream(stream)))
+    _check(st, "skip_retrieve_skv")
+    return (out_ids, out_nu, count, m_ids, m_sc) if with_merged else (out_ids, out_nu, count)
+
+
 def skip_sync_status(corpus: Corpus, stream=None) -> int:
     """Synchronise and return the status latched by the kernels (SKIP_OK, ...)."""
     return int(load_library().skip_sync_status(corpus.handle, ctypes.c_void_p(_stream(stream))))
@@ -246,4 +317,4 @@ def skip_timing_report(corpus: Corpus) -> dict:
 
 
 __all__ = [n for n in dir() if n.startswith("skip_") or n.startswith("SKIP_")] + [
-    "Corpus", "SkipError", "load_library", "library_path"]
+    "Corpus", "SkipError", "SkvMlp", "load_library", "library_path"]

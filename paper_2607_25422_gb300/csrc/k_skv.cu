@@ -1,0 +1,383 @@
+// SKV passage gate (App. B.4 Def. B.4, Eq. skv_score; Alg. 1 "SKV: verify"
+// and the TopK after it) on the merged retrieval lists.
+//
+//  k_skv_qbias   per question: c_q = b1 + W1[:, qbar] qbar + W1[:, vbar] vbar
+//                (fp32, one warp per hidden unit, W1 row slice in registers).
+//  k_skv_mlp     per 128 passage slots x 128 hidden units: the passage part
+//                of layer 1 on the tensor cores.  The A operand is built in
+//                shared memory by four warps from the gathered corpus rows
+//                and qbar: per 64-column chunk of d, three K-slices
+//                e | bf16(e * qbar) | bf16(|e - qbar|) in the 128-byte
+//                swizzled layout TMA would produce; the B operand is the
+//                matching W1 column blocks, loaded by TMA.  tcgen05.mma
+//                (kind::f16, M = N = 128) accumulates in TMEM; the epilogue
+//                adds c_q, applies ReLU and the w2 dot for its 128 units and
+//                writes one partial logit per slot and hidden block.
+//  k_skv_select  per question: logit = b2 + sum of the partial logits,
+//                nu = sigmoid(logit), gate nu >= tau, then the first
+//                ceil(rho |K| - 1e-3) by (nu desc, id asc) (bitonic sort).
+#include <cuda.h>
+#include <cuda_bf16.h>
+#include <cuda_runtime.h>
+
+#include "skip_device.cuh"
+#include "skip_internal.h"
+
+namespace skipk {
+namespace {
+
+constexpr int kSkvRows = 128;                       // passage slots per CTA (TMEM lanes)
+constexpr int kSkvSlice = kSkvRows * 128;           // one [128 x 64] bf16 K-slice, bytes
+constexpr int kSkvStageA = 3 * kSkvSlice;           // e | e*qbar | |e - qbar|
+constexpr int kSkvStageB = 3 * kSkvSlice;           // the three W1 column blocks (128 units)
+constexpr int kSkvStages = 2;
+constexpr int kSkvThreads = 192;                    // TMA warp, MMA warp, 4 builder/epilogue warps
+constexpr uint32_t kSkvIdesc = idesc_bf16_f32(128, kSkvHidden);
+constexpr uint64_t kDrainTimeoutNs = 1000000000ull;  // 1 s for copies in flight
+
+struct SkvShared {
+    uint64_t full[kSkvStages];   // A built (128 arrivals) and B landed (tx bytes)
+    uint64_t empty[kSkvStages];  // stage consumed (tcgen05.commit)
+    uint64_t tfull;              // accumulator complete
+    uint32_t tmem_base;
+};
+
+__device__ __forceinline__ void sts128(uint32_t addr, uint4 v) {
+    asm volatile("st.shared.v4.b32 [%0], {%1, %2, %3, %4};" ::"r"(addr), "r"(v.x), "r"(v.y), "r"(v.z),
+                 "r"(v.w)
+                 : "memory");
+}
+
+__device__ __forceinline__ void fence_proxy_async_smem() {
+    asm volatile("fence.proxy.async.shared::cta;" ::: "memory");
+}
+
+// Two bf16 lanes of a 32-bit word -> the two interaction features, rounded
+// to bf16 (ties to even).
+__device__ __forceinline__ void features2(uint32_t e2, uint32_t q2, uint32_t &eq2, uint32_t &ad2) {
+    const __nv_bfloat162 e = *reinterpret_cast<const __nv_bfloat162 *>(&e2);
+    const __nv_bfloat162 q = *reinterpret_cast<const __nv_bfloat162 *>(&q2);
+    const float2 ef = __bfloat1622float2(e), qf = __bfloat1622float2(q);
+    // e * qbar is exact in fp32 (two 8-bit significands); |e - qbar| is exact
+    // in fp32 unless the exponents are more than 16 apart, where the bf16
+    // result is the larger operand's magnitude either way.
+    const __nv_bfloat162 m = __floats2bfloat162_rn(ef.x * qf.x, ef.y * qf.y);
+    const __nv_bfloat162 a = __floats2bfloat162_rn(fabsf(ef.x - qf.x), fabsf(ef.y - qf.y));
+    eq2 = *reinterpret_cast<const uint32_t *>(&m);
+    ad2 = *reinterpret_cast<const uint32_t *>(&a);
+}
+
+__global__ void __launch_bounds__(kSkvThreads, 1)
+    k_skv_mlp(const __grid_constant__ CUtensorMap tw, const SkvParams p) {
+    extern __shared__ __align__(1024) uint8_t smem_raw[];
+    uint8_t *smem = reinterpret_cast<uint8_t *>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
+    uint8_t *sA = smem;
+    uint8_t *sB = smem + kSkvStages * kSkvStageA;
+    SkvShared *sh = reinterpret_cast<SkvShared *>(sB + kSkvStages * kSkvStageB);
+    const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+    const int64_t m0 = (int64_t)blockIdx.x * kSkvRows;
+    const int n0 = blockIdx.y * kSkvHidden;
+    const int nc = p.d / 64;
+
+    if (threadIdx.x == 0) {
+        for (int s = 0; s < kSkvStages; ++s) {
+            mbar_init(smem_addr(&sh->full[s]), kSkvRows + 1);
+            mbar_init(smem_addr(&sh->empty[s]), 1);
+        }
+        mbar_init(smem_addr(&sh->tfull), 1);
+        mbar_fence_init();
+    }
+    if (warp == 0 && lane == 0) tma_prefetch_desc(&tw);
+    if (warp == 1) {
+        tmem_alloc(smem_addr(&sh->tmem_base), kSkvHidden);
+        tmem_relinquish();
+    }
+    tc_fence_before();
+    __syncthreads();
+    tc_fence_after();
+    const uint32_t tmem = sh->tmem_base;
+
+    if (warp == 0) {
+        // ------------------------------------------------ TMA: W1 column blocks
+        if (lane == 0) {
+            bool ok = true;
+            int issued = 0;
+            for (int c = 0; c < nc && ok; ++c) {
+                const int s = c % kSkvStages;
+                const uint32_t ph = (uint32_t)(c / kSkvStages) & 1u;
+                if (!mbar_wait(smem_addr(&sh->empty[s]), ph ^ 1u, p.timeout_ns)) {
+                    ok = false;
+                    break;
+                }
+                const uint32_t fb = smem_addr(&sh->full[s]);
+                mbar_arrive_expect_tx(fb, kSkvStageB);
+                for (int b = 0; b < 3; ++b)
+                    tma_load_2d(smem_addr(sB + s * kSkvStageB + b * kSkvSlice), &tw, fb, (2 + b) * p.d + c * 64, n0);
+                ++issued;
+            }
+            if (!ok) atomicOr(p.err, kErrTimeout);
+            // Copies in flight: wait for the last use of each stage to complete.
+            for (int s = 0; s < kSkvStages; ++s) {
+                const int uses = issued / kSkvStages + (s < issued % kSkvStages ? 1 : 0);
+                if (uses == 0) continue;
+                if (!mbar_wait(smem_addr(&sh->full[s]), (uint32_t)((uses - 1) & 1), kDrainTimeoutNs))
+                    atomicOr(p.err, kErrTimeout);
+            }
+        }
+    } else if (warp == 1) {
+        // ------------------------------------------------ MMA issuer
+        if (lane == 0) {
+            bool ok = true;
+            for (int c = 0; c < nc && ok; ++c) {
+                const int s = c % kSkvStages;
+                const uint32_t ph = (uint32_t)(c / kSkvStages) & 1u;
+                if (!mbar_wait(smem_addr(&sh->full[s]), ph, p.timeout_ns)) {
+                    ok = false;
+                    break;
+                }
+                tc_fence_after();
+                for (int b = 0; b < 3; ++b) {
+                    const uint64_t ad = smem_desc_k128(smem_addr(sA + s * kSkvStageA + b * kSkvSlice));
+                    const uint64_t bd = smem_desc_k128(smem_addr(sB + s * kSkvStageB + b * kSkvSlice));
+#pragma unroll
+                    for (int kk = 0; kk < 4; ++kk)
+                        tc_mma_f16(tmem, ad + (uint64_t)(kk * 2), bd + (uint64_t)(kk * 2), kSkvIdesc,
+                                   (c | b | kk) != 0);
+                }
+                tc_commit(smem_addr(&sh->empty[s]));
+            }
+            if (!ok) atomicOr(p.err, kErrTimeout);
+            // Arrives once every MMA issued has completed (also after a timeout).
+            tc_commit(smem_addr(&sh->tfull));
+        }
+    } else {
+        // ------------------------------------------------ builders, then epilogue
+        const int r = (warp & 3) * 32 + lane;  // TMEM lane = slot row in the tile
+        const int64_t slot = m0 + r;
+        int64_t id = -1;
+        int q = 0;
+        if (slot < p.P) {
+            id = p.ids[slot];
+            q = (int)(slot / p.K);
+            if (id >= p.N) {
+                atomicOr(p.err, kErrConfig);
+                id = -1;
+            }
+        }
+        const uint4 *erow = reinterpret_cast<const uint4 *>(p.rows + (id < 0 ? 0 : id) * (int64_t)p.d);
+        const uint4 *qrow = reinterpret_cast<const uint4 *>(p.qbar + (int64_t)q * p.d);
+        const uint4 zero = make_uint4(0, 0, 0, 0);
+        // Chunk c + 1's loads are issued before chunk c is written out.
+        uint4 en[8], qn[8];
+#pragma unroll
+        for (int j = 0; j < 8; ++j) {
+            en[j] = id >= 0 ? __ldg(erow + j) : zero;
+            qn[j] = id >= 0 ? __ldg(qrow + j) : zero;
+        }
+        bool ok = true;
+        for (int c = 0; c < nc; ++c) {
+            const int s = c % kSkvStages;
+            const uint32_t ph = (uint32_t)(c / kSkvStages) & 1u;
+            uint4 e[8], qv[8];
+#pragma unroll
+            for (int j = 0; j < 8; ++j) {
+                e[j] = en[j];
+                qv[j] = qn[j];
+            }
+            if (c + 1 < nc && id >= 0) {
+#pragma unroll
+                for (int j = 0; j < 8; ++j) {
+                    en[j] = __ldg(erow + (c + 1) * 8 + j);
+                    qn[j] = __ldg(qrow + (c + 1) * 8 + j);
+                }
+            }
+            if (!mbar_wait(smem_addr(&sh->empty[s]), ph ^ 1u, p.timeout_ns)) {
+                ok = false;
+                break;
+            }
+            // Row r of each slice: 16-byte chunk j at position j ^ (r & 7).
+            const uint32_t base = smem_addr(sA + s * kSkvStageA) + r * 128;
+            const int sw = r & 7;
+#pragma unroll
+            for (int j = 0; j < 8; ++j) {
+                uint4 eq, ad;
+                features2(e[j].x, qv[j].x, eq.x, ad.x);
+                features2(e[j].y, qv[j].y, eq.y, ad.y);
+                features2(e[j].z, qv[j].z, eq.z, ad.z);
+                features2(e[j].w, qv[j].w, eq.w, ad.w);
+                const uint32_t off = (uint32_t)((j ^ sw) << 4);
+                sts128(base + off, e[j]);
+                sts128(base + kSkvSlice + off, eq);
+                sts128(base + 2 * kSkvSlice + off, ad);
+            }
+            fence_proxy_async_smem();
+            mbar_arrive(smem_addr(&sh->full[s]));
+        }
+        if (!ok) atomicOr(p.err, kErrTimeout);
+        // Epilogue: h = acc + c_q, ReLU, dot with w2 over this CTA's units.
+        const bool done = mbar_wait(smem_addr(&sh->tfull), 0, p.timeout_ns);
+        if (!done) atomicOr(p.err, kErrTimeout);
+        tc_fence_after();
+        if (done) {
+            const uint32_t lane_addr = (uint32_t)((warp & 3) * 32) << 16;
+            const float *cq = p.cq + (int64_t)q * p.H + n0;
+            const float *w2 = p.w2 + n0;
+            float part = 0.f;
+#pragma unroll 1
+            for (int c = 0; c < kSkvHidden / 32; ++c) {
+                uint32_t v[32];
+                tmem_ld_32x32b_x32(tmem + lane_addr + c * 32, v);
+                tmem_ld_wait(v);
+#pragma unroll
+                for (int i = 0; i < 32; ++i) {
+                    const float h = __uint_as_float(v[i]) + __ldg(cq + c * 32 + i);
+                    part = fmaf(fmaxf(h, 0.f), __ldg(w2 + c * 32 + i), part);
+                }
+            }
+            if (slot < p.P) p.partial[(int64_t)blockIdx.y * p.P + slot] = part;
+        }
+    }
+
+    tc_fence_before();
+    __syncthreads();
+    tc_fence_after();
+    if (warp == 1) {
+        __syncwarp();
+        tmem_dealloc(tmem, kSkvHidden);
+    }
+}
+
+// c[q][i] = b1[i] + sum_t W1[i][t] qbar[q][t] + sum_t W1[i][d + t] vbar[q][t]:
+// one warp per hidden unit i, its 2d weights held in registers (d <= 1024),
+// questions in turn.
+__global__ void __launch_bounds__(128) k_skv_qbias(const SkvParams p) {
+    const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+    const int i = blockIdx.x * 4 + warp;
+    if (i >= p.H) return;
+    const int nv = (2 * p.d) / 8;  // 16-byte words in the row slice [qbar | vbar]
+    const int nq = p.d / 8;
+    const uint4 *wrow = reinterpret_cast<const uint4 *>(p.w1 + (int64_t)i * 5 * p.d);
+    uint4 w[8];
+#pragma unroll
+    for (int t = 0; t < 8; ++t) w[t] = (lane + 32 * t < nv) ? __ldg(wrow + lane + 32 * t) : make_uint4(0, 0, 0, 0);
+    const float b = p.b1[i];
+    for (int q = 0; q < p.Q; ++q) {
+        const uint4 *qrow = reinterpret_cast<const uint4 *>(p.qbar + (int64_t)q * p.d);
+        const uint4 *vrow = reinterpret_cast<const uint4 *>(p.vbar + (int64_t)q * p.d);
+        float acc = 0.f;
+#pragma unroll
+        for (int t = 0; t < 8; ++t) {
+            const int k = lane + 32 * t;
+            if (k >= nv) break;
+            const uint4 x = k < nq ? __ldg(qrow + k) : __ldg(vrow + (k - nq));
+            const uint32_t wv[4] = {w[t].x, w[t].y, w[t].z, w[t].w};
+            const uint32_t xv[4] = {x.x, x.y, x.z, x.w};
+#pragma unroll
+            for (int h = 0; h < 4; ++h) {
+                const float2 wf = __bfloat1622float2(*reinterpret_cast<const __nv_bfloat162 *>(&wv[h]));
+                const float2 xf = __bfloat1622float2(*reinterpret_cast<const __nv_bfloat162 *>(&xv[h]));
+                acc = fmaf(wf.x, xf.x, acc);
+                acc = fmaf(wf.y, xf.y, acc);
+            }
+        }
+#pragma unroll
+        for (int o = 16; o; o >>= 1) acc += __shfl_xor_sync(0xFFFFFFFFu, acc, o);
+        if (lane == 0) p.cq[(int64_t)q * p.H + i] = acc + b;
+    }
+}
+
+// One block per question: nu for every slot, the gate, and the first n by
+// (nu desc, id asc).  Keys (ordered nu bits << 32 | ~id) sort descending.
+constexpr int kSelThreads = 256;
+__global__ void __launch_bounds__(kSelThreads) k_skv_select(const SkvParams p) {
+    __shared__ uint64_t keys[kSkvMaxK];
+    __shared__ int nonempty, ngated;
+    const int q = blockIdx.x;
+    const int K = p.K;
+    int Kp = 1;
+    while (Kp < K) Kp <<= 1;
+    if (threadIdx.x == 0) nonempty = 0, ngated = 0;
+    __syncthreads();
+    const int nb = p.H / kSkvHidden;
+    int my_ne = 0, my_g = 0;
+    for (int j = threadIdx.x; j < Kp; j += kSelThreads) {
+        uint64_t key = 0;
+        if (j < K) {
+            const int64_t slot = (int64_t)q * K + j;
+            int64_t id = p.ids[slot];
+            if (id >= p.N) id = -1;  // flagged by k_skv_mlp
+            float nu = -__int_as_float(0x7f800000);
+            if (id >= 0) {
+                float logit = p.b2;
+                for (int b = 0; b < nb; ++b) logit += p.partial[(int64_t)b * p.P + slot];
+                nu = 1.f / (1.f + expf(-logit));
+                ++my_ne;
+                if (nu >= p.tau) {
+                    key = ((uint64_t)(__float_as_uint(nu) | 0x80000000u) << 32) |
+                          (uint64_t)(0xFFFFFFFFu - (uint32_t)id);
+                    ++my_g;
+                }
+            }
+            if (p.nu_all) p.nu_all[slot] = nu;
+        }
+        keys[j] = key;
+    }
+    if (my_ne) atomicAdd(&nonempty, my_ne);
+    if (my_g) atomicAdd(&ngated, my_g);
+    __syncthreads();
+    // bitonic sort, descending
+    for (int size = 2; size <= Kp; size <<= 1)
+        for (int stride = size >> 1; stride > 0; stride >>= 1) {
+            for (int t = threadIdx.x; t < Kp / 2; t += kSelThreads) {
+                const int lo = 2 * t - (t & (stride - 1));
+                const int hi = lo + stride;
+                const bool desc = (lo & size) == 0;
+                const uint64_t a = keys[lo], b = keys[hi];
+                if ((a < b) == desc) {
+                    keys[lo] = b;
+                    keys[hi] = a;
+                }
+            }
+            __syncthreads();
+        }
+    const double nd = ceil((double)p.rho * (double)nonempty - 1e-3);
+    int n = nd < 0.0 ? 0 : (int)nd;
+    if (n > nonempty) n = nonempty;
+    if (n > ngated) n = ngated;
+    for (int j = threadIdx.x; j < K; j += kSelThreads) {
+        const int64_t o = (int64_t)q * K + j;
+        if (j < n) {
+            const uint64_t key = keys[j];
+            p.out_ids[o] = (int64_t)(0xFFFFFFFFu - (uint32_t)key);
+            p.out_nu[o] = __uint_as_float((uint32_t)(key >> 32) & 0x7FFFFFFFu);
+        } else {
+            p.out_ids[o] = -1;
+            p.out_nu[o] = -__int_as_float(0x7f800000);
+        }
+    }
+    if (threadIdx.x == 0) p.out_count[q] = n;
+}
+
+}  // namespace
+
+size_t skv_mlp_smem_bytes() {
+    return 1024 + (size_t)kSkvStages * (kSkvStageA + kSkvStageB) + sizeof(SkvShared);
+}
+
+cudaError_t launch_skv(const CUtensorMap &tw, const SkvParams &p, cudaStream_t s) {
+    if (p.Q == 0) return cudaSuccess;
+    k_skv_qbias<<<(p.H + 3) / 4, 128, 0, s>>>(p);
+    cudaError_t e = cudaGetLastError();
+    if (e != cudaSuccess) return e;
+    const size_t smem = skv_mlp_smem_bytes();
+    e = cudaFuncSetAttribute(k_skv_mlp, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
+    if (e != cudaSuccess) return e;
+    dim3 grid((unsigned)((p.P + kSkvRows - 1) / kSkvRows), (unsigned)(p.H / kSkvHidden));
+    k_skv_mlp<<<grid, kSkvThreads, smem, s>>>(tw, p);
+    e = cudaGetLastError();
+    if (e != cudaSuccess) return e;
+    k_skv_select<<<p.Q, kSelThreads, 0, s>>>(p);
+    return cudaGetLastError();
+}
+
+}  // namespace skipk

@@ -13,6 +13,7 @@
 #include <vector>
 
 #include "../../include/skip_retrieve.h"
+#include "../../include/skip_skv.h"
 #include "skip_internal.h"
 
 using namespace skipk;
@@ -88,6 +89,8 @@ struct skip_corpus {
     size_t ws_bytes = 0;
     void *io = nullptr;        // device staging for skip_retrieve_host
     size_t io_bytes = 0;
+    void *gws = nullptr;       // SKV gate workspace
+    size_t gws_bytes = 0;
     int path = SKIP_PATH_AUTO;
     uint64_t timeout_ns = kDefaultTimeoutNs;
     int grid = 0;
@@ -113,23 +116,27 @@ skip_status_t cuda_status(cudaError_t e) {
     return SKIP_ECUDA;
 }
 
-skip_status_t ensure_ws(skip_corpus *c, size_t bytes) {
-    if (bytes <= c->ws_bytes) return SKIP_OK;
-    if (c->ws) {
+// Grows a device buffer to at least `bytes` (25% headroom); a buffer in use
+// by queued work is freed only after the device has drained.
+skip_status_t ensure_buf(void *&buf, size_t &have, size_t bytes) {
+    if (bytes <= have) return SKIP_OK;
+    if (buf) {
         cudaError_t e = cudaDeviceSynchronize();
         if (e != cudaSuccess) return SKIP_ECUDA;
-        cudaFree(c->ws);
-        c->ws = nullptr;
-        c->ws_bytes = 0;
+        cudaFree(buf);
+        buf = nullptr;
+        have = 0;
     }
     size_t want = bytes + bytes / 4;
-    if (cudaMalloc(&c->ws, want) != cudaSuccess) {
+    if (cudaMalloc(&buf, want) != cudaSuccess) {
         cudaGetLastError();
         return SKIP_ENOMEM;
     }
-    c->ws_bytes = want;
+    have = want;
     return SKIP_OK;
 }
+
+skip_status_t ensure_ws(skip_corpus *c, size_t bytes) { return ensure_buf(c->ws, c->ws_bytes, bytes); }
 
 void record(skip_corpus *c, cudaStream_t s, const char *name) {
     if (!c->timing || c->ev_used >= kMaxEvents) return;
@@ -473,6 +480,100 @@ void write_plan(skip_corpus *c, const Plan &pl, int R, int Q, int k, int K) {
              pl.tensor ? (pl.list_in_smem ? "shared" : "global") : "global");
 }
 
+// Argument rules of skip_retrieve.
+skip_status_t check_retrieve(skip_corpus *c, const void *regions, const int32_t *region_offsets, int32_t Q,
+                             int32_t R_total, int32_t k_region, int32_t K) {
+    skip_status_t st = check_common(c, regions, R_total, k_region);
+    if (st) return st;
+    if (Q < 0 || K < 1 || K > SKIP_MAX_K || (Q > 0 && !region_offsets)) return SKIP_EINVAL;
+    if (Q == 0 && R_total != 0) return SKIP_EINVAL;
+    return SKIP_OK;
+}
+
+// Per-region step, then the per-question merge into out_ids / out_scores.
+skip_status_t retrieve_impl(skip_corpus *c, const void *regions, const int32_t *region_offsets, int32_t Q,
+                            int32_t R_total, int32_t k_region, int32_t K, int64_t *out_ids, float *out_scores,
+                            cudaStream_t s, Plan &pl) {
+    const size_t keys_bytes = align_up((size_t)std::max(R_total, 1) * k_region * sizeof(uint64_t), 256);
+    uint64_t *reg_keys = nullptr;
+    skip_status_t st;
+    if (R_total > 0) {
+        st = run_regions(c, reinterpret_cast<const uint16_t *>(regions), R_total, k_region, &reg_keys,
+                         nullptr, nullptr, s, pl, keys_bytes);
+        if (st) return st;
+    } else {
+        st = ensure_ws(c, keys_bytes);
+        if (st) return st;
+        reg_keys = reinterpret_cast<uint64_t *>(c->ws);
+    }
+    if (Q > 0) {
+        record(c, s, "question_merge");
+        cudaError_t e = launch_question_merge(reg_keys, k_region, region_offsets, Q, R_total, K, out_ids,
+                                              out_scores, c->err, s);
+        if (e != cudaSuccess) return cuda_status(e);
+        ++pl.launches;
+    }
+    return SKIP_OK;
+}
+
+// Argument rules of the SKV gate (the corpus handle is already checked).
+skip_status_t check_skv(skip_corpus *c, int32_t Q, int32_t K, const uint16_t *qbar, const uint16_t *vbar,
+                        const skip_skv_mlp_t *mlp, float tau, float rho, const void *out_ids, const void *out_nu,
+                        const void *out_count) {
+    if (Q < 0 || K < 1 || K > SKIP_MAX_K || !mlp) return SKIP_EINVAL;
+    if (!(tau == tau) || !(rho >= 0.f && rho <= 1.f)) return SKIP_EINVAL;
+    if (mlp->hidden < kSkvHidden || mlp->hidden % kSkvHidden != 0 || !mlp->w1 || !mlp->b1 || !mlp->w2)
+        return SKIP_EINVAL;
+    if (Q > 0 && (!qbar || !vbar || !out_ids || !out_nu || !out_count)) return SKIP_EINVAL;
+    if (c->dtype != SKIP_BF16 || c->d % 64 != 0 || c->d > 1024) return SKIP_EUNSUPPORTED;
+    return SKIP_OK;
+}
+
+size_t skv_ws_bytes(int Q, int K, int H) {
+    const size_t P = (size_t)Q * K;
+    return align_up((size_t)Q * H * 4, 256) + align_up((size_t)(H / kSkvHidden) * P * 4, 256);
+}
+
+// The gate on cand_ids; its workspace is the head of gws (skv_ws_bytes).
+skip_status_t skv_impl(skip_corpus *c, const int64_t *cand_ids, int32_t Q, int32_t K, const uint16_t *qbar,
+                       const uint16_t *vbar, const skip_skv_mlp_t *mlp, float tau, float rho, int64_t *out_ids,
+                       float *out_nu, int32_t *out_count, float *nu_all, cudaStream_t s, Plan &pl) {
+    if (Q == 0) return SKIP_OK;
+    const int H = mlp->hidden;
+    CUtensorMap tw;
+    if (!encode_bf16_rows(&tw, mlp->w1, H, 5 * c->d, 128)) return SKIP_ECUDA;
+    SkvParams p;
+    p.rows = reinterpret_cast<const uint16_t *>(c->rows);
+    p.N = c->N;
+    p.d = c->d;
+    p.ids = cand_ids;
+    p.P = (int64_t)Q * K;
+    p.K = K;
+    p.Q = Q;
+    p.qbar = qbar;
+    p.vbar = vbar;
+    p.w1 = mlp->w1;
+    p.b1 = mlp->b1;
+    p.w2 = mlp->w2;
+    p.b2 = mlp->b2;
+    p.H = H;
+    p.tau = tau;
+    p.rho = rho;
+    p.cq = reinterpret_cast<float *>(c->gws);
+    p.partial = reinterpret_cast<float *>((char *)c->gws + align_up((size_t)Q * H * 4, 256));
+    p.out_ids = out_ids;
+    p.out_nu = out_nu;
+    p.out_count = out_count;
+    p.nu_all = nu_all;
+    p.err = c->err;
+    p.timeout_ns = c->timeout_ns;
+    record(c, s, "skv_gate");
+    cudaError_t e = launch_skv(tw, p, s);
+    if (e != cudaSuccess) return cuda_status(e);
+    pl.launches += 3;
+    return SKIP_OK;
+}
+
 }  // namespace
 
 extern "C" {
@@ -549,6 +650,7 @@ skip_status_t skip_corpus_free(skip_corpus_t c) {
     cudaFree(c->err);
     cudaFree(c->ws);
     cudaFree(c->io);
+    cudaFree(c->gws);
     for (cudaEvent_t e : c->ev_pool) cudaEventDestroy(e);
     delete c;
     return SKIP_OK;
@@ -587,32 +689,14 @@ skip_status_t skip_corpus_set_option(skip_corpus_t c, int option, int64_t value)
 skip_status_t skip_retrieve(skip_corpus_t c, const void *regions, const int32_t *region_offsets,
                             int32_t Q, int32_t R_total, int32_t k_region, int32_t K, int64_t *out_ids,
                             float *out_scores, void *stream) {
-    skip_status_t st = check_common(c, regions, R_total, k_region);
+    skip_status_t st = check_retrieve(c, regions, region_offsets, Q, R_total, k_region, K);
     if (st) return st;
-    if (Q < 0 || K < 1 || K > SKIP_MAX_K || (Q > 0 && !region_offsets)) return SKIP_EINVAL;
     if (Q > 0 && (!out_ids || !out_scores)) return SKIP_EINVAL;
-    if (Q == 0 && R_total != 0) return SKIP_EINVAL;
     cudaStream_t s = reinterpret_cast<cudaStream_t>(stream);
     ++c->call_id;
     Plan pl;
-    const size_t keys_bytes = align_up((size_t)std::max(R_total, 1) * k_region * sizeof(uint64_t), 256);
-    uint64_t *reg_keys = nullptr;
-    if (R_total > 0) {
-        st = run_regions(c, reinterpret_cast<const uint16_t *>(regions), R_total, k_region, &reg_keys,
-                         nullptr, nullptr, s, pl, keys_bytes);
-        if (st) return st;
-    } else {
-        st = ensure_ws(c, keys_bytes);
-        if (st) return st;
-        reg_keys = reinterpret_cast<uint64_t *>(c->ws);
-    }
-    if (Q > 0) {
-        record(c, s, "question_merge");
-        cudaError_t e = launch_question_merge(reg_keys, k_region, region_offsets, Q, R_total, K, out_ids,
-                                              out_scores, c->err, s);
-        if (e != cudaSuccess) return cuda_status(e);
-        ++pl.launches;
-    }
+    st = retrieve_impl(c, regions, region_offsets, Q, R_total, k_region, K, out_ids, out_scores, s, pl);
+    if (st) return st;
     record(c, s, "end");
     write_plan(c, pl, R_total, Q, k_region, K);
     return SKIP_OK;
@@ -749,6 +833,56 @@ skip_status_t skip_timing_report(skip_corpus_t c, char *buf, int32_t len) {
     out += "}";
     if ((int)out.size() + 1 > len) return SKIP_EINVAL;
     memcpy(buf, out.c_str(), out.size() + 1);
+    return SKIP_OK;
+}
+
+}  // extern "C"
+
+extern "C" {
+
+skip_status_t skip_skv_gate(skip_corpus_t c, const int64_t *cand_ids, int32_t Q, int32_t K, const uint16_t *qbar,
+                            const uint16_t *vbar, const skip_skv_mlp_t *mlp, float tau_nu, float rho_r,
+                            int64_t *out_ids, float *out_nu, int32_t *out_count, float *nu_all, void *stream) {
+    if (!c) return SKIP_EINVAL;
+    skip_status_t st = check_skv(c, Q, K, qbar, vbar, mlp, tau_nu, rho_r, out_ids, out_nu, out_count);
+    if (st) return st;
+    if (Q > 0 && !cand_ids) return SKIP_EINVAL;
+    cudaStream_t s = reinterpret_cast<cudaStream_t>(stream);
+    st = ensure_buf(c->gws, c->gws_bytes, skv_ws_bytes(Q, K, mlp->hidden));
+    if (st) return st;
+    ++c->call_id;
+    Plan pl;
+    st = skv_impl(c, cand_ids, Q, K, qbar, vbar, mlp, tau_nu, rho_r, out_ids, out_nu, out_count, nu_all, s, pl);
+    if (st) return st;
+    record(c, s, "end");
+    return SKIP_OK;
+}
+
+skip_status_t skip_retrieve_skv(skip_corpus_t c, const void *regions, const int32_t *region_offsets, int32_t Q,
+                                int32_t R_total, int32_t k_region, int32_t K, const uint16_t *qbar,
+                                const uint16_t *vbar, const skip_skv_mlp_t *mlp, float tau_nu, float rho_r,
+                                int64_t *out_ids, float *out_nu, int32_t *out_count, int64_t *merged_ids,
+                                float *merged_scores, void *stream) {
+    skip_status_t st = check_retrieve(c, regions, region_offsets, Q, R_total, k_region, K);
+    if (st) return st;
+    st = check_skv(c, Q, K, qbar, vbar, mlp, tau_nu, rho_r, out_ids, out_nu, out_count);
+    if (st) return st;
+    cudaStream_t s = reinterpret_cast<cudaStream_t>(stream);
+    // gate workspace first, then the merged lists (unless the caller keeps them)
+    const size_t gate = skv_ws_bytes(Q, K, mlp->hidden);
+    const size_t mid = align_up((size_t)Q * K * 8, 256), msc = align_up((size_t)Q * K * 4, 256);
+    st = ensure_buf(c->gws, c->gws_bytes, gate + mid + msc);
+    if (st) return st;
+    int64_t *mids = merged_ids ? merged_ids : reinterpret_cast<int64_t *>((char *)c->gws + gate);
+    float *mscs = merged_scores ? merged_scores : reinterpret_cast<float *>((char *)c->gws + gate + mid);
+    ++c->call_id;
+    Plan pl;
+    st = retrieve_impl(c, regions, region_offsets, Q, R_total, k_region, K, mids, mscs, s, pl);
+    if (st) return st;
+    st = skv_impl(c, mids, Q, K, qbar, vbar, mlp, tau_nu, rho_r, out_ids, out_nu, out_count, nullptr, s, pl);
+    if (st) return st;
+    record(c, s, "end");
+    write_plan(c, pl, R_total, Q, k_region, K);
     return SKIP_OK;
 }
 

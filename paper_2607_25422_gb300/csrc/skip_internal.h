@@ -105,4 +105,36 @@ cudaError_t launch_question_merge(const uint64_t *reg_keys, int k, const int32_t
                                   int R, int K, int64_t *out_ids, float *out_scores, int *err,
                                   cudaStream_t s);
 
+// ---- SKV passage gate (k_skv.cu) ------------------------------------------
+constexpr int kSkvHidden = 128;  // hidden units per CTA of the gate MLP (TMEM columns)
+constexpr int kSkvMaxK = 2048;   // candidate slots per question (SKIP_MAX_K)
+struct SkvParams {
+    const uint16_t *rows;  // bf16 corpus [N x d]
+    int64_t N;
+    int d;                 // multiple of 64, at most 1024
+    const int64_t *ids;    // [Q x K] candidate ids, -1 = empty
+    int64_t P;             // Q * K slots
+    int K;
+    int Q;
+    const uint16_t *qbar;  // bf16 [Q x d]
+    const uint16_t *vbar;  // bf16 [Q x d]
+    const uint16_t *w1;    // bf16 [H x 5d]
+    const float *b1;       // [H]
+    const float *w2;       // [H]
+    float b2;
+    int H;                 // multiple of kSkvHidden
+    float tau, rho;
+    float *cq;             // [Q x H] workspace: b1 + W1 qbar-part + W1 vbar-part
+    float *partial;        // [H / kSkvHidden][P] workspace: partial logits
+    int64_t *out_ids;      // [Q x K]
+    float *out_nu;         // [Q x K]
+    int32_t *out_count;    // [Q]
+    float *nu_all;         // [Q x K] or null
+    int *err;
+    uint64_t timeout_ns;
+};
+size_t skv_mlp_smem_bytes();
+// tw: tensor map over W1 [H x 5d] bf16, box 64 columns x 128 rows, 128-byte swizzle.
+cudaError_t launch_skv(const CUtensorMap &tw, const SkvParams &p, cudaStream_t s);
+
 }  // namespace skipk
