@@ -272,6 +272,8 @@ def main():
                     help="use only the first ROWS corpus rows (smaller profiling captures; not a bench line)")
     ap.add_argument("--cluster", type=int, default=0, choices=[0, 1, 2, 4, 8],
                     help="single-CTA tensor path CTAs per cluster (0 = library's choice)")
+    ap.add_argument("--skv", action="store_true",
+                    help="step = retrieval + SKV passage gate (skip_retrieve_skv), H = 512, tau 0.5, rho 0.6")
     ap.add_argument("--mma", default="auto", choices=["auto", "single", "pair"],
                     help="tensor-path MMA shape (auto = library's choice)")
     args = ap.parse_args()
@@ -306,8 +308,17 @@ def main():
     out_sc = torch.empty(Q, spec.K, dtype=torch.float32, device=dev)
     stream = torch.cuda.current_stream()
 
-    def step():
-        skip.skip_retrieve(c, reg_d, off_d, spec.k_region, spec.K, out_ids, out_sc, stream)
+    if args.skv:
+        qbar, vbar = synth.make_skv_queries(regions, offsets)
+        w1, b1, w2, b2 = synth.make_skv_mlp(spec.d)
+        qbar, vbar, w1, b1, w2 = (x.to(dev).contiguous() for x in (qbar, vbar, w1, b1, w2))
+
+        def step():
+            return skip.skip_retrieve_skv(c, reg_d, off_d, spec.k_region, spec.K, qbar, vbar, w1, b1, w2, b2,
+                                          stream=stream)
+    else:
+        def step():
+            skip.skip_retrieve(c, reg_d, off_d, spec.k_region, spec.K, out_ids, out_sc, stream)
 
     for _ in range(args.warmup):
         step()
@@ -346,17 +357,32 @@ def main():
     off_h = offsets.pin_memory()
     ids_h = torch.empty(Q, spec.K, dtype=torch.int64).pin_memory()
     sc_h = torch.empty(Q, spec.K, dtype=torch.float32).pin_memory()
+    cnt_h = torch.empty(Q, dtype=torch.int32).pin_memory()
+
+    def e2e_step():
+        if args.skv:
+            # host regions in, gated lists out, through the device entry point
+            reg_d.copy_(reg_h, non_blocking=True)
+            off_d.copy_(off_h, non_blocking=True)
+            g_ids, g_nu, g_cnt = step()
+            ids_h.copy_(g_ids, non_blocking=True)
+            sc_h.copy_(g_nu, non_blocking=True)
+            cnt_h.copy_(g_cnt, non_blocking=True)
+            stream.synchronize()
+        else:
+            skip.skip_retrieve_host(c, reg_h, off_h, spec.k_region, spec.K, ids_h, sc_h, stream)
+
     for _ in range(3):
-        skip.skip_retrieve_host(c, reg_h, off_h, spec.k_region, spec.K, ids_h, sc_h, stream)
+        e2e_step()
     barrier(world)
     torch.cuda.synchronize()
     t0 = time.perf_counter()
     for _ in range(args.steps):
-        skip.skip_retrieve_host(c, reg_h, off_h, spec.k_region, spec.K, ids_h, sc_h, stream)
+        e2e_step()
     torch.cuda.synchronize()
     e2e_s = max_over_ranks(time.perf_counter() - t0, world)
     h2d = R * spec.d * 2 + (Q + 1) * 4
-    d2h = Q * spec.K * (8 + 4)
+    d2h = Q * spec.K * (8 + 4) + (Q * 4 if args.skv else 0)
 
     # ---- derived figures
     total_q = Q * world * args.steps
@@ -396,11 +422,25 @@ def main():
         "roofline": roof,
         "clocks": clocks,
         "e2e": {"value": total_q / e2e_s, "unit": "queries/s", "h2d_bytes_per_step": h2d,
-                "d2h_bytes_per_step": d2h, "entry_point": "skip_retrieve_host (pinned host buffers)"},
+                "d2h_bytes_per_step": d2h,
+                "entry_point": ("skip_retrieve_skv with pinned host copies in and out" if args.skv
+                                else "skip_retrieve_host (pinned host buffers)")},
         "gpu_launches": int(sum(v["launches"] for v in kernels.values())),
         "kernels": kernels,
         "plan": plan,
     }
+    if args.skv:
+        line["config"]["skv_gate"] = {"hidden": 512, "tau_nu": 0.5, "rho_r": 0.6}
+        H = 512
+        P = Q * spec.K
+        skv_flops = 2.0 * P * 3 * spec.d * H + 2.0 * Q * 2 * spec.d * H
+        skv_ms = sum(kernels[k]["ms"] / max(1, kernels[k]["launches"]) for k in kernels if k.startswith("skv_"))
+        mlp = kernels.get("skv_mlp", {"ms": float("nan"), "launches": 1})
+        mlp_ms = mlp["ms"] / max(1, mlp["launches"])
+        line["skv"] = {"gate_ms_per_step": skv_ms, "mlp_kernel_ms": mlp_ms,
+                       "mlp_algorithmic_flops": 2.0 * P * 3 * spec.d * H,
+                       "mlp_tflops": 2.0 * P * 3 * spec.d * H / (mlp_ms / 1e3) / 1e12,
+                       "gate_share_of_step": skv_ms / (ms / args.steps), "algorithmic_flops": skv_flops}
     if keep_host:
         line["cpu_baseline"] = cpu_baseline(spec, corpus_np, scale_np, regions, offsets, args.cpu_questions)
     c.free()

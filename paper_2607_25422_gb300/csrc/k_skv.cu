@@ -2,7 +2,7 @@
 // and the TopK after it) on the merged retrieval lists.
 //
 //  k_skv_qbias   per question: c_q = b1 + W1[:, qbar] qbar + W1[:, vbar] vbar
-//                (fp32, one warp per hidden unit, W1 row slice in registers).
+//                (fp32 on the CUDA cores; a warp per unit and 8 questions).
 //  k_skv_mlp     per 128 passage slots x 128 hidden units: the passage part
 //                of layer 1 on the tensor cores.  The A operand is built in
 //                shared memory by four warps from the gathered corpus rows
@@ -247,42 +247,74 @@ __global__ void __launch_bounds__(kSkvThreads, 1)
     }
 }
 
-// c[q][i] = b1[i] + sum_t W1[i][t] qbar[q][t] + sum_t W1[i][d + t] vbar[q][t]:
-// one warp per hidden unit i, its 2d weights held in registers (d <= 1024),
-// questions in turn.
-__global__ void __launch_bounds__(128) k_skv_qbias(const SkvParams p) {
+// c[q][i] = b1[i] + sum_t W1[i][t] qbar[q][t] + sum_t W1[i][d + t] vbar[q][t].
+// A block covers four hidden units (one per warp) and eight questions.  The
+// eight questions' [qbar | vbar] are first staged in shared memory by the
+// whole block (independent loads, all in flight at once); each warp reads its
+// unit's 2d weights once, coalesced, into registers (lane l holds 16-byte
+// words l, l + 32, ...) and reduces each of the eight dots across the warp.
+constexpr int kBiasWarps = 4, kBiasQs = 8;
+__global__ void __launch_bounds__(32 * kBiasWarps) k_skv_qbias(const SkvParams p) {
+    __shared__ uint4 xs[kBiasQs][256];  // [question][16-byte word of qbar | vbar], d <= 1024
     const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
-    const int i = blockIdx.x * 4 + warp;
-    if (i >= p.H) return;
-    const int nv = (2 * p.d) / 8;  // 16-byte words in the row slice [qbar | vbar]
-    const int nq = p.d / 8;
-    const uint4 *wrow = reinterpret_cast<const uint4 *>(p.w1 + (int64_t)i * 5 * p.d);
+    const int i = blockIdx.x * kBiasWarps + warp;
+    const int q0 = blockIdx.y * kBiasQs;
+    const int nq = p.d / 8;  // 16-byte words per d-vector
+    const int nv = 2 * nq;   // words of [qbar | vbar]
+    // All of a thread's staging loads are issued before any is stored.
+    constexpr int kPer = kBiasQs * 256 / (32 * kBiasWarps);
+    uint4 xr[kPer];
+#pragma unroll
+    for (int r = 0; r < kPer; ++r) {
+        const int idx = threadIdx.x + r * 32 * kBiasWarps;
+        const int u = idx / nv, k = idx - u * nv, q = q0 + u;
+        xr[r] = make_uint4(0, 0, 0, 0);
+        if (idx < kBiasQs * nv && q < p.Q)
+            xr[r] = k < nq ? __ldg(reinterpret_cast<const uint4 *>(p.qbar + (int64_t)q * p.d) + k)
+                           : __ldg(reinterpret_cast<const uint4 *>(p.vbar + (int64_t)q * p.d) + (k - nq));
+    }
+#pragma unroll
+    for (int r = 0; r < kPer; ++r) {
+        const int idx = threadIdx.x + r * 32 * kBiasWarps;
+        if (idx < kBiasQs * nv) xs[idx / nv][idx % nv] = xr[r];
+    }
     uint4 w[8];
+    const uint4 *wrow = reinterpret_cast<const uint4 *>(p.w1 + (int64_t)min(i, p.H - 1) * 5 * p.d);
 #pragma unroll
     for (int t = 0; t < 8; ++t) w[t] = (lane + 32 * t < nv) ? __ldg(wrow + lane + 32 * t) : make_uint4(0, 0, 0, 0);
-    const float b = p.b1[i];
-    for (int q = 0; q < p.Q; ++q) {
-        const uint4 *qrow = reinterpret_cast<const uint4 *>(p.qbar + (int64_t)q * p.d);
-        const uint4 *vrow = reinterpret_cast<const uint4 *>(p.vbar + (int64_t)q * p.d);
-        float acc = 0.f;
+    __syncthreads();
+    if (i >= p.H) return;
+    float acc[kBiasQs];
+#pragma unroll
+    for (int u = 0; u < kBiasQs; ++u) {
+        acc[u] = 0.f;
 #pragma unroll
         for (int t = 0; t < 8; ++t) {
             const int k = lane + 32 * t;
-            if (k >= nv) break;
-            const uint4 x = k < nq ? __ldg(qrow + k) : __ldg(vrow + (k - nq));
-            const uint32_t wv[4] = {w[t].x, w[t].y, w[t].z, w[t].w};
-            const uint32_t xv[4] = {x.x, x.y, x.z, x.w};
+            if (k < nv) {
+                const uint4 x = xs[u][k];
+                const uint32_t wv[4] = {w[t].x, w[t].y, w[t].z, w[t].w};
+                const uint32_t xw[4] = {x.x, x.y, x.z, x.w};
 #pragma unroll
-            for (int h = 0; h < 4; ++h) {
-                const float2 wf = __bfloat1622float2(*reinterpret_cast<const __nv_bfloat162 *>(&wv[h]));
-                const float2 xf = __bfloat1622float2(*reinterpret_cast<const __nv_bfloat162 *>(&xv[h]));
-                acc = fmaf(wf.x, xf.x, acc);
-                acc = fmaf(wf.y, xf.y, acc);
+                for (int h = 0; h < 4; ++h) {
+                    const float2 wf = __bfloat1622float2(*reinterpret_cast<const __nv_bfloat162 *>(&wv[h]));
+                    const float2 xf = __bfloat1622float2(*reinterpret_cast<const __nv_bfloat162 *>(&xw[h]));
+                    acc[u] = fmaf(wf.x, xf.x, acc[u]);
+                    acc[u] = fmaf(wf.y, xf.y, acc[u]);
+                }
             }
         }
+    }
 #pragma unroll
-        for (int o = 16; o; o >>= 1) acc += __shfl_xor_sync(0xFFFFFFFFu, acc, o);
-        if (lane == 0) p.cq[(int64_t)q * p.H + i] = acc + b;
+    for (int u = 0; u < kBiasQs; ++u)
+#pragma unroll
+        for (int o = 16; o; o >>= 1) acc[u] += __shfl_xor_sync(0xFFFFFFFFu, acc[u], o);
+    if (lane < kBiasQs && q0 + lane < p.Q) {
+        float v = acc[0];
+#pragma unroll
+        for (int u = 1; u < kBiasQs; ++u)
+            if (lane == u) v = acc[u];
+        p.cq[(int64_t)(q0 + lane) * p.H + i] = v + p.b1[i];
     }
 }
 
@@ -364,18 +396,25 @@ size_t skv_mlp_smem_bytes() {
     return 1024 + (size_t)kSkvStages * (kSkvStageA + kSkvStageB) + sizeof(SkvShared);
 }
 
-cudaError_t launch_skv(const CUtensorMap &tw, const SkvParams &p, cudaStream_t s) {
+cudaError_t launch_skv_qbias(const SkvParams &p, cudaStream_t s) {
     if (p.Q == 0) return cudaSuccess;
-    k_skv_qbias<<<(p.H + 3) / 4, 128, 0, s>>>(p);
-    cudaError_t e = cudaGetLastError();
-    if (e != cudaSuccess) return e;
+    dim3 grid((unsigned)((p.H + kBiasWarps - 1) / kBiasWarps), (unsigned)((p.Q + kBiasQs - 1) / kBiasQs));
+    k_skv_qbias<<<grid, 32 * kBiasWarps, 0, s>>>(p);
+    return cudaGetLastError();
+}
+
+cudaError_t launch_skv_mlp(const CUtensorMap &tw, const SkvParams &p, cudaStream_t s) {
+    if (p.Q == 0) return cudaSuccess;
     const size_t smem = skv_mlp_smem_bytes();
-    e = cudaFuncSetAttribute(k_skv_mlp, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
+    cudaError_t e = cudaFuncSetAttribute(k_skv_mlp, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
     if (e != cudaSuccess) return e;
     dim3 grid((unsigned)((p.P + kSkvRows - 1) / kSkvRows), (unsigned)(p.H / kSkvHidden));
     k_skv_mlp<<<grid, kSkvThreads, smem, s>>>(tw, p);
-    e = cudaGetLastError();
-    if (e != cudaSuccess) return e;
+    return cudaGetLastError();
+}
+
+cudaError_t launch_skv_select(const SkvParams &p, cudaStream_t s) {
+    if (p.Q == 0) return cudaSuccess;
     k_skv_select<<<p.Q, kSelThreads, 0, s>>>(p);
     return cudaGetLastError();
 }

@@ -567,8 +567,14 @@ skip_status_t skv_impl(skip_corpus *c, const int64_t *cand_ids, int32_t Q, int32
     p.nu_all = nu_all;
     p.err = c->err;
     p.timeout_ns = c->timeout_ns;
-    record(c, s, "skv_gate");
-    cudaError_t e = launch_skv(tw, p, s);
+    record(c, s, "skv_qbias");
+    cudaError_t e = launch_skv_qbias(p, s);
+    if (e != cudaSuccess) return cuda_status(e);
+    record(c, s, "skv_mlp");
+    e = launch_skv_mlp(tw, p, s);
+    if (e != cudaSuccess) return cuda_status(e);
+    record(c, s, "skv_select");
+    e = launch_skv_select(p, s);
     if (e != cudaSuccess) return cuda_status(e);
     pl.launches += 3;
     return SKIP_OK;

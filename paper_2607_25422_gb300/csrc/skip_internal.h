@@ -134,7 +134,11 @@ struct SkvParams {
     uint64_t timeout_ns;
 };
 size_t skv_mlp_smem_bytes();
+// The gate in three launches: per-question bias, the tensor-core layer 1 +
+// ReLU + w2 partial dots, and the sigmoid / gate / selection.
 // tw: tensor map over W1 [H x 5d] bf16, box 64 columns x 128 rows, 128-byte swizzle.
-cudaError_t launch_skv(const CUtensorMap &tw, const SkvParams &p, cudaStream_t s);
+cudaError_t launch_skv_qbias(const SkvParams &p, cudaStream_t s);
+cudaError_t launch_skv_mlp(const CUtensorMap &tw, const SkvParams &p, cudaStream_t s);
+cudaError_t launch_skv_select(const SkvParams &p, cudaStream_t s);
 
 }  // namespace skipk
