@@ -20,6 +20,10 @@ Functions and what they follow:
   nu_j >= tau, the best ceil(rho |K|) by (nu desc, id asc)
   (``skv_oracle.c``).
 * ``bf16_round``   -- a double rounded to bf16 (ties to even), as bits.
+* ``ivf_assign``, ``pq_encode``, ``ivfpq_build``, ``ivfpq_search``,
+  ``ivfpq_scores_at`` -- the IVF-PQ index (§4.1 "Implementation", App. I.4;
+  the published inverted file with product-quantised residuals and
+  asymmetric inner-product scoring) and its search (``ivfpq_oracle.c``).
 """
 from __future__ import annotations
 
@@ -30,7 +34,8 @@ import subprocess
 import numpy as np
 
 _HERE = os.path.dirname(os.path.abspath(__file__))
-_SRCS = [os.path.join(_HERE, "rcsr_oracle.c"), os.path.join(_HERE, "skv_oracle.c")]
+_SRCS = [os.path.join(_HERE, "rcsr_oracle.c"), os.path.join(_HERE, "skv_oracle.c"),
+         os.path.join(_HERE, "ivfpq_oracle.c")]
 _OUT = os.path.join(_HERE, "_build", "libskip_oracle.so")
 _lib = None
 
@@ -70,6 +75,13 @@ def _load():
     lib.skip_oracle_skv_count.argtypes = [i32, ctypes.c_double]
     lib.skip_oracle_bf16_round.argtypes = [ctypes.c_double]
     lib.skip_oracle_bf16_round.restype = ctypes.c_uint16
+    lib.skip_oracle_ivf_assign.argtypes = [P, i64, i32, P, i32, P]
+    lib.skip_oracle_pq_encode.argtypes = [P, i64, i32, P, P, P, i32, i32, P]
+    lib.skip_oracle_ivfpq_search.argtypes = [P, i32, i32, P, P, P, P, i32, i32, P, i32, i32, i32, P, P, P]
+    lib.skip_oracle_ivfpq_scores_at.argtypes = [P, i32, P, P, i64, P, i32, i32, P, P, P, i64, P]
+    for f in ("skip_oracle_ivf_assign", "skip_oracle_pq_encode", "skip_oracle_ivfpq_search",
+              "skip_oracle_ivfpq_scores_at"):
+        getattr(lib, f).restype = ctypes.c_int
     for f in ("skip_oracle_region_topk", "skip_oracle_merge", "skip_oracle_retrieve", "skip_oracle_skv",
               "skip_oracle_skv_count",
               "skip_oracle_score_matrix", "skip_oracle_scores_at", "skip_oracle_threads"):
@@ -238,3 +250,92 @@ def skv(corpus, ids, qbar, vbar, w1, b1, w2, b2, tau=0.5, rho=0.6):
     if rc:
         raise RuntimeError("oracle skv failed (%d)" % rc)
     return {"nu_all": nu_all, "bound": bound, "ids": out_ids, "nu": out_nu, "count": count}
+
+
+def ivf_assign(corpus, centroids):
+    """list(i) = argmax_l <x_i, c_l> (ties: lower l); int32 [N]."""
+    lib = _load()
+    corpus = np.ascontiguousarray(corpus, dtype=np.uint16)
+    centroids = np.ascontiguousarray(centroids, dtype=np.uint16)
+    N, d = corpus.shape
+    out = np.empty(N, np.int32)
+    if lib.skip_oracle_ivf_assign(_ptr(corpus), N, d, _ptr(centroids), centroids.shape[0], _ptr(out)):
+        raise RuntimeError("oracle ivf_assign failed")
+    return out
+
+
+def pq_encode(corpus, centroids, lists, codebook):
+    """PQ codes of the residuals x_i - c_list(i): uint8 [N, M]; codebook
+    float32 [M, ksub, d/M] (ties: lower codeword)."""
+    lib = _load()
+    corpus = np.ascontiguousarray(corpus, dtype=np.uint16)
+    centroids = np.ascontiguousarray(centroids, dtype=np.uint16)
+    lists = np.ascontiguousarray(lists, dtype=np.int32)
+    codebook = np.ascontiguousarray(codebook, dtype=np.float32)
+    N, d = corpus.shape
+    M, ksub = codebook.shape[0], codebook.shape[1]
+    out = np.empty((N, M), np.uint8)
+    if lib.skip_oracle_pq_encode(_ptr(corpus), N, d, _ptr(centroids), _ptr(lists), _ptr(codebook), M, ksub,
+                                 _ptr(out)):
+        raise RuntimeError("oracle pq_encode failed")
+    return out
+
+
+def ivf_lists(lists, C):
+    """Inverted lists: (offsets int64 [C+1], ids int64 [N] grouped by list,
+    ascending within a list)."""
+    lists = np.asarray(lists, np.int64)
+    ids = np.argsort(lists, kind="stable").astype(np.int64)
+    counts = np.bincount(lists, minlength=C)
+    offsets = np.zeros(C + 1, np.int64)
+    offsets[1:] = np.cumsum(counts)
+    return offsets, ids
+
+
+def ivfpq_build(corpus, centroids, codebook):
+    """The whole index: dict(lists, codes, offsets, ids)."""
+    lists = ivf_assign(corpus, centroids)
+    codes = pq_encode(corpus, centroids, lists, codebook)
+    offsets, ids = ivf_lists(lists, np.asarray(centroids).shape[0])
+    return {"lists": lists, "codes": codes, "offsets": offsets, "ids": ids}
+
+
+def ivfpq_search(index, centroids, codebook, regions, nprobe, k):
+    """(ids int64 [R, k], scores float64 [R, k], probes int32 [R, nprobe])."""
+    lib = _load()
+    centroids = np.ascontiguousarray(centroids, dtype=np.uint16)
+    codebook = np.ascontiguousarray(codebook, dtype=np.float32)
+    regions = np.ascontiguousarray(regions, dtype=np.uint16)
+    offsets = np.ascontiguousarray(index["offsets"], dtype=np.int64)
+    ids = np.ascontiguousarray(index["ids"], dtype=np.int64)
+    codes = np.ascontiguousarray(index["codes"], dtype=np.uint8)
+    C, d = centroids.shape
+    M, ksub = codebook.shape[0], codebook.shape[1]
+    R = regions.shape[0]
+    out_ids = np.empty((R, k), np.int64)
+    out_sc = np.empty((R, k), np.float64)
+    probes = np.empty((R, nprobe), np.int32)
+    if lib.skip_oracle_ivfpq_search(_ptr(centroids), C, d, _ptr(offsets), _ptr(ids), _ptr(codes), _ptr(codebook),
+                                    M, ksub, _ptr(regions), R, int(nprobe), int(k), _ptr(out_ids), _ptr(out_sc),
+                                    _ptr(probes)):
+        raise RuntimeError("oracle ivfpq_search failed")
+    return out_ids, out_sc, probes
+
+
+def ivfpq_scores_at(index, centroids, codebook, regions, region_idx, ids):
+    """s^(q_r, i) at chosen (region, id) pairs (NaN outside [0, N))."""
+    lib = _load()
+    centroids = np.ascontiguousarray(centroids, dtype=np.uint16)
+    codebook = np.ascontiguousarray(codebook, dtype=np.float32)
+    regions = np.ascontiguousarray(regions, dtype=np.uint16)
+    lists = np.ascontiguousarray(index["lists"], dtype=np.int32)
+    codes = np.ascontiguousarray(index["codes"], dtype=np.uint8)
+    region_idx = np.ascontiguousarray(region_idx, dtype=np.int64).ravel()
+    ids = np.ascontiguousarray(ids, dtype=np.int64).ravel()
+    M, ksub = codebook.shape[0], codebook.shape[1]
+    out = np.empty(ids.shape[0], np.float64)
+    if lib.skip_oracle_ivfpq_scores_at(_ptr(centroids), centroids.shape[1], _ptr(lists), _ptr(codes),
+                                       lists.shape[0], _ptr(codebook), M, ksub, _ptr(regions), _ptr(region_idx),
+                                       _ptr(ids), ids.shape[0], _ptr(out)):
+        raise RuntimeError("oracle ivfpq_scores_at failed")
+    return out

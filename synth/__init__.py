@@ -111,10 +111,12 @@ def draw_centres(spec_or_seed, C: int, d: int, device="cpu") -> torch.Tensor:
 
 
 def corpus_rows_fp32(seed: int, n0: int, n: int, d: int, kind: str,
-                     centres: Optional[torch.Tensor], device="cpu") -> torch.Tensor:
+                     centres: Optional[torch.Tensor], device="cpu", return_centres: bool = False):
     """fp32 unit rows [n0, n0 + n) of a corpus; n0 must be a multiple of CHUNK
-    unless the whole draw lies in one chunk."""
+    unless the whole draw lies in one chunk.  With return_centres (clustered
+    corpora), also the index of the centre each row was drawn around."""
     out = torch.empty(n, d, dtype=torch.float32, device=device)
+    which = torch.full((n,), -1, dtype=torch.int64, device=device)
     done = 0
     while done < n:
         row = n0 + done
@@ -129,11 +131,12 @@ def corpus_rows_fp32(seed: int, n0: int, n: int, d: int, kind: str,
             a = torch.randint(0, C, (off + take,), generator=g, device=device)[off:]
             z = torch.randn(off + take, d, generator=g, device=device, dtype=torch.float32)[off:]
             x = centres[a] + (0.3 / math.sqrt(d)) * z
+            which[done:done + take] = a
         else:
             raise ValueError(kind)
         out[done:done + take] = _normalise(x)
         done += take
-    return out
+    return (out, which) if return_centres else out
 
 
 def quantise_e4m3(x: torch.Tensor):
@@ -283,3 +286,36 @@ def make_candidate_ids(N: int, Q: int, K: int, empty, seed: int) -> torch.Tensor
         if n > 0:
             out[q, :n] = torch.randperm(N, generator=g)[:n]
     return out
+
+
+
+# ---- inputs of the IVF-PQ variant ----------------------------------------
+#
+# The paper's index (FAISS IVF-PQ, 1,024 or 4,096 centroids, PQ64) was
+# trained on its corpus; no trained index exists here.  For the clustered
+# workloads the IVF centroids are the generator's own centres (1,024 for the
+# 1M and 10M corpora, 4,096 for the 20M one), as bf16.  The PQ codebook is
+# sample-based: codeword j of sub-space m is sub-vector m of the residual
+# bf16(x_i) - bf16(c_{a_i}) of corpus row i = m * ksub + j, where a_i is the
+# centre the generator drew row i around (no k-means refinement).
+
+def make_ivf_centroids(spec: WorkloadSpec, device="cpu") -> torch.Tensor:
+    """bf16 [C, d]: the clustered corpus's centres."""
+    if spec.corpus != "clustered":
+        raise ValueError("IVF centroids are drawn for clustered corpora")
+    return draw_centres(spec, spec.centres, spec.d, device).to(torch.bfloat16)
+
+
+def make_pq_codebook(spec: WorkloadSpec, M: int, ksub: int = 256, device="cpu") -> torch.Tensor:
+    """float32 [M, ksub, d / M] sample-based PQ codebook (see above)."""
+    if spec.d % M:
+        raise ValueError("M must divide d")
+    centres = draw_centres(spec, spec.centres, spec.d, "cpu")
+    n = M * ksub
+    x, a = corpus_rows_fp32(spec.index, 0, n, spec.d, spec.corpus, centres, "cpu", return_centres=True)
+    r = x.to(torch.bfloat16).float() - centres[a].to(torch.bfloat16).float()
+    ds = spec.d // M
+    cb = torch.empty(M, ksub, ds)
+    for m in range(M):
+        cb[m] = r[m * ksub:(m + 1) * ksub, m * ds:(m + 1) * ds]
+    return cb.to(device)

@@ -16,7 +16,10 @@ def read_fixture(name):
         key = parts[0]
         if len(parts) == 2 and key in ("corpus", "regions", "region_ids", "region_scores",
                                        "merged_ids", "merged_scores", "skv_corpus", "w1", "qbar",
-                                       "vbar", "ids", "nu_all", "out_ids", "out_nu"):
+                                       "vbar", "ids", "nu_all", "out_ids", "out_nu", "centroids",
+                                       "codebook", "ivf_corpus", "queries", "codes", "p1k2_ids",
+                                       "p1k2_scores", "p1k4_ids", "p1k4_scores", "p2k3_ids",
+                                       "p2k3_scores"):
             n = int(parts[1])
             rows = [[float(v) for v in lines[i + 1 + t].split()] for t in range(n)]
             out[key] = np.array(rows, dtype=np.float64)
