@@ -13,7 +13,8 @@ top-k_region ids are kept per region, and each question's region lists are
 merged into a deduplicated top-K (max score per id, ties to the lower id).
 The SKV passage gate (App. B.4 Def. B.4; ``include/skip_skv.h``) then keeps
 the passages whose verification score nu reaches tau, at most
-ceil(rho |K|) of them.
+ceil(rho |K|) of them.  The IVF-PQ variant (``include/skip_ivfpq.h``) builds
+and searches an inverted-file, product-quantised index of the corpus.
 """
 from __future__ import annotations
 
@@ -71,11 +72,25 @@ def load_library():
                                   ctypes.c_float, P, P, P, P, P]
     lib.skip_retrieve_skv.argtypes = [P, P, P, i32, i32, i32, i32, P, P, ctypes.POINTER(SkvMlp), ctypes.c_float,
                                       ctypes.c_float, P, P, P, P, P, P]
+    lib.skip_ivfpq_build.argtypes = [P, P, i32, P, i32, P, ctypes.POINTER(P)]
+    lib.skip_ivfpq_load.argtypes = [P, i32, i32, P, i32, P, P, P, i64, P, ctypes.POINTER(P)]
+    lib.skip_ivfpq_lists.argtypes = [P, P, P, P, P]
+    lib.skip_ivfpq_info.argtypes = [P, ctypes.POINTER(i64), ctypes.POINTER(i32), ctypes.POINTER(i32),
+                                    ctypes.POINTER(i32)]
+    lib.skip_ivfpq_free.argtypes = [P]
+    lib.skip_ivfpq_search_regions.argtypes = [P, P, i32, i32, i32, P, P, P]
+    lib.skip_ivfpq_search.argtypes = [P, P, P, i32, i32, i32, i32, i32, P, P, P]
+    lib.skip_ivfpq_sync_status.argtypes = [P, P]
+    lib.skip_ivfpq_set_option.argtypes = [P, ctypes.c_int, i64]
+    lib.skip_ivfpq_timing_report.argtypes = [P, ctypes.c_char_p, i32]
     lib.skip_status_string.argtypes = [ctypes.c_int]
     lib.skip_status_string.restype = ctypes.c_char_p
     for f in ("skip_corpus_load", "skip_corpus_free", "skip_corpus_set_option", "skip_retrieve",
               "skip_retrieve_regions", "skip_retrieve_host", "skip_sync_status", "skip_last_plan",
-              "skip_timing_report", "skip_retrieve_regions_noalloc", "skip_skv_gate", "skip_retrieve_skv"):
+              "skip_timing_report", "skip_retrieve_regions_noalloc", "skip_skv_gate", "skip_retrieve_skv",
+              "skip_ivfpq_build", "skip_ivfpq_load", "skip_ivfpq_lists", "skip_ivfpq_info", "skip_ivfpq_free",
+              "skip_ivfpq_search_regions", "skip_ivfpq_search", "skip_ivfpq_sync_status", "skip_ivfpq_set_option",
+              "skip_ivfpq_timing_report"):
         getattr(lib, f).restype = ctypes.c_int
     _lib = lib
     return lib
@@ -297,6 +312,110 @@ def skip_retrieve_skv(corpus: Corpus, regions: torch.Tensor, region_offsets: tor
     return (out_ids, out_nu, count, m_ids, m_sc) if with_merged else (out_ids, out_nu, count)
 
 
+class IvfIndex:
+    """An IVF-PQ index handle (``skip_ivfpq_t``)."""
+
+    def __init__(self, handle):
+        self.handle = handle
+        lib = load_library()
+        N, d, C, M = ctypes.c_int64(), ctypes.c_int32(), ctypes.c_int32(), ctypes.c_int32()
+        _check(lib.skip_ivfpq_info(handle, ctypes.byref(N), ctypes.byref(d), ctypes.byref(C), ctypes.byref(M)),
+               "skip_ivfpq_info")
+        self.N, self.d, self.C, self.M = N.value, d.value, C.value, M.value
+
+    def free(self):
+        if self.handle:
+            load_library().skip_ivfpq_free(self.handle)
+            self.handle = None
+
+    def __del__(self):
+        try:
+            self.free()
+        except Exception:
+            pass
+
+    def set_option(self, option: int, value: int):
+        _check(load_library().skip_ivfpq_set_option(self.handle, int(option), int(value)), "skip_ivfpq_set_option")
+
+
+def skip_ivfpq_build(corpus: Corpus, centroids: torch.Tensor, codebook: torch.Tensor, stream=None) -> IvfIndex:
+    """Index of a loaded bf16 corpus: centroids bf16 [C, d], codebook float32
+    [M, 256, d / M] (device tensors)."""
+    lib = load_library()
+    centroids, codebook = centroids.contiguous(), codebook.to(torch.float32).contiguous()
+    h = ctypes.c_void_p()
+    st = lib.skip_ivfpq_build(corpus.handle, _ptr(centroids), centroids.shape[0], _ptr(codebook), codebook.shape[0],
+                              ctypes.c_void_p(_stream(stream)), ctypes.byref(h))
+    _check(st, "skip_ivfpq_build")
+    return IvfIndex(h)
+
+
+def skip_ivfpq_load(centroids: torch.Tensor, codebook: torch.Tensor, list_offsets: torch.Tensor, ids: torch.Tensor,
+                    codes: torch.Tensor, stream=None) -> IvfIndex:
+    """Index from device arrays: offsets int64 [C + 1], ids int32 [N] and codes
+    uint8 [N, M] in list order."""
+    lib = load_library()
+    centroids, codebook = centroids.contiguous(), codebook.to(torch.float32).contiguous()
+    list_offsets = list_offsets.to(torch.int64).contiguous()
+    ids, codes = ids.to(torch.int32).contiguous(), codes.to(torch.uint8).contiguous()
+    h = ctypes.c_void_p()
+    st = lib.skip_ivfpq_load(_ptr(centroids), centroids.shape[0], centroids.shape[1], _ptr(codebook), codebook.shape[0],
+                             _ptr(list_offsets), _ptr(ids), _ptr(codes), ids.shape[0],
+                             ctypes.c_void_p(_stream(stream)), ctypes.byref(h))
+    _check(st, "skip_ivfpq_load")
+    return IvfIndex(h)
+
+
+def skip_ivfpq_lists(index: IvfIndex, device=None, stream=None):
+    """(offsets int64 [C + 1], ids int32 [N], codes uint8 [N, M]) on the device."""
+    device = device or torch.device("cuda", torch.cuda.current_device())
+    off = torch.empty(index.C + 1, dtype=torch.int64, device=device)
+    ids = torch.empty(index.N, dtype=torch.int32, device=device)
+    codes = torch.empty(index.N, index.M, dtype=torch.uint8, device=device)
+    _check(load_library().skip_ivfpq_lists(index.handle, _ptr(off), _ptr(ids), _ptr(codes),
+                                          ctypes.c_void_p(_stream(stream))), "skip_ivfpq_lists")
+    return off, ids, codes
+
+
+def skip_ivfpq_search_regions(index: IvfIndex, regions: torch.Tensor, nprobe: int, k_region: int, stream=None):
+    """Per region: (ids int64 [R, k], scores fp32 [R, k])."""
+    regions = regions.contiguous()
+    R = regions.shape[0]
+    ids = torch.empty(R, k_region, dtype=torch.int64, device=regions.device)
+    sc = torch.empty(R, k_region, dtype=torch.float32, device=regions.device)
+    _check(load_library().skip_ivfpq_search_regions(index.handle, _ptr(regions), R, int(nprobe), int(k_region),
+                                                    _ptr(ids), _ptr(sc), ctypes.c_void_p(_stream(stream))),
+           "skip_ivfpq_search_regions")
+    return ids, sc
+
+
+def skip_ivfpq_search(index: IvfIndex, regions: torch.Tensor, region_offsets: torch.Tensor, nprobe: int,
+                      k_region: int, K: int, out_ids: Optional[torch.Tensor] = None,
+                      out_scores: Optional[torch.Tensor] = None, stream=None):
+    """Per region, then per question: (ids int64 [Q, K], scores fp32 [Q, K])."""
+    regions = regions.contiguous()
+    offs = region_offsets.to(device=regions.device, dtype=torch.int32).contiguous()
+    Q = offs.numel() - 1
+    if out_ids is None:
+        out_ids = torch.empty(Q, K, dtype=torch.int64, device=regions.device)
+    if out_scores is None:
+        out_scores = torch.empty(Q, K, dtype=torch.float32, device=regions.device)
+    _check(load_library().skip_ivfpq_search(index.handle, _ptr(regions), _ptr(offs), Q, regions.shape[0], int(nprobe),
+                                            int(k_region), int(K), _ptr(out_ids), _ptr(out_scores),
+                                            ctypes.c_void_p(_stream(stream))), "skip_ivfpq_search")
+    return out_ids, out_scores
+
+
+def skip_ivfpq_sync_status(index: IvfIndex, stream=None) -> int:
+    return int(load_library().skip_ivfpq_sync_status(index.handle, ctypes.c_void_p(_stream(stream))))
+
+
+def skip_ivfpq_timing_report(index: IvfIndex) -> dict:
+    buf = ctypes.create_string_buffer(1 << 16)
+    _check(load_library().skip_ivfpq_timing_report(index.handle, buf, 1 << 16), "skip_ivfpq_timing_report")
+    return json.loads(buf.value.decode())
+
+
 def skip_sync_status(corpus: Corpus, stream=None) -> int:
     """Synchronise and return the status latched by the kernels (SKIP_OK, ...)."""
     return int(load_library().skip_sync_status(corpus.handle, ctypes.c_void_p(_stream(stream))))
@@ -317,4 +436,4 @@ def skip_timing_report(corpus: Corpus) -> dict:
 
 
 __all__ = [n for n in dir() if n.startswith("skip_") or n.startswith("SKIP_")] + [
-    "Corpus", "SkipError", "SkvMlp", "load_library", "library_path"]
+    "Corpus", "SkipError", "SkvMlp", "IvfIndex", "load_library", "library_path"]

@@ -14,6 +14,7 @@
 
 #include "../../include/skip_retrieve.h"
 #include "../../include/skip_skv.h"
+#include "../../include/skip_ivfpq.h"
 #include "skip_internal.h"
 
 using namespace skipk;
@@ -890,6 +891,264 @@ skip_status_t skip_retrieve_skv(skip_corpus_t c, const void *regions, const int3
     record(c, s, "end");
     write_plan(c, pl, R_total, Q, k_region, K);
     return SKIP_OK;
+}
+
+}  // extern "C"
+
+// ---------------------------------------------------------------- IVF-PQ
+
+struct skip_ivfpq {
+    skip_corpus *cent = nullptr;  // the centroids as a searchable set (coarse step)
+    int64_t N = 0;
+    int d = 0, C = 0, M = 0, ds = 0;
+    float *codebook = nullptr;    // [M x 256 x ds]
+    int64_t *offsets = nullptr;   // [C + 1]
+    int32_t *ids = nullptr;       // [N] list order
+    uint8_t *codes = nullptr;     // [N x M] list order
+    void *ws = nullptr;           // search workspace
+    size_t ws_bytes = 0;
+};
+
+namespace {
+
+void ivf_release(skip_ivfpq *ix) {
+    if (!ix) return;
+    cudaDeviceSynchronize();
+    if (ix->cent) skip_corpus_free(ix->cent);
+    cudaFree(ix->codebook);
+    cudaFree(ix->offsets);
+    cudaFree(ix->ids);
+    cudaFree(ix->codes);
+    cudaFree(ix->ws);
+    delete ix;
+}
+
+// Allocates the index arrays and the centroid set; fills sizes.
+skip_status_t ivf_create(const void *centroids, int C, int d, const float *codebook, int M, int64_t N,
+                         cudaStream_t s, skip_ivfpq **out) {
+    auto *ix = new skip_ivfpq();
+    ix->N = N, ix->d = d, ix->C = C, ix->M = M, ix->ds = d / M;
+    skip_status_t st = skip_corpus_load(centroids, 1, C, d, SKIP_BF16, nullptr, s, &ix->cent);
+    if (st) {
+        ivf_release(ix);
+        return st;
+    }
+    const size_t cb = (size_t)M * 256 * ix->ds * sizeof(float);
+    if (cudaMalloc(&ix->codebook, cb) != cudaSuccess || cudaMalloc(&ix->offsets, (size_t)(C + 1) * 8) != cudaSuccess ||
+        cudaMalloc(&ix->ids, (size_t)std::max<int64_t>(N, 1) * 4) != cudaSuccess ||
+        cudaMalloc(&ix->codes, (size_t)std::max<int64_t>(N, 1) * M) != cudaSuccess) {
+        cudaGetLastError();
+        ivf_release(ix);
+        return SKIP_ENOMEM;
+    }
+    if (cudaMemcpyAsync(ix->codebook, codebook, cb, cudaMemcpyDeviceToDevice, s) != cudaSuccess) {
+        ivf_release(ix);
+        return SKIP_ECUDA;
+    }
+    *out = ix;
+    return SKIP_OK;
+}
+
+skip_status_t ivf_check_shape(int C, int d, int M) {
+    if (C < 1 || d < 1 || M < 1) return SKIP_EINVAL;
+    if (C > (1 << 20) || M % 16 != 0 || d % M != 0 || d / M > kIvfMaxDs) return SKIP_EUNSUPPORTED;
+    return SKIP_OK;
+}
+
+IvfParams ivf_params(const skip_ivfpq *ix) {
+    IvfParams p;
+    p.rows = nullptr;
+    p.N = ix->N;
+    p.d = ix->d;
+    p.centroids = ix->cent->rows;
+    p.C = ix->C;
+    p.codebook = ix->codebook;
+    p.M = ix->M;
+    p.ds = ix->ds;
+    p.offsets = ix->offsets;
+    p.ids = ix->ids;
+    p.codes = ix->codes;
+    return p;
+}
+
+// Coarse probes then the list scan: top-k keys per region into the head of
+// the index workspace.
+skip_status_t ivf_regions(skip_ivfpq *ix, const void *regions, int R, int nprobe, int k, cudaStream_t s,
+                          uint64_t **keys_out) {
+    const size_t pid = align_up((size_t)R * nprobe * 8, 256), psc = align_up((size_t)R * nprobe * 4, 256);
+    const size_t kb = align_up((size_t)std::max(R, 1) * k * 8, 256);
+    skip_status_t st = ensure_buf(ix->ws, ix->ws_bytes, kb + pid + psc);
+    if (st) return st;
+    uint64_t *keys = reinterpret_cast<uint64_t *>(ix->ws);
+    int64_t *probe_ids = reinterpret_cast<int64_t *>((char *)ix->ws + kb);
+    float *probe_sc = reinterpret_cast<float *>((char *)ix->ws + kb + pid);
+    *keys_out = keys;
+    if (R == 0) return SKIP_OK;
+    Plan pl;
+    st = run_regions(ix->cent, reinterpret_cast<const uint16_t *>(regions), R, nprobe, nullptr, probe_ids, probe_sc,
+                     s, pl, 0);
+    if (st) return st;
+    record(ix->cent, s, "ivfpq_scan");
+    cudaError_t e = launch_ivfpq_scan(ivf_params(ix), reinterpret_cast<const uint16_t *>(regions), R, probe_ids,
+                                      probe_sc, nprobe, k, keys, ix->cent->sm_count, s);
+    return cuda_status(e);
+}
+
+skip_status_t ivf_check_search(skip_ivfpq *ix, const void *regions, int R, int nprobe, int k) {
+    if (!ix || R < 0 || (R > 0 && !regions)) return SKIP_EINVAL;
+    if (nprobe < 1 || nprobe > std::min(ix->C, SKIP_MAX_K_REGION)) return SKIP_EINVAL;
+    if (k < 1 || k > SKIP_MAX_K_REGION) return SKIP_EINVAL;
+    return SKIP_OK;
+}
+
+}  // namespace
+
+extern "C" {
+
+skip_status_t skip_ivfpq_build(skip_corpus_t c, const void *centroids, int32_t C, const float *codebook, int32_t M,
+                               void *stream, skip_ivfpq_t *out) {
+    if (!c || !centroids || !codebook || !out) return SKIP_EINVAL;
+    skip_status_t st = ivf_check_shape(C, c->d, M);
+    if (st) return st;
+    if (c->dtype != SKIP_BF16) return SKIP_EUNSUPPORTED;
+    cudaStream_t s = reinterpret_cast<cudaStream_t>(stream);
+    skip_ivfpq *ix = nullptr;
+    st = ivf_create(centroids, C, c->d, codebook, M, c->N, s, &ix);
+    if (st) return st;
+    const int64_t N = c->N;
+    void *tmp = nullptr;
+    const size_t rl = align_up((size_t)N * 8, 256), rs = align_up((size_t)N * 4, 256);
+    const size_t cr = align_up((size_t)N * M, 256), cc = align_up((size_t)C * 8, 256);
+    if (cudaMalloc(&tmp, rl + rs + cr + 2 * cc) != cudaSuccess) {
+        cudaGetLastError();
+        ivf_release(ix);
+        return SKIP_ENOMEM;
+    }
+    int64_t *row_list = reinterpret_cast<int64_t *>(tmp);
+    float *row_score = reinterpret_cast<float *>((char *)tmp + rl);
+    uint8_t *codes_rows = reinterpret_cast<uint8_t *>((char *)tmp + rl + rs);
+    int64_t *counts = reinterpret_cast<int64_t *>((char *)tmp + rl + rs + cr);
+    int64_t *cursor = reinterpret_cast<int64_t *>((char *)tmp + rl + rs + cr + cc);
+    Plan pl;
+    st = run_regions(ix->cent, reinterpret_cast<const uint16_t *>(c->rows), (int)N, 1, nullptr, row_list, row_score,
+                     s, pl, 0);
+    IvfParams p = ivf_params(ix);
+    p.rows = c->rows;
+    if (!st) st = cuda_status(launch_pq_encode(p, row_list, codes_rows, s));
+    if (!st)
+        st = cuda_status(launch_ivf_lists(p, row_list, codes_rows, counts, cursor, ix->offsets, ix->ids, ix->codes,
+                                          ix->cent->err, ix->cent->sm_count, s));
+    if (!st) st = skip_sync_status(ix->cent, stream);
+    cudaFree(tmp);
+    if (st) {
+        ivf_release(ix);
+        return st;
+    }
+    *out = ix;
+    return SKIP_OK;
+}
+
+skip_status_t skip_ivfpq_load(const void *centroids, int32_t C, int32_t d, const float *codebook, int32_t M,
+                              const int64_t *list_offsets, const int32_t *ids, const uint8_t *codes, int64_t N,
+                              void *stream, skip_ivfpq_t *out) {
+    if (!centroids || !codebook || !list_offsets || !out || N < 0 || N >= ((int64_t)1 << 31)) return SKIP_EINVAL;
+    if (N > 0 && (!ids || !codes)) return SKIP_EINVAL;
+    if (d % 16 != 0) return SKIP_EINVAL;
+    skip_status_t st = ivf_check_shape(C, d, M);
+    if (st) return st;
+    cudaStream_t s = reinterpret_cast<cudaStream_t>(stream);
+    skip_ivfpq *ix = nullptr;
+    st = ivf_create(centroids, C, d, codebook, M, N, s, &ix);
+    if (st) return st;
+    if (cudaMemcpyAsync(ix->offsets, list_offsets, (size_t)(C + 1) * 8, cudaMemcpyDeviceToDevice, s) != cudaSuccess ||
+        (N > 0 && cudaMemcpyAsync(ix->ids, ids, (size_t)N * 4, cudaMemcpyDeviceToDevice, s) != cudaSuccess) ||
+        (N > 0 && cudaMemcpyAsync(ix->codes, codes, (size_t)N * M, cudaMemcpyDeviceToDevice, s) != cudaSuccess) ||
+        cudaStreamSynchronize(s) != cudaSuccess) {
+        ivf_release(ix);
+        return SKIP_ECUDA;
+    }
+    *out = ix;
+    return SKIP_OK;
+}
+
+skip_status_t skip_ivfpq_lists(skip_ivfpq_t ix, int64_t *list_offsets, int32_t *ids, uint8_t *codes, void *stream) {
+    if (!ix) return SKIP_EINVAL;
+    cudaStream_t s = reinterpret_cast<cudaStream_t>(stream);
+    if ((list_offsets && cudaMemcpyAsync(list_offsets, ix->offsets, (size_t)(ix->C + 1) * 8, cudaMemcpyDeviceToDevice,
+                                         s) != cudaSuccess) ||
+        (ids && ix->N > 0 && cudaMemcpyAsync(ids, ix->ids, (size_t)ix->N * 4, cudaMemcpyDeviceToDevice, s) != cudaSuccess) ||
+        (codes && ix->N > 0 &&
+         cudaMemcpyAsync(codes, ix->codes, (size_t)ix->N * ix->M, cudaMemcpyDeviceToDevice, s) != cudaSuccess) ||
+        cudaStreamSynchronize(s) != cudaSuccess)
+        return SKIP_ECUDA;
+    return SKIP_OK;
+}
+
+skip_status_t skip_ivfpq_info(skip_ivfpq_t ix, int64_t *N, int32_t *d, int32_t *C, int32_t *M) {
+    if (!ix) return SKIP_EINVAL;
+    if (N) *N = ix->N;
+    if (d) *d = ix->d;
+    if (C) *C = ix->C;
+    if (M) *M = ix->M;
+    return SKIP_OK;
+}
+
+skip_status_t skip_ivfpq_free(skip_ivfpq_t ix) {
+    ivf_release(ix);
+    return SKIP_OK;
+}
+
+skip_status_t skip_ivfpq_search_regions(skip_ivfpq_t ix, const void *regions, int32_t R_total, int32_t nprobe,
+                                        int32_t k_region, int64_t *reg_ids, float *reg_scores, void *stream) {
+    skip_status_t st = ivf_check_search(ix, regions, R_total, nprobe, k_region);
+    if (st) return st;
+    if (R_total > 0 && (!reg_ids || !reg_scores)) return SKIP_EINVAL;
+    cudaStream_t s = reinterpret_cast<cudaStream_t>(stream);
+    ++ix->cent->call_id;
+    uint64_t *keys = nullptr;
+    st = ivf_regions(ix, regions, R_total, nprobe, k_region, s, &keys);
+    if (st || R_total == 0) return st;
+    record(ix->cent, s, "merge_lists");
+    st = cuda_status(launch_merge_lists(keys, 1, (int64_t)R_total * k_region, R_total, k_region, nullptr, reg_ids,
+                                        reg_scores, s));
+    record(ix->cent, s, "end");
+    return st;
+}
+
+skip_status_t skip_ivfpq_search(skip_ivfpq_t ix, const void *regions, const int32_t *region_offsets, int32_t Q,
+                                int32_t R_total, int32_t nprobe, int32_t k_region, int32_t K, int64_t *out_ids,
+                                float *out_scores, void *stream) {
+    skip_status_t st = ivf_check_search(ix, regions, R_total, nprobe, k_region);
+    if (st) return st;
+    if (Q < 0 || K < 1 || K > SKIP_MAX_K || (Q > 0 && (!region_offsets || !out_ids || !out_scores))) return SKIP_EINVAL;
+    if (Q == 0 && R_total != 0) return SKIP_EINVAL;
+    cudaStream_t s = reinterpret_cast<cudaStream_t>(stream);
+    ++ix->cent->call_id;
+    uint64_t *keys = nullptr;
+    st = ivf_regions(ix, regions, R_total, nprobe, k_region, s, &keys);
+    if (st) return st;
+    if (Q > 0) {
+        record(ix->cent, s, "question_merge");
+        st = cuda_status(launch_question_merge(keys, k_region, region_offsets, Q, R_total, K, out_ids, out_scores,
+                                               ix->cent->err, s));
+    }
+    record(ix->cent, s, "end");
+    return st;
+}
+
+skip_status_t skip_ivfpq_sync_status(skip_ivfpq_t ix, void *stream) {
+    if (!ix) return SKIP_EINVAL;
+    return skip_sync_status(ix->cent, stream);
+}
+
+skip_status_t skip_ivfpq_set_option(skip_ivfpq_t ix, int option, int64_t value) {
+    if (!ix) return SKIP_EINVAL;
+    return skip_corpus_set_option(ix->cent, option, value);
+}
+
+skip_status_t skip_ivfpq_timing_report(skip_ivfpq_t ix, char *buf, int32_t len) {
+    if (!ix) return SKIP_EINVAL;
+    return skip_timing_report(ix->cent, buf, len);
 }
 
 }  // extern "C"

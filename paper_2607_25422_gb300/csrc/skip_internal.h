@@ -141,4 +141,30 @@ cudaError_t launch_skv_qbias(const SkvParams &p, cudaStream_t s);
 cudaError_t launch_skv_mlp(const CUtensorMap &tw, const SkvParams &p, cudaStream_t s);
 cudaError_t launch_skv_select(const SkvParams &p, cudaStream_t s);
 
+// ---- IVF-PQ variant (k_ivfpq.cu) ------------------------------------------
+constexpr int kIvfMaxDs = 32;  // largest sub-space width d / M
+struct IvfParams {
+    const void *rows;       // bf16 corpus [N x d] (build only)
+    int64_t N;
+    int d;
+    const void *centroids;  // bf16 [C x d]
+    int C;
+    const float *codebook;  // [M][256][ds]
+    int M;                  // sub-spaces, a multiple of 16
+    int ds;                 // d / M
+    const int64_t *offsets; // [C + 1] list starts
+    const int32_t *ids;     // [N] ids in list order
+    const uint8_t *codes;   // [N x M] codes in list order
+};
+cudaError_t launch_pq_encode(const IvfParams &p, const int64_t *row_list, uint8_t *codes, cudaStream_t s);
+// counts, cursor: [C] scratch; offsets [C + 1]; ids [N]; codes [N x M].
+cudaError_t launch_ivf_lists(const IvfParams &p, const int64_t *row_list, const uint8_t *codes_rows,
+                             int64_t *counts, int64_t *cursor, int64_t *offsets, int32_t *ids, uint8_t *codes,
+                             int *err, int sms, cudaStream_t s);
+size_t ivfpq_scan_smem(int M, int d, int nprobe);
+// Per region: keys (ordered score << 32 | ~id, 0 = empty) of the top k [R x k].
+cudaError_t launch_ivfpq_scan(const IvfParams &p, const uint16_t *regions, int R, const int64_t *probe_ids,
+                              const float *probe_scores, int nprobe, int k, uint64_t *out_keys, int sms,
+                              cudaStream_t s);
+
 }  // namespace skipk
