@@ -258,6 +258,44 @@ def run_reference(args, spec):
     print(json.dumps(line), flush=True)
 
 
+def ivfpq_report(args, spec, skip, c, ix, cent, reg_d, off_d, kernels, build_s, peaks, ms):
+    """Figures of the IVF-PQ step: recall against the exact path, the codes
+    the scan reads (probed list sizes from the index offsets), the scan
+    kernel's bandwidth against the HBM peak."""
+    k = spec.k_region
+    ivf_ids, _ = skip.skip_ivfpq_search_regions(ix, reg_d, args.nprobe, k)
+    ex_ids, _ = skip.skip_retrieve_regions(c, reg_d, k)
+    q_ivf, _ = skip.skip_ivfpq_search(ix, reg_d, off_d, args.nprobe, k, spec.K)
+    q_ex, _ = skip.skip_retrieve(c, reg_d, off_d, k, spec.K)
+    torch.cuda.synchronize()
+
+    def recall(a, b, n):
+        a, b = a.cpu().numpy(), b.cpu().numpy()
+        return float(np.mean([len(set(x[x >= 0]) & set(y[y >= 0])) / max(1, min(n, (y >= 0).sum()))
+                              for x, y in zip(a, b)]))
+    off, _, _ = skip.skip_ivfpq_lists(ix)
+    sizes = (off[1:] - off[:-1]).double()
+    probes = torch.topk(reg_d.float() @ cent.float().T, args.nprobe, dim=1).indices
+    scanned = float(sizes[probes].sum())
+    scan = kernels.get("ivfpq_scan", {"ms": float("nan"), "launches": 1})
+    scan_ms = scan["ms"] / max(1, scan["launches"])
+    code_bytes = scanned * (args.pq_m + 4)
+    return {
+        "ivfpq": {"C": int(cent.shape[0]), "M": args.pq_m, "nprobe": args.nprobe, "build_s": build_s,
+                  "recall_region_at_k": recall(ivf_ids, ex_ids, k), "recall_question_at_K": recall(q_ivf, q_ex, spec.K),
+                  "codes_scanned_per_step": scanned, "scan_kernel_ms": scan_ms,
+                  "scan_gbs": code_bytes / (scan_ms / 1e3) / 1e9,
+                  "scan_frac_of_hbm": code_bytes / (scan_ms / 1e3) / 1e9 / peaks["hbm_gbs"],
+                  "exact_step_ms_for_reference": None,
+                  "index_bytes": spec.N * (args.pq_m + 4),
+                  "note": "codes of probed lists mostly served from L2 when the index fits in 129 MB"},
+        "roofline": {"bound": "hbm", "achieved": code_bytes / (scan_ms / 1e3) / 1e9, "peak": peaks["hbm_gbs"],
+                     "unit": "GB/s", "frac": code_bytes / (scan_ms / 1e3) / 1e9 / peaks["hbm_gbs"], "traffic": None,
+                     "kernel": "ivfpq_scan", "kernel_ms": scan_ms, "algorithmic_bytes_per_launch": code_bytes,
+                     "peak_source": peaks["source"]},
+    }
+
+
 def main():
     ap = argparse.ArgumentParser()
     ap.add_argument("--gpus", type=int, default=1)
@@ -272,6 +310,10 @@ def main():
                     help="use only the first ROWS corpus rows (smaller profiling captures; not a bench line)")
     ap.add_argument("--cluster", type=int, default=0, choices=[0, 1, 2, 4, 8],
                     help="single-CTA tensor path CTAs per cluster (0 = library's choice)")
+    ap.add_argument("--ivfpq", action="store_true",
+                    help="step = IVF-PQ search (generator centres as IVF centroids, sample-based PQ codebook)")
+    ap.add_argument("--nprobe", type=int, default=32)
+    ap.add_argument("--pq-m", type=int, default=64, help="PQ sub-spaces (codes of M bytes)")
     ap.add_argument("--skv", action="store_true",
                     help="step = retrieval + SKV passage gate (skip_retrieve_skv), H = 512, tau 0.5, rho 0.6")
     ap.add_argument("--mma", default="auto", choices=["auto", "single", "pair"],
@@ -295,7 +337,7 @@ def main():
     R = regions.shape[0]
     Q = offsets.numel() - 1
     c = skip.skip_corpus_load(corpus, row_scale=scale)
-    keep_host = rank == 0 and world == 1 and not args.no_cpu_baseline
+    keep_host = rank == 0 and world == 1 and not args.no_cpu_baseline and not args.ivfpq
     corpus_np, scale_np = host_corpus(corpus, scale) if keep_host else (None, None)
     del corpus
     torch.cuda.empty_cache()
@@ -308,7 +350,18 @@ def main():
     out_sc = torch.empty(Q, spec.K, dtype=torch.float32, device=dev)
     stream = torch.cuda.current_stream()
 
-    if args.skv:
+    ix = None
+    if args.ivfpq:
+        cent = synth.make_ivf_centroids(spec).to(dev)
+        codebook = synth.make_pq_codebook(spec, args.pq_m).to(dev)
+        torch.cuda.synchronize()
+        tb = time.perf_counter()
+        ix = skip.skip_ivfpq_build(c, cent, codebook)
+        build_s = time.perf_counter() - tb
+
+        def step():
+            skip.skip_ivfpq_search(ix, reg_d, off_d, args.nprobe, spec.k_region, spec.K, out_ids, out_sc, stream)
+    elif args.skv:
         qbar, vbar = synth.make_skv_queries(regions, offsets)
         w1, b1, w2, b2 = synth.make_skv_mlp(spec.d)
         qbar, vbar, w1, b1, w2 = (x.to(dev).contiguous() for x in (qbar, vbar, w1, b1, w2))
@@ -328,8 +381,9 @@ def main():
     plan = skip.skip_last_plan(c)
 
     # ---- timed region (device-resident inputs)
-    c.set_option(skip.SKIP_OPT_TIMING, 1)
-    skip.skip_timing_report(c)
+    timed = ix if ix is not None else c
+    timed.set_option(skip.SKIP_OPT_TIMING, 1)
+    (skip.skip_ivfpq_timing_report(ix) if ix is not None else skip.skip_timing_report(c))
     sampler = ClockSampler(torch.cuda.current_device())
     barrier(world)
     torch.cuda.synchronize()
@@ -345,9 +399,9 @@ def main():
     clocks = sampler.stop()
     barrier(world)
     ms_local = e0.elapsed_time(e1)
-    kernels = skip.skip_timing_report(c)
-    c.set_option(skip.SKIP_OPT_TIMING, 0)
-    st = skip.skip_sync_status(c)
+    kernels = skip.skip_ivfpq_timing_report(ix) if ix is not None else skip.skip_timing_report(c)
+    timed.set_option(skip.SKIP_OPT_TIMING, 0)
+    st = skip.skip_ivfpq_sync_status(ix) if ix is not None else skip.skip_sync_status(c)
     if st != skip.SKIP_OK:
         raise SystemExit("timed kernel status: %s" % skip.skip_status_string(st))
     ms = max_over_ranks(ms_local, world)
@@ -360,7 +414,14 @@ def main():
     cnt_h = torch.empty(Q, dtype=torch.int32).pin_memory()
 
     def e2e_step():
-        if args.skv:
+        if args.ivfpq:
+            reg_d.copy_(reg_h, non_blocking=True)
+            off_d.copy_(off_h, non_blocking=True)
+            step()
+            ids_h.copy_(out_ids, non_blocking=True)
+            sc_h.copy_(out_sc, non_blocking=True)
+            stream.synchronize()
+        elif args.skv:
             # host regions in, gated lists out, through the device entry point
             reg_d.copy_(reg_h, non_blocking=True)
             off_d.copy_(off_h, non_blocking=True)
@@ -423,12 +484,17 @@ def main():
         "clocks": clocks,
         "e2e": {"value": total_q / e2e_s, "unit": "queries/s", "h2d_bytes_per_step": h2d,
                 "d2h_bytes_per_step": d2h,
-                "entry_point": ("skip_retrieve_skv with pinned host copies in and out" if args.skv
+                "entry_point": ("skip_ivfpq_search with pinned host copies in and out" if args.ivfpq else
+                                "skip_retrieve_skv with pinned host copies in and out" if args.skv
                                 else "skip_retrieve_host (pinned host buffers)")},
         "gpu_launches": int(sum(v["launches"] for v in kernels.values())),
         "kernels": kernels,
         "plan": plan,
     }
+    if args.ivfpq:
+        line.update(ivfpq_report(args, spec, skip, c, ix, cent, reg_d, off_d, kernels, build_s, peaks, ms))
+        line["config"]["variant"] = "IVF-PQ: %d centroids, PQ%d, nprobe %d" % (cent.shape[0], args.pq_m, args.nprobe)
+        ix.free()
     if args.skv:
         line["config"]["skv_gate"] = {"hidden": 512, "tau_nu": 0.5, "rho_r": 0.6}
         H = 512

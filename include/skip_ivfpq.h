@@ -20,7 +20,7 @@
  * training them is not part of this library).  Codes are one byte per
  * sub-space.  Conventions as in skip_retrieve.h (device pointers,
  * asynchronous and stream ordered, no CPU fallback).  Limits: bf16 corpus,
- * M a multiple of 16 with d / M <= 32, 1 <= nprobe <= min(C, 1024),
+ * M a multiple of 16, at most 128, with d / M <= 32, 1 <= nprobe <= min(C, 1024),
  * 1 <= k_region <= 1024, C <= 2^20.
  */
 #ifndef SKIP_IVFPQ_H

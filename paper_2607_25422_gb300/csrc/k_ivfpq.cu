@@ -212,7 +212,8 @@ __global__ void __launch_bounds__(kScanThreads) k_ivfpq_scan(const IvfParams p, 
                 }
                 const int64_t e = pstart[lo] + (v - pref[lo]);
                 const uint4 *code = reinterpret_cast<const uint4 *>(p.codes + e * p.M);
-                float s = pscore[lo];
+                // four independent sums (one per 32-bit word of a 16-byte chunk)
+                float acc[4] = {0.f, 0.f, 0.f, 0.f};
                 for (int w = 0; w < p.M / 16; ++w) {
                     const uint4 cw = __ldg(code + w);
                     const uint32_t ws[4] = {cw.x, cw.y, cw.z, cw.w};
@@ -220,8 +221,9 @@ __global__ void __launch_bounds__(kScanThreads) k_ivfpq_scan(const IvfParams p, 
                     for (int h = 0; h < 4; ++h)
 #pragma unroll
                         for (int b = 0; b < 4; ++b)
-                            s += T[((w * 16 + h * 4 + b) << 8) + ((ws[h] >> (8 * b)) & 0xFFu)];
+                            acc[h] += T[((w * 16 + h * 4 + b) << 8) + ((ws[h] >> (8 * b)) & 0xFFu)];
                 }
+                const float s = pscore[lo] + ((acc[0] + acc[1]) + (acc[2] + acc[3]));
                 const uint64_t key = make_key(s, (uint32_t)p.ids[e]);
                 if (key > tau) {
                     const int pos = atomicAdd(&cnt, 1);

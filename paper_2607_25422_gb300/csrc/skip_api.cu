@@ -951,7 +951,7 @@ skip_status_t ivf_create(const void *centroids, int C, int d, const float *codeb
 
 skip_status_t ivf_check_shape(int C, int d, int M) {
     if (C < 1 || d < 1 || M < 1) return SKIP_EINVAL;
-    if (C > (1 << 20) || M % 16 != 0 || d % M != 0 || d / M > kIvfMaxDs) return SKIP_EUNSUPPORTED;
+    if (C > (1 << 20) || M % 16 != 0 || M > kIvfMaxM || d % M != 0 || d / M > kIvfMaxDs) return SKIP_EUNSUPPORTED;
     return SKIP_OK;
 }
 

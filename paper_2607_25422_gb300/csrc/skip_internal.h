@@ -142,7 +142,8 @@ cudaError_t launch_skv_mlp(const CUtensorMap &tw, const SkvParams &p, cudaStream
 cudaError_t launch_skv_select(const SkvParams &p, cudaStream_t s);
 
 // ---- IVF-PQ variant (k_ivfpq.cu) ------------------------------------------
-constexpr int kIvfMaxDs = 32;  // largest sub-space width d / M
+constexpr int kIvfMaxDs = 32;   // largest sub-space width d / M
+constexpr int kIvfMaxM = 128;   // most sub-spaces (code bytes)
 struct IvfParams {
     const void *rows;       // bf16 corpus [N x d] (build only)
     int64_t N;
