@@ -24,6 +24,9 @@ Functions and what they follow:
   ``ivfpq_scores_at`` -- the IVF-PQ index (§4.1 "Implementation", App. I.4;
   the published inverted file with product-quantised residuals and
   asymmetric inner-product scoring) and its search (``ivfpq_oracle.c``).
+* ``qvs``, ``qvs_count`` -- App. B.1 Def. B.1 (Eq. qvs_score) and the Alg. 1
+  QVS prune: token scores sigmoid(<f_q, W_v v + b_v> / sqrt(d_k) + <w_b, v>)
+  and the top ceil(rho_v L) tokens (``qvs_oracle.c``).
 """
 from __future__ import annotations
 
@@ -35,7 +38,7 @@ import numpy as np
 
 _HERE = os.path.dirname(os.path.abspath(__file__))
 _SRCS = [os.path.join(_HERE, "rcsr_oracle.c"), os.path.join(_HERE, "skv_oracle.c"),
-         os.path.join(_HERE, "ivfpq_oracle.c")]
+         os.path.join(_HERE, "ivfpq_oracle.c"), os.path.join(_HERE, "qvs_oracle.c")]
 _OUT = os.path.join(_HERE, "_build", "libskip_oracle.so")
 _lib = None
 
@@ -79,7 +82,10 @@ def _load():
     lib.skip_oracle_pq_encode.argtypes = [P, i64, i32, P, P, P, i32, i32, P]
     lib.skip_oracle_ivfpq_search.argtypes = [P, i32, i32, P, P, P, P, i32, i32, P, i32, i32, i32, P, P, P]
     lib.skip_oracle_ivfpq_scores_at.argtypes = [P, i32, P, P, i64, P, i32, i32, P, P, P, i64, P]
-    for f in ("skip_oracle_ivf_assign", "skip_oracle_pq_encode", "skip_oracle_ivfpq_search",
+    lib.skip_oracle_qvs.argtypes = [P, i32, i32, i32, P, P, P, P, i32, ctypes.c_double, P, P, P]
+    lib.skip_oracle_qvs_count.argtypes = [i32, ctypes.c_double]
+    for f in ("skip_oracle_qvs", "skip_oracle_qvs_count", "skip_oracle_ivf_assign", "skip_oracle_pq_encode",
+              "skip_oracle_ivfpq_search",
               "skip_oracle_ivfpq_scores_at"):
         getattr(lib, f).restype = ctypes.c_int
     for f in ("skip_oracle_region_topk", "skip_oracle_merge", "skip_oracle_retrieve", "skip_oracle_skv",
@@ -339,3 +345,30 @@ def ivfpq_scores_at(index, centroids, codebook, regions, region_idx, ids):
                                        _ptr(ids), ids.shape[0], _ptr(out)):
         raise RuntimeError("oracle ivfpq_scores_at failed")
     return out
+
+
+def qvs_count(L: int, rho: float) -> int:
+    """ceil(rho * L - 1e-3) clamped to [0, L]: tokens kept per image."""
+    return int(_load().skip_oracle_qvs_count(int(L), float(rho)))
+
+
+def qvs(tokens, fq, wv, bv, wb, rho):
+    """QVS scores and pruning.  tokens uint16 [B, L, d] (bf16 bits); fq uint16
+    [B, dk]; wv uint16 [dk, d]; bv float32 [dk] or None; wb float32 [d].
+    Returns (logits float64 [B, L], idx int32 [B, n], score float64 [B, n])."""
+    lib = _load()
+    tokens = np.ascontiguousarray(tokens, dtype=np.uint16)
+    fq = np.ascontiguousarray(fq, dtype=np.uint16)
+    wv = np.ascontiguousarray(wv, dtype=np.uint16)
+    wb = np.ascontiguousarray(wb, dtype=np.float32)
+    bv = None if bv is None else np.ascontiguousarray(bv, dtype=np.float32)
+    B, L, d = tokens.shape
+    dk = wv.shape[0]
+    n = qvs_count(L, rho)
+    logits = np.empty((B, L), np.float64)
+    idx = np.empty((B, n), np.int32)
+    score = np.empty((B, n), np.float64)
+    if lib.skip_oracle_qvs(_ptr(tokens), B, L, d, _ptr(fq), _ptr(wv), _ptr(bv), _ptr(wb), dk, float(rho),
+                           _ptr(logits), _ptr(idx), _ptr(score)):
+        raise RuntimeError("oracle qvs failed")
+    return logits, idx, score

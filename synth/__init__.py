@@ -319,3 +319,35 @@ def make_pq_codebook(spec: WorkloadSpec, M: int, ksub: int = 256, device="cpu") 
     for m in range(M):
         cb[m] = r[m * ksub:(m + 1) * ksub, m * ds:(m + 1) * ds]
     return cb.to(device)
+
+
+# ---- inputs of QVS (App. B.1 Def. B.1) -------------------------------------
+#
+# QVS scores L visual tokens per image against the question: L = 576 (a 24 x
+# 24 patch grid, §4.1 / App. I.4: CLIP ViT-L/14 at 336 px), token width
+# d = 1024, d_k = d (Def. B.1 maps both to R^d).  No vision encoder or trained
+# QVS head exists here: tokens are Gaussian unit vectors, of which about 22%
+# ("entity" patches; the paper finds ~78% background) are pulled towards an
+# image direction g_b (x = normalise(z + 2 g_b)); f_q(Q) is normalise(g_b +
+# N(0, I)) scaled by sqrt(d); W_v = I + N(0, 0.25/d) (so that f_v roughly
+# keeps the token and entity patches score high), b_v ~ N(0, 0.01^2),
+# w_b ~ N(0, 1/d).  Tokens, f_q and W_v are bf16; b_v and w_b fp32.
+
+QVS_L, QVS_D = 576, 1024
+
+
+def make_qvs_inputs(B: int, L: int = QVS_L, d: int = QVS_D, seed: int = 5000, device="cpu"):
+    """(tokens bf16 [B, L, d], fq bf16 [B, d], wv bf16 [d, d], bv fp32 [d], wb fp32 [d])."""
+    g = _gen(seed, "cpu")
+    gdir = _normalise(torch.randn(B, d, generator=g))
+    tokens = torch.empty(B, L, d, dtype=torch.bfloat16)
+    for b in range(B):
+        z = torch.randn(L, d, generator=g) / math.sqrt(d)
+        ent = torch.rand(L, generator=g) < 0.22
+        z[ent] += 2.0 * gdir[b]
+        tokens[b] = _normalise(z).to(torch.bfloat16)
+    fq = (math.sqrt(d) * _normalise(gdir + torch.randn(B, d, generator=g) / math.sqrt(d))).to(torch.bfloat16)
+    wv = (torch.eye(d) + 0.5 * torch.randn(d, d, generator=g) / math.sqrt(d)).to(torch.bfloat16)
+    bv = 0.01 * torch.randn(d, generator=g)
+    wb = torch.randn(d, generator=g) / math.sqrt(d)
+    return tokens.to(device), fq.to(device), wv.to(device), bv.to(device), wb.to(device)
