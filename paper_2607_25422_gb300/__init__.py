@@ -14,7 +14,8 @@ merged into a deduplicated top-K (max score per id, ties to the lower id).
 The SKV passage gate (App. B.4 Def. B.4; ``include/skip_skv.h``) then keeps
 the passages whose verification score nu reaches tau, at most
 ceil(rho |K|) of them.  The IVF-PQ variant (``include/skip_ivfpq.h``) builds
-and searches an inverted-file, product-quantised index of the corpus.
+and searches an inverted-file, product-quantised index of the corpus; QVS
+(``include/skip_qvs.h``) scores and prunes visual tokens before retrieval.
 """
 from __future__ import annotations
 
@@ -83,6 +84,11 @@ def load_library():
     lib.skip_ivfpq_sync_status.argtypes = [P, P]
     lib.skip_ivfpq_set_option.argtypes = [P, ctypes.c_int, i64]
     lib.skip_ivfpq_timing_report.argtypes = [P, ctypes.c_char_p, i32]
+    lib.skip_qvs_create.argtypes = [P, P, P, i32, i32, i32, i32, P, ctypes.POINTER(P)]
+    lib.skip_qvs_free.argtypes = [P]
+    lib.skip_qvs_count.argtypes = [i32, ctypes.c_float]
+    lib.skip_qvs_count.restype = i32
+    lib.skip_qvs_prune.argtypes = [P, P, i32, i32, P, ctypes.c_float, P, P, P, P, P]
     lib.skip_status_string.argtypes = [ctypes.c_int]
     lib.skip_status_string.restype = ctypes.c_char_p
     for f in ("skip_corpus_load", "skip_corpus_free", "skip_corpus_set_option", "skip_retrieve",
@@ -90,7 +96,7 @@ def load_library():
               "skip_timing_report", "skip_retrieve_regions_noalloc", "skip_skv_gate", "skip_retrieve_skv",
               "skip_ivfpq_build", "skip_ivfpq_load", "skip_ivfpq_lists", "skip_ivfpq_info", "skip_ivfpq_free",
               "skip_ivfpq_search_regions", "skip_ivfpq_search", "skip_ivfpq_sync_status", "skip_ivfpq_set_option",
-              "skip_ivfpq_timing_report"):
+              "skip_ivfpq_timing_report", "skip_qvs_create", "skip_qvs_free", "skip_qvs_prune"):
         getattr(lib, f).restype = ctypes.c_int
     _lib = lib
     return lib
@@ -416,6 +422,65 @@ def skip_ivfpq_timing_report(index: IvfIndex) -> dict:
     return json.loads(buf.value.decode())
 
 
+class QvsHead:
+    """A QVS head (``skip_qvs_t``): weights copied to the library."""
+
+    def __init__(self, handle, d, dk):
+        self.handle, self.d, self.dk = handle, d, dk
+
+    def free(self):
+        if self.handle:
+            load_library().skip_qvs_free(self.handle)
+            self.handle = None
+
+    def __del__(self):
+        try:
+            self.free()
+        except Exception:
+            pass
+
+
+def skip_qvs_create(wv: torch.Tensor, bv: Optional[torch.Tensor], wb: torch.Tensor, max_images: int,
+                    max_tokens: int, stream=None) -> QvsHead:
+    """QVS head from device tensors: wv bf16 [d_k, d], bv float32 [d_k] or None, wb float32 [d]."""
+    wv = wv.contiguous()
+    bv = None if bv is None else bv.to(torch.float32).contiguous()
+    wb = wb.to(torch.float32).contiguous()
+    h = ctypes.c_void_p()
+    st = load_library().skip_qvs_create(_ptr(wv), _ptr(bv), _ptr(wb), wv.shape[1], wv.shape[0], int(max_images),
+                                        int(max_tokens), ctypes.c_void_p(_stream(stream)), ctypes.byref(h))
+    _check(st, "skip_qvs_create")
+    return QvsHead(h, wv.shape[1], wv.shape[0])
+
+
+def skip_qvs_count(L: int, rho_v: float) -> int:
+    return int(load_library().skip_qvs_count(int(L), float(rho_v)))
+
+
+def skip_qvs_prune(head: QvsHead, tokens: torch.Tensor, fq: torch.Tensor, rho_v: float, with_tokens: bool = False,
+                   with_logits: bool = False, stream=None):
+    """tokens bf16 [B, L, d], fq bf16 [B, d_k] (device).  Returns (idx int32
+    [B, n], score fp32 [B, n]) plus the kept tokens [B, n, d] and / or all
+    logits [B, L] when asked."""
+    tokens, fq = tokens.contiguous(), fq.contiguous()
+    B, L, d = tokens.shape
+    n = skip_qvs_count(L, rho_v)
+    dev = tokens.device
+    idx = torch.empty(B, n, dtype=torch.int32, device=dev)
+    score = torch.empty(B, n, dtype=torch.float32, device=dev)
+    kept = torch.empty(B, n, d, dtype=tokens.dtype, device=dev) if with_tokens else None
+    logits = torch.empty(B, L, dtype=torch.float32, device=dev) if with_logits else None
+    st = load_library().skip_qvs_prune(head.handle, _ptr(tokens), B, L, _ptr(fq), float(rho_v), _ptr(idx),
+                                       _ptr(score), _ptr(kept), _ptr(logits), ctypes.c_void_p(_stream(stream)))
+    _check(st, "skip_qvs_prune")
+    out = [idx, score]
+    if with_tokens:
+        out.append(kept)
+    if with_logits:
+        out.append(logits)
+    return tuple(out)
+
+
 def skip_sync_status(corpus: Corpus, stream=None) -> int:
     """Synchronise and return the status latched by the kernels (SKIP_OK, ...)."""
     return int(load_library().skip_sync_status(corpus.handle, ctypes.c_void_p(_stream(stream))))
@@ -436,4 +501,4 @@ def skip_timing_report(corpus: Corpus) -> dict:
 
 
 __all__ = [n for n in dir() if n.startswith("skip_") or n.startswith("SKIP_")] + [
-    "Corpus", "SkipError", "SkvMlp", "IvfIndex", "load_library", "library_path"]
+    "Corpus", "SkipError", "SkvMlp", "IvfIndex", "QvsHead", "load_library", "library_path"]

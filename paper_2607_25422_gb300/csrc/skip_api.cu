@@ -15,6 +15,7 @@
 #include "../../include/skip_retrieve.h"
 #include "../../include/skip_skv.h"
 #include "../../include/skip_ivfpq.h"
+#include "../../include/skip_qvs.h"
 #include "skip_internal.h"
 
 using namespace skipk;
@@ -1149,6 +1150,110 @@ skip_status_t skip_ivfpq_set_option(skip_ivfpq_t ix, int option, int64_t value) 
 skip_status_t skip_ivfpq_timing_report(skip_ivfpq_t ix, char *buf, int32_t len) {
     if (!ix) return SKIP_EINVAL;
     return skip_timing_report(ix->cent, buf, len);
+}
+
+}  // extern "C"
+
+// ---------------------------------------------------------------- QVS
+
+struct skip_qvs {
+    int device = 0, sms = 0;
+    int d = 0, dk = 0, max_b = 0, max_l = 0;
+    uint16_t *wv = nullptr;
+    float *bv = nullptr, *wb = nullptr;
+    float *u = nullptr, *c = nullptr, *logits = nullptr;  // workspace
+};
+
+namespace {
+
+void qvs_release(skip_qvs *q) {
+    if (!q) return;
+    cudaDeviceSynchronize();
+    cudaFree(q->wv);
+    cudaFree(q->bv);
+    cudaFree(q->wb);
+    cudaFree(q->u);
+    cudaFree(q->c);
+    cudaFree(q->logits);
+    delete q;
+}
+
+}  // namespace
+
+extern "C" {
+
+int32_t skip_qvs_count(int32_t L, float rho_v) {
+    const double v = ceil((double)rho_v * (double)L - 1e-3);
+    return (int32_t)std::max(0.0, std::min((double)L, v));
+}
+
+skip_status_t skip_qvs_create(const uint16_t *wv, const float *bv, const float *wb, int32_t d, int32_t dk,
+                              int32_t max_images, int32_t max_tokens, void *stream, skip_qvs_t *out) {
+    if (!wv || !wb || !out || d < 8 || dk < 1 || max_images < 1 || max_tokens < 1) return SKIP_EINVAL;
+    if (d % 8 != 0 || d > 8192 || dk > kQvsMaxDk || max_tokens > kQvsMaxL) return SKIP_EUNSUPPORTED;
+    int dev = 0;
+    cudaDeviceProp prop;
+    if (cudaGetDevice(&dev) != cudaSuccess || cudaGetDeviceProperties(&prop, dev) != cudaSuccess) {
+        cudaGetLastError();
+        return SKIP_EUNSUPPORTED;
+    }
+    if (prop.major != 10 || prop.minor != 3) return SKIP_EUNSUPPORTED;
+    auto *q = new skip_qvs();
+    q->device = dev, q->sms = prop.multiProcessorCount;
+    q->d = d, q->dk = dk, q->max_b = max_images, q->max_l = max_tokens;
+    if (cudaMalloc(&q->wv, (size_t)dk * d * 2) != cudaSuccess || cudaMalloc(&q->bv, (size_t)dk * 4) != cudaSuccess ||
+        cudaMalloc(&q->wb, (size_t)d * 4) != cudaSuccess ||
+        cudaMalloc(&q->u, (size_t)max_images * d * 4) != cudaSuccess ||
+        cudaMalloc(&q->c, (size_t)max_images * 4) != cudaSuccess ||
+        cudaMalloc(&q->logits, (size_t)max_images * max_tokens * 4) != cudaSuccess) {
+        cudaGetLastError();
+        qvs_release(q);
+        return SKIP_ENOMEM;
+    }
+    cudaStream_t s = reinterpret_cast<cudaStream_t>(stream);
+    if (cudaMemcpyAsync(q->wv, wv, (size_t)dk * d * 2, cudaMemcpyDeviceToDevice, s) != cudaSuccess ||
+        (bv ? cudaMemcpyAsync(q->bv, bv, (size_t)dk * 4, cudaMemcpyDeviceToDevice, s)
+            : cudaMemsetAsync(q->bv, 0, (size_t)dk * 4, s)) != cudaSuccess ||
+        cudaMemcpyAsync(q->wb, wb, (size_t)d * 4, cudaMemcpyDeviceToDevice, s) != cudaSuccess ||
+        cudaStreamSynchronize(s) != cudaSuccess) {
+        qvs_release(q);
+        return SKIP_ECUDA;
+    }
+    *out = q;
+    return SKIP_OK;
+}
+
+skip_status_t skip_qvs_free(skip_qvs_t q) {
+    qvs_release(q);
+    return SKIP_OK;
+}
+
+skip_status_t skip_qvs_prune(skip_qvs_t q, const uint16_t *tokens, int32_t B, int32_t L, const uint16_t *fq,
+                             float rho_v, int32_t *out_idx, float *out_score, uint16_t *out_tokens, float *logits,
+                             void *stream) {
+    if (!q || B < 0 || B > q->max_b || L < 1 || L > q->max_l) return SKIP_EINVAL;
+    if (!(rho_v >= 0.f && rho_v <= 1.f)) return SKIP_EINVAL;
+    const int n = skip_qvs_count(L, rho_v);
+    if (B > 0 && (!tokens || !fq || (n > 0 && (!out_idx || !out_score)))) return SKIP_EINVAL;
+    if (B == 0) return SKIP_OK;
+    cudaStream_t s = reinterpret_cast<cudaStream_t>(stream);
+    QvsParams p;
+    p.tokens = tokens;
+    p.fq = fq;
+    p.wv = q->wv;
+    p.bv = q->bv;
+    p.wb = q->wb;
+    p.B = B, p.L = L, p.d = q->d, p.dk = q->dk, p.n = n;
+    p.u = q->u;
+    p.c = q->c;
+    p.logits = logits ? logits : q->logits;
+    p.out_idx = out_idx;
+    p.out_score = out_score;
+    p.out_tokens = out_tokens;
+    cudaError_t e = launch_qvs_u(p, s);
+    if (e == cudaSuccess) e = launch_qvs_logits(p, q->sms, s);
+    if (e == cudaSuccess) e = launch_qvs_select(p, s);
+    return cuda_status(e);
 }
 
 }  // extern "C"

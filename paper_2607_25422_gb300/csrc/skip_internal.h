@@ -168,4 +168,25 @@ cudaError_t launch_ivfpq_scan(const IvfParams &p, const uint16_t *regions, int R
                               const float *probe_scores, int nprobe, int k, uint64_t *out_keys, int sms,
                               cudaStream_t s);
 
+// ---- QVS visual token pruning (k_qvs.cu) -----------------------------------
+constexpr int kQvsMaxDk = 4096;  // projection width d_k
+constexpr int kQvsMaxL = 4096;   // tokens per image
+struct QvsParams {
+    const void *tokens;     // bf16 [B x L x d]
+    const void *fq;         // bf16 [B x dk]
+    const void *wv;         // bf16 [dk x d]
+    const float *bv;        // [dk] or null
+    const float *wb;        // [d]
+    int B, L, d, dk, n;     // n tokens kept per image
+    float *u;               // [B x d] workspace
+    float *c;               // [B] workspace
+    float *logits;          // [B x L] workspace
+    int32_t *out_idx;       // [B x n]
+    float *out_score;       // [B x n]
+    void *out_tokens;       // bf16 [B x n x d] or null
+};
+cudaError_t launch_qvs_u(const QvsParams &p, cudaStream_t s);
+cudaError_t launch_qvs_logits(const QvsParams &p, int sms, cudaStream_t s);
+cudaError_t launch_qvs_select(const QvsParams &p, cudaStream_t s);
+
 }  // namespace skipk
