@@ -296,6 +296,98 @@ def ivfpq_report(args, spec, skip, c, ix, cent, reg_d, off_d, kernels, build_s, 
     }
 
 
+def run_qvs(args, spec, skip):
+    """QVS bench: one image per question of the workload (B = Q), L = 576
+    tokens of d = 1024, d_k = d, rho_v from --rho-v; HBM-bound token scan."""
+    world, rank, local = dist_setup()
+    dev = torch.device("cuda", torch.cuda.current_device())
+    B = spec.Q
+    L, d = synth.QVS_L, synth.QVS_D
+    tokens, fq, wv, bv, wb = synth.make_qvs_inputs(B, L, d)
+    head = skip.skip_qvs_create(wv.to(dev), bv.to(dev), wb.to(dev), B, L)
+    tok_d, fq_d = tokens.to(dev), fq.to(dev)
+    n = skip.skip_qvs_count(L, args.rho_v)
+    idx = torch.empty(B, n, dtype=torch.int32, device=dev)
+    stream = torch.cuda.current_stream()
+
+    def step():
+        return skip.skip_qvs_prune(head, tok_d, fq_d, args.rho_v, with_tokens=True, stream=stream)
+    for _ in range(args.warmup):
+        step()
+    torch.cuda.synchronize()
+    # per-kernel times: one profiled pass of events around each launch is not
+    # available without a handle, so the scan kernel's share comes from ncu;
+    # the step time here is the whole prune.
+    sampler = ClockSampler(torch.cuda.current_device())
+    barrier(world)
+    torch.cuda.synchronize()
+    sampler.start()
+    time.sleep(0.3)
+    e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    e0.record(stream)
+    for _ in range(args.steps):
+        step()
+    e1.record(stream)
+    torch.cuda.synchronize()
+    clocks = sampler.stop()
+    ms = max_over_ranks(e0.elapsed_time(e1), world)
+    # end to end: host tokens in, kept indices and scores out
+    tok_h, fq_h = tokens.pin_memory(), fq.pin_memory()
+    idx_h = torch.empty(B, n, dtype=torch.int32).pin_memory()
+    sc_h = torch.empty(B, n, dtype=torch.float32).pin_memory()
+
+    def e2e_step():
+        tok_d.copy_(tok_h, non_blocking=True)
+        fq_d.copy_(fq_h, non_blocking=True)
+        i, sc, _ = step()
+        idx_h.copy_(i, non_blocking=True)
+        sc_h.copy_(sc, non_blocking=True)
+        stream.synchronize()
+    for _ in range(3):
+        e2e_step()
+    torch.cuda.synchronize()
+    t0 = time.perf_counter()
+    for _ in range(args.steps):
+        e2e_step()
+    e2e_s = max_over_ranks(time.perf_counter() - t0, world)
+    peaks = load_peaks()
+    step_ms = ms / args.steps
+    tok_bytes = B * L * d * 2
+    step_bytes = tok_bytes + B * n * d * 2 + wv.numel() * 2 + B * L * 4 * 2
+    achieved = step_bytes / (step_ms / 1e3) / 1e9
+    line = {
+        "metric": "QVS images/s (visual token pruning) [next row]", "value": B * world * args.steps / (ms / 1e3),
+        "unit": "images/s", "n_gpus": world, "steps": args.steps, "warmup": args.warmup, "ms_per_step": step_ms,
+        "higher_is_better": True, "scaling": "weak", "vs_baseline": None, "dtype": "bf16", "data": "synthetic",
+        "config": {"workload": "qvs_%dx%dx%d" % (B, L, d), "images_per_gpu": B, "tokens": L, "d": d, "d_k": d,
+                   "rho_v": args.rho_v, "kept": n,
+                   "l2": "tokens %.1f MB < L2: steady-state reads may hit L2" % (tok_bytes / 1e6)},
+        "roofline": {"bound": "hbm", "achieved": achieved, "peak": peaks["hbm_gbs"], "unit": "GB/s",
+                     "frac": achieved / peaks["hbm_gbs"], "traffic": None, "kernel": "qvs step (5 kernels)",
+                     "algorithmic_bytes_per_step": step_bytes, "peak_source": peaks["source"]},
+        "clocks": clocks,
+        "e2e": {"value": B * world * args.steps / e2e_s, "unit": "images/s",
+                "h2d_bytes_per_step": tok_bytes + B * d * 2, "d2h_bytes_per_step": B * n * 8,
+                "entry_point": "skip_qvs_prune with pinned host copies in and out"},
+        "gpu_launches": 5 * args.steps,
+    }
+    if rank == 0 and world == 1 and not args.no_cpu_baseline:
+        import oracle
+        nb = 2
+        t0 = time.perf_counter()
+        oracle.qvs(synth.bf16_bits(tokens[:nb]), synth.bf16_bits(fq[:nb]), synth.bf16_bits(wv), bv.numpy(),
+                   wb.numpy(), args.rho_v)
+        dt = time.perf_counter() - t0
+        line["cpu_baseline"] = {"value": nb / dt, "unit": "images/s", "cores": oracle.threads(), "kind": "oracle",
+                                "sample": "%d images of the batch (fp64, W_v v per token as defined)" % nb}
+    head.free()
+    if rank == 0:
+        print(json.dumps(line), flush=True)
+    if world > 1:
+        import torch.distributed as dist
+        dist.destroy_process_group()
+
+
 def main():
     ap = argparse.ArgumentParser()
     ap.add_argument("--gpus", type=int, default=1)
@@ -314,6 +406,9 @@ def main():
                     help="step = IVF-PQ search (generator centres as IVF centroids, sample-based PQ codebook)")
     ap.add_argument("--nprobe", type=int, default=32)
     ap.add_argument("--pq-m", type=int, default=64, help="PQ sub-spaces (codes of M bytes)")
+    ap.add_argument("--qvs", action="store_true",
+                    help="step = QVS token pruning of one image per question of the workload (576 x 1024 tokens)")
+    ap.add_argument("--rho-v", type=float, default=0.4)
     ap.add_argument("--skv", action="store_true",
                     help="step = retrieval + SKV passage gate (skip_retrieve_skv), H = 512, tau 0.5, rho 0.6")
     ap.add_argument("--mma", default="auto", choices=["auto", "single", "pair"],
@@ -331,6 +426,9 @@ def main():
 
     import paper_2607_25422_gb300 as skip
 
+    if args.qvs:
+        run_qvs(args, spec, skip)
+        return
     world, rank, local = dist_setup()
     dev = torch.device("cuda", torch.cuda.current_device())
     corpus, scale, regions, offsets = make_inputs(spec, rank, world, dev)

@@ -6,11 +6,14 @@
 // once: HBM-bound), and the ranking by s = sigmoid(logit) is the ranking by
 // the logit.
 //
-//  k_qvs_u       u and c for eight images per block (W_v read once per eight).
-//  k_qvs_logits  one warp per token, 16-byte loads, u in shared memory.
+//  k_qvs_u       partial sums of W_v^T f_q and <f_q, b_v> per 32-wide slice
+//                of d_k, eight images per block (W_v read once per eight).
+//  k_qvs_ureduce the slices summed: u = sum / sqrt(d_k) + w_b, c likewise.
+//  k_qvs_logits  u in shared memory; one warp per four tokens at a time,
+//                16-byte loads.
 //  k_qvs_select  per image: (logit, ~index) keys sorted descending in shared
-//                memory, the first n kept; their sigmoid scores and (optional)
-//                the kept token rows copied out.
+//                memory, the first n kept with their sigmoid scores.
+//  k_qvs_gather  (optional) the kept token rows copied out, a block per row.
 #include <cuda_bf16.h>
 #include <cuda_runtime.h>
 
@@ -22,44 +25,84 @@
 namespace skipk {
 namespace {
 
-constexpr int kUImgs = 8, kUThreads = 128;
+constexpr int kUImgs = 8, kUThreads = 128, kUSlice = 32, kUCols = 8;
 
+// Partial sums of W_v^T f_q over one 32-wide slice of d_k, for 8 columns of d
+// per thread (one 16-byte load of W_v per k) and eight images per block:
+// part[slice][b][j]; the c term likewise.
 __global__ void __launch_bounds__(kUThreads) k_qvs_u(const QvsParams p) {
-    extern __shared__ float fq_smem[];  // [kUImgs][dk]
-    auto fqs = [&](int u, int k) -> float & { return fq_smem[u * p.dk + k]; };
-    const int b0 = blockIdx.y * kUImgs;
-    const int j = blockIdx.x * kUThreads + threadIdx.x;
+    __shared__ float fqs[kUImgs][kUSlice];
+    const int j0 = (blockIdx.x * kUThreads + threadIdx.x) * kUCols;
+    const int ks = blockIdx.y, k0 = ks * kUSlice;
+    const int b0 = blockIdx.z * kUImgs;
+    const int kn = min(kUSlice, p.dk - k0);
     const __nv_bfloat16 *fq = reinterpret_cast<const __nv_bfloat16 *>(p.fq);
-    for (int e = threadIdx.x; e < kUImgs * p.dk; e += kUThreads) {
-        const int u = e / p.dk, k = e - u * p.dk;
-        fqs(u, k) = b0 + u < p.B ? __bfloat162float(fq[(int64_t)(b0 + u) * p.dk + k]) : 0.f;
+    for (int e = threadIdx.x; e < kUImgs * kUSlice; e += kUThreads) {
+        const int u = e / kUSlice, k = e - u * kUSlice;
+        fqs[u][k] = (b0 + u < p.B && k < kn) ? __bfloat162float(fq[(int64_t)(b0 + u) * p.dk + k0 + k]) : 0.f;
     }
     __syncthreads();
-    const float inv = rsqrtf((float)p.dk);
-    if (j < p.d) {
-        const __nv_bfloat16 *wv = reinterpret_cast<const __nv_bfloat16 *>(p.wv);
-        float acc[kUImgs];
-#pragma unroll
-        for (int u = 0; u < kUImgs; ++u) acc[u] = 0.f;
-        for (int k = 0; k < p.dk; ++k) {
-            const float w = __bfloat162float(wv[(int64_t)k * p.d + j]);
-#pragma unroll
-            for (int u = 0; u < kUImgs; ++u) acc[u] = fmaf(w, fqs(u, k), acc[u]);
-        }
-        const float wbj = p.wb[j];
+    if (j0 < p.d) {
+        const uint4 *wv = reinterpret_cast<const uint4 *>(reinterpret_cast<const __nv_bfloat16 *>(p.wv) +
+                                                          (int64_t)k0 * p.d + j0);
+        const int64_t wstride = p.d / 8;
+        float acc[kUImgs][kUCols];
 #pragma unroll
         for (int u = 0; u < kUImgs; ++u)
-            if (b0 + u < p.B) p.u[(int64_t)(b0 + u) * p.d + j] = acc[u] * inv + wbj;
+#pragma unroll
+            for (int c = 0; c < kUCols; ++c) acc[u][c] = 0.f;
+#pragma unroll 4
+        for (int k = 0; k < kn; ++k) {
+            const uint4 w4 = __ldg(wv + k * wstride);
+            const uint32_t wv4[4] = {w4.x, w4.y, w4.z, w4.w};
+            float w[kUCols];
+#pragma unroll
+            for (int h = 0; h < 4; ++h) {
+                const float2 f = __bfloat1622float2(*reinterpret_cast<const __nv_bfloat162 *>(&wv4[h]));
+                w[2 * h] = f.x;
+                w[2 * h + 1] = f.y;
+            }
+#pragma unroll
+            for (int u = 0; u < kUImgs; ++u) {
+                const float f = fqs[u][k];
+#pragma unroll
+                for (int c = 0; c < kUCols; ++c) acc[u][c] = fmaf(w[c], f, acc[u][c]);
+            }
+        }
+#pragma unroll
+        for (int u = 0; u < kUImgs; ++u)
+            if (b0 + u < p.B) {
+                float4 *dst = reinterpret_cast<float4 *>(p.u + ((int64_t)ks * p.B + b0 + u) * p.d + j0);
+                dst[0] = make_float4(acc[u][0], acc[u][1], acc[u][2], acc[u][3]);
+                dst[1] = make_float4(acc[u][4], acc[u][5], acc[u][6], acc[u][7]);
+            }
     }
-    if (blockIdx.x == 0 && threadIdx.x < 32) {  // c = <f_q, b_v> / sqrt(d_k), one warp per image in turn
+    if (blockIdx.x == 0 && threadIdx.x < 32) {  // <f_q, b_v> over the slice, one warp, image by image
         for (int u = 0; u < kUImgs && b0 + u < p.B; ++u) {
-            float s = 0.f;
-            if (p.bv)
-                for (int k = threadIdx.x; k < p.dk; k += 32) s = fmaf(fqs(u, k), p.bv[k], s);
+            float s = (p.bv && (int)threadIdx.x < kn) ? fqs[u][threadIdx.x] * p.bv[k0 + threadIdx.x] : 0.f;
 #pragma unroll
             for (int o = 16; o; o >>= 1) s += __shfl_xor_sync(0xFFFFFFFFu, s, o);
-            if (threadIdx.x == 0) p.c[b0 + u] = s * inv;
+            if (threadIdx.x == 0) p.c[ks * p.B + b0 + u] = s;
         }
+    }
+}
+
+// u = (sum of the slices) / sqrt(d_k) + w_b and c likewise, written over
+// slice 0 (each thread reads all slices of its own element first).
+__global__ void __launch_bounds__(256) k_qvs_ureduce(const QvsParams p) {
+    const int64_t e = (int64_t)blockIdx.x * 256 + threadIdx.x;
+    const int ns = (p.dk + kUSlice - 1) / kUSlice;
+    const float inv = rsqrtf((float)p.dk);
+    if (e < (int64_t)p.B * p.d) {
+        const int64_t stride = (int64_t)p.B * p.d;
+        float v = 0.f;
+        for (int ks = 0; ks < ns; ++ks) v += p.u[ks * stride + e];
+        p.u[e] = v * inv + p.wb[e % p.d];
+    }
+    if (e < p.B) {
+        float c = 0.f;
+        for (int ks = 0; ks < ns; ++ks) c += p.c[ks * p.B + e];
+        p.c[e] = c * inv;
     }
 }
 
@@ -73,31 +116,92 @@ __global__ void __launch_bounds__(kLogThreads) k_qvs_logits(const QvsParams p) {
     const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
     const int nw = p.d / 8;  // 16-byte words per token
     const float cb = p.c[b];
-    for (int i = blockIdx.x * (kLogThreads / 32) + warp; i < p.L; i += gridDim.x * (kLogThreads / 32)) {
-        const uint4 *row = reinterpret_cast<const uint4 *>(p.tokens) + ((int64_t)b * p.L + i) * nw;
-        float s = 0.f;
-        for (int w = lane; w < nw; w += 32) {
-            const uint4 x = __ldg(row + w);
-            const uint32_t xv[4] = {x.x, x.y, x.z, x.w};
+    // Four tokens per warp at a time: their loads are issued together.
+    constexpr int kT = 4;
+    const int wstep = gridDim.x * (kLogThreads / 32);
+    for (int i0 = blockIdx.x * (kLogThreads / 32) + warp; i0 < p.L; i0 += kT * wstep) {
+        float s[kT];
 #pragma unroll
-            for (int h = 0; h < 4; ++h) {
-                const float2 f = __bfloat1622float2(*reinterpret_cast<const __nv_bfloat162 *>(&xv[h]));
-                s = fmaf(f.x, us[w * 8 + 2 * h], s);
-                s = fmaf(f.y, us[w * 8 + 2 * h + 1], s);
+        for (int t = 0; t < kT; ++t) s[t] = 0.f;
+        for (int w = lane; w < nw; w += 32) {
+            uint4 x[kT];
+#pragma unroll
+            for (int t = 0; t < kT; ++t) {
+                const int i = i0 + t * wstep;
+                x[t] = i < p.L ? __ldg(reinterpret_cast<const uint4 *>(p.tokens) + ((int64_t)b * p.L + i) * nw + w)
+                               : make_uint4(0, 0, 0, 0);
+            }
+            float uu[8];
+#pragma unroll
+            for (int e = 0; e < 8; ++e) uu[e] = us[w * 8 + e];
+#pragma unroll
+            for (int t = 0; t < kT; ++t) {
+                const uint32_t xv[4] = {x[t].x, x[t].y, x[t].z, x[t].w};
+#pragma unroll
+                for (int h = 0; h < 4; ++h) {
+                    const float2 f = __bfloat1622float2(*reinterpret_cast<const __nv_bfloat162 *>(&xv[h]));
+                    s[t] = fmaf(f.x, uu[2 * h], s[t]);
+                    s[t] = fmaf(f.y, uu[2 * h + 1], s[t]);
+                }
             }
         }
 #pragma unroll
-        for (int o = 16; o; o >>= 1) s += __shfl_xor_sync(0xFFFFFFFFu, s, o);
-        if (lane == 0) p.logits[(int64_t)b * p.L + i] = s + cb;
+        for (int t = 0; t < kT; ++t) {
+#pragma unroll
+            for (int o = 16; o; o >>= 1) s[t] += __shfl_xor_sync(0xFFFFFFFFu, s[t], o);
+            const int i = i0 + t * wstep;
+            if (lane == 0 && i < p.L) p.logits[(int64_t)b * p.L + i] = s[t] + cb;
+        }
     }
 }
 
 constexpr int kSelThreads = 512;
 
+// One bitonic step on a register pair held by lanes (lane, lane ^ j): the
+// lower lane keeps the larger key when `desc`, else the smaller.
+__device__ __forceinline__ uint64_t bitonic_lane_step(uint64_t v, int pos, int j, bool desc) {
+    const uint64_t o = __shfl_xor_sync(0xFFFFFFFFu, v, j);
+    const bool lower = (pos & j) == 0;
+    const bool keep_max = lower == desc;
+    return keep_max ? (v > o ? v : o) : (v < o ? v : o);
+}
+
+// Sorts keys[0, n) descending (n a power of two, 64 <= n <= kQvsMaxL, block of
+// kSelThreads threads).  Strides below 32 run inside warps on registers,
+// one key per lane; larger strides through shared memory.
+__device__ void bitonic_desc(uint64_t *keys, int n) {
+    const int lane = threadIdx.x & 31;
+    for (int size = 2; size <= n; size <<= 1) {
+        int stride = size >> 1;
+        for (; stride >= 32; stride >>= 1) {
+            for (int t = threadIdx.x; t < n / 2; t += kSelThreads) {
+                const int lo = 2 * t - (t & (stride - 1));
+                const int hi = lo + stride;
+                const bool desc = (lo & size) == 0;
+                const uint64_t a = keys[lo], b = keys[hi];
+                if ((a < b) == desc) {
+                    keys[lo] = b;
+                    keys[hi] = a;
+                }
+            }
+            __syncthreads();
+        }
+        // strides 16 .. 1: each warp sorts its 32-key runs in registers
+        for (int base = (threadIdx.x & ~31); base < n; base += kSelThreads) {
+            const int pos = base + lane;
+            uint64_t v = keys[pos];
+            const bool desc = (pos & size) == 0;
+            for (int j = stride; j > 0; j >>= 1) v = bitonic_lane_step(v, pos, j, desc);
+            keys[pos] = v;
+        }
+        __syncthreads();
+    }
+}
+
 __global__ void __launch_bounds__(kSelThreads) k_qvs_select(const QvsParams p) {
     __shared__ uint64_t keys[kQvsMaxL];
     const int b = blockIdx.x;
-    int Lp = 2;
+    int Lp = 64;
     while (Lp < p.L) Lp <<= 1;
     for (int i = threadIdx.x; i < Lp; i += kSelThreads) {
         uint64_t key = 0;
@@ -105,45 +209,36 @@ __global__ void __launch_bounds__(kSelThreads) k_qvs_select(const QvsParams p) {
         keys[i] = key;
     }
     __syncthreads();
-    for (int size = 2; size <= Lp; size <<= 1)
-        for (int stride = size >> 1; stride > 0; stride >>= 1) {
-            for (int t = threadIdx.x; t < Lp / 2; t += kSelThreads) {
-                const int lo = 2 * t - (t & (stride - 1));
-                const int hi = lo + stride;
-                const bool desc = (lo & size) == 0;
-                const uint64_t x = keys[lo], y = keys[hi];
-                if ((x < y) == desc) {
-                    keys[lo] = y;
-                    keys[hi] = x;
-                }
-            }
-            __syncthreads();
-        }
+    bitonic_desc(keys, Lp);
     for (int r = threadIdx.x; r < p.n; r += kSelThreads) {
         const uint64_t key = keys[r];
         p.out_idx[(int64_t)b * p.n + r] = (int32_t)(0xFFFFFFFFu - (uint32_t)key);
         p.out_score[(int64_t)b * p.n + r] = 1.f / (1.f + expf(-score_of_ord((uint32_t)(key >> 32))));
     }
-    if (p.out_tokens) {
-        const int nw = p.d / 8;
-        for (int e = threadIdx.x; e < p.n * nw; e += kSelThreads) {
-            const int r = e / nw, w = e - r * nw;
-            const int i = (int)(0xFFFFFFFFu - (uint32_t)keys[r]);
-            reinterpret_cast<uint4 *>(p.out_tokens)[((int64_t)b * p.n + r) * nw + w] =
-                __ldg(reinterpret_cast<const uint4 *>(p.tokens) + ((int64_t)b * p.L + i) * nw + w);
-        }
-    }
+}
+
+// Kept token rows: one block per (rank, image), 16-byte copies.
+__global__ void __launch_bounds__(128) k_qvs_gather(const QvsParams p) {
+    const int r = blockIdx.x, b = blockIdx.y;
+    const int i = p.out_idx[(int64_t)b * p.n + r];
+    const int nw = p.d / 8;
+    const uint4 *src = reinterpret_cast<const uint4 *>(p.tokens) + ((int64_t)b * p.L + i) * nw;
+    uint4 *dst = reinterpret_cast<uint4 *>(p.out_tokens) + ((int64_t)b * p.n + r) * nw;
+    for (int w = threadIdx.x; w < nw; w += 128) dst[w] = __ldg(src + w);
 }
 
 }  // namespace
 
+int qvs_u_slices(int dk) { return (dk + kUSlice - 1) / kUSlice; }
+
 cudaError_t launch_qvs_u(const QvsParams &p, cudaStream_t s) {
     if (p.B == 0) return cudaSuccess;
-    const size_t smem = (size_t)kUImgs * p.dk * sizeof(float);
-    cudaError_t e = cudaFuncSetAttribute(k_qvs_u, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
+    dim3 grid((unsigned)((p.d / kUCols + kUThreads - 1) / kUThreads), (unsigned)((p.dk + kUSlice - 1) / kUSlice),
+              (unsigned)((p.B + kUImgs - 1) / kUImgs));
+    k_qvs_u<<<grid, kUThreads, 0, s>>>(p);
+    cudaError_t e = cudaGetLastError();
     if (e != cudaSuccess) return e;
-    dim3 grid((unsigned)((p.d + kUThreads - 1) / kUThreads), (unsigned)((p.B + kUImgs - 1) / kUImgs));
-    k_qvs_u<<<grid, kUThreads, smem, s>>>(p);
+    k_qvs_ureduce<<<(unsigned)(((int64_t)p.B * p.d + 255) / 256), 256, 0, s>>>(p);
     return cudaGetLastError();
 }
 
@@ -159,6 +254,9 @@ cudaError_t launch_qvs_logits(const QvsParams &p, int sms, cudaStream_t s) {
 cudaError_t launch_qvs_select(const QvsParams &p, cudaStream_t s) {
     if (p.B == 0) return cudaSuccess;
     k_qvs_select<<<p.B, kSelThreads, 0, s>>>(p);
+    cudaError_t e = cudaGetLastError();
+    if (e != cudaSuccess || !p.out_tokens || p.n == 0) return e;
+    k_qvs_gather<<<dim3((unsigned)p.n, (unsigned)p.B), 128, 0, s>>>(p);
     return cudaGetLastError();
 }
 

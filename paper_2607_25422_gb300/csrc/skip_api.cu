@@ -1203,8 +1203,8 @@ skip_status_t skip_qvs_create(const uint16_t *wv, const float *bv, const float *
     q->d = d, q->dk = dk, q->max_b = max_images, q->max_l = max_tokens;
     if (cudaMalloc(&q->wv, (size_t)dk * d * 2) != cudaSuccess || cudaMalloc(&q->bv, (size_t)dk * 4) != cudaSuccess ||
         cudaMalloc(&q->wb, (size_t)d * 4) != cudaSuccess ||
-        cudaMalloc(&q->u, (size_t)max_images * d * 4) != cudaSuccess ||
-        cudaMalloc(&q->c, (size_t)max_images * 4) != cudaSuccess ||
+        cudaMalloc(&q->u, (size_t)qvs_u_slices(dk) * max_images * d * 4) != cudaSuccess ||
+        cudaMalloc(&q->c, (size_t)qvs_u_slices(dk) * max_images * 4) != cudaSuccess ||
         cudaMalloc(&q->logits, (size_t)max_images * max_tokens * 4) != cudaSuccess) {
         cudaGetLastError();
         qvs_release(q);
