@@ -27,6 +27,9 @@ Functions and what they follow:
 * ``qvs``, ``qvs_count`` -- App. B.1 Def. B.1 (Eq. qvs_score) and the Alg. 1
   QVS prune: token scores sigmoid(<f_q, W_v v + b_v> / sqrt(d_k) + <w_b, v>)
   and the top ceil(rho_v L) tokens (``qvs_oracle.c``).
+* ``bsca``, ``bsca_edges_count`` -- App. B.3 Def. B.3 (Eq. bsca_edges,
+  bsca_attn): the bipartite edge set by cosine threshold and the attention of
+  each visual token over its chunk neighbours (``bsca_oracle.c``).
 """
 from __future__ import annotations
 
@@ -38,7 +41,8 @@ import numpy as np
 
 _HERE = os.path.dirname(os.path.abspath(__file__))
 _SRCS = [os.path.join(_HERE, "rcsr_oracle.c"), os.path.join(_HERE, "skv_oracle.c"),
-         os.path.join(_HERE, "ivfpq_oracle.c"), os.path.join(_HERE, "qvs_oracle.c")]
+         os.path.join(_HERE, "ivfpq_oracle.c"), os.path.join(_HERE, "qvs_oracle.c"),
+         os.path.join(_HERE, "bsca_oracle.c")]
 _OUT = os.path.join(_HERE, "_build", "libskip_oracle.so")
 _lib = None
 
@@ -83,6 +87,10 @@ def _load():
     lib.skip_oracle_ivfpq_search.argtypes = [P, i32, i32, P, P, P, P, i32, i32, P, i32, i32, i32, P, P, P]
     lib.skip_oracle_ivfpq_scores_at.argtypes = [P, i32, P, P, i64, P, i32, i32, P, P, P, i64, P]
     lib.skip_oracle_qvs.argtypes = [P, i32, i32, i32, P, P, P, P, i32, ctypes.c_double, P, P, P]
+    lib.skip_oracle_bsca.argtypes = [P, P, i32, P, P, P, P, P, i32, i32, i32, i32, ctypes.c_double, P, P, P, P, P]
+    lib.skip_oracle_bsca_edges_count.argtypes = [i32, ctypes.c_double]
+    lib.skip_oracle_bsca.restype = ctypes.c_int
+    lib.skip_oracle_bsca_edges_count.restype = ctypes.c_int
     lib.skip_oracle_qvs_count.argtypes = [i32, ctypes.c_double]
     for f in ("skip_oracle_qvs", "skip_oracle_qvs_count", "skip_oracle_ivf_assign", "skip_oracle_pq_encode",
               "skip_oracle_ivfpq_search",
@@ -372,3 +380,32 @@ def qvs(tokens, fq, wv, bv, wb, rho):
                            _ptr(logits), _ptr(idx), _ptr(score)):
         raise RuntimeError("oracle qvs failed")
     return logits, idx, score
+
+
+def bsca_edges_count(P: int, dbar: float) -> int:
+    """ceil(dbar * P - 1e-3): edges a question keeps (before ties at tau_e)."""
+    return int(_load().skip_oracle_bsca_edges_count(int(P), float(dbar)))
+
+
+def bsca(vis_offsets, chunk_offsets, hv, qh, hk, kh, vh, rmax, dbar=4.0, edge_mask=None):
+    """BSCA per question.  Offsets int32 [Q+1]; hv, qh uint16 (bf16 bits)
+    [Nv, dp] / [Nv, dh]; hk, kh, vh uint16 [Nc, dp] / [Nc, dh] / [Nc, dout].
+    Returns dict(cos float64 [Nv, rmax], tau float64 [Q], degree int32 [Nv],
+    out float64 [Nv, dout]).  edge_mask (uint8 [Nv, rmax]) replaces the
+    threshold rule when given."""
+    lib = _load()
+    vo = np.ascontiguousarray(vis_offsets, dtype=np.int32)
+    co = np.ascontiguousarray(chunk_offsets, dtype=np.int32)
+    hv, qh, hk, kh, vh = (np.ascontiguousarray(a, dtype=np.uint16) for a in (hv, qh, hk, kh, vh))
+    Q = vo.shape[0] - 1
+    Nv, dp = hv.shape
+    dh, dout = qh.shape[1], vh.shape[1]
+    em = None if edge_mask is None else np.ascontiguousarray(edge_mask, dtype=np.uint8)
+    cos = np.empty((Nv, rmax), np.float64)
+    tau = np.empty(Q, np.float64)
+    deg = np.empty(Nv, np.int32)
+    out = np.empty((Nv, dout), np.float64)
+    if lib.skip_oracle_bsca(_ptr(vo), _ptr(co), Q, _ptr(hv), _ptr(qh), _ptr(hk), _ptr(kh), _ptr(vh), dp, dh, dout,
+                            int(rmax), float(dbar), _ptr(em), _ptr(cos), _ptr(tau), _ptr(deg), _ptr(out)):
+        raise RuntimeError("oracle bsca failed")
+    return {"cos": cos, "tau": tau, "degree": deg, "out": out}

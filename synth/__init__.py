@@ -351,3 +351,31 @@ def make_qvs_inputs(B: int, L: int = QVS_L, d: int = QVS_D, seed: int = 5000, de
     bv = 0.01 * torch.randn(d, generator=g)
     wb = torch.randn(d, generator=g) / math.sqrt(d)
     return tokens.to(device), fq.to(device), wv.to(device), bv.to(device), wb.to(device)
+
+
+# ---- inputs of BSCA (App. B.3 Def. B.3) ------------------------------------
+#
+# BSCA fuses each question's retained visual tokens (P = ceil(rho_v L): 231
+# for rho_v = 0.4) with its verified chunks (R, ragged: what the SKV gate
+# keeps, 16..32 here) through projections h_v, h_k (width d_p), W_Q, W_K
+# (width d_h = 128, App. I.4) and W_V (width d_o).  The projected vectors are
+# the inputs here: Gaussian rows (unit norm for h_v / h_k, N(0, 1) entries
+# for the others), bf16; chunk counts U{16..32} per question (seeded).
+
+def make_bsca_inputs(Q: int, P: int, R_lo: int = 16, R_hi: int = 32, dp: int = 128, dh: int = 128,
+                     dout: int = 1024, seed: int = 6000, device="cpu"):
+    """dict(vis_offsets, chunk_offsets (int32 [Q+1]), hv [Nv, dp], qh [Nv, dh],
+    hk [Nc, dp], kh [Nc, dh], vh [Nc, dout] (bf16))."""
+    g = _gen(seed, "cpu")
+    counts_r = torch.randint(R_lo, R_hi + 1, (Q,), generator=g)
+    vo = offsets_from_counts(torch.full((Q,), P, dtype=torch.int64))
+    co = offsets_from_counts(counts_r)
+    Nv, Nc = int(vo[-1]), int(co[-1])
+    hv = _normalise(torch.randn(Nv, dp, generator=g))
+    hk = _normalise(torch.randn(Nc, dp, generator=g))
+    qh = torch.randn(Nv, dh, generator=g)
+    kh = torch.randn(Nc, dh, generator=g)
+    vh = torch.randn(Nc, dout, generator=g)
+    bf = lambda t: t.to(torch.bfloat16).to(device)
+    return {"vis_offsets": vo, "chunk_offsets": co, "hv": bf(hv), "qh": bf(qh), "hk": bf(hk), "kh": bf(kh),
+            "vh": bf(vh)}

@@ -19,7 +19,8 @@ def read_fixture(name):
                                        "vbar", "ids", "nu_all", "out_ids", "out_nu", "centroids",
                                        "codebook", "ivf_corpus", "queries", "codes", "p1k2_ids",
                                        "p1k2_scores", "p1k4_ids", "p1k4_scores", "p2k3_ids",
-                                       "p2k3_scores", "qvs_tokens", "wv"):
+                                       "p2k3_scores", "qvs_tokens", "wv", "hv", "hk", "qh", "kh", "vh",
+                                       "out1", "out2"):
             n = int(parts[1])
             rows = [[float(v) for v in lines[i + 1 + t].split()] for t in range(n)]
             out[key] = np.array(rows, dtype=np.float64)
