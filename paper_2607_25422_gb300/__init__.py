@@ -15,7 +15,9 @@ The SKV passage gate (App. B.4 Def. B.4; ``include/skip_skv.h``) then keeps
 the passages whose verification score nu reaches tau, at most
 ceil(rho |K|) of them.  The IVF-PQ variant (``include/skip_ivfpq.h``) builds
 and searches an inverted-file, product-quantised index of the corpus; QVS
-(``include/skip_qvs.h``) scores and prunes visual tokens before retrieval.
+(``include/skip_qvs.h``) scores and prunes visual tokens before retrieval;
+BSCA (``include/skip_bsca.h``) fuses the kept tokens with the verified
+chunks by attention over a sparse bipartite graph.
 """
 from __future__ import annotations
 
@@ -89,6 +91,10 @@ def load_library():
     lib.skip_qvs_count.argtypes = [i32, ctypes.c_float]
     lib.skip_qvs_count.restype = i32
     lib.skip_qvs_prune.argtypes = [P, P, i32, i32, P, ctypes.c_float, P, P, P, P, P]
+    lib.skip_bsca_create.argtypes = [i32, i32, i32, i32, i32, ctypes.POINTER(P)]
+    lib.skip_bsca_free.argtypes = [P]
+    lib.skip_bsca_run.argtypes = [P, i32, P, P, i32, P, P, P, P, P, ctypes.c_float, P, P, P, P, P]
+    lib.skip_bsca_sync_status.argtypes = [P, P]
     lib.skip_status_string.argtypes = [ctypes.c_int]
     lib.skip_status_string.restype = ctypes.c_char_p
     for f in ("skip_corpus_load", "skip_corpus_free", "skip_corpus_set_option", "skip_retrieve",
@@ -96,7 +102,8 @@ def load_library():
               "skip_timing_report", "skip_retrieve_regions_noalloc", "skip_skv_gate", "skip_retrieve_skv",
               "skip_ivfpq_build", "skip_ivfpq_load", "skip_ivfpq_lists", "skip_ivfpq_info", "skip_ivfpq_free",
               "skip_ivfpq_search_regions", "skip_ivfpq_search", "skip_ivfpq_sync_status", "skip_ivfpq_set_option",
-              "skip_ivfpq_timing_report", "skip_qvs_create", "skip_qvs_free", "skip_qvs_prune"):
+              "skip_ivfpq_timing_report", "skip_qvs_create", "skip_qvs_free", "skip_qvs_prune",
+              "skip_bsca_create", "skip_bsca_free", "skip_bsca_run", "skip_bsca_sync_status"):
         getattr(lib, f).restype = ctypes.c_int
     _lib = lib
     return lib
@@ -481,6 +488,56 @@ def skip_qvs_prune(head: QvsHead, tokens: torch.Tensor, fq: torch.Tensor, rho_v:
     return tuple(out)
 
 
+class BscaHandle:
+    """A BSCA workspace (``skip_bsca_t``)."""
+
+    def __init__(self, handle, dp, dh, dout):
+        self.handle, self.dp, self.dh, self.dout = handle, dp, dh, dout
+
+    def free(self):
+        if self.handle:
+            load_library().skip_bsca_free(self.handle)
+            self.handle = None
+
+    def __del__(self):
+        try:
+            self.free()
+        except Exception:
+            pass
+
+
+def skip_bsca_create(d_p: int, d_h: int, d_o: int, max_questions: int, max_tokens: int) -> BscaHandle:
+    h = ctypes.c_void_p()
+    _check(load_library().skip_bsca_create(int(d_p), int(d_h), int(d_o), int(max_questions), int(max_tokens),
+                                           ctypes.byref(h)), "skip_bsca_create")
+    return BscaHandle(h, d_p, d_h, d_o)
+
+
+def skip_bsca_run(handle: BscaHandle, vis_offsets: torch.Tensor, chunk_offsets: torch.Tensor, hv: torch.Tensor,
+                  qh: torch.Tensor, hk: torch.Tensor, kh: torch.Tensor, vh: torch.Tensor, dbar: float = 4.0,
+                  with_graph: bool = False, stream=None):
+    """Device tensors (bf16 projections, int32 offsets).  Returns out fp32
+    [Nv, d_o] and, with with_graph, (degree int32 [Nv], edges int64 [Nv]
+    neighbour bit masks, tau_e fp32 [Q])."""
+    vo = vis_offsets.to(torch.int32).contiguous()
+    co = chunk_offsets.to(torch.int32).contiguous()
+    hv, qh, hk, kh, vh = (t.contiguous() for t in (hv, qh, hk, kh, vh))
+    Q = vo.numel() - 1
+    Nv = hv.shape[0]
+    out = torch.empty(Nv, handle.dout, dtype=torch.float32, device=hv.device)
+    deg = torch.empty(Nv, dtype=torch.int32, device=hv.device) if with_graph else None
+    tau = torch.empty(Q, dtype=torch.float32, device=hv.device) if with_graph else None
+    edges = torch.empty(Nv, dtype=torch.int64, device=hv.device) if with_graph else None
+    _check(load_library().skip_bsca_run(handle.handle, Q, _ptr(vo), _ptr(co), Nv, _ptr(hv), _ptr(qh), _ptr(hk),
+                                        _ptr(kh), _ptr(vh), float(dbar), _ptr(out), _ptr(deg), _ptr(edges), _ptr(tau),
+                                        ctypes.c_void_p(_stream(stream))), "skip_bsca_run")
+    return (out, deg, edges, tau) if with_graph else out
+
+
+def skip_bsca_sync_status(handle: BscaHandle, stream=None) -> int:
+    return int(load_library().skip_bsca_sync_status(handle.handle, ctypes.c_void_p(_stream(stream))))
+
+
 def skip_sync_status(corpus: Corpus, stream=None) -> int:
     """Synchronise and return the status latched by the kernels (SKIP_OK, ...)."""
     return int(load_library().skip_sync_status(corpus.handle, ctypes.c_void_p(_stream(stream))))
@@ -501,4 +558,4 @@ def skip_timing_report(corpus: Corpus) -> dict:
 
 
 __all__ = [n for n in dir() if n.startswith("skip_") or n.startswith("SKIP_")] + [
-    "Corpus", "SkipError", "SkvMlp", "IvfIndex", "QvsHead", "load_library", "library_path"]
+    "Corpus", "SkipError", "SkvMlp", "IvfIndex", "QvsHead", "BscaHandle", "load_library", "library_path"]

@@ -16,6 +16,7 @@
 #include "../../include/skip_skv.h"
 #include "../../include/skip_ivfpq.h"
 #include "../../include/skip_qvs.h"
+#include "../../include/skip_bsca.h"
 #include "skip_internal.h"
 
 using namespace skipk;
@@ -1254,6 +1255,98 @@ skip_status_t skip_qvs_prune(skip_qvs_t q, const uint16_t *tokens, int32_t B, in
     if (e == cudaSuccess) e = launch_qvs_logits(p, q->sms, s);
     if (e == cudaSuccess) e = launch_qvs_select(p, s);
     return cuda_status(e);
+}
+
+}  // extern "C"
+
+// ---------------------------------------------------------------- BSCA
+
+struct skip_bsca {
+    int dp = 0, dh = 0, dout = 0, max_q = 0, max_t = 0;
+    float *cos = nullptr, *tau = nullptr;
+    int *err = nullptr;
+};
+
+namespace {
+
+void bsca_release(skip_bsca *b) {
+    if (!b) return;
+    cudaDeviceSynchronize();
+    cudaFree(b->cos);
+    cudaFree(b->tau);
+    cudaFree(b->err);
+    delete b;
+}
+
+}  // namespace
+
+extern "C" {
+
+skip_status_t skip_bsca_create(int32_t d_p, int32_t d_h, int32_t d_o, int32_t max_questions, int32_t max_tokens,
+                               skip_bsca_t *out) {
+    if (!out || d_p < 1 || d_h < 1 || d_o < 2 || max_questions < 1 || max_tokens < 1) return SKIP_EINVAL;
+    if (d_p > kBscaMaxDp || d_h > kBscaMaxDh || d_o > kBscaMaxDo || d_o % 2 != 0) return SKIP_EUNSUPPORTED;
+    int dev = 0, major = 0, minor = 0;
+    if (cudaGetDevice(&dev) != cudaSuccess) {
+        cudaGetLastError();
+        return SKIP_EUNSUPPORTED;
+    }
+    cudaDeviceGetAttribute(&major, cudaDevAttrComputeCapabilityMajor, dev);
+    cudaDeviceGetAttribute(&minor, cudaDevAttrComputeCapabilityMinor, dev);
+    if (major != 10 || minor != 3) return SKIP_EUNSUPPORTED;
+    auto *b = new skip_bsca();
+    b->dp = d_p, b->dh = d_h, b->dout = d_o, b->max_q = max_questions, b->max_t = max_tokens;
+    if (cudaMalloc(&b->cos, (size_t)max_tokens * kBscaMaxR * 4) != cudaSuccess ||
+        cudaMalloc(&b->tau, (size_t)max_questions * 4) != cudaSuccess ||
+        cudaMalloc(&b->err, sizeof(int)) != cudaSuccess || cudaMemset(b->err, 0, sizeof(int)) != cudaSuccess) {
+        cudaGetLastError();
+        bsca_release(b);
+        return SKIP_ENOMEM;
+    }
+    *out = b;
+    return SKIP_OK;
+}
+
+skip_status_t skip_bsca_free(skip_bsca_t b) {
+    bsca_release(b);
+    return SKIP_OK;
+}
+
+skip_status_t skip_bsca_run(skip_bsca_t b, int32_t Q, const int32_t *vis_offsets, const int32_t *chunk_offsets,
+                            int32_t total_tokens, const uint16_t *hv, const uint16_t *qh, const uint16_t *hk,
+                            const uint16_t *kh, const uint16_t *vh, float dbar, float *out, int32_t *degree,
+                            uint64_t *edges, float *tau_e, void *stream) {
+    if (!b || Q < 0 || Q > b->max_q || total_tokens < 0 || total_tokens > b->max_t) return SKIP_EINVAL;
+    if (!(dbar >= 0.f)) return SKIP_EINVAL;
+    if (Q > 0 && (!vis_offsets || !chunk_offsets || !hk || !kh || !vh)) return SKIP_EINVAL;
+    if (total_tokens > 0 && (!hv || !qh || !out)) return SKIP_EINVAL;
+    if (Q == 0) return SKIP_OK;
+    cudaStream_t s = reinterpret_cast<cudaStream_t>(stream);
+    BscaParams p;
+    p.Q = Q;
+    p.vis_offsets = vis_offsets;
+    p.chunk_offsets = chunk_offsets;
+    p.Nv = total_tokens;
+    p.hv = hv, p.qh = qh, p.hk = hk, p.kh = kh, p.vh = vh;
+    p.dp = b->dp, p.dh = b->dh, p.dout = b->dout;
+    p.dbar = dbar;
+    p.cos = b->cos;
+    p.tau = tau_e ? tau_e : b->tau;
+    p.degree = degree;
+    p.edges = edges;
+    p.out = out;
+    p.err = b->err;
+    return cuda_status(launch_bsca(p, s));
+}
+
+skip_status_t skip_bsca_sync_status(skip_bsca_t b, void *stream) {
+    if (!b) return SKIP_EINVAL;
+    if (cudaStreamSynchronize(reinterpret_cast<cudaStream_t>(stream)) != cudaSuccess) return SKIP_ECUDA;
+    int err = 0;
+    if (cudaMemcpy(&err, b->err, sizeof(int), cudaMemcpyDeviceToHost) != cudaSuccess) return SKIP_ECUDA;
+    if (err && cudaMemset(b->err, 0, sizeof(int)) != cudaSuccess) return SKIP_ECUDA;
+    if (err & kErrConfig) return SKIP_EINVAL;
+    return SKIP_OK;
 }
 
 }  // extern "C"

@@ -190,4 +190,27 @@ cudaError_t launch_qvs_u(const QvsParams &p, cudaStream_t s);
 cudaError_t launch_qvs_logits(const QvsParams &p, int sms, cudaStream_t s);
 cudaError_t launch_qvs_select(const QvsParams &p, cudaStream_t s);
 
+// ---- BSCA bipartite sparse cross-attention (k_bsca.cu) --------------------
+constexpr int kBscaMaxR = 64;     // chunks per question
+constexpr int kBscaMaxDp = 256;   // width of h_v / h_k
+constexpr int kBscaMaxDh = 256;   // width of W_Q / W_K
+constexpr int kBscaMaxDo = 2048;  // width of W_V
+struct BscaParams {
+    int Q;
+    const int32_t *vis_offsets;    // [Q + 1]
+    const int32_t *chunk_offsets;  // [Q + 1]
+    int64_t Nv;                    // visual tokens in all
+    const uint16_t *hv, *qh;       // bf16 [Nv x dp], [Nv x dh]
+    const uint16_t *hk, *kh, *vh;  // bf16 [Nc x dp], [Nc x dh], [Nc x dout]
+    int dp, dh, dout;              // dout even
+    float dbar;
+    float *cos;                    // [Nv x kBscaMaxR] workspace
+    float *tau;                    // [Q]
+    int32_t *degree;               // [Nv] or null
+    uint64_t *edges;               // [Nv] neighbour bit masks or null
+    float *out;                    // [Nv x dout]
+    int *err;
+};
+cudaError_t launch_bsca(const BscaParams &p, cudaStream_t s);
+
 }  // namespace skipk
