@@ -296,6 +296,96 @@ def ivfpq_report(args, spec, skip, c, ix, cent, reg_d, off_d, kernels, build_s, 
     }
 
 
+def run_bsca(args, spec, skip):
+    """BSCA bench: one question per workload question (Q), 231 retained visual
+    tokens (rho_v = 0.4 of 576), 16..32 verified chunks, d_p = d_h = 128,
+    d_o = 1024, mean degree --dbar.  Bound by the fp32 output it writes."""
+    world, rank, local = dist_setup()
+    dev = torch.device("cuda", torch.cuda.current_device())
+    Q, P, dp, dh, dout = spec.Q, 231, 128, 128, 1024
+    x = synth.make_bsca_inputs(Q, P, 16, 32, dp, dh, dout)
+    Nv, Nc = int(x["vis_offsets"][-1]), int(x["chunk_offsets"][-1])
+    xd = {k: v.to(dev).contiguous() for k, v in x.items()}
+    h = skip.skip_bsca_create(dp, dh, dout, Q, Nv)
+    stream = torch.cuda.current_stream()
+
+    def step():
+        return skip.skip_bsca_run(h, xd["vis_offsets"], xd["chunk_offsets"], xd["hv"], xd["qh"], xd["hk"], xd["kh"],
+                                  xd["vh"], args.dbar, stream=stream)
+    for _ in range(args.warmup):
+        step()
+    torch.cuda.synchronize()
+    sampler = ClockSampler(torch.cuda.current_device())
+    barrier(world)
+    torch.cuda.synchronize()
+    sampler.start()
+    time.sleep(0.3)
+    e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    e0.record(stream)
+    for _ in range(args.steps):
+        out = step()
+    e1.record(stream)
+    torch.cuda.synchronize()
+    clocks = sampler.stop()
+    ms = max_over_ranks(e0.elapsed_time(e1), world)
+    if skip.skip_bsca_sync_status(h) != skip.SKIP_OK:
+        raise SystemExit("bsca kernel status")
+    # end to end: host projections in, the fused tokens out
+    xh = {k: v.pin_memory() for k, v in x.items()}
+    out_h = torch.empty(Nv, dout, dtype=torch.float32).pin_memory()
+
+    def e2e_step():
+        for k in xd:
+            xd[k].copy_(xh[k], non_blocking=True)
+        o = step()
+        out_h.copy_(o, non_blocking=True)
+        stream.synchronize()
+    for _ in range(3):
+        e2e_step()
+    t0 = time.perf_counter()
+    for _ in range(args.steps):
+        e2e_step()
+    e2e_s = max_over_ranks(time.perf_counter() - t0, world)
+    peaks = load_peaks()
+    step_ms = ms / args.steps
+    in_bytes = Nv * (dp + dh) * 2 + Nc * (dp + dh + dout) * 2
+    step_bytes = in_bytes + Nv * dout * 4 + 2 * Nv * 64 * 4
+    achieved = step_bytes / (step_ms / 1e3) / 1e9
+    line = {
+        "metric": "BSCA questions/s (sparse visual-chunk fusion) [next row]",
+        "value": Q * world * args.steps / (ms / 1e3), "unit": "questions/s", "n_gpus": world, "steps": args.steps,
+        "warmup": args.warmup, "ms_per_step": step_ms, "higher_is_better": True, "scaling": "weak",
+        "vs_baseline": None, "dtype": "bf16 in, fp32 out", "data": "synthetic",
+        "config": {"workload": "bsca_%dq_%dtok" % (Q, P), "questions_per_gpu": Q, "visual_tokens": P,
+                   "chunks": "U{16..32}", "d_p": dp, "d_h": dh, "d_o": dout, "dbar": args.dbar,
+                   "l2": "output %.1f MB written per step" % (Nv * dout * 4 / 1e6)},
+        "roofline": {"bound": "hbm", "achieved": achieved, "peak": peaks["hbm_gbs"], "unit": "GB/s",
+                     "frac": achieved / peaks["hbm_gbs"], "traffic": None, "kernel": "bsca step (2 kernels)",
+                     "algorithmic_bytes_per_step": step_bytes, "peak_source": peaks["source"]},
+        "clocks": clocks,
+        "e2e": {"value": Q * world * args.steps / e2e_s, "unit": "questions/s", "h2d_bytes_per_step": in_bytes,
+                "d2h_bytes_per_step": Nv * dout * 4, "entry_point": "skip_bsca_run with pinned host copies"},
+        "gpu_launches": 2 * args.steps,
+    }
+    if rank == 0 and world == 1 and not args.no_cpu_baseline:
+        import oracle
+        nq = 4
+        sub = synth.make_bsca_inputs(nq, P, 16, 32, dp, dh, dout)
+        b = synth.bf16_bits
+        t0 = time.perf_counter()
+        oracle.bsca(sub["vis_offsets"], sub["chunk_offsets"], b(sub["hv"]), b(sub["qh"]), b(sub["hk"]), b(sub["kh"]),
+                    b(sub["vh"]), 64, args.dbar)
+        dt = time.perf_counter() - t0
+        line["cpu_baseline"] = {"value": nq / dt, "unit": "questions/s", "cores": 1, "kind": "oracle",
+                                "sample": "%d questions of the same shape (fp64, one thread)" % nq}
+    h.free()
+    if rank == 0:
+        print(json.dumps(line), flush=True)
+    if world > 1:
+        import torch.distributed as dist
+        dist.destroy_process_group()
+
+
 def run_qvs(args, spec, skip):
     """QVS bench: one image per question of the workload (B = Q), L = 576
     tokens of d = 1024, d_k = d, rho_v from --rho-v; HBM-bound token scan."""
@@ -409,6 +499,9 @@ def main():
     ap.add_argument("--qvs", action="store_true",
                     help="step = QVS token pruning of one image per question of the workload (576 x 1024 tokens)")
     ap.add_argument("--rho-v", type=float, default=0.4)
+    ap.add_argument("--bsca", action="store_true",
+                    help="step = BSCA of one question per workload question: 231 visual tokens x 16..32 chunks")
+    ap.add_argument("--dbar", type=float, default=4.0)
     ap.add_argument("--skv", action="store_true",
                     help="step = retrieval + SKV passage gate (skip_retrieve_skv), H = 512, tau 0.5, rho 0.6")
     ap.add_argument("--mma", default="auto", choices=["auto", "single", "pair"],
@@ -428,6 +521,9 @@ def main():
 
     if args.qvs:
         run_qvs(args, spec, skip)
+        return
+    if args.bsca:
+        run_bsca(args, spec, skip)
         return
     world, rank, local = dist_setup()
     dev = torch.device("cuda", torch.cuda.current_device())

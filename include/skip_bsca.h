@@ -23,8 +23,9 @@
  *
  * Device pointers; asynchronous and stream ordered; errors found by kernels
  * latched in the handle (skip_bsca_sync_status); no CPU fallback.  Limits:
- * at most 64 chunks per question (a question with more latches SKIP_EINVAL
- * and gets zero outputs), d_p and d_h at most 256, d_o even and at most 2048.
+ * at most 64 chunks and 32,768 (token, chunk) pairs per question (a
+ * question beyond either latches SKIP_EINVAL and gets zero outputs), d_p and
+ * d_h at most 256, d_o even and at most 2048.
  */
 #ifndef SKIP_BSCA_H
 #define SKIP_BSCA_H

@@ -195,6 +195,7 @@ constexpr int kBscaMaxR = 64;     // chunks per question
 constexpr int kBscaMaxDp = 256;   // width of h_v / h_k
 constexpr int kBscaMaxDh = 256;   // width of W_Q / W_K
 constexpr int kBscaMaxDo = 2048;  // width of W_V
+constexpr int kBscaMaxPairs = 32768;  // (visual token, chunk) pairs per question
 struct BscaParams {
     int Q;
     const int32_t *vis_offsets;    // [Q + 1]
