@@ -281,10 +281,11 @@ __global__ void __launch_bounds__(kTcThreads, 1)
             uint32_t *tau = p.tau + row;
             // The shared threshold is read one tile ahead, off the critical path.
             uint32_t tau_next = row_valid ? *reinterpret_cast<volatile uint32_t *>(tau) : 0u;
-            // Common case: no score of the 32 beats the threshold (a max and
-            // a compare).  Otherwise a branch-free bit mask of the survivors
-            // is walked in increasing column (= id) order, so that lanes
-            // without survivors idle for a few instructions only.
+            // Common case: no score of 64 columns beats the threshold of any
+            // row of the warp (a max and a warp vote).  Otherwise, per 32
+            // columns, a branch-free bit mask of the survivors is walked in
+            // increasing column (= id) order, so that lanes without
+            // survivors idle for a few instructions only.
             // One compare per score: s > thr and s >= gthr is s > cthr
             // (padding columns hold -inf and never pass).
             float gbelow = kNegInf, cthr = kNegInf;
@@ -310,7 +311,10 @@ __global__ void __launch_bounds__(kTcThreads, 1)
             };
             for (int64_t t = it.t0; t < it.t1; ++t, ++lt) {
                 const uint32_t buf = lt & 1u, use = lt >> 1;
-                if (!mbar_wait(smem_addr(&sh->tfull[buf]), use & 1u, p.timeout_ns)) {
+                // The warp gives up together, so that its vote below stays
+                // convergent.
+                const bool got = mbar_wait(smem_addr(&sh->tfull[buf]), use & 1u, p.timeout_ns);
+                if (!__all_sync(0xffffffffu, got)) {
                     ok = false;
                     break;
                 }
@@ -359,8 +363,11 @@ __global__ void __launch_bounds__(kTcThreads, 1)
                                 mbar_arrive(te);
                         }
                     }
-                    scan32(v0, id0);
-                    scan32(v1, id0 + 32);
+                    const float mx = fmaxf(fmax32(v0), fmax32(v1));
+                    if (__any_sync(0xffffffffu, row_valid && mx > cthr)) {
+                        scan32(v0, id0);
+                        scan32(v1, id0 + 32);
+                    }
                 }
             }
             if (row_valid) {

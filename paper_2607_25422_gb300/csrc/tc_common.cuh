@@ -108,15 +108,22 @@ __device__ __forceinline__ uint32_t select32(const uint32_t (&v)[32], int j) {
     return (j & 1) ? a[1] : a[0];
 }
 
+// Three-input maximum (one instruction on sm_100 and later).
+__device__ __forceinline__ float fmax3f(float a, float b, float c) {
+    float d;
+    asm("max.f32 %0, %1, %2, %3;" : "=f"(d) : "f"(a), "f"(b), "f"(c));
+    return d;
+}
+
 __device__ __forceinline__ float fmax32(const uint32_t (&v)[32]) {
-    float m[16];
+    float m[11];
 #pragma unroll
-    for (int j = 0; j < 16; ++j) m[j] = fmaxf(__uint_as_float(v[j]), __uint_as_float(v[j + 16]));
-#pragma unroll
-    for (int w = 8; w; w >>= 1)
-#pragma unroll
-        for (int j = 0; j < w; ++j) m[j] = fmaxf(m[j], m[j + w]);
-    return m[0];
+    for (int j = 0; j < 10; ++j)
+        m[j] = fmax3f(__uint_as_float(v[j]), __uint_as_float(v[j + 10]), __uint_as_float(v[j + 20]));
+    m[10] = fmaxf(__uint_as_float(v[30]), __uint_as_float(v[31]));
+    const float a = fmax3f(m[0], m[1], m[2]), b = fmax3f(m[3], m[4], m[5]), c = fmax3f(m[6], m[7], m[8]);
+    const float e = fmaxf(m[9], m[10]);
+    return fmaxf(fmax3f(a, b, c), e);
 }
 
 }  // namespace tc
