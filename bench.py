@@ -360,12 +360,12 @@ def run_bsca(args, spec, skip):
                    "chunks": "U{16..32}", "d_p": dp, "d_h": dh, "d_o": dout, "dbar": args.dbar,
                    "l2": "output %.1f MB written per step" % (Nv * dout * 4 / 1e6)},
         "roofline": {"bound": "hbm", "achieved": achieved, "peak": peaks["hbm_gbs"], "unit": "GB/s",
-                     "frac": achieved / peaks["hbm_gbs"], "traffic": None, "kernel": "bsca step (2 kernels)",
+                     "frac": achieved / peaks["hbm_gbs"], "traffic": None, "kernel": "bsca step (3 kernels)",
                      "algorithmic_bytes_per_step": step_bytes, "peak_source": peaks["source"]},
         "clocks": clocks,
         "e2e": {"value": Q * world * args.steps / e2e_s, "unit": "questions/s", "h2d_bytes_per_step": in_bytes,
                 "d2h_bytes_per_step": Nv * dout * 4, "entry_point": "skip_bsca_run with pinned host copies"},
-        "gpu_launches": 2 * args.steps,
+        "gpu_launches": 3 * args.steps,
     }
     if rank == 0 and world == 1 and not args.no_cpu_baseline:
         import oracle

@@ -19,7 +19,9 @@
  * [Nc x d_p], kh = W_K k [Nc x d_h], vh = W_V k [Nc x d_o], all bf16.
  * Questions own consecutive rows: question q's tokens are
  * [vis_offsets[q], vis_offsets[q+1]) and its chunks [chunk_offsets[q],
- * chunk_offsets[q+1]) (device int32 [Q + 1] each).  Sums and outputs fp32.
+ * chunk_offsets[q+1]) (device int32 [Q + 1] each), with vis_offsets[0] = 0
+ * and vis_offsets[Q] = total_tokens (rows outside every question's range
+ * are not written).  Sums and outputs fp32.
  *
  * Device pointers; asynchronous and stream ordered; errors found by kernels
  * latched in the handle (skip_bsca_sync_status); no CPU fallback.  Limits:

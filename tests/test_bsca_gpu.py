@@ -111,6 +111,9 @@ CASES = [
     (3, 100, 40, 64, 256, 64, 512, 2.5),
     (5, 20, 4, 6, 64, 32, 64, 100.0),
     (2, 50, 10, 20, 128, 128, 128, 0.0),
+    # widths that are not multiples of 4 / 8: the element-wise fallbacks
+    (4, 37, 3, 9, 50, 30, 62, 3.0),
+    (3, 90, 33, 40, 256, 256, 2048, 4.0),
 ]
 
 
