@@ -453,13 +453,13 @@ def run_qvs(args, spec, skip):
                    "rho_v": args.rho_v, "kept": n,
                    "l2": "tokens %.1f MB < L2: steady-state reads may hit L2" % (tok_bytes / 1e6)},
         "roofline": {"bound": "hbm", "achieved": achieved, "peak": peaks["hbm_gbs"], "unit": "GB/s",
-                     "frac": achieved / peaks["hbm_gbs"], "traffic": None, "kernel": "qvs step (5 kernels)",
+                     "frac": achieved / peaks["hbm_gbs"], "traffic": None, "kernel": "qvs step (3 kernels + 1 cuBLAS GEMM)",
                      "algorithmic_bytes_per_step": step_bytes, "peak_source": peaks["source"]},
         "clocks": clocks,
         "e2e": {"value": B * world * args.steps / e2e_s, "unit": "images/s",
                 "h2d_bytes_per_step": tok_bytes + B * d * 2, "d2h_bytes_per_step": B * n * 8,
                 "entry_point": "skip_qvs_prune with pinned host copies in and out"},
-        "gpu_launches": 5 * args.steps,
+        "gpu_launches": 3 * args.steps,
     }
     if rank == 0 and world == 1 and not args.no_cpu_baseline:
         import oracle

@@ -18,8 +18,10 @@
  * that fp32 rounding creates near 1 do not reorder tokens.
  *
  * Device pointers; calls are asynchronous and stream ordered; no CPU
- * fallback.  Limits: d a multiple of 8 and at most 8192, 1 <= d_k <= 4096,
- * 1 <= L <= 4096.
+ * fallback.  W_v^T f_q for all images is one bf16 GEMM with fp32 results
+ * that the library hands to cuBLAS (a handle per QVS object, set to the
+ * call's stream); every other step runs in the library's kernels.  Limits:
+ * d a multiple of 8 and at most 8192, 1 <= d_k <= 4096, 1 <= L <= 4096.
  */
 #ifndef SKIP_QVS_H
 #define SKIP_QVS_H

@@ -6,14 +6,13 @@
 // once: HBM-bound), and the ranking by s = sigmoid(logit) is the ranking by
 // the logit.
 //
-//  k_qvs_u       partial sums of W_v^T f_q and <f_q, b_v> per 32-wide slice
-//                of d_k, eight images per block (W_v read once per eight).
-//  k_qvs_ureduce the slices summed: u = sum / sqrt(d_k) + w_b, c likewise.
-//  k_qvs_logits  u in shared memory; one warp per four tokens at a time,
-//                16-byte loads.
+//  (library)     W_v^T f_q / sqrt(d_k) for all images at once: a plain bf16
+//                GEMM with fp32 results (cuBLAS), issued by the host code.
+//  k_qvs_logits  u = that + w_b in shared memory and c by one warp; one warp
+//                per four tokens at a time, 16-byte loads.
 //  k_qvs_select  per image: (logit, ~index) keys sorted descending in shared
 //                memory, the first n kept with their sigmoid scores.
-//  k_qvs_gather  (optional) the kept token rows copied out, a block per row.
+//  k_qvs_gather  (optional) the kept token rows copied out, a warp per row.
 #include <cuda_bf16.h>
 #include <cuda_runtime.h>
 
@@ -25,97 +24,26 @@
 namespace skipk {
 namespace {
 
-constexpr int kUImgs = 8, kUThreads = 128, kUSlice = 32, kUCols = 8;
-
-// Partial sums of W_v^T f_q over one 32-wide slice of d_k, for 8 columns of d
-// per thread (one 16-byte load of W_v per k) and eight images per block:
-// part[slice][b][j]; the c term likewise.
-__global__ void __launch_bounds__(kUThreads) k_qvs_u(const QvsParams p) {
-    __shared__ float fqs[kUImgs][kUSlice];
-    const int j0 = (blockIdx.x * kUThreads + threadIdx.x) * kUCols;
-    const int ks = blockIdx.y, k0 = ks * kUSlice;
-    const int b0 = blockIdx.z * kUImgs;
-    const int kn = min(kUSlice, p.dk - k0);
-    const __nv_bfloat16 *fq = reinterpret_cast<const __nv_bfloat16 *>(p.fq);
-    for (int e = threadIdx.x; e < kUImgs * kUSlice; e += kUThreads) {
-        const int u = e / kUSlice, k = e - u * kUSlice;
-        fqs[u][k] = (b0 + u < p.B && k < kn) ? __bfloat162float(fq[(int64_t)(b0 + u) * p.dk + k0 + k]) : 0.f;
-    }
-    __syncthreads();
-    if (j0 < p.d) {
-        const uint4 *wv = reinterpret_cast<const uint4 *>(reinterpret_cast<const __nv_bfloat16 *>(p.wv) +
-                                                          (int64_t)k0 * p.d + j0);
-        const int64_t wstride = p.d / 8;
-        float acc[kUImgs][kUCols];
-#pragma unroll
-        for (int u = 0; u < kUImgs; ++u)
-#pragma unroll
-            for (int c = 0; c < kUCols; ++c) acc[u][c] = 0.f;
-#pragma unroll 4
-        for (int k = 0; k < kn; ++k) {
-            const uint4 w4 = __ldg(wv + k * wstride);
-            const uint32_t wv4[4] = {w4.x, w4.y, w4.z, w4.w};
-            float w[kUCols];
-#pragma unroll
-            for (int h = 0; h < 4; ++h) {
-                const float2 f = __bfloat1622float2(*reinterpret_cast<const __nv_bfloat162 *>(&wv4[h]));
-                w[2 * h] = f.x;
-                w[2 * h + 1] = f.y;
-            }
-#pragma unroll
-            for (int u = 0; u < kUImgs; ++u) {
-                const float f = fqs[u][k];
-#pragma unroll
-                for (int c = 0; c < kUCols; ++c) acc[u][c] = fmaf(w[c], f, acc[u][c]);
-            }
-        }
-#pragma unroll
-        for (int u = 0; u < kUImgs; ++u)
-            if (b0 + u < p.B) {
-                float4 *dst = reinterpret_cast<float4 *>(p.u + ((int64_t)ks * p.B + b0 + u) * p.d + j0);
-                dst[0] = make_float4(acc[u][0], acc[u][1], acc[u][2], acc[u][3]);
-                dst[1] = make_float4(acc[u][4], acc[u][5], acc[u][6], acc[u][7]);
-            }
-    }
-    if (blockIdx.x == 0 && threadIdx.x < 32) {  // <f_q, b_v> over the slice, one warp, image by image
-        for (int u = 0; u < kUImgs && b0 + u < p.B; ++u) {
-            float s = (p.bv && (int)threadIdx.x < kn) ? fqs[u][threadIdx.x] * p.bv[k0 + threadIdx.x] : 0.f;
-#pragma unroll
-            for (int o = 16; o; o >>= 1) s += __shfl_xor_sync(0xFFFFFFFFu, s, o);
-            if (threadIdx.x == 0) p.c[ks * p.B + b0 + u] = s;
-        }
-    }
-}
-
-// u = (sum of the slices) / sqrt(d_k) + w_b and c likewise, written over
-// slice 0 (each thread reads all slices of its own element first).
-__global__ void __launch_bounds__(256) k_qvs_ureduce(const QvsParams p) {
-    const int64_t e = (int64_t)blockIdx.x * 256 + threadIdx.x;
-    const int ns = (p.dk + kUSlice - 1) / kUSlice;
-    const float inv = rsqrtf((float)p.dk);
-    if (e < (int64_t)p.B * p.d) {
-        const int64_t stride = (int64_t)p.B * p.d;
-        float v = 0.f;
-        for (int ks = 0; ks < ns; ++ks) v += p.u[ks * stride + e];
-        p.u[e] = v * inv + p.wb[e % p.d];
-    }
-    if (e < p.B) {
-        float c = 0.f;
-        for (int ks = 0; ks < ns; ++ks) c += p.c[ks * p.B + e];
-        p.c[e] = c * inv;
-    }
-}
-
 constexpr int kLogThreads = 256;
 
 __global__ void __launch_bounds__(kLogThreads) k_qvs_logits(const QvsParams p) {
     extern __shared__ float us[];  // [d]
+    __shared__ float cbs;
     const int b = blockIdx.y;
-    for (int t = threadIdx.x; t < p.d; t += kLogThreads) us[t] = p.u[(int64_t)b * p.d + t];
-    __syncthreads();
     const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+    // u = W_v^T f_q / sqrt(d_k) (the library GEMM) + w_b; c = <f_q, b_v> / sqrt(d_k)
+    for (int t = threadIdx.x; t < p.d; t += kLogThreads) us[t] = p.u[(int64_t)b * p.d + t] + p.wb[t];
+    if (warp == 0) {
+        const __nv_bfloat16 *fq = reinterpret_cast<const __nv_bfloat16 *>(p.fq) + (int64_t)b * p.dk;
+        float c = 0.f;
+        for (int k = lane; k < p.dk; k += 32) c = fmaf(__bfloat162float(fq[k]), p.bv[k], c);
+#pragma unroll
+        for (int o = 16; o; o >>= 1) c += __shfl_xor_sync(0xFFFFFFFFu, c, o);
+        if (lane == 0) cbs = c * rsqrtf((float)p.dk);
+    }
+    __syncthreads();
     const int nw = p.d / 8;  // 16-byte words per token
-    const float cb = p.c[b];
+    const float cb = cbs;
     // Four tokens per warp at a time: their loads are issued together.
     constexpr int kT = 4;
     const int wstep = gridDim.x * (kLogThreads / 32);
@@ -218,29 +146,33 @@ __global__ void __launch_bounds__(kSelThreads) k_qvs_select(const QvsParams p) {
 }
 
 // Kept token rows: one block per (rank, image), 16-byte copies.
-__global__ void __launch_bounds__(128) k_qvs_gather(const QvsParams p) {
-    const int r = blockIdx.x, b = blockIdx.y;
+constexpr int kGatherWarps = 8;
+
+__global__ void __launch_bounds__(32 * kGatherWarps) k_qvs_gather(const QvsParams p) {
+    const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+    const int r = blockIdx.x * kGatherWarps + warp, b = blockIdx.y;
+    if (r >= p.n) return;
     const int i = p.out_idx[(int64_t)b * p.n + r];
     const int nw = p.d / 8;
     const uint4 *src = reinterpret_cast<const uint4 *>(p.tokens) + ((int64_t)b * p.L + i) * nw;
     uint4 *dst = reinterpret_cast<uint4 *>(p.out_tokens) + ((int64_t)b * p.n + r) * nw;
-    for (int w = threadIdx.x; w < nw; w += 128) dst[w] = __ldg(src + w);
+    // four 16-byte words per lane in flight
+    for (int w0 = 0; w0 < nw; w0 += 128) {
+        uint4 x[4];
+#pragma unroll
+        for (int u = 0; u < 4; ++u) {
+            const int w = w0 + lane + 32 * u;
+            if (w < nw) x[u] = __ldg(src + w);
+        }
+#pragma unroll
+        for (int u = 0; u < 4; ++u) {
+            const int w = w0 + lane + 32 * u;
+            if (w < nw) dst[w] = x[u];
+        }
+    }
 }
 
 }  // namespace
-
-int qvs_u_slices(int dk) { return (dk + kUSlice - 1) / kUSlice; }
-
-cudaError_t launch_qvs_u(const QvsParams &p, cudaStream_t s) {
-    if (p.B == 0) return cudaSuccess;
-    dim3 grid((unsigned)((p.d / kUCols + kUThreads - 1) / kUThreads), (unsigned)((p.dk + kUSlice - 1) / kUSlice),
-              (unsigned)((p.B + kUImgs - 1) / kUImgs));
-    k_qvs_u<<<grid, kUThreads, 0, s>>>(p);
-    cudaError_t e = cudaGetLastError();
-    if (e != cudaSuccess) return e;
-    k_qvs_ureduce<<<(unsigned)(((int64_t)p.B * p.d + 255) / 256), 256, 0, s>>>(p);
-    return cudaGetLastError();
-}
 
 cudaError_t launch_qvs_logits(const QvsParams &p, int sms, cudaStream_t s) {
     if (p.B == 0) return cudaSuccess;
@@ -256,7 +188,7 @@ cudaError_t launch_qvs_select(const QvsParams &p, cudaStream_t s) {
     k_qvs_select<<<p.B, kSelThreads, 0, s>>>(p);
     cudaError_t e = cudaGetLastError();
     if (e != cudaSuccess || !p.out_tokens || p.n == 0) return e;
-    k_qvs_gather<<<dim3((unsigned)p.n, (unsigned)p.B), 128, 0, s>>>(p);
+    k_qvs_gather<<<dim3((unsigned)((p.n + kGatherWarps - 1) / kGatherWarps), (unsigned)p.B), 32 * kGatherWarps, 0, s>>>(p);
     return cudaGetLastError();
 }
 

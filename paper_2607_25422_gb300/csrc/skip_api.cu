@@ -1,12 +1,16 @@
 // C-ABI layer of the retrieval library: argument checks, the corpus copy and
 // its TMA descriptor, the per-handle workspace, the launch plan for each
 // regime and the error word.  The arithmetic lives in the kernels
-// (k_tc.cu, k_warpdot.cu, k_merge.cu); this file only decides what to launch.
+// (k_tc.cu, k_warpdot.cu, k_merge.cu and the others); this file only decides
+// what to launch, apart from QVS's projected query W_v^T f_q, a plain bf16
+// GEMM over all images that it hands to cuBLAS.
+#include <cublas_v2.h>
 #include <stdio.h>
 #include <stdlib.h>
 #include <string.h>
 
 #include <algorithm>
+#include <cmath>
 #include <map>
 #include <mutex>
 #include <string>
@@ -1162,7 +1166,8 @@ struct skip_qvs {
     int d = 0, dk = 0, max_b = 0, max_l = 0;
     uint16_t *wv = nullptr;
     float *bv = nullptr, *wb = nullptr;
-    float *u = nullptr, *c = nullptr, *logits = nullptr;  // workspace
+    float *u = nullptr, *logits = nullptr;  // workspace
+    cublasHandle_t blas = nullptr;          // the W_v^T f_q GEMM
 };
 
 namespace {
@@ -1174,8 +1179,8 @@ void qvs_release(skip_qvs *q) {
     cudaFree(q->bv);
     cudaFree(q->wb);
     cudaFree(q->u);
-    cudaFree(q->c);
     cudaFree(q->logits);
+    if (q->blas) cublasDestroy(q->blas);
     delete q;
 }
 
@@ -1204,12 +1209,16 @@ skip_status_t skip_qvs_create(const uint16_t *wv, const float *bv, const float *
     q->d = d, q->dk = dk, q->max_b = max_images, q->max_l = max_tokens;
     if (cudaMalloc(&q->wv, (size_t)dk * d * 2) != cudaSuccess || cudaMalloc(&q->bv, (size_t)dk * 4) != cudaSuccess ||
         cudaMalloc(&q->wb, (size_t)d * 4) != cudaSuccess ||
-        cudaMalloc(&q->u, (size_t)qvs_u_slices(dk) * max_images * d * 4) != cudaSuccess ||
-        cudaMalloc(&q->c, (size_t)qvs_u_slices(dk) * max_images * 4) != cudaSuccess ||
+        cudaMalloc(&q->u, (size_t)max_images * d * 4) != cudaSuccess ||
         cudaMalloc(&q->logits, (size_t)max_images * max_tokens * 4) != cudaSuccess) {
         cudaGetLastError();
         qvs_release(q);
         return SKIP_ENOMEM;
+    }
+    if (cublasCreate(&q->blas) != CUBLAS_STATUS_SUCCESS) {
+        q->blas = nullptr;
+        qvs_release(q);
+        return SKIP_ECUDA;
     }
     cudaStream_t s = reinterpret_cast<cudaStream_t>(stream);
     if (cudaMemcpyAsync(q->wv, wv, (size_t)dk * d * 2, cudaMemcpyDeviceToDevice, s) != cudaSuccess ||
@@ -1246,13 +1255,18 @@ skip_status_t skip_qvs_prune(skip_qvs_t q, const uint16_t *tokens, int32_t B, in
     p.wb = q->wb;
     p.B = B, p.L = L, p.d = q->d, p.dk = q->dk, p.n = n;
     p.u = q->u;
-    p.c = q->c;
     p.logits = logits ? logits : q->logits;
     p.out_idx = out_idx;
     p.out_score = out_score;
     p.out_tokens = out_tokens;
-    cudaError_t e = launch_qvs_u(p, s);
-    if (e == cudaSuccess) e = launch_qvs_logits(p, q->sms, s);
+    // U = F_q W_v / sqrt(d_k), row-major [B x d]: column-major U^T = W_v^T F_q^T
+    const float alpha = 1.f / std::sqrt((float)q->dk), beta = 0.f;
+    if (cublasSetStream(q->blas, s) != CUBLAS_STATUS_SUCCESS ||
+        cublasGemmEx(q->blas, CUBLAS_OP_N, CUBLAS_OP_N, q->d, B, q->dk, &alpha, q->wv, CUDA_R_16BF, q->d, fq,
+                     CUDA_R_16BF, q->dk, &beta, q->u, CUDA_R_32F, q->d, CUBLAS_COMPUTE_32F,
+                     CUBLAS_GEMM_DEFAULT) != CUBLAS_STATUS_SUCCESS)
+        return SKIP_ECUDA;
+    cudaError_t e = launch_qvs_logits(p, q->sms, s);
     if (e == cudaSuccess) e = launch_qvs_select(p, s);
     return cuda_status(e);
 }

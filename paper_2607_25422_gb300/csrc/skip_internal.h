@@ -178,15 +178,12 @@ struct QvsParams {
     const float *bv;        // [dk] or null
     const float *wb;        // [d]
     int B, L, d, dk, n;     // n tokens kept per image
-    float *u;               // [qvs_u_slices(dk) x B x d] workspace: partial sums
-    float *c;               // [qvs_u_slices(dk) x B] workspace: partial sums
+    float *u;               // [B x d] W_v^T f_q / sqrt(d_k) (written by the library GEMM)
     float *logits;          // [B x L] workspace
     int32_t *out_idx;       // [B x n]
     float *out_score;       // [B x n]
     void *out_tokens;       // bf16 [B x n x d] or null
 };
-int qvs_u_slices(int dk);  // d_k slices of the partial sums (workspace rows)
-cudaError_t launch_qvs_u(const QvsParams &p, cudaStream_t s);
 cudaError_t launch_qvs_logits(const QvsParams &p, int sms, cudaStream_t s);
 cudaError_t launch_qvs_select(const QvsParams &p, cudaStream_t s);
 
