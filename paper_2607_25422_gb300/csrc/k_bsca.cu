@@ -8,12 +8,14 @@
 //  k_bsca_cos     blocks (question, slice of its tokens): the question's h_k
 //                 rows normalised in shared memory (rows padded against bank
 //                 conflicts); a warp per four visual tokens, a lane per
-//                 chunk, computes their cosines into the workspace.
+//                 chunk, computes their cosines into the workspace and counts
+//                 each in the question's histogram.
 //  k_bsca_select  one block per question: tau_e = the m-th largest cosine of
-//                 the question by a 4 x 8-bit radix select on the
-//                 order-preserving integers of the values staged in shared
-//                 memory (a histogram per warp, increments aggregated over
-//                 lanes with equal digits).
+//                 the question: the bin that holds it from a 4,096-bin
+//                 histogram k_bsca_cos filled as it wrote the cosines, then
+//                 the rank inside that bin by counting over its few values
+//                 (a crowded bin falls back to a 4 x 8-bit radix select on
+//                 order-preserving integers).
 //  k_bsca_attend  blocks (question, slice of its tokens), a warp per visual
 //                 token: its neighbours are the chunks with cos >= tau_e;
 //                 e_ij = <q_i, k_j> / sqrt(d_h) for four neighbours at a time
@@ -61,6 +63,14 @@ __device__ __forceinline__ void slice_of(int P, int s, int S, int &ib, int &ie) 
     const int per = (P + S - 1) / S;
     ib = min(P, s * per);
     ie = min(P, ib + per);
+}
+
+// Histogram bin of a cosine: kBscaBins equal bins over [-1, 1], a
+// non-decreasing function of the value (the same float operations wherever
+// it is evaluated).
+__device__ __forceinline__ int cos_bin(float c) {
+    const int b = __float2int_rd((c + 1.f) * (float)(kBscaBins / 2));
+    return min(max(b, 0), kBscaBins - 1);
 }
 
 __global__ void __launch_bounds__(kCosThreads) k_bsca_cos(const BscaParams p, int S) {
@@ -136,45 +146,29 @@ __global__ void __launch_bounds__(kCosThreads) k_bsca_cos(const BscaParams p, in
             const float sv[4] = {s0, s1, s2, s3};
 #pragma unroll
             for (int k = 0; k < 4; ++k)
-                if (ia + k < ie) p.cos[(int64_t)(i0 + ia + k) * kBscaMaxR + j] = sv[k] * inv[k];
+                if (ia + k < ie) {
+                    const float c = sv[k] * inv[k];
+                    p.cos[(int64_t)(i0 + ia + k) * kBscaMaxR + j] = c;
+                    atomicAdd(p.hist + (int64_t)q * kBscaBins + cos_bin(c), 1u);
+                }
         }
         __syncwarp();
     }
 }
 
-__global__ void __launch_bounds__(kSelThreads) k_bsca_select(const BscaParams p) {
-    extern __shared__ float cs[];  // the question's P * R cosines
-    __shared__ uint32_t hist[kSelThreads / 32][256];
+constexpr int kCandCap = 2048;  // values of the threshold's bin resolved exactly
+
+// The m-th largest of cs[0, total) by a 4 x 8-bit radix select on the
+// order-preserving integers (a histogram per warp, increments aggregated
+// over lanes with equal digits); all threads of the block call it.
+__device__ float radix_select(const float *cs, int64_t total, int64_t m, uint32_t (*hist)[256]) {
     __shared__ uint32_t sel_prefix;
     __shared__ int sel_rank;
-    const int q = blockIdx.x;
-    const int i0 = p.vis_offsets[q], P = p.vis_offsets[q + 1] - i0;
-    const int R = p.chunk_offsets[q + 1] - p.chunk_offsets[q];
-    const float kInf = __int_as_float(0x7f800000);
-    if (!question_ok(P, R)) {
-        if (threadIdx.x == 0) p.tau[q] = kInf;  // no edges (flagged by k_bsca_cos)
-        return;
-    }
-    const int64_t total = (int64_t)P * R;
-    const double md = ceil((double)p.dbar * (double)P - 1e-3);
-    const int64_t m = md < 0.0 ? 0 : (int64_t)md;
-    if (m < 1 || total == 0) {
-        if (threadIdx.x == 0) p.tau[q] = kInf;
-        return;
-    }
-    if (m >= total) {
-        if (threadIdx.x == 0) p.tau[q] = -kInf;
-        return;
-    }
     const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
-    for (int r = warp; r < P; r += kSelThreads / 32)
-        for (int j = lane; j < R; j += 32) cs[r * R + j] = p.cos[(int64_t)(i0 + r) * kBscaMaxR + j];
     if (threadIdx.x == 0) {
         sel_prefix = 0;
         sel_rank = (int)m;
     }
-    // 4 x 8-bit radix select; a histogram per warp, increments aggregated over
-    // lanes with equal digits
     for (int pass = 0; pass < 4; ++pass) {
         const int shift = 24 - 8 * pass;
         for (int b = lane; b < 256; b += 32) hist[warp][b] = 0;
@@ -203,8 +197,7 @@ __global__ void __launch_bounds__(kSelThreads) k_bsca_select(const BscaParams p)
                 const int dd = 255 - blk * 32 - lane;
                 uint32_t c = 0;
                 for (int w = 0; w < kSelThreads / 32; ++w) c += hist[w][dd];
-                // inclusive prefix over lanes (descending digits)
-                uint32_t pre = c;
+                uint32_t pre = c;  // inclusive prefix over lanes (descending digits)
 #pragma unroll
                 for (int o = 1; o < 32; o <<= 1) {
                     const uint32_t v = __shfl_up_sync(0xFFFFFFFFu, pre, o);
@@ -228,7 +221,121 @@ __global__ void __launch_bounds__(kSelThreads) k_bsca_select(const BscaParams p)
         }
         __syncthreads();
     }
-    if (threadIdx.x == 0) p.tau[q] = score_of_ord(sel_prefix);
+    return score_of_ord(sel_prefix);
+}
+
+// tau_e of one question from the histogram k_bsca_cos built: the bin B that
+// holds the m-th largest cosine (a block-wide scan of the bin counts from the
+// top), then the values of bin B gathered and the one of the right rank
+// among them found by counting; a bin of more than kCandCap values falls
+// back to the radix select over all the question's cosines.  The histogram
+// row is cleared for the next call.
+__global__ void __launch_bounds__(kSelThreads) k_bsca_select(const BscaParams p) {
+    extern __shared__ float cs[];  // fallback: the question's P * R cosines
+    __shared__ uint32_t hs[kBscaBins];
+    __shared__ uint32_t hist[kSelThreads / 32][256];
+    __shared__ float cand[kCandCap];
+    __shared__ uint32_t wsum[kSelThreads / 32];
+    __shared__ int s_bin, s_rank, s_cnt, s_found;
+    __shared__ float s_tau;
+    const int q = blockIdx.x;
+    const int i0 = p.vis_offsets[q], P = p.vis_offsets[q + 1] - i0;
+    const int R = p.chunk_offsets[q + 1] - p.chunk_offsets[q];
+    const float kInf = __int_as_float(0x7f800000);
+    const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+    uint32_t *hrow = p.hist + (int64_t)q * kBscaBins;
+    for (int b = threadIdx.x; b < kBscaBins; b += kSelThreads) {
+        hs[b] = hrow[b];
+        hrow[b] = 0u;
+    }
+    if (!question_ok(P, R)) {
+        if (threadIdx.x == 0) p.tau[q] = kInf;  // no edges (flagged by k_bsca_cos)
+        return;
+    }
+    const int64_t total = (int64_t)P * R;
+    const double md = ceil((double)p.dbar * (double)P - 1e-3);
+    const int64_t m = md < 0.0 ? 0 : (int64_t)md;
+    if (m < 1 || total == 0) {
+        if (threadIdx.x == 0) p.tau[q] = kInf;
+        return;
+    }
+    if (m >= total) {
+        if (threadIdx.x == 0) p.tau[q] = -kInf;
+        return;
+    }
+    if (threadIdx.x == 0) {
+        s_bin = -1;
+        s_cnt = 0;
+        s_found = 0;
+    }
+    __syncthreads();
+    // thread t owns the kBscaBins / kSelThreads bins just below those of
+    // thread t - 1, counted from the top
+    constexpr int kPer = kBscaBins / kSelThreads;
+    const int top = kBscaBins - 1 - kPer * (int)threadIdx.x;
+    uint32_t mine = 0;
+#pragma unroll
+    for (int u = 0; u < kPer; ++u) mine += hs[top - u];
+    uint32_t incl = mine;  // inclusive scan over the warp's lanes
+#pragma unroll
+    for (int o = 1; o < 32; o <<= 1) {
+        const uint32_t v = __shfl_up_sync(0xFFFFFFFFu, incl, o);
+        if (lane >= o) incl += v;
+    }
+    if (lane == 31) wsum[warp] = incl;
+    __syncthreads();
+    uint32_t above = incl - mine;  // values in the bins above this thread's
+    for (int w = 0; w < warp; ++w) above += wsum[w];
+    if (above < (uint64_t)m && above + mine >= (uint64_t)m) {
+        uint32_t acc = above;
+        for (int u = 0; u < kPer; ++u) {
+            const int b = top - u;
+            if (acc + hs[b] >= (uint64_t)m) {
+                s_bin = b;
+                s_rank = (int)(m - acc);  // 1-based rank inside bin b, descending
+                break;
+            }
+            acc += hs[b];
+        }
+    }
+    __syncthreads();
+    const int B = s_bin, r = s_rank;
+    if (B >= 0 && hs[B] <= (uint32_t)kCandCap) {
+        for (int row = warp; row < P; row += kSelThreads / 32)
+            for (int j = lane; j < R; j += 32) {
+                const float c = p.cos[(int64_t)(i0 + row) * kBscaMaxR + j];
+                if (cos_bin(c) == B) {
+                    const int pos = atomicAdd(&s_cnt, 1);
+                    if (pos < kCandCap) cand[pos] = c;
+                }
+            }
+        __syncthreads();
+        const int n = min(s_cnt, kCandCap);
+        for (int a = threadIdx.x; a < n; a += kSelThreads) {
+            const float v = cand[a];
+            int before = 0;  // position of a in the descending order, ties by slot
+            for (int e = 0; e < n; ++e) {
+                const float x = cand[e];
+                before += (x > v) || (x == v && e < a);
+            }
+            if (before == r - 1) {
+                s_tau = v;
+                s_found = 1;
+            }
+        }
+        __syncthreads();
+        if (s_found) {
+            if (threadIdx.x == 0) p.tau[q] = s_tau;
+            return;
+        }
+    }
+    // a crowded bin (or counts that do not add up): the radix select over
+    // all the cosines
+    for (int row = warp; row < P; row += kSelThreads / 32)
+        for (int j = lane; j < R; j += 32) cs[row * R + j] = p.cos[(int64_t)(i0 + row) * kBscaMaxR + j];
+    __syncthreads();
+    const float t = radix_select(cs, total, m, hist);
+    if (threadIdx.x == 0) p.tau[q] = t;
 }
 
 // Output columns: slot u of a lane covers columns 8 * (lane + 32 u) .. + 7
@@ -446,7 +553,12 @@ cudaError_t launch_bsca(const BscaParams &p, cudaStream_t s) {
     e = cudaFuncSetAttribute(k_bsca_select, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem2);
     if (e != cudaSuccess) return e;
     k_bsca_select<<<(unsigned)p.Q, kSelThreads, smem2, s>>>(p);
-    if ((e = cudaGetLastError()) != cudaSuccess || p.Nv == 0) return e;
+    if ((e = cudaGetLastError()) != cudaSuccess) {
+        // the select clears the histograms; without it they must be cleared here
+        cudaMemsetAsync(p.hist, 0, (size_t)p.Q * kBscaBins * sizeof(uint32_t), s);
+        return e;
+    }
+    if (p.Nv == 0) return e;
     k_bsca_attend<<<(unsigned)(p.Q * S3), 32 * kAttWarps, 0, s>>>(p, S3);
     return cudaGetLastError();
 }

@@ -1278,6 +1278,7 @@ skip_status_t skip_qvs_prune(skip_qvs_t q, const uint16_t *tokens, int32_t B, in
 struct skip_bsca {
     int dp = 0, dh = 0, dout = 0, max_q = 0, max_t = 0;
     float *cos = nullptr, *tau = nullptr;
+    uint32_t *hist = nullptr;  // per-question cosine histograms, zero between calls
     int *err = nullptr;
 };
 
@@ -1287,6 +1288,7 @@ void bsca_release(skip_bsca *b) {
     if (!b) return;
     cudaDeviceSynchronize();
     cudaFree(b->cos);
+    cudaFree(b->hist);
     cudaFree(b->tau);
     cudaFree(b->err);
     delete b;
@@ -1312,6 +1314,8 @@ skip_status_t skip_bsca_create(int32_t d_p, int32_t d_h, int32_t d_o, int32_t ma
     b->dp = d_p, b->dh = d_h, b->dout = d_o, b->max_q = max_questions, b->max_t = max_tokens;
     if (cudaMalloc(&b->cos, (size_t)max_tokens * kBscaMaxR * 4) != cudaSuccess ||
         cudaMalloc(&b->tau, (size_t)max_questions * 4) != cudaSuccess ||
+        cudaMalloc(&b->hist, (size_t)max_questions * kBscaBins * 4) != cudaSuccess ||
+        cudaMemset(b->hist, 0, (size_t)max_questions * kBscaBins * 4) != cudaSuccess ||
         cudaMalloc(&b->err, sizeof(int)) != cudaSuccess || cudaMemset(b->err, 0, sizeof(int)) != cudaSuccess) {
         cudaGetLastError();
         bsca_release(b);
@@ -1345,6 +1349,7 @@ skip_status_t skip_bsca_run(skip_bsca_t b, int32_t Q, const int32_t *vis_offsets
     p.dp = b->dp, p.dh = b->dh, p.dout = b->dout;
     p.dbar = dbar;
     p.cos = b->cos;
+    p.hist = b->hist;
     p.tau = tau_e ? tau_e : b->tau;
     p.degree = degree;
     p.edges = edges;

@@ -193,6 +193,7 @@ constexpr int kBscaMaxDp = 256;   // width of h_v / h_k
 constexpr int kBscaMaxDh = 256;   // width of W_Q / W_K
 constexpr int kBscaMaxDo = 2048;  // width of W_V
 constexpr int kBscaMaxPairs = 32768;  // (visual token, chunk) pairs per question
+constexpr int kBscaBins = 4096;       // cosine histogram bins per question (over [-1, 1])
 struct BscaParams {
     int Q;
     const int32_t *vis_offsets;    // [Q + 1]
@@ -203,6 +204,7 @@ struct BscaParams {
     int dp, dh, dout;              // dout even
     float dbar;
     float *cos;                    // [Nv x kBscaMaxR] workspace
+    uint32_t *hist;                // [Q x kBscaBins] workspace, all zero between calls
     float *tau;                    // [Q]
     int32_t *degree;               // [Nv] or null
     uint64_t *edges;               // [Nv] neighbour bit masks or null

@@ -133,6 +133,20 @@ def test_full_size():
     print("full size: %d of %d tokens with the oracle's own neighbour set" % (n_ok, n))
 
 
+def test_crowded_bin():
+    """Every cosine equal (one h_v row and one h_k row repeated): more values
+    in the threshold's histogram bin than the exact step takes, so tau_e
+    comes from the radix select over all the question's cosines; ties at
+    tau_e are all kept."""
+    x = synth.make_bsca_inputs(2, 100, 30, 30, 64, 64, 128, seed=11)
+    x["hv"] = x["hv"][:1].repeat(x["hv"].shape[0], 1)
+    x["hk"] = x["hk"][:1].repeat(x["hk"].shape[0], 1)
+    out, deg, edges, tau, st = _gpu(x, 4.0, 64, 64, 128)
+    assert st == skip.SKIP_OK
+    np.testing.assert_array_equal(deg, np.full(200, 30, np.int32))
+    check(x, 4.0, (out, deg, edges, tau, st))
+
+
 def test_too_many_chunks_is_flagged():
     x = synth.make_bsca_inputs(2, 10, 70, 70, 64, 64, 64, seed=9)
     out, deg, edges, tau, st = _gpu(x, 4.0, 64, 64, 64)
