@@ -516,20 +516,25 @@ __global__ void __launch_bounds__(32 * kAttWarps) k_bsca_attend(const BscaParams
             }
         } else {
             // d_o not a multiple of 8, or unaligned rows: two columns per step
+            // (the loop runs the same number of times in every lane: the
+            // shuffle needs the whole warp)
             const int npair = p.dout / 2;
             float2 *o2 = reinterpret_cast<float2 *>(orow);
-            for (int pr = lane; pr < npair; pr += 32) {
+            for (int pr0 = 0; pr0 < npair; pr0 += 32) {
+                const int pr = pr0 + lane;
                 float2 acc = make_float2(0.f, 0.f);
                 int k = 0;
                 for (uint64_t mm = nb; mm; mm &= mm - 1, ++k) {
                     const int j = __ffsll((long long)mm) - 1;
                     const float w = __shfl_sync(0xFFFFFFFFu, k < 32 ? w0 : w1, k & 31);
-                    const float2 v = __bfloat1622float2(
-                        reinterpret_cast<const __nv_bfloat162 *>(p.vh + (int64_t)(j0 + j) * p.dout)[pr]);
-                    acc.x = fmaf(w, v.x, acc.x);
-                    acc.y = fmaf(w, v.y, acc.y);
+                    if (pr < npair) {
+                        const float2 v = __bfloat1622float2(
+                            reinterpret_cast<const __nv_bfloat162 *>(p.vh + (int64_t)(j0 + j) * p.dout)[pr]);
+                        acc.x = fmaf(w, v.x, acc.x);
+                        acc.y = fmaf(w, v.y, acc.y);
+                    }
                 }
-                o2[pr] = acc;
+                if (pr < npair) o2[pr] = acc;
             }
         }
     }
