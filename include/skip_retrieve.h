@@ -70,7 +70,10 @@ typedef enum {
     SKIP_OPT_GRID = 2,            /* score-kernel CTAs (0 = one per SM) */
     SKIP_OPT_TIMING = 3,          /* 1: time each kernel with CUDA events */
     SKIP_OPT_CLUSTER = 4,         /* single-CTA tensor path CTAs per cluster: 0 pick, 1, 2, 4, 8 */
-    SKIP_OPT_MMA = 5              /* tensor path MMA: 0 pick, 1 single CTA, 2 CTA pair */
+    SKIP_OPT_MMA = 5,             /* tensor path MMA: 0 pick, 1 single CTA, 2 CTA pair */
+    SKIP_OPT_BOUND = 6            /* bf16 tensor path: 0 auto (a bounding pass over every 32nd
+                                     corpus tile first when the corpus has at least 2,048
+                                     tiles), 1 never, 2 always */
 } skip_option_t;
 
 enum { SKIP_PATH_AUTO = 0, SKIP_PATH_TENSOR = 1, SKIP_PATH_WARP = 2, SKIP_PATH_LATENCY = 3 };

@@ -166,14 +166,15 @@ __global__ void __launch_bounds__(kTcThreads, 1)
                             const uint32_t fl = mapa_shared(fb, 0);
                             tma_load_2d_pair(smem_addr(sA + s * kABytes), &tq, fl, x, it.mb * kTcTileM);
                             tma_load_2d_pair(smem_addr(sB + s * Gm::kBBytes), &tx, fl, x,
-                                             (int)(t * kTcTileN) + rank * (kTcTileN / 2));
+                                             (int)(t * p.tile_stride * kTcTileN) + rank * (kTcTileN / 2));
                         } else {
                             tma_load_2d(smem_addr(sA + s * kABytes), &tq, fb, x, it.mb * kTcTileM);
                             if (CL == 1)
-                                tma_load_2d(smem_addr(sB + s * Gm::kBBytes), &tx, fb, x, (int)(t * kTcTileN));
+                                tma_load_2d(smem_addr(sB + s * Gm::kBBytes), &tx, fb, x,
+                                            (int)(t * p.tile_stride * kTcTileN));
                             else
                                 tma_load_2d_mc(smem_addr(sB + s * Gm::kBBytes + rank * slice_rows * 128), &tx, fb,
-                                               x, (int)(t * kTcTileN) + rank * slice_rows, mask);
+                                               x, (int)(t * p.tile_stride * kTcTileN) + rank * slice_rows, mask);
                         }
                         ++issued;
                         if (++s == S) {
@@ -280,7 +281,7 @@ __global__ void __launch_bounds__(kTcThreads, 1)
             uint32_t published = 0;
             uint32_t *tau = p.tau + row;
             // The shared threshold is read one tile ahead, off the critical path.
-            uint32_t tau_next = row_valid ? *reinterpret_cast<volatile uint32_t *>(tau) : 0u;
+            uint32_t tau_next = row_valid && p.share ? *reinterpret_cast<volatile uint32_t *>(tau) : 0u;
             // Common case: no score of 64 columns beats the threshold of any
             // row of the warp (a max and a warp vote).  Otherwise, per 32
             // columns, a branch-free bit mask of the survivors is walked in
@@ -319,7 +320,7 @@ __global__ void __launch_bounds__(kTcThreads, 1)
                     break;
                 }
                 tc_fence_after();
-                if (row_valid) {
+                if (row_valid && p.share) {
                     // Publish this chunk's k-th score, then adopt the row's best.
                     const uint32_t mine = top.n == p.k ? ord_of_score(thr) : 0u;
                     if (mine > published) {
@@ -333,7 +334,7 @@ __global__ void __launch_bounds__(kTcThreads, 1)
                     }
                     tau_next = *reinterpret_cast<volatile uint32_t *>(tau);
                 }
-                const int64_t n0 = t * kTcTileN;
+                const int64_t n0 = t * p.tile_stride * kTcTileN;
                 const bool tail = n0 + kTcTileN > p.N;
 #pragma unroll 1
                 for (int c = 0; c < kTcTileN / 64; ++c) {

@@ -103,6 +103,7 @@ struct skip_corpus {
     int grid = 0;
     int cluster = 0;           // 0 = pick; else CTAs per cluster
     int mma = 0;               // 0 = pick, 1 = single-CTA MMA, 2 = CTA-pair MMA
+    int bound = 0;             // bounding pass: 0 = by corpus size, 1 = never, 2 = always
     std::map<int, int> cluster_cache;  // resident clusters per (size, stages, list place)
     int timing = 0;
     // Timing: events recorded on the launching stream before each kernel and
@@ -172,6 +173,7 @@ struct Plan {
     int launches = 0;
     int stages = 0;
     bool list_in_smem = false;
+    bool bound = false;  // bounding pass over a sample of corpus tiles first
     int CL = 1;
     bool pair = false;
     bool latency = false;
@@ -312,6 +314,8 @@ skip_status_t run_regions(skip_corpus *c, const uint16_t *regions, int R, int k,
         if (!encode_bf16_rows(&tq, regions, R, c->d, kTcTileM)) return SKIP_ECUDA;
         if (!encode_e4m3_rows(&traw, c->rows, c->N, c->d)) return SKIP_ECUDA;
         TcParams p;
+        p.tile_stride = 1;
+        p.share = 1;
         p.N = c->N;
         p.d = c->d;
         p.R = R;
@@ -397,10 +401,29 @@ skip_status_t run_regions(skip_corpus *c, const uint16_t *regions, int R, int k,
         pl.grid = std::min(items, ncl) * cl_best;
         const size_t lists_bytes = (size_t)pl.G * pl.R_pad * k * sizeof(uint64_t);
         const size_t tau_bytes = align_up((size_t)pl.R_pad * sizeof(uint32_t), 256);
-        skip_status_t st = ensure_ws(c, align_up(ws_extra, 256) + tau_bytes + lists_bytes);
+        // Bounding pass: the same kernel over every kBoundStride-th corpus
+        // tile first; the merged sample top-k of each row is k ids whose
+        // scores (computed bit for bit as the full pass computes them) are at
+        // least its k-th key, so that score bounds the row's k-th best over
+        // the whole corpus from below and seeds the shared threshold.  The
+        // full pass's epilogue then admits far fewer keys.
+        // Each sample chunk keeps only its top k_s (about twice its share of
+        // k) with no bound shared between chunks, so its epilogue stays cheap
+        // on short streams; the k-th best of the union of the chunks' lists is
+        // still k distinct rows' scores, hence still a bound.
+        const int64_t stiles = (pl.tiles + kBoundStride - 1) / kBoundStride;
+        const bool bound = c->bound == 2 || (c->bound == 0 && pl.tiles >= kBoundMinTiles);
+        const int chunks_s = bound ? pick_chunks(QG, stiles, ncl) : 0;
+        const int k_s = bound ? std::min(k, std::max(4, (2 * k + chunks_s - 1) / chunks_s)) : 0;
+        const size_t lists_s_bytes = align_up((size_t)chunks_s * pl.R_pad * k_s * sizeof(uint64_t), 256);
+        const size_t keys_s_bytes = bound ? align_up((size_t)pl.R_pad * k * sizeof(uint64_t), 256) : 0;
+        skip_status_t st = ensure_ws(c, align_up(ws_extra, 256) + tau_bytes + align_up(lists_bytes, 256) +
+                                            lists_s_bytes + keys_s_bytes);
         if (st) return st;
         uint32_t *tau = reinterpret_cast<uint32_t *>((char *)c->ws + align_up(ws_extra, 256));
         uint64_t *lists = reinterpret_cast<uint64_t *>((char *)tau + tau_bytes);
+        uint64_t *lists_s = reinterpret_cast<uint64_t *>((char *)lists + align_up(lists_bytes, 256));
+        uint64_t *keys_s = reinterpret_cast<uint64_t *>((char *)lists_s + lists_s_bytes);
         if (keys_out) *keys_out = reg_keys = reinterpret_cast<uint64_t *>(c->ws);
         if (cudaMemsetAsync(tau, 0, tau_bytes, s) != cudaSuccess) return SKIP_ECUDA;
         CUtensorMap tq, tx;
@@ -408,6 +431,8 @@ skip_status_t run_regions(skip_corpus *c, const uint16_t *regions, int R, int k,
         if (!encode_bf16_rows(&tx, c->rows, c->N, c->d, pair ? kTcTileN / 2 : kTcTileN / cl_best))
             return SKIP_ECUDA;
         TcParams p;
+        p.tile_stride = 1;
+        p.share = 1;
         p.N = c->N;
         p.d = c->d;
         p.R = R;
@@ -426,11 +451,39 @@ skip_status_t run_regions(skip_corpus *c, const uint16_t *regions, int R, int k,
         p.list_in_smem = in_smem;
         p.scale = nullptr;
         p.raw_stages = 0;
+        p.tile_stride = 1;
         pl.stages = p.stages;
         pl.list_in_smem = in_smem;
-        record(c, s, "score_topk_tc");
         pl.pair = pair;
-        cudaError_t e = launch_tc(pair, tq, tx, p, pl.grid, s);
+        pl.bound = bound;
+        cudaError_t e;
+        if (bound) {
+            TcParams ps = p;
+            ps.tiles = stiles;
+            ps.tile_stride = kBoundStride;
+            ps.G = chunks_s;
+            ps.lists = lists_s;
+            ps.k = k_s;
+            ps.share = 0;
+            int st_s = 0;
+            bool smem_s = false;
+            tc_pick_layout(pair, k_s, c->max_smem, &st_s, &smem_s);
+            ps.stages = st_s;
+            ps.list_in_smem = smem_s;
+            record(c, s, "score_topk_tc_bound");
+            e = launch_tc(pair, tq, tx, ps, std::min(QG * chunks_s, ncl) * cl_best, s);
+            if (e != cudaSuccess) return cuda_status(e);
+            record(c, s, "merge_bound");
+            e = launch_merge_lists_len(lists_s, chunks_s, (int64_t)pl.R_pad * k_s, k_s, R, k, keys_s, nullptr,
+                                       nullptr, s);
+            if (e != cudaSuccess) return cuda_status(e);
+            record(c, s, "tau_bound");
+            e = launch_tau_from_keys(keys_s, R, k, tau, s);
+            if (e != cudaSuccess) return cuda_status(e);
+            pl.launches += 3;
+        }
+        record(c, s, "score_topk_tc");
+        e = launch_tc(pair, tq, tx, p, pl.grid, s);
         if (e != cudaSuccess) return cuda_status(e);
         ++pl.launches;
         record(c, s, "merge_lists");
@@ -480,11 +533,11 @@ void write_plan(skip_corpus *c, const Plan &pl, int R, int Q, int k, int K) {
     snprintf(c->plan, sizeof c->plan,
              "{\"path\": \"%s\", \"grid\": %d, \"lists_per_row\": %d, \"query_blocks\": %d, "
              "\"R_total\": %d, \"Q\": %d, \"k_region\": %d, \"K\": %d, \"launches\": %d, "
-             "\"stages\": %d, \"cluster\": %d, \"mma\": \"%s\", \"lists\": \"%s\"}",
+             "\"stages\": %d, \"cluster\": %d, \"mma\": \"%s\", \"lists\": \"%s\", \"bound\": %d}",
              pl.latency ? "latency" : pl.tensor ? "tensor" : "warpdot", pl.grid, pl.G, pl.MB, R, Q, k, K, pl.launches,
              pl.stages, pl.CL,
              pl.pair ? "pair" : "single",
-             pl.tensor ? (pl.list_in_smem ? "shared" : "global") : "global");
+             pl.tensor ? (pl.list_in_smem ? "shared" : "global") : "global", pl.bound ? 1 : 0);
 }
 
 // Argument rules of skip_retrieve.
@@ -694,6 +747,10 @@ skip_status_t skip_corpus_set_option(skip_corpus_t c, int option, int64_t value)
         case SKIP_OPT_CLUSTER:
             if (value != 0 && value != 1 && value != 2 && value != 4 && value != 8) return SKIP_EINVAL;
             c->cluster = (int)value;
+            return SKIP_OK;
+        case SKIP_OPT_BOUND:
+            if (value < 0 || value > 2) return SKIP_EINVAL;
+            c->bound = (int)value;
             return SKIP_OK;
     }
     return SKIP_EINVAL;

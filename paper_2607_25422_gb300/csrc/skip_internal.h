@@ -39,7 +39,11 @@ struct TcParams {
     int CL;           // CTAs per cluster (1, 2, 4, 8), one query block each
     int QG;           // query groups: ceil(MB / CL)
     int G;            // corpus chunks (lists per row)
-    int64_t tiles;    // corpus tiles of kTcTileN rows
+    int64_t tiles;    // corpus tiles of kTcTileN rows this launch visits
+    int tile_stride;  // bf16 kernel: item tile t is corpus tile t * tile_stride (1, or the
+                      // sample stride of a bounding pass)
+    int share;        // bf16 kernel: 1 = the chunks of a row share their k-th score through
+                      // tau; 0 in a bounding pass (its lists are shorter than the caller's k)
     uint64_t *lists;  // [G][R_pad][k]
     uint32_t *tau;    // [R_pad] shared per-row threshold (order-preserving ints), zeroed
     int *err;
@@ -53,6 +57,8 @@ constexpr int kTcTileM = 128;   // region rows per tile (TMEM lanes)
 constexpr int kTcTileN = 256;   // corpus rows per tile (TMEM columns)
 constexpr int kTcTileK = 64;    // bf16 elements per stage row (128 bytes)
 constexpr int kTcThreads = 192; // producer warp, MMA warp, 4 epilogue warps
+constexpr int kBoundStride = 32;     // bounding pass: every 32nd corpus tile (3% more MMA work)
+constexpr int kBoundMinTiles = 2048; // ... on corpora of at least 2,048 tiles (524,288 rows)
 // pair: CTA-pair MMA (cta_group::2, clusters of 2); else single-CTA MMA.
 size_t tc_smem_bytes(bool pair, int stages, int k, bool list_in_smem);
 // Deepest pipeline that fits next to shared-memory lists, else global lists.
@@ -96,9 +102,16 @@ cudaError_t launch_latency(bool fp8, const CUtensorMap &ta, const CUtensorMap &t
 // ---- merges -------------------------------------------------------------
 // Per-region merge of G sorted lists into the exact top-k (keys and/or
 // decoded ids/scores).
+// tau[row] = max(tau[row], the order-preserving integer of the score of key
+// keys[row * k + k - 1]) for rows with a k-th key: a sample's k-th best
+// score bounds the row's k-th best score over the whole corpus from below.
+cudaError_t launch_tau_from_keys(const uint64_t *keys, int R, int k, uint32_t *tau, cudaStream_t s);
 cudaError_t launch_merge_lists(const uint64_t *lists, int G, int64_t g_stride, int R, int k,
                                uint64_t *reg_keys, int64_t *reg_ids, float *reg_scores,
                                cudaStream_t s);
+// The same over lists of `len` keys each (len may differ from the k kept).
+cudaError_t launch_merge_lists_len(const uint64_t *lists, int G, int64_t g_stride, int len, int R, int k,
+                                   uint64_t *reg_keys, int64_t *reg_ids, float *reg_scores, cudaStream_t s);
 // Per-question union + dedup (max score) + top-K.
 // Offsets are clamped to [0, R]; a clamp sets kErrConfig in *err.
 cudaError_t launch_question_merge(const uint64_t *reg_keys, int k, const int32_t *offsets, int Q,

@@ -165,6 +165,33 @@ def test_pair_mma(case):
     assert_parity(cn, rn, offsets, k, K, gpu, truth)
 
 
+BOUND_CASES = [
+    # N, d, R, Q, k, K, mma
+    (70000, 768, 512, 32, 20, 50, 2),
+    (45000, 256, 300, 20, 100, 100, 2),
+    (30000, 128, 200, 10, 7, 16, 1),
+]
+
+
+@pytest.mark.parametrize("case", BOUND_CASES, ids=lambda c: "N%d_d%d_R%d_k%d_mma%d" % (c[0], c[1], c[2], c[4], c[6]))
+def test_bounding_pass(case):
+    """The bounding pass (every 32nd corpus tile first, its merged top-k
+    seeding each row's shared threshold) forced on: the oracle's results, and
+    exactly the same keys as without it."""
+    N, d, R, Q, k, K, mma = case
+    ct = synth.random_bf16(N, d, seed=N + 7)
+    rt = synth.random_bf16(R, d, seed=R + 13)
+    offsets = ragged_offsets(Q, R, seed=R + 1)
+    cn, rn = _bits(ct), _bits(rt)
+    truth = oracle_truth(cn, rn, offsets, k, K)
+    on = run_gpu(ct, rt, offsets, k, K, skip.SKIP_PATH_TENSOR, mma=mma, options=((skip.SKIP_OPT_BOUND, 2),))
+    off = run_gpu(ct, rt, offsets, k, K, skip.SKIP_PATH_TENSOR, mma=mma, options=((skip.SKIP_OPT_BOUND, 1),))
+    assert on[4]["bound"] == 1 and off[4]["bound"] == 0
+    assert_parity(cn, rn, offsets, k, K, on, truth)
+    for a, b in zip(on[:4], off[:4]):
+        np.testing.assert_array_equal(a, b)
+
+
 def test_clustered_near_ties():
     """Clustered rows put many candidates within 2e-3 of the k-th score."""
     spec = synth.WorkloadSpec("clustered_small", 11, 60000, 256, "bf16", 12, (1, 12), 20, 50, "clustered", 64)
