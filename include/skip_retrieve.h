@@ -73,7 +73,8 @@ typedef enum {
     SKIP_OPT_MMA = 5,             /* tensor path MMA: 0 pick, 1 single CTA, 2 CTA pair */
     SKIP_OPT_BOUND = 6            /* bf16 tensor path: 0 auto (a bounding pass over every 32nd
                                      corpus tile first when the corpus has at least 2,048
-                                     tiles), 1 never, 2 always */
+                                     tiles and the full pass would admit about one key per
+                                     thousand scores or more), 1 never, 2 always */
 } skip_option_t;
 
 enum { SKIP_PATH_AUTO = 0, SKIP_PATH_TENSOR = 1, SKIP_PATH_WARP = 2, SKIP_PATH_LATENCY = 3 };

@@ -411,8 +411,15 @@ skip_status_t run_regions(skip_corpus *c, const uint16_t *regions, int R, int k,
         // k) with no bound shared between chunks, so its epilogue stays cheap
         // on short streams; the k-th best of the union of the chunks' lists is
         // still k distinct rows' scores, hence still a bound.
+        // By default it runs where the full pass's epilogue would be busy: a
+        // row's chunks admit about G k (1 + ln(N / (G k))) keys without a
+        // bound (a running top-k over random order), and at one key per
+        // thousand scores or more the inserts, not the MMA, set the pace
+        // (clustered_1m: 3.4e-3, on; throughput_10m: 4e-4, off).
         const int64_t stiles = (pl.tiles + kBoundStride - 1) / kBoundStride;
-        const bool bound = c->bound == 2 || (c->bound == 0 && pl.tiles >= kBoundMinTiles);
+        const double gk = (double)pl.G * k;
+        const double ins_per_score = gk * (1.0 + std::log(std::max(1.0, (double)c->N / gk))) / (double)c->N;
+        const bool bound = c->bound == 2 || (c->bound == 0 && pl.tiles >= kBoundMinTiles && ins_per_score >= 1e-3);
         const int chunks_s = bound ? pick_chunks(QG, stiles, ncl) : 0;
         const int k_s = bound ? std::min(k, std::max(4, (2 * k + chunks_s - 1) / chunks_s)) : 0;
         const size_t lists_s_bytes = align_up((size_t)chunks_s * pl.R_pad * k_s * sizeof(uint64_t), 256);
