@@ -29,7 +29,7 @@ template <int LPL>
 __global__ void __launch_bounds__(kMergeWarps * 32)
     k_merge_lists(const uint64_t *__restrict__ lists, int G, int64_t g_stride, int len, int R, int k,
                   uint64_t *__restrict__ reg_keys, int64_t *__restrict__ reg_ids,
-                  float *__restrict__ reg_scores) {
+                  float *__restrict__ reg_scores, uint32_t *__restrict__ tau) {
     const int warp = threadIdx.x >> 5;
     const int row = blockIdx.x * kMergeWarps + warp;
     if (row >= R) return;
@@ -39,6 +39,8 @@ __global__ void __launch_bounds__(kMergeWarps * 32)
     float *sout = reg_scores ? reg_scores + (int64_t)row * k : nullptr;
     warp_merge_topk<LPL>(base, g_stride, G, len, k, [&](int i, uint64_t key) {
         if (kout) kout[i] = key;
+        // the k-th key's upper 32 bits are the order-preserving integer of its score
+        if (tau && i == k - 1 && key != 0ull) atomicMax(tau + row, (uint32_t)(key >> 32));
         if (iout) {
             int64_t id;
             float s;
@@ -148,38 +150,25 @@ __global__ void __launch_bounds__(kQThreads)
     }
 }
 
-// The k-th key of a row's merged sample list (its upper 32 bits are the
-// order-preserving integer of the score) raises the row's shared bound.
-__global__ void k_tau_from_keys(const uint64_t *__restrict__ keys, int R, int k, uint32_t *tau) {
-    const int row = blockIdx.x * blockDim.x + threadIdx.x;
-    if (row >= R) return;
-    const uint64_t key = keys[(int64_t)row * k + k - 1];
-    if (key != 0ull) atomicMax(tau + row, (uint32_t)(key >> 32));
-}
-
 }  // namespace
 
-cudaError_t launch_tau_from_keys(const uint64_t *keys, int R, int k, uint32_t *tau, cudaStream_t s) {
-    if (R <= 0) return cudaSuccess;
-    k_tau_from_keys<<<(R + 255) / 256, 256, 0, s>>>(keys, R, k, tau);
-    return cudaGetLastError();
-}
 
 cudaError_t launch_merge_lists_len(const uint64_t *lists, int G, int64_t g_stride, int len, int R, int k,
-                                   uint64_t *reg_keys, int64_t *reg_ids, float *reg_scores, cudaStream_t s) {
+                                   uint64_t *reg_keys, int64_t *reg_ids, float *reg_scores, uint32_t *tau,
+                                   cudaStream_t s) {
     if (R <= 0) return cudaSuccess;
     const int grid = (R + kMergeWarps - 1) / kMergeWarps;
     const int threads = kMergeWarps * 32;
     if (G <= 32)
-        k_merge_lists<1><<<grid, threads, 0, s>>>(lists, G, g_stride, len, R, k, reg_keys, reg_ids, reg_scores);
+        k_merge_lists<1><<<grid, threads, 0, s>>>(lists, G, g_stride, len, R, k, reg_keys, reg_ids, reg_scores, tau);
     else if (G <= 64)
-        k_merge_lists<2><<<grid, threads, 0, s>>>(lists, G, g_stride, len, R, k, reg_keys, reg_ids, reg_scores);
+        k_merge_lists<2><<<grid, threads, 0, s>>>(lists, G, g_stride, len, R, k, reg_keys, reg_ids, reg_scores, tau);
     else if (G <= 128)
-        k_merge_lists<4><<<grid, threads, 0, s>>>(lists, G, g_stride, len, R, k, reg_keys, reg_ids, reg_scores);
+        k_merge_lists<4><<<grid, threads, 0, s>>>(lists, G, g_stride, len, R, k, reg_keys, reg_ids, reg_scores, tau);
     else if (G <= 256)
-        k_merge_lists<8><<<grid, threads, 0, s>>>(lists, G, g_stride, len, R, k, reg_keys, reg_ids, reg_scores);
+        k_merge_lists<8><<<grid, threads, 0, s>>>(lists, G, g_stride, len, R, k, reg_keys, reg_ids, reg_scores, tau);
     else if (G <= 512)
-        k_merge_lists<16><<<grid, threads, 0, s>>>(lists, G, g_stride, len, R, k, reg_keys, reg_ids, reg_scores);
+        k_merge_lists<16><<<grid, threads, 0, s>>>(lists, G, g_stride, len, R, k, reg_keys, reg_ids, reg_scores, tau);
     else
         return cudaErrorInvalidValue;
     return cudaGetLastError();
@@ -188,7 +177,7 @@ cudaError_t launch_merge_lists_len(const uint64_t *lists, int G, int64_t g_strid
 cudaError_t launch_merge_lists(const uint64_t *lists, int G, int64_t g_stride, int R, int k,
                                uint64_t *reg_keys, int64_t *reg_ids, float *reg_scores,
                                cudaStream_t s) {
-    return launch_merge_lists_len(lists, G, g_stride, k, R, k, reg_keys, reg_ids, reg_scores, s);
+    return launch_merge_lists_len(lists, G, g_stride, k, R, k, reg_keys, reg_ids, reg_scores, nullptr, s);
 }
 
 int question_merge_capacity() { return kQCap; }

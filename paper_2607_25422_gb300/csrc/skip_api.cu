@@ -410,7 +410,8 @@ skip_status_t run_regions(skip_corpus *c, const uint16_t *regions, int R, int k,
         // Each sample chunk keeps only its top k_s (about twice its share of
         // k) with no bound shared between chunks, so its epilogue stays cheap
         // on short streams; the k-th best of the union of the chunks' lists is
-        // still k distinct rows' scores, hence still a bound.
+        // still k distinct rows' scores, hence still a bound.  The merge of
+        // the short lists raises each row's threshold itself.
         // By default it runs where the full pass's epilogue would be busy: a
         // row's chunks admit about G k (1 + ln(N / (G k))) keys without a
         // bound (a running top-k over random order), and at one key per
@@ -423,14 +424,12 @@ skip_status_t run_regions(skip_corpus *c, const uint16_t *regions, int R, int k,
         const int chunks_s = bound ? pick_chunks(QG, stiles, ncl) : 0;
         const int k_s = bound ? std::min(k, std::max(4, (2 * k + chunks_s - 1) / chunks_s)) : 0;
         const size_t lists_s_bytes = align_up((size_t)chunks_s * pl.R_pad * k_s * sizeof(uint64_t), 256);
-        const size_t keys_s_bytes = bound ? align_up((size_t)pl.R_pad * k * sizeof(uint64_t), 256) : 0;
         skip_status_t st = ensure_ws(c, align_up(ws_extra, 256) + tau_bytes + align_up(lists_bytes, 256) +
-                                            lists_s_bytes + keys_s_bytes);
+                                            lists_s_bytes);
         if (st) return st;
         uint32_t *tau = reinterpret_cast<uint32_t *>((char *)c->ws + align_up(ws_extra, 256));
         uint64_t *lists = reinterpret_cast<uint64_t *>((char *)tau + tau_bytes);
         uint64_t *lists_s = reinterpret_cast<uint64_t *>((char *)lists + align_up(lists_bytes, 256));
-        uint64_t *keys_s = reinterpret_cast<uint64_t *>((char *)lists_s + lists_s_bytes);
         if (keys_out) *keys_out = reg_keys = reinterpret_cast<uint64_t *>(c->ws);
         if (cudaMemsetAsync(tau, 0, tau_bytes, s) != cudaSuccess) return SKIP_ECUDA;
         CUtensorMap tq, tx;
@@ -481,13 +480,10 @@ skip_status_t run_regions(skip_corpus *c, const uint16_t *regions, int R, int k,
             e = launch_tc(pair, tq, tx, ps, std::min(QG * chunks_s, ncl) * cl_best, s);
             if (e != cudaSuccess) return cuda_status(e);
             record(c, s, "merge_bound");
-            e = launch_merge_lists_len(lists_s, chunks_s, (int64_t)pl.R_pad * k_s, k_s, R, k, keys_s, nullptr,
-                                       nullptr, s);
+            e = launch_merge_lists_len(lists_s, chunks_s, (int64_t)pl.R_pad * k_s, k_s, R, k, nullptr, nullptr,
+                                       nullptr, tau, s);
             if (e != cudaSuccess) return cuda_status(e);
-            record(c, s, "tau_bound");
-            e = launch_tau_from_keys(keys_s, R, k, tau, s);
-            if (e != cudaSuccess) return cuda_status(e);
-            pl.launches += 3;
+            pl.launches += 2;
         }
         record(c, s, "score_topk_tc");
         e = launch_tc(pair, tq, tx, p, pl.grid, s);

@@ -102,16 +102,16 @@ cudaError_t launch_latency(bool fp8, const CUtensorMap &ta, const CUtensorMap &t
 // ---- merges -------------------------------------------------------------
 // Per-region merge of G sorted lists into the exact top-k (keys and/or
 // decoded ids/scores).
-// tau[row] = max(tau[row], the order-preserving integer of the score of key
-// keys[row * k + k - 1]) for rows with a k-th key: a sample's k-th best
-// score bounds the row's k-th best score over the whole corpus from below.
-cudaError_t launch_tau_from_keys(const uint64_t *keys, int R, int k, uint32_t *tau, cudaStream_t s);
 cudaError_t launch_merge_lists(const uint64_t *lists, int G, int64_t g_stride, int R, int k,
                                uint64_t *reg_keys, int64_t *reg_ids, float *reg_scores,
                                cudaStream_t s);
-// The same over lists of `len` keys each (len may differ from the k kept).
+// The same over lists of `len` keys each (len may differ from the k kept);
+// with tau, also tau[row] = max(tau[row], the order-preserving integer of the
+// score of the row's k-th merged key) when it has one: a sample's k-th best
+// score bounds the row's k-th best score over the whole corpus from below.
 cudaError_t launch_merge_lists_len(const uint64_t *lists, int G, int64_t g_stride, int len, int R, int k,
-                                   uint64_t *reg_keys, int64_t *reg_ids, float *reg_scores, cudaStream_t s);
+                                   uint64_t *reg_keys, int64_t *reg_ids, float *reg_scores, uint32_t *tau,
+                                   cudaStream_t s);
 // Per-question union + dedup (max score) + top-K.
 // Offsets are clamped to [0, R]; a clamp sets kErrConfig in *err.
 cudaError_t launch_question_merge(const uint64_t *reg_keys, int k, const int32_t *offsets, int Q,
