@@ -30,6 +30,8 @@ __global__ void __launch_bounds__(kMergeWarps * 32)
     k_merge_lists(const uint64_t *__restrict__ lists, int G, int64_t g_stride, int len, int R, int k,
                   uint64_t *__restrict__ reg_keys, int64_t *__restrict__ reg_ids,
                   float *__restrict__ reg_scores, uint32_t *__restrict__ tau) {
+    grid_dep_wait();
+    grid_dep_launch();
     const int warp = threadIdx.x >> 5;
     const int row = blockIdx.x * kMergeWarps + warp;
     if (row >= R) return;
@@ -100,6 +102,8 @@ __global__ void __launch_bounds__(kQThreads)
                      int R, int K, int64_t *__restrict__ out_ids, float *__restrict__ out_scores,
                      int *__restrict__ err) {
     extern __shared__ uint64_t qsmem[];
+    grid_dep_wait();
+    grid_dep_launch();
     uint64_t *pool = qsmem;            // [kQCap] id-major keys
     uint64_t *ranked = qsmem + kQCap;  // [kQCap] ranking keys, negated for the ascending sort
     __shared__ int s_kept;
@@ -155,43 +159,62 @@ __global__ void __launch_bounds__(kQThreads)
 
 cudaError_t launch_merge_lists_len(const uint64_t *lists, int G, int64_t g_stride, int len, int R, int k,
                                    uint64_t *reg_keys, int64_t *reg_ids, float *reg_scores, uint32_t *tau,
-                                   cudaStream_t s) {
+                                   cudaStream_t s, bool pdl) {
     if (R <= 0) return cudaSuccess;
-    const int grid = (R + kMergeWarps - 1) / kMergeWarps;
-    const int threads = kMergeWarps * 32;
+    cudaLaunchConfig_t cfg = {};
+    cfg.gridDim = dim3((unsigned)((R + kMergeWarps - 1) / kMergeWarps), 1, 1);
+    cfg.blockDim = dim3(kMergeWarps * 32, 1, 1);
+    cfg.stream = s;
+    cudaLaunchAttribute attr[1];
+    attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+    attr[0].val.programmaticStreamSerializationAllowed = 1;
+    cfg.attrs = attr;
+    cfg.numAttrs = pdl ? 1 : 0;
     if (G <= 32)
-        k_merge_lists<1><<<grid, threads, 0, s>>>(lists, G, g_stride, len, R, k, reg_keys, reg_ids, reg_scores, tau);
-    else if (G <= 64)
-        k_merge_lists<2><<<grid, threads, 0, s>>>(lists, G, g_stride, len, R, k, reg_keys, reg_ids, reg_scores, tau);
-    else if (G <= 128)
-        k_merge_lists<4><<<grid, threads, 0, s>>>(lists, G, g_stride, len, R, k, reg_keys, reg_ids, reg_scores, tau);
-    else if (G <= 256)
-        k_merge_lists<8><<<grid, threads, 0, s>>>(lists, G, g_stride, len, R, k, reg_keys, reg_ids, reg_scores, tau);
-    else if (G <= 512)
-        k_merge_lists<16><<<grid, threads, 0, s>>>(lists, G, g_stride, len, R, k, reg_keys, reg_ids, reg_scores, tau);
-    else
-        return cudaErrorInvalidValue;
-    return cudaGetLastError();
+        return cudaLaunchKernelEx(&cfg, k_merge_lists<1>, lists, G, g_stride, len, R, k, reg_keys, reg_ids,
+                                  reg_scores, tau);
+    if (G <= 64)
+        return cudaLaunchKernelEx(&cfg, k_merge_lists<2>, lists, G, g_stride, len, R, k, reg_keys, reg_ids,
+                                  reg_scores, tau);
+    if (G <= 128)
+        return cudaLaunchKernelEx(&cfg, k_merge_lists<4>, lists, G, g_stride, len, R, k, reg_keys, reg_ids,
+                                  reg_scores, tau);
+    if (G <= 256)
+        return cudaLaunchKernelEx(&cfg, k_merge_lists<8>, lists, G, g_stride, len, R, k, reg_keys, reg_ids,
+                                  reg_scores, tau);
+    if (G <= 512)
+        return cudaLaunchKernelEx(&cfg, k_merge_lists<16>, lists, G, g_stride, len, R, k, reg_keys, reg_ids,
+                                  reg_scores, tau);
+    return cudaErrorInvalidValue;
 }
 
 cudaError_t launch_merge_lists(const uint64_t *lists, int G, int64_t g_stride, int R, int k,
                                uint64_t *reg_keys, int64_t *reg_ids, float *reg_scores,
-                               cudaStream_t s) {
-    return launch_merge_lists_len(lists, G, g_stride, k, R, k, reg_keys, reg_ids, reg_scores, nullptr, s);
+                               cudaStream_t s, bool pdl) {
+    return launch_merge_lists_len(lists, G, g_stride, k, R, k, reg_keys, reg_ids, reg_scores, nullptr, s, pdl);
 }
 
 int question_merge_capacity() { return kQCap; }
 
 cudaError_t launch_question_merge(const uint64_t *reg_keys, int k, const int32_t *offsets, int Q,
                                   int R, int K, int64_t *out_ids, float *out_scores, int *err,
-                                  cudaStream_t s) {
+                                  cudaStream_t s, bool pdl) {
     if (Q <= 0) return cudaSuccess;
     if (K + k > kQCap) return cudaErrorInvalidValue;
     const int smem = 2 * kQCap * (int)sizeof(uint64_t);
     cudaError_t e = cudaFuncSetAttribute(k_question_merge, cudaFuncAttributeMaxDynamicSharedMemorySize, smem);
     if (e != cudaSuccess) return e;
-    k_question_merge<<<Q, kQThreads, smem, s>>>(reg_keys, k, offsets, R, K, out_ids, out_scores, err);
-    return cudaGetLastError();
+    cudaLaunchConfig_t cfg = {};
+    cfg.gridDim = dim3((unsigned)Q, 1, 1);
+    cfg.blockDim = dim3(kQThreads, 1, 1);
+    cfg.dynamicSmemBytes = smem;
+    cfg.stream = s;
+    cudaLaunchAttribute attr[1];
+    attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+    attr[0].val.programmaticStreamSerializationAllowed = 1;
+    cfg.attrs = attr;
+    cfg.numAttrs = pdl ? 1 : 0;
+    return cudaLaunchKernelEx(&cfg, k_question_merge, reg_keys, k, offsets, R, K, out_ids, out_scores, err);
 }
 
 }  // namespace skipk

@@ -262,6 +262,10 @@ __global__ void __launch_bounds__(kTcThreads, 1)
         }
     } else {
         // ------------------------------------------------ epilogue
+        // The shared thresholds may come from the grid before this one (the
+        // bounding pass's merge, launched as its programmatic dependent):
+        // the TMA and MMA roles start at once, the epilogue waits for it.
+        grid_dep_wait();
         const int sub = warp & 3;
         const int rib = sub * 32 + lane;  // region row within the query block
         const uint32_t lane_addr = (uint32_t)(sub * 32) << 16;
@@ -400,7 +404,8 @@ size_t smem_bytes(int stages, int k, bool list_in_smem) {
            (list_in_smem ? (size_t)kTcTileM * k * 8 : 0) + sizeof(TcShared);
 }
 
-cudaLaunchConfig_t tc_config(int grid, int CL, size_t smem, cudaStream_t s, cudaLaunchAttribute *attr) {
+cudaLaunchConfig_t tc_config(int grid, int CL, size_t smem, cudaStream_t s, cudaLaunchAttribute *attr,
+                             bool pdl = false) {
     cudaLaunchConfig_t cfg = {};
     cfg.gridDim = dim3(grid, 1, 1);
     cfg.blockDim = dim3(kTcThreads, 1, 1);
@@ -410,8 +415,10 @@ cudaLaunchConfig_t tc_config(int grid, int CL, size_t smem, cudaStream_t s, cuda
     attr[0].val.clusterDim.x = CL;
     attr[0].val.clusterDim.y = 1;
     attr[0].val.clusterDim.z = 1;
+    attr[1].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+    attr[1].val.programmaticStreamSerializationAllowed = 1;
     cfg.attrs = attr;
-    cfg.numAttrs = 1;
+    cfg.numAttrs = pdl ? 2 : 1;
     return cfg;
 }
 
@@ -440,7 +447,7 @@ int tc_max_clusters(bool pair, int CL, int stages, int k, bool list_in_smem) {
         cudaGetLastError();
         return 0;
     }
-    cudaLaunchAttribute attr[1];
+    cudaLaunchAttribute attr[2];
     cudaLaunchConfig_t cfg = tc_config(CL * 64, CL, smem, 0, attr);
     int n = 0;
     if (cudaOccupancyMaxActiveClusters(&n, kern, &cfg) != cudaSuccess) {
@@ -451,14 +458,14 @@ int tc_max_clusters(bool pair, int CL, int stages, int k, bool list_in_smem) {
 }
 
 cudaError_t launch_tc(bool pair, const CUtensorMap &tq, const CUtensorMap &tx, const TcParams &p, int grid,
-                      cudaStream_t s) {
+                      cudaStream_t s, bool pdl) {
     if (pair && p.CL != 2) return cudaErrorInvalidValue;
     const size_t smem = tc_smem_bytes(pair, p.stages, p.k, p.list_in_smem != 0);
     auto kern = pair ? k_tc_score_topk<true> : k_tc_score_topk<false>;
     cudaError_t e = cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
     if (e != cudaSuccess) return e;
-    cudaLaunchAttribute attr[1];
-    cudaLaunchConfig_t cfg = tc_config(grid, p.CL, smem, s, attr);
+    cudaLaunchAttribute attr[2];
+    cudaLaunchConfig_t cfg = tc_config(grid, p.CL, smem, s, attr, pdl);
     return cudaLaunchKernelEx(&cfg, kern, tq, tx, p);
 }
 

@@ -284,7 +284,7 @@ skip_status_t run_regions(skip_corpus *c, const uint16_t *regions, int R, int k,
         if (e != cudaSuccess) return cuda_status(e);
         ++pl.launches;
         record(c, s, "merge_lists");
-        e = launch_merge_lists(lists, pl.G, (int64_t)R * k, R, k, reg_keys, reg_ids, reg_scores, s);
+        e = launch_merge_lists(lists, pl.G, (int64_t)R * k, R, k, reg_keys, reg_ids, reg_scores, s, true);
         if (e != cudaSuccess) return cuda_status(e);
         ++pl.launches;
         return SKIP_OK;
@@ -341,7 +341,7 @@ skip_status_t run_regions(skip_corpus *c, const uint16_t *regions, int R, int k,
         if (e != cudaSuccess) return cuda_status(e);
         ++pl.launches;
         record(c, s, "merge_lists");
-        e = launch_merge_lists(lists, pl.G, (int64_t)pl.R_pad * k, R, k, reg_keys, reg_ids, reg_scores, s);
+        e = launch_merge_lists(lists, pl.G, (int64_t)pl.R_pad * k, R, k, reg_keys, reg_ids, reg_scores, s, true);
         if (e != cudaSuccess) return cuda_status(e);
         ++pl.launches;
         return SKIP_OK;
@@ -481,16 +481,16 @@ skip_status_t run_regions(skip_corpus *c, const uint16_t *regions, int R, int k,
             if (e != cudaSuccess) return cuda_status(e);
             record(c, s, "merge_bound");
             e = launch_merge_lists_len(lists_s, chunks_s, (int64_t)pl.R_pad * k_s, k_s, R, k, nullptr, nullptr,
-                                       nullptr, tau, s);
+                                       nullptr, tau, s, true);
             if (e != cudaSuccess) return cuda_status(e);
             pl.launches += 2;
         }
         record(c, s, "score_topk_tc");
-        e = launch_tc(pair, tq, tx, p, pl.grid, s);
+        e = launch_tc(pair, tq, tx, p, pl.grid, s, bound);
         if (e != cudaSuccess) return cuda_status(e);
         ++pl.launches;
         record(c, s, "merge_lists");
-        e = launch_merge_lists(lists, pl.G, (int64_t)pl.R_pad * k, R, k, reg_keys, reg_ids, reg_scores, s);
+        e = launch_merge_lists(lists, pl.G, (int64_t)pl.R_pad * k, R, k, reg_keys, reg_ids, reg_scores, s, true);
         if (e != cudaSuccess) return cuda_status(e);
         ++pl.launches;
         return SKIP_OK;
@@ -526,7 +526,7 @@ skip_status_t run_regions(skip_corpus *c, const uint16_t *regions, int R, int k,
         ++pl.launches;
     }
     record(c, s, "merge_lists");
-    cudaError_t e = launch_merge_lists(lists, pl.G, (int64_t)R * k, R, k, reg_keys, reg_ids, reg_scores, s);
+    cudaError_t e = launch_merge_lists(lists, pl.G, (int64_t)R * k, R, k, reg_keys, reg_ids, reg_scores, s, true);
     if (e != cudaSuccess) return cuda_status(e);
     ++pl.launches;
     return SKIP_OK;
@@ -572,7 +572,7 @@ skip_status_t retrieve_impl(skip_corpus *c, const void *regions, const int32_t *
     if (Q > 0) {
         record(c, s, "question_merge");
         cudaError_t e = launch_question_merge(reg_keys, k_region, region_offsets, Q, R_total, K, out_ids,
-                                              out_scores, c->err, s);
+                                              out_scores, c->err, s, R_total > 0);
         if (e != cudaSuccess) return cuda_status(e);
         ++pl.launches;
     }

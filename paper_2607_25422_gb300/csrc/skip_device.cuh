@@ -142,6 +142,14 @@ __device__ __forceinline__ bool mbar_wait(uint32_t bar, uint32_t parity, uint64_
     }
 }
 
+// ---------------------------------------------------------------- PDL
+
+// Programmatic dependent launch: wait until the grids this one depends on
+// have completed and their writes are visible (returns at once for a launch
+// without the attribute), and let the next grid in the stream launch early.
+__device__ __forceinline__ void grid_dep_wait() { asm volatile("griddepcontrol.wait;" ::: "memory"); }
+__device__ __forceinline__ void grid_dep_launch() { asm volatile("griddepcontrol.launch_dependents;" ::: "memory"); }
+
 // ---------------------------------------------------------------- TMA
 
 __device__ __forceinline__ void tma_prefetch_desc(const void *map) {

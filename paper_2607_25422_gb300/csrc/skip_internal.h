@@ -65,8 +65,10 @@ size_t tc_smem_bytes(bool pair, int stages, int k, bool list_in_smem);
 void tc_pick_layout(bool pair, int k, int max_smem, int *stages, bool *list_in_smem);
 // Clusters of CL CTAs that can be resident at once with this layout.
 int tc_max_clusters(bool pair, int CL, int stages, int k, bool list_in_smem);
+// pdl: launched as the programmatic dependent of the kernel before it in the
+// stream (the epilogue waits for it before reading the shared thresholds).
 cudaError_t launch_tc(bool pair, const CUtensorMap &tq, const CUtensorMap &tx, const TcParams &p, int grid,
-                      cudaStream_t s);
+                      cudaStream_t s, bool pdl = false);
 
 // e4m3 corpus (single-CTA MMA, corpus widened to bf16 in shared memory).
 void tc_fp8_pick_layout(int k, int max_smem, int *stages, int *raw_stages, bool *list_in_smem);
@@ -101,22 +103,24 @@ cudaError_t launch_latency(bool fp8, const CUtensorMap &ta, const CUtensorMap &t
 
 // ---- merges -------------------------------------------------------------
 // Per-region merge of G sorted lists into the exact top-k (keys and/or
-// decoded ids/scores).
+// decoded ids/scores).  pdl (here and below): launched as the programmatic
+// dependent of the kernel just before it in the stream (the merge waits for
+// it before reading, and lets the next kernel launch early).
 cudaError_t launch_merge_lists(const uint64_t *lists, int G, int64_t g_stride, int R, int k,
                                uint64_t *reg_keys, int64_t *reg_ids, float *reg_scores,
-                               cudaStream_t s);
+                               cudaStream_t s, bool pdl = false);
 // The same over lists of `len` keys each (len may differ from the k kept);
 // with tau, also tau[row] = max(tau[row], the order-preserving integer of the
 // score of the row's k-th merged key) when it has one: a sample's k-th best
 // score bounds the row's k-th best score over the whole corpus from below.
 cudaError_t launch_merge_lists_len(const uint64_t *lists, int G, int64_t g_stride, int len, int R, int k,
                                    uint64_t *reg_keys, int64_t *reg_ids, float *reg_scores, uint32_t *tau,
-                                   cudaStream_t s);
+                                   cudaStream_t s, bool pdl = false);
 // Per-question union + dedup (max score) + top-K.
 // Offsets are clamped to [0, R]; a clamp sets kErrConfig in *err.
 cudaError_t launch_question_merge(const uint64_t *reg_keys, int k, const int32_t *offsets, int Q,
                                   int R, int K, int64_t *out_ids, float *out_scores, int *err,
-                                  cudaStream_t s);
+                                  cudaStream_t s, bool pdl = false);
 
 // ---- SKV passage gate (k_skv.cu) ------------------------------------------
 constexpr int kSkvHidden = 128;  // hidden units per CTA of the gate MLP (TMEM columns)
