@@ -38,7 +38,7 @@ namespace {
 
 constexpr int kCosThreads = 256;
 constexpr int kSelThreads = 512;
-constexpr int kAttWarps = 8;
+constexpr int kAttWarps = 4;
 
 __device__ __forceinline__ float bf16_at(const uint16_t *p, int64_t i) {
     return __uint_as_float((uint32_t)p[i] << 16);
