@@ -294,6 +294,23 @@ __global__ void __launch_bounds__(kTcThreads, 1)
             // One compare per score: s > thr and s >= gthr is s > cthr
             // (padding columns hold -inf and never pass).
             float gbelow = kNegInf, cthr = kNegInf;
+            // dense (a bounding pass with four-slot lists): the row's four
+            // largest scores of the chunk, kept sorted in registers
+            // (d4[0] >= .. >= d4[3]); each score that beats d4[3] is bubbled in
+            float d4[4] = {kNegInf, kNegInf, kNegInf, kNegInf};
+            auto dense32 = [&](const uint32_t (&vv)[32]) {
+#pragma unroll
+                for (int j = 0; j < 32; ++j) {
+                    const float x = __uint_as_float(vv[j]);
+                    const float m1 = fminf(d4[0], x);
+                    d4[0] = fmaxf(d4[0], x);
+                    const float m2 = fminf(d4[1], m1);
+                    d4[1] = fmaxf(d4[1], m1);
+                    const float m3 = fminf(d4[2], m2);
+                    d4[2] = fmaxf(d4[2], m2);
+                    d4[3] = fmaxf(d4[3], m3);
+                }
+            };
             auto scan32 = [&](uint32_t (&vv)[32], uint32_t id0) {
                 if (!row_valid) return;
                 const float mx = fmax32(vv);
@@ -369,13 +386,23 @@ __global__ void __launch_bounds__(kTcThreads, 1)
                         }
                     }
                     const float mx = fmaxf(fmax32(v0), fmax32(v1));
-                    if (__any_sync(0xffffffffu, row_valid && mx > cthr)) {
+                    if (p.dense) {
+                        if (__any_sync(0xffffffffu, row_valid && mx > d4[3])) {
+                            dense32(v0);
+                            dense32(v1);
+                        }
+                    } else if (__any_sync(0xffffffffu, row_valid && mx > cthr)) {
                         scan32(v0, id0);
                         scan32(v1, id0 + 32);
                     }
                 }
             }
-            if (row_valid) {
+            if (row_valid && p.dense) {
+                // scores only: the ids stand for four distinct rows of this chunk
+#pragma unroll
+                for (int t = 0; t < 4; ++t)
+                    glist[t] = d4[t] > kNegInf ? make_key(d4[t], (uint32_t)(it.g * 4 + t)) : 0ull;
+            } else if (row_valid) {
                 topk_sort(L, ls, top.n);
                 for (int t = 0; t < p.k; ++t) glist[t] = t < top.n ? L[t * ls] : 0ull;
             }

@@ -316,6 +316,7 @@ skip_status_t run_regions(skip_corpus *c, const uint16_t *regions, int R, int k,
         TcParams p;
         p.tile_stride = 1;
         p.share = 1;
+        p.dense = 0;
         p.N = c->N;
         p.d = c->d;
         p.R = R;
@@ -439,6 +440,7 @@ skip_status_t run_regions(skip_corpus *c, const uint16_t *regions, int R, int k,
         TcParams p;
         p.tile_stride = 1;
         p.share = 1;
+        p.dense = 0;
         p.N = c->N;
         p.d = c->d;
         p.R = R;
@@ -471,6 +473,7 @@ skip_status_t run_regions(skip_corpus *c, const uint16_t *regions, int R, int k,
             ps.lists = lists_s;
             ps.k = k_s;
             ps.share = 0;
+            ps.dense = k_s == 4;
             int st_s = 0;
             bool smem_s = false;
             tc_pick_layout(pair, k_s, c->max_smem, &st_s, &smem_s);

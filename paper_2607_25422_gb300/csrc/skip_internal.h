@@ -44,6 +44,8 @@ struct TcParams {
                       // sample stride of a bounding pass)
     int share;        // bf16 kernel: 1 = the chunks of a row share their k-th score through
                       // tau; 0 in a bounding pass (its lists are shorter than the caller's k)
+    int dense;        // bf16 kernel, bounding pass with k == 4: each row's four largest scores
+                      // of the chunk kept in registers (no ids; keys with stand-in ids)
     uint64_t *lists;  // [G][R_pad][k]
     uint32_t *tau;    // [R_pad] shared per-row threshold (order-preserving ints), zeroed
     int *err;

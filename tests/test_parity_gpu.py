@@ -170,6 +170,8 @@ BOUND_CASES = [
     (70000, 768, 512, 32, 20, 50, 2),
     (45000, 256, 300, 20, 100, 100, 2),
     (30000, 128, 200, 10, 7, 16, 1),
+    # 49 sample tiles in 12 chunks: four-slot lists kept in registers
+    (400000, 128, 256, 16, 20, 50, 2),
 ]
 
 
