@@ -667,11 +667,11 @@ def main():
                  "algorithmic_flops_per_launch": flops, "algorithmic_bytes_per_launch": corpus_bytes,
                  "step_roofline_frac": max(t_hbm, t_tc) / (secs / args.steps)})
     if kname and kname + "_bound" in kernels:
-        # the bounding pass (every 32nd corpus tile first) is extra work of the
+        # the bounding pass (every 48th corpus tile first) is extra work of the
         # step, outside the algorithmic count: reported, and in ms_per_step
         kb = kernels[kname + "_bound"]
         roof["bound_pass_ms"] = kb["ms"] / max(1, kb["launches"])
-        roof["kernel_note"] = ("full pass only; each call first runs a bounding pass over every 32nd "
+        roof["kernel_note"] = ("full pass only; each call first runs a bounding pass over every 48th "
                                "corpus tile (bound_pass_ms), counted in ms_per_step")
     line = {
         "metric": METRIC, "value": total_q / secs, "unit": "queries/s", "n_gpus": world,

@@ -71,7 +71,7 @@ typedef enum {
     SKIP_OPT_TIMING = 3,          /* 1: time each kernel with CUDA events */
     SKIP_OPT_CLUSTER = 4,         /* single-CTA tensor path CTAs per cluster: 0 pick, 1, 2, 4, 8 */
     SKIP_OPT_MMA = 5,             /* tensor path MMA: 0 pick, 1 single CTA, 2 CTA pair */
-    SKIP_OPT_BOUND = 6            /* bf16 tensor path: 0 auto (a bounding pass over every 32nd
+    SKIP_OPT_BOUND = 6            /* bf16 tensor path: 0 auto (a bounding pass over every 48th
                                      corpus tile first when the corpus has at least 2,048
                                      tiles and the full pass would admit about one key per
                                      thousand scores or more), 1 never, 2 always */

@@ -59,7 +59,7 @@ constexpr int kTcTileM = 128;   // region rows per tile (TMEM lanes)
 constexpr int kTcTileN = 256;   // corpus rows per tile (TMEM columns)
 constexpr int kTcTileK = 64;    // bf16 elements per stage row (128 bytes)
 constexpr int kTcThreads = 192; // producer warp, MMA warp, 4 epilogue warps
-constexpr int kBoundStride = 32;     // bounding pass: every 32nd corpus tile (3% more MMA work)
+constexpr int kBoundStride = 48;     // bounding pass: every 48th corpus tile (2% more MMA work)
 constexpr int kBoundMinTiles = 2048; // ... on corpora of at least 2,048 tiles (524,288 rows)
 // pair: CTA-pair MMA (cta_group::2, clusters of 2); else single-CTA MMA.
 size_t tc_smem_bytes(bool pair, int stages, int k, bool list_in_smem);

@@ -170,14 +170,14 @@ BOUND_CASES = [
     (70000, 768, 512, 32, 20, 50, 2),
     (45000, 256, 300, 20, 100, 100, 2),
     (30000, 128, 200, 10, 7, 16, 1),
-    # 49 sample tiles in 12 chunks: four-slot lists kept in registers
-    (400000, 128, 256, 16, 20, 50, 2),
+    # 33 sample tiles in 8 chunks, k = 16: four-slot lists kept in registers
+    (400000, 128, 256, 16, 16, 40, 2),
 ]
 
 
 @pytest.mark.parametrize("case", BOUND_CASES, ids=lambda c: "N%d_d%d_R%d_k%d_mma%d" % (c[0], c[1], c[2], c[4], c[6]))
 def test_bounding_pass(case):
-    """The bounding pass (every 32nd corpus tile first, its merged top-k
+    """The bounding pass (every 48th corpus tile first, its merged top-k
     seeding each row's shared threshold) forced on: the oracle's results, and
     exactly the same keys as without it."""
     N, d, R, Q, k, K, mma = case
