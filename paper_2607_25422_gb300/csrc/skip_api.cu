@@ -180,11 +180,14 @@ struct Plan {
 };
 
 // Corpus chunks G for the tensor path: make MB * G a whole number of waves of
-// `ctas` while keeping at least 4 tiles per item.
+// `ctas` while keeping at least 4 tiles per item where the corpus allows.
 int pick_chunks(int MB, int64_t tiles, int ctas) {
     int best = 1;
     double best_eff = -1.0;
-    const int gmax = (int)std::min<int64_t>(512, std::max<int64_t>(1, tiles / 4));
+    // At least 4 tiles per item, unless that leaves most CTAs idle (a small
+    // corpus, e.g. IVF centroids): then down to one tile per item.
+    const int64_t per = (int64_t)MB * std::max<int64_t>(1, tiles / 4) < ctas ? 1 : 4;
+    const int gmax = (int)std::min<int64_t>(512, std::max<int64_t>(1, tiles / per));
     for (int G = 1; G <= gmax; ++G) {
         const int64_t items = (int64_t)MB * G;
         const int64_t waves = (items + ctas - 1) / ctas;
