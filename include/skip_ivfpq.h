@@ -51,6 +51,10 @@ SKIP_API skip_status_t skip_ivfpq_build(skip_corpus_t corpus, const void *centro
  * list_offsets int64 [C + 1] (list l holds entries [off[l], off[l+1])),
  * ids int32 [N] and codes uint8 [N x M] in list order, centroids bf16
  * [C x d], codebook fp32 [M x 256 x d/M].  Returns after the copies.
+ * The index stores the codes in its own layout (blocks of 32 entries of a
+ * list, grouped by sub-space); skip_ivfpq_lists returns them in the row
+ * layout above.  Errors: SKIP_EINVAL also when the offsets are not
+ * 0 = off[0] <= off[1] <= ... <= off[C] = N.
  */
 SKIP_API skip_status_t skip_ivfpq_load(const void *centroids, int32_t C, int32_t d, const float *codebook,
                                        int32_t M, const int64_t *list_offsets, const int32_t *ids,
@@ -87,9 +91,10 @@ SKIP_API skip_status_t skip_ivfpq_search(skip_ivfpq_t index, const void *regions
 /* As skip_sync_status, for the index's kernels. */
 SKIP_API skip_status_t skip_ivfpq_sync_status(skip_ivfpq_t index, void *stream);
 
-/* Sets an option of the index's coarse search (skip_option_t of
- * skip_retrieve.h, applied to its centroid set); SKIP_OPT_TIMING records the
- * index's kernels, reported by skip_ivfpq_timing_report. */
+/* Sets an option of the index: SKIP_OPT_IVF_SPLIT for its list scan, any
+ * other skip_option_t of skip_retrieve.h for its coarse search (applied to
+ * its centroid set); SKIP_OPT_TIMING records the index's kernels, reported
+ * by skip_ivfpq_timing_report.  Results do not depend on the options. */
 SKIP_API skip_status_t skip_ivfpq_set_option(skip_ivfpq_t index, int option, int64_t value);
 SKIP_API skip_status_t skip_ivfpq_timing_report(skip_ivfpq_t index, char *buf, int32_t len);
 

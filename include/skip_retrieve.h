@@ -71,10 +71,14 @@ typedef enum {
     SKIP_OPT_TIMING = 3,          /* 1: time each kernel with CUDA events */
     SKIP_OPT_CLUSTER = 4,         /* single-CTA tensor path CTAs per cluster: 0 pick, 1, 2, 4, 8 */
     SKIP_OPT_MMA = 5,             /* tensor path MMA: 0 pick, 1 single CTA, 2 CTA pair */
-    SKIP_OPT_BOUND = 6            /* bf16 tensor path: 0 auto (a bounding pass over every 48th
+    SKIP_OPT_BOUND = 6,           /* bf16 tensor path: 0 auto (a bounding pass over every 48th
                                      corpus tile first when the corpus has at least 2,048
                                      tiles and the full pass would admit about one key per
                                      thousand scores or more), 1 never, 2 always */
+    SKIP_OPT_IVF_SPLIT = 7        /* IVF-PQ index only (skip_ivfpq_set_option): parts each
+                                     region's probed lists are cut into for the list scan,
+                                     0 pick (1, 2 or 4: doubled while twice the parts
+                                     still fit in the resident CTAs), else 1..8 */
 } skip_option_t;
 
 enum { SKIP_PATH_AUTO = 0, SKIP_PATH_TENSOR = 1, SKIP_PATH_WARP = 2, SKIP_PATH_LATENCY = 3 };

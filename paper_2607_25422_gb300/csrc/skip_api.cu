@@ -974,11 +974,14 @@ struct skip_ivfpq {
     int64_t N = 0;
     int d = 0, C = 0, M = 0, ds = 0;
     float *codebook = nullptr;    // [M x 256 x ds]
-    int64_t *offsets = nullptr;   // [C + 1]
+    float *cbT = nullptr;         // [256 x ds x Mp] (Mp = M rounded up to 32)
+    int64_t *offsets = nullptr;   // [C + 1] list starts (entries)
+    int64_t *boff = nullptr;      // [C + 1] list starts (blocks of 32 entries)
     int32_t *ids = nullptr;       // [N] list order
-    uint8_t *codes = nullptr;     // [N x M] list order
+    uint8_t *codes = nullptr;     // [boff[C] x M * 32] blocks of 32 entries (layout: k_ivfpq.cu il_offset)
     void *ws = nullptr;           // search workspace
     size_t ws_bytes = 0;
+    int split = 0;                // parts per region of the list scan (0: pick)
 };
 
 namespace {
@@ -988,7 +991,9 @@ void ivf_release(skip_ivfpq *ix) {
     cudaDeviceSynchronize();
     if (ix->cent) skip_corpus_free(ix->cent);
     cudaFree(ix->codebook);
+    cudaFree(ix->cbT);
     cudaFree(ix->offsets);
+    cudaFree(ix->boff);
     cudaFree(ix->ids);
     cudaFree(ix->codes);
     cudaFree(ix->ws);
@@ -1006,14 +1011,17 @@ skip_status_t ivf_create(const void *centroids, int C, int d, const float *codeb
         return st;
     }
     const size_t cb = (size_t)M * 256 * ix->ds * sizeof(float);
-    if (cudaMalloc(&ix->codebook, cb) != cudaSuccess || cudaMalloc(&ix->offsets, (size_t)(C + 1) * 8) != cudaSuccess ||
-        cudaMalloc(&ix->ids, (size_t)std::max<int64_t>(N, 1) * 4) != cudaSuccess ||
-        cudaMalloc(&ix->codes, (size_t)std::max<int64_t>(N, 1) * M) != cudaSuccess) {
+    const size_t cbt = (size_t)256 * ix->ds * ivf_padded_m(M) * sizeof(float);
+    if (cudaMalloc(&ix->codebook, cb) != cudaSuccess || cudaMalloc(&ix->cbT, cbt) != cudaSuccess ||
+        cudaMalloc(&ix->offsets, (size_t)(C + 1) * 8) != cudaSuccess ||
+        cudaMalloc(&ix->boff, (size_t)(C + 1) * 8) != cudaSuccess ||
+        cudaMalloc(&ix->ids, (size_t)std::max<int64_t>(N, 1) * 4) != cudaSuccess) {
         cudaGetLastError();
         ivf_release(ix);
         return SKIP_ENOMEM;
     }
-    if (cudaMemcpyAsync(ix->codebook, codebook, cb, cudaMemcpyDeviceToDevice, s) != cudaSuccess) {
+    if (cudaMemcpyAsync(ix->codebook, codebook, cb, cudaMemcpyDeviceToDevice, s) != cudaSuccess ||
+        launch_pq_codebook_t(ix->codebook, M, ix->ds, ix->cbT, s) != cudaSuccess) {
         ivf_release(ix);
         return SKIP_ECUDA;
     }
@@ -1035,26 +1043,64 @@ IvfParams ivf_params(const skip_ivfpq *ix) {
     p.centroids = ix->cent->rows;
     p.C = ix->C;
     p.codebook = ix->codebook;
+    p.cbT = ix->cbT;
     p.M = ix->M;
     p.ds = ix->ds;
     p.offsets = ix->offsets;
+    p.boff = ix->boff;
     p.ids = ix->ids;
     p.codes = ix->codes;
     return p;
 }
 
-// Coarse probes then the list scan: top-k keys per region into the head of
-// the index workspace.
+// Checks the list offsets (0 = off[0] <= ... <= off[C] = N), derives the
+// block offsets and stores `rows` (codes in list order, one row of M bytes
+// per entry; device) in blocks of 32 entries.  Returns after the copy.
+skip_status_t ivf_layout(skip_ivfpq *ix, const uint8_t *rows, cudaStream_t s) {
+    const int C = ix->C;
+    std::vector<int64_t> off((size_t)C + 1), boff((size_t)C + 1);
+    if (cudaMemcpyAsync(off.data(), ix->offsets, (size_t)(C + 1) * 8, cudaMemcpyDeviceToHost, s) != cudaSuccess ||
+        cudaStreamSynchronize(s) != cudaSuccess)
+        return SKIP_ECUDA;
+    if (off[0] != 0 || off[C] != ix->N) return SKIP_EINVAL;
+    boff[0] = 0;
+    for (int l = 0; l < C; ++l) {
+        if (off[l + 1] < off[l]) return SKIP_EINVAL;
+        boff[l + 1] = boff[l] + (off[l + 1] - off[l] + 31) / 32;
+    }
+    const size_t bytes = (size_t)std::max<int64_t>(boff[C], 1) * 32 * ix->M;
+    if (cudaMalloc(&ix->codes, bytes) != cudaSuccess) {
+        cudaGetLastError();
+        return SKIP_ENOMEM;
+    }
+    if (cudaMemcpyAsync(ix->boff, boff.data(), (size_t)(C + 1) * 8, cudaMemcpyHostToDevice, s) != cudaSuccess ||
+        cudaMemsetAsync(ix->codes, 0, bytes, s) != cudaSuccess ||
+        launch_ivf_interleave(ivf_params(ix), rows, ix->codes, ix->cent->sm_count, s) != cudaSuccess ||
+        cudaStreamSynchronize(s) != cudaSuccess)
+        return SKIP_ECUDA;
+    return SKIP_OK;
+}
+
+// Coarse probes then the list scan: top-k keys of each of the G parts of
+// each region ([G x R x k], the head of the index workspace), and room for
+// R x k merged keys after them (*merged).
 skip_status_t ivf_regions(skip_ivfpq *ix, const void *regions, int R, int nprobe, int k, cudaStream_t s,
-                          uint64_t **keys_out) {
+                          uint64_t **keys_out, uint64_t **merged, int *G_out) {
+    int G = 1;
+    if (R > 0) {
+        skip_status_t st = cuda_status(ivfpq_scan_split(ix->M, nprobe, R, ix->cent->sm_count, ix->split, &G));
+        if (st) return st;
+    }
     const size_t pid = align_up((size_t)R * nprobe * 8, 256), psc = align_up((size_t)R * nprobe * 4, 256);
     const size_t kb = align_up((size_t)std::max(R, 1) * k * 8, 256);
-    skip_status_t st = ensure_buf(ix->ws, ix->ws_bytes, kb + pid + psc);
+    skip_status_t st = ensure_buf(ix->ws, ix->ws_bytes, (G + 1) * kb + pid + psc);
     if (st) return st;
     uint64_t *keys = reinterpret_cast<uint64_t *>(ix->ws);
-    int64_t *probe_ids = reinterpret_cast<int64_t *>((char *)ix->ws + kb);
-    float *probe_sc = reinterpret_cast<float *>((char *)ix->ws + kb + pid);
+    int64_t *probe_ids = reinterpret_cast<int64_t *>((char *)ix->ws + (G + 1) * kb);
+    float *probe_sc = reinterpret_cast<float *>((char *)ix->ws + (G + 1) * kb + pid);
     *keys_out = keys;
+    *merged = reinterpret_cast<uint64_t *>((char *)ix->ws + G * kb);
+    *G_out = G;
     if (R == 0) return SKIP_OK;
     Plan pl;
     st = run_regions(ix->cent, reinterpret_cast<const uint16_t *>(regions), R, nprobe, nullptr, probe_ids, probe_sc,
@@ -1062,7 +1108,7 @@ skip_status_t ivf_regions(skip_ivfpq *ix, const void *regions, int R, int nprobe
     if (st) return st;
     record(ix->cent, s, "ivfpq_scan");
     cudaError_t e = launch_ivfpq_scan(ivf_params(ix), reinterpret_cast<const uint16_t *>(regions), R, probe_ids,
-                                      probe_sc, nprobe, k, keys, ix->cent->sm_count, s);
+                                      probe_sc, nprobe, k, G, keys, ix->cent->sm_count, s);
     return cuda_status(e);
 }
 
@@ -1091,7 +1137,7 @@ skip_status_t skip_ivfpq_build(skip_corpus_t c, const void *centroids, int32_t C
     void *tmp = nullptr;
     const size_t rl = align_up((size_t)N * 8, 256), rs = align_up((size_t)N * 4, 256);
     const size_t cr = align_up((size_t)N * M, 256), cc = align_up((size_t)C * 8, 256);
-    if (cudaMalloc(&tmp, rl + rs + cr + 2 * cc) != cudaSuccess) {
+    if (cudaMalloc(&tmp, rl + rs + 2 * cr + 2 * cc) != cudaSuccess) {
         cudaGetLastError();
         ivf_release(ix);
         return SKIP_ENOMEM;
@@ -1101,6 +1147,7 @@ skip_status_t skip_ivfpq_build(skip_corpus_t c, const void *centroids, int32_t C
     uint8_t *codes_rows = reinterpret_cast<uint8_t *>((char *)tmp + rl + rs);
     int64_t *counts = reinterpret_cast<int64_t *>((char *)tmp + rl + rs + cr);
     int64_t *cursor = reinterpret_cast<int64_t *>((char *)tmp + rl + rs + cr + cc);
+    uint8_t *codes_list = reinterpret_cast<uint8_t *>((char *)tmp + rl + rs + cr + 2 * cc);
     Plan pl;
     st = run_regions(ix->cent, reinterpret_cast<const uint16_t *>(c->rows), (int)N, 1, nullptr, row_list, row_score,
                      s, pl, 0);
@@ -1108,9 +1155,10 @@ skip_status_t skip_ivfpq_build(skip_corpus_t c, const void *centroids, int32_t C
     p.rows = c->rows;
     if (!st) st = cuda_status(launch_pq_encode(p, row_list, codes_rows, s));
     if (!st)
-        st = cuda_status(launch_ivf_lists(p, row_list, codes_rows, counts, cursor, ix->offsets, ix->ids, ix->codes,
+        st = cuda_status(launch_ivf_lists(p, row_list, codes_rows, counts, cursor, ix->offsets, ix->ids, codes_list,
                                           ix->cent->err, ix->cent->sm_count, s));
     if (!st) st = skip_sync_status(ix->cent, stream);
+    if (!st) st = ivf_layout(ix, codes_list, s);
     cudaFree(tmp);
     if (st) {
         ivf_release(ix);
@@ -1133,11 +1181,14 @@ skip_status_t skip_ivfpq_load(const void *centroids, int32_t C, int32_t d, const
     st = ivf_create(centroids, C, d, codebook, M, N, s, &ix);
     if (st) return st;
     if (cudaMemcpyAsync(ix->offsets, list_offsets, (size_t)(C + 1) * 8, cudaMemcpyDeviceToDevice, s) != cudaSuccess ||
-        (N > 0 && cudaMemcpyAsync(ix->ids, ids, (size_t)N * 4, cudaMemcpyDeviceToDevice, s) != cudaSuccess) ||
-        (N > 0 && cudaMemcpyAsync(ix->codes, codes, (size_t)N * M, cudaMemcpyDeviceToDevice, s) != cudaSuccess) ||
-        cudaStreamSynchronize(s) != cudaSuccess) {
+        (N > 0 && cudaMemcpyAsync(ix->ids, ids, (size_t)N * 4, cudaMemcpyDeviceToDevice, s) != cudaSuccess)) {
         ivf_release(ix);
         return SKIP_ECUDA;
+    }
+    st = ivf_layout(ix, codes, s);
+    if (st) {
+        ivf_release(ix);
+        return st;
     }
     *out = ix;
     return SKIP_OK;
@@ -1149,8 +1200,7 @@ skip_status_t skip_ivfpq_lists(skip_ivfpq_t ix, int64_t *list_offsets, int32_t *
     if ((list_offsets && cudaMemcpyAsync(list_offsets, ix->offsets, (size_t)(ix->C + 1) * 8, cudaMemcpyDeviceToDevice,
                                          s) != cudaSuccess) ||
         (ids && ix->N > 0 && cudaMemcpyAsync(ids, ix->ids, (size_t)ix->N * 4, cudaMemcpyDeviceToDevice, s) != cudaSuccess) ||
-        (codes && ix->N > 0 &&
-         cudaMemcpyAsync(codes, ix->codes, (size_t)ix->N * ix->M, cudaMemcpyDeviceToDevice, s) != cudaSuccess) ||
+        (codes && launch_ivf_deinterleave(ivf_params(ix), codes, ix->cent->sm_count, s) != cudaSuccess) ||
         cudaStreamSynchronize(s) != cudaSuccess)
         return SKIP_ECUDA;
     return SKIP_OK;
@@ -1177,11 +1227,12 @@ skip_status_t skip_ivfpq_search_regions(skip_ivfpq_t ix, const void *regions, in
     if (R_total > 0 && (!reg_ids || !reg_scores)) return SKIP_EINVAL;
     cudaStream_t s = reinterpret_cast<cudaStream_t>(stream);
     ++ix->cent->call_id;
-    uint64_t *keys = nullptr;
-    st = ivf_regions(ix, regions, R_total, nprobe, k_region, s, &keys);
+    uint64_t *keys = nullptr, *merged = nullptr;
+    int G = 1;
+    st = ivf_regions(ix, regions, R_total, nprobe, k_region, s, &keys, &merged, &G);
     if (st || R_total == 0) return st;
     record(ix->cent, s, "merge_lists");
-    st = cuda_status(launch_merge_lists(keys, 1, (int64_t)R_total * k_region, R_total, k_region, nullptr, reg_ids,
+    st = cuda_status(launch_merge_lists(keys, G, (int64_t)R_total * k_region, R_total, k_region, nullptr, reg_ids,
                                         reg_scores, s));
     record(ix->cent, s, "end");
     return st;
@@ -1196,9 +1247,17 @@ skip_status_t skip_ivfpq_search(skip_ivfpq_t ix, const void *regions, const int3
     if (Q == 0 && R_total != 0) return SKIP_EINVAL;
     cudaStream_t s = reinterpret_cast<cudaStream_t>(stream);
     ++ix->cent->call_id;
-    uint64_t *keys = nullptr;
-    st = ivf_regions(ix, regions, R_total, nprobe, k_region, s, &keys);
+    uint64_t *keys = nullptr, *merged = nullptr;
+    int G = 1;
+    st = ivf_regions(ix, regions, R_total, nprobe, k_region, s, &keys, &merged, &G);
     if (st) return st;
+    if (G > 1 && R_total > 0) {
+        record(ix->cent, s, "merge_lists");
+        st = cuda_status(launch_merge_lists(keys, G, (int64_t)R_total * k_region, R_total, k_region, merged, nullptr,
+                                            nullptr, s));
+        if (st) return st;
+        keys = merged;
+    }
     if (Q > 0) {
         record(ix->cent, s, "question_merge");
         st = cuda_status(launch_question_merge(keys, k_region, region_offsets, Q, R_total, K, out_ids, out_scores,
@@ -1215,6 +1274,11 @@ skip_status_t skip_ivfpq_sync_status(skip_ivfpq_t ix, void *stream) {
 
 skip_status_t skip_ivfpq_set_option(skip_ivfpq_t ix, int option, int64_t value) {
     if (!ix) return SKIP_EINVAL;
+    if (option == SKIP_OPT_IVF_SPLIT) {
+        if (value < 0 || value > kIvfMaxSplit) return SKIP_EINVAL;
+        ix->split = (int)value;
+        return SKIP_OK;
+    }
     return skip_corpus_set_option(ix->cent, option, value);
 }
 

@@ -170,21 +170,35 @@ struct IvfParams {
     const void *centroids;  // bf16 [C x d]
     int C;
     const float *codebook;  // [M][256][ds]
+    const float *cbT;       // [256][ds][Mp]: codebook with the sub-space fastest, 0 past M
     int M;                  // sub-spaces, a multiple of 16
     int ds;                 // d / M
-    const int64_t *offsets; // [C + 1] list starts
+    const int64_t *offsets; // [C + 1] list starts (entries)
+    const int64_t *boff;    // [C + 1] list starts (blocks of 32 entries)
     const int32_t *ids;     // [N] ids in list order
-    const uint8_t *codes;   // [N x M] codes in list order
+    const uint8_t *codes;   // [boff[C]][M * 32] codes in blocks of 32 entries (k_ivfpq.cu: il_offset)
 };
+// M rounded up to a whole number of warps: the row stride of the lookup table.
+inline int ivf_padded_m(int M) { return (M + 31) / 32 * 32; }
 cudaError_t launch_pq_encode(const IvfParams &p, const int64_t *row_list, uint8_t *codes, cudaStream_t s);
-// counts, cursor: [C] scratch; offsets [C + 1]; ids [N]; codes [N x M].
+// counts, cursor: [C] scratch; offsets [C + 1]; ids [N]; codes [N x M] (list order, one row per entry).
 cudaError_t launch_ivf_lists(const IvfParams &p, const int64_t *row_list, const uint8_t *codes_rows,
                              int64_t *counts, int64_t *cursor, int64_t *offsets, int32_t *ids, uint8_t *codes,
                              int *err, int sms, cudaStream_t s);
-size_t ivfpq_scan_smem(int M, int d, int nprobe);
-// Per region: keys (ordered score << 32 | ~id, 0 = empty) of the top k [R x k].
+// rows [N x M] in list order <-> p.codes (p.offsets, p.boff valid).
+cudaError_t launch_ivf_interleave(const IvfParams &p, const uint8_t *rows, uint8_t *il, int sms, cudaStream_t s);
+cudaError_t launch_ivf_deinterleave(const IvfParams &p, uint8_t *rows, int sms, cudaStream_t s);
+// cbT [256 x ds x ivf_padded_m(M)] from codebook [M x 256 x ds].
+cudaError_t launch_pq_codebook_t(const float *codebook, int M, int ds, float *cbT, cudaStream_t s);
+size_t ivfpq_scan_smem(int M, int nprobe);
+constexpr int kIvfMaxSplit = 8;  // most parts a region's probed blocks are cut into
+// Parts per region of the list scan: `requested` if > 0, else 1, 2 or 4,
+// doubling while twice the items still fit in the resident CTAs.
+cudaError_t ivfpq_scan_split(int M, int nprobe, int R, int sms, int requested, int *G);
+// Per part g of region r: keys (ordered score << 32 | ~id, 0 = empty) of its
+// top k at out_keys[(g * R + r) * k], sorted descending [G x R x k].
 cudaError_t launch_ivfpq_scan(const IvfParams &p, const uint16_t *regions, int R, const int64_t *probe_ids,
-                              const float *probe_scores, int nprobe, int k, uint64_t *out_keys, int sms,
+                              const float *probe_scores, int nprobe, int k, int G, uint64_t *out_keys, int sms,
                               cudaStream_t s);
 
 // ---- QVS visual token pruning (k_qvs.cu) -----------------------------------

@@ -143,10 +143,25 @@ def test_build_matches_oracle():
 
 @pytest.mark.parametrize("nprobe", [1, 4, 16, 64])
 def test_search_matches_oracle(nprobe):
-    corpus, regions, offsets, cent, cb = _small_inputs()
+    _check_search(SPEC, 16, nprobe)
+
+
+@pytest.mark.parametrize("d,M", [(128, 32), (96, 48), (160, 80), (128, 128)])
+def test_search_sub_space_counts(d, M):
+    """One to four warps' worth of sub-spaces (the lookup table's row is M
+    rounded up to 32), including the half-warp passes of M = 48 and 80."""
+    spec = synth.WorkloadSpec("ivf_m%d" % M, 43 + M, 9000, d, "bf16", 10, (1, 6), 10, 25, "clustered", 64)
+    _check_search(spec, M, 8)
+
+
+def _check_search(spec, M, nprobe):
+    corpus, _, centres = synth.make_corpus(spec)
+    regions, offsets = synth.make_regions(spec, centres)
+    cent = synth.make_ivf_centroids(spec)
+    cb = synth.make_pq_codebook(spec, M)
     cn, ce, qn = synth.bf16_bits(corpus), synth.bf16_bits(cent), synth.bf16_bits(regions)
     idx = oracle.ivfpq_build(cn, ce, cb.numpy())
-    k, K = SPEC.k_region, SPEC.K
+    k, K = spec.k_region, spec.K
     ext = k + 32
     o_ids, o_sc, o_probes = oracle.ivfpq_search(idx, ce, cb.numpy(), qn, nprobe, ext)
     c = skip.skip_corpus_load(_t(corpus))
@@ -182,6 +197,77 @@ def test_search_matches_oracle(nprobe):
         _, probs = checker.check_question(q_ids[q], q_sc[q], o_m_ids[q], o_m_sc[q], truths[off[q]:off[q + 1]], K)
         assert not probs, (q, probs[:3])
     print("nprobe %d: %d regions checked, %d identical to the oracle's" % (nprobe, checked, exact))
+
+
+def test_split_parts_give_identical_lists():
+    """Cutting each region's probed blocks into 1, 2, 3 or 8 parts (each part
+    scanned by its own CTA, the parts' lists merged afterwards) changes
+    nothing: every entry's s^ is computed the same way and ties break by id."""
+    corpus, regions, offsets, cent, cb = _small_inputs()
+    k, K = SPEC.k_region, SPEC.K
+    c = skip.skip_corpus_load(_t(corpus))
+    try:
+        ix = skip.skip_ivfpq_build(c, _t(cent), _t(cb))
+        outs = []
+        for split in (1, 2, 3, 8, 0):
+            ix.set_option(skip.SKIP_OPT_IVF_SPLIT, split)
+            r_ids, r_sc = skip.skip_ivfpq_search_regions(ix, _t(regions), 16, k)
+            q_ids, q_sc = skip.skip_ivfpq_search(ix, _t(regions), _t(offsets), 16, k, K)
+            assert skip.skip_ivfpq_sync_status(ix) == skip.SKIP_OK
+            outs.append([x.cpu().numpy() for x in (r_ids, r_sc, q_ids, q_sc)])
+        with pytest.raises(skip.SkipError):
+            ix.set_option(skip.SKIP_OPT_IVF_SPLIT, 9)
+        ix.free()
+    finally:
+        c.free()
+    for o in outs[1:]:
+        for a, b in zip(outs[0], o):
+            np.testing.assert_array_equal(a, b)
+
+
+def test_ragged_lists_round_trip_and_search():
+    """Lists of 0, 1, 31, 32, 33 and 100 entries (empty, partial and whole
+    blocks of 32): the codes come back out of the index unchanged, a search
+    probing every list returns the oracle's lists, and offsets that do not
+    partition the N entries are refused."""
+    rng = np.random.default_rng(11)
+    gen = torch.Generator().manual_seed(11)
+    lens = [0, 1, 31, 32, 33, 0, 100, 5]
+    C, d, M = len(lens), 64, 32
+    N = int(sum(lens))
+    off = np.concatenate([[0], np.cumsum(lens)]).astype(np.int64)
+    ids = rng.permutation(N).astype(np.int64)
+    lists = np.empty(N, np.int32)
+    for l in range(C):
+        lists[ids[off[l]:off[l + 1]]] = l
+    codes_by_id = rng.integers(0, 256, (N, M), dtype=np.uint8)
+    cent = torch.randn(C, d, generator=gen).to(torch.bfloat16)
+    cb = torch.randn(M, 256, d // M, generator=gen) * 0.1
+    q = torch.randn(6, d, generator=gen).to(torch.bfloat16)
+    k = 40
+    ix = skip.skip_ivfpq_load(_t(cent), _t(cb), _t(off), _t(ids, torch.int32), _t(codes_by_id[ids]))
+    try:
+        o, i, c = (x.cpu().numpy() for x in skip.skip_ivfpq_lists(ix))
+        g_ids, g_sc = skip.skip_ivfpq_search_regions(ix, _t(q), C, k)
+        assert skip.skip_ivfpq_sync_status(ix) == skip.SKIP_OK
+    finally:
+        ix.free()
+    np.testing.assert_array_equal(o, off)
+    np.testing.assert_array_equal(i, ids.astype(np.int32))
+    np.testing.assert_array_equal(c, codes_by_id[ids])
+    idx = {"offsets": off, "ids": ids, "codes": codes_by_id, "lists": lists}
+    ce, qn = synth.bf16_bits(cent), synth.bf16_bits(q)
+    o_ids, o_sc, _ = oracle.ivfpq_search(idx, ce, cb.numpy(), qn, C, k + 16)
+    for r, t in enumerate(checker.region_truths(o_ids, o_sc, k)):
+        _, probs = checker.check_region(
+            g_ids[r].cpu().numpy(), g_sc[r].cpu().numpy(), t,
+            extra_score=lambda i, r=r: float(oracle.ivfpq_scores_at(idx, ce, cb.numpy(), qn, [r], [i])[0]))
+        assert not probs, (r, probs[:3])
+    falling = off.copy()
+    falling[4] = off[3] - 1
+    for bad in (off + 1, np.r_[off[:-1], N - 1], falling):
+        with pytest.raises(skip.SkipError):
+            skip.skip_ivfpq_load(_t(cent), _t(cb), _t(bad), _t(ids, torch.int32), _t(codes_by_id[ids]))
 
 
 def test_exact_codebook_all_lists_equals_exact_search():
