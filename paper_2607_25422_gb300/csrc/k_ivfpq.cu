@@ -306,6 +306,7 @@ __global__ void __launch_bounds__(kScanThreads, NP <= 2 ? 2 : 1)
     const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
     const int M = p.M, ds = p.ds;
     constexpr int Mp = 32 * NP;
+    constexpr int kLutUnroll = NP == 2 ? 3 : 2;  // codebook loads in flight per lane: 32 x this
     // item it: part g of region r (its blocks [TB g / G, TB (g + 1) / G))
     for (int it = blockIdx.x; it < R * G; it += gridDim.x) {
         const int r = it / G, g = it - r * G;
@@ -334,7 +335,7 @@ __global__ void __launch_bounds__(kScanThreads, NP <= 2 ? 2 : 1)
                 float acc[32];
 #pragma unroll
                 for (int i = 0; i < 32; ++i) acc[i] = 0.f;
-#pragma unroll 2
+#pragma unroll kLutUnroll
                 for (int t = 0; t < ds; ++t) {
                     const float qv = m < M ? __bfloat162float(q[m * ds + t]) : 0.f;
                     const float *pc = p.cbT + ((int64_t)c0 * ds + t) * Mp + m;
