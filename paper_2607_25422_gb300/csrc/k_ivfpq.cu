@@ -6,7 +6,8 @@
 // the centroids as the corpus and the corpus rows as queries, k = 1):
 //   k_pq_encode     residual x - c_list, nearest of 256 codewords per
 //                   sub-space (fp32, ties to the lower codeword); a block of
-//                   128 rows shares each sub-space's codebook in shared memory.
+//                   128 rows shares each sub-space's codebook in shared memory,
+//                   read as 16-byte broadcasts.
 //   k_ivf_count / k_ivf_offsets / k_ivf_scatter
 //                   counting sort of the rows into their lists (order inside
 //                   a list is arbitrary: the search breaks ties by id).
@@ -39,9 +40,14 @@ namespace {
 
 constexpr int kEncRows = 128;
 
+// DSB: the sub-space width rounded up to 4, 8, 12, 16, 24 or 32; the
+// codebook copy in shared memory and the residual are zero past ds, so the
+// padded sum adds exact zeros after the same terms in the same order.
+template <int DSB>
 __global__ void __launch_bounds__(kEncRows) k_pq_encode(const IvfParams p, const int64_t *row_list,
                                                          uint8_t *codes) {
-    extern __shared__ float cbs[];  // [256][ds] codebook of one sub-space
+    extern __shared__ float4 cbs4[];  // [256][DSB / 4]: codebook of one sub-space
+    float *cbs = reinterpret_cast<float *>(cbs4);
     const int64_t i = (int64_t)blockIdx.x * kEncRows + threadIdx.x;
     const bool valid = i < p.N;
     const int ds = p.ds;
@@ -51,23 +57,28 @@ __global__ void __launch_bounds__(kEncRows) k_pq_encode(const IvfParams p, const
     const __nv_bfloat16 *c = reinterpret_cast<const __nv_bfloat16 *>(p.centroids) + l * (int64_t)p.d;
     for (int m = 0; m < p.M; ++m) {
         __syncthreads();
-        for (int e = threadIdx.x; e < 256 * ds; e += kEncRows) cbs[e] = p.codebook[(int64_t)m * 256 * ds + e];
+        for (int e = threadIdx.x; e < 256 * DSB; e += kEncRows) {
+            const int j = e / DSB, t = e - j * DSB;
+            cbs[e] = t < ds ? p.codebook[((int64_t)m * 256 + j) * ds + t] : 0.f;
+        }
         __syncthreads();
-        float r[kIvfMaxDs];
+        float r[DSB];
 #pragma unroll
-        for (int t = 0; t < kIvfMaxDs; ++t)
+        for (int t = 0; t < DSB; ++t)
             r[t] = t < ds ? __bfloat162float(x[m * ds + t]) - __bfloat162float(c[m * ds + t]) : 0.f;
         int best = 0;
         float bd = __int_as_float(0x7f800000);
         for (int j = 0; j < 256; ++j) {
-            const float *pj = cbs + j * ds;
             float dist = 0.f;
 #pragma unroll
-            for (int t = 0; t < kIvfMaxDs; ++t) {
-                if (t < ds) {
-                    const float e = r[t] - pj[t];
-                    dist = fmaf(e, e, dist);
-                }
+            for (int q = 0; q < DSB / 4; ++q) {
+                const float4 v = cbs4[j * (DSB / 4) + q];
+                const float e0 = r[4 * q] - v.x, e1 = r[4 * q + 1] - v.y;
+                const float e2 = r[4 * q + 2] - v.z, e3 = r[4 * q + 3] - v.w;
+                dist = fmaf(e0, e0, dist);
+                dist = fmaf(e1, e1, dist);
+                dist = fmaf(e2, e2, dist);
+                dist = fmaf(e3, e3, dist);
             }
             if (dist < bd) {
                 bd = dist;
@@ -448,10 +459,23 @@ __global__ void __launch_bounds__(kScanThreads, NP <= 2 ? 2 : 1)
 
 }  // namespace
 
+namespace {
+template <int DSB>
+void launch_encode_dsb(const IvfParams &p, const int64_t *row_list, uint8_t *codes, cudaStream_t s) {
+    k_pq_encode<DSB><<<(unsigned)((p.N + kEncRows - 1) / kEncRows), kEncRows, (size_t)256 * DSB * sizeof(float), s>>>(
+        p, row_list, codes);
+}
+}  // namespace
+
 cudaError_t launch_pq_encode(const IvfParams &p, const int64_t *row_list, uint8_t *codes, cudaStream_t s) {
     if (p.N == 0) return cudaSuccess;
-    const size_t smem = (size_t)256 * p.ds * sizeof(float);
-    k_pq_encode<<<(unsigned)((p.N + kEncRows - 1) / kEncRows), kEncRows, smem, s>>>(p, row_list, codes);
+    if (p.ds <= 4) launch_encode_dsb<4>(p, row_list, codes, s);
+    else if (p.ds <= 8) launch_encode_dsb<8>(p, row_list, codes, s);
+    else if (p.ds <= 12) launch_encode_dsb<12>(p, row_list, codes, s);
+    else if (p.ds <= 16) launch_encode_dsb<16>(p, row_list, codes, s);
+    else if (p.ds <= 24) launch_encode_dsb<24>(p, row_list, codes, s);
+    else if (p.ds <= 32) launch_encode_dsb<32>(p, row_list, codes, s);
+    else return cudaErrorInvalidValue;
     return cudaGetLastError();
 }
 
