@@ -69,3 +69,29 @@ def test_null_handles():
     assert lib.skip_retrieve(None, None, None, 0, 0, 1, 1, None, None, None) == skip.SKIP_EINVAL
     assert lib.skip_sync_status(None, None) == skip.SKIP_EINVAL
     assert lib.skip_corpus_set_option(None, 0, 0) == skip.SKIP_EINVAL
+
+
+def test_header_constants_match_the_binding():
+    """Every `SKIP_NAME = value` of the C headers (status codes, options,
+    paths) has the same value in the Python binding."""
+    found = {}
+    for h in glob.glob(os.path.join(ROOT, "include", "*.h")):
+        for name, val in re.findall(r"\b(SKIP_[A-Z0-9_]+)\s*=\s*(\d+)", open(h).read()):
+            found[name] = int(val)
+    for name in ("SKIP_OK", "SKIP_EINVAL", "SKIP_ETIMEOUT", "SKIP_OPT_PATH", "SKIP_OPT_BOUND",
+                 "SKIP_OPT_IVF_SPLIT", "SKIP_PATH_LATENCY"):
+        assert name in found, name
+    for name, val in found.items():
+        assert getattr(skip, name) == val, name
+
+
+def test_ivfpq_entry_points_reject_null_handles():
+    lib = skip.load_library()
+    assert lib.skip_ivfpq_set_option(None, skip.SKIP_OPT_IVF_SPLIT, 0) == skip.SKIP_EINVAL
+    assert lib.skip_ivfpq_sync_status(None, None) == skip.SKIP_EINVAL
+    assert lib.skip_ivfpq_info(None, None, None, None, None) == skip.SKIP_EINVAL
+    assert lib.skip_ivfpq_lists(None, None, None, None, None) == skip.SKIP_EINVAL
+    h = ctypes.c_void_p()
+    # no centroids, codebook or offsets: refused before any device work
+    assert lib.skip_ivfpq_load(None, 4, 64, None, 16, None, None, None, 0, None, ctypes.byref(h)) == skip.SKIP_EINVAL
+    assert not h.value
