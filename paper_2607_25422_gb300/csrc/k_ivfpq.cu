@@ -219,6 +219,28 @@ __device__ void block_sort_desc(uint64_t *keys, int n) {
         }
 }
 
+// Coarse probe of a small centroid set: region r's C centroid scores
+// (a GEMM's row) sorted by (score desc, id asc) in shared memory; the first
+// nprobe are the probed lists.
+__global__ void __launch_bounds__(256) k_ivf_probe_select(const float *scores, int C, int nprobe,
+                                                          int64_t *probe_ids, float *probe_sc) {
+    extern __shared__ uint64_t pkeys[];  // [n], n = C rounded up to a power of two
+    const int r = blockIdx.x;
+    int n = 2;
+    while (n < C) n <<= 1;
+    const float *sr = scores + (int64_t)r * C;
+    for (int c = threadIdx.x; c < n; c += blockDim.x) pkeys[c] = c < C ? make_key(sr[c], (uint32_t)c) : 0ull;
+    __syncthreads();
+    block_sort_desc(pkeys, n);
+    for (int i = threadIdx.x; i < nprobe; i += blockDim.x) {
+        int64_t id;
+        float sc;
+        key_decode(pkeys[i], id, sc);
+        probe_ids[(int64_t)r * nprobe + i] = id;
+        probe_sc[(int64_t)r * nprobe + i] = sc;
+    }
+}
+
 // One step of the butterfly reduce-scatter.  Slot i of lane l holds entry
 // i ^ l (the index stores each sub-space's bytes in that order), so the
 // lane keeps slots [0, O) and adds the partner's slots [O, 2 O), which hold
@@ -509,6 +531,16 @@ cudaError_t launch_pq_codebook_t(const float *codebook, int M, int ds, float *cb
     const int Mp = ivf_padded_m(M);
     const int64_t n = (int64_t)256 * ds * Mp;
     k_pq_codebook_t<<<(unsigned)std::min<int64_t>((n + 255) / 256, 4096), 256, 0, s>>>(codebook, M, ds, Mp, cbT);
+    return cudaGetLastError();
+}
+
+cudaError_t launch_ivf_probe_select(const float *scores, int R, int C, int nprobe, int64_t *probe_ids,
+                                    float *probe_sc, cudaStream_t s) {
+    if (R == 0) return cudaSuccess;
+    if (C < 1 || C > kIvfCoarseMaxC || nprobe < 1 || nprobe > C) return cudaErrorInvalidValue;
+    int n = 2;
+    while (n < C) n <<= 1;
+    k_ivf_probe_select<<<R, 256, (size_t)n * sizeof(uint64_t), s>>>(scores, C, nprobe, probe_ids, probe_sc);
     return cudaGetLastError();
 }
 

@@ -982,6 +982,7 @@ struct skip_ivfpq {
     void *ws = nullptr;           // search workspace
     size_t ws_bytes = 0;
     int split = 0;                // parts per region of the list scan (0: pick)
+    cublasHandle_t blas = nullptr; // the coarse probe's GEMM (C <= kIvfCoarseMaxC)
 };
 
 namespace {
@@ -990,6 +991,7 @@ void ivf_release(skip_ivfpq *ix) {
     if (!ix) return;
     cudaDeviceSynchronize();
     if (ix->cent) skip_corpus_free(ix->cent);
+    if (ix->blas) cublasDestroy(ix->blas);
     cudaFree(ix->codebook);
     cudaFree(ix->cbT);
     cudaFree(ix->offsets);
@@ -1011,6 +1013,11 @@ skip_status_t ivf_create(const void *centroids, int C, int d, const float *codeb
         return st;
     }
     const size_t cb = (size_t)M * 256 * ix->ds * sizeof(float);
+    if (C <= kIvfCoarseMaxC && cublasCreate(&ix->blas) != CUBLAS_STATUS_SUCCESS) {
+        ix->blas = nullptr;
+        ivf_release(ix);
+        return SKIP_ECUDA;
+    }
     const size_t cbt = (size_t)256 * ix->ds * ivf_padded_m(M) * sizeof(float);
     if (cudaMalloc(&ix->codebook, cb) != cudaSuccess || cudaMalloc(&ix->cbT, cbt) != cudaSuccess ||
         cudaMalloc(&ix->offsets, (size_t)(C + 1) * 8) != cudaSuccess ||
@@ -1093,7 +1100,8 @@ skip_status_t ivf_regions(skip_ivfpq *ix, const void *regions, int R, int nprobe
     }
     const size_t pid = align_up((size_t)R * nprobe * 8, 256), psc = align_up((size_t)R * nprobe * 4, 256);
     const size_t kb = align_up((size_t)std::max(R, 1) * k * 8, 256);
-    skip_status_t st = ensure_buf(ix->ws, ix->ws_bytes, (G + 1) * kb + pid + psc);
+    const size_t scb = ix->blas ? align_up((size_t)R * ix->C * 4, 256) : 0;  // coarse GEMM scores
+    skip_status_t st = ensure_buf(ix->ws, ix->ws_bytes, (G + 1) * kb + pid + psc + scb);
     if (st) return st;
     uint64_t *keys = reinterpret_cast<uint64_t *>(ix->ws);
     int64_t *probe_ids = reinterpret_cast<int64_t *>((char *)ix->ws + (G + 1) * kb);
@@ -1102,9 +1110,23 @@ skip_status_t ivf_regions(skip_ivfpq *ix, const void *regions, int R, int nprobe
     *merged = reinterpret_cast<uint64_t *>((char *)ix->ws + G * kb);
     *G_out = G;
     if (R == 0) return SKIP_OK;
-    Plan pl;
-    st = run_regions(ix->cent, reinterpret_cast<const uint16_t *>(regions), R, nprobe, nullptr, probe_ids, probe_sc,
-                     s, pl, 0);
+    if (ix->blas) {
+        // coarse scores [R x C] = regions [R x d] . centroids [C x d]^T:
+        // column-major scores^T = centroids . regions^T
+        float *scores = reinterpret_cast<float *>((char *)ix->ws + (G + 1) * kb + pid + psc);
+        const float one = 1.f, zero = 0.f;
+        record(ix->cent, s, "ivf_probe");
+        if (cublasSetStream(ix->blas, s) != CUBLAS_STATUS_SUCCESS ||
+            cublasGemmEx(ix->blas, CUBLAS_OP_T, CUBLAS_OP_N, ix->C, R, ix->d, &one, ix->cent->rows, CUDA_R_16BF,
+                         ix->d, regions, CUDA_R_16BF, ix->d, &zero, scores, CUDA_R_32F, ix->C, CUBLAS_COMPUTE_32F,
+                         CUBLAS_GEMM_DEFAULT) != CUBLAS_STATUS_SUCCESS)
+            return SKIP_ECUDA;
+        st = cuda_status(launch_ivf_probe_select(scores, R, ix->C, nprobe, probe_ids, probe_sc, s));
+    } else {
+        Plan pl;
+        st = run_regions(ix->cent, reinterpret_cast<const uint16_t *>(regions), R, nprobe, nullptr, probe_ids,
+                         probe_sc, s, pl, 0);
+    }
     if (st) return st;
     record(ix->cent, s, "ivfpq_scan");
     cudaError_t e = launch_ivfpq_scan(ivf_params(ix), reinterpret_cast<const uint16_t *>(regions), R, probe_ids,

@@ -190,6 +190,11 @@ cudaError_t launch_ivf_interleave(const IvfParams &p, const uint8_t *rows, uint8
 cudaError_t launch_ivf_deinterleave(const IvfParams &p, uint8_t *rows, int sms, cudaStream_t s);
 // cbT [256 x ds x ivf_padded_m(M)] from codebook [M x 256 x ds].
 cudaError_t launch_pq_codebook_t(const float *codebook, int M, int ds, float *cbT, cudaStream_t s);
+// Coarse probe over at most kIvfCoarseMaxC centroids: scores [R x C] (a
+// GEMM) -> per region the nprobe best (id, score), sorted (score desc, id asc).
+constexpr int kIvfCoarseMaxC = 4096;
+cudaError_t launch_ivf_probe_select(const float *scores, int R, int C, int nprobe, int64_t *probe_ids,
+                                    float *probe_sc, cudaStream_t s);
 size_t ivfpq_scan_smem(int M, int nprobe);
 constexpr int kIvfMaxSplit = 8;  // most parts a region's probed blocks are cut into
 // Parts per region of the list scan: `requested` if > 0, else 1, 2 or 4,
