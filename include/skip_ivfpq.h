@@ -91,10 +91,13 @@ SKIP_API skip_status_t skip_ivfpq_search(skip_ivfpq_t index, const void *regions
 /* As skip_sync_status, for the index's kernels. */
 SKIP_API skip_status_t skip_ivfpq_sync_status(skip_ivfpq_t index, void *stream);
 
-/* Sets an option of the index: SKIP_OPT_IVF_SPLIT for its list scan, any
- * other skip_option_t of skip_retrieve.h for its coarse search (applied to
- * its centroid set); SKIP_OPT_TIMING records the index's kernels, reported
- * by skip_ivfpq_timing_report.  Results do not depend on the options. */
+/* Sets an option of the index: SKIP_OPT_IVF_SPLIT for its list scan; any
+ * other skip_option_t of skip_retrieve.h applies to its centroid set, which
+ * the exact MIPS path searches for the build's coarse assignment and, with
+ * more than 4,096 centroids, for the search's coarse probe (with at most
+ * 4,096 the probe is one bf16 GEMM and a per-region sort).  SKIP_OPT_TIMING
+ * records the index's kernels, reported by skip_ivfpq_timing_report.
+ * Results do not depend on the options. */
 SKIP_API skip_status_t skip_ivfpq_set_option(skip_ivfpq_t index, int option, int64_t value);
 SKIP_API skip_status_t skip_ivfpq_timing_report(skip_ivfpq_t index, char *buf, int32_t len);
 
