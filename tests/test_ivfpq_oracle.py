@@ -103,3 +103,41 @@ def test_more_probes_never_lower_the_kth_score():
     # the index holds every id once
     assert sorted(idx["ids"].tolist()) == list(range(spec.N))
     assert idx["offsets"][-1] == spec.N
+
+
+@pytest.mark.parametrize("nprobe,k", [(1, 5), (1, 30), (3, 12), (7, 40)])
+def test_search_matches_brute_force_with_random_codes(nprobe, k):
+    """An index given directly (random lists and random codes, so the build
+    plays no part): for every region, the nprobe centroids with the largest
+    <q, c_l> (lower l first on ties) are probed and every row of their lists
+    is scored s^ = <q, c_list(i)> + sum_m <q_m, p_{m, code_{i,m}}> in fp64,
+    then cut to the k best by (s^ desc, id asc), padded with (-1, -inf)."""
+    rng = np.random.default_rng(17 + nprobe)
+    N, d, C, M, ksub = 90, 32, 7, 8, 16
+    ds = d // M
+    cent = synth.random_bf16(C, d, seed=nprobe)
+    cent[5] = cent[2]  # two equal centroid scores: the lower list is probed first
+    q = synth.random_bf16(4, d, seed=10 + nprobe)
+    cb = rng.normal(0, 0.1, size=(M, ksub, ds)).astype(np.float32)
+    lists = rng.integers(0, C, N).astype(np.int32)
+    codes = rng.integers(0, ksub, (N, M)).astype(np.uint8)
+    order = np.argsort(lists, kind="stable")
+    offsets = np.zeros(C + 1, np.int64)
+    offsets[1:] = np.cumsum(np.bincount(lists, minlength=C))
+    idx = {"lists": lists, "codes": codes, "offsets": offsets, "ids": order.astype(np.int64)}
+    ids, sc, probes = oracle.ivfpq_search(idx, synth.bf16_bits(cent), cb, synth.bf16_bits(q), nprobe, k)
+    qd, cd, cbd = q.double().numpy(), cent.double().numpy(), cb.astype(np.float64)
+    for r in range(qd.shape[0]):
+        cs = cd @ qd[r]
+        want_probes = np.lexsort((np.arange(C), -cs))[:nprobe]
+        np.testing.assert_array_equal(probes[r], want_probes)
+        rows = np.nonzero(np.isin(lists, want_probes))[0]
+        s = np.array([cs[lists[i]] + sum(qd[r, m * ds:(m + 1) * ds] @ cbd[m, codes[i, m]] for m in range(M))
+                      for i in rows])
+        top = np.lexsort((rows, -s))[:k]
+        want_ids = np.full(k, -1, np.int64)
+        want_sc = np.full(k, -np.inf)
+        want_ids[:len(top)] = rows[top]
+        want_sc[:len(top)] = s[top]
+        np.testing.assert_array_equal(ids[r], want_ids)
+        np.testing.assert_allclose(sc[r], want_sc, rtol=1e-12, atol=1e-12)
