@@ -490,8 +490,6 @@ def main():
     ap.add_argument("--path", default="auto", choices=["auto", "tensor", "warp", "latency"])
     ap.add_argument("--rows", type=int, default=0,
                     help="use only the first ROWS corpus rows (smaller profiling captures; not a bench line)")
-    ap.add_argument("--cluster", type=int, default=0, choices=[0, 1, 2, 4, 8],
-                    help="single-CTA tensor path CTAs per cluster (0 = library's choice)")
     ap.add_argument("--ivfpq", action="store_true",
                     help="step = IVF-PQ search (generator centres as IVF centroids, sample-based PQ codebook)")
     ap.add_argument("--nprobe", type=int, default=32)
@@ -536,7 +534,6 @@ def main():
     del corpus
     torch.cuda.empty_cache()
     c.set_option(skip.SKIP_OPT_PATH, {"auto": 0, "tensor": 1, "warp": 2, "latency": 3}[args.path])
-    c.set_option(skip.SKIP_OPT_CLUSTER, args.cluster)
     c.set_option(skip.SKIP_OPT_MMA, {"auto": 0, "single": 1, "pair": 2}[args.mma])
     reg_d = regions.to(dev)
     off_d = offsets.to(dev)

@@ -69,7 +69,8 @@ typedef enum {
     SKIP_OPT_WAIT_TIMEOUT_NS = 1, /* cap on each in-kernel wait (default 2e9 ns) */
     SKIP_OPT_GRID = 2,            /* score-kernel CTAs (0 = one per SM) */
     SKIP_OPT_TIMING = 3,          /* 1: time each kernel with CUDA events */
-    SKIP_OPT_CLUSTER = 4,         /* single-CTA tensor path CTAs per cluster: 0 pick, 1, 2, 4, 8 */
+    SKIP_OPT_CLUSTER = 4,         /* accepts 0 or 1 only: single-CTA tensor launches use no
+                                     thread-block clusters (each CTA loads its own corpus tiles) */
     SKIP_OPT_MMA = 5,             /* tensor path MMA: 0 pick, 1 single CTA, 2 CTA pair */
     SKIP_OPT_BOUND = 6,           /* bf16 tensor path: 0 auto (a bounding pass over every 48th
                                      corpus tile first when the corpus has at least 2,048
@@ -182,9 +183,15 @@ SKIP_API skip_status_t skip_retrieve_host(skip_corpus_t corpus, const uint16_t *
  *  reg_ids/scores  device int64 / fp32 [R_total x k_region], each row sorted
  *                  by (score desc, id asc) -- the same result as
  *                  skip_retrieve_regions.
- * Limits as skip_retrieve_regions, plus: the scratch, about
- * 8 * k_region * (#SMs * R_total + #SMs * 64) bytes, must fit in 16 MiB,
- * else SKIP_EUNSUPPORTED.  Asynchronous on `stream`.
+ * Alignment (SKIP_EINVAL otherwise, checked before anything is launched):
+ * corpus_rows on a 16-byte boundary, row_scale and reg_scores on 4 bytes,
+ * regions on 2, reg_ids on 8.
+ * Limits as skip_retrieve_regions, plus: with G = min(#SMs, 512,
+ * ceil(N / 256)) score-kernel blocks, the scratch of
+ * 8 * k_region * (G * R_total + G * 64) bytes (the first term rounded up to
+ * 256) must fit in 16 MiB, else SKIP_EUNSUPPORTED; the limit on R_total *
+ * k_region therefore depends on the GPU's SM count and on N.
+ * Asynchronous on `stream`.
  */
 SKIP_API skip_status_t skip_retrieve_regions_noalloc(const void *corpus_rows, int64_t N, int32_t d,
                                                      skip_dtype_t dtype, const float *row_scale,

@@ -16,10 +16,8 @@
 //
 // Two MMA shapes:
 //  * single CTA (cta_group::1, M = 128): the CTA stages its 128 region rows
-//    and the whole 256-row corpus tile; a cluster of CL CTAs (1, 2, 4, 8)
-//    with CL query blocks shares each corpus tile -- CTA r loads rows
-//    [r * 256 / CL, (r + 1) * 256 / CL) and multicasts them to all CL CTAs,
-//    and the MMA commits that release a stage are multicast too;
+//    and the whole 256-row corpus tile itself (CTAs of other query blocks
+//    that read the same tile find it in L2);
 //  * CTA pair (cta_group::2, M = 256): a cluster of two CTAs on two SMs
 //    computes 256 region rows (two query blocks) against a 256-row corpus
 //    tile, each CTA staging its own 128 region rows and half of the corpus
@@ -103,18 +101,16 @@ __global__ void __launch_bounds__(kTcThreads, 1)
     const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
     const int items = p.QG * p.G;
     const int KB = (p.d + kTcTileK - 1) / kTcTileK;
-    const int CL = p.CL;
-    const int rank = CL > 1 ? (int)cluster_rank() : 0;
-    const int cid = CL > 1 ? (int)cluster_index() : (int)blockIdx.x;
-    const int ncl = CL > 1 ? (int)cluster_count() : (int)gridDim.x;
-    const uint16_t mask = (uint16_t)((1u << CL) - 1u);
-    const int slice_rows = kTcTileN / CL;
+    // A pair is a cluster of two CTAs; a single-CTA launch has no clusters.
+    const int rank = PAIR ? (int)cluster_rank() : 0;
+    const int cid = PAIR ? (int)cluster_index() : (int)blockIdx.x;
+    const int ncl = PAIR ? (int)cluster_count() : (int)gridDim.x;
     const bool mma_cta = !PAIR || rank == 0;
 
     if (threadIdx.x == 0) {
         for (int s = 0; s < S; ++s) {
             mbar_init(smem_addr(&sh->full[s]), 1);
-            mbar_init(smem_addr(&sh->empty[s]), PAIR ? 1 : CL);
+            mbar_init(smem_addr(&sh->empty[s]), 1);
         }
         for (int b = 0; b < 2; ++b) {
             mbar_init(smem_addr(&sh->tfull[b]), 1);
@@ -140,7 +136,7 @@ __global__ void __launch_bounds__(kTcThreads, 1)
     __syncthreads();
     tc_fence_after();
     // Every CTA's barriers are initialised before any peer copy or arrive.
-    if (CL > 1) cluster_sync_all();
+    if constexpr (PAIR) cluster_sync_all();
     const uint32_t tmem = sh->tmem_base;
 
     if (warp == 0) {
@@ -169,12 +165,8 @@ __global__ void __launch_bounds__(kTcThreads, 1)
                                              (int)(t * p.tile_stride * kTcTileN) + rank * (kTcTileN / 2));
                         } else {
                             tma_load_2d(smem_addr(sA + s * kABytes), &tq, fb, x, it.mb * kTcTileM);
-                            if (CL == 1)
-                                tma_load_2d(smem_addr(sB + s * Gm::kBBytes), &tx, fb, x,
-                                            (int)(t * p.tile_stride * kTcTileN));
-                            else
-                                tma_load_2d_mc(smem_addr(sB + s * Gm::kBBytes + rank * slice_rows * 128), &tx, fb,
-                                               x, (int)(t * p.tile_stride * kTcTileN) + rank * slice_rows, mask);
+                            tma_load_2d(smem_addr(sB + s * Gm::kBBytes), &tx, fb, x,
+                                        (int)(t * p.tile_stride * kTcTileN));
                         }
                         ++issued;
                         if (++s == S) {
@@ -233,10 +225,8 @@ __global__ void __launch_bounds__(kTcThreads, 1)
                         }
                         if constexpr (PAIR)
                             tc_commit_pair_mc(smem_addr(&sh->empty[s]), 3);
-                        else if (CL == 1)
-                            tc_commit(smem_addr(&sh->empty[s]));
                         else
-                            tc_commit_mc(smem_addr(&sh->empty[s]), mask);
+                            tc_commit(smem_addr(&sh->empty[s]));
                         if (++s == S) {
                             s = 0;
                             ph ^= 1u;
@@ -414,7 +404,7 @@ __global__ void __launch_bounds__(kTcThreads, 1)
     __syncthreads();
     // No peer may still copy into, arrive on, or (pair) write the TMEM of
     // this CTA when it frees TMEM and exits.
-    if (CL > 1) cluster_sync_all();
+    if constexpr (PAIR) cluster_sync_all();
     tc_fence_after();
     if (warp == 1) {
         __syncwarp();
@@ -486,7 +476,7 @@ int tc_max_clusters(bool pair, int CL, int stages, int k, bool list_in_smem) {
 
 cudaError_t launch_tc(bool pair, const CUtensorMap &tq, const CUtensorMap &tx, const TcParams &p, int grid,
                       cudaStream_t s, bool pdl) {
-    if (pair && p.CL != 2) return cudaErrorInvalidValue;
+    if (p.CL != (pair ? 2 : 1)) return cudaErrorInvalidValue;
     const size_t smem = tc_smem_bytes(pair, p.stages, p.k, p.list_in_smem != 0);
     auto kern = pair ? k_tc_score_topk<true> : k_tc_score_topk<false>;
     cudaError_t e = cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);

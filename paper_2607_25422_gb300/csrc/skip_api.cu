@@ -101,7 +101,6 @@ struct skip_corpus {
     int path = SKIP_PATH_AUTO;
     uint64_t timeout_ns = kDefaultTimeoutNs;
     int grid = 0;
-    int cluster = 0;           // 0 = pick; else CTAs per cluster
     int mma = 0;               // 0 = pick, 1 = single-CTA MMA, 2 = CTA-pair MMA
     int bound = 0;             // bounding pass: 0 = by corpus size, 1 = never, 2 = always
     std::map<int, int> cluster_cache;  // resident clusters per (size, stages, list place)
@@ -366,36 +365,11 @@ skip_status_t run_regions(skip_corpus *c, const uint16_t *regions, int R, int k,
                 hit = c->cluster_cache.emplace(key, tc_max_clusters(pair, CL, stages, k, in_smem)).first;
             return hit->second;
         };
-        // Cluster size (single-CTA MMA): the CTAs of a cluster share each
-        // corpus tile (one L2 read, multicast).  Take the largest size that
-        // keeps at least 90% of the SMs the best size keeps busy, unless set
-        // by option.  A pair is a cluster of two.
-        int cl_best = 1, ncl_best = 0;
-        if (pair) {
-            cl_best = 2;
-            ncl_best = max_clusters(2);
-            if (ncl_best == 0) return SKIP_ECUDA;
-        } else {
-            int used[4] = {0, 0, 0, 0}, ncls[4] = {0, 0, 0, 0};
-            int best_used = 0;
-            for (int i = 0; i < 4; ++i) {
-                const int CL = 1 << i;
-                if (c->cluster && CL != c->cluster) continue;
-                if (!c->cluster && CL > 1 && CL > pl.MB) break;
-                ncls[i] = max_clusters(CL);
-                const int QG = (pl.MB + CL - 1) / CL;
-                const double eff = (double)pl.MB / (double)(QG * CL);
-                used[i] = (int)(std::min(ncls[i] * CL, ctas) * eff);
-                best_used = std::max(best_used, used[i]);
-            }
-            for (int i = 3; i >= 0; --i)
-                if (used[i] > 0 && used[i] * 10 >= best_used * 9) {
-                    cl_best = 1 << i;
-                    ncl_best = ncls[i];
-                    break;
-                }
-            if (ncl_best == 0) return SKIP_ECUDA;
-        }
+        // A pair is a cluster of two CTAs; single-CTA MMA runs without
+        // clusters, each CTA loading its own corpus tiles.
+        const int cl_best = pair ? 2 : 1;
+        const int ncl_best = max_clusters(cl_best);
+        if (ncl_best == 0) return SKIP_ECUDA;
         pl.CL = cl_best;
         const int QG = (pl.MB + cl_best - 1) / cl_best;
         const int ncl = std::max(1, std::min(ncl_best, ctas / cl_best));
@@ -754,8 +728,8 @@ skip_status_t skip_corpus_set_option(skip_corpus_t c, int option, int64_t value)
             c->mma = (int)value;
             return SKIP_OK;
         case SKIP_OPT_CLUSTER:
-            if (value != 0 && value != 1 && value != 2 && value != 4 && value != 8) return SKIP_EINVAL;
-            c->cluster = (int)value;
+            // Kept for the ABI: single-CTA tensor launches use no clusters.
+            if (value != 0 && value != 1) return SKIP_EINVAL;
             return SKIP_OK;
         case SKIP_OPT_BOUND:
             if (value < 0 || value > 2) return SKIP_EINVAL;

@@ -176,18 +176,6 @@ __device__ __forceinline__ void tma_load_2d_hint(uint32_t dst, const void *map, 
         : "memory");
 }
 
-// Multicast variant: the tile lands at the same shared-memory offset, and
-// its bytes are counted on the barrier at the same offset, in every CTA of
-// the cluster named in cta_mask.
-__device__ __forceinline__ void tma_load_2d_mc(uint32_t dst, const void *map, uint32_t bar, int x, int y,
-                                               uint16_t cta_mask) {
-    asm volatile(
-        "cp.async.bulk.tensor.2d.shared::cluster.global.mbarrier::complete_tx::bytes.multicast::cluster"
-        " [%0], [%1, {%3, %4}], [%2], %5;" ::"r"(dst),
-        "l"(map), "r"(bar), "r"(x), "r"(y), "h"(cta_mask)
-        : "memory");
-}
-
 // CTA-pair variant (.cta_group::2): the tile lands in this CTA's shared
 // memory, and its bytes are counted on `bar`, a shared::cluster address that
 // may name the barrier of the other CTA of the pair.
@@ -327,16 +315,6 @@ __device__ __forceinline__ void tc_commit(uint32_t bar) {
     asm volatile("tcgen05.commit.cta_group::1.mbarrier::arrive::one.shared::cluster.b64 [%0];" ::"r"(
                      bar)
                  : "memory");
-}
-
-// As tc_commit, arriving on the barrier at the same offset in every CTA of
-// the cluster named in cta_mask.
-__device__ __forceinline__ void tc_commit_mc(uint32_t bar, uint16_t cta_mask) {
-    asm volatile(
-        "tcgen05.commit.cta_group::1.mbarrier::arrive::one.shared::cluster.multicast::cluster.b64 [%0], %1;" ::"r"(
-            bar),
-        "h"(cta_mask)
-        : "memory");
 }
 
 // 32 lanes x 32 consecutive 32-bit columns; thread t of the warp receives

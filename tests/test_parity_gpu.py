@@ -24,12 +24,11 @@ def _bits(t):
     return synth.bf16_bits(t)
 
 
-def run_gpu(corpus, regions, offsets, k, K, path, scale=None, cluster=0, mma=0, options=()):
+def run_gpu(corpus, regions, offsets, k, K, path, scale=None, mma=0, options=()):
     dev = torch.device("cuda")
     c = skip.skip_corpus_load(corpus.to(dev), row_scale=None if scale is None else scale.to(dev))
     try:
         c.set_option(skip.SKIP_OPT_PATH, path)
-        c.set_option(skip.SKIP_OPT_CLUSTER, cluster)
         c.set_option(skip.SKIP_OPT_MMA, mma)
         for opt, val in options:
             c.set_option(opt, val)
@@ -45,10 +44,12 @@ def run_gpu(corpus, regions, offsets, k, K, path, scale=None, cluster=0, mma=0, 
 
 
 def oracle_truth(corpus_np, regions_np, offsets, k, K, scale_np=None, extra=64):
+    """The oracle's extended per-region lists and its merged lists with one
+    slot past K (for the merged K / K+1 gap)."""
     N = corpus_np.shape[0]
     kk = min(N, k + extra)
     ids_ext, sc_ext = oracle.region_topk(corpus_np, regions_np, kk, row_scale=scale_np)
-    oid, osc = oracle.merge(ids_ext, sc_ext, k, np.asarray(offsets, np.int32), K)
+    oid, osc = oracle.merge(ids_ext, sc_ext, k, np.asarray(offsets, np.int32), K + 1)
     return ids_ext, sc_ext, oid, osc
 
 
@@ -66,8 +67,10 @@ def assert_parity(corpus_np, regions_np, offsets, k, K, gpu, truth, scale_np=Non
             bad.append(("region", r, probs[:3]))
     q_exact = 0
     for q in range(len(offsets) - 1):
-        ts = truths[offsets[q]:offsets[q + 1]]
-        ex, probs = checker.check_question(oid[q], osc[q], o_ids[q], o_sc[q], ts, K)
+        r0, r1 = offsets[q], offsets[q + 1]
+        ts = truths[r0:r1]
+        rescore = checker.exact_rescore(corpus_np, regions_np[r0:r1], ts, row_scale=scale_np)
+        ex, probs, _ = checker.check_question(oid[q], osc[q], o_ids[q], o_sc[q], ts, K, rid[r0:r1], rescore)
         q_exact += ex
         if probs:
             bad.append(("question", q, probs[:3]))
@@ -127,18 +130,18 @@ def test_random_bf16(case, path):
     assert_parity(cn, rn, offsets, k, K, gpu, truth)
 
 
-@pytest.mark.parametrize("cluster", [1, 2, 4, 8])
-def test_cluster_sizes(cluster):
-    """Every cluster size of the single-CTA tensor path, with query blocks
-    that do not fill the last cluster and a ragged corpus tail."""
+def test_single_cta_mma():
+    """The single-CTA (cta_group::1) tensor path over several query blocks,
+    the last one partial, and a ragged corpus tail; launched without
+    thread-block clusters."""
     N, d, R, Q, k, K = 40000, 256, 700, 30, 16, 40
     ct = synth.random_bf16(N, d, seed=77)
     rt = synth.random_bf16(R, d, seed=78)
     offsets = ragged_offsets(Q, R, seed=79)
     cn, rn = _bits(ct), _bits(rt)
     truth = oracle_truth(cn, rn, offsets, k, K)
-    gpu = run_gpu(ct, rt, offsets, k, K, skip.SKIP_PATH_TENSOR, cluster=cluster, mma=1)
-    assert gpu[4]["cluster"] == cluster and gpu[4]["mma"] == "single"
+    gpu = run_gpu(ct, rt, offsets, k, K, skip.SKIP_PATH_TENSOR, mma=1)
+    assert gpu[4]["cluster"] == 1 and gpu[4]["mma"] == "single"
     assert_parity(cn, rn, offsets, k, K, gpu, truth)
 
 
