@@ -260,7 +260,31 @@ def skip_retrieve_regions_noalloc(corpus_rows: torch.Tensor, regions: torch.Tens
     lib = load_library()
     if not (corpus_rows.is_cuda and regions.is_cuda and reg_ids.is_cuda and reg_scores.is_cuda):
         raise ValueError("skip_retrieve_regions_noalloc takes device tensors")
-    dtype = SKIP_BF16 if corpus_rows.dtype in (torch.bfloat16, torch.uint16, torch.int16) else SKIP_E4M3
+    if corpus_rows.dim() != 2:
+        raise ValueError("corpus_rows must be [N, d]")
+    if corpus_rows.dtype in (torch.bfloat16, torch.uint16, torch.int16):
+        dtype = SKIP_BF16
+        if row_scale is not None:
+            raise ValueError("a bf16 corpus takes no row_scale")
+    elif corpus_rows.dtype in (torch.uint8, torch.float8_e4m3fn):
+        dtype = SKIP_E4M3
+        if row_scale is None or row_scale.dtype != torch.float32 or not row_scale.is_cuda \
+                or row_scale.shape != (corpus_rows.shape[0],) or not row_scale.is_contiguous():
+            raise ValueError("an e4m3 corpus needs row_scale: contiguous float32 [N] on the device")
+    else:
+        raise TypeError("corpus_rows must be bf16 (or uint16 bits) or e4m3 bytes (uint8 / float8_e4m3fn)")
+    if not corpus_rows.is_contiguous():
+        raise ValueError("corpus_rows must be contiguous")
+    if regions.dim() != 2 or regions.shape[1] != corpus_rows.shape[1]:
+        raise ValueError("regions must be [R_total, d] with the corpus's d")
+    if regions.dtype not in (torch.bfloat16, torch.uint16, torch.int16) or not regions.is_contiguous():
+        raise TypeError("regions must be contiguous bf16")
+    R = regions.shape[0]
+    if reg_ids.dtype != torch.int64 or tuple(reg_ids.shape) != (R, int(k_region)) or not reg_ids.is_contiguous():
+        raise ValueError("reg_ids must be contiguous int64 [R_total, k_region]")
+    if reg_scores.dtype != torch.float32 or tuple(reg_scores.shape) != (R, int(k_region)) \
+            or not reg_scores.is_contiguous():
+        raise ValueError("reg_scores must be contiguous float32 [R_total, k_region]")
     st = lib.skip_retrieve_regions_noalloc(_ptr(corpus_rows), corpus_rows.shape[0], corpus_rows.shape[1], dtype,
                                            _ptr(row_scale), _ptr(regions), regions.shape[0], int(k_region),
                                            _ptr(reg_ids), _ptr(reg_scores), ctypes.c_void_p(_stream(stream)))

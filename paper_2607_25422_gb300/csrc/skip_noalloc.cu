@@ -41,6 +41,8 @@ void *g_noalloc_ptr[kMaxDevices];  // device address of the array, per device
 
 size_t round256(size_t v) { return (v + 255) / 256 * 256; }
 
+bool aligned(const void *p, uintptr_t a) { return ((uintptr_t)p & (a - 1)) == 0; }
+
 }  // namespace
 
 extern "C" {
@@ -54,6 +56,13 @@ skip_status_t skip_retrieve_regions_noalloc(const void *corpus_rows, int64_t N, 
     if ((dtype == SKIP_E4M3) != (row_scale != nullptr)) return SKIP_EINVAL;
     if (R_total < 0 || k_region < 1 || k_region > SKIP_MAX_K_REGION || (int64_t)k_region > N) return SKIP_EINVAL;
     if (R_total > 0 && (!regions || !reg_ids || !reg_scores)) return SKIP_EINVAL;
+    // The score kernel reads corpus rows as 16-byte vectors (d % 16 == 0 keeps
+    // every row on that boundary once the first one is), the row scales as
+    // fp32, the regions as 16-bit words; the merge writes int64 ids and fp32
+    // scores.  A misaligned pointer is refused here, before any launch.
+    if (!aligned(corpus_rows, 16) || (row_scale && !aligned(row_scale, 4))) return SKIP_EINVAL;
+    if (R_total > 0 && (!aligned(regions, 2) || !aligned(reg_ids, 8) || !aligned(reg_scores, 4)))
+        return SKIP_EINVAL;
     if (R_total == 0) return SKIP_OK;
 
     int dev = 0, major = 0, minor = 0, sms = 0;
@@ -67,8 +76,10 @@ skip_status_t skip_retrieve_regions_noalloc(const void *corpus_rows, int64_t N, 
     if (major != 10 || minor != 3 || dev >= kMaxDevices) return SKIP_EUNSUPPORTED;
 
     // Scratch: one list per (block, region row) and one per (warp, region of
-    // the current group of eight).  Sizes beyond the array are rejected.
-    const int grid = std::max(1, std::min(sms, 512));
+    // the current group of eight); sizes beyond the array are rejected.
+    // Blocks of the score kernel: one per SM, at most 512, and no more than
+    // the corpus has 256-row slices (so small corpora need little scratch).
+    const int grid = (int)std::max<int64_t>(1, std::min<int64_t>(std::min(sms, 512), (N + 255) / 256));
     const size_t lists_bytes = round256((size_t)grid * R_total * k_region * sizeof(uint64_t));
     const size_t wl_bytes = (size_t)grid * kWarpDotWarps * 8 * k_region * sizeof(uint64_t);
     if (lists_bytes + wl_bytes > kNoAllocScratchBytes) return SKIP_EUNSUPPORTED;
