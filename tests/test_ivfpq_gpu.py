@@ -189,12 +189,16 @@ def _check_search(spec, M, nprobe):
         exact += ex
     assert checked >= len(truths) // 2
     off = offsets.numpy()
-    o_m_ids, o_m_sc = oracle.merge(o_ids, o_sc, k, off, K)
+    o_m_ids, o_m_sc = oracle.merge(o_ids, o_sc, k, off, K + 1)
     for q in range(off.shape[0] - 1):
         rs = range(off[q], off[q + 1])
         if any(nprobe < cent.shape[0] and cs[r, nprobe - 1] - cs[r, nprobe] <= PROBE_TIE for r in rs):
             continue
-        _, probs = checker.check_question(q_ids[q], q_sc[q], o_m_ids[q], o_m_sc[q], truths[off[q]:off[q + 1]], K)
+
+        def rescore(j, ids, r0=off[q]):
+            return oracle.ivfpq_scores_at(idx, ce, cb.numpy(), qn, np.full(len(ids), r0 + j), ids)
+        _, probs, _ = checker.check_question(q_ids[q], q_sc[q], o_m_ids[q], o_m_sc[q], truths[off[q]:off[q + 1]],
+                                             K, g_ids[off[q]:off[q + 1]], rescore)
         assert not probs, (q, probs[:3])
     print("nprobe %d: %d regions checked, %d identical to the oracle's" % (nprobe, checked, exact))
 

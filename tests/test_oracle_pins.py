@@ -293,3 +293,35 @@ def test_e4m3_brute_force_and_scale():
     # An e4m3 corpus without scales is rejected.
     with pytest.raises(ValueError):
         oracle.region_topk(cb, qb, 8)
+
+
+# ---------------------------------------------------------------- scores at chosen pairs
+
+def test_scores_at_matches_numpy_product():
+    """oracle.scores_at (the value the parity checker uses for ids outside
+    the oracle's extended list) against a numpy fp64 product with an
+    independent decode, at random (region, id) pairs of a bf16 and of an
+    e4m3 corpus with per-row scales.  Region indices and ids are drawn
+    independently, so a swapped index, a row taken from the wrong region or
+    a missing scale changes the value; ids out of range give NaN."""
+    rng = np.random.default_rng(7)
+    N, d, R, n = 2000, 96, 9, 400
+    x = rng.standard_normal((N, d)).astype(np.float32)
+    q = rng.standard_normal((R, d)).astype(np.float32)
+    cb, qb = bf16_from_float(x), bf16_from_float(q)
+    reg = rng.integers(0, R, size=n)
+    ids = rng.integers(0, N, size=n)
+    got = oracle.scores_at(cb, qb, reg, ids)
+    want = np.einsum("tj,tj->t", decode_bf16(qb)[reg], decode_bf16(cb)[ids])
+    np.testing.assert_allclose(got, want, rtol=0, atol=1e-12)
+    # e4m3 rows times their scales
+    spec = synth.WorkloadSpec("e4m3_at", 98, N, d, "e4m3", 1, (R, R), 8, 8, "gaussian")
+    w = synth.make_workload(spec)
+    ce, sc = w.corpus.numpy(), w.row_scale.numpy()
+    xs = torch.from_numpy(ce).view(torch.float8_e4m3fn).to(torch.float32).numpy().astype(np.float64)
+    got = oracle.scores_at(ce, qb, reg, ids, row_scale=sc)
+    want = np.einsum("tj,tj->t", decode_bf16(qb)[reg], xs[ids] * sc[ids, None].astype(np.float64))
+    np.testing.assert_allclose(got, want, rtol=0, atol=1e-12)
+    assert not np.allclose(got, np.einsum("tj,tj->t", decode_bf16(qb)[reg], xs[ids]))
+    bad = oracle.scores_at(cb, qb, [0, 1], [-1, N])
+    assert np.isnan(bad).all()

@@ -24,22 +24,41 @@ pytestmark = pytest.mark.gpu
 # workload -> (questions to check, oracle extension past rank k)
 SAMPLES = {
     "tiny_100k": ("all", 32),
-    "clustered_1m": (3, 160),
-    "throughput_10m": (2, 160),
+    "clustered_1m": (16, 160),
+    "throughput_10m": (16, 160),
     "latency_fp8_6m": ("all", 32),
-    "ragged_20m": ("minmax", 160),
+    "ragged_20m": (8, 160),
+}
+
+# Floors on the strict exact-match rates (ids in the oracle's order, scores
+# within 2e-3, no near-tie excuse): the GPU sums in fp32 (~1e-6 from the
+# fp64 value), so a list differs from the oracle's only where two of its
+# scores lie closer than that, which clustered corpora with k = 100 make
+# common; the small-batch e4m3 path's three-part queries (within 2.4e-4 of
+# exact) reorder more.  Measured rates are printed.
+STRICT_FLOOR = {
+    "tiny_100k": (0.0, 0.0),
+    "clustered_1m": (0.0, 0.0),
+    "throughput_10m": (0.0, 0.0),
+    "latency_fp8_6m": (0.0, 0.0),
+    "ragged_20m": (0.0, 0.0),
 }
 
 
 def _pick_questions(offsets, how):
+    """All questions, or `how` of them drawn with a fixed seed, always
+    including a question with the fewest and one with the most regions."""
     counts = np.diff(offsets)
     Q = counts.size
     if how == "all":
         return list(range(Q))
-    if how == "minmax":
-        return sorted({int(np.argmin(counts)), int(np.argmax(counts))})
+    keep = {int(np.argmin(counts)), int(np.argmax(counts))}
     rng = np.random.default_rng(12345)
-    return sorted(rng.choice(Q, size=how, replace=False).tolist())
+    for q in rng.permutation(Q).tolist():
+        if len(keep) >= how:
+            break
+        keep.add(int(q))
+    return sorted(keep)
 
 
 @pytest.mark.parametrize("name", list(SAMPLES))
@@ -83,17 +102,24 @@ def test_workload_full_size(name):
         if probs:
             bad.append(("region", r, probs[:3]))
     at = 0
+    q_exact = q_amb = 0
     for q in qs:
         n = off[q + 1] - off[q]
         ts = truths[at:at + n]
         sub_ids, sub_sc = ids_ext[at:at + n], sc_ext[at:at + n]
+        sub_rn = rn[at:at + n]
         at += n
-        o_ids, o_sc = oracle.merge(sub_ids, sub_sc, spec.k_region, np.array([0, n], np.int32), spec.K)
-        _, probs = checker.check_question(oid[q], osc[q], o_ids[0], o_sc[0], ts, spec.K)
+        o_ids, o_sc = oracle.merge(sub_ids, sub_sc, spec.k_region, np.array([0, n], np.int32), spec.K + 1)
+        rescore = checker.exact_rescore(cn, sub_rn, ts, row_scale=sn)
+        ex, probs, amb = checker.check_question(oid[q], osc[q], o_ids[0], o_sc[0], ts, spec.K,
+                                                rid[off[q]:off[q + 1]], rescore)
+        q_exact += ex
+        q_amb += amb
         if probs:
             bad.append(("question", q, probs[:3]))
     assert not bad, "%s plan %s: %s" % (name, plan, bad[:5])
-    # Lists that match the oracle's id for id in order; the rest differ only
-    # inside the 2e-3 band (fp32 accumulation reorders scores ~1e-6 apart,
-    # which happens often among 100 clustered neighbours).
-    print("%s: %d of %d region lists identical to the oracle's" % (name, exact, len(rows)))
+    r_rate, q_rate = exact / len(rows), q_exact / len(qs)
+    print("%s: strict exact match %d of %d region lists (%.3f), %d of %d questions (%.3f); "
+          "%d questions near-tied" % (name, exact, len(rows), r_rate, q_exact, len(qs), q_rate, q_amb))
+    lo_r, lo_q = STRICT_FLOOR[name]
+    assert r_rate >= lo_r and q_rate >= lo_q, (r_rate, q_rate)
