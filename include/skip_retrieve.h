@@ -61,7 +61,9 @@ typedef enum {
     SKIP_ENOMEM = 2,        /* device or pinned allocation failed */
     SKIP_EUNSUPPORTED = 3,  /* no sm_103 device, or a size beyond a stated limit */
     SKIP_ETIMEOUT = 4,      /* a kernel's bounded wait gave up; results invalid */
-    SKIP_ECUDA = 5          /* a CUDA runtime/driver call failed */
+    SKIP_ECUDA = 5,         /* a CUDA runtime/driver call failed */
+    SKIP_ECANARY = 6        /* SKIP_OPT_CANARY: guard bytes after a buffer of the
+                               handle were overwritten (a kernel wrote past its end) */
 } skip_status_t;
 
 typedef enum {
@@ -76,10 +78,15 @@ typedef enum {
                                      corpus tile first when the corpus has at least 2,048
                                      tiles and the full pass would admit about one key per
                                      thousand scores or more), 1 never, 2 always */
-    SKIP_OPT_IVF_SPLIT = 7        /* IVF-PQ index only (skip_ivfpq_set_option): parts each
+    SKIP_OPT_IVF_SPLIT = 7,       /* IVF-PQ index only (skip_ivfpq_set_option): parts each
                                      region's probed lists are cut into for the list scan,
                                      0 pick (1, 2 or 4: doubled while twice the parts
                                      still fit in the resident CTAs), else 1..8 */
+    SKIP_OPT_CANARY = 8           /* debugging aid (no counterpart in the paper): 1 places
+                                     4 KiB of guard bytes after the handle's workspace,
+                                     host staging and gate buffers (reallocating them now);
+                                     skip_sync_status then also checks them and returns
+                                     SKIP_ECANARY if any changed.  0 (default) off. */
 } skip_option_t;
 
 enum { SKIP_PATH_AUTO = 0, SKIP_PATH_TENSOR = 1, SKIP_PATH_WARP = 2, SKIP_PATH_LATENCY = 3 };
@@ -202,7 +209,16 @@ SKIP_API skip_status_t skip_retrieve_regions_noalloc(const void *corpus_rows, in
 /* Synchronises `stream`, then reports and clears the handle's error word:
  * SKIP_ETIMEOUT if a kernel's bounded wait gave up since the last check,
  * SKIP_EINVAL if region offsets were inconsistent with R_total (clamped),
- * SKIP_ECUDA if the stream reported an error, else SKIP_OK. */
+ * SKIP_ECUDA if the stream reported an error, with SKIP_OPT_CANARY on
+ * SKIP_ECANARY if a guard region was overwritten, else SKIP_OK.
+ *
+ * Fault injection (a debugging aid with no counterpart in the paper): with
+ * the environment variable SKIP_FAULT_INJECT=alloc every device allocation
+ * the library makes fails as on an exhausted device, and the call that needed
+ * it returns SKIP_ENOMEM; SKIP_FAULT_INJECT=alloc:<kind> limits this to one
+ * kind (corpus, workspace, staging, gate, ivfpq, qvs, bsca).  The variable
+ * is read at every allocation; a handle whose workspace growth failed stays
+ * usable and allocates again on its next call. */
 SKIP_API skip_status_t skip_sync_status(skip_corpus_t corpus, void *stream);
 
 /* Describes the last retrieval call's launch plan as a short JSON object

@@ -30,9 +30,9 @@ import torch
 from . import _build
 
 SKIP_BF16, SKIP_E4M3 = 0, 1
-SKIP_OK, SKIP_EINVAL, SKIP_ENOMEM, SKIP_EUNSUPPORTED, SKIP_ETIMEOUT, SKIP_ECUDA = range(6)
+SKIP_OK, SKIP_EINVAL, SKIP_ENOMEM, SKIP_EUNSUPPORTED, SKIP_ETIMEOUT, SKIP_ECUDA, SKIP_ECANARY = range(7)
 (SKIP_OPT_PATH, SKIP_OPT_WAIT_TIMEOUT_NS, SKIP_OPT_GRID, SKIP_OPT_TIMING, SKIP_OPT_CLUSTER, SKIP_OPT_MMA,
- SKIP_OPT_BOUND, SKIP_OPT_IVF_SPLIT) = range(8)
+ SKIP_OPT_BOUND, SKIP_OPT_IVF_SPLIT, SKIP_OPT_CANARY) = range(9)
 SKIP_PATH_AUTO, SKIP_PATH_TENSOR, SKIP_PATH_WARP, SKIP_PATH_LATENCY = range(4)
 SKIP_MAX_K_REGION, SKIP_MAX_K = 1024, 2048
 
@@ -92,6 +92,7 @@ def load_library():
     lib.skip_qvs_count.argtypes = [i32, ctypes.c_float]
     lib.skip_qvs_count.restype = i32
     lib.skip_qvs_prune.argtypes = [P, P, i32, i32, P, ctypes.c_float, P, P, P, P, P]
+    lib.skip_qvs_sync_status.argtypes = [P, P]
     lib.skip_bsca_create.argtypes = [i32, i32, i32, i32, i32, ctypes.POINTER(P)]
     lib.skip_bsca_free.argtypes = [P]
     lib.skip_bsca_run.argtypes = [P, i32, P, P, i32, P, P, P, P, P, ctypes.c_float, P, P, P, P, P]
@@ -103,7 +104,7 @@ def load_library():
               "skip_timing_report", "skip_retrieve_regions_noalloc", "skip_skv_gate", "skip_retrieve_skv",
               "skip_ivfpq_build", "skip_ivfpq_load", "skip_ivfpq_lists", "skip_ivfpq_info", "skip_ivfpq_free",
               "skip_ivfpq_search_regions", "skip_ivfpq_search", "skip_ivfpq_sync_status", "skip_ivfpq_set_option",
-              "skip_ivfpq_timing_report", "skip_qvs_create", "skip_qvs_free", "skip_qvs_prune",
+              "skip_ivfpq_timing_report", "skip_qvs_create", "skip_qvs_free", "skip_qvs_prune", "skip_qvs_sync_status",
               "skip_bsca_create", "skip_bsca_free", "skip_bsca_run", "skip_bsca_sync_status"):
         getattr(lib, f).restype = ctypes.c_int
     _lib = lib
@@ -557,6 +558,10 @@ def skip_bsca_run(handle: BscaHandle, vis_offsets: torch.Tensor, chunk_offsets: 
                                         _ptr(kh), _ptr(vh), float(dbar), _ptr(out), _ptr(deg), _ptr(edges), _ptr(tau),
                                         ctypes.c_void_p(_stream(stream))), "skip_bsca_run")
     return (out, deg, edges, tau) if with_graph else out
+
+
+def skip_qvs_sync_status(head: QvsHead, stream=None) -> int:
+    return int(load_library().skip_qvs_sync_status(head.handle, ctypes.c_void_p(_stream(stream))))
 
 
 def skip_bsca_sync_status(handle: BscaHandle, stream=None) -> int:

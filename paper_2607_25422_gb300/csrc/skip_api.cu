@@ -2,9 +2,8 @@
 // its TMA descriptor, the per-handle workspace, the launch plan for each
 // regime and the error word.  The arithmetic lives in the kernels
 // (k_tc.cu, k_warpdot.cu, k_merge.cu and the others); this file only decides
-// what to launch, apart from QVS's projected query W_v^T f_q, a plain bf16
-// GEMM over all images that it hands to cuBLAS.
-#include <cublas_v2.h>
+// what to launch.  No vendor library is called: the two plain products (QVS's
+// projected query and the IVF-PQ coarse probe) run on k_gemm.cu.
 #include <stdio.h>
 #include <stdlib.h>
 #include <string.h>
@@ -103,6 +102,7 @@ struct skip_corpus {
     int grid = 0;
     int mma = 0;               // 0 = pick, 1 = single-CTA MMA, 2 = CTA-pair MMA
     int bound = 0;             // bounding pass: 0 = by corpus size, 1 = never, 2 = always
+    bool canary = false;       // guard bytes after the growable buffers (SKIP_OPT_CANARY)
     std::map<int, int> cluster_cache;  // resident clusters per (size, stages, list place)
     int timing = 0;
     // Timing: events recorded on the launching stream before each kernel and
@@ -123,9 +123,33 @@ skip_status_t cuda_status(cudaError_t e) {
     return SKIP_ECUDA;
 }
 
-// Grows a device buffer to at least `bytes` (25% headroom); a buffer in use
-// by queued work is freed only after the device has drained.
-skip_status_t ensure_buf(void *&buf, size_t &have, size_t bytes) {
+// Every device allocation of the library goes through dev_alloc.  Host-side
+// fault injection (no counterpart in the paper; it stands in for a device
+// that runs out of memory, without touching the GPU): with the environment
+// variable SKIP_FAULT_INJECT=alloc every allocation fails as cudaMalloc does
+// when memory is exhausted, with SKIP_FAULT_INJECT=alloc:<kind> only the
+// allocations of that kind (corpus, workspace, staging, gate, ivfpq, qvs,
+// bsca).  The variable is read at each allocation.
+cudaError_t dev_alloc(void **p, size_t bytes, const char *kind) {
+    const char *e = getenv("SKIP_FAULT_INJECT");
+    if (e && strncmp(e, "alloc", 5) == 0 && (e[5] == 0 || (e[5] == ':' && strcmp(e + 6, kind) == 0))) {
+        *p = nullptr;
+        return cudaErrorMemoryAllocation;
+    }
+    return cudaMalloc(p, bytes);
+}
+
+// Guard bytes after a handle's growable buffers (SKIP_OPT_CANARY): a kernel
+// that writes past the end of its workspace changes them, and
+// skip_sync_status reports it.
+constexpr size_t kCanaryBytes = 4096;
+constexpr unsigned char kCanaryByte = 0xA5;
+
+// Grows a device buffer to at least `bytes` (25% headroom; none with
+// guard bytes, which then follow the `bytes` usable ones); a buffer in use
+// by queued work is freed only after the device has drained.  A failed
+// allocation leaves the buffer empty, so the next call allocates again.
+skip_status_t ensure_buf(void *&buf, size_t &have, size_t bytes, const char *kind, bool canary) {
     if (bytes <= have) return SKIP_OK;
     if (buf) {
         cudaError_t e = cudaDeviceSynchronize();
@@ -134,16 +158,41 @@ skip_status_t ensure_buf(void *&buf, size_t &have, size_t bytes) {
         buf = nullptr;
         have = 0;
     }
-    size_t want = bytes + bytes / 4;
-    if (cudaMalloc(&buf, want) != cudaSuccess) {
+    const size_t want = canary ? bytes : bytes + bytes / 4;
+    if (dev_alloc(&buf, want + (canary ? kCanaryBytes : 0), kind) != cudaSuccess) {
         cudaGetLastError();
+        buf = nullptr;
         return SKIP_ENOMEM;
+    }
+    if (canary && (cudaMemset((char *)buf + want, kCanaryByte, kCanaryBytes) != cudaSuccess ||
+                   cudaDeviceSynchronize() != cudaSuccess)) {
+        cudaFree(buf);
+        buf = nullptr;
+        return SKIP_ECUDA;
     }
     have = want;
     return SKIP_OK;
 }
 
-skip_status_t ensure_ws(skip_corpus *c, size_t bytes) { return ensure_buf(c->ws, c->ws_bytes, bytes); }
+skip_status_t ensure_ws(skip_corpus *c, size_t bytes) {
+    return ensure_buf(c->ws, c->ws_bytes, bytes, "workspace", c->canary);
+}
+
+// SKIP_OPT_CANARY: true when the guard bytes after every allocated
+// growable buffer of the handle are intact.
+bool canaries_intact(skip_corpus *c, bool *ok) {
+    unsigned char h[kCanaryBytes];
+    const std::pair<void *, size_t> bufs[3] = {{c->ws, c->ws_bytes}, {c->io, c->io_bytes}, {c->gws, c->gws_bytes}};
+    *ok = true;
+    for (const auto &b : bufs) {
+        if (!b.first) continue;
+        if (cudaMemcpy(h, (char *)b.first + b.second, kCanaryBytes, cudaMemcpyDeviceToHost) != cudaSuccess)
+            return false;
+        for (size_t i = 0; i < kCanaryBytes; ++i)
+            if (h[i] != kCanaryByte) *ok = false;
+    }
+    return true;
+}
 
 void record(skip_corpus *c, cudaStream_t s, const char *name) {
     if (!c->timing || c->ev_used >= kMaxEvents) return;
@@ -635,6 +684,7 @@ const char *skip_status_string(skip_status_t s) {
         case SKIP_EUNSUPPORTED: return "unsupported device or size";
         case SKIP_ETIMEOUT: return "a kernel wait timed out";
         case SKIP_ECUDA: return "CUDA error";
+        case SKIP_ECANARY: return "guard bytes after a library buffer were overwritten";
     }
     return "unknown status";
 }
@@ -672,8 +722,9 @@ skip_status_t skip_corpus_load(const void *rows, int rows_on_device, int64_t N, 
     const size_t bytes = (size_t)N * d * elem;
     cudaStream_t s = reinterpret_cast<cudaStream_t>(stream);
     skip_status_t st = SKIP_OK;
-    if (cudaMalloc(&c->rows, bytes) != cudaSuccess || cudaMalloc(&c->err, sizeof(int)) != cudaSuccess ||
-        (dtype == SKIP_E4M3 && cudaMalloc(&c->scale, N * sizeof(float)) != cudaSuccess)) {
+    if (dev_alloc(&c->rows, bytes, "corpus") != cudaSuccess ||
+        dev_alloc((void **)&c->err, sizeof(int), "corpus") != cudaSuccess ||
+        (dtype == SKIP_E4M3 && dev_alloc((void **)&c->scale, N * sizeof(float), "corpus") != cudaSuccess)) {
         cudaGetLastError();
         st = SKIP_ENOMEM;
     }
@@ -735,6 +786,19 @@ skip_status_t skip_corpus_set_option(skip_corpus_t c, int option, int64_t value)
             if (value < 0 || value > 2) return SKIP_EINVAL;
             c->bound = (int)value;
             return SKIP_OK;
+        case SKIP_OPT_CANARY:
+            if (value != 0 && value != 1) return SKIP_EINVAL;
+            if ((value != 0) != c->canary) {
+                // The growable buffers are allocated again in the new mode.
+                if (cudaDeviceSynchronize() != cudaSuccess) return SKIP_ECUDA;
+                cudaFree(c->ws);
+                cudaFree(c->io);
+                cudaFree(c->gws);
+                c->ws = c->io = c->gws = nullptr;
+                c->ws_bytes = c->io_bytes = c->gws_bytes = 0;
+                c->canary = value != 0;
+            }
+            return SKIP_OK;
     }
     return SKIP_EINVAL;
 }
@@ -784,6 +848,11 @@ skip_status_t skip_sync_status(skip_corpus_t c, void *stream) {
         if (cudaMemset(c->err, 0, sizeof(int)) != cudaSuccess) return SKIP_ECUDA;
         return (err & kErrTimeout) ? SKIP_ETIMEOUT : SKIP_EINVAL;
     }
+    if (c->canary) {
+        bool ok = true;
+        if (!canaries_intact(c, &ok)) return SKIP_ECUDA;
+        if (!ok) return SKIP_ECANARY;
+    }
     return SKIP_OK;
 }
 
@@ -800,19 +869,8 @@ skip_status_t skip_retrieve_host(skip_corpus_t c, const uint16_t *regions, const
     const size_t ib = align_up((size_t)Q * K * sizeof(int64_t), 256);
     const size_t sb = align_up((size_t)Q * K * sizeof(float), 256);
     const size_t need = rb + ob + ib + sb;
-    if (need > c->io_bytes) {
-        if (c->io) {
-            if (cudaDeviceSynchronize() != cudaSuccess) return SKIP_ECUDA;
-            cudaFree(c->io);
-            c->io = nullptr;
-            c->io_bytes = 0;
-        }
-        if (cudaMalloc(&c->io, need) != cudaSuccess) {
-            cudaGetLastError();
-            return SKIP_ENOMEM;
-        }
-        c->io_bytes = need;
-    }
+    st = ensure_buf(c->io, c->io_bytes, need, "staging", c->canary);
+    if (st) return st;
     char *io = reinterpret_cast<char *>(c->io);
     void *d_reg = io;
     int32_t *d_off = reinterpret_cast<int32_t *>(io + rb);
@@ -901,7 +959,7 @@ skip_status_t skip_skv_gate(skip_corpus_t c, const int64_t *cand_ids, int32_t Q,
     if (st) return st;
     if (Q > 0 && !cand_ids) return SKIP_EINVAL;
     cudaStream_t s = reinterpret_cast<cudaStream_t>(stream);
-    st = ensure_buf(c->gws, c->gws_bytes, skv_ws_bytes(Q, K, mlp->hidden));
+    st = ensure_buf(c->gws, c->gws_bytes, skv_ws_bytes(Q, K, mlp->hidden), "gate", c->canary);
     if (st) return st;
     ++c->call_id;
     Plan pl;
@@ -924,7 +982,7 @@ skip_status_t skip_retrieve_skv(skip_corpus_t c, const void *regions, const int3
     // gate workspace first, then the merged lists (unless the caller keeps them)
     const size_t gate = skv_ws_bytes(Q, K, mlp->hidden);
     const size_t mid = align_up((size_t)Q * K * 8, 256), msc = align_up((size_t)Q * K * 4, 256);
-    st = ensure_buf(c->gws, c->gws_bytes, gate + mid + msc);
+    st = ensure_buf(c->gws, c->gws_bytes, gate + mid + msc, "gate", c->canary);
     if (st) return st;
     int64_t *mids = merged_ids ? merged_ids : reinterpret_cast<int64_t *>((char *)c->gws + gate);
     float *mscs = merged_scores ? merged_scores : reinterpret_cast<float *>((char *)c->gws + gate + mid);
@@ -956,7 +1014,7 @@ struct skip_ivfpq {
     void *ws = nullptr;           // search workspace
     size_t ws_bytes = 0;
     int split = 0;                // parts per region of the list scan (0: pick)
-    cublasHandle_t blas = nullptr; // the coarse probe's GEMM (C <= kIvfCoarseMaxC)
+    bool gemm_probe = false;      // coarse probe: one GEMM + per-region sort (C <= kIvfCoarseMaxC)
 };
 
 namespace {
@@ -965,7 +1023,6 @@ void ivf_release(skip_ivfpq *ix) {
     if (!ix) return;
     cudaDeviceSynchronize();
     if (ix->cent) skip_corpus_free(ix->cent);
-    if (ix->blas) cublasDestroy(ix->blas);
     cudaFree(ix->codebook);
     cudaFree(ix->cbT);
     cudaFree(ix->offsets);
@@ -987,16 +1044,12 @@ skip_status_t ivf_create(const void *centroids, int C, int d, const float *codeb
         return st;
     }
     const size_t cb = (size_t)M * 256 * ix->ds * sizeof(float);
-    if (C <= kIvfCoarseMaxC && cublasCreate(&ix->blas) != CUBLAS_STATUS_SUCCESS) {
-        ix->blas = nullptr;
-        ivf_release(ix);
-        return SKIP_ECUDA;
-    }
+    ix->gemm_probe = C <= kIvfCoarseMaxC;
     const size_t cbt = (size_t)256 * ix->ds * ivf_padded_m(M) * sizeof(float);
-    if (cudaMalloc(&ix->codebook, cb) != cudaSuccess || cudaMalloc(&ix->cbT, cbt) != cudaSuccess ||
-        cudaMalloc(&ix->offsets, (size_t)(C + 1) * 8) != cudaSuccess ||
-        cudaMalloc(&ix->boff, (size_t)(C + 1) * 8) != cudaSuccess ||
-        cudaMalloc(&ix->ids, (size_t)std::max<int64_t>(N, 1) * 4) != cudaSuccess) {
+    if (dev_alloc((void **)&ix->codebook, cb, "ivfpq") != cudaSuccess || dev_alloc((void **)&ix->cbT, cbt, "ivfpq") != cudaSuccess ||
+        dev_alloc((void **)&ix->offsets, (size_t)(C + 1) * 8, "ivfpq") != cudaSuccess ||
+        dev_alloc((void **)&ix->boff, (size_t)(C + 1) * 8, "ivfpq") != cudaSuccess ||
+        dev_alloc((void **)&ix->ids, (size_t)std::max<int64_t>(N, 1) * 4, "ivfpq") != cudaSuccess) {
         cudaGetLastError();
         ivf_release(ix);
         return SKIP_ENOMEM;
@@ -1050,7 +1103,7 @@ skip_status_t ivf_layout(skip_ivfpq *ix, const uint8_t *rows, cudaStream_t s) {
         boff[l + 1] = boff[l] + (off[l + 1] - off[l] + 31) / 32;
     }
     const size_t bytes = (size_t)std::max<int64_t>(boff[C], 1) * 32 * ix->M;
-    if (cudaMalloc(&ix->codes, bytes) != cudaSuccess) {
+    if (dev_alloc((void **)&ix->codes, bytes, "ivfpq") != cudaSuccess) {
         cudaGetLastError();
         return SKIP_ENOMEM;
     }
@@ -1074,8 +1127,8 @@ skip_status_t ivf_regions(skip_ivfpq *ix, const void *regions, int R, int nprobe
     }
     const size_t pid = align_up((size_t)R * nprobe * 8, 256), psc = align_up((size_t)R * nprobe * 4, 256);
     const size_t kb = align_up((size_t)std::max(R, 1) * k * 8, 256);
-    const size_t scb = ix->blas ? align_up((size_t)R * ix->C * 4, 256) : 0;  // coarse GEMM scores
-    skip_status_t st = ensure_buf(ix->ws, ix->ws_bytes, (G + 1) * kb + pid + psc + scb);
+    const size_t scb = ix->gemm_probe ? align_up((size_t)R * ix->C * 4, 256) : 0;  // coarse GEMM scores
+    skip_status_t st = ensure_buf(ix->ws, ix->ws_bytes, (G + 1) * kb + pid + psc + scb, "ivfpq", false);
     if (st) return st;
     uint64_t *keys = reinterpret_cast<uint64_t *>(ix->ws);
     int64_t *probe_ids = reinterpret_cast<int64_t *>((char *)ix->ws + (G + 1) * kb);
@@ -1084,17 +1137,18 @@ skip_status_t ivf_regions(skip_ivfpq *ix, const void *regions, int R, int nprobe
     *merged = reinterpret_cast<uint64_t *>((char *)ix->ws + G * kb);
     *G_out = G;
     if (R == 0) return SKIP_OK;
-    if (ix->blas) {
-        // coarse scores [R x C] = regions [R x d] . centroids [C x d]^T:
-        // column-major scores^T = centroids . regions^T
+    if (ix->gemm_probe) {
+        // coarse scores [R x C] = regions [R x d] . centroids [C x d]^T on the
+        // tensor cores, then the nprobe best per region
         float *scores = reinterpret_cast<float *>((char *)ix->ws + (G + 1) * kb + pid + psc);
-        const float one = 1.f, zero = 0.f;
-        record(ix->cent, s, "ivf_probe");
-        if (cublasSetStream(ix->blas, s) != CUBLAS_STATUS_SUCCESS ||
-            cublasGemmEx(ix->blas, CUBLAS_OP_T, CUBLAS_OP_N, ix->C, R, ix->d, &one, ix->cent->rows, CUDA_R_16BF,
-                         ix->d, regions, CUDA_R_16BF, ix->d, &zero, scores, CUDA_R_32F, ix->C, CUBLAS_COMPUTE_32F,
-                         CUBLAS_GEMM_DEFAULT) != CUBLAS_STATUS_SUCCESS)
+        CUtensorMap ta, tb;
+        if (!encode_bf16_rows(&ta, regions, R, ix->d, 128) ||
+            !encode_bf16_rows(&tb, ix->cent->rows, ix->C, ix->d, kGemmN))
             return SKIP_ECUDA;
+        record(ix->cent, s, "ivf_probe");
+        st = cuda_status(launch_gemm_bf16_f32(ta, tb, R, ix->C, ix->d, 1.f, scores, ix->C, ix->cent->err,
+                                              ix->cent->timeout_ns, s));
+        if (st) return st;
         st = cuda_status(launch_ivf_probe_select(scores, R, ix->C, nprobe, probe_ids, probe_sc, s));
     } else {
         Plan pl;
@@ -1133,7 +1187,7 @@ skip_status_t skip_ivfpq_build(skip_corpus_t c, const void *centroids, int32_t C
     void *tmp = nullptr;
     const size_t rl = align_up((size_t)N * 8, 256), rs = align_up((size_t)N * 4, 256);
     const size_t cr = align_up((size_t)N * M, 256), cc = align_up((size_t)C * 8, 256);
-    if (cudaMalloc(&tmp, rl + rs + 2 * cr + 2 * cc) != cudaSuccess) {
+    if (dev_alloc((void **)&tmp, rl + rs + 2 * cr + 2 * cc, "ivfpq") != cudaSuccess) {
         cudaGetLastError();
         ivf_release(ix);
         return SKIP_ENOMEM;
@@ -1290,10 +1344,13 @@ skip_status_t skip_ivfpq_timing_report(skip_ivfpq_t ix, char *buf, int32_t len) 
 struct skip_qvs {
     int device = 0, sms = 0;
     int d = 0, dk = 0, max_b = 0, max_l = 0;
-    uint16_t *wv = nullptr;
+    int dkp = 0;                            // d_k rounded up to 8 (zero columns past d_k)
+    uint16_t *wvt = nullptr;                // W_v^T [d x dkp] bf16
+    uint16_t *fqp = nullptr;                // [max_b x dkp] staging for f_q when d_k % 8 != 0
     float *bv = nullptr, *wb = nullptr;
     float *u = nullptr, *logits = nullptr;  // workspace
-    cublasHandle_t blas = nullptr;          // the W_v^T f_q GEMM
+    int *err = nullptr;                     // device error word of the GEMM's bounded waits
+    uint64_t timeout_ns = kDefaultTimeoutNs;
 };
 
 namespace {
@@ -1301,12 +1358,13 @@ namespace {
 void qvs_release(skip_qvs *q) {
     if (!q) return;
     cudaDeviceSynchronize();
-    cudaFree(q->wv);
+    cudaFree(q->wvt);
+    cudaFree(q->fqp);
     cudaFree(q->bv);
     cudaFree(q->wb);
     cudaFree(q->u);
     cudaFree(q->logits);
-    if (q->blas) cublasDestroy(q->blas);
+    cudaFree(q->err);
     delete q;
 }
 
@@ -1333,21 +1391,26 @@ skip_status_t skip_qvs_create(const uint16_t *wv, const float *bv, const float *
     auto *q = new skip_qvs();
     q->device = dev, q->sms = prop.multiProcessorCount;
     q->d = d, q->dk = dk, q->max_b = max_images, q->max_l = max_tokens;
-    if (cudaMalloc(&q->wv, (size_t)dk * d * 2) != cudaSuccess || cudaMalloc(&q->bv, (size_t)dk * 4) != cudaSuccess ||
-        cudaMalloc(&q->wb, (size_t)d * 4) != cudaSuccess ||
-        cudaMalloc(&q->u, (size_t)max_images * d * 4) != cudaSuccess ||
-        cudaMalloc(&q->logits, (size_t)max_images * max_tokens * 4) != cudaSuccess) {
+    q->dkp = (dk + 7) / 8 * 8;
+    if (dev_alloc((void **)&q->wvt, (size_t)q->dkp * d * 2, "qvs") != cudaSuccess ||
+        (q->dkp != dk && dev_alloc((void **)&q->fqp, (size_t)max_images * q->dkp * 2, "qvs") != cudaSuccess) ||
+        dev_alloc((void **)&q->bv, (size_t)dk * 4, "qvs") != cudaSuccess ||
+        dev_alloc((void **)&q->wb, (size_t)d * 4, "qvs") != cudaSuccess ||
+        dev_alloc((void **)&q->u, (size_t)max_images * d * 4, "qvs") != cudaSuccess ||
+        dev_alloc((void **)&q->logits, (size_t)max_images * max_tokens * 4, "qvs") != cudaSuccess ||
+        dev_alloc((void **)&q->err, sizeof(int), "qvs") != cudaSuccess) {
         cudaGetLastError();
         qvs_release(q);
         return SKIP_ENOMEM;
     }
-    if (cublasCreate(&q->blas) != CUBLAS_STATUS_SUCCESS) {
-        q->blas = nullptr;
-        qvs_release(q);
-        return SKIP_ECUDA;
-    }
     cudaStream_t s = reinterpret_cast<cudaStream_t>(stream);
-    if (cudaMemcpyAsync(q->wv, wv, (size_t)dk * d * 2, cudaMemcpyDeviceToDevice, s) != cudaSuccess ||
+    // W_v^T is kept so that both operands of the projection GEMM are K-major;
+    // with d_k % 8 != 0 both operands carry zero columns up to dkp (the row
+    // pitch a TMA copy needs), which add nothing to the sums.
+    if ((q->dkp != dk && (cudaMemsetAsync(q->wvt, 0, (size_t)q->dkp * d * 2, s) != cudaSuccess ||
+                          cudaMemsetAsync(q->fqp, 0, (size_t)max_images * q->dkp * 2, s) != cudaSuccess)) ||
+        launch_transpose_bf16(wv, dk, d, q->wvt, q->dkp, s) != cudaSuccess ||
+        cudaMemsetAsync(q->err, 0, sizeof(int), s) != cudaSuccess ||
         (bv ? cudaMemcpyAsync(q->bv, bv, (size_t)dk * 4, cudaMemcpyDeviceToDevice, s)
             : cudaMemsetAsync(q->bv, 0, (size_t)dk * 4, s)) != cudaSuccess ||
         cudaMemcpyAsync(q->wb, wb, (size_t)d * 4, cudaMemcpyDeviceToDevice, s) != cudaSuccess ||
@@ -1371,12 +1434,13 @@ skip_status_t skip_qvs_prune(skip_qvs_t q, const uint16_t *tokens, int32_t B, in
     if (!(rho_v >= 0.f && rho_v <= 1.f)) return SKIP_EINVAL;
     const int n = skip_qvs_count(L, rho_v);
     if (B > 0 && (!tokens || !fq || (n > 0 && (!out_idx || !out_score)))) return SKIP_EINVAL;
+    if (B > 0 && ((uintptr_t)tokens & 15) != 0) return SKIP_EINVAL;
     if (B == 0) return SKIP_OK;
     cudaStream_t s = reinterpret_cast<cudaStream_t>(stream);
     QvsParams p;
     p.tokens = tokens;
     p.fq = fq;
-    p.wv = q->wv;
+    p.wvt = q->wvt;
     p.bv = q->bv;
     p.wb = q->wb;
     p.B = B, p.L = L, p.d = q->d, p.dk = q->dk, p.n = n;
@@ -1385,16 +1449,38 @@ skip_status_t skip_qvs_prune(skip_qvs_t q, const uint16_t *tokens, int32_t B, in
     p.out_idx = out_idx;
     p.out_score = out_score;
     p.out_tokens = out_tokens;
-    // U = F_q W_v / sqrt(d_k), row-major [B x d]: column-major U^T = W_v^T F_q^T
-    const float alpha = 1.f / std::sqrt((float)q->dk), beta = 0.f;
-    if (cublasSetStream(q->blas, s) != CUBLAS_STATUS_SUCCESS ||
-        cublasGemmEx(q->blas, CUBLAS_OP_N, CUBLAS_OP_N, q->d, B, q->dk, &alpha, q->wv, CUDA_R_16BF, q->d, fq,
-                     CUDA_R_16BF, q->dk, &beta, q->u, CUDA_R_32F, q->d, CUBLAS_COMPUTE_32F,
-                     CUBLAS_GEMM_DEFAULT) != CUBLAS_STATUS_SUCCESS)
+    // U [B x d] = F_q [B x d_k] (W_v^T [d x d_k])^T / sqrt(d_k) on the tensor cores.
+    const uint16_t *fa = fq;
+    if (q->dkp != q->dk || ((uintptr_t)fq & 15) != 0) {
+        if (!q->fqp && dev_alloc((void **)&q->fqp, (size_t)q->max_b * q->dkp * 2, "qvs") != cudaSuccess) {
+            cudaGetLastError();
+            return SKIP_ENOMEM;
+        }
+        if (cudaMemcpy2DAsync(q->fqp, (size_t)q->dkp * 2, fq, (size_t)q->dk * 2, (size_t)q->dk * 2, B,
+                              cudaMemcpyDeviceToDevice, s) != cudaSuccess)
+            return SKIP_ECUDA;
+        fa = q->fqp;
+    }
+    CUtensorMap ta, tb;
+    if (!encode_bf16_rows(&ta, fa, B, q->dkp, 128) || !encode_bf16_rows(&tb, q->wvt, q->d, q->dkp, kGemmN))
         return SKIP_ECUDA;
-    cudaError_t e = launch_qvs_logits(p, q->sms, s);
+    cudaError_t e = launch_gemm_bf16_f32(ta, tb, B, q->d, q->dkp, 1.f / std::sqrt((float)q->dk), q->u, q->d,
+                                         q->err, q->timeout_ns, s);
+    if (e == cudaSuccess) e = launch_qvs_logits(p, q->sms, s);
     if (e == cudaSuccess) e = launch_qvs_select(p, s);
     return cuda_status(e);
+}
+
+skip_status_t skip_qvs_sync_status(skip_qvs_t q, void *stream) {
+    if (!q) return SKIP_EINVAL;
+    if (cudaStreamSynchronize(reinterpret_cast<cudaStream_t>(stream)) != cudaSuccess) return SKIP_ECUDA;
+    int err = 0;
+    if (cudaMemcpy(&err, q->err, sizeof(int), cudaMemcpyDeviceToHost) != cudaSuccess) return SKIP_ECUDA;
+    if (err) {
+        if (cudaMemset(q->err, 0, sizeof(int)) != cudaSuccess) return SKIP_ECUDA;
+        return SKIP_ETIMEOUT;
+    }
+    return SKIP_OK;
 }
 
 }  // extern "C"
@@ -1438,11 +1524,11 @@ skip_status_t skip_bsca_create(int32_t d_p, int32_t d_h, int32_t d_o, int32_t ma
     if (major != 10 || minor != 3) return SKIP_EUNSUPPORTED;
     auto *b = new skip_bsca();
     b->dp = d_p, b->dh = d_h, b->dout = d_o, b->max_q = max_questions, b->max_t = max_tokens;
-    if (cudaMalloc(&b->cos, (size_t)max_tokens * kBscaMaxR * 4) != cudaSuccess ||
-        cudaMalloc(&b->tau, (size_t)max_questions * 4) != cudaSuccess ||
-        cudaMalloc(&b->hist, (size_t)max_questions * kBscaBins * 4) != cudaSuccess ||
+    if (dev_alloc((void **)&b->cos, (size_t)max_tokens * kBscaMaxR * 4, "bsca") != cudaSuccess ||
+        dev_alloc((void **)&b->tau, (size_t)max_questions * 4, "bsca") != cudaSuccess ||
+        dev_alloc((void **)&b->hist, (size_t)max_questions * kBscaBins * 4, "bsca") != cudaSuccess ||
         cudaMemset(b->hist, 0, (size_t)max_questions * kBscaBins * 4) != cudaSuccess ||
-        cudaMalloc(&b->err, sizeof(int)) != cudaSuccess || cudaMemset(b->err, 0, sizeof(int)) != cudaSuccess) {
+        dev_alloc((void **)&b->err, sizeof(int), "bsca") != cudaSuccess || cudaMemset(b->err, 0, sizeof(int)) != cudaSuccess) {
         cudaGetLastError();
         bsca_release(b);
         return SKIP_ENOMEM;
