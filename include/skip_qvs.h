@@ -18,9 +18,9 @@
  * that fp32 rounding creates near 1 do not reorder tokens.
  *
  * Device pointers; calls are asynchronous and stream ordered; no CPU
- * fallback.  W_v^T f_q for all images is one bf16 GEMM with fp32 results
- * that the library hands to cuBLAS (a handle per QVS object, set to the
- * call's stream); every other step runs in the library's kernels.  Limits:
+ * fallback.  W_v^T f_q for all images is one bf16 GEMM with fp32 results on
+ * the library's own tensor-core kernel (the handle keeps W_v^T so that both
+ * operands are K-major); every step runs in the library's kernels.  Limits:
  * d a multiple of 8 and at most 8192, 1 <= d_k <= 4096, 1 <= L <= 4096.
  */
 #ifndef SKIP_QVS_H
@@ -36,7 +36,8 @@ typedef struct skip_qvs *skip_qvs_t; /* opaque: a copy of the QVS head and its w
 
 /*
  * skip_qvs_create -- copies the head's weights (device pointers): wv bf16
- * [d_k x d] row-major, bv fp32 [d_k] (NULL: zero), wb fp32 [d]; sizes the
+ * [d_k x d] row-major (kept transposed), bv fp32 [d_k] (NULL: zero), wb fp32
+ * [d]; sizes the
  * workspace for up to max_images images of up to max_tokens tokens.
  * Returns after the copies.  Errors: SKIP_EINVAL, SKIP_EUNSUPPORTED (sizes
  * beyond the limits, or no sm_103 device), SKIP_ENOMEM, SKIP_ECUDA.
@@ -58,12 +59,19 @@ SKIP_API int32_t skip_qvs_count(int32_t L, float rho_v);
  *  out_tokens optional (NULL) device bf16 [B x n x d]: the kept tokens.
  *  logits     optional (NULL) device fp32 [B x L]: every token's argument of
  *             the sigmoid.
- * Asynchronous on `stream`.  Errors: SKIP_EINVAL (null pointers, B or L
- * beyond the handle's maxima, rho_v outside [0, 1]), SKIP_ECUDA.
+ * tokens must start on a 16-byte boundary.
+ * Asynchronous on `stream`.  Errors: SKIP_EINVAL (null or misaligned
+ * pointers, B or L beyond the handle's maxima, rho_v outside [0, 1]),
+ * SKIP_ECUDA.
  */
 SKIP_API skip_status_t skip_qvs_prune(skip_qvs_t qvs, const uint16_t *tokens, int32_t B, int32_t L,
                                       const uint16_t *fq, float rho_v, int32_t *out_idx, float *out_score,
                                       uint16_t *out_tokens, float *logits, void *stream);
+
+/* Synchronises `stream`, then reports and clears the handle's error word:
+ * SKIP_ETIMEOUT if a bounded wait of the projection GEMM gave up since the
+ * last check, SKIP_ECUDA if the stream reported an error, else SKIP_OK. */
+SKIP_API skip_status_t skip_qvs_sync_status(skip_qvs_t qvs, void *stream);
 
 #ifdef __cplusplus
 }

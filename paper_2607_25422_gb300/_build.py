@@ -60,7 +60,7 @@ def build(force: bool = False, verbose: bool = False) -> str:
     with concurrent.futures.ThreadPoolExecutor(max_workers=len(sources())) as ex:
         objs = list(ex.map(compile_one, sources()))
     tmp = LIB + ".tmp.%d" % os.getpid()
-    cmd = [cc, *ARCH, "-shared", "--cudart", "static", *objs, "-lcublas", "-o", tmp]
+    cmd = [cc, *ARCH, "-shared", "--cudart", "static", *objs, "-o", tmp]
     r = subprocess.run(cmd, capture_output=True, text=True)
     if r.returncode != 0:
         raise RuntimeError("link failed:\n%s\n%s" % (r.stdout, r.stderr))

@@ -6,8 +6,9 @@
 // once: HBM-bound), and the ranking by s = sigmoid(logit) is the ranking by
 // the logit.
 //
-//  (library)     W_v^T f_q / sqrt(d_k) for all images at once: a plain bf16
-//                GEMM with fp32 results (cuBLAS), issued by the host code.
+//  k_gemm        W_v^T f_q / sqrt(d_k) for all images at once: the library's
+//                tensor-core GEMM (k_gemm.cu) on F_q [B x d_k] and the handle's
+//                copy of W_v^T [d x d_k] (k_transpose_bf16, once per handle).
 //  k_qvs_logits  u = that + w_b in shared memory and c by one warp; one warp
 //                per four tokens at a time, 16-byte loads.
 //  k_qvs_select  per image: (logit, ~index) keys sorted descending in shared
@@ -172,7 +173,34 @@ __global__ void __launch_bounds__(32 * kGatherWarps) k_qvs_gather(const QvsParam
     }
 }
 
+// W^T of a bf16 matrix W [rows x cols] (row-major) into wt [cols x ldt]
+// (ldt >= rows) through 32 x 32 tiles in shared memory: both the reads and
+// the writes are coalesced.
+__global__ void __launch_bounds__(256) k_transpose_bf16(const uint16_t *__restrict__ w, int rows, int cols,
+                                                        uint16_t *__restrict__ wt, int ldt) {
+    __shared__ uint16_t tile[32][33];
+    const int c0 = blockIdx.x * 32, r0 = blockIdx.y * 32;
+    const int tx = threadIdx.x & 31, ty = threadIdx.x >> 5;  // 8 rows of threads
+    for (int y = ty; y < 32; y += 8) {
+        const int r = r0 + y, c = c0 + tx;
+        if (r < rows && c < cols) tile[y][tx] = w[(int64_t)r * cols + c];
+    }
+    __syncthreads();
+    for (int y = ty; y < 32; y += 8) {
+        const int c = c0 + y, r = r0 + tx;
+        if (r < rows && c < cols) wt[(int64_t)c * ldt + r] = tile[tx][y];
+    }
+}
+
 }  // namespace
+
+cudaError_t launch_transpose_bf16(const uint16_t *w, int rows, int cols, uint16_t *wt, int ldt, cudaStream_t s) {
+    if (rows <= 0 || cols <= 0) return cudaSuccess;
+    if (ldt < rows) return cudaErrorInvalidValue;
+    k_transpose_bf16<<<dim3((unsigned)((cols + 31) / 32), (unsigned)((rows + 31) / 32)), 256, 0, s>>>(w, rows, cols,
+                                                                                                     wt, ldt);
+    return cudaGetLastError();
+}
 
 cudaError_t launch_qvs_logits(const QvsParams &p, int sms, cudaStream_t s) {
     if (p.B == 0) return cudaSuccess;

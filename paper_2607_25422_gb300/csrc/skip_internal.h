@@ -36,7 +36,7 @@ struct TcParams {
     int R_pad;        // padded query blocks * 128
     int k;
     int MB;           // query blocks of 128 rows holding region rows
-    int CL;           // CTAs per cluster (1, 2, 4, 8), one query block each
+    int CL;           // CTAs per cluster: 1, or 2 for a CTA pair (one query block each)
     int QG;           // query groups: ceil(MB / CL)
     int G;            // corpus chunks (lists per row)
     int64_t tiles;    // corpus tiles of kTcTileN rows this launch visits
@@ -102,6 +102,15 @@ cudaError_t launch_split_queries(const uint16_t *regions, int R, int d, uint8_t 
                                  cudaStream_t s);
 cudaError_t launch_latency(bool fp8, const CUtensorMap &ta, const CUtensorMap &tb, const LatParams &p, int grid,
                            cudaStream_t s);
+
+// ---- small dense GEMM with fp32 results (k_gemm.cu) ------------------------
+// D [M x N] (leading dimension ldd) = alpha * A [M x K] B [N x K]^T, bf16
+// operands row-major with K contiguous (K % 8 == 0).  ta: tensor map over A,
+// box 128 rows x 64 elements; tb: over B, box kGemmN rows x 64 elements; both
+// 128-byte swizzle.  err (nullable) receives kErrTimeout if a wait gives up.
+constexpr int kGemmN = 64;
+cudaError_t launch_gemm_bf16_f32(const CUtensorMap &ta, const CUtensorMap &tb, int M, int N, int K, float alpha,
+                                 float *D, int64_t ldd, int *err, uint64_t timeout_ns, cudaStream_t s);
 
 // ---- merges -------------------------------------------------------------
 // Per-region merge of G sorted lists into the exact top-k (keys and/or
@@ -212,17 +221,19 @@ constexpr int kQvsMaxL = 4096;   // tokens per image
 struct QvsParams {
     const void *tokens;     // bf16 [B x L x d]
     const void *fq;         // bf16 [B x dk]
-    const void *wv;         // bf16 [dk x d]
+    const void *wvt;        // bf16 [d x dk]: W_v^T
     const float *bv;        // [dk] or null
     const float *wb;        // [d]
     int B, L, d, dk, n;     // n tokens kept per image
-    float *u;               // [B x d] W_v^T f_q / sqrt(d_k) (written by the library GEMM)
+    float *u;               // [B x d] W_v^T f_q / sqrt(d_k) (written by the tensor-core GEMM)
     float *logits;          // [B x L] workspace
     int32_t *out_idx;       // [B x n]
     float *out_score;       // [B x n]
     void *out_tokens;       // bf16 [B x n x d] or null
 };
 cudaError_t launch_qvs_logits(const QvsParams &p, int sms, cudaStream_t s);
+// wt [cols x ldt] (first `rows` of each row) = w^T for a bf16 w [rows x cols].
+cudaError_t launch_transpose_bf16(const uint16_t *w, int rows, int cols, uint16_t *wt, int ldt, cudaStream_t s);
 cudaError_t launch_qvs_select(const QvsParams &p, cudaStream_t s);
 
 // ---- BSCA bipartite sparse cross-attention (k_bsca.cu) --------------------
