@@ -31,17 +31,20 @@ SAMPLES = {
 }
 
 # Floors on the strict exact-match rates (ids in the oracle's order, scores
-# within 2e-3, no near-tie excuse): the GPU sums in fp32 (~1e-6 from the
-# fp64 value), so a list differs from the oracle's only where two of its
-# scores lie closer than that, which clustered corpora with k = 100 make
-# common; the small-batch e4m3 path's three-part queries (within 2.4e-4 of
-# exact) reorder more.  Measured rates are printed.
+# within 2e-3, no near-tie excuse), per region list and per question: the
+# GPU sums in fp32 (~1e-6 from the fp64 value), so a list differs from the
+# oracle's only where two of its scores lie closer than that, which
+# clustered corpora with k = 100 make common; the small-batch e4m3 path's
+# three-part queries (within 2.4e-4 of exact) could reorder more, and its
+# single question is reported, not required.  Measured rates are printed
+# (at the time of writing 1.0 / 1.0, 1.0 / 0.94, 0.98 / 0.88, 1.0 / 1.0 and
+# 0.84 / 1.0).
 STRICT_FLOOR = {
-    "tiny_100k": (0.0, 0.0),
-    "clustered_1m": (0.0, 0.0),
-    "throughput_10m": (0.0, 0.0),
-    "latency_fp8_6m": (0.0, 0.0),
-    "ragged_20m": (0.0, 0.0),
+    "tiny_100k": (1.0, 1.0),
+    "clustered_1m": (0.95, 0.8),
+    "throughput_10m": (0.9, 0.75),
+    "latency_fp8_6m": (0.9, 0.0),
+    "ragged_20m": (0.75, 0.75),
 }
 
 
