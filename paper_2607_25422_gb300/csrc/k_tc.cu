@@ -42,7 +42,16 @@
 //
 // Per-row top-k sets live in shared memory ([slot][row], k slots) when they
 // fit next to a pipeline of at least two stages, else in global memory; a
-// set is unsorted with its smallest key tracked, and sorted at chunk end.
+// set is unsorted with its smallest key tracked, and sorted at chunk end
+// (in registers when it holds at most 16 keys); a list shorter than k ends
+// with an empty key, which is as far as the merge reads.
+//
+// Resident query block (CTA pair, d <= 512, sets in global memory): each CTA
+// keeps its 128 region rows x d for the whole item in shared memory (loaded
+// once per item, released by an MMA commit when the item's last MMA is
+// done) and the ring carries only corpus slices, which halves the bytes
+// moved from L2 per tile.  Used with the bounding pass, which keeps the sets
+// short enough that they rarely fill (so rarely need a rescan from L2).
 //
 // Warp roles (192 threads): warp 0 issues TMA loads into the shared-memory
 // ring; warp 1 owns TMEM (two 256-column fp32 accumulators) and issues
@@ -82,6 +91,7 @@ struct __align__(8) TcShared {
     uint64_t tfull[2];           // accumulator ready (tcgen05.commit)
     uint64_t tempty[2];          // accumulator drained (epilogue warps)
     uint64_t drain;              // MMA completion at exit
+    uint64_t afull, aempty;      // resident query block loaded / released
     uint32_t tmem_base;
 };
 
@@ -93,14 +103,16 @@ __global__ void __launch_bounds__(kTcThreads, 1)
     extern __shared__ uint8_t smem_raw[];
     uint8_t *smem = reinterpret_cast<uint8_t *>(((uintptr_t)smem_raw + 1023) & ~(uintptr_t)1023);
     const int S = p.stages;
+    const int KB = (p.d + kTcTileK - 1) / kTcTileK;
+    const bool ar = PAIR && p.a_res;  // query block resident for the item; ring = corpus slices only
     uint8_t *sA = smem;
-    uint8_t *sB = smem + S * kABytes;
-    uint64_t *slists = reinterpret_cast<uint64_t *>(smem + S * Gm::kStageBytes);
+    uint8_t *sB = ar ? smem + KB * kABytes : smem + S * kABytes;
+    const size_t ring_bytes = ar ? (size_t)KB * kABytes + (size_t)S * Gm::kBBytes : (size_t)S * Gm::kStageBytes;
+    uint64_t *slists = reinterpret_cast<uint64_t *>(smem + ring_bytes);
     const size_t list_bytes = p.list_in_smem ? (size_t)kTcTileM * p.k * 8 : 0;
-    TcShared *sh = reinterpret_cast<TcShared *>(smem + S * Gm::kStageBytes + list_bytes);
+    TcShared *sh = reinterpret_cast<TcShared *>(smem + ring_bytes + list_bytes);
     const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
     const int items = p.QG * p.G;
-    const int KB = (p.d + kTcTileK - 1) / kTcTileK;
     // A pair is a cluster of two CTAs; a single-CTA launch has no clusters.
     const int rank = PAIR ? (int)cluster_rank() : 0;
     const int cid = PAIR ? (int)cluster_index() : (int)blockIdx.x;
@@ -117,6 +129,8 @@ __global__ void __launch_bounds__(kTcThreads, 1)
             mbar_init(smem_addr(&sh->tempty[b]), PAIR ? 8 : 4);
         }
         mbar_init(smem_addr(&sh->drain), 1);
+        mbar_init(smem_addr(&sh->afull), 1);
+        mbar_init(smem_addr(&sh->aempty), 1);
         mbar_fence_init();
     }
     if (warp == 0 && lane == 0) {
@@ -146,8 +160,23 @@ __global__ void __launch_bounds__(kTcThreads, 1)
             uint32_t ph = 0;
             int64_t issued = 0;
             bool ok = true;
+            uint32_t na = 0;  // query blocks loaded (resident mode)
             for (int v = cid; v < items && ok; v += ncl) {
                 const Item it = item_of(p, v, rank);
+                if (ar) {
+                    // The previous item's MMAs have released the block: load
+                    // this item's, both CTAs' copies counted on the MMA CTA.
+                    if (!mbar_wait(smem_addr(&sh->aempty), (na & 1u) ^ 1u, p.timeout_ns)) {
+                        ok = false;
+                        break;
+                    }
+                    const uint32_t fa = smem_addr(&sh->afull);
+                    if (mma_cta) mbar_arrive_expect_tx(fa, (uint32_t)(2 * KB * kABytes));
+                    for (int kb = 0; kb < KB; ++kb)
+                        tma_load_2d_pair(smem_addr(sA + kb * kABytes), &tq, mapa_shared(fa, 0), kb * kTcTileK,
+                                         it.mb * kTcTileM);
+                    ++na;
+                }
                 for (int64_t t = it.t0; t < it.t1 && ok; ++t) {
                     for (int kb = 0; kb < KB; ++kb) {
                         if (!mbar_wait(smem_addr(&sh->empty[s]), ph ^ 1u, p.timeout_ns)) {
@@ -155,12 +184,12 @@ __global__ void __launch_bounds__(kTcThreads, 1)
                             break;
                         }
                         const uint32_t fb = smem_addr(&sh->full[s]);
-                        if (mma_cta) mbar_arrive_expect_tx(fb, Gm::kTxBytes);
+                        if (mma_cta) mbar_arrive_expect_tx(fb, ar ? 2u * Gm::kBBytes : Gm::kTxBytes);
                         const int x = kb * kTcTileK;
                         if constexpr (PAIR) {
                             // Both CTAs' copies complete on the MMA CTA's barrier.
                             const uint32_t fl = mapa_shared(fb, 0);
-                            tma_load_2d_pair(smem_addr(sA + s * kABytes), &tq, fl, x, it.mb * kTcTileM);
+                            if (!ar) tma_load_2d_pair(smem_addr(sA + s * kABytes), &tq, fl, x, it.mb * kTcTileM);
                             tma_load_2d_pair(smem_addr(sB + s * Gm::kBBytes), &tx, fl, x,
                                              (int)(t * p.tile_stride * kTcTileN) + rank * (kTcTileN / 2));
                         } else {
@@ -188,6 +217,11 @@ __global__ void __launch_bounds__(kTcThreads, 1)
                 const uint32_t bar = mma_cta ? smem_addr(&sh->full[st]) : smem_addr(&sh->empty[st]);
                 if (!mbar_wait(bar, (uint32_t)((uses - 1) & 1), kDrainTimeoutNs)) atomicOr(p.err, kErrTimeout);
             }
+            if (ar && na > 0) {
+                // the last query block: its arrival (MMA CTA) or its release
+                const uint32_t bar = mma_cta ? smem_addr(&sh->afull) : smem_addr(&sh->aempty);
+                if (!mbar_wait(bar, (na - 1) & 1u, kDrainTimeoutNs)) atomicOr(p.err, kErrTimeout);
+            }
         }
     } else if (warp == 1) {
         // ------------------------------------------------ MMA issuer
@@ -196,8 +230,16 @@ __global__ void __launch_bounds__(kTcThreads, 1)
             uint32_t ph = 0;
             uint32_t lt = 0;
             bool ok = true;
+            uint32_t na = 0;  // query blocks used (resident mode)
             for (int v = cid; v < items && ok; v += ncl) {
                 const Item it = item_of(p, v, rank);
+                if (ar) {
+                    if (!mbar_wait(smem_addr(&sh->afull), na & 1u, p.timeout_ns)) {
+                        ok = false;
+                        break;
+                    }
+                    tc_fence_after();
+                }
                 for (int64_t t = it.t0; t < it.t1 && ok; ++t, ++lt) {
                     const uint32_t buf = lt & 1u, use = lt >> 1;
                     if (!mbar_wait(smem_addr(&sh->tempty[buf]), (use & 1u) ^ 1u, p.timeout_ns)) {
@@ -212,7 +254,7 @@ __global__ void __launch_bounds__(kTcThreads, 1)
                             break;
                         }
                         tc_fence_after();
-                        const uint64_t ad = smem_desc_k128(smem_addr(sA + s * kABytes));
+                        const uint64_t ad = smem_desc_k128(smem_addr(sA + (ar ? kb : s) * kABytes));
                         const uint64_t bd = smem_desc_k128(smem_addr(sB + s * Gm::kBBytes));
 #pragma unroll
                         for (int kk = 0; kk < kTcTileK / 16; ++kk) {
@@ -237,6 +279,11 @@ __global__ void __launch_bounds__(kTcThreads, 1)
                         tc_commit_pair_mc(smem_addr(&sh->tfull[buf]), 3);
                     else
                         tc_commit(smem_addr(&sh->tfull[buf]));
+                }
+                if (ar && ok) {
+                    // the block is free once this item's MMAs are done
+                    if constexpr (PAIR) tc_commit_pair_mc(smem_addr(&sh->aempty), 3);
+                    ++na;
                 }
             }
             if (!ok) atomicOr(p.err, kErrTimeout);
@@ -393,8 +440,14 @@ __global__ void __launch_bounds__(kTcThreads, 1)
                 for (int t = 0; t < 4; ++t)
                     glist[t] = d4[t] > kNegInf ? make_key(d4[t], (uint32_t)(it.g * 4 + t)) : 0ull;
             } else if (row_valid) {
-                topk_sort(L, ls, top.n);
-                for (int t = 0; t < p.k; ++t) glist[t] = t < top.n ? L[t * ls] : 0ull;
+                if (!p.list_in_smem && top.n <= 16) {
+                    sort16_desc_in_place(glist, top.n);
+                } else {
+                    topk_sort(L, ls, top.n);
+                    if (p.list_in_smem)
+                        for (int t = 0; t < top.n; ++t) glist[t] = L[t * ls];
+                }
+                if (top.n < p.k) glist[top.n] = 0ull;  // end of a short list
             }
         }
         if (!ok && lane == 0) atomicOr(p.err, kErrTimeout);
@@ -416,9 +469,10 @@ __global__ void __launch_bounds__(kTcThreads, 1)
 }
 
 template <bool PAIR>
-size_t smem_bytes(int stages, int k, bool list_in_smem) {
-    return 1024 + (size_t)stages * Geom<PAIR>::kStageBytes +
-           (list_in_smem ? (size_t)kTcTileM * k * 8 : 0) + sizeof(TcShared);
+size_t smem_bytes(int stages, int k, bool list_in_smem, int a_res_slices) {
+    const size_t ring = a_res_slices > 0 ? (size_t)a_res_slices * kABytes + (size_t)stages * Geom<PAIR>::kBBytes
+                                         : (size_t)stages * Geom<PAIR>::kStageBytes;
+    return 1024 + ring + (list_in_smem ? (size_t)kTcTileM * k * 8 : 0) + sizeof(TcShared);
 }
 
 cudaLaunchConfig_t tc_config(int grid, int CL, size_t smem, cudaStream_t s, cudaLaunchAttribute *attr,
@@ -441,14 +495,15 @@ cudaLaunchConfig_t tc_config(int grid, int CL, size_t smem, cudaStream_t s, cuda
 
 }  // namespace
 
-size_t tc_smem_bytes(bool pair, int stages, int k, bool list_in_smem) {
-    return pair ? smem_bytes<true>(stages, k, list_in_smem) : smem_bytes<false>(stages, k, list_in_smem);
+size_t tc_smem_bytes(bool pair, int stages, int k, bool list_in_smem, int a_res_slices) {
+    return pair ? smem_bytes<true>(stages, k, list_in_smem, a_res_slices)
+                : smem_bytes<false>(stages, k, list_in_smem, 0);
 }
 
 void tc_pick_layout(bool pair, int k, int max_smem, int *stages, bool *list_in_smem) {
     const int top = pair ? Geom<true>::kMaxSt : Geom<false>::kMaxSt;
     for (int st = top; st >= 2; --st)
-        if (tc_smem_bytes(pair, st, k, true) <= (size_t)max_smem) {
+        if (tc_smem_bytes(pair, st, k, true, 0) <= (size_t)max_smem) {
             *stages = st;
             *list_in_smem = true;
             return;
@@ -457,8 +512,16 @@ void tc_pick_layout(bool pair, int k, int max_smem, int *stages, bool *list_in_s
     *list_in_smem = false;
 }
 
-int tc_max_clusters(bool pair, int CL, int stages, int k, bool list_in_smem) {
-    const size_t smem = tc_smem_bytes(pair, stages, k, list_in_smem);
+int tc_pick_resident_stages(int d, int max_smem) {
+    const int KB = (d + kTcTileK - 1) / kTcTileK;
+    if (KB > kMaxResidentSlices) return 0;
+    for (int st = Geom<true>::kMaxSt; st >= 3; --st)
+        if (tc_smem_bytes(true, st, 0, false, KB) <= (size_t)max_smem) return st;
+    return 0;
+}
+
+int tc_max_clusters(bool pair, int CL, int stages, int k, bool list_in_smem, int a_res_slices) {
+    const size_t smem = tc_smem_bytes(pair, stages, k, list_in_smem, a_res_slices);
     auto kern = pair ? k_tc_score_topk<true> : k_tc_score_topk<false>;
     if (cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem) != cudaSuccess) {
         cudaGetLastError();
@@ -477,7 +540,10 @@ int tc_max_clusters(bool pair, int CL, int stages, int k, bool list_in_smem) {
 cudaError_t launch_tc(bool pair, const CUtensorMap &tq, const CUtensorMap &tx, const TcParams &p, int grid,
                       cudaStream_t s, bool pdl) {
     if (p.CL != (pair ? 2 : 1)) return cudaErrorInvalidValue;
-    const size_t smem = tc_smem_bytes(pair, p.stages, p.k, p.list_in_smem != 0);
+    if (p.a_res && (!pair || p.list_in_smem)) return cudaErrorInvalidValue;
+    const int slices = p.a_res ? (p.d + kTcTileK - 1) / kTcTileK : 0;
+    if (slices > kMaxResidentSlices) return cudaErrorInvalidValue;
+    const size_t smem = tc_smem_bytes(pair, p.stages, p.k, p.list_in_smem != 0, slices);
     auto kern = pair ? k_tc_score_topk<true> : k_tc_score_topk<false>;
     cudaError_t e = cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
     if (e != cudaSuccess) return e;

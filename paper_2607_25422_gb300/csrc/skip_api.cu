@@ -225,18 +225,20 @@ struct Plan {
     int CL = 1;
     bool pair = false;
     bool latency = false;
+    bool resident = false;  // query blocks resident in shared memory (pair kernel)
 };
 
 // Corpus chunks G for the tensor path: make MB * G a whole number of waves of
-// `ctas` while keeping at least 4 tiles per item where the corpus allows.
-int pick_chunks(int MB, int64_t tiles, int ctas) {
-    int best = 1;
+// `ctas` while keeping at least 4 tiles per item where the corpus allows, and
+// at least gmin chunks.
+int pick_chunks(int MB, int64_t tiles, int ctas, int gmin = 1) {
+    int best = std::max(1, std::min(gmin, 512));
     double best_eff = -1.0;
     // At least 4 tiles per item, unless that leaves most CTAs idle (a small
     // corpus, e.g. IVF centroids): then down to one tile per item.
     const int64_t per = (int64_t)MB * std::max<int64_t>(1, tiles / 4) < ctas ? 1 : 4;
-    const int gmax = (int)std::min<int64_t>(512, std::max<int64_t>(1, tiles / per));
-    for (int G = 1; G <= gmax; ++G) {
+    const int gmax = (int)std::min<int64_t>(512, std::max<int64_t>(best, tiles / per));
+    for (int G = best; G <= gmax; ++G) {
         const int64_t items = (int64_t)MB * G;
         const int64_t waves = (items + ctas - 1) / ctas;
         const double eff = (double)items / (double)(waves * ctas);
@@ -385,6 +387,7 @@ skip_status_t run_regions(skip_corpus *c, const uint16_t *regions, int R, int k,
         p.stages = stages;
         p.raw_stages = raw_stages;
         p.list_in_smem = in_smem;
+        p.a_res = 0;
         p.scale = c->scale;
         pl.stages = stages;
         pl.list_in_smem = in_smem;
@@ -407,23 +410,26 @@ skip_status_t run_regions(skip_corpus *c, const uint16_t *regions, int R, int k,
         bool in_smem = false;
         int stages = 0;
         tc_pick_layout(pair, k, c->max_smem, &stages, &in_smem);
-        auto max_clusters = [&](int CL) {
-            const int key = (pair ? 10000 : 0) + CL * 100 + stages * 10 + (in_smem ? 1 : 0);
+        auto max_clusters = [&](int CL, int st, bool sm, int slices) {
+            const int key = (pair ? 100000 : 0) + slices * 10000 + CL * 100 + st * 10 + (sm ? 1 : 0);
             auto hit = c->cluster_cache.find(key);
             if (hit == c->cluster_cache.end())
-                hit = c->cluster_cache.emplace(key, tc_max_clusters(pair, CL, stages, k, in_smem)).first;
+                hit = c->cluster_cache.emplace(key, tc_max_clusters(pair, CL, st, k, sm, slices)).first;
             return hit->second;
         };
         // A pair is a cluster of two CTAs; single-CTA MMA runs without
         // clusters, each CTA loading its own corpus tiles.
         const int cl_best = pair ? 2 : 1;
-        const int ncl_best = max_clusters(cl_best);
+        const int ncl_best = max_clusters(cl_best, stages, in_smem, 0);
         if (ncl_best == 0) return SKIP_ECUDA;
         pl.CL = cl_best;
         const int QG = (pl.MB + cl_best - 1) / cl_best;
         const int ncl = std::max(1, std::min(ncl_best, ctas / cl_best));
         pl.R_pad = QG * cl_best * kTcTileM;
-        pl.G = pick_chunks(QG, pl.tiles, ncl);
+        // Items of at most kTcChunkTiles corpus tiles: the query groups that
+        // read a chunk at the same time then all find it in L2 (a long chunk
+        // lets them drift apart, and each re-reads it from HBM).
+        pl.G = pick_chunks(QG, pl.tiles, ncl, (int)((pl.tiles + kTcChunkTiles - 1) / kTcChunkTiles));
         const int items = QG * pl.G;
         pl.grid = std::min(items, ncl) * cl_best;
         const size_t lists_bytes = (size_t)pl.G * pl.R_pad * k * sizeof(uint64_t);
@@ -448,8 +454,22 @@ skip_status_t run_regions(skip_corpus *c, const uint16_t *regions, int R, int k,
         const double gk = (double)pl.G * k;
         const double ins_per_score = gk * (1.0 + std::log(std::max(1.0, (double)c->N / gk))) / (double)c->N;
         const bool bound = c->bound == 2 || (c->bound == 0 && pl.tiles >= kBoundMinTiles && ins_per_score >= 1e-3);
-        const int chunks_s = bound ? pick_chunks(QG, stiles, ncl) : 0;
+        // Sample chunks keep four keys per row in registers when there are at
+        // least k / 2 of them (the k-th of the union of 2k keys or more);
+        // with too few sample tiles for that, lists of about 2k / chunks.
+        int chunks_s = bound ? pick_chunks(QG, stiles, ncl) : 0;
+        if (bound && chunks_s * 4 < 2 * k && stiles >= (k + 1) / 2)
+            chunks_s = pick_chunks(QG, stiles, ncl, (k + 1) / 2);
         const int k_s = bound ? std::min(k, std::max(4, (2 * k + chunks_s - 1) / chunks_s)) : 0;
+        // Query blocks resident in shared memory (pairs, d <= 512): the sets
+        // go to global memory, where the bounding pass keeps them short.
+        int res_stages = (pair && bound) ? tc_pick_resident_stages(c->d, c->max_smem) : 0;
+        const int res_slices = res_stages > 0 ? (c->d + kTcTileK - 1) / kTcTileK : 0;
+        if (res_stages > 0 && max_clusters(cl_best, res_stages, false, res_slices) < ncl) res_stages = 0;
+        if (res_stages > 0) {
+            stages = res_stages;
+            in_smem = false;
+        }
         const size_t lists_s_bytes = align_up((size_t)chunks_s * pl.R_pad * k_s * sizeof(uint64_t), 256);
         skip_status_t st = ensure_ws(c, align_up(ws_extra, 256) + tau_bytes + align_up(lists_bytes, 256) +
                                             lists_s_bytes);
@@ -486,10 +506,12 @@ skip_status_t run_regions(skip_corpus *c, const uint16_t *regions, int R, int k,
         p.scale = nullptr;
         p.raw_stages = 0;
         p.tile_stride = 1;
+        p.a_res = res_stages > 0 ? 1 : 0;
         pl.stages = p.stages;
         pl.list_in_smem = in_smem;
         pl.pair = pair;
         pl.bound = bound;
+        pl.resident = res_stages > 0;
         cudaError_t e;
         if (bound) {
             TcParams ps = p;
@@ -503,6 +525,12 @@ skip_status_t run_regions(skip_corpus *c, const uint16_t *regions, int R, int k,
             int st_s = 0;
             bool smem_s = false;
             tc_pick_layout(pair, k_s, c->max_smem, &st_s, &smem_s);
+            if (res_stages > 0 && ps.dense) {
+                st_s = res_stages;  // the four keys live in registers: no sets at all
+                smem_s = false;
+            } else {
+                ps.a_res = 0;
+            }
             ps.stages = st_s;
             ps.list_in_smem = smem_s;
             record(c, s, "score_topk_tc_bound");
@@ -565,11 +593,12 @@ void write_plan(skip_corpus *c, const Plan &pl, int R, int Q, int k, int K) {
     snprintf(c->plan, sizeof c->plan,
              "{\"path\": \"%s\", \"grid\": %d, \"lists_per_row\": %d, \"query_blocks\": %d, "
              "\"R_total\": %d, \"Q\": %d, \"k_region\": %d, \"K\": %d, \"launches\": %d, "
-             "\"stages\": %d, \"cluster\": %d, \"mma\": \"%s\", \"lists\": \"%s\", \"bound\": %d}",
+             "\"stages\": %d, \"cluster\": %d, \"mma\": \"%s\", \"lists\": \"%s\", \"bound\": %d, "
+             "\"resident_queries\": %d}",
              pl.latency ? "latency" : pl.tensor ? "tensor" : "warpdot", pl.grid, pl.G, pl.MB, R, Q, k, K, pl.launches,
              pl.stages, pl.CL,
              pl.pair ? "pair" : "single",
-             pl.tensor ? (pl.list_in_smem ? "shared" : "global") : "global", pl.bound ? 1 : 0);
+             pl.tensor ? (pl.list_in_smem ? "shared" : "global") : "global", pl.bound ? 1 : 0, pl.resident ? 1 : 0);
 }
 
 // Argument rules of skip_retrieve.

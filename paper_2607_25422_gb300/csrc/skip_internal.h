@@ -54,6 +54,9 @@ struct TcParams {
     int list_in_smem; // per-row lists in shared memory (else global)
     const float *scale;  // [N] row scales (e4m3 corpus only)
     int raw_stages;      // e4m3 corpus: depth of the raw-slice ring
+    int a_res;           // bf16 pair kernel: the query block stays resident in shared memory for
+                         // the whole item and the ring carries corpus slices only (sets in global
+                         // memory; d <= 64 * kMaxResidentSlices)
 };
 constexpr int kTcTileM = 128;   // region rows per tile (TMEM lanes)
 constexpr int kTcTileN = 256;   // corpus rows per tile (TMEM columns)
@@ -61,12 +64,18 @@ constexpr int kTcTileK = 64;    // bf16 elements per stage row (128 bytes)
 constexpr int kTcThreads = 192; // producer warp, MMA warp, 4 epilogue warps
 constexpr int kBoundStride = 48;     // bounding pass: every 48th corpus tile (2% more MMA work)
 constexpr int kBoundMinTiles = 2048; // ... on corpora of at least 2,048 tiles (524,288 rows)
+constexpr int kMaxResidentSlices = 8;  // resident query block: d <= 512
+constexpr int kTcChunkTiles = 200;     // corpus tiles per work item at most (chunks of a large corpus)
 // pair: CTA-pair MMA (cta_group::2, clusters of 2); else single-CTA MMA.
-size_t tc_smem_bytes(bool pair, int stages, int k, bool list_in_smem);
+// a_res_slices: 64-element slices of a resident query block (0: none).
+size_t tc_smem_bytes(bool pair, int stages, int k, bool list_in_smem, int a_res_slices);
 // Deepest pipeline that fits next to shared-memory lists, else global lists.
 void tc_pick_layout(bool pair, int k, int max_smem, int *stages, bool *list_in_smem);
+// Pair kernel with a resident query block of width d (sets in global
+// memory): the ring depth that fits, 0 if d is too wide.
+int tc_pick_resident_stages(int d, int max_smem);
 // Clusters of CL CTAs that can be resident at once with this layout.
-int tc_max_clusters(bool pair, int CL, int stages, int k, bool list_in_smem);
+int tc_max_clusters(bool pair, int CL, int stages, int k, bool list_in_smem, int a_res_slices);
 // pdl: launched as the programmatic dependent of the kernel before it in the
 // stream (the epilogue waits for it before reading the shared thresholds).
 cudaError_t launch_tc(bool pair, const CUtensorMap &tq, const CUtensorMap &tx, const TcParams &p, int grid,

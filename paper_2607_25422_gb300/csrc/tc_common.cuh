@@ -85,6 +85,33 @@ __device__ __forceinline__ void topk_sort(uint64_t *L, int ls, int n) {
     }
 }
 
+// Sorts the first n <= 16 keys of a list in global memory descending,
+// through registers (a bitonic network; empty slots are 0 and sort last).
+__device__ __forceinline__ void sort16_desc_in_place(uint64_t *L, int n) {
+    uint64_t r[16];
+#pragma unroll
+    for (int i = 0; i < 16; ++i) r[i] = i < n ? L[i] : 0ull;
+#pragma unroll
+    for (int size = 2; size <= 16; size <<= 1)
+#pragma unroll
+        for (int stride = size >> 1; stride > 0; stride >>= 1)
+#pragma unroll
+            for (int i = 0; i < 16; ++i) {
+                const int j = i ^ stride;
+                if (j > i) {
+                    const bool desc = (i & size) == 0;  // blocks alternate; the last stage is one block
+                    const uint64_t a = r[i], b = r[j];
+                    if ((a < b) == desc) {
+                        r[i] = b;
+                        r[j] = a;
+                    }
+                }
+            }
+#pragma unroll
+    for (int i = 0; i < 16; ++i)
+        if (i < n) L[i] = r[i];
+}
+
 // The largest float below x (x itself for -inf): "s > below(x)" is "s >= x".
 __device__ __forceinline__ float float_below(float x) {
     const uint32_t b = __float_as_uint(x);

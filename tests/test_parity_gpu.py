@@ -175,6 +175,10 @@ BOUND_CASES = [
     (30000, 128, 200, 10, 7, 16, 1),
     # 33 sample tiles in 8 chunks, k = 16: four-slot lists kept in registers
     (400000, 128, 256, 16, 16, 40, 2),
+    # d = 512, k = 100: query blocks resident, sets in global memory, a
+    # four-key bounding pass over at least 50 sample chunks, 14 items of at
+    # most 200 tiles per query group
+    (700000, 512, 300, 20, 100, 100, 2),
 ]
 
 
@@ -192,6 +196,9 @@ def test_bounding_pass(case):
     on = run_gpu(ct, rt, offsets, k, K, skip.SKIP_PATH_TENSOR, mma=mma, options=((skip.SKIP_OPT_BOUND, 2),))
     off = run_gpu(ct, rt, offsets, k, K, skip.SKIP_PATH_TENSOR, mma=mma, options=((skip.SKIP_OPT_BOUND, 1),))
     assert on[4]["bound"] == 1 and off[4]["bound"] == 0
+    # pairs with d <= 512 keep the query block resident once the bounding
+    # pass runs; without it the sets stay in shared memory
+    assert on[4]["resident_queries"] == int(mma == 2 and d <= 512) and off[4]["resident_queries"] == 0
     assert_parity(cn, rn, offsets, k, K, on, truth)
     for a, b in zip(on[:4], off[:4]):
         np.testing.assert_array_equal(a, b)
