@@ -22,14 +22,20 @@
 // bf16 corpus: B is the bf16 queries themselves (kind::f16).
 //
 // Epilogue: lane = corpus row, so for each query the 32 rows of a warp are
-// compared with the query's threshold at once (a ballot); lane q owns the
+// compared with the query's filter at once (a ballot); lane q owns the
 // running top-k set of query q for its warp's rows (an unsorted set with its
 // minimum tracked, in shared memory) and inserts the ballot's survivors in
-// increasing row (= id) order.  A per-query threshold shared by all CTAs
-// (atomic max of the sets' k-th scores) prunes the rest.  At the end of a
-// chunk the four warps' sets of each query are merged into the chunk's list.
+// increasing row (= id) order.  Eight epilogue warps in two sets of four
+// drain the two TMEM accumulators in turn (set j takes the tiles that land
+// in accumulator j), so that the survivor work of one tile overlaps the
+// ballots of the next.  A query's filter is the largest of its own set's
+// k-th score, the k-th scores of the CTA's other warps' sets (each is k
+// distinct rows' scores, so a score below it cannot reach the CTA's top k)
+// and a threshold shared by all CTAs (atomic max of the sets' k-th scores).
+// At the end of a chunk the eight warps' sets of each query are merged into
+// the chunk's list.
 //
-// Warps (192 threads): 0 TMA producer, 1 TMEM owner and MMA issuer, 2..5
+// Warps (320 threads): 0 TMA producer, 1 TMEM owner and MMA issuer, 2..9
 // epilogue.  Bounded waits and drains as in the other tensor kernels.
 #include "skip_device.cuh"
 #include "skip_internal.h"
@@ -44,7 +50,8 @@ constexpr int kRows = 128;                      // corpus rows per tile
 constexpr int kSlice = 128;                     // bytes of a row per K slice
 constexpr int kAStage = kRows * kSlice;         // 16 KB
 constexpr int kMaxStages = 12;
-constexpr int kThreads = 192;
+constexpr int kEpiWarps = 8;                    // two sets of four
+constexpr int kThreads = 64 + 32 * kEpiWarps;
 constexpr uint32_t kTmemCols = 256;             // two 128-column accumulators
 constexpr uint64_t kDrainTimeoutNs = 1000000000ull;
 
@@ -55,12 +62,12 @@ struct __align__(8) LatShared {
     uint64_t tfull[2];
     uint64_t tempty[2];
     uint64_t drain;
-    uint64_t sorted;  // the 128 epilogue threads have sorted their sets
+    uint64_t sorted;  // the epilogue threads have sorted their sets
     uint64_t merged;  // ... and merged them into the chunk's lists
     uint32_t tmem_base;
     float qscale[3][kLatMaxR];
-    float thr[4][32];   // per epilogue warp: each query's set threshold (k-th score)
-    float gthr[4][32];  // ... and the shared threshold it has adopted
+    float thr[kEpiWarps][32];   // per epilogue warp: each query's set threshold (k-th score)
+    float filt[kEpiWarps][32];  // ... and the filter its next ballots use (strict compare)
 };
 
 template <bool FP8>
@@ -75,8 +82,8 @@ __global__ void __launch_bounds__(kThreads, 1)
     uint8_t *sB = smem;
     uint8_t *sA = sB + KS * bslice;
     uint64_t *slists = reinterpret_cast<uint64_t *>(sA + S * kAStage);
-    float *strans = reinterpret_cast<float *>(slists + (size_t)4 * p.R * p.k);  // [4][32][33]
-    LatShared *sh = reinterpret_cast<LatShared *>(strans + 4 * 32 * 33);
+    float *strans = reinterpret_cast<float *>(slists + (size_t)kEpiWarps * p.R * p.k);  // [8][32][33]
+    LatShared *sh = reinterpret_cast<LatShared *>(strans + kEpiWarps * 32 * 33);
     const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
     constexpr int kElemsPerSlice = FP8 ? 128 : 64;
     constexpr uint32_t kIdescBase = FP8 ? idesc_e4m3_f32(kRows, 16) : idesc_bf16_f32(kRows, 16);
@@ -93,9 +100,13 @@ __global__ void __launch_bounds__(kThreads, 1)
             mbar_init(smem_addr(&sh->tempty[b]), 4);
         }
         mbar_init(smem_addr(&sh->drain), 1);
-        mbar_init(smem_addr(&sh->sorted), 128);
-        mbar_init(smem_addr(&sh->merged), 128);
+        mbar_init(smem_addr(&sh->sorted), 32 * kEpiWarps);
+        mbar_init(smem_addr(&sh->merged), 32 * kEpiWarps);
         mbar_fence_init();
+    }
+    for (int i = threadIdx.x; i < kEpiWarps * 32; i += blockDim.x) {
+        sh->thr[i / 32][i % 32] = -__int_as_float(0x7f800000);
+        sh->filt[i / 32][i % 32] = -__int_as_float(0x7f800000);
     }
     if (FP8)
         for (int i = threadIdx.x; i < 3 * kLatMaxR; i += blockDim.x) {
@@ -199,30 +210,34 @@ __global__ void __launch_bounds__(kThreads, 1)
             if (!mbar_wait(smem_addr(&sh->drain), 0, kDrainTimeoutNs)) atomicOr(p.err, kErrTimeout);
         }
     } else {
-        // ------------------------------------------------ epilogue (warps 2..5)
-        const int sub = warp & 3;
+        // ------------------------------------------------ epilogue (warps 2..9)
+        const int ew = warp - 2;        // epilogue warp 0..7
+        const uint32_t set = ew >> 2;   // drains accumulator `set`: the tiles with lt % 2 == set
+        const int sub = warp & 3;       // TMEM lane quadrant this warp may read
         const uint32_t lane_addr = (uint32_t)(sub * 32) << 16;
         const float kNegInf = -__int_as_float(0x7f800000);
         const int R = p.R, k = p.k;
-        uint64_t *Lw = slists + (size_t)sub * R * k;  // this warp's set of query q at Lw + q * k
+        uint64_t *Lw = slists + (size_t)ew * R * k;  // this warp's set of query q at Lw + q * k
+        float *thr_w = sh->thr[ew], *filt_w = sh->filt[ew];
+        float *Sw = strans + ew * 32 * 33;  // [32 rows][33]: one row's scores per lane
         uint32_t lt = 0, chunk = 0;
         bool ok = true;
         for (int v = blockIdx.x; v < items && ok; v += gridDim.x) {
             const int64_t t0 = (int64_t)v * p.tiles / p.G, t1 = (int64_t)(v + 1) * p.tiles / p.G;
             // Lane q keeps query q's set for this warp's rows of the chunk; its
-            // two thresholds are mirrored in shared memory for the other lanes.
+            // k-th score and its filter are mirrored in shared memory.
+            // A mirror in thr[][] only ever rises: it is the k-th score of k
+            // distinct corpus rows (of this chunk or an earlier one), so it
+            // bounds the k-th best score over the whole corpus from below.
             RowTopK top;
-            float thr = kNegInf, gthr = kNegInf;
+            float thr = kNegInf;  // own set's k-th score (strict: later rows lose ties)
+            float cthr = kNegInf; // filter: s > cthr  <=>  s > thr and s >= every bound from elsewhere
             uint32_t published = 0;
-            float *thr_w = sh->thr[sub], *gthr_w = sh->gthr[sub];
-            float *Sw = strans + sub * 32 * 33;  // [32 rows][33]: one row's scores per lane
-            thr_w[lane] = kNegInf;
-            gthr_w[lane] = kNegInf;
             // The shared threshold is read one tile ahead, off the critical path.
             uint32_t tau_next = lane < R ? *reinterpret_cast<volatile uint32_t *>(p.tau + lane) : 0u;
-            __syncwarp();
             for (int64_t t = t0; t < t1; ++t, ++lt) {
                 const uint32_t buf = lt & 1u, use = lt >> 1;
+                if (buf != set) continue;
                 if (!mbar_wait(smem_addr(&sh->tfull[buf]), use & 1u, p.timeout_ns)) {
                     ok = false;
                     break;
@@ -234,10 +249,18 @@ __global__ void __launch_bounds__(kThreads, 1)
                         atomicMax(p.tau + lane, mine);
                         published = mine;
                     }
-                    if (tau_next > published) gthr = score_of_ord(tau_next);
+                    // Bound from elsewhere: the shared threshold and the
+                    // mirrors of the CTA's warps (possibly stale, hence lower:
+                    // still bounds).
+                    float other = tau_next ? score_of_ord(tau_next) : kNegInf;
                     tau_next = *reinterpret_cast<volatile uint32_t *>(p.tau + lane);
-                    gthr_w[lane] = gthr;
+                    const volatile float *vt = &sh->thr[0][0];
+#pragma unroll
+                    for (int w = 0; w < kEpiWarps; ++w) other = fmaxf(other, vt[w * 32 + lane]);
+                    cthr = fmaxf(thr, float_below(other));
+                    filt_w[lane] = cthr;
                 }
+                __syncwarp();
                 const int64_t rowbase = t * kRows + sub * 32;
                 const int64_t i = rowbase + lane;
                 const bool valid = i < p.N;
@@ -258,7 +281,7 @@ __global__ void __launch_bounds__(kThreads, 1)
                 if (lane == 0) mbar_arrive(smem_addr(&sh->tempty[buf]));
                 const float cs = FP8 ? (valid ? __ldg(p.corpus_scale + i) : 0.0f) : 1.0f;
                 // All queries' scores of this lane's row, and one ballot per
-                // query against that query's thresholds (branch-free).
+                // query against that query's filter (branch-free).
                 float sc[kLatMaxR];
                 uint32_t m[kLatMaxR];
                 uint32_t anym = 0;
@@ -271,7 +294,7 @@ __global__ void __launch_bounds__(kThreads, 1)
                     else
                         sq = __uint_as_float(d0[q]);
                     sc[q] = sq;
-                    m[q] = __ballot_sync(0xffffffffu, valid && q < R && sq > thr_w[q] && sq >= gthr_w[q]);
+                    m[q] = __ballot_sync(0xffffffffu, valid && q < R && sq > filt_w[q]);
                     anym |= m[q];
                 }
                 if (anym) {
@@ -283,21 +306,26 @@ __global__ void __launch_bounds__(kThreads, 1)
                     __syncwarp();
                     uint32_t mine_m = select32(m, lane);
                     if (lane < R) {
+                        const float below_other = cthr > thr ? cthr : kNegInf;  // the part of cthr from elsewhere
                         while (mine_m) {
                             const int l = __ffs(mine_m) - 1;
                             mine_m &= mine_m - 1;
                             const float sl = Sw[l * 33 + lane];
-                            if (sl > thr && sl >= gthr) {
+                            if (sl > cthr) {
                                 topk_add(Lw + (size_t)lane * k, 1, k, top, make_key(sl, (uint32_t)(rowbase + l)));
-                                if (top.n == k) thr = key_score(top.min_key);
+                                if (top.n == k) {
+                                    thr = key_score(top.min_key);
+                                    cthr = fmaxf(thr, below_other);
+                                }
                             }
                         }
-                        thr_w[lane] = thr;
+                        if (thr > thr_w[lane]) thr_w[lane] = thr;
+                        filt_w[lane] = cthr;
                     }
                     __syncwarp();
                 }
             }
-            // Chunk done: sort each set, then merge the four warps' sets of
+            // Chunk done: sort each set, then merge the eight warps' sets of
             // every query into the chunk's list (the two hand-offs between
             // the epilogue warps are bounded waits, like every other wait).
             if (lane < R) {
@@ -307,9 +335,9 @@ __global__ void __launch_bounds__(kThreads, 1)
             const uint32_t par = (uint32_t)(chunk & 1);
             mbar_arrive(smem_addr(&sh->sorted));
             if (!mbar_wait(smem_addr(&sh->sorted), par, p.timeout_ns)) ok = false;
-            for (int q = sub; q < R && ok; q += 4) {
+            for (int q = ew; q < R && ok; q += kEpiWarps) {
                 uint64_t *out = p.lists + ((int64_t)v * R + q) * k;
-                warp_merge_topk<1>(slists + (size_t)q * k, (int64_t)R * k, 4, k, k,
+                warp_merge_topk<1>(slists + (size_t)q * k, (int64_t)R * k, kEpiWarps, k, k,
                                    [&](int idx, uint64_t key) { out[idx] = key; });
             }
             mbar_arrive(smem_addr(&sh->merged));
@@ -380,8 +408,8 @@ __global__ void __launch_bounds__(256) k_split_queries(const uint16_t *__restric
 }
 
 size_t smem_bytes(int Npad, int slices, int stages, int R, int k) {
-    return 1024 + (size_t)slices * Npad * kSlice + (size_t)stages * kAStage + (size_t)4 * R * k * 8 +
-           (size_t)4 * 32 * 33 * 4 + sizeof(LatShared);
+    return 1024 + (size_t)slices * Npad * kSlice + (size_t)stages * kAStage + (size_t)kEpiWarps * R * k * 8 +
+           (size_t)kEpiWarps * 32 * 33 * 4 + sizeof(LatShared);
 }
 
 }  // namespace
