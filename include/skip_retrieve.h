@@ -82,11 +82,17 @@ typedef enum {
                                      region's probed lists are cut into for the list scan,
                                      0 pick (1, 2 or 4: doubled while twice the parts
                                      still fit in the resident CTAs), else 1..8 */
-    SKIP_OPT_CANARY = 8           /* debugging aid (no counterpart in the paper): 1 places
+    SKIP_OPT_CANARY = 8,          /* debugging aid (no counterpart in the paper): 1 places
                                      4 KiB of guard bytes after the handle's workspace,
                                      host staging and gate buffers (reallocating them now);
                                      skip_sync_status then also checks them and returns
                                      SKIP_ECANARY if any changed.  0 (default) off. */
+    SKIP_OPT_RESIDENT = 9         /* bf16 tensor path with CTA pairs, d <= 512, after a
+                                     bounding pass: 0 auto (each CTA keeps its query block in
+                                     shared memory for a work item and the per-row sets in
+                                     global memory when the items can be sized so that about
+                                     16 keys or fewer reach a set), 1 never, 2 whenever the
+                                     shape allows (for tests) */
 } skip_option_t;
 
 enum { SKIP_PATH_AUTO = 0, SKIP_PATH_TENSOR = 1, SKIP_PATH_WARP = 2, SKIP_PATH_LATENCY = 3 };

@@ -63,9 +63,10 @@ typedef struct {
  *             input slot (-inf for empty ones).
  * Uses the handle's gate workspace (grown on demand, which synchronises the
  * device once).  Asynchronous on `stream`.
- * Errors: SKIP_EINVAL (null pointers, K < 1 or > SKIP_MAX_K, bad hidden,
- * tau or rho), SKIP_EUNSUPPORTED (e4m3 corpus, d % 64 != 0, d > 1024),
- * SKIP_ENOMEM, SKIP_ECUDA.
+ * qbar, vbar and the mlp's w1 must start on 16-byte boundaries.
+ * Errors: SKIP_EINVAL (null or misaligned pointers, K < 1 or > SKIP_MAX_K,
+ * bad hidden, tau or rho), SKIP_EUNSUPPORTED (e4m3 corpus, d % 64 != 0,
+ * d > 1024), SKIP_ENOMEM, SKIP_ECUDA.
  */
 SKIP_API skip_status_t skip_skv_gate(skip_corpus_t corpus, const int64_t *cand_ids, int32_t num_questions,
                                      int32_t K, const uint16_t *qbar, const uint16_t *vbar,

@@ -7,13 +7,17 @@
 //  * the IVF-PQ coarse probe scores S = Q C^T of all regions against every
 //    centroid (the inverted file's coarse quantiser, §4.1 "Implementation").
 //
-//   D[m][n] = alpha * sum_k A[m][k] B[n][k],   A [M x K], B [N x K] bf16
-//   row-major (K contiguous), D fp32 row-major with leading dimension ldd.
+//   D[m][n] = alpha * (sum_k A[m][k] B[n][k] + sum_k A2[m][k] B2[n][k]) + bias[n]
+//   A [M x K], B [N x K], A2 [M x K2], B2 [N x K2] bf16 row-major (K
+//   contiguous; the second product and the bias are optional), D fp32
+//   row-major with leading dimension ldd.  The SKV gate's per-question half
+//   of layer 1 is such a sum (its qbar and vbar column blocks of W1).
 //
-// One CTA computes one 128 x kGemmN tile of D: warp 0 streams K slices of 64
-// elements (128 bytes, 128-byte swizzle) of both operands into a four-stage
+// One CTA computes one 128 x BN tile of D (BN = 64, or 32 when that leaves
+// too few tiles to occupy the GPU): warp 0 streams K slices of 64 elements
+// (128 bytes, 128-byte swizzle) of both operands into an eight-stage
 // shared-memory ring by TMA (rows past M or N are zero-filled by the copy),
-// one thread of warp 1 issues tcgen05.mma (kind::f16, M = 128, N = kGemmN)
+// one thread of warp 1 issues tcgen05.mma (kind::f16, M = 128, N = BN)
 // into a TMEM accumulator, and warps 2..5 read it back (warp w: TMEM lanes
 // 32 (w mod 4) .. + 31, i.e. rows of D) and store their rows, masked at the
 // M and N edges.  Every wait is bounded; a wait that gives up sets *err (if
@@ -24,13 +28,17 @@
 namespace skipk {
 namespace {
 
-constexpr int kStages = 4;
+constexpr int kStages = 8;
 constexpr int kABytes = 128 * 64 * 2;      // 16 KB: 128 rows x 64 elements
-constexpr int kBBytes = kGemmN * 64 * 2;   // 8 KB
-constexpr int kStageBytes = kABytes + kBBytes;
 constexpr int kThreads = 192;
-constexpr uint32_t kTmemCols = kGemmN;     // one fp32 accumulator (power of two >= 32)
 constexpr uint64_t kDrainTimeoutNs = 1000000000ull;
+
+template <int BN>
+struct GemmGeom {
+    static constexpr int kBBytes = BN * 64 * 2;
+    static constexpr int kStageBytes = kABytes + kBBytes;
+    static constexpr uint32_t kTmemCols = BN;  // one fp32 accumulator (power of two >= 32)
+};
 
 struct __align__(8) GemmShared {
     uint64_t full[kStages];
@@ -39,18 +47,25 @@ struct __align__(8) GemmShared {
     uint32_t tmem_base;
 };
 
+template <int BN>
 __global__ void __launch_bounds__(kThreads, 1)
-    k_gemm_bf16_f32(const __grid_constant__ CUtensorMap ta, const __grid_constant__ CUtensorMap tb, int M, int N,
-                    int K, float alpha, float *__restrict__ D, int64_t ldd, int *err, uint64_t timeout_ns) {
+    k_gemm_bf16_f32(const __grid_constant__ CUtensorMap ta, const __grid_constant__ CUtensorMap tb,
+                    const __grid_constant__ CUtensorMap ta2, const __grid_constant__ CUtensorMap tb2, int M, int N,
+                    int K, int K2, float alpha, const float *__restrict__ bias, float *__restrict__ D, int64_t ldd,
+                    int *err, uint64_t timeout_ns) {
+    constexpr int kBBytes = GemmGeom<BN>::kBBytes;
+    constexpr int kStageBytes = GemmGeom<BN>::kStageBytes;
+    constexpr uint32_t kTmemCols = GemmGeom<BN>::kTmemCols;
     extern __shared__ uint8_t smem_raw[];
     uint8_t *smem = reinterpret_cast<uint8_t *>(((uintptr_t)smem_raw + 1023) & ~(uintptr_t)1023);
     uint8_t *sA = smem;
     uint8_t *sB = smem + kStages * kABytes;
     GemmShared *sh = reinterpret_cast<GemmShared *>(smem + kStages * kStageBytes);
     const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
-    const int m0 = blockIdx.x * 128, n0 = blockIdx.y * kGemmN;
-    const int KB = (K + 63) / 64;
-    constexpr uint32_t kIdesc = idesc_bf16_f32(128, kGemmN);
+    const int m0 = blockIdx.x * 128, n0 = blockIdx.y * BN;
+    const int KB1 = (K + 63) / 64;
+    const int KB = KB1 + (K2 + 63) / 64;
+    constexpr uint32_t kIdesc = idesc_bf16_f32(128, BN);
 
     if (threadIdx.x == 0) {
         for (int s = 0; s < kStages; ++s) {
@@ -63,6 +78,10 @@ __global__ void __launch_bounds__(kThreads, 1)
     if (warp == 0 && lane == 0) {
         tma_prefetch_desc(&ta);
         tma_prefetch_desc(&tb);
+        if (K2 > 0) {
+            tma_prefetch_desc(&ta2);
+            tma_prefetch_desc(&tb2);
+        }
     }
     if (warp == 1) {
         tmem_alloc(smem_addr(&sh->tmem_base), kTmemCols);
@@ -86,8 +105,10 @@ __global__ void __launch_bounds__(kThreads, 1)
                 }
                 const uint32_t fb = smem_addr(&sh->full[s]);
                 mbar_arrive_expect_tx(fb, kStageBytes);
-                tma_load_2d(smem_addr(sA + s * kABytes), &ta, fb, kb * 64, m0);
-                tma_load_2d(smem_addr(sB + s * kBBytes), &tb, fb, kb * 64, n0);
+                const bool first = kb < KB1;
+                const int x = (first ? kb : kb - KB1) * 64;
+                tma_load_2d(smem_addr(sA + s * kABytes), first ? &ta : &ta2, fb, x, m0);
+                tma_load_2d(smem_addr(sB + s * kBBytes), first ? &tb : &tb2, fb, x, n0);
                 ++issued;
             }
             // copies in flight: the last load issued on every stage
@@ -128,23 +149,32 @@ __global__ void __launch_bounds__(kThreads, 1)
             const int row = m0 + sub * 32 + lane;
             float *drow = D + (int64_t)row * ldd;
 #pragma unroll 1
-            for (int c = 0; c < kGemmN; c += 32) {
+            for (int c = 0; c < BN; c += 32) {
                 uint32_t v[32];
                 tmem_ld_32x32b_x32(tmem + ((uint32_t)(sub * 32) << 16) + (uint32_t)c, v);
                 tmem_ld_wait(v);
+                if (bias) {
+#pragma unroll
+                    for (int j = 0; j < 32; ++j) {
+                        const int n = n0 + c + j;
+                        v[j] = __float_as_uint(alpha * __uint_as_float(v[j]) + (n < N ? __ldg(bias + n) : 0.f));
+                    }
+                } else {
+#pragma unroll
+                    for (int j = 0; j < 32; ++j) v[j] = __float_as_uint(alpha * __uint_as_float(v[j]));
+                }
                 if (row < M) {
                     const int nc = N - (n0 + c);
                     if (nc >= 32 && (ldd & 3) == 0) {
                         float4 *o = reinterpret_cast<float4 *>(drow + n0 + c);
 #pragma unroll
                         for (int j = 0; j < 8; ++j)
-                            o[j] = make_float4(alpha * __uint_as_float(v[4 * j]), alpha * __uint_as_float(v[4 * j + 1]),
-                                               alpha * __uint_as_float(v[4 * j + 2]),
-                                               alpha * __uint_as_float(v[4 * j + 3]));
+                            o[j] = make_float4(__uint_as_float(v[4 * j]), __uint_as_float(v[4 * j + 1]),
+                                               __uint_as_float(v[4 * j + 2]), __uint_as_float(v[4 * j + 3]));
                     } else {
 #pragma unroll
                         for (int j = 0; j < 32; ++j)
-                            if (j < nc) drow[n0 + c + j] = alpha * __uint_as_float(v[j]);
+                            if (j < nc) drow[n0 + c + j] = __uint_as_float(v[j]);
                     }
                 }
             }
@@ -162,20 +192,47 @@ __global__ void __launch_bounds__(kThreads, 1)
     }
 }
 
+template <int BN>
+size_t gemm_smem_bytes() {
+    return 1024 + (size_t)kStages * GemmGeom<BN>::kStageBytes + sizeof(GemmShared);
+}
+
+template <int BN>
+cudaError_t launch_bn(const CUtensorMap &ta, const CUtensorMap &tb, const CUtensorMap &ta2, const CUtensorMap &tb2,
+                      int M, int N, int K, int K2, float alpha, const float *bias, float *D, int64_t ldd, int *err,
+                      uint64_t timeout_ns, cudaStream_t s) {
+    const size_t smem = gemm_smem_bytes<BN>();
+    cudaError_t e = cudaFuncSetAttribute(k_gemm_bf16_f32<BN>, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
+    if (e != cudaSuccess) return e;
+    dim3 grid((unsigned)((M + 127) / 128), (unsigned)((N + BN - 1) / BN));
+    k_gemm_bf16_f32<BN><<<grid, kThreads, smem, s>>>(ta, tb, ta2, tb2, M, N, K, K2, alpha, bias, D, ldd, err,
+                                                     timeout_ns);
+    return cudaGetLastError();
+}
+
 }  // namespace
 
-size_t gemm_smem_bytes() { return 1024 + (size_t)kStages * kStageBytes + sizeof(GemmShared); }
+int gemm_tile_n(int M, int N, int sms) {
+    const int64_t tiles64 = (int64_t)((M + 127) / 128) * ((N + 63) / 64);
+    return tiles64 * 2 <= sms ? 32 : 64;
+}
 
-cudaError_t launch_gemm_bf16_f32(const CUtensorMap &ta, const CUtensorMap &tb, int M, int N, int K, float alpha,
-                                 float *D, int64_t ldd, int *err, uint64_t timeout_ns, cudaStream_t s) {
+cudaError_t launch_gemm2_bf16_f32(const CUtensorMap &ta, const CUtensorMap &tb, const CUtensorMap *ta2,
+                                  const CUtensorMap *tb2, int tile_n, int M, int N, int K, int K2, float alpha,
+                                  const float *bias, float *D, int64_t ldd, int *err, uint64_t timeout_ns,
+                                  cudaStream_t s) {
     if (M <= 0 || N <= 0) return cudaSuccess;
-    if (K <= 0 || (K & 7) != 0) return cudaErrorInvalidValue;
-    const size_t smem = gemm_smem_bytes();
-    cudaError_t e = cudaFuncSetAttribute(k_gemm_bf16_f32, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
-    if (e != cudaSuccess) return e;
-    dim3 grid((unsigned)((M + 127) / 128), (unsigned)((N + kGemmN - 1) / kGemmN));
-    k_gemm_bf16_f32<<<grid, kThreads, smem, s>>>(ta, tb, M, N, K, alpha, D, ldd, err, timeout_ns);
-    return cudaGetLastError();
+    if (K <= 0 || (K & 7) != 0 || K2 < 0 || (K2 & 7) != 0 || (K2 > 0 && (!ta2 || !tb2))) return cudaErrorInvalidValue;
+    const CUtensorMap &a2 = K2 > 0 ? *ta2 : ta, &b2 = K2 > 0 ? *tb2 : tb;
+    if (tile_n == 32) return launch_bn<32>(ta, tb, a2, b2, M, N, K, K2, alpha, bias, D, ldd, err, timeout_ns, s);
+    if (tile_n == 64) return launch_bn<64>(ta, tb, a2, b2, M, N, K, K2, alpha, bias, D, ldd, err, timeout_ns, s);
+    return cudaErrorInvalidValue;
+}
+
+cudaError_t launch_gemm_bf16_f32(const CUtensorMap &ta, const CUtensorMap &tb, int tile_n, int M, int N, int K,
+                                 float alpha, float *D, int64_t ldd, int *err, uint64_t timeout_ns, cudaStream_t s) {
+    return launch_gemm2_bf16_f32(ta, tb, nullptr, nullptr, tile_n, M, N, K, 0, alpha, nullptr, D, ldd, err, timeout_ns,
+                                 s);
 }
 
 }  // namespace skipk

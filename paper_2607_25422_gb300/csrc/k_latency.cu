@@ -280,21 +280,22 @@ __global__ void __launch_bounds__(kThreads, 1)
                 __syncwarp();
                 if (lane == 0) mbar_arrive(smem_addr(&sh->tempty[buf]));
                 const float cs = FP8 ? (valid ? __ldg(p.corpus_scale + i) : 0.0f) : 1.0f;
-                // All queries' scores of this lane's row, and one ballot per
-                // query against that query's filter (branch-free).
+                // All queries' scores of this lane's row.
                 float sc[kLatMaxR];
+#pragma unroll
+                for (int q = 0; q < kLatMaxR; ++q) {
+                    if constexpr (FP8)
+                        sc[q] = (sh->qscale[0][q] * __uint_as_float(d0[q]) + sh->qscale[1][q] * __uint_as_float(d1[q]) +
+                                 sh->qscale[2][q] * __uint_as_float(d2[q])) * cs;
+                    else
+                        sc[q] = __uint_as_float(d0[q]);
+                }
+                // One ballot per query against that query's filter (branch-free).
                 uint32_t m[kLatMaxR];
                 uint32_t anym = 0;
 #pragma unroll
                 for (int q = 0; q < kLatMaxR; ++q) {
-                    float sq;
-                    if constexpr (FP8)
-                        sq = (sh->qscale[0][q] * __uint_as_float(d0[q]) + sh->qscale[1][q] * __uint_as_float(d1[q]) +
-                              sh->qscale[2][q] * __uint_as_float(d2[q])) * cs;
-                    else
-                        sq = __uint_as_float(d0[q]);
-                    sc[q] = sq;
-                    m[q] = __ballot_sync(0xffffffffu, valid && q < R && sq > filt_w[q]);
+                    m[q] = __ballot_sync(0xffffffffu, valid && q < R && sc[q] > filt_w[q]);
                     anym |= m[q];
                 }
                 if (anym) {
@@ -325,11 +326,14 @@ __global__ void __launch_bounds__(kThreads, 1)
                     __syncwarp();
                 }
             }
-            // Chunk done: sort each set, then merge the eight warps' sets of
-            // every query into the chunk's list (the two hand-offs between
-            // the epilogue warps are bounded waits, like every other wait).
+            // Chunk done: merge the eight warps' sets of every query into the
+            // chunk's list -- for k <= 16 one warp-wide sort of the 8k keys
+            // per query, else sorted sets merged by a warp (the two hand-offs
+            // between the epilogue warps are bounded waits, like every other
+            // wait).
+            const bool small_k = kEpiWarps * k <= 128;
             if (lane < R) {
-                topk_sort(Lw + (size_t)lane * k, 1, top.n);
+                if (!small_k) topk_sort(Lw + (size_t)lane * k, 1, top.n);
                 for (int t = top.n; t < k; ++t) Lw[(size_t)lane * k + t] = 0ull;
             }
             const uint32_t par = (uint32_t)(chunk & 1);
@@ -337,8 +341,19 @@ __global__ void __launch_bounds__(kThreads, 1)
             if (!mbar_wait(smem_addr(&sh->sorted), par, p.timeout_ns)) ok = false;
             for (int q = ew; q < R && ok; q += kEpiWarps) {
                 uint64_t *out = p.lists + ((int64_t)v * R + q) * k;
-                warp_merge_topk<1>(slists + (size_t)q * k, (int64_t)R * k, kEpiWarps, k, k,
-                                   [&](int idx, uint64_t key) { out[idx] = key; });
+                if (small_k) {
+                    uint64_t keys4[4];
+#pragma unroll
+                    for (int u = 0; u < 4; ++u) {
+                        const int pos = lane + 32 * u, w = pos / k, tt = pos - w * k;
+                        keys4[u] = pos < kEpiWarps * k ? slists[((size_t)w * R + q) * k + tt] : 0ull;
+                    }
+                    warp_sort128_desc(keys4);
+                    if (lane < k) out[lane] = keys4[0];
+                } else {
+                    warp_merge_topk<1>(slists + (size_t)q * k, (int64_t)R * k, kEpiWarps, k, k,
+                                       [&](int idx, uint64_t key) { out[idx] = key; });
+                }
             }
             mbar_arrive(smem_addr(&sh->merged));
             if (!mbar_wait(smem_addr(&sh->merged), par, p.timeout_ns)) ok = false;

@@ -1,8 +1,8 @@
 // SKV passage gate (App. B.4 Def. B.4, Eq. skv_score; Alg. 1 "SKV: verify"
 // and the TopK after it) on the merged retrieval lists.
 //
-//  k_skv_qbias   per question: c_q = b1 + W1[:, qbar] qbar + W1[:, vbar] vbar
-//                (fp32 on the CUDA cores; a warp per unit and 8 questions).
+//  (k_gemm)      per question: c_q = b1 + W1[:, qbar] qbar + W1[:, vbar] vbar
+//                for all questions at once, on the tensor cores (k_gemm.cu).
 //  k_skv_mlp     per 128 passage slots x 128 hidden units: the passage part
 //                of layer 1 on the tensor cores.  The A operand is built in
 //                shared memory by four warps from the gathered corpus rows
@@ -31,7 +31,9 @@ constexpr int kSkvSlice = kSkvRows * 128;           // one [128 x 64] bf16 K-sli
 constexpr int kSkvStageA = 3 * kSkvSlice;           // e | e*qbar | |e - qbar|
 constexpr int kSkvStageB = 3 * kSkvSlice;           // the three W1 column blocks (128 units)
 constexpr int kSkvStages = 2;
-constexpr int kSkvThreads = 192;                    // TMA warp, MMA warp, 4 builder/epilogue warps
+constexpr int kSkvBuilders = 8;                     // two builder warps per TMEM lane quadrant
+constexpr int kSkvThreads = 64 + 32 * kSkvBuilders;  // TMA warp, MMA warp, builders (4 of them: epilogue)
+constexpr int kSkvAhead = 3;                         // chunks of corpus row in flight per builder thread
 constexpr uint32_t kSkvIdesc = idesc_bf16_f32(128, kSkvHidden);
 constexpr uint64_t kDrainTimeoutNs = 1000000000ull;  // 1 s for copies in flight
 
@@ -81,7 +83,7 @@ __global__ void __launch_bounds__(kSkvThreads, 1)
 
     if (threadIdx.x == 0) {
         for (int s = 0; s < kSkvStages; ++s) {
-            mbar_init(smem_addr(&sh->full[s]), kSkvRows + 1);
+            mbar_init(smem_addr(&sh->full[s]), 32 * kSkvBuilders + 1);
             mbar_init(smem_addr(&sh->empty[s]), 1);
         }
         mbar_init(smem_addr(&sh->tfull), 1);
@@ -152,6 +154,11 @@ __global__ void __launch_bounds__(kSkvThreads, 1)
         }
     } else {
         // ------------------------------------------------ builders, then epilogue
+        // Builder warps w and w + 4 share a TMEM lane quadrant: each thread
+        // owns one slot row and half of every 64-column chunk (16-byte words
+        // 4 h .. 4 h + 3), and keeps the next kSkvAhead chunks of its corpus
+        // row and qbar in flight in registers.
+        const int bw = warp - 2, half = bw >> 2;
         const int r = (warp & 3) * 32 + lane;  // TMEM lane = slot row in the tile
         const int64_t slot = m0 + r;
         int64_t id = -1;
@@ -160,35 +167,47 @@ __global__ void __launch_bounds__(kSkvThreads, 1)
             id = p.ids[slot];
             q = (int)(slot / p.K);
             if (id >= p.N) {
-                atomicOr(p.err, kErrConfig);
+                if (half == 0) atomicOr(p.err, kErrConfig);
                 id = -1;
             }
         }
-        const uint4 *erow = reinterpret_cast<const uint4 *>(p.rows + (id < 0 ? 0 : id) * (int64_t)p.d);
-        const uint4 *qrow = reinterpret_cast<const uint4 *>(p.qbar + (int64_t)q * p.d);
+        const uint4 *erow = reinterpret_cast<const uint4 *>(p.rows + (id < 0 ? 0 : id) * (int64_t)p.d) + 4 * half;
+        const uint4 *qrow = reinterpret_cast<const uint4 *>(p.qbar + (int64_t)q * p.d) + 4 * half;
         const uint4 zero = make_uint4(0, 0, 0, 0);
-        // Chunk c + 1's loads are issued before chunk c is written out.
-        uint4 en[8], qn[8];
+        uint4 eb[kSkvAhead][4], qb[kSkvAhead][4];
 #pragma unroll
-        for (int j = 0; j < 8; ++j) {
-            en[j] = id >= 0 ? __ldg(erow + j) : zero;
-            qn[j] = id >= 0 ? __ldg(qrow + j) : zero;
-        }
+        for (int a = 0; a < kSkvAhead; ++a)
+#pragma unroll
+            for (int j = 0; j < 4; ++j) {
+                const bool ld = id >= 0 && a < nc;
+                eb[a][j] = ld ? __ldg(erow + a * 8 + j) : zero;
+                qb[a][j] = ld ? __ldg(qrow + a * 8 + j) : zero;
+            }
         bool ok = true;
         for (int c = 0; c < nc; ++c) {
             const int s = c % kSkvStages;
             const uint32_t ph = (uint32_t)(c / kSkvStages) & 1u;
-            uint4 e[8], qv[8];
+            uint4 e[4], qv[4];
 #pragma unroll
-            for (int j = 0; j < 8; ++j) {
-                e[j] = en[j];
-                qv[j] = qn[j];
+            for (int j = 0; j < 4; ++j) {
+                e[j] = eb[0][j];
+                qv[j] = qb[0][j];
             }
-            if (c + 1 < nc && id >= 0) {
+            // rotate the prefetch ring and issue chunk c + kSkvAhead
 #pragma unroll
-                for (int j = 0; j < 8; ++j) {
-                    en[j] = __ldg(erow + (c + 1) * 8 + j);
-                    qn[j] = __ldg(qrow + (c + 1) * 8 + j);
+            for (int a = 0; a + 1 < kSkvAhead; ++a)
+#pragma unroll
+                for (int j = 0; j < 4; ++j) {
+                    eb[a][j] = eb[a + 1][j];
+                    qb[a][j] = qb[a + 1][j];
+                }
+            {
+                const int cn = c + kSkvAhead;
+                const bool ld = id >= 0 && cn < nc;
+#pragma unroll
+                for (int j = 0; j < 4; ++j) {
+                    eb[kSkvAhead - 1][j] = ld ? __ldg(erow + cn * 8 + j) : zero;
+                    qb[kSkvAhead - 1][j] = ld ? __ldg(qrow + cn * 8 + j) : zero;
                 }
             }
             if (!mbar_wait(smem_addr(&sh->empty[s]), ph ^ 1u, p.timeout_ns)) {
@@ -199,14 +218,15 @@ __global__ void __launch_bounds__(kSkvThreads, 1)
             const uint32_t base = smem_addr(sA + s * kSkvStageA) + r * 128;
             const int sw = r & 7;
 #pragma unroll
-            for (int j = 0; j < 8; ++j) {
+            for (int jj = 0; jj < 4; ++jj) {
+                const int j = 4 * half + jj;
                 uint4 eq, ad;
-                features2(e[j].x, qv[j].x, eq.x, ad.x);
-                features2(e[j].y, qv[j].y, eq.y, ad.y);
-                features2(e[j].z, qv[j].z, eq.z, ad.z);
-                features2(e[j].w, qv[j].w, eq.w, ad.w);
+                features2(e[jj].x, qv[jj].x, eq.x, ad.x);
+                features2(e[jj].y, qv[jj].y, eq.y, ad.y);
+                features2(e[jj].z, qv[jj].z, eq.z, ad.z);
+                features2(e[jj].w, qv[jj].w, eq.w, ad.w);
                 const uint32_t off = (uint32_t)((j ^ sw) << 4);
-                sts128(base + off, e[j]);
+                sts128(base + off, e[jj]);
                 sts128(base + kSkvSlice + off, eq);
                 sts128(base + 2 * kSkvSlice + off, ad);
             }
@@ -215,8 +235,8 @@ __global__ void __launch_bounds__(kSkvThreads, 1)
         }
         if (!ok) atomicOr(p.err, kErrTimeout);
         // Epilogue: h = acc + c_q, ReLU, dot with w2 over this CTA's units.
-        const bool done = mbar_wait(smem_addr(&sh->tfull), 0, p.timeout_ns);
-        if (!done) atomicOr(p.err, kErrTimeout);
+        const bool done = half == 0 ? mbar_wait(smem_addr(&sh->tfull), 0, p.timeout_ns) : false;
+        if (half == 0 && !done) atomicOr(p.err, kErrTimeout);
         tc_fence_after();
         if (done) {
             const uint32_t lane_addr = (uint32_t)((warp & 3) * 32) << 16;
@@ -244,77 +264,6 @@ __global__ void __launch_bounds__(kSkvThreads, 1)
     if (warp == 1) {
         __syncwarp();
         tmem_dealloc(tmem, kSkvHidden);
-    }
-}
-
-// c[q][i] = b1[i] + sum_t W1[i][t] qbar[q][t] + sum_t W1[i][d + t] vbar[q][t].
-// A block covers four hidden units (one per warp) and eight questions.  The
-// eight questions' [qbar | vbar] are first staged in shared memory by the
-// whole block (independent loads, all in flight at once); each warp reads its
-// unit's 2d weights once, coalesced, into registers (lane l holds 16-byte
-// words l, l + 32, ...) and reduces each of the eight dots across the warp.
-constexpr int kBiasWarps = 4, kBiasQs = 8;
-__global__ void __launch_bounds__(32 * kBiasWarps) k_skv_qbias(const SkvParams p) {
-    __shared__ uint4 xs[kBiasQs][256];  // [question][16-byte word of qbar | vbar], d <= 1024
-    const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
-    const int i = blockIdx.x * kBiasWarps + warp;
-    const int q0 = blockIdx.y * kBiasQs;
-    const int nq = p.d / 8;  // 16-byte words per d-vector
-    const int nv = 2 * nq;   // words of [qbar | vbar]
-    // All of a thread's staging loads are issued before any is stored.
-    constexpr int kPer = kBiasQs * 256 / (32 * kBiasWarps);
-    uint4 xr[kPer];
-#pragma unroll
-    for (int r = 0; r < kPer; ++r) {
-        const int idx = threadIdx.x + r * 32 * kBiasWarps;
-        const int u = idx / nv, k = idx - u * nv, q = q0 + u;
-        xr[r] = make_uint4(0, 0, 0, 0);
-        if (idx < kBiasQs * nv && q < p.Q)
-            xr[r] = k < nq ? __ldg(reinterpret_cast<const uint4 *>(p.qbar + (int64_t)q * p.d) + k)
-                           : __ldg(reinterpret_cast<const uint4 *>(p.vbar + (int64_t)q * p.d) + (k - nq));
-    }
-#pragma unroll
-    for (int r = 0; r < kPer; ++r) {
-        const int idx = threadIdx.x + r * 32 * kBiasWarps;
-        if (idx < kBiasQs * nv) xs[idx / nv][idx % nv] = xr[r];
-    }
-    uint4 w[8];
-    const uint4 *wrow = reinterpret_cast<const uint4 *>(p.w1 + (int64_t)min(i, p.H - 1) * 5 * p.d);
-#pragma unroll
-    for (int t = 0; t < 8; ++t) w[t] = (lane + 32 * t < nv) ? __ldg(wrow + lane + 32 * t) : make_uint4(0, 0, 0, 0);
-    __syncthreads();
-    if (i >= p.H) return;
-    float acc[kBiasQs];
-#pragma unroll
-    for (int u = 0; u < kBiasQs; ++u) {
-        acc[u] = 0.f;
-#pragma unroll
-        for (int t = 0; t < 8; ++t) {
-            const int k = lane + 32 * t;
-            if (k < nv) {
-                const uint4 x = xs[u][k];
-                const uint32_t wv[4] = {w[t].x, w[t].y, w[t].z, w[t].w};
-                const uint32_t xw[4] = {x.x, x.y, x.z, x.w};
-#pragma unroll
-                for (int h = 0; h < 4; ++h) {
-                    const float2 wf = __bfloat1622float2(*reinterpret_cast<const __nv_bfloat162 *>(&wv[h]));
-                    const float2 xf = __bfloat1622float2(*reinterpret_cast<const __nv_bfloat162 *>(&xw[h]));
-                    acc[u] = fmaf(wf.x, xf.x, acc[u]);
-                    acc[u] = fmaf(wf.y, xf.y, acc[u]);
-                }
-            }
-        }
-    }
-#pragma unroll
-    for (int u = 0; u < kBiasQs; ++u)
-#pragma unroll
-        for (int o = 16; o; o >>= 1) acc[u] += __shfl_xor_sync(0xFFFFFFFFu, acc[u], o);
-    if (lane < kBiasQs && q0 + lane < p.Q) {
-        float v = acc[0];
-#pragma unroll
-        for (int u = 1; u < kBiasQs; ++u)
-            if (lane == u) v = acc[u];
-        p.cq[(int64_t)(q0 + lane) * p.H + i] = v + p.b1[i];
     }
 }
 
@@ -394,13 +343,6 @@ __global__ void __launch_bounds__(kSelThreads) k_skv_select(const SkvParams p) {
 
 size_t skv_mlp_smem_bytes() {
     return 1024 + (size_t)kSkvStages * (kSkvStageA + kSkvStageB) + sizeof(SkvShared);
-}
-
-cudaError_t launch_skv_qbias(const SkvParams &p, cudaStream_t s) {
-    if (p.Q == 0) return cudaSuccess;
-    dim3 grid((unsigned)((p.H + kBiasWarps - 1) / kBiasWarps), (unsigned)((p.Q + kBiasQs - 1) / kBiasQs));
-    k_skv_qbias<<<grid, 32 * kBiasWarps, 0, s>>>(p);
-    return cudaGetLastError();
 }
 
 cudaError_t launch_skv_mlp(const CUtensorMap &tw, const SkvParams &p, cudaStream_t s) {

@@ -27,11 +27,12 @@
 //    its commits are multicast to both CTAs, and both CTAs' epilogues hand
 //    the accumulator back to it.
 //
-// Work: persistent clusters walk items (query group, corpus chunk)
-// cid, cid + #clusters, ...; items are numbered chunk-major so that the
-// clusters of the other query groups read the same chunk at the same time
-// and find it in L2.  Each item leaves one sorted list per region row; the
-// merge kernel combines the chunks.
+// Work: persistent clusters take items (query group, corpus chunk) from a
+// counter shared by the grid, one at a time; items are numbered
+// chunk-major, so the clusters at work hold the query groups of one or two
+// chunks and each corpus tile, read once from HBM, serves the others from
+// L2.  Each item leaves one sorted list per region row; the merge kernel
+// combines the chunks.
 //
 // The k-th best score of any chunk of a row bounds the row's global top-k
 // from below, so the chunks of a row share one threshold: each CTA publishes
@@ -43,7 +44,7 @@
 // Per-row top-k sets live in shared memory ([slot][row], k slots) when they
 // fit next to a pipeline of at least two stages, else in global memory; a
 // set is unsorted with its smallest key tracked, and sorted at chunk end
-// (in registers when it holds at most 16 keys); a list shorter than k ends
+// (in registers when it holds at most 32 keys); a list shorter than k ends
 // with an empty key, which is as far as the merge reads.
 //
 // Resident query block (CTA pair, d <= 512, sets in global memory): each CTA
@@ -75,6 +76,7 @@ constexpr int kBFull = kTcTileN * kTcTileK * 2;   // 32 KB: 256 corpus rows x 64
 constexpr uint32_t kTmemCols = 512;               // two 256-column accumulators
 constexpr uint64_t kDrainTimeoutNs = 1000000000ull;  // 1 s for copies/MMAs in flight
 constexpr int kMaxStages = 8;
+constexpr int kSchedQ = 4;  // work items published ahead of the slowest role
 
 template <bool PAIR>
 struct Geom {
@@ -92,6 +94,9 @@ struct __align__(8) TcShared {
     uint64_t tempty[2];          // accumulator drained (epilogue warps)
     uint64_t drain;              // MMA completion at exit
     uint64_t afull, aempty;      // resident query block loaded / released
+    uint64_t sfull[kSchedQ];     // work item published (the pair's MMA CTA publishes to both CTAs)
+    uint64_t sempty[kSchedQ];    // ... taken by every role of the pair
+    int sched[kSchedQ];          // item index, -1 = no more work
     uint32_t tmem_base;
 };
 
@@ -115,9 +120,39 @@ __global__ void __launch_bounds__(kTcThreads, 1)
     const int items = p.QG * p.G;
     // A pair is a cluster of two CTAs; a single-CTA launch has no clusters.
     const int rank = PAIR ? (int)cluster_rank() : 0;
-    const int cid = PAIR ? (int)cluster_index() : (int)blockIdx.x;
-    const int ncl = PAIR ? (int)cluster_count() : (int)gridDim.x;
     const bool mma_cta = !PAIR || rank == 0;
+
+    // Work items are handed out dynamically: the MMA CTA's producer takes the
+    // next index from a counter shared by the grid and publishes it to every
+    // role of the pair through a small ring in shared memory, so that the
+    // CTAs at work always hold nearly consecutive items (the query groups of
+    // one corpus chunk, which then find its tiles in L2).
+    auto sched_take = [&](uint32_t n, int &v) -> bool {
+        const int j = (int)(n % kSchedQ);
+        if (!mbar_wait_cluster(smem_addr(&sh->sfull[j]), (n / kSchedQ) & 1u, p.timeout_ns)) return false;
+        v = *reinterpret_cast<volatile int *>(&sh->sched[j]);
+        return true;
+    };
+    auto sched_release = [&](uint32_t n) {
+        const uint32_t e = smem_addr(&sh->sempty[n % kSchedQ]);
+        if (PAIR && rank != 0)
+            mbar_arrive_cluster(mapa_shared(e, 0));
+        else
+            mbar_arrive(e);
+    };
+    auto sched_publish = [&](uint32_t n, int &v) -> bool {
+        const int j = (int)(n % kSchedQ);
+        if (!mbar_wait_cluster(smem_addr(&sh->sempty[j]), ((n / kSchedQ) & 1u) ^ 1u, p.timeout_ns)) return false;
+        const int x = atomicAdd(p.sched, 1);
+        v = x < items ? x : -1;
+        sh->sched[j] = v;
+        mbar_arrive(smem_addr(&sh->sfull[j]));
+        if constexpr (PAIR) {
+            st_shared_cluster_u32(mapa_shared(smem_addr(&sh->sched[j]), 1), (uint32_t)v);
+            mbar_arrive_cluster(mapa_shared(smem_addr(&sh->sfull[j]), 1));
+        }
+        return true;
+    };
 
     if (threadIdx.x == 0) {
         for (int s = 0; s < S; ++s) {
@@ -131,6 +166,12 @@ __global__ void __launch_bounds__(kTcThreads, 1)
         mbar_init(smem_addr(&sh->drain), 1);
         mbar_init(smem_addr(&sh->afull), 1);
         mbar_init(smem_addr(&sh->aempty), 1);
+        for (int j = 0; j < kSchedQ; ++j) {
+            mbar_init(smem_addr(&sh->sfull[j]), 1);
+            // takers: the MMA thread and the epilogue warps (and, in a pair,
+            // the other CTA's epilogue warps and producer)
+            mbar_init(smem_addr(&sh->sempty[j]), PAIR ? 10 : 5);
+        }
         mbar_fence_init();
     }
     if (warp == 0 && lane == 0) {
@@ -161,7 +202,21 @@ __global__ void __launch_bounds__(kTcThreads, 1)
             int64_t issued = 0;
             bool ok = true;
             uint32_t na = 0;  // query blocks loaded (resident mode)
-            for (int v = cid; v < items && ok; v += ncl) {
+            for (uint32_t n = 0; ok; ++n) {
+                int v = -1;
+                if (mma_cta) {
+                    if (!sched_publish(n, v)) {
+                        ok = false;
+                        break;
+                    }
+                } else {
+                    if (!sched_take(n, v)) {
+                        ok = false;
+                        break;
+                    }
+                    sched_release(n);
+                }
+                if (v < 0) break;
                 const Item it = item_of(p, v, rank);
                 if (ar) {
                     // The previous item's MMAs have released the block: load
@@ -231,7 +286,14 @@ __global__ void __launch_bounds__(kTcThreads, 1)
             uint32_t lt = 0;
             bool ok = true;
             uint32_t na = 0;  // query blocks used (resident mode)
-            for (int v = cid; v < items && ok; v += ncl) {
+            for (uint32_t n = 0; ok; ++n) {
+                int v = -1;
+                if (!sched_take(n, v)) {
+                    ok = false;
+                    break;
+                }
+                sched_release(n);
+                if (v < 0) break;
                 const Item it = item_of(p, v, rank);
                 if (ar) {
                     if (!mbar_wait(smem_addr(&sh->afull), na & 1u, p.timeout_ns)) {
@@ -309,7 +371,16 @@ __global__ void __launch_bounds__(kTcThreads, 1)
         const float kNegInf = -__int_as_float(0x7f800000);
         uint32_t lt = 0;
         bool ok = true;
-        for (int v = cid; v < items && ok; v += ncl) {
+        for (uint32_t n = 0; ok; ++n) {
+            int v = -1;
+            const bool got_item = sched_take(n, v);
+            if (!__all_sync(0xffffffffu, got_item)) {
+                ok = false;
+                break;
+            }
+            __syncwarp();
+            if (lane == 0) sched_release(n);
+            if (v < 0) break;
             const Item it = item_of(p, v, rank);
             const int row = it.mb * kTcTileM + rib;
             const bool row_valid = it.mb < p.MB && row < p.R;
@@ -441,7 +512,9 @@ __global__ void __launch_bounds__(kTcThreads, 1)
                     glist[t] = d4[t] > kNegInf ? make_key(d4[t], (uint32_t)(it.g * 4 + t)) : 0ull;
             } else if (row_valid) {
                 if (!p.list_in_smem && top.n <= 16) {
-                    sort16_desc_in_place(glist, top.n);
+                    sortw_desc_in_place<16>(glist, top.n);
+                } else if (!p.list_in_smem && top.n <= 32) {
+                    sortw_desc_in_place<32>(glist, top.n);
                 } else {
                     topk_sort(L, ls, top.n);
                     if (p.list_in_smem)

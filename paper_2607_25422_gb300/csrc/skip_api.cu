@@ -63,6 +63,21 @@ bool encode_bf16_rows(CUtensorMap *map, const void *base, int64_t rows, int d, i
               CU_TENSOR_MAP_L2_PROMOTION_L2_256B, CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) == CUDA_SUCCESS;
 }
 
+// 2D bf16 tensor map over `cols` columns of a row-major matrix whose rows
+// are `ld` elements apart (a column block of a wider matrix), box
+// box_rows x 64 elements, 128-byte swizzle.
+bool encode_bf16_block(CUtensorMap *map, const void *base, int64_t rows, int cols, int64_t ld, int box_rows) {
+    EncodeTiledFn fn = encode_fn();
+    if (!fn) return false;
+    cuuint64_t dims[2] = {(cuuint64_t)cols, (cuuint64_t)rows};
+    cuuint64_t strides[1] = {(cuuint64_t)ld * 2};
+    cuuint32_t box[2] = {(cuuint32_t)kTcTileK, (cuuint32_t)box_rows};
+    cuuint32_t estr[2] = {1, 1};
+    return fn(map, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 2, const_cast<void *>(base), dims, strides, box, estr,
+              CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B, CU_TENSOR_MAP_L2_PROMOTION_L2_256B,
+              CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) == CUDA_SUCCESS;
+}
+
 // 2D byte tensor map over the e4m3 corpus [rows x d], box 256 rows x 128
 // elements (128 bytes), 128-byte swizzle, zero fill out of bounds.
 bool encode_e4m3_rows(CUtensorMap *map, const void *base, int64_t rows, int d, int box_rows = kTcTileN) {
@@ -103,6 +118,7 @@ struct skip_corpus {
     int mma = 0;               // 0 = pick, 1 = single-CTA MMA, 2 = CTA-pair MMA
     int bound = 0;             // bounding pass: 0 = by corpus size, 1 = never, 2 = always
     bool canary = false;       // guard bytes after the growable buffers (SKIP_OPT_CANARY)
+    int resident = 0;          // resident query blocks: 0 by the rule, 1 never, 2 whenever possible
     std::map<int, int> cluster_cache;  // resident clusters per (size, stages, list place)
     int timing = 0;
     // Timing: events recorded on the launching stream before each kernel and
@@ -388,6 +404,7 @@ skip_status_t run_regions(skip_corpus *c, const uint16_t *regions, int R, int k,
         p.raw_stages = raw_stages;
         p.list_in_smem = in_smem;
         p.a_res = 0;
+        p.sched = nullptr;
         p.scale = c->scale;
         pl.stages = stages;
         pl.list_in_smem = in_smem;
@@ -430,10 +447,8 @@ skip_status_t run_regions(skip_corpus *c, const uint16_t *regions, int R, int k,
         // read a chunk at the same time then all find it in L2 (a long chunk
         // lets them drift apart, and each re-reads it from HBM).
         pl.G = pick_chunks(QG, pl.tiles, ncl, (int)((pl.tiles + kTcChunkTiles - 1) / kTcChunkTiles));
-        const int items = QG * pl.G;
-        pl.grid = std::min(items, ncl) * cl_best;
-        const size_t lists_bytes = (size_t)pl.G * pl.R_pad * k * sizeof(uint64_t);
-        const size_t tau_bytes = align_up((size_t)pl.R_pad * sizeof(uint32_t), 256);
+        // the per-row thresholds, then the two launches' work-item counters
+        const size_t tau_bytes = align_up((size_t)pl.R_pad * sizeof(uint32_t), 256) + 256;
         // Bounding pass: the same kernel over every kBoundStride-th corpus
         // tile first; the merged sample top-k of each row is k ids whose
         // scores (computed bit for bit as the full pass computes them) are at
@@ -463,13 +478,35 @@ skip_status_t run_regions(skip_corpus *c, const uint16_t *regions, int R, int k,
         const int k_s = bound ? std::min(k, std::max(4, (2 * k + chunks_s - 1) / chunks_s)) : 0;
         // Query blocks resident in shared memory (pairs, d <= 512): the sets
         // go to global memory, where the bounding pass keeps them short.
-        int res_stages = (pair && bound) ? tc_pick_resident_stages(c->d, c->max_smem) : 0;
+        int res_stages = (pair && bound && c->resident != 1) ? tc_pick_resident_stages(c->d, c->max_smem) : 0;
         const int res_slices = res_stages > 0 ? (c->d + kTcTileK - 1) / kTcTileK : 0;
         if (res_stages > 0 && max_clusters(cl_best, res_stages, false, res_slices) < ncl) res_stages = 0;
         if (res_stages > 0) {
-            stages = res_stages;
-            in_smem = false;
+            // The sets then live in global memory, where a full set costs a
+            // rescan from L2 and a long one a slow sort; keep the keys an
+            // item admits few: the sample's k-th score is about the
+            // (kBoundStride k)-th best of the corpus, so an item of T tiles
+            // holds about kBoundStride k T / tiles keys above it.  Items of
+            // at most 16 such keys, and of at least 64 tiles (else the
+            // per-item cost of loading the query block shows).
+            const int64_t t_keys = (int64_t)(16.0 * (double)pl.tiles / ((double)kBoundStride * k));
+            int64_t gmin = (pl.tiles + std::max<int64_t>(1, std::min<int64_t>(kTcChunkTiles, t_keys)) - 1) /
+                           std::max<int64_t>(1, std::min<int64_t>(kTcChunkTiles, t_keys));
+            gmin = std::min<int64_t>(gmin, 512);
+            if (c->resident == 2) {  // forced: items as for shared-memory sets
+                stages = res_stages;
+                in_smem = false;
+            } else if ((pl.tiles + gmin - 1) / gmin < 64 || t_keys < 1) {
+                res_stages = 0;
+            } else {
+                pl.G = pick_chunks(QG, pl.tiles, ncl, (int)gmin);
+                stages = res_stages;
+                in_smem = false;
+            }
         }
+        const int items = QG * pl.G;
+        pl.grid = std::min(items, ncl) * cl_best;
+        const size_t lists_bytes = (size_t)pl.G * pl.R_pad * k * sizeof(uint64_t);
         const size_t lists_s_bytes = align_up((size_t)chunks_s * pl.R_pad * k_s * sizeof(uint64_t), 256);
         skip_status_t st = ensure_ws(c, align_up(ws_extra, 256) + tau_bytes + align_up(lists_bytes, 256) +
                                             lists_s_bytes);
@@ -507,6 +544,8 @@ skip_status_t run_regions(skip_corpus *c, const uint16_t *regions, int R, int k,
         p.raw_stages = 0;
         p.tile_stride = 1;
         p.a_res = res_stages > 0 ? 1 : 0;
+        int *counters = reinterpret_cast<int *>((char *)tau + tau_bytes - 256);
+        p.sched = counters;
         pl.stages = p.stages;
         pl.list_in_smem = in_smem;
         pl.pair = pair;
@@ -515,6 +554,7 @@ skip_status_t run_regions(skip_corpus *c, const uint16_t *regions, int R, int k,
         cudaError_t e;
         if (bound) {
             TcParams ps = p;
+            ps.sched = counters + 1;
             ps.tiles = stiles;
             ps.tile_stride = kBoundStride;
             ps.G = chunks_s;
@@ -646,6 +686,8 @@ skip_status_t check_skv(skip_corpus *c, int32_t Q, int32_t K, const uint16_t *qb
     if (mlp->hidden < kSkvHidden || mlp->hidden % kSkvHidden != 0 || !mlp->w1 || !mlp->b1 || !mlp->w2)
         return SKIP_EINVAL;
     if (Q > 0 && (!qbar || !vbar || !out_ids || !out_nu || !out_count)) return SKIP_EINVAL;
+    // qbar, vbar and W1 are read by TMA and as 16-byte vectors
+    if ((((uintptr_t)qbar | (uintptr_t)vbar | (uintptr_t)mlp->w1) & 15) != 0) return SKIP_EINVAL;
     if (c->dtype != SKIP_BF16 || c->d % 64 != 0 || c->d > 1024) return SKIP_EUNSUPPORTED;
     return SKIP_OK;
 }
@@ -688,8 +730,17 @@ skip_status_t skv_impl(skip_corpus *c, const int64_t *cand_ids, int32_t Q, int32
     p.nu_all = nu_all;
     p.err = c->err;
     p.timeout_ns = c->timeout_ns;
+    // c_q = b1 + W1[:, 0:d] qbar + W1[:, d:2d] vbar for every question: one
+    // GEMM over the two column blocks of W1.
+    CUtensorMap ta, tb, ta2, tb2;
+    const int tn = gemm_tile_n(Q, H, c->sm_count);
+    if (!encode_bf16_rows(&ta, qbar, Q, c->d, 128) || !encode_bf16_rows(&ta2, vbar, Q, c->d, 128) ||
+        !encode_bf16_block(&tb, mlp->w1, H, c->d, 5 * (int64_t)c->d, tn) ||
+        !encode_bf16_block(&tb2, mlp->w1 + c->d, H, c->d, 5 * (int64_t)c->d, tn))
+        return SKIP_ECUDA;
     record(c, s, "skv_qbias");
-    cudaError_t e = launch_skv_qbias(p, s);
+    cudaError_t e = launch_gemm2_bf16_f32(ta, tb, &ta2, &tb2, tn, Q, H, c->d, c->d, 1.f, mlp->b1, p.cq, H, c->err,
+                                          c->timeout_ns, s);
     if (e != cudaSuccess) return cuda_status(e);
     record(c, s, "skv_mlp");
     e = launch_skv_mlp(tw, p, s);
@@ -814,6 +865,10 @@ skip_status_t skip_corpus_set_option(skip_corpus_t c, int option, int64_t value)
         case SKIP_OPT_BOUND:
             if (value < 0 || value > 2) return SKIP_EINVAL;
             c->bound = (int)value;
+            return SKIP_OK;
+        case SKIP_OPT_RESIDENT:
+            if (value < 0 || value > 2) return SKIP_EINVAL;
+            c->resident = (int)value;
             return SKIP_OK;
         case SKIP_OPT_CANARY:
             if (value != 0 && value != 1) return SKIP_EINVAL;
@@ -1171,11 +1226,12 @@ skip_status_t ivf_regions(skip_ivfpq *ix, const void *regions, int R, int nprobe
         // tensor cores, then the nprobe best per region
         float *scores = reinterpret_cast<float *>((char *)ix->ws + (G + 1) * kb + pid + psc);
         CUtensorMap ta, tb;
+        const int tn = gemm_tile_n(R, ix->C, ix->cent->sm_count);
         if (!encode_bf16_rows(&ta, regions, R, ix->d, 128) ||
-            !encode_bf16_rows(&tb, ix->cent->rows, ix->C, ix->d, kGemmN))
+            !encode_bf16_rows(&tb, ix->cent->rows, ix->C, ix->d, tn))
             return SKIP_ECUDA;
         record(ix->cent, s, "ivf_probe");
-        st = cuda_status(launch_gemm_bf16_f32(ta, tb, R, ix->C, ix->d, 1.f, scores, ix->C, ix->cent->err,
+        st = cuda_status(launch_gemm_bf16_f32(ta, tb, tn, R, ix->C, ix->d, 1.f, scores, ix->C, ix->cent->err,
                                               ix->cent->timeout_ns, s));
         if (st) return st;
         st = cuda_status(launch_ivf_probe_select(scores, R, ix->C, nprobe, probe_ids, probe_sc, s));
@@ -1491,9 +1547,10 @@ skip_status_t skip_qvs_prune(skip_qvs_t q, const uint16_t *tokens, int32_t B, in
         fa = q->fqp;
     }
     CUtensorMap ta, tb;
-    if (!encode_bf16_rows(&ta, fa, B, q->dkp, 128) || !encode_bf16_rows(&tb, q->wvt, q->d, q->dkp, kGemmN))
+    const int tn = gemm_tile_n(B, q->d, q->sms);
+    if (!encode_bf16_rows(&ta, fa, B, q->dkp, 128) || !encode_bf16_rows(&tb, q->wvt, q->d, q->dkp, tn))
         return SKIP_ECUDA;
-    cudaError_t e = launch_gemm_bf16_f32(ta, tb, B, q->d, q->dkp, 1.f / std::sqrt((float)q->dk), q->u, q->d,
+    cudaError_t e = launch_gemm_bf16_f32(ta, tb, tn, B, q->d, q->dkp, 1.f / std::sqrt((float)q->dk), q->u, q->d,
                                          q->err, q->timeout_ns, s);
     if (e == cudaSuccess) e = launch_qvs_logits(p, q->sms, s);
     if (e == cudaSuccess) e = launch_qvs_select(p, s);

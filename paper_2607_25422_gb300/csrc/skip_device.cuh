@@ -88,6 +88,57 @@ __device__ __forceinline__ uint64_t warp_max_u64(uint64_t v) {
     return v;
 }
 
+// Bitonic sort, descending, of one key per lane across the warp (lane 0
+// ends with the largest).
+__device__ __forceinline__ uint64_t warp_sort32_desc(uint64_t v) {
+    const int lane = threadIdx.x & 31;
+#pragma unroll
+    for (int size = 2; size <= 32; size <<= 1)
+#pragma unroll
+        for (int j = size >> 1; j > 0; j >>= 1) {
+            const uint64_t o = __shfl_xor_sync(0xffffffffu, v, j);
+            const bool desc = (lane & size) == 0 || size == 32;
+            const bool lower = (lane & j) == 0;
+            v = (lower == desc) ? (v > o ? v : o) : (v < o ? v : o);
+        }
+    return v;
+}
+
+// The same over 128 keys, four per lane (position lane + 32 i holds v[i]);
+// position 0 ends with the largest.
+__device__ __forceinline__ void warp_sort128_desc(uint64_t (&v)[4]) {
+    const int lane = threadIdx.x & 31;
+#pragma unroll
+    for (int size = 2; size <= 128; size <<= 1)
+#pragma unroll
+        for (int j = size >> 1; j > 0; j >>= 1) {
+            if (j >= 32) {
+                const int ji = j >> 5;
+#pragma unroll
+                for (int i = 0; i < 4; ++i) {
+                    const int ip = i ^ ji;
+                    if (ip > i) {
+                        const int pos = lane + 32 * i;
+                        const bool desc = (pos & size) == 0 || size == 128;
+                        const uint64_t a = v[i], b = v[ip];
+                        const bool sw = desc ? a < b : a > b;
+                        v[i] = sw ? b : a;
+                        v[ip] = sw ? a : b;
+                    }
+                }
+            } else {
+#pragma unroll
+                for (int i = 0; i < 4; ++i) {
+                    const int pos = lane + 32 * i;
+                    const uint64_t o = __shfl_xor_sync(0xffffffffu, v[i], j);
+                    const bool desc = (pos & size) == 0 || size == 128;
+                    const bool lower = (lane & j) == 0;
+                    v[i] = (lower == desc) ? (v[i] > o ? v[i] : o) : (v[i] < o ? v[i] : o);
+                }
+            }
+        }
+}
+
 // ---------------------------------------------------------------- timing
 
 __device__ __forceinline__ uint64_t globaltimer_ns() {
@@ -140,6 +191,36 @@ __device__ __forceinline__ bool mbar_wait(uint32_t bar, uint32_t parity, uint64_
         if (mbar_try_wait(bar, parity)) return true;
         if (globaltimer_ns() - t0 > timeout_ns) return false;
     }
+}
+
+// As mbar_wait, with cluster-scope acquire: for a phase completed by
+// arrivals (with release at cluster scope) from another CTA of the cluster,
+// whose earlier writes to this CTA's shared memory must be visible.
+__device__ __forceinline__ bool mbar_try_wait_cluster(uint32_t bar, uint32_t parity) {
+    uint32_t ok;
+    asm volatile(
+        "{\n\t.reg .pred p;\n\t"
+        "mbarrier.try_wait.parity.acquire.cluster.shared::cta.b64 p, [%1], %2;\n\t"
+        "selp.u32 %0, 1, 0, p;\n\t}"
+        : "=r"(ok)
+        : "r"(bar), "r"(parity)
+        : "memory");
+    return ok != 0;
+}
+
+__device__ __forceinline__ bool mbar_wait_cluster(uint32_t bar, uint32_t parity, uint64_t timeout_ns) {
+    if (mbar_try_wait_cluster(bar, parity)) return true;
+    uint64_t t0 = globaltimer_ns();
+    for (;;) {
+        if (mbar_try_wait_cluster(bar, parity)) return true;
+        if (globaltimer_ns() - t0 > timeout_ns) return false;
+    }
+}
+
+// 32-bit store to the shared memory of a CTA of the cluster (address from
+// mapa_shared).
+__device__ __forceinline__ void st_shared_cluster_u32(uint32_t cluster_addr, uint32_t v) {
+    asm volatile("st.shared::cluster.u32 [%0], %1;" ::"r"(cluster_addr), "r"(v) : "memory");
 }
 
 // ---------------------------------------------------------------- PDL

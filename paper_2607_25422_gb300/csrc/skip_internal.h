@@ -54,6 +54,7 @@ struct TcParams {
     int list_in_smem; // per-row lists in shared memory (else global)
     const float *scale;  // [N] row scales (e4m3 corpus only)
     int raw_stages;      // e4m3 corpus: depth of the raw-slice ring
+    int *sched;          // bf16 kernel: work-item counter, zero at launch
     int a_res;           // bf16 pair kernel: the query block stays resident in shared memory for
                          // the whole item and the ring carries corpus slices only (sets in global
                          // memory; d <= 64 * kMaxResidentSlices)
@@ -115,11 +116,18 @@ cudaError_t launch_latency(bool fp8, const CUtensorMap &ta, const CUtensorMap &t
 // ---- small dense GEMM with fp32 results (k_gemm.cu) ------------------------
 // D [M x N] (leading dimension ldd) = alpha * A [M x K] B [N x K]^T, bf16
 // operands row-major with K contiguous (K % 8 == 0).  ta: tensor map over A,
-// box 128 rows x 64 elements; tb: over B, box kGemmN rows x 64 elements; both
+// box 128 rows x 64 elements; tb: over B, box tile_n rows x 64 elements; both
 // 128-byte swizzle.  err (nullable) receives kErrTimeout if a wait gives up.
-constexpr int kGemmN = 64;
-cudaError_t launch_gemm_bf16_f32(const CUtensorMap &ta, const CUtensorMap &tb, int M, int N, int K, float alpha,
-                                 float *D, int64_t ldd, int *err, uint64_t timeout_ns, cudaStream_t s);
+// gemm_tile_n: the tile width (32 or 64) to use for an M x N product.
+int gemm_tile_n(int M, int N, int sms);
+cudaError_t launch_gemm_bf16_f32(const CUtensorMap &ta, const CUtensorMap &tb, int tile_n, int M, int N, int K,
+                                 float alpha, float *D, int64_t ldd, int *err, uint64_t timeout_ns, cudaStream_t s);
+// D = alpha * (A B^T + A2 B2^T) + bias (per column n; nullable); ta2 / tb2
+// over A2 [M x K2] / B2 [N x K2] with the same boxes (K2 = 0: one product).
+cudaError_t launch_gemm2_bf16_f32(const CUtensorMap &ta, const CUtensorMap &tb, const CUtensorMap *ta2,
+                                  const CUtensorMap *tb2, int tile_n, int M, int N, int K, int K2, float alpha,
+                                  const float *bias, float *D, int64_t ldd, int *err, uint64_t timeout_ns,
+                                  cudaStream_t s);
 
 // ---- merges -------------------------------------------------------------
 // Per-region merge of G sorted lists into the exact top-k (keys and/or
@@ -171,10 +179,10 @@ struct SkvParams {
     uint64_t timeout_ns;
 };
 size_t skv_mlp_smem_bytes();
-// The gate in three launches: per-question bias, the tensor-core layer 1 +
-// ReLU + w2 partial dots, and the sigmoid / gate / selection.
+// The gate in three launches: per-question bias (the library GEMM), the
+// tensor-core layer 1 + ReLU + w2 partial dots, and the sigmoid / gate /
+// selection.
 // tw: tensor map over W1 [H x 5d] bf16, box 64 columns x 128 rows, 128-byte swizzle.
-cudaError_t launch_skv_qbias(const SkvParams &p, cudaStream_t s);
 cudaError_t launch_skv_mlp(const CUtensorMap &tw, const SkvParams &p, cudaStream_t s);
 cudaError_t launch_skv_select(const SkvParams &p, cudaStream_t s);
 

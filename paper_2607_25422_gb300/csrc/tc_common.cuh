@@ -61,14 +61,54 @@ __device__ __forceinline__ void topk_rescan(uint64_t *L, int ls, int k, RowTopK 
     st.min_slot = s0;
 }
 
+// The same over a contiguous set in global memory (slot t at L[t], k even,
+// L 16-byte aligned): 16 keys per batch as eight 16-byte loads, two batches
+// in flight, so a rescan costs a few round trips to L2 instead of one per
+// eight keys.
+__device__ __forceinline__ void topk_rescan_contig(const uint64_t *L, int k, RowTopK &st) {
+    uint64_t m0 = ~0ull, m1 = ~0ull;
+    int s0 = 0, s1 = 0;
+    const ulonglong2 *V = reinterpret_cast<const ulonglong2 *>(L);
+    const int pairs = k >> 1;
+    int t = 0;
+#pragma unroll 2
+    for (; t + 8 <= pairs; t += 8) {
+        ulonglong2 x[8];
+#pragma unroll
+        for (int u = 0; u < 8; ++u) x[u] = V[t + u];
+#pragma unroll
+        for (int u = 0; u < 8; ++u) {
+            if (x[u].x < m0) { m0 = x[u].x; s0 = 2 * (t + u); }
+            if (x[u].y < m1) { m1 = x[u].y; s1 = 2 * (t + u) + 1; }
+        }
+    }
+    for (; t < pairs; ++t) {
+        const ulonglong2 x = V[t];
+        if (x.x < m0) { m0 = x.x; s0 = 2 * t; }
+        if (x.y < m1) { m1 = x.y; s1 = 2 * t + 1; }
+    }
+    if (m1 < m0) { m0 = m1; s0 = s1; }
+    st.min_key = m0;
+    st.min_slot = s0;
+}
+
 // The caller has checked that key beats the smallest key (or n < k).
 __device__ __forceinline__ void topk_add(uint64_t *L, int ls, int k, RowTopK &st, uint64_t key) {
+    const bool contig = ls == 1 && (k & 1) == 0 && ((uintptr_t)L & 15) == 0;
     if (st.n < k) {
         L[st.n * ls] = key;
-        if (++st.n == k) topk_rescan(L, ls, k, st);
+        if (++st.n == k) {
+            if (contig)
+                topk_rescan_contig(L, k, st);
+            else
+                topk_rescan(L, ls, k, st);
+        }
     } else {
         L[st.min_slot * ls] = key;
-        topk_rescan(L, ls, k, st);
+        if (contig)
+            topk_rescan_contig(L, k, st);
+        else
+            topk_rescan(L, ls, k, st);
     }
 }
 
@@ -85,18 +125,20 @@ __device__ __forceinline__ void topk_sort(uint64_t *L, int ls, int n) {
     }
 }
 
-// Sorts the first n <= 16 keys of a list in global memory descending,
-// through registers (a bitonic network; empty slots are 0 and sort last).
-__device__ __forceinline__ void sort16_desc_in_place(uint64_t *L, int n) {
-    uint64_t r[16];
+// Sorts the first n <= W keys (W = 16 or 32) of a list in global memory
+// descending, through registers (a bitonic network; empty slots are 0 and
+// sort last).
+template <int W>
+__device__ __forceinline__ void sortw_desc_in_place(uint64_t *L, int n) {
+    uint64_t r[W];
 #pragma unroll
-    for (int i = 0; i < 16; ++i) r[i] = i < n ? L[i] : 0ull;
+    for (int i = 0; i < W; ++i) r[i] = i < n ? L[i] : 0ull;
 #pragma unroll
-    for (int size = 2; size <= 16; size <<= 1)
+    for (int size = 2; size <= W; size <<= 1)
 #pragma unroll
         for (int stride = size >> 1; stride > 0; stride >>= 1)
 #pragma unroll
-            for (int i = 0; i < 16; ++i) {
+            for (int i = 0; i < W; ++i) {
                 const int j = i ^ stride;
                 if (j > i) {
                     const bool desc = (i & size) == 0;  // blocks alternate; the last stage is one block
@@ -108,7 +150,7 @@ __device__ __forceinline__ void sort16_desc_in_place(uint64_t *L, int n) {
                 }
             }
 #pragma unroll
-    for (int i = 0; i < 16; ++i)
+    for (int i = 0; i < W; ++i)
         if (i < n) L[i] = r[i];
 }
 

@@ -169,36 +169,42 @@ def test_pair_mma(case):
 
 
 BOUND_CASES = [
-    # N, d, R, Q, k, K, mma
-    (70000, 768, 512, 32, 20, 50, 2),
-    (45000, 256, 300, 20, 100, 100, 2),
-    (30000, 128, 200, 10, 7, 16, 1),
+    # N, d, R, Q, k, K, mma, resident option (0 auto, 2 forced), resident expected
+    (70000, 768, 512, 32, 20, 50, 2, 0, 0),
+    (45000, 256, 300, 20, 100, 100, 2, 0, 0),
+    # forced: sets in global memory that fill (rescans from L2) and grow
+    # past 32 keys (sorted in place at the end of an item)
+    (45000, 256, 300, 20, 100, 100, 2, 2, 1),
+    (30000, 128, 200, 10, 7, 16, 1, 0, 0),
     # 33 sample tiles in 8 chunks, k = 16: four-slot lists kept in registers
-    (400000, 128, 256, 16, 16, 40, 2),
-    # d = 512, k = 100: query blocks resident, sets in global memory, a
-    # four-key bounding pass over at least 50 sample chunks, 14 items of at
-    # most 200 tiles per query group
-    (700000, 512, 300, 20, 100, 100, 2),
+    (400000, 128, 256, 16, 16, 40, 2, 0, 0),
+    # k = 4: items of 97 tiles leave about 16 keys per set, so the query
+    # blocks stay resident by default
+    (300000, 128, 300, 20, 4, 16, 2, 0, 1),
+    # d = 512, k = 100 with a four-key bounding pass over 50 sample chunks,
+    # forced resident
+    (700000, 512, 300, 20, 100, 100, 2, 2, 1),
 ]
 
 
-@pytest.mark.parametrize("case", BOUND_CASES, ids=lambda c: "N%d_d%d_R%d_k%d_mma%d" % (c[0], c[1], c[2], c[4], c[6]))
+@pytest.mark.parametrize("case", BOUND_CASES,
+                         ids=lambda c: "N%d_d%d_R%d_k%d_mma%d_res%d" % (c[0], c[1], c[2], c[4], c[6], c[7]))
 def test_bounding_pass(case):
     """The bounding pass (every 48th corpus tile first, its merged top-k
-    seeding each row's shared threshold) forced on: the oracle's results, and
-    exactly the same keys as without it."""
-    N, d, R, Q, k, K, mma = case
+    seeding each row's shared threshold) forced on, with the query blocks
+    resident where the case expects it: the oracle's results, and exactly
+    the same keys as without the bounding pass (sets in shared memory)."""
+    N, d, R, Q, k, K, mma, res_opt, res_expected = case
     ct = synth.random_bf16(N, d, seed=N + 7)
     rt = synth.random_bf16(R, d, seed=R + 13)
     offsets = ragged_offsets(Q, R, seed=R + 1)
     cn, rn = _bits(ct), _bits(rt)
     truth = oracle_truth(cn, rn, offsets, k, K)
-    on = run_gpu(ct, rt, offsets, k, K, skip.SKIP_PATH_TENSOR, mma=mma, options=((skip.SKIP_OPT_BOUND, 2),))
+    on = run_gpu(ct, rt, offsets, k, K, skip.SKIP_PATH_TENSOR, mma=mma,
+                 options=((skip.SKIP_OPT_BOUND, 2), (skip.SKIP_OPT_RESIDENT, res_opt)))
     off = run_gpu(ct, rt, offsets, k, K, skip.SKIP_PATH_TENSOR, mma=mma, options=((skip.SKIP_OPT_BOUND, 1),))
     assert on[4]["bound"] == 1 and off[4]["bound"] == 0
-    # pairs with d <= 512 keep the query block resident once the bounding
-    # pass runs; without it the sets stay in shared memory
-    assert on[4]["resident_queries"] == int(mma == 2 and d <= 512) and off[4]["resident_queries"] == 0
+    assert on[4]["resident_queries"] == res_expected and off[4]["resident_queries"] == 0
     assert_parity(cn, rn, offsets, k, K, on, truth)
     for a, b in zip(on[:4], off[:4]):
         np.testing.assert_array_equal(a, b)
