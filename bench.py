@@ -4,10 +4,11 @@
 A step is one call of the whole path (per-region MIPS top-k over the corpus,
 cross-partition merge, per-question dedup and top-K; paper §3.3 Eq. rcsr,
 App. B.2 Def. B.2, Alg. 1) on one batch of questions whose region embeddings
-and corpus are already resident in HBM.  The default workload is the 1M-row
-clustered corpus (N = 1,000,000 x d = 768 bf16, 64 questions x 16 regions,
-k_region = 20, K = 50).  The corpus (1.54 GB) is larger than L2 (129 MB), so
-every step streams it from HBM without an explicit flush.
+and corpus are already resident in HBM.  The default workload is the largest
+single-GPU one, the ragged pruned batch (N = 20,000,000 x d = 512 bf16 with
+4,096 clusters, 1,024 questions with U{1..32} regions each, k_region = 100,
+K = 100); --workload picks another.  Every corpus is larger than L2
+(129 MB), so each step streams it from HBM without an explicit flush.
 
 Printed as one JSON line: questions/s (``value``), corpus GB/s, region rows/s,
 TFLOP/s, the roofline of the dominant kernel (CUDA events on the launching
@@ -197,19 +198,36 @@ def host_corpus(corpus, scale):
 
 
 def cpu_baseline(spec, corpus_np, scale_np, regions, offsets, questions):
+    """The oracle on a bounded sample of the batch over the full corpus.
+    Ragged batches: a question with the fewest and one with the most regions
+    (their mean region count is the batch's expected one); fixed batches:
+    the first `questions` questions.  Scaled to questions/s of the batch,
+    which extrapolates from the sample."""
     import oracle
     nthreads = len(os.sched_getaffinity(0))
-    q = min(questions, offsets.numel() - 1)
-    r1 = int(offsets[q])
-    reg = synth.bf16_bits(regions[:r1])
-    off = offsets[:q + 1].numpy()
+    off_all = offsets.numpy().astype(np.int64)
+    counts = np.diff(off_all)
+    if spec.fixed_regions:
+        qs = list(range(min(questions, counts.size)))
+        how = "first %d questions" % len(qs)
+    else:
+        qs = sorted({int(np.argmin(counts)), int(np.argmax(counts))})
+        how = "the questions with the fewest (%d) and the most (%d) regions" % (counts.min(), counts.max())
+    rows = [r for q in qs for r in range(off_all[q], off_all[q + 1])]
+    reg = synth.bf16_bits(regions[rows])
+    off = np.concatenate([[0], np.cumsum(counts[qs])]).astype(np.int32)
     oracle.build()
     t0 = time.perf_counter()
     oracle.retrieve(corpus_np, reg, off, spec.k_region, spec.K, row_scale=scale_np, nthreads=nthreads)
     dt = time.perf_counter() - t0
-    return {"value": q / dt, "unit": "queries/s", "cores": nthreads, "kind": "oracle",
-            "sample": "first %d questions (%d regions) over the full %d-row corpus, fp64, %d OpenMP threads, "
-                      "%.1f s" % (q, r1, spec.N, nthreads, dt)}
+    per_region = dt / max(1, len(rows))
+    batch_s = per_region * int(off_all[-1])
+    return {"value": (counts.size / batch_s) if not spec.fixed_regions else len(qs) / dt, "unit": "queries/s",
+            "cores": nthreads, "kind": "oracle",
+            "sample": "%s (%d regions) over the full %d-row corpus, fp64, %d OpenMP threads, %.1f s; %s" % (
+                how, len(rows), spec.N, nthreads, dt,
+                "scaled per region to the batch's %d regions (extrapolated)" % int(off_all[-1])
+                if not spec.fixed_regions else "measured on the sample")}
 
 
 def run_reference(args, spec):
@@ -273,6 +291,33 @@ def ivfpq_report(args, spec, skip, c, ix, cent, reg_d, off_d, kernels, build_s, 
         a, b = a.cpu().numpy(), b.cpu().numpy()
         return float(np.mean([len(set(x[x >= 0]) & set(y[y >= 0])) / max(1, min(n, (y >= 0).sum()))
                               for x, y in zip(a, b)]))
+
+    # recall and step time over a sweep of probes (after the timed region)
+    sweep = {}
+    for npb in (8, 32, 128):
+        if npb > int(cent.shape[0]):
+            continue
+        out_i = torch.empty_like(q_ivf)
+        out_s = torch.empty(q_ivf.shape, dtype=torch.float32, device=q_ivf.device)
+        for _ in range(3):
+            skip.skip_ivfpq_search(ix, reg_d, off_d, npb, k, spec.K, out_i, out_s)
+        e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+        e0.record()
+        for _ in range(10):
+            skip.skip_ivfpq_search(ix, reg_d, off_d, npb, k, spec.K, out_i, out_s)
+        e1.record()
+        torch.cuda.synchronize()
+        r_ids, _ = skip.skip_ivfpq_search_regions(ix, reg_d, npb, k)
+        sweep[npb] = {"recall_region_at_k": recall(r_ids, ex_ids, k), "recall_question_at_K": recall(out_i, q_ex, spec.K),
+                      "ms_per_step": e0.elapsed_time(e1) / 10}
+    e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    skip.skip_retrieve(c, reg_d, off_d, k, spec.K)
+    e0.record()
+    for _ in range(5):
+        skip.skip_retrieve(c, reg_d, off_d, k, spec.K)
+    e1.record()
+    torch.cuda.synchronize()
+    exact_ms = e0.elapsed_time(e1) / 5
     off, _, _ = skip.skip_ivfpq_lists(ix)
     sizes = (off[1:] - off[:-1]).double()
     probes = torch.topk(reg_d.float() @ cent.float().T, args.nprobe, dim=1).indices
@@ -282,11 +327,13 @@ def ivfpq_report(args, spec, skip, c, ix, cent, reg_d, off_d, kernels, build_s, 
     code_bytes = scanned * (args.pq_m + 4)
     return {
         "ivfpq": {"C": int(cent.shape[0]), "M": args.pq_m, "nprobe": args.nprobe, "build_s": build_s,
+                  "codebook": "k-means on 65,536 rows' residuals" if args.pq_train else "sample-based",
+                  "nprobe_sweep": sweep,
                   "recall_region_at_k": recall(ivf_ids, ex_ids, k), "recall_question_at_K": recall(q_ivf, q_ex, spec.K),
                   "codes_scanned_per_step": scanned, "scan_kernel_ms": scan_ms,
                   "scan_gbs": code_bytes / (scan_ms / 1e3) / 1e9,
                   "scan_frac_of_hbm": code_bytes / (scan_ms / 1e3) / 1e9 / peaks["hbm_gbs"],
-                  "exact_step_ms_for_reference": None,
+                  "exact_step_ms_for_reference": exact_ms,
                   "index_bytes": spec.N * (args.pq_m + 4),
                   "note": "codes of probed lists mostly served from L2 when the index fits in 129 MB"},
         "roofline": {"bound": "hbm", "achieved": code_bytes / (scan_ms / 1e3) / 1e9, "peak": peaks["hbm_gbs"],
@@ -481,10 +528,10 @@ def run_qvs(args, spec, skip):
 def main():
     ap = argparse.ArgumentParser()
     ap.add_argument("--gpus", type=int, default=1)
-    ap.add_argument("--steps", type=int, default=300)
+    ap.add_argument("--steps", type=int, default=50)
     ap.add_argument("--warmup", type=int, default=5)
     ap.add_argument("--impl", default="native", choices=["native", "reference"])
-    ap.add_argument("--workload", default="clustered_1m", choices=sorted(synth.WORKLOADS))
+    ap.add_argument("--workload", default="ragged_20m", choices=sorted(synth.WORKLOADS))
     ap.add_argument("--cpu-questions", type=int, default=8, help="questions in the oracle sample")
     ap.add_argument("--no-cpu-baseline", action="store_true")
     ap.add_argument("--path", default="auto", choices=["auto", "tensor", "warp", "latency"])
@@ -494,6 +541,8 @@ def main():
                     help="step = IVF-PQ search (generator centres as IVF centroids, sample-based PQ codebook)")
     ap.add_argument("--nprobe", type=int, default=32)
     ap.add_argument("--pq-m", type=int, default=64, help="PQ sub-spaces (codes of M bytes)")
+    ap.add_argument("--pq-train", action="store_true",
+                    help="PQ codebook trained by k-means on 65,536 corpus rows' residuals (else sample-based)")
     ap.add_argument("--qvs", action="store_true",
                     help="step = QVS token pruning of one image per question of the workload (576 x 1024 tokens)")
     ap.add_argument("--rho-v", type=float, default=0.4)
@@ -502,6 +551,12 @@ def main():
     ap.add_argument("--dbar", type=float, default=4.0)
     ap.add_argument("--skv", action="store_true",
                     help="step = retrieval + SKV passage gate (skip_retrieve_skv), H = 512, tau 0.5, rho 0.6")
+    ap.add_argument("--wait-timeout-ns", type=int, default=0,
+                    help="cap on each in-kernel wait (0: the library's 2 s); profilers that replay a kernel "
+                         "many times slow it down enough to need more")
+    ap.add_argument("--resident", default="auto", choices=["auto", "never", "force"],
+                    help="query blocks resident in shared memory (pair kernel, d <= 512): the library's rule, "
+                         "never, or whenever the shape allows (smaller profiling captures of the same kernel)")
     ap.add_argument("--mma", default="auto", choices=["auto", "single", "pair"],
                     help="tensor-path MMA shape (auto = library's choice)")
     args = ap.parse_args()
@@ -535,6 +590,9 @@ def main():
     torch.cuda.empty_cache()
     c.set_option(skip.SKIP_OPT_PATH, {"auto": 0, "tensor": 1, "warp": 2, "latency": 3}[args.path])
     c.set_option(skip.SKIP_OPT_MMA, {"auto": 0, "single": 1, "pair": 2}[args.mma])
+    c.set_option(skip.SKIP_OPT_RESIDENT, {"auto": 0, "never": 1, "force": 2}[args.resident])
+    if args.wait_timeout_ns:
+        c.set_option(skip.SKIP_OPT_WAIT_TIMEOUT_NS, args.wait_timeout_ns)
     reg_d = regions.to(dev)
     off_d = offsets.to(dev)
     out_ids = torch.empty(Q, spec.K, dtype=torch.int64, device=dev)
@@ -544,7 +602,8 @@ def main():
     ix = None
     if args.ivfpq:
         cent = synth.make_ivf_centroids(spec).to(dev)
-        codebook = synth.make_pq_codebook(spec, args.pq_m).to(dev)
+        codebook = (synth.train_pq_codebook(spec, args.pq_m, device=dev) if args.pq_train
+                    else synth.make_pq_codebook(spec, args.pq_m)).to(dev)
         torch.cuda.synchronize()
         tb = time.perf_counter()
         ix = skip.skip_ivfpq_build(c, cent, codebook)
@@ -668,8 +727,10 @@ def main():
         # step, outside the algorithmic count: reported, and in ms_per_step
         kb = kernels[kname + "_bound"]
         roof["bound_pass_ms"] = kb["ms"] / max(1, kb["launches"])
-        roof["kernel_note"] = ("full pass only; each call first runs a bounding pass over every 48th "
-                               "corpus tile (bound_pass_ms), counted in ms_per_step")
+        roof["frac_with_bound_pass"] = roof["frac"] * k_ms / (k_ms + roof["bound_pass_ms"])
+        roof["kernel_note"] = ("frac: full pass only; each call first runs a bounding pass over every 48th "
+                               "corpus tile (bound_pass_ms, counted in ms_per_step); frac_with_bound_pass: the "
+                               "algorithmic work over both passes' time")
     line = {
         "metric": METRIC, "value": total_q / secs, "unit": "queries/s", "n_gpus": world,
         "steps": args.steps, "warmup": args.warmup, "ms_per_step": ms / args.steps,

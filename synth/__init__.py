@@ -321,6 +321,36 @@ def make_pq_codebook(spec: WorkloadSpec, M: int, ksub: int = 256, device="cpu") 
     return cb.to(device)
 
 
+def train_pq_codebook(spec: WorkloadSpec, M: int, ksub: int = 256, sample: int = 65536, iters: int = 12,
+                      device="cpu") -> torch.Tensor:
+    """float32 [M, ksub, d / M] PQ codebook trained by k-means (Lloyd's
+    algorithm, squared L2) on the residuals bf16(x_i) - bf16(c_{a_i}) of the
+    first `sample` corpus rows, each sub-space on its own; it starts from the
+    sample-based codebook above, and a codeword that loses all its points
+    keeps its place.  Index training, like the paper's FAISS index (trained
+    offline on its corpus), is input preparation here: the library and the
+    oracle both take the codebook as given."""
+    if spec.d % M:
+        raise ValueError("M must divide d")
+    centres = draw_centres(spec, spec.centres, spec.d, "cpu")
+    x, a = corpus_rows_fp32(spec.index, 0, min(sample, spec.N), spec.d, spec.corpus, centres, "cpu",
+                            return_centres=True)
+    r = (x.to(torch.bfloat16).float() - centres[a].to(torch.bfloat16).float()).to(device)
+    ds = spec.d // M
+    sub = r.view(r.shape[0], M, ds).permute(1, 0, 2).contiguous()      # [M, n, ds]
+    cb = make_pq_codebook(spec, M, ksub, device=device).clone()          # [M, ksub, ds]
+    for _ in range(iters):
+        # nearest codeword of every sub-vector: argmin ||r||^2 - 2 r.c + ||c||^2
+        d2 = (cb * cb).sum(-1)[:, None, :] - 2.0 * torch.bmm(sub, cb.transpose(1, 2))
+        assign = d2.argmin(-1)                                           # [M, n]
+        sums = torch.zeros_like(cb).scatter_add_(1, assign[..., None].expand(-1, -1, ds), sub)
+        cnt = torch.zeros(M, ksub, device=sub.device).scatter_add_(1, assign, torch.ones_like(assign,
+                                                                                              dtype=torch.float32))
+        upd = cnt > 0
+        cb[upd] = sums[upd] / cnt[upd][:, None]
+    return cb.to(device)
+
+
 # ---- inputs of QVS (App. B.1 Def. B.1) -------------------------------------
 #
 # QVS scores L visual tokens per image against the question: L = 576 (a 24 x

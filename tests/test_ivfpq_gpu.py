@@ -334,8 +334,27 @@ def test_full_size_build_and_recall():
     nl, nc = check_build(corpus, cent, cb, lists, code_by_id, rows)
     g, gs, e = g_ids.cpu().numpy(), g_sc.cpu().numpy(), e_ids.cpu().numpy()
     ce, qn = synth.bf16_bits(cent), synth.bf16_bits(regions)
+    # Completeness: the oracle's search of the GPU's own index (its lists and
+    # codes, whose sampled rows match the oracle's encoding above) for the
+    # sampled regions; every sure id of the oracle's list must be returned.
+    gidx = {"offsets": off, "ids": ids.astype(np.int64), "codes": code_by_id, "lists": lists}
+    sample = np.random.default_rng(8).choice(regions.shape[0], 6, replace=False)
+    o_ids, o_sc, _ = oracle.ivfpq_search(gidx, ce, cb.numpy(), qn[sample], nprobe, spec.k_region + 32)
+    complete = 0
+    for j, t in enumerate(checker.region_truths(o_ids, o_sc, spec.k_region)):
+        r = int(sample[j])
+        cs = oracle.score_matrix(ce, qn[r:r + 1])[0]
+        order = np.argsort(-cs, kind="stable")
+        if cs[order[nprobe - 1]] - cs[order[nprobe]] <= PROBE_TIE:
+            continue
+        _, probs = checker.check_region(
+            g_ids[r].cpu().numpy(), g_sc[r].cpu().numpy(), t,
+            extra_score=lambda i, r=r: float(oracle.ivfpq_scores_at(gidx, ce, cb.numpy(), qn, [r], [i])[0]))
+        assert not probs, (r, probs[:3])
+        complete += 1
+    assert complete >= 3
     checked = 0
-    for r in np.random.default_rng(8).choice(regions.shape[0], 6, replace=False):
+    for r in sample:
         cs = oracle.score_matrix(ce, qn[r:r + 1])[0]
         order = np.argsort(-cs, kind="stable")
         if cs[order[nprobe - 1]] - cs[order[nprobe]] <= PROBE_TIE:
