@@ -326,33 +326,55 @@ __global__ void __launch_bounds__(kThreads, 1)
                     __syncwarp();
                 }
             }
-            // Chunk done: merge the eight warps' sets of every query into the
-            // chunk's list -- for k <= 16 one warp-wide sort of the 8k keys
-            // per query, else sorted sets merged by a warp (the two hand-offs
-            // between the epilogue warps are bounded waits, like every other
-            // wait).
-            const bool small_k = kEpiWarps * k <= 128;
+            // Chunk done: each warp sorts its sets (lane q: query q), then
+            // lane q of warp q mod 8 merges the eight sorted sets of query q
+            // into the chunk's list -- one lane per query, all queries at once,
+            // no warp-wide chains (the two hand-offs between the epilogue
+            // warps are bounded waits, like every other wait).
             if (lane < R) {
-                if (!small_k) topk_sort(Lw + (size_t)lane * k, 1, top.n);
-                for (int t = top.n; t < k; ++t) Lw[(size_t)lane * k + t] = 0ull;
+                uint64_t *Lq = Lw + (size_t)lane * k;
+                for (int t = top.n; t < k; ++t) Lq[t] = 0ull;
+                if (k <= 16)
+                    sortw_desc_in_place<16>(Lq, top.n);
+                else if (k <= 32)
+                    sortw_desc_in_place<32>(Lq, top.n);
+                else
+                    topk_sort(Lq, 1, top.n);
             }
             const uint32_t par = (uint32_t)(chunk & 1);
             mbar_arrive(smem_addr(&sh->sorted));
             if (!mbar_wait(smem_addr(&sh->sorted), par, p.timeout_ns)) ok = false;
-            for (int q = ew; q < R && ok; q += kEpiWarps) {
-                uint64_t *out = p.lists + ((int64_t)v * R + q) * k;
-                if (small_k) {
-                    uint64_t keys4[4];
+            {
+                const int q = lane * kEpiWarps + ew;
+                if (ok && q < R) {
+                    uint64_t *out = p.lists + ((int64_t)v * R + q) * k;
+                    // heads of the eight sorted sets of query q
+                    const uint64_t *Ls[kEpiWarps];
+                    uint64_t h[kEpiWarps];
+                    int at[kEpiWarps];
 #pragma unroll
-                    for (int u = 0; u < 4; ++u) {
-                        const int pos = lane + 32 * u, w = pos / k, tt = pos - w * k;
-                        keys4[u] = pos < kEpiWarps * k ? slists[((size_t)w * R + q) * k + tt] : 0ull;
+                    for (int w = 0; w < kEpiWarps; ++w) {
+                        Ls[w] = slists + ((size_t)w * R + q) * k;
+                        at[w] = 0;
+                        h[w] = Ls[w][0];
                     }
-                    warp_sort128_desc(keys4);
-                    if (lane < k) out[lane] = keys4[0];
-                } else {
-                    warp_merge_topk<1>(slists + (size_t)q * k, (int64_t)R * k, kEpiWarps, k, k,
-                                       [&](int idx, uint64_t key) { out[idx] = key; });
+                    for (int t = 0; t < k; ++t) {
+                        uint64_t best = h[0];
+                        int bw = 0;
+#pragma unroll
+                        for (int w = 1; w < kEpiWarps; ++w)
+                            if (h[w] > best) {
+                                best = h[w];
+                                bw = w;
+                            }
+                        out[t] = best;
+#pragma unroll
+                        for (int w = 0; w < kEpiWarps; ++w)
+                            if (w == bw) {
+                                ++at[w];
+                                h[w] = (best != 0ull && at[w] < k) ? Ls[w][at[w]] : 0ull;
+                            }
+                    }
                 }
             }
             mbar_arrive(smem_addr(&sh->merged));

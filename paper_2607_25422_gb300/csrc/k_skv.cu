@@ -5,11 +5,13 @@
 //                for all questions at once, on the tensor cores (k_gemm.cu).
 //  k_skv_mlp     per 128 passage slots x 128 hidden units: the passage part
 //                of layer 1 on the tensor cores.  The A operand is built in
-//                shared memory by four warps from the gathered corpus rows
-//                and qbar: per 64-column chunk of d, three K-slices
+//                shared memory by eight warps (two per slot row, each with
+//                three chunks of its row in flight) from the gathered corpus
+//                rows and qbar: per 64-column chunk of d, three K-slices
 //                e | bf16(e * qbar) | bf16(|e - qbar|) in the 128-byte
-//                swizzled layout TMA would produce; the B operand is the
-//                matching W1 column blocks, loaded by TMA.  tcgen05.mma
+//                swizzled layout TMA would produce, one slice per stage of a
+//                six-stage ring; the B operand is the matching W1 column
+//                block, loaded by TMA.  tcgen05.mma
 //                (kind::f16, M = N = 128) accumulates in TMEM; the epilogue
 //                adds c_q, applies ReLU and the w2 dot for its 128 units and
 //                writes one partial logit per slot and hidden block.
@@ -28,9 +30,11 @@ namespace {
 
 constexpr int kSkvRows = 128;                       // passage slots per CTA (TMEM lanes)
 constexpr int kSkvSlice = kSkvRows * 128;           // one [128 x 64] bf16 K-slice, bytes
-constexpr int kSkvStageA = 3 * kSkvSlice;           // e | e*qbar | |e - qbar|
-constexpr int kSkvStageB = 3 * kSkvSlice;           // the three W1 column blocks (128 units)
-constexpr int kSkvStages = 2;
+// A stage is one K-slice: of A (e, e*qbar or |e - qbar| of one 64-column
+// chunk of d) and of B (the matching W1 column block for 128 units).
+constexpr int kSkvStageA = kSkvSlice;
+constexpr int kSkvStageB = kSkvSlice;
+constexpr int kSkvStages = 6;
 constexpr int kSkvBuilders = 8;                     // two builder warps per TMEM lane quadrant
 constexpr int kSkvThreads = 64 + 32 * kSkvBuilders;  // TMA warp, MMA warp, builders (4 of them: epilogue)
 constexpr int kSkvAhead = 3;                         // chunks of corpus row in flight per builder thread
@@ -104,17 +108,16 @@ __global__ void __launch_bounds__(kSkvThreads, 1)
         if (lane == 0) {
             bool ok = true;
             int issued = 0;
-            for (int c = 0; c < nc && ok; ++c) {
-                const int s = c % kSkvStages;
-                const uint32_t ph = (uint32_t)(c / kSkvStages) & 1u;
+            for (int u = 0; u < 3 * nc && ok; ++u) {
+                const int s = u % kSkvStages, c = u / 3, b = u - 3 * c;
+                const uint32_t ph = (uint32_t)(u / kSkvStages) & 1u;
                 if (!mbar_wait(smem_addr(&sh->empty[s]), ph ^ 1u, p.timeout_ns)) {
                     ok = false;
                     break;
                 }
                 const uint32_t fb = smem_addr(&sh->full[s]);
                 mbar_arrive_expect_tx(fb, kSkvStageB);
-                for (int b = 0; b < 3; ++b)
-                    tma_load_2d(smem_addr(sB + s * kSkvStageB + b * kSkvSlice), &tw, fb, (2 + b) * p.d + c * 64, n0);
+                tma_load_2d(smem_addr(sB + s * kSkvStageB), &tw, fb, (2 + b) * p.d + c * 64, n0);
                 ++issued;
             }
             if (!ok) atomicOr(p.err, kErrTimeout);
@@ -130,22 +133,19 @@ __global__ void __launch_bounds__(kSkvThreads, 1)
         // ------------------------------------------------ MMA issuer
         if (lane == 0) {
             bool ok = true;
-            for (int c = 0; c < nc && ok; ++c) {
-                const int s = c % kSkvStages;
-                const uint32_t ph = (uint32_t)(c / kSkvStages) & 1u;
+            for (int u = 0; u < 3 * nc && ok; ++u) {
+                const int s = u % kSkvStages;
+                const uint32_t ph = (uint32_t)(u / kSkvStages) & 1u;
                 if (!mbar_wait(smem_addr(&sh->full[s]), ph, p.timeout_ns)) {
                     ok = false;
                     break;
                 }
                 tc_fence_after();
-                for (int b = 0; b < 3; ++b) {
-                    const uint64_t ad = smem_desc_k128(smem_addr(sA + s * kSkvStageA + b * kSkvSlice));
-                    const uint64_t bd = smem_desc_k128(smem_addr(sB + s * kSkvStageB + b * kSkvSlice));
+                const uint64_t ad = smem_desc_k128(smem_addr(sA + s * kSkvStageA));
+                const uint64_t bd = smem_desc_k128(smem_addr(sB + s * kSkvStageB));
 #pragma unroll
-                    for (int kk = 0; kk < 4; ++kk)
-                        tc_mma_f16(tmem, ad + (uint64_t)(kk * 2), bd + (uint64_t)(kk * 2), kSkvIdesc,
-                                   (c | b | kk) != 0);
-                }
+                for (int kk = 0; kk < 4; ++kk)
+                    tc_mma_f16(tmem, ad + (uint64_t)(kk * 2), bd + (uint64_t)(kk * 2), kSkvIdesc, (u | kk) != 0);
                 tc_commit(smem_addr(&sh->empty[s]));
             }
             if (!ok) atomicOr(p.err, kErrTimeout);
@@ -185,8 +185,6 @@ __global__ void __launch_bounds__(kSkvThreads, 1)
             }
         bool ok = true;
         for (int c = 0; c < nc; ++c) {
-            const int s = c % kSkvStages;
-            const uint32_t ph = (uint32_t)(c / kSkvStages) & 1u;
             uint4 e[4], qv[4];
 #pragma unroll
             for (int j = 0; j < 4; ++j) {
@@ -210,28 +208,32 @@ __global__ void __launch_bounds__(kSkvThreads, 1)
                     qb[kSkvAhead - 1][j] = ld ? __ldg(qrow + cn * 8 + j) : zero;
                 }
             }
-            if (!mbar_wait(smem_addr(&sh->empty[s]), ph ^ 1u, p.timeout_ns)) {
-                ok = false;
-                break;
-            }
-            // Row r of each slice: 16-byte chunk j at position j ^ (r & 7).
-            const uint32_t base = smem_addr(sA + s * kSkvStageA) + r * 128;
-            const int sw = r & 7;
+            uint4 f[3][4];  // the chunk's three K-slices of this thread's half row
 #pragma unroll
             for (int jj = 0; jj < 4; ++jj) {
-                const int j = 4 * half + jj;
-                uint4 eq, ad;
-                features2(e[jj].x, qv[jj].x, eq.x, ad.x);
-                features2(e[jj].y, qv[jj].y, eq.y, ad.y);
-                features2(e[jj].z, qv[jj].z, eq.z, ad.z);
-                features2(e[jj].w, qv[jj].w, eq.w, ad.w);
-                const uint32_t off = (uint32_t)((j ^ sw) << 4);
-                sts128(base + off, e[jj]);
-                sts128(base + kSkvSlice + off, eq);
-                sts128(base + 2 * kSkvSlice + off, ad);
+                f[0][jj] = e[jj];
+                features2(e[jj].x, qv[jj].x, f[1][jj].x, f[2][jj].x);
+                features2(e[jj].y, qv[jj].y, f[1][jj].y, f[2][jj].y);
+                features2(e[jj].z, qv[jj].z, f[1][jj].z, f[2][jj].z);
+                features2(e[jj].w, qv[jj].w, f[1][jj].w, f[2][jj].w);
             }
-            fence_proxy_async_smem();
-            mbar_arrive(smem_addr(&sh->full[s]));
+            // Row r of each slice: 16-byte chunk j at position j ^ (r & 7).
+            const int sw = r & 7;
+#pragma unroll
+            for (int b = 0; b < 3; ++b) {
+                const int u = 3 * c + b, s = u % kSkvStages;
+                const uint32_t ph = (uint32_t)(u / kSkvStages) & 1u;
+                if (!mbar_wait(smem_addr(&sh->empty[s]), ph ^ 1u, p.timeout_ns)) {
+                    ok = false;
+                    break;
+                }
+                const uint32_t base = smem_addr(sA + s * kSkvStageA) + r * 128;
+#pragma unroll
+                for (int jj = 0; jj < 4; ++jj) sts128(base + (uint32_t)(((4 * half + jj) ^ sw) << 4), f[b][jj]);
+                fence_proxy_async_smem();
+                mbar_arrive(smem_addr(&sh->full[s]));
+            }
+            if (!ok) break;
         }
         if (!ok) atomicOr(p.err, kErrTimeout);
         // Epilogue: h = acc + c_q, ReLU, dot with w2 over this CTA's units.
