@@ -328,6 +328,7 @@ def ivfpq_report(args, spec, skip, c, ix, cent, reg_d, off_d, kernels, build_s, 
     return {
         "ivfpq": {"C": int(cent.shape[0]), "M": args.pq_m, "nprobe": args.nprobe, "build_s": build_s,
                   "codebook": "k-means on 65,536 rows' residuals" if args.pq_train else "sample-based",
+                  "refine": args.ivf_refine,
                   "nprobe_sweep": sweep,
                   "recall_region_at_k": recall(ivf_ids, ex_ids, k), "recall_question_at_K": recall(q_ivf, q_ex, spec.K),
                   "codes_scanned_per_step": scanned, "scan_kernel_ms": scan_ms,
@@ -541,6 +542,8 @@ def main():
                     help="step = IVF-PQ search (generator centres as IVF centroids, sample-based PQ codebook)")
     ap.add_argument("--nprobe", type=int, default=32)
     ap.add_argument("--pq-m", type=int, default=64, help="PQ sub-spaces (codes of M bytes)")
+    ap.add_argument("--ivf-refine", type=int, default=0,
+                    help="IVF-PQ: re-rank the best r * k_region entries by s^ exactly (0: plain IVF-PQ)")
     ap.add_argument("--pq-train", action="store_true",
                     help="PQ codebook trained by k-means on 65,536 corpus rows' residuals (else sample-based)")
     ap.add_argument("--qvs", action="store_true",
@@ -608,6 +611,8 @@ def main():
         tb = time.perf_counter()
         ix = skip.skip_ivfpq_build(c, cent, codebook)
         build_s = time.perf_counter() - tb
+        if args.ivf_refine:
+            ix.set_option(skip.SKIP_OPT_IVF_REFINE, args.ivf_refine)
 
         def step():
             skip.skip_ivfpq_search(ix, reg_d, off_d, args.nprobe, spec.k_region, spec.K, out_ids, out_sc, stream)
@@ -752,7 +757,9 @@ def main():
     }
     if args.ivfpq:
         line.update(ivfpq_report(args, spec, skip, c, ix, cent, reg_d, off_d, kernels, build_s, peaks, ms))
-        line["config"]["variant"] = "IVF-PQ: %d centroids, PQ%d, nprobe %d" % (cent.shape[0], args.pq_m, args.nprobe)
+        line["config"]["variant"] = "IVF-PQ: %d centroids, PQ%d, nprobe %d%s" % (
+            cent.shape[0], args.pq_m, args.nprobe,
+            ", exact re-rank of the best %d x k_region" % args.ivf_refine if args.ivf_refine else "")
         ix.free()
     if args.skv:
         line["config"]["skv_gate"] = {"hidden": 512, "tau_nu": 0.5, "rho_r": 0.6}

@@ -73,7 +73,11 @@ SKIP_API skip_status_t skip_ivfpq_free(skip_ivfpq_t index);
 
 /*
  * skip_ivfpq_search_regions -- per region: reg_ids int64 / reg_scores fp32,
- * both device [R_total x k_region], sorted by (s^ desc, id asc).
+ * both device [R_total x k_region], sorted by (s^ desc, id asc); with
+ * SKIP_OPT_IVF_REFINE = r >= 2 (an option beyond the paper's IVF-PQ, the
+ * usual exact re-rank), the best min(r k_region, 1024) entries by s^ are
+ * re-scored exactly (fp32 sums of the bf16 products) and the k_region best by
+ * (exact score desc, id asc) are returned with their exact scores.
  */
 SKIP_API skip_status_t skip_ivfpq_search_regions(skip_ivfpq_t index, const void *regions, int32_t R_total,
                                                  int32_t nprobe, int32_t k_region, int64_t *reg_ids,
@@ -91,13 +95,14 @@ SKIP_API skip_status_t skip_ivfpq_search(skip_ivfpq_t index, const void *regions
 /* As skip_sync_status, for the index's kernels. */
 SKIP_API skip_status_t skip_ivfpq_sync_status(skip_ivfpq_t index, void *stream);
 
-/* Sets an option of the index: SKIP_OPT_IVF_SPLIT for its list scan; any
+/* Sets an option of the index: SKIP_OPT_IVF_SPLIT for its list scan,
+ * SKIP_OPT_IVF_REFINE for the exact re-rank of a shortlist; any
  * other skip_option_t of skip_retrieve.h applies to its centroid set, which
  * the exact MIPS path searches for the build's coarse assignment and, with
  * more than 4,096 centroids, for the search's coarse probe (with at most
  * 4,096 the probe is one bf16 GEMM and a per-region sort).  SKIP_OPT_TIMING
  * records the index's kernels, reported by skip_ivfpq_timing_report.
- * Results do not depend on the options. */
+ * Apart from SKIP_OPT_IVF_REFINE, results do not depend on the options. */
 SKIP_API skip_status_t skip_ivfpq_set_option(skip_ivfpq_t index, int option, int64_t value);
 SKIP_API skip_status_t skip_ivfpq_timing_report(skip_ivfpq_t index, char *buf, int32_t len);
 

@@ -87,12 +87,18 @@ typedef enum {
                                      host staging and gate buffers (reallocating them now);
                                      skip_sync_status then also checks them and returns
                                      SKIP_ECANARY if any changed.  0 (default) off. */
-    SKIP_OPT_RESIDENT = 9         /* bf16 tensor path with CTA pairs, d <= 512, after a
+    SKIP_OPT_RESIDENT = 9,        /* bf16 tensor path with CTA pairs, d <= 512, after a
                                      bounding pass: 0 auto (each CTA keeps its query block in
                                      shared memory for a work item and the per-row sets in
                                      global memory when the items can be sized so that about
                                      16 keys or fewer reach a set), 1 never, 2 whenever the
                                      shape allows (for tests) */
+    SKIP_OPT_IVF_REFINE = 10      /* IVF-PQ index built from a corpus (skip_ivfpq_set_option):
+                                     0 or 1 off; r >= 2 keeps the best min(r k_region, 1024)
+                                     entries of each region by s^ and re-ranks them by the
+                                     exact inner product with the corpus rows (the corpus
+                                     handle must stay alive); SKIP_EUNSUPPORTED for an index
+                                     made by skip_ivfpq_load */
 } skip_option_t;
 
 enum { SKIP_PATH_AUTO = 0, SKIP_PATH_TENSOR = 1, SKIP_PATH_WARP = 2, SKIP_PATH_LATENCY = 3 };

@@ -21,7 +21,7 @@ Functions and what they follow:
   (``skv_oracle.c``).
 * ``bf16_round``   -- a double rounded to bf16 (ties to even), as bits.
 * ``ivf_assign``, ``pq_encode``, ``ivfpq_build``, ``ivfpq_search``,
-  ``ivfpq_scores_at`` -- the IVF-PQ index (§4.1 "Implementation", App. I.4;
+  ``ivfpq_search_refine``, ``ivfpq_scores_at`` -- the IVF-PQ index (§4.1 "Implementation", App. I.4;
   the published inverted file with product-quantised residuals and
   asymmetric inner-product scoring) and its search (``ivfpq_oracle.c``).
 * ``qvs``, ``qvs_count`` -- App. B.1 Def. B.1 (Eq. qvs_score) and the Alg. 1
@@ -334,6 +334,26 @@ def ivfpq_search(index, centroids, codebook, regions, nprobe, k):
                                     _ptr(probes)):
         raise RuntimeError("oracle ivfpq_search failed")
     return out_ids, out_sc, probes
+
+
+def ivfpq_search_refine(index, centroids, codebook, regions, nprobe, k, ks, corpus, row_scale=None):
+    """IVF-PQ search followed by an exact re-rank (the usual refinement of an
+    IVF-PQ shortlist): each region's best ks entries by s^ (ivfpq_search),
+    re-scored with the exact fp64 inner product (scores_at), the k best by
+    (score desc, id asc).  Returns (ids int64 [R, k], scores float64 [R, k])."""
+    s_ids, _, _ = ivfpq_search(index, centroids, codebook, regions, nprobe, ks)
+    R = s_ids.shape[0]
+    out_ids = np.full((R, k), -1, np.int64)
+    out_sc = np.full((R, k), -np.inf)
+    for r in range(R):
+        cand = s_ids[r][s_ids[r] >= 0]
+        if cand.size == 0:
+            continue
+        ex = scores_at(corpus, regions, np.full(cand.size, r), cand, row_scale=row_scale)
+        order = np.lexsort((cand, -ex))[:k]
+        out_ids[r, :order.size] = cand[order]
+        out_sc[r, :order.size] = ex[order]
+    return out_ids, out_sc
 
 
 def ivfpq_scores_at(index, centroids, codebook, regions, region_idx, ids):

@@ -32,7 +32,7 @@ from . import _build
 SKIP_BF16, SKIP_E4M3 = 0, 1
 SKIP_OK, SKIP_EINVAL, SKIP_ENOMEM, SKIP_EUNSUPPORTED, SKIP_ETIMEOUT, SKIP_ECUDA, SKIP_ECANARY = range(7)
 (SKIP_OPT_PATH, SKIP_OPT_WAIT_TIMEOUT_NS, SKIP_OPT_GRID, SKIP_OPT_TIMING, SKIP_OPT_CLUSTER, SKIP_OPT_MMA,
- SKIP_OPT_BOUND, SKIP_OPT_IVF_SPLIT, SKIP_OPT_CANARY, SKIP_OPT_RESIDENT) = range(10)
+ SKIP_OPT_BOUND, SKIP_OPT_IVF_SPLIT, SKIP_OPT_CANARY, SKIP_OPT_RESIDENT, SKIP_OPT_IVF_REFINE) = range(11)
 SKIP_PATH_AUTO, SKIP_PATH_TENSOR, SKIP_PATH_WARP, SKIP_PATH_LATENCY = range(4)
 SKIP_MAX_K_REGION, SKIP_MAX_K = 1024, 2048
 

@@ -573,7 +573,78 @@ cudaError_t launch_scan_np(const IvfParams &p, const uint16_t *regions, int R, c
                                                                               nprobe, k, G, out_keys);
     return cudaGetLastError();
 }
+
+// Exact re-rank of an IVF-PQ shortlist (an option beyond the paper's FAISS
+// IVF-PQ, the usual "refine" step): per region, the ks candidates the scan
+// kept by s^ (keys [R x ks], descending, 0 = none) are scored exactly,
+// s(r, i) = sum_j q_{r,j} x_{i,j} in fp32 from the bf16 corpus rows, and the
+// k best by (s desc, id asc) are written as keys [R x k].  One block per
+// region: a warp per candidate row (16-byte loads, the query in shared memory
+// as fp32), then a bitonic sort of the keys in shared memory.
+constexpr int kRefineThreads = 256;
+constexpr int kRefineMax = 1024;
+
+__global__ void __launch_bounds__(kRefineThreads) k_ivf_refine(const uint16_t *__restrict__ rows, int64_t N, int d,
+                                                                const uint16_t *__restrict__ regions,
+                                                                const uint64_t *__restrict__ cand, int ks, int k,
+                                                                uint64_t *__restrict__ out) {
+    extern __shared__ float qf[];                       // [d]
+    __shared__ uint64_t keys[kRefineMax];
+    const int r = blockIdx.x;
+    const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+    for (int j = threadIdx.x; j < d; j += kRefineThreads)
+        qf[j] = __uint_as_float((uint32_t)regions[(int64_t)r * d + j] << 16);
+    int n2 = 1;
+    while (n2 < ks) n2 <<= 1;
+    for (int t = threadIdx.x; t < n2; t += kRefineThreads) keys[t] = 0ull;
+    __syncthreads();
+    const int nw = d / 8;  // 16-byte words per row
+    for (int t = warp; t < ks; t += kRefineThreads / 32) {
+        const uint64_t ck = cand[(int64_t)r * ks + t];
+        if (ck == 0ull) continue;  // warp-uniform
+        const int64_t id = (int64_t)(0xFFFFFFFFu - (uint32_t)ck);
+        if (id < 0 || id >= N) continue;
+        const uint4 *row = reinterpret_cast<const uint4 *>(rows + id * (int64_t)d);
+        float acc = 0.f;
+        for (int w = lane; w < nw; w += 32) {
+            const uint4 x = __ldg(row + w);
+            const uint32_t xv[4] = {x.x, x.y, x.z, x.w};
+#pragma unroll
+            for (int h = 0; h < 4; ++h) {
+                acc = fmaf(__uint_as_float(xv[h] << 16), qf[8 * w + 2 * h], acc);
+                acc = fmaf(__uint_as_float(xv[h] & 0xFFFF0000u), qf[8 * w + 2 * h + 1], acc);
+            }
+        }
+#pragma unroll
+        for (int o = 16; o; o >>= 1) acc += __shfl_xor_sync(0xffffffffu, acc, o);
+        if (lane == 0) keys[t] = make_key(acc, (uint32_t)id);
+    }
+    __syncthreads();
+    for (int size = 2; size <= n2; size <<= 1)
+        for (int stride = size >> 1; stride > 0; stride >>= 1) {
+            for (int t = threadIdx.x; t < n2 / 2; t += kRefineThreads) {
+                const int lo = 2 * t - (t & (stride - 1)), hi = lo + stride;
+                const bool desc = (lo & size) == 0;
+                const uint64_t a = keys[lo], b = keys[hi];
+                if ((a < b) == desc) {
+                    keys[lo] = b;
+                    keys[hi] = a;
+                }
+            }
+            __syncthreads();
+        }
+    for (int t = threadIdx.x; t < k; t += kRefineThreads) out[(int64_t)r * k + t] = t < n2 ? keys[t] : 0ull;
+}
+
 }  // namespace
+
+cudaError_t launch_ivf_refine(const uint16_t *rows, int64_t N, int d, const uint16_t *regions, int R,
+                              const uint64_t *cand, int ks, int k, uint64_t *out, cudaStream_t s) {
+    if (R <= 0) return cudaSuccess;
+    if (ks < 1 || ks > kRefineMax || k < 1 || k > ks || d % 8 != 0) return cudaErrorInvalidValue;
+    k_ivf_refine<<<R, kRefineThreads, (size_t)d * sizeof(float), s>>>(rows, N, d, regions, cand, ks, k, out);
+    return cudaGetLastError();
+}
 
 cudaError_t ivfpq_scan_split(int M, int nprobe, int R, int sms, int requested, int *G) {
     if (requested > 0) {

@@ -1099,6 +1099,8 @@ struct skip_ivfpq {
     size_t ws_bytes = 0;
     int split = 0;                // parts per region of the list scan (0: pick)
     bool gemm_probe = false;      // coarse probe: one GEMM + per-region sort (C <= kIvfCoarseMaxC)
+    const skip_corpus *src = nullptr;  // corpus the index was built from (exact re-rank), or null
+    int refine = 0;               // SKIP_OPT_IVF_REFINE: shortlist refine * k by s^, re-ranked exactly
 };
 
 namespace {
@@ -1254,6 +1256,43 @@ skip_status_t ivf_check_search(skip_ivfpq *ix, const void *regions, int R, int n
     return SKIP_OK;
 }
 
+// Each region's k keys [R x k] (sorted), in the index workspace: the scan's
+// top k by s^, or with a refine factor its top min(refine k, 1024) re-ranked
+// by exact scores against the corpus the index was built from.
+skip_status_t ivf_region_keys(skip_ivfpq *ix, const void *regions, int R, int nprobe, int k, cudaStream_t s,
+                              uint64_t **out) {
+    const int ks = ix->refine > 1 ? (int)std::min<int64_t>(std::min<int64_t>((int64_t)ix->refine * k, kIvfMaxRefine),
+                                                           ix->N)
+                                  : k;
+    uint64_t *keys = nullptr, *merged = nullptr;
+    int G = 1;
+    skip_status_t st = ivf_regions(ix, regions, R, nprobe, std::max(ks, k), s, &keys, &merged, &G);
+    if (st || R == 0) {
+        *out = keys;
+        return st;
+    }
+    const int kk = std::max(ks, k);
+    if (G > 1) {
+        record(ix->cent, s, "merge_lists");
+        st = cuda_status(launch_merge_lists(keys, G, (int64_t)R * kk, R, kk, merged, nullptr, nullptr, s));
+        if (st) return st;
+    } else {
+        merged = keys;
+    }
+    if (ks > k) {
+        // the shortlist (merged) is re-ranked into the head of the workspace
+        uint64_t *dst = merged == keys ? keys + (size_t)R * kk : keys;
+        record(ix->cent, s, "ivf_refine");
+        st = cuda_status(launch_ivf_refine(reinterpret_cast<const uint16_t *>(ix->src->rows), ix->src->N,
+                                           ix->src->d, reinterpret_cast<const uint16_t *>(regions), R, merged, ks,
+                                           k, dst, s));
+        *out = dst;
+        return st;
+    }
+    *out = merged;
+    return SKIP_OK;
+}
+
 }  // namespace
 
 extern "C" {
@@ -1268,6 +1307,7 @@ skip_status_t skip_ivfpq_build(skip_corpus_t c, const void *centroids, int32_t C
     skip_ivfpq *ix = nullptr;
     st = ivf_create(centroids, C, c->d, codebook, M, c->N, s, &ix);
     if (st) return st;
+    ix->src = c;
     const int64_t N = c->N;
     void *tmp = nullptr;
     const size_t rl = align_up((size_t)N * 8, 256), rs = align_up((size_t)N * 4, 256);
@@ -1362,12 +1402,11 @@ skip_status_t skip_ivfpq_search_regions(skip_ivfpq_t ix, const void *regions, in
     if (R_total > 0 && (!reg_ids || !reg_scores)) return SKIP_EINVAL;
     cudaStream_t s = reinterpret_cast<cudaStream_t>(stream);
     ++ix->cent->call_id;
-    uint64_t *keys = nullptr, *merged = nullptr;
-    int G = 1;
-    st = ivf_regions(ix, regions, R_total, nprobe, k_region, s, &keys, &merged, &G);
+    uint64_t *keys = nullptr;
+    st = ivf_region_keys(ix, regions, R_total, nprobe, k_region, s, &keys);
     if (st || R_total == 0) return st;
     record(ix->cent, s, "merge_lists");
-    st = cuda_status(launch_merge_lists(keys, G, (int64_t)R_total * k_region, R_total, k_region, nullptr, reg_ids,
+    st = cuda_status(launch_merge_lists(keys, 1, (int64_t)R_total * k_region, R_total, k_region, nullptr, reg_ids,
                                         reg_scores, s));
     record(ix->cent, s, "end");
     return st;
@@ -1382,17 +1421,9 @@ skip_status_t skip_ivfpq_search(skip_ivfpq_t ix, const void *regions, const int3
     if (Q == 0 && R_total != 0) return SKIP_EINVAL;
     cudaStream_t s = reinterpret_cast<cudaStream_t>(stream);
     ++ix->cent->call_id;
-    uint64_t *keys = nullptr, *merged = nullptr;
-    int G = 1;
-    st = ivf_regions(ix, regions, R_total, nprobe, k_region, s, &keys, &merged, &G);
+    uint64_t *keys = nullptr;
+    st = ivf_region_keys(ix, regions, R_total, nprobe, k_region, s, &keys);
     if (st) return st;
-    if (G > 1 && R_total > 0) {
-        record(ix->cent, s, "merge_lists");
-        st = cuda_status(launch_merge_lists(keys, G, (int64_t)R_total * k_region, R_total, k_region, merged, nullptr,
-                                            nullptr, s));
-        if (st) return st;
-        keys = merged;
-    }
     if (Q > 0) {
         record(ix->cent, s, "question_merge");
         st = cuda_status(launch_question_merge(keys, k_region, region_offsets, Q, R_total, K, out_ids, out_scores,
@@ -1412,6 +1443,12 @@ skip_status_t skip_ivfpq_set_option(skip_ivfpq_t ix, int option, int64_t value) 
     if (option == SKIP_OPT_IVF_SPLIT) {
         if (value < 0 || value > kIvfMaxSplit) return SKIP_EINVAL;
         ix->split = (int)value;
+        return SKIP_OK;
+    }
+    if (option == SKIP_OPT_IVF_REFINE) {
+        if (value < 0 || value > kIvfMaxRefine) return SKIP_EINVAL;
+        if (value > 1 && !ix->src) return SKIP_EUNSUPPORTED;
+        ix->refine = value > 1 ? (int)value : 0;
         return SKIP_OK;
     }
     return skip_corpus_set_option(ix->cent, option, value);

@@ -222,6 +222,11 @@ constexpr int kIvfCoarseMaxC = 4096;
 cudaError_t launch_ivf_probe_select(const float *scores, int R, int C, int nprobe, int64_t *probe_ids,
                                     float *probe_sc, cudaStream_t s);
 size_t ivfpq_scan_smem(int M, int nprobe);
+// Exact re-rank: per region, the ks shortlisted keys cand [R x ks] scored
+// exactly against the bf16 rows [N x d], the k best written as keys [R x k].
+constexpr int kIvfMaxRefine = 1024;  // shortlist length at most
+cudaError_t launch_ivf_refine(const uint16_t *rows, int64_t N, int d, const uint16_t *regions, int R,
+                              const uint64_t *cand, int ks, int k, uint64_t *out, cudaStream_t s);
 constexpr int kIvfMaxSplit = 8;  // most parts a region's probed blocks are cut into
 // Parts per region of the list scan: `requested` if > 0, else 1, 2 or 4,
 // doubling while twice the items still fit in the resident CTAs.

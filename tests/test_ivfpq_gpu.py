@@ -376,3 +376,67 @@ def test_full_size_build_and_recall():
           "%d/%d sampled list/code differences (near ties)"
           % (nprobe, spec.k_region, recall, spec.k_region * spec.centres / (nprobe * spec.N), nl, nc))
     assert recall > 10 * spec.k_region * spec.centres / (nprobe * spec.N)
+
+
+@pytest.mark.parametrize("refine", [2, 8])
+def test_refine_matches_oracle(refine):
+    """SKIP_OPT_IVF_REFINE = r: each region's best r k entries by s^ are
+    re-scored exactly; the GPU's lists must pass the per-region check against
+    the oracle's refined search (its shortlist re-ordered by exact fp64
+    scores), and the per-question merge the question check.  Regions whose
+    probed lists or whose shortlist end sit on a near tie in s^ (the GPU
+    computes s^ in fp32) are left out.  An index made by skip_ivfpq_load has
+    no corpus to re-rank against and refuses the option."""
+    corpus, regions, offsets, cent, cb = _small_inputs()
+    k, K, nprobe = SPEC.k_region, SPEC.K, 16
+    ks = refine * k
+    cn, ce, qn = synth.bf16_bits(corpus), synth.bf16_bits(cent), synth.bf16_bits(regions)
+    c = skip.skip_corpus_load(_t(corpus))
+    try:
+        ix = skip.skip_ivfpq_build(c, _t(cent), _t(cb))
+        ix.set_option(skip.SKIP_OPT_IVF_REFINE, refine)
+        g_ids, g_sc = skip.skip_ivfpq_search_regions(ix, _t(regions), nprobe, k)
+        q_ids, q_sc = skip.skip_ivfpq_search(ix, _t(regions), _t(offsets), nprobe, k, K)
+        assert skip.skip_ivfpq_sync_status(ix) == skip.SKIP_OK
+        off, ids, codes = (x.cpu().numpy() for x in skip.skip_ivfpq_lists(ix))
+        ix.free()
+        ix2 = skip.skip_ivfpq_load(_t(cent), _t(cb), _t(off), _t(ids, torch.int32), _t(codes))
+        with pytest.raises(skip.SkipError) as e:
+            ix2.set_option(skip.SKIP_OPT_IVF_REFINE, refine)
+        assert e.value.status == skip.SKIP_EUNSUPPORTED
+        ix2.free()
+    finally:
+        c.free()
+    g_ids, g_sc, q_ids, q_sc = (x.cpu().numpy() for x in (g_ids, g_sc, q_ids, q_sc))
+    lists, code_by_id = _lists_by_id(off, ids, codes, SPEC.N, cb.shape[0])
+    gidx = {"offsets": off, "ids": ids.astype(np.int64), "codes": code_by_id, "lists": lists}
+    # the oracle's shortlist one past ks (for the tie test) and its exact re-rank of all ks
+    s_ids, s_sc, _ = oracle.ivfpq_search(gidx, ce, cb.numpy(), qn, nprobe, ks + 1)
+    o_ids, o_sc = oracle.ivfpq_search_refine(gidx, ce, cb.numpy(), qn, nprobe, ks, ks, cn)
+    cs = np.sort(oracle.score_matrix(ce, qn), axis=1)[:, ::-1]
+    truths = checker.region_truths(o_ids, o_sc, k)
+    usable = []
+    for r in range(qn.shape[0]):
+        if cs[r, nprobe - 1] - cs[r, nprobe] <= PROBE_TIE:
+            continue
+        if s_ids[r, ks] >= 0 and s_sc[r, ks - 1] - s_sc[r, ks] <= PROBE_TIE:
+            continue
+        _, probs = checker.check_region(
+            g_ids[r], g_sc[r], truths[r],
+            extra_score=lambda i, r=r: float(oracle.scores_at(cn, qn, [r], [i])[0]))
+        assert not probs, (r, probs[:3])
+        usable.append(r)
+    assert len(usable) >= qn.shape[0] // 2
+    off_q = offsets.numpy()
+    o_m_ids, o_m_sc = oracle.merge(o_ids, o_sc, k, off_q, K + 1)
+    ok_r = set(usable)
+    for q in range(off_q.shape[0] - 1):
+        if not all(r in ok_r for r in range(off_q[q], off_q[q + 1])):
+            continue
+
+        def rescore(j, ids_, r0=off_q[q]):
+            return oracle.scores_at(cn, qn, np.full(len(ids_), r0 + j), ids_)
+        _, probs, _ = checker.check_question(q_ids[q], q_sc[q], o_m_ids[q], o_m_sc[q],
+                                             truths[off_q[q]:off_q[q + 1]], K, g_ids[off_q[q]:off_q[q + 1]],
+                                             rescore)
+        assert not probs, (q, probs[:3])

@@ -141,3 +141,27 @@ def test_search_matches_brute_force_with_random_codes(nprobe, k):
         want_sc[:len(top)] = s[top]
         np.testing.assert_array_equal(ids[r], want_ids)
         np.testing.assert_allclose(sc[r], want_sc, rtol=1e-12, atol=1e-12)
+
+
+def test_refine_with_every_list_and_entry_is_exact_mips():
+    """With every list probed and a shortlist as long as the corpus, the
+    exact re-rank sees every row: the result is exact MIPS (region_topk, a
+    separate code path), whatever the codebook.  With a shortlist of k the
+    re-rank keeps the ids of the plain search and only re-scores them."""
+    spec = synth.WorkloadSpec("ivf_refine", 33, 900, 64, "bf16", 4, (2, 2), 8, 16, "clustered", 16)
+    corpus, _, centres = synth.make_corpus(spec)
+    cent = synth.make_ivf_centroids(spec)
+    cb = synth.make_pq_codebook(spec, 16).numpy()
+    regions, _ = synth.make_regions(spec, centres)
+    cbits, ce, q = synth.bf16_bits(corpus), synth.bf16_bits(cent), synth.bf16_bits(regions)
+    idx = oracle.ivfpq_build(cbits, ce, cb)
+    k = spec.k_region
+    r_ids, r_sc = oracle.ivfpq_search_refine(idx, ce, cb, q, spec.centres, k, spec.N, cbits)
+    e_ids, e_sc = oracle.region_topk(cbits, q, k)
+    np.testing.assert_array_equal(r_ids, e_ids)
+    np.testing.assert_allclose(r_sc, e_sc, rtol=0, atol=1e-12)
+    p_ids, _, _ = oracle.ivfpq_search(idx, ce, cb, q, 4, k)
+    s_ids, s_sc = oracle.ivfpq_search_refine(idx, ce, cb, q, 4, k, k, cbits)
+    for a, b in zip(p_ids, s_ids):
+        assert set(a.tolist()) == set(b.tolist())
+    assert np.all(np.diff(s_sc, axis=1) <= 0)
