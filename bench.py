@@ -344,6 +344,24 @@ def ivfpq_report(args, spec, skip, c, ix, cent, reg_d, off_d, kernels, build_s, 
     }
 
 
+
+def timed_steps_flushed(step, steps, stream, dev):
+    """Device time of `steps` calls of step(), each bracketed by its own CUDA
+    events on `stream`, with L2 flushed between them (a 256 MB buffer larger
+    than the 129 MB L2 is rewritten outside the events), for inputs that would
+    otherwise stay in L2.  Returns (total ms, last output)."""
+    flush = torch.empty(256 << 20, dtype=torch.uint8, device=dev)
+    evs = [(torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)) for _ in range(steps)]
+    out = None
+    with torch.cuda.stream(stream):
+        for a, b in evs:
+            flush.fill_(1)
+            a.record(stream)
+            out = step()
+            b.record(stream)
+    torch.cuda.synchronize()
+    return sum(a.elapsed_time(b) for a, b in evs), out
+
 def run_bsca(args, spec, skip):
     """BSCA bench: one question per workload question (Q), 231 retained visual
     tokens (rho_v = 0.4 of 576), 16..32 verified chunks, d_p = d_h = 128,
@@ -368,14 +386,9 @@ def run_bsca(args, spec, skip):
     torch.cuda.synchronize()
     sampler.start()
     time.sleep(0.3)
-    e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
-    e0.record(stream)
-    for _ in range(args.steps):
-        out = step()
-    e1.record(stream)
-    torch.cuda.synchronize()
+    t_ms, out = timed_steps_flushed(step, args.steps, stream, dev)
     clocks = sampler.stop()
-    ms = max_over_ranks(e0.elapsed_time(e1), world)
+    ms = max_over_ranks(t_ms, world)
     if skip.skip_bsca_sync_status(h) != skip.SKIP_OK:
         raise SystemExit("bsca kernel status")
     # end to end: host projections in, the fused tokens out
@@ -406,7 +419,8 @@ def run_bsca(args, spec, skip):
         "vs_baseline": None, "dtype": "bf16 in, fp32 out", "data": "synthetic",
         "config": {"workload": "bsca_%dq_%dtok" % (Q, P), "questions_per_gpu": Q, "visual_tokens": P,
                    "chunks": "U{16..32}", "d_p": dp, "d_h": dh, "d_o": dout, "dbar": args.dbar,
-                   "l2": "output %.1f MB written per step" % (Nv * dout * 4 / 1e6)},
+                   "l2": "L2 flushed between timed steps (256 MB write outside the events); "
+                         "output %.1f MB written per step" % (Nv * dout * 4 / 1e6)},
         "roofline": {"bound": "hbm", "achieved": achieved, "peak": peaks["hbm_gbs"], "unit": "GB/s",
                      "frac": achieved / peaks["hbm_gbs"], "traffic": None, "kernel": "bsca step (3 kernels)",
                      "algorithmic_bytes_per_step": step_bytes, "peak_source": peaks["source"]},
@@ -461,14 +475,9 @@ def run_qvs(args, spec, skip):
     torch.cuda.synchronize()
     sampler.start()
     time.sleep(0.3)
-    e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
-    e0.record(stream)
-    for _ in range(args.steps):
-        step()
-    e1.record(stream)
-    torch.cuda.synchronize()
+    t_ms, _ = timed_steps_flushed(step, args.steps, stream, dev)
     clocks = sampler.stop()
-    ms = max_over_ranks(e0.elapsed_time(e1), world)
+    ms = max_over_ranks(t_ms, world)
     # end to end: host tokens in, kept indices and scores out
     tok_h, fq_h = tokens.pin_memory(), fq.pin_memory()
     idx_h = torch.empty(B, n, dtype=torch.int32).pin_memory()
@@ -499,9 +508,10 @@ def run_qvs(args, spec, skip):
         "higher_is_better": True, "scaling": "weak", "vs_baseline": None, "dtype": "bf16", "data": "synthetic",
         "config": {"workload": "qvs_%dx%dx%d" % (B, L, d), "images_per_gpu": B, "tokens": L, "d": d, "d_k": d,
                    "rho_v": args.rho_v, "kept": n,
-                   "l2": "tokens %.1f MB < L2: steady-state reads may hit L2" % (tok_bytes / 1e6)},
+                   "l2": "L2 flushed between timed steps (256 MB write outside the events); tokens %.1f MB"
+                         % (tok_bytes / 1e6)},
         "roofline": {"bound": "hbm", "achieved": achieved, "peak": peaks["hbm_gbs"], "unit": "GB/s",
-                     "frac": achieved / peaks["hbm_gbs"], "traffic": None, "kernel": "qvs step (3 kernels + 1 cuBLAS GEMM)",
+                     "frac": achieved / peaks["hbm_gbs"], "traffic": None, "kernel": "qvs step (3 kernels: split-K projected-query GEMM, logits, rank + gather)",
                      "algorithmic_bytes_per_step": step_bytes, "peak_source": peaks["source"]},
         "clocks": clocks,
         "e2e": {"value": B * world * args.steps / e2e_s, "unit": "images/s",
@@ -635,31 +645,43 @@ def main():
         raise SystemExit("warm-up kernel status: %s" % skip.skip_status_string(st))
     plan = skip.skip_last_plan(c)
 
-    # ---- timed region (device-resident inputs)
+    # ---- timed region (device-resident inputs).  Two passes of K steps:
+    # the first, with no events between the library's launches, gives the
+    # step time (`value`, `ms_per_step`); the second records CUDA events
+    # around every launch on the launching stream, for the per-kernel
+    # durations (roofline).  Events between launches cost the small
+    # workloads several microseconds a step (they break the programmatic
+    # overlap of consecutive launches), so they stay out of the first pass.
     timed = ix if ix is not None else c
-    timed.set_option(skip.SKIP_OPT_TIMING, 1)
-    (skip.skip_ivfpq_timing_report(ix) if ix is not None else skip.skip_timing_report(c))
+
+    def run_timed(with_events):
+        timed.set_option(skip.SKIP_OPT_TIMING, 1 if with_events else 0)
+        (skip.skip_ivfpq_timing_report(ix) if ix is not None else skip.skip_timing_report(c))
+        barrier(world)
+        torch.cuda.synchronize()
+        e0 = torch.cuda.Event(enable_timing=True)
+        e1 = torch.cuda.Event(enable_timing=True)
+        e0.record(stream)
+        for _ in range(args.steps):
+            step()
+        e1.record(stream)
+        torch.cuda.synchronize()
+        barrier(world)
+        rep = (skip.skip_ivfpq_timing_report(ix) if ix is not None else skip.skip_timing_report(c))
+        timed.set_option(skip.SKIP_OPT_TIMING, 0)
+        st = skip.skip_ivfpq_sync_status(ix) if ix is not None else skip.skip_sync_status(c)
+        if st != skip.SKIP_OK:
+            raise SystemExit("timed kernel status: %s" % skip.skip_status_string(st))
+        return e0.elapsed_time(e1), rep
+
     sampler = ClockSampler(torch.cuda.current_device())
-    barrier(world)
-    torch.cuda.synchronize()
     sampler.start()
     time.sleep(0.3)
-    e0 = torch.cuda.Event(enable_timing=True)
-    e1 = torch.cuda.Event(enable_timing=True)
-    e0.record(stream)
-    for _ in range(args.steps):
-        step()
-    e1.record(stream)
-    torch.cuda.synchronize()
+    ms_local, _ = run_timed(False)
     clocks = sampler.stop()
-    barrier(world)
-    ms_local = e0.elapsed_time(e1)
-    kernels = skip.skip_ivfpq_timing_report(ix) if ix is not None else skip.skip_timing_report(c)
-    timed.set_option(skip.SKIP_OPT_TIMING, 0)
-    st = skip.skip_ivfpq_sync_status(ix) if ix is not None else skip.skip_sync_status(c)
-    if st != skip.SKIP_OK:
-        raise SystemExit("timed kernel status: %s" % skip.skip_status_string(st))
+    ms_ev_local, kernels = run_timed(True)
     ms = max_over_ranks(ms_local, world)
+    ms_ev = max_over_ranks(ms_ev_local, world)
 
     # ---- end to end through the host-buffer entry point
     reg_h = regions.pin_memory()
@@ -739,6 +761,7 @@ def main():
     line = {
         "metric": METRIC, "value": total_q / secs, "unit": "queries/s", "n_gpus": world,
         "steps": args.steps, "warmup": args.warmup, "ms_per_step": ms / args.steps,
+        "ms_per_step_with_kernel_events": ms_ev / args.steps,
         "higher_is_better": True, "scaling": "weak", "vs_baseline": None, "dtype": "bf16",
         "data": "synthetic", "config": workload_config(spec, R, world),
         "corpus_gbs": corpus_bytes * world * args.steps / secs / 1e9,

@@ -13,6 +13,11 @@
 //   row-major with leading dimension ldd.  The SKV gate's per-question half
 //   of layer 1 is such a sum (its qbar and vbar column blocks of W1).
 //
+// Split K (splits > 1, for products with few output tiles): CTA z of a
+// tile takes the z-th share of the K slices (both products counted
+// together) and writes its partial tile to D + z * split_stride; the caller
+// sums the `splits` slabs (the bias goes into slab 0 only).
+//
 // One CTA computes one 128 x BN tile of D (BN = 64, or 32 when that leaves
 // too few tiles to occupy the GPU): warp 0 streams K slices of 64 elements
 // (128 bytes, 128-byte swizzle) of both operands into an eight-stage
@@ -22,6 +27,8 @@
 // 32 (w mod 4) .. + 31, i.e. rows of D) and store their rows, masked at the
 // M and N edges.  Every wait is bounded; a wait that gives up sets *err (if
 // given) and the roles drain their copies and MMAs before TMEM is freed.
+#include <algorithm>
+
 #include "skip_device.cuh"
 #include "skip_internal.h"
 
@@ -52,7 +59,7 @@ __global__ void __launch_bounds__(kThreads, 1)
     k_gemm_bf16_f32(const __grid_constant__ CUtensorMap ta, const __grid_constant__ CUtensorMap tb,
                     const __grid_constant__ CUtensorMap ta2, const __grid_constant__ CUtensorMap tb2, int M, int N,
                     int K, int K2, float alpha, const float *__restrict__ bias, float *__restrict__ D, int64_t ldd,
-                    int *err, uint64_t timeout_ns) {
+                    int64_t split_stride, int *err, uint64_t timeout_ns) {
     constexpr int kBBytes = GemmGeom<BN>::kBBytes;
     constexpr int kStageBytes = GemmGeom<BN>::kStageBytes;
     constexpr uint32_t kTmemCols = GemmGeom<BN>::kTmemCols;
@@ -64,7 +71,14 @@ __global__ void __launch_bounds__(kThreads, 1)
     const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
     const int m0 = blockIdx.x * 128, n0 = blockIdx.y * BN;
     const int KB1 = (K + 63) / 64;
-    const int KB = KB1 + (K2 + 63) / 64;
+    const int KBall = KB1 + (K2 + 63) / 64;
+    // this CTA's share of the K slices [kb0, kb0 + KB)
+    const int kb0 = (int)((int64_t)blockIdx.z * KBall / gridDim.z);
+    const int KB = (int)((int64_t)(blockIdx.z + 1) * KBall / gridDim.z) - kb0;
+    if (blockIdx.z > 0) {
+        D += (int64_t)blockIdx.z * split_stride;
+        bias = nullptr;
+    }
     constexpr uint32_t kIdesc = idesc_bf16_f32(128, BN);
 
     if (threadIdx.x == 0) {
@@ -105,8 +119,9 @@ __global__ void __launch_bounds__(kThreads, 1)
                 }
                 const uint32_t fb = smem_addr(&sh->full[s]);
                 mbar_arrive_expect_tx(fb, kStageBytes);
-                const bool first = kb < KB1;
-                const int x = (first ? kb : kb - KB1) * 64;
+                const int kg = kb0 + kb;  // slice index over both products
+                const bool first = kg < KB1;
+                const int x = (first ? kg : kg - KB1) * 64;
                 tma_load_2d(smem_addr(sA + s * kABytes), first ? &ta : &ta2, fb, x, m0);
                 tma_load_2d(smem_addr(sB + s * kBBytes), first ? &tb : &tb2, fb, x, n0);
                 ++issued;
@@ -153,6 +168,11 @@ __global__ void __launch_bounds__(kThreads, 1)
                 uint32_t v[32];
                 tmem_ld_32x32b_x32(tmem + ((uint32_t)(sub * 32) << 16) + (uint32_t)c, v);
                 tmem_ld_wait(v);
+                if (KB == 0) {
+                    // an empty share of K (more splits than slices): zeros
+#pragma unroll
+                    for (int j = 0; j < 32; ++j) v[j] = 0u;
+                }
                 if (bias) {
 #pragma unroll
                     for (int j = 0; j < 32; ++j) {
@@ -199,14 +219,14 @@ size_t gemm_smem_bytes() {
 
 template <int BN>
 cudaError_t launch_bn(const CUtensorMap &ta, const CUtensorMap &tb, const CUtensorMap &ta2, const CUtensorMap &tb2,
-                      int M, int N, int K, int K2, float alpha, const float *bias, float *D, int64_t ldd, int *err,
-                      uint64_t timeout_ns, cudaStream_t s) {
+                      int M, int N, int K, int K2, float alpha, const float *bias, float *D, int64_t ldd, int splits,
+                      int64_t split_stride, int *err, uint64_t timeout_ns, cudaStream_t s) {
     const size_t smem = gemm_smem_bytes<BN>();
     cudaError_t e = cudaFuncSetAttribute(k_gemm_bf16_f32<BN>, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
     if (e != cudaSuccess) return e;
-    dim3 grid((unsigned)((M + 127) / 128), (unsigned)((N + BN - 1) / BN));
-    k_gemm_bf16_f32<BN><<<grid, kThreads, smem, s>>>(ta, tb, ta2, tb2, M, N, K, K2, alpha, bias, D, ldd, err,
-                                                     timeout_ns);
+    dim3 grid((unsigned)((M + 127) / 128), (unsigned)((N + BN - 1) / BN), (unsigned)splits);
+    k_gemm_bf16_f32<BN><<<grid, kThreads, smem, s>>>(ta, tb, ta2, tb2, M, N, K, K2, alpha, bias, D, ldd,
+                                                     split_stride, err, timeout_ns);
     return cudaGetLastError();
 }
 
@@ -217,22 +237,33 @@ int gemm_tile_n(int M, int N, int sms) {
     return tiles64 * 2 <= sms ? 32 : 64;
 }
 
+int gemm_splits(int M, int N, int K, int tile_n, int sms) {
+    const int64_t tiles = (int64_t)((M + 127) / 128) * ((N + tile_n - 1) / tile_n);
+    const int kb = (K + 63) / 64;
+    // at least two K slices per split; no more splits than fill the SMs once
+    return (int)std::max<int64_t>(1, std::min<int64_t>(std::min<int64_t>(kb / 2, 16), sms / std::max<int64_t>(1, tiles)));
+}
+
 cudaError_t launch_gemm2_bf16_f32(const CUtensorMap &ta, const CUtensorMap &tb, const CUtensorMap *ta2,
                                   const CUtensorMap *tb2, int tile_n, int M, int N, int K, int K2, float alpha,
                                   const float *bias, float *D, int64_t ldd, int *err, uint64_t timeout_ns,
-                                  cudaStream_t s) {
+                                  cudaStream_t s, int splits, int64_t split_stride) {
     if (M <= 0 || N <= 0) return cudaSuccess;
     if (K <= 0 || (K & 7) != 0 || K2 < 0 || (K2 & 7) != 0 || (K2 > 0 && (!ta2 || !tb2))) return cudaErrorInvalidValue;
+    if (splits < 1 || splits > 64 || (splits > 1 && split_stride < (int64_t)M * ldd)) return cudaErrorInvalidValue;
     const CUtensorMap &a2 = K2 > 0 ? *ta2 : ta, &b2 = K2 > 0 ? *tb2 : tb;
-    if (tile_n == 32) return launch_bn<32>(ta, tb, a2, b2, M, N, K, K2, alpha, bias, D, ldd, err, timeout_ns, s);
-    if (tile_n == 64) return launch_bn<64>(ta, tb, a2, b2, M, N, K, K2, alpha, bias, D, ldd, err, timeout_ns, s);
+    if (tile_n == 32)
+        return launch_bn<32>(ta, tb, a2, b2, M, N, K, K2, alpha, bias, D, ldd, splits, split_stride, err, timeout_ns, s);
+    if (tile_n == 64)
+        return launch_bn<64>(ta, tb, a2, b2, M, N, K, K2, alpha, bias, D, ldd, splits, split_stride, err, timeout_ns, s);
     return cudaErrorInvalidValue;
 }
 
 cudaError_t launch_gemm_bf16_f32(const CUtensorMap &ta, const CUtensorMap &tb, int tile_n, int M, int N, int K,
-                                 float alpha, float *D, int64_t ldd, int *err, uint64_t timeout_ns, cudaStream_t s) {
+                                 float alpha, float *D, int64_t ldd, int *err, uint64_t timeout_ns, cudaStream_t s,
+                                 int splits, int64_t split_stride) {
     return launch_gemm2_bf16_f32(ta, tb, nullptr, nullptr, tile_n, M, N, K, 0, alpha, nullptr, D, ldd, err, timeout_ns,
-                                 s);
+                                 s, splits, split_stride);
 }
 
 }  // namespace skipk

@@ -23,9 +23,10 @@
 //
 // Epilogue: lane = corpus row, so for each query the 32 rows of a warp are
 // compared with the query's filter at once (a ballot); lane q owns the
-// running top-k set of query q for its warp's rows (an unsorted set with its
-// minimum tracked, in shared memory) and inserts the ballot's survivors in
-// increasing row (= id) order.  Eight epilogue warps in two sets of four
+// running top-k set of query q for its warp's rows (bf16 with k <= 16: a
+// sorted array in registers; else an unsorted set with its minimum tracked,
+// in shared memory) and inserts the ballot's survivors in increasing row
+// (= id) order.  Eight epilogue warps in two sets of four
 // drain the two TMEM accumulators in turn (set j takes the tiles that land
 // in accumulator j), so that the survivor work of one tile overlaps the
 // ballots of the next.  A query's filter is the largest of its own set's
@@ -70,7 +71,70 @@ struct __align__(8) LatShared {
     float filt[kEpiWarps][32];  // ... and the filter its next ballots use (strict compare)
 };
 
-template <bool FP8>
+// Running top-k of one query in registers (k <= KM): ascending, a[0] the
+// k-th best key (0 while fewer than k keys are held), a[i] = ~0 for i >= k.
+// Inserting x drops a[0]: a[i] <- max(a[i], min(x, a[i + 1])) (a[KM] = ~0)
+// shifts the keys below x down one place and puts x in its slot; with
+// x <= a[0] every a[i] stays as it is, so the network runs unconditionally
+// on max(x, a[0]).  Straight-line code on registers: no shared-memory
+// round trips per key.
+template <int KM>
+__device__ __forceinline__ void regset_insert(uint64_t (&a)[KM], uint64_t x) {
+    x = x > a[0] ? x : a[0];
+#pragma unroll
+    for (int i = 0; i < KM - 1; ++i) {
+        const uint64_t t = x < a[i + 1] ? x : a[i + 1];
+        a[i] = a[i] > t ? a[i] : t;
+    }
+    a[KM - 1] = a[KM - 1] > x ? a[KM - 1] : x;
+}
+
+// The k-th largest (k <= 16) of the 16 pair maxima max(s_j, s_{j+16}) over
+// the rows j of mask m (others -inf); s_j = col[33 j].  The pair maxima are
+// sorted descending by a bitonic network on sixteen named registers (an
+// array here was placed in local memory).
+#define CED(a, b) { const float x_ = a, y_ = b; a = fmaxf(x_, y_); b = fminf(x_, y_); }
+#define CEA(a, b) { const float x_ = a, y_ = b; a = fminf(x_, y_); b = fmaxf(x_, y_); }
+__device__ __forceinline__ float pair_max_bound(const float *col, uint32_t m, int k) {
+    const float ninf = -__int_as_float(0x7f800000);
+#define PM(j) const float a##j = (m >> j) & 1u ? col[j * 33] : ninf, b##j = (m >> (j + 16)) & 1u ? col[(j + 16) * 33] : ninf; \
+    float g##j = fmaxf(a##j, b##j);
+    PM(0) PM(1) PM(2) PM(3) PM(4) PM(5) PM(6) PM(7)
+    PM(8) PM(9) PM(10) PM(11) PM(12) PM(13) PM(14) PM(15)
+#undef PM
+    CED(g0, g1); CEA(g2, g3); CED(g4, g5); CEA(g6, g7);
+    CED(g8, g9); CEA(g10, g11); CED(g12, g13); CEA(g14, g15);
+    CED(g0, g2); CED(g1, g3); CEA(g4, g6); CEA(g5, g7);
+    CED(g8, g10); CED(g9, g11); CEA(g12, g14); CEA(g13, g15);
+    CED(g0, g1); CED(g2, g3); CEA(g4, g5); CEA(g6, g7);
+    CED(g8, g9); CED(g10, g11); CEA(g12, g13); CEA(g14, g15);
+    CED(g0, g4); CED(g1, g5); CED(g2, g6); CED(g3, g7);
+    CEA(g8, g12); CEA(g9, g13); CEA(g10, g14); CEA(g11, g15);
+    CED(g0, g2); CED(g1, g3); CED(g4, g6); CED(g5, g7);
+    CEA(g8, g10); CEA(g9, g11); CEA(g12, g14); CEA(g13, g15);
+    CED(g0, g1); CED(g2, g3); CED(g4, g5); CED(g6, g7);
+    CEA(g8, g9); CEA(g10, g11); CEA(g12, g13); CEA(g14, g15);
+    CED(g0, g8); CED(g1, g9); CED(g2, g10); CED(g3, g11);
+    CED(g4, g12); CED(g5, g13); CED(g6, g14); CED(g7, g15);
+    CED(g0, g4); CED(g1, g5); CED(g2, g6); CED(g3, g7);
+    CED(g8, g12); CED(g9, g13); CED(g10, g14); CED(g11, g15);
+    CED(g0, g2); CED(g1, g3); CED(g4, g6); CED(g5, g7);
+    CED(g8, g10); CED(g9, g11); CED(g12, g14); CED(g13, g15);
+    CED(g0, g1); CED(g2, g3); CED(g4, g5); CED(g6, g7);
+    CED(g8, g9); CED(g10, g11); CED(g12, g13); CED(g14, g15);
+    float T = g0;
+#define PICK(j) T = (j == k - 1) ? g##j : T;
+    PICK(1) PICK(2) PICK(3) PICK(4) PICK(5) PICK(6) PICK(7) PICK(8)
+    PICK(9) PICK(10) PICK(11) PICK(12) PICK(13) PICK(14) PICK(15)
+#undef PICK
+    return T;
+}
+#undef CED
+#undef CEA
+
+// KM > 0: the epilogue keeps each query's set in registers (k <= KM);
+// KM == 0: in shared memory (any k).
+template <bool FP8, int KM>
 __global__ void __launch_bounds__(kThreads, 1)
     k_latency_score_topk(const __grid_constant__ CUtensorMap ta, const __grid_constant__ CUtensorMap tb,
                          const LatParams p) {
@@ -230,6 +294,9 @@ __global__ void __launch_bounds__(kThreads, 1)
             // distinct corpus rows (of this chunk or an earlier one), so it
             // bounds the k-th best score over the whole corpus from below.
             RowTopK top;
+            uint64_t ra[KM > 0 ? KM : 1];
+#pragma unroll
+            for (int i = 0; i < (KM > 0 ? KM : 1); ++i) ra[i] = i < k ? 0ull : ~0ull;
             float thr = kNegInf;  // own set's k-th score (strict: later rows lose ties)
             float cthr = kNegInf; // filter: s > cthr  <=>  s > thr and s >= every bound from elsewhere
             uint32_t published = 0;
@@ -244,7 +311,8 @@ __global__ void __launch_bounds__(kThreads, 1)
                 }
                 tc_fence_after();
                 if (lane < R) {
-                    const uint32_t mine = top.n == k ? ord_of_score(thr) : 0u;
+                    const bool full = KM > 0 ? ra[0] != 0ull : top.n == k;
+                    const uint32_t mine = full ? ord_of_score(thr) : 0u;
                     if (mine > published) {
                         atomicMax(p.tau + lane, mine);
                         published = mine;
@@ -307,16 +375,48 @@ __global__ void __launch_bounds__(kThreads, 1)
                     __syncwarp();
                     uint32_t mine_m = select32(m, lane);
                     if (lane < R) {
-                        const float below_other = cthr > thr ? cthr : kNegInf;  // the part of cthr from elsewhere
+                        float below_other = cthr > thr ? cthr : kNegInf;  // the part of cthr from elsewhere
+                        if constexpr (KM > 0) {
+                            if (__popc(mine_m) > KM) {
+                                // Many survivors (a warp's first tile of a chunk): a bound
+                                // from the tile itself.  The k-th largest of the 16 pair
+                                // maxima max(s_j, s_{j+16}) is met or beaten by k distinct
+                                // rows, so a score below it cannot reach the warp's top k;
+                                // about k + 2 rows of 32 pass it instead of all 32.  (The
+                                // lanes insert in step, so a round costs the same whether
+                                // one lane or all insert: it is the rounds that count.)
+                                const float T = pair_max_bound(Sw + lane, mine_m, k);
+                                if (T > kNegInf) {
+                                    below_other = fmaxf(below_other, float_below(T));
+                                    cthr = fmaxf(cthr, below_other);
+                                    // Drop the rows below the bound from the mask: the
+                                    // insert loop below runs as many rounds as the lane
+                                    // with the most rows left, all lanes in step.
+                                    uint32_t keep = 0;
+#pragma unroll
+                                    for (int j = 0; j < 32; ++j) keep |= (Sw[j * 33 + lane] > cthr ? 1u : 0u) << j;
+                                    mine_m &= keep;
+                                }
+                            }
+                        }
                         while (mine_m) {
                             const int l = __ffs(mine_m) - 1;
                             mine_m &= mine_m - 1;
                             const float sl = Sw[l * 33 + lane];
                             if (sl > cthr) {
-                                topk_add(Lw + (size_t)lane * k, 1, k, top, make_key(sl, (uint32_t)(rowbase + l)));
-                                if (top.n == k) {
-                                    thr = key_score(top.min_key);
-                                    cthr = fmaxf(thr, below_other);
+                                const uint64_t key = make_key(sl, (uint32_t)(rowbase + l));
+                                if constexpr (KM > 0) {
+                                    regset_insert<KM>(ra, key);
+                                    if (ra[0] != 0ull) {
+                                        thr = key_score(ra[0]);
+                                        cthr = fmaxf(thr, below_other);
+                                    }
+                                } else {
+                                    topk_add(Lw + (size_t)lane * k, 1, k, top, key);
+                                    if (top.n == k) {
+                                        thr = key_score(top.min_key);
+                                        cthr = fmaxf(thr, below_other);
+                                    }
                                 }
                             }
                         }
@@ -326,12 +426,19 @@ __global__ void __launch_bounds__(kThreads, 1)
                     __syncwarp();
                 }
             }
-            // Chunk done: each warp sorts its sets (lane q: query q), then
-            // lane q of warp q mod 8 merges the eight sorted sets of query q
-            // into the chunk's list -- one lane per query, all queries at once,
-            // no warp-wide chains (the two hand-offs between the epilogue
-            // warps are bounded waits, like every other wait).
-            if (lane < R) {
+            // Chunk done: each warp writes its sets sorted (lane q: query q),
+            // then lane q of warp q mod 8 merges the eight sorted sets of
+            // query q into the chunk's list (a ranking of every key by binary
+            // searches in the other sets, all 256 threads at once, measured
+            // six times slower).  The two hand-offs between the epilogue
+            // warps are bounded waits, like every other wait.
+            if (KM > 0 && lane < R) {
+                // descending into the warp's slot of query `lane`
+                uint64_t *Lq = Lw + (size_t)lane * k;
+#pragma unroll
+                for (int i = 0; i < (KM > 0 ? KM : 1); ++i)
+                    if (i < k) Lq[k - 1 - i] = ra[i];
+            } else if (lane < R) {
                 uint64_t *Lq = Lw + (size_t)lane * k;
                 for (int t = top.n; t < k; ++t) Lq[t] = 0ull;
                 if (k <= 16)
@@ -349,14 +456,14 @@ __global__ void __launch_bounds__(kThreads, 1)
                 if (ok && q < R) {
                     uint64_t *out = p.lists + ((int64_t)v * R + q) * k;
                     // heads of the eight sorted sets of query q
-                    const uint64_t *Ls[kEpiWarps];
+                    const uint64_t *Lq0 = slists + (size_t)q * k;  // warp w's set at Lq0 + w * R * k
+                    const size_t wstride = (size_t)R * k;
                     uint64_t h[kEpiWarps];
                     int at[kEpiWarps];
 #pragma unroll
                     for (int w = 0; w < kEpiWarps; ++w) {
-                        Ls[w] = slists + ((size_t)w * R + q) * k;
                         at[w] = 0;
-                        h[w] = Ls[w][0];
+                        h[w] = Lq0[w * wstride];
                     }
                     for (int t = 0; t < k; ++t) {
                         uint64_t best = h[0];
@@ -372,7 +479,7 @@ __global__ void __launch_bounds__(kThreads, 1)
                         for (int w = 0; w < kEpiWarps; ++w)
                             if (w == bw) {
                                 ++at[w];
-                                h[w] = (best != 0ull && at[w] < k) ? Ls[w][at[w]] : 0ull;
+                                h[w] = (best != 0ull && at[w] < k) ? Lq0[w * wstride + at[w]] : 0ull;
                             }
                     }
                 }
@@ -472,7 +579,14 @@ cudaError_t launch_split_queries(const uint16_t *regions, int R, int d, uint8_t 
 cudaError_t launch_latency(bool fp8, const CUtensorMap &ta, const CUtensorMap &tb, const LatParams &p, int grid,
                            cudaStream_t s) {
     const size_t smem = smem_bytes(p.Npad, p.slices, p.stages, p.R, p.k);
-    auto kern = fp8 ? k_latency_score_topk<true> : k_latency_score_topk<false>;
+    // e4m3: the sets stay in shared memory (the three accumulator groups
+    // leave no registers for them: a register set spilled and ran slower).
+    auto kern = fp8 ? k_latency_score_topk<true, 0>
+                    : (p.k <= 4    ? k_latency_score_topk<false, 4>
+                       : p.k <= 8  ? k_latency_score_topk<false, 8>
+                       : p.k <= 12 ? k_latency_score_topk<false, 12>
+                       : p.k <= 16 ? k_latency_score_topk<false, 16>
+                                   : k_latency_score_topk<false, 0>);
     cudaError_t e = cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
     if (e != cudaSuccess) return e;
     kern<<<grid, kThreads, smem, s>>>(ta, tb, p);

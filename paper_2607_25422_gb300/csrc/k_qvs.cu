@@ -8,12 +8,18 @@
 //
 //  k_gemm        W_v^T f_q / sqrt(d_k) for all images at once: the library's
 //                tensor-core GEMM (k_gemm.cu) on F_q [B x d_k] and the handle's
-//                copy of W_v^T [d x d_k] (k_transpose_bf16, once per handle).
-//  k_qvs_logits  u = that + w_b in shared memory and c by one warp; one warp
-//                per four tokens at a time, 16-byte loads.
-//  k_qvs_select  per image: (logit, ~index) keys sorted descending in shared
-//                memory, the first n kept with their sigmoid scores.
-//  k_qvs_gather  (optional) the kept token rows copied out, a warp per row.
+//                copy of W_v^T [d x d_k] (k_transpose_bf16, once per handle),
+//                K split over up to four CTAs per tile (partial slabs).
+//  k_qvs_logits  u = the slabs' sum + w_b in shared memory, c by all warps;
+//                one warp per eight tokens at a time, 16-byte loads.
+//  k_qvs_rank    rank of every token = the number of the image's keys
+//                (logit, ~index) above its own, counted against all the
+//                image's keys in shared memory (many blocks per image, a warp
+//                per four tokens); a token with rank < n is written at its
+//                rank with its sigmoid score, and (optionally) its row copied
+//                out by the same warp.  The same order as a descending sort.
+// The logits and rank kernels are programmatic dependents of the kernel
+// before them: they launch while it drains and wait for its results.
 #include <cuda_bf16.h>
 #include <cuda_runtime.h>
 
@@ -26,27 +32,38 @@ namespace skipk {
 namespace {
 
 constexpr int kLogThreads = 256;
+constexpr int kLogTok = 8;  // tokens per warp in flight
 
 __global__ void __launch_bounds__(kLogThreads) k_qvs_logits(const QvsParams p) {
     extern __shared__ float us[];  // [d]
-    __shared__ float cbs;
+    __shared__ float cpart[kLogThreads / 32];
     const int b = blockIdx.y;
     const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
-    // u = W_v^T f_q / sqrt(d_k) (the library GEMM) + w_b; c = <f_q, b_v> / sqrt(d_k)
-    for (int t = threadIdx.x; t < p.d; t += kLogThreads) us[t] = p.u[(int64_t)b * p.d + t] + p.wb[t];
-    if (warp == 0) {
+    grid_dep_wait();
+    // u = W_v^T f_q / sqrt(d_k) (the GEMM's partial slabs) + w_b; c = <f_q, b_v> / sqrt(d_k)
+    const int64_t slab = (int64_t)p.B * p.d;
+    for (int t = threadIdx.x; t < p.d; t += kLogThreads) {
+        float v = p.wb[t];
+        for (int z = 0; z < p.u_splits; ++z) v += p.u[z * slab + (int64_t)b * p.d + t];
+        us[t] = v;
+    }
+    {
+        // c = <f_q, b_v> / sqrt(d_k): every warp a share, summed in shared memory
         const __nv_bfloat16 *fq = reinterpret_cast<const __nv_bfloat16 *>(p.fq) + (int64_t)b * p.dk;
         float c = 0.f;
-        for (int k = lane; k < p.dk; k += 32) c = fmaf(__bfloat162float(fq[k]), p.bv[k], c);
+        for (int k = threadIdx.x; k < p.dk; k += kLogThreads) c = fmaf(__bfloat162float(fq[k]), p.bv[k], c);
 #pragma unroll
         for (int o = 16; o; o >>= 1) c += __shfl_xor_sync(0xFFFFFFFFu, c, o);
-        if (lane == 0) cbs = c * rsqrtf((float)p.dk);
+        if (lane == 0) cpart[warp] = c;
     }
     __syncthreads();
     const int nw = p.d / 8;  // 16-byte words per token
-    const float cb = cbs;
-    // Four tokens per warp at a time: their loads are issued together.
-    constexpr int kT = 4;
+    float cb = 0.f;
+#pragma unroll
+    for (int w = 0; w < kLogThreads / 32; ++w) cb += cpart[w];
+    cb *= rsqrtf((float)p.dk);
+    // kLogTok tokens per warp at a time: their loads are issued together.
+    constexpr int kT = kLogTok;
     const int wstep = gridDim.x * (kLogThreads / 32);
     for (int i0 = blockIdx.x * (kLogThreads / 32) + warp; i0 < p.L; i0 += kT * wstep) {
         float s[kT];
@@ -84,91 +101,62 @@ __global__ void __launch_bounds__(kLogThreads) k_qvs_logits(const QvsParams p) {
     }
 }
 
-constexpr int kSelThreads = 512;
+constexpr int kRankWarps = 8;
+constexpr int kRankTok = 4;  // tokens per warp
 
-// One bitonic step on a register pair held by lanes (lane, lane ^ j): the
-// lower lane keeps the larger key when `desc`, else the smaller.
-__device__ __forceinline__ uint64_t bitonic_lane_step(uint64_t v, int pos, int j, bool desc) {
-    const uint64_t o = __shfl_xor_sync(0xFFFFFFFFu, v, j);
-    const bool lower = (pos & j) == 0;
-    const bool keep_max = lower == desc;
-    return keep_max ? (v > o ? v : o) : (v < o ? v : o);
-}
-
-// Sorts keys[0, n) descending (n a power of two, 64 <= n <= kQvsMaxL, block of
-// kSelThreads threads).  Strides below 32 run inside warps on registers,
-// one key per lane; larger strides through shared memory.
-__device__ void bitonic_desc(uint64_t *keys, int n) {
-    const int lane = threadIdx.x & 31;
-    for (int size = 2; size <= n; size <<= 1) {
-        int stride = size >> 1;
-        for (; stride >= 32; stride >>= 1) {
-            for (int t = threadIdx.x; t < n / 2; t += kSelThreads) {
-                const int lo = 2 * t - (t & (stride - 1));
-                const int hi = lo + stride;
-                const bool desc = (lo & size) == 0;
-                const uint64_t a = keys[lo], b = keys[hi];
-                if ((a < b) == desc) {
-                    keys[lo] = b;
-                    keys[hi] = a;
+__global__ void __launch_bounds__(32 * kRankWarps) k_qvs_rank(const QvsParams p) {
+    extern __shared__ uint64_t keys[];  // [L]: (ord(logit), ~index) of every token of the image
+    const int b = blockIdx.y;
+    const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+    grid_dep_wait();
+    const float *lg = p.logits + (int64_t)b * p.L;
+    for (int i = threadIdx.x; i < p.L; i += 32 * kRankWarps)
+        keys[i] = ((uint64_t)ord_of_score(lg[i]) << 32) | (uint32_t)(0xFFFFFFFFu - i);
+    __syncthreads();
+    const int i0 = (blockIdx.x * kRankWarps + warp) * kRankTok;
+    if (i0 >= p.L) return;
+    uint64_t mine[kRankTok];
+    int cnt[kRankTok];
+#pragma unroll
+    for (int t = 0; t < kRankTok; ++t) {
+        mine[t] = i0 + t < p.L ? keys[i0 + t] : ~0ull;  // past L: rank 0 of nothing, never written
+        cnt[t] = 0;
+    }
+    // Keys are distinct (the index is in the low word), so a token's rank is
+    // its position in the descending order.
+    for (int j = lane; j < p.L; j += 32) {
+        const uint64_t kj = keys[j];
+#pragma unroll
+        for (int t = 0; t < kRankTok; ++t) cnt[t] += kj > mine[t] ? 1 : 0;
+    }
+#pragma unroll
+    for (int t = 0; t < kRankTok; ++t) cnt[t] = __reduce_add_sync(0xFFFFFFFFu, cnt[t]);
+    const int nw = p.d / 8;  // 16-byte words per token
+#pragma unroll
+    for (int t = 0; t < kRankTok; ++t) {
+        const int i = i0 + t, r = cnt[t];
+        if (i >= p.L || r >= p.n) continue;  // warp-uniform
+        if (lane == 0) {
+            p.out_idx[(int64_t)b * p.n + r] = i;
+            p.out_score[(int64_t)b * p.n + r] = 1.f / (1.f + expf(-score_of_ord((uint32_t)(mine[t] >> 32))));
+        }
+        if (p.out_tokens) {
+            const uint4 *src = reinterpret_cast<const uint4 *>(p.tokens) + ((int64_t)b * p.L + i) * nw;
+            uint4 *dst = reinterpret_cast<uint4 *>(p.out_tokens) + ((int64_t)b * p.n + r) * nw;
+            // four 16-byte words per lane in flight
+            for (int w0 = 0; w0 < nw; w0 += 128) {
+                uint4 x[4];
+#pragma unroll
+                for (int u = 0; u < 4; ++u) {
+                    const int w = w0 + lane + 32 * u;
+                    if (w < nw) x[u] = __ldg(src + w);
+                }
+#pragma unroll
+                for (int u = 0; u < 4; ++u) {
+                    const int w = w0 + lane + 32 * u;
+                    if (w < nw) dst[w] = x[u];
                 }
             }
-            __syncthreads();
-        }
-        // strides 16 .. 1: each warp sorts its 32-key runs in registers
-        for (int base = (threadIdx.x & ~31); base < n; base += kSelThreads) {
-            const int pos = base + lane;
-            uint64_t v = keys[pos];
-            const bool desc = (pos & size) == 0;
-            for (int j = stride; j > 0; j >>= 1) v = bitonic_lane_step(v, pos, j, desc);
-            keys[pos] = v;
-        }
-        __syncthreads();
-    }
-}
-
-__global__ void __launch_bounds__(kSelThreads) k_qvs_select(const QvsParams p) {
-    __shared__ uint64_t keys[kQvsMaxL];
-    const int b = blockIdx.x;
-    int Lp = 64;
-    while (Lp < p.L) Lp <<= 1;
-    for (int i = threadIdx.x; i < Lp; i += kSelThreads) {
-        uint64_t key = 0;
-        if (i < p.L) key = ((uint64_t)ord_of_score(p.logits[(int64_t)b * p.L + i]) << 32) | (uint32_t)(0xFFFFFFFFu - i);
-        keys[i] = key;
-    }
-    __syncthreads();
-    bitonic_desc(keys, Lp);
-    for (int r = threadIdx.x; r < p.n; r += kSelThreads) {
-        const uint64_t key = keys[r];
-        p.out_idx[(int64_t)b * p.n + r] = (int32_t)(0xFFFFFFFFu - (uint32_t)key);
-        p.out_score[(int64_t)b * p.n + r] = 1.f / (1.f + expf(-score_of_ord((uint32_t)(key >> 32))));
-    }
-}
-
-// Kept token rows: one block per (rank, image), 16-byte copies.
-constexpr int kGatherWarps = 8;
-
-__global__ void __launch_bounds__(32 * kGatherWarps) k_qvs_gather(const QvsParams p) {
-    const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
-    const int r = blockIdx.x * kGatherWarps + warp, b = blockIdx.y;
-    if (r >= p.n) return;
-    const int i = p.out_idx[(int64_t)b * p.n + r];
-    const int nw = p.d / 8;
-    const uint4 *src = reinterpret_cast<const uint4 *>(p.tokens) + ((int64_t)b * p.L + i) * nw;
-    uint4 *dst = reinterpret_cast<uint4 *>(p.out_tokens) + ((int64_t)b * p.n + r) * nw;
-    // four 16-byte words per lane in flight
-    for (int w0 = 0; w0 < nw; w0 += 128) {
-        uint4 x[4];
-#pragma unroll
-        for (int u = 0; u < 4; ++u) {
-            const int w = w0 + lane + 32 * u;
-            if (w < nw) x[u] = __ldg(src + w);
-        }
-#pragma unroll
-        for (int u = 0; u < 4; ++u) {
-            const int w = w0 + lane + 32 * u;
-            if (w < nw) dst[w] = x[u];
         }
     }
 }
@@ -202,22 +190,41 @@ cudaError_t launch_transpose_bf16(const uint16_t *w, int rows, int cols, uint16_
     return cudaGetLastError();
 }
 
+// Launch as the programmatic dependent of the previous kernel in the stream.
+template <typename... Args>
+cudaError_t launch_dependent(void (*kern)(Args...), dim3 grid, int threads, size_t smem, cudaStream_t s,
+                             Args... args) {
+    cudaLaunchConfig_t cfg = {};
+    cfg.gridDim = grid;
+    cfg.blockDim = dim3((unsigned)threads);
+    cfg.dynamicSmemBytes = smem;
+    cfg.stream = s;
+    cudaLaunchAttribute attr[1];
+    attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+    attr[0].val.programmaticStreamSerializationAllowed = 1;
+    cfg.attrs = attr;
+    cfg.numAttrs = 1;
+    return cudaLaunchKernelEx(&cfg, kern, args...);
+}
+
 cudaError_t launch_qvs_logits(const QvsParams &p, int sms, cudaStream_t s) {
     if (p.B == 0) return cudaSuccess;
-    // Enough blocks for about four per SM; each covers a strided share of an image's tokens.
-    const int per_img = std::max(1, std::min((p.L + 7) / 8, (4 * sms + p.B - 1) / p.B));
+    if (p.u_splits < 1) return cudaErrorInvalidValue;
+    // Enough blocks that every warp loads its tokens in one round (kLogTok
+    // per warp), but no more than about four per SM: each block first builds
+    // u (the GEMM's slabs summed) and c, so more blocks per image repeat that
+    // work (at 18 blocks per image, 4 tokens per warp, the step was 8% slower).
+    const int one_round = (p.L + kLogTok * (kLogThreads / 32) - 1) / (kLogTok * (kLogThreads / 32));
+    const int per_img = std::max(1, std::min(one_round, (4 * sms + p.B - 1) / p.B));
     dim3 grid((unsigned)per_img, (unsigned)p.B);
-    k_qvs_logits<<<grid, kLogThreads, (size_t)p.d * sizeof(float), s>>>(p);
-    return cudaGetLastError();
+    return launch_dependent(k_qvs_logits, grid, kLogThreads, (size_t)p.d * sizeof(float), s, p);
 }
 
 cudaError_t launch_qvs_select(const QvsParams &p, cudaStream_t s) {
-    if (p.B == 0) return cudaSuccess;
-    k_qvs_select<<<p.B, kSelThreads, 0, s>>>(p);
-    cudaError_t e = cudaGetLastError();
-    if (e != cudaSuccess || !p.out_tokens || p.n == 0) return e;
-    k_qvs_gather<<<dim3((unsigned)((p.n + kGatherWarps - 1) / kGatherWarps), (unsigned)p.B), 32 * kGatherWarps, 0, s>>>(p);
-    return cudaGetLastError();
+    if (p.B == 0 || p.L == 0) return cudaSuccess;
+    const size_t smem = (size_t)p.L * sizeof(uint64_t);  // <= 32 KB: no opt-in needed
+    const int per_img = (p.L + kRankWarps * kRankTok - 1) / (kRankWarps * kRankTok);
+    return launch_dependent(k_qvs_rank, dim3((unsigned)per_img, (unsigned)p.B), 32 * kRankWarps, smem, s, p);
 }
 
 }  // namespace skipk

@@ -237,26 +237,46 @@ __global__ void __launch_bounds__(kSkvThreads, 1)
         }
         if (!ok) atomicOr(p.err, kErrTimeout);
         // Epilogue: h = acc + c_q, ReLU, dot with w2 over this CTA's units.
-        const bool done = half == 0 ? mbar_wait(smem_addr(&sh->tfull), 0, p.timeout_ns) : false;
-        if (half == 0 && !done) atomicOr(p.err, kErrTimeout);
-        tc_fence_after();
-        if (done) {
-            const uint32_t lane_addr = (uint32_t)((warp & 3) * 32) << 16;
-            const float *cq = p.cq + (int64_t)q * p.H + n0;
-            const float *w2 = p.w2 + n0;
-            float part = 0.f;
-#pragma unroll 1
-            for (int c = 0; c < kSkvHidden / 32; ++c) {
-                uint32_t v[32];
-                tmem_ld_32x32b_x32(tmem + lane_addr + c * 32, v);
-                tmem_ld_wait(v);
-#pragma unroll
-                for (int i = 0; i < 32; ++i) {
-                    const float h = __uint_as_float(v[i]) + __ldg(cq + c * 32 + i);
-                    part = fmaf(fmaxf(h, 0.f), __ldg(w2 + c * 32 + i), part);
+        if (half == 0) {
+            const bool done = mbar_wait(smem_addr(&sh->tfull), 0, p.timeout_ns);
+            if (!done) atomicOr(p.err, kErrTimeout);
+            tc_fence_after();
+            // c_q of the tile's questions for this CTA's units, the GEMM's
+            // K-split slabs summed once, staged in the A ring (free: every
+            // MMA that read it has completed).  cqs[(q - q0) * 128 + n].
+            float *cqs = reinterpret_cast<float *>(sA);
+            const int q0 = (int)(m0 / p.K);
+            const int64_t last = (m0 + kSkvRows < p.P ? m0 + kSkvRows : p.P) - 1;
+            const int nq = m0 < p.P ? (int)(last / p.K) - q0 + 1 : 0;  // <= 128: fits the ring
+            const int et = (warp & 3) * 32 + lane;                      // 0..127
+            const int64_t slab = (int64_t)p.Q * p.H;
+            if (done)
+                for (int t = et; t < nq * kSkvHidden; t += kSkvRows) {
+                    const float *src = p.cq + (int64_t)(q0 + t / kSkvHidden) * p.H + n0 + t % kSkvHidden;
+                    float v = 0.f;
+                    for (int z = 0; z < p.cq_splits; ++z) v += src[z * slab];
+                    cqs[t] = v;
                 }
+            asm volatile("bar.sync 1, %0;" ::"r"(kSkvRows) : "memory");  // the four epilogue warps
+            if (done) {
+                const uint32_t lane_addr = (uint32_t)((warp & 3) * 32) << 16;
+                // rows past the last slot (q = 0) read question q0's entries and write nothing
+                const float *cq = cqs + (slot < p.P ? q - q0 : 0) * kSkvHidden;
+                const float *w2 = p.w2 + n0;
+                float part = 0.f;
+#pragma unroll 1
+                for (int c = 0; c < kSkvHidden / 32; ++c) {
+                    uint32_t v[32];
+                    tmem_ld_32x32b_x32(tmem + lane_addr + c * 32, v);
+                    tmem_ld_wait(v);
+#pragma unroll
+                    for (int i = 0; i < 32; ++i) {
+                        const float h = __uint_as_float(v[i]) + cq[c * 32 + i];
+                        part = fmaf(fmaxf(h, 0.f), __ldg(w2 + c * 32 + i), part);
+                    }
+                }
+                if (slot < p.P) p.partial[(int64_t)blockIdx.y * p.P + slot] = part;
             }
-            if (slot < p.P) p.partial[(int64_t)blockIdx.y * p.P + slot] = part;
         }
     }
 

@@ -694,7 +694,7 @@ skip_status_t check_skv(skip_corpus *c, int32_t Q, int32_t K, const uint16_t *qb
 
 size_t skv_ws_bytes(int Q, int K, int H) {
     const size_t P = (size_t)Q * K;
-    return align_up((size_t)Q * H * 4, 256) + align_up((size_t)(H / kSkvHidden) * P * 4, 256);
+    return align_up((size_t)kSkvCqSplits * Q * H * 4, 256) + align_up((size_t)(H / kSkvHidden) * P * 4, 256);
 }
 
 // The gate on cand_ids; its workspace is the head of gws (skv_ws_bytes).
@@ -723,7 +723,7 @@ skip_status_t skv_impl(skip_corpus *c, const int64_t *cand_ids, int32_t Q, int32
     p.tau = tau;
     p.rho = rho;
     p.cq = reinterpret_cast<float *>(c->gws);
-    p.partial = reinterpret_cast<float *>((char *)c->gws + align_up((size_t)Q * H * 4, 256));
+    p.partial = reinterpret_cast<float *>((char *)c->gws + align_up((size_t)kSkvCqSplits * Q * H * 4, 256));
     p.out_ids = out_ids;
     p.out_nu = out_nu;
     p.out_count = out_count;
@@ -731,16 +731,18 @@ skip_status_t skv_impl(skip_corpus *c, const int64_t *cand_ids, int32_t Q, int32
     p.err = c->err;
     p.timeout_ns = c->timeout_ns;
     // c_q = b1 + W1[:, 0:d] qbar + W1[:, d:2d] vbar for every question: one
-    // GEMM over the two column blocks of W1.
+    // GEMM over the two column blocks of W1, K split over up to
+    // kSkvCqSplits CTAs per tile (k_skv_mlp sums the partial slabs).
     CUtensorMap ta, tb, ta2, tb2;
     const int tn = gemm_tile_n(Q, H, c->sm_count);
+    p.cq_splits = std::min(kSkvCqSplits, gemm_splits(Q, H, 2 * c->d, tn, c->sm_count));
     if (!encode_bf16_rows(&ta, qbar, Q, c->d, 128) || !encode_bf16_rows(&ta2, vbar, Q, c->d, 128) ||
         !encode_bf16_block(&tb, mlp->w1, H, c->d, 5 * (int64_t)c->d, tn) ||
         !encode_bf16_block(&tb2, mlp->w1 + c->d, H, c->d, 5 * (int64_t)c->d, tn))
         return SKIP_ECUDA;
     record(c, s, "skv_qbias");
     cudaError_t e = launch_gemm2_bf16_f32(ta, tb, &ta2, &tb2, tn, Q, H, c->d, c->d, 1.f, mlp->b1, p.cq, H, c->err,
-                                          c->timeout_ns, s);
+                                          c->timeout_ns, s, p.cq_splits, (int64_t)Q * H);
     if (e != cudaSuccess) return cuda_status(e);
     record(c, s, "skv_mlp");
     e = launch_skv_mlp(tw, p, s);
@@ -1518,7 +1520,7 @@ skip_status_t skip_qvs_create(const uint16_t *wv, const float *bv, const float *
         (q->dkp != dk && dev_alloc((void **)&q->fqp, (size_t)max_images * q->dkp * 2, "qvs") != cudaSuccess) ||
         dev_alloc((void **)&q->bv, (size_t)dk * 4, "qvs") != cudaSuccess ||
         dev_alloc((void **)&q->wb, (size_t)d * 4, "qvs") != cudaSuccess ||
-        dev_alloc((void **)&q->u, (size_t)max_images * d * 4, "qvs") != cudaSuccess ||
+        dev_alloc((void **)&q->u, (size_t)kQvsUSplits * max_images * d * 4, "qvs") != cudaSuccess ||
         dev_alloc((void **)&q->logits, (size_t)max_images * max_tokens * 4, "qvs") != cudaSuccess ||
         dev_alloc((void **)&q->err, sizeof(int), "qvs") != cudaSuccess) {
         cudaGetLastError();
@@ -1587,8 +1589,11 @@ skip_status_t skip_qvs_prune(skip_qvs_t q, const uint16_t *tokens, int32_t B, in
     const int tn = gemm_tile_n(B, q->d, q->sms);
     if (!encode_bf16_rows(&ta, fa, B, q->dkp, 128) || !encode_bf16_rows(&tb, q->wvt, q->d, q->dkp, tn))
         return SKIP_ECUDA;
+    // K split over up to kQvsUSplits CTAs per tile (a [B x d] product has few
+    // tiles); the logits kernel sums the partial slabs.
+    p.u_splits = std::min(kQvsUSplits, gemm_splits(B, q->d, q->dkp, tn, q->sms));
     cudaError_t e = launch_gemm_bf16_f32(ta, tb, tn, B, q->d, q->dkp, 1.f / std::sqrt((float)q->dk), q->u, q->d,
-                                         q->err, q->timeout_ns, s);
+                                         q->err, q->timeout_ns, s, p.u_splits, (int64_t)B * q->d);
     if (e == cudaSuccess) e = launch_qvs_logits(p, q->sms, s);
     if (e == cudaSuccess) e = launch_qvs_select(p, s);
     return cuda_status(e);

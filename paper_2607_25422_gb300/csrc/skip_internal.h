@@ -119,15 +119,21 @@ cudaError_t launch_latency(bool fp8, const CUtensorMap &ta, const CUtensorMap &t
 // box 128 rows x 64 elements; tb: over B, box tile_n rows x 64 elements; both
 // 128-byte swizzle.  err (nullable) receives kErrTimeout if a wait gives up.
 // gemm_tile_n: the tile width (32 or 64) to use for an M x N product.
+// splits > 1: K is split over that many CTAs per tile, each writing its
+// partial product to D + z * split_stride (split_stride >= M * ldd); the
+// caller sums the slabs.  gemm_splits: the split count that fills the SMs
+// once (1 when the tiles already do).
 int gemm_tile_n(int M, int N, int sms);
+int gemm_splits(int M, int N, int K, int tile_n, int sms);
 cudaError_t launch_gemm_bf16_f32(const CUtensorMap &ta, const CUtensorMap &tb, int tile_n, int M, int N, int K,
-                                 float alpha, float *D, int64_t ldd, int *err, uint64_t timeout_ns, cudaStream_t s);
+                                 float alpha, float *D, int64_t ldd, int *err, uint64_t timeout_ns, cudaStream_t s,
+                                 int splits = 1, int64_t split_stride = 0);
 // D = alpha * (A B^T + A2 B2^T) + bias (per column n; nullable); ta2 / tb2
 // over A2 [M x K2] / B2 [N x K2] with the same boxes (K2 = 0: one product).
 cudaError_t launch_gemm2_bf16_f32(const CUtensorMap &ta, const CUtensorMap &tb, const CUtensorMap *ta2,
                                   const CUtensorMap *tb2, int tile_n, int M, int N, int K, int K2, float alpha,
                                   const float *bias, float *D, int64_t ldd, int *err, uint64_t timeout_ns,
-                                  cudaStream_t s);
+                                  cudaStream_t s, int splits = 1, int64_t split_stride = 0);
 
 // ---- merges -------------------------------------------------------------
 // Per-region merge of G sorted lists into the exact top-k (keys and/or
@@ -169,7 +175,8 @@ struct SkvParams {
     float b2;
     int H;                 // multiple of kSkvHidden
     float tau, rho;
-    float *cq;             // [Q x H] workspace: b1 + W1 qbar-part + W1 vbar-part
+    float *cq;             // [cq_splits x Q x H] workspace: partial sums of b1 + W1 qbar-part + W1 vbar-part
+    int cq_splits;         // K splits of the c_q GEMM (the slabs are summed in k_skv_mlp)
     float *partial;        // [H / kSkvHidden][P] workspace: partial logits
     int64_t *out_ids;      // [Q x K]
     float *out_nu;         // [Q x K]
@@ -240,6 +247,8 @@ cudaError_t launch_ivfpq_scan(const IvfParams &p, const uint16_t *regions, int R
 // ---- QVS visual token pruning (k_qvs.cu) -----------------------------------
 constexpr int kQvsMaxDk = 4096;  // projection width d_k
 constexpr int kQvsMaxL = 4096;   // tokens per image
+constexpr int kQvsUSplits = 4;   // K splits of the projected-query GEMM
+constexpr int kSkvCqSplits = 4;  // K splits of the SKV gate's c_q GEMM
 struct QvsParams {
     const void *tokens;     // bf16 [B x L x d]
     const void *fq;         // bf16 [B x dk]
@@ -247,7 +256,8 @@ struct QvsParams {
     const float *bv;        // [dk] or null
     const float *wb;        // [d]
     int B, L, d, dk, n;     // n tokens kept per image
-    float *u;               // [B x d] W_v^T f_q / sqrt(d_k) (written by the tensor-core GEMM)
+    float *u;               // [u_splits x B x d] partial sums of W_v^T f_q / sqrt(d_k) (split-K GEMM)
+    int u_splits;
     float *logits;          // [B x L] workspace
     int32_t *out_idx;       // [B x n]
     float *out_score;       // [B x n]
@@ -256,6 +266,8 @@ struct QvsParams {
 cudaError_t launch_qvs_logits(const QvsParams &p, int sms, cudaStream_t s);
 // wt [cols x ldt] (first `rows` of each row) = w^T for a bf16 w [rows x cols].
 cudaError_t launch_transpose_bf16(const uint16_t *w, int rows, int cols, uint16_t *wt, int ldt, cudaStream_t s);
+// Ranks every token by counting the larger logits and writes the kept ones
+// (rank < n) in rank order, with their rows when out_tokens is set.
 cudaError_t launch_qvs_select(const QvsParams &p, cudaStream_t s);
 
 // ---- BSCA bipartite sparse cross-attention (k_bsca.cu) --------------------

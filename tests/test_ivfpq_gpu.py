@@ -411,7 +411,8 @@ def test_refine_matches_oracle(refine):
     lists, code_by_id = _lists_by_id(off, ids, codes, SPEC.N, cb.shape[0])
     gidx = {"offsets": off, "ids": ids.astype(np.int64), "codes": code_by_id, "lists": lists}
     # the oracle's shortlist one past ks (for the tie test) and its exact re-rank of all ks
-    s_ids, s_sc, _ = oracle.ivfpq_search(gidx, ce, cb.numpy(), qn, nprobe, ks + 1)
+    ext = 32
+    s_ids, s_sc, _ = oracle.ivfpq_search(gidx, ce, cb.numpy(), qn, nprobe, ks + ext)
     o_ids, o_sc = oracle.ivfpq_search_refine(gidx, ce, cb.numpy(), qn, nprobe, ks, ks, cn)
     cs = np.sort(oracle.score_matrix(ce, qn), axis=1)[:, ::-1]
     truths = checker.region_truths(o_ids, o_sc, k)
@@ -420,7 +421,14 @@ def test_refine_matches_oracle(refine):
         if cs[r, nprobe - 1] - cs[r, nprobe] <= PROBE_TIE:
             continue
         if s_ids[r, ks] >= 0 and s_sc[r, ks - 1] - s_sc[r, ks] <= PROBE_TIE:
-            continue
+            # A near tie in s^ at the shortlist's end only matters when one
+            # of the tied entries could reach the exact top k.
+            tied = np.nonzero((s_ids[r] >= 0) & (np.abs(s_sc[r] - s_sc[r, ks - 1]) <= PROBE_TIE))[0]
+            if tied[-1] == ks + ext - 1:
+                continue
+            ex = oracle.scores_at(cn, qn, np.full(len(tied), r), s_ids[r, tied])
+            if ex.max() >= truths[r].theta - checker.TAU:
+                continue
         _, probs = checker.check_region(
             g_ids[r], g_sc[r], truths[r],
             extra_score=lambda i, r=r: float(oracle.scores_at(cn, qn, [r], [i])[0]))

@@ -17,7 +17,7 @@ from tests._golden import read_fixture
 
 pytestmark = pytest.mark.gpu
 
-PATHS = {"tensor": skip.SKIP_PATH_TENSOR, "warp": skip.SKIP_PATH_WARP}
+PATHS = {"tensor": skip.SKIP_PATH_TENSOR, "warp": skip.SKIP_PATH_WARP, "latency": skip.SKIP_PATH_LATENCY}
 
 
 def _bits(t):
@@ -221,7 +221,7 @@ def test_clustered_near_ties():
     assert_parity(cn, rn, offsets, spec.k_region, spec.K, gpu, truth)
 
 
-@pytest.mark.parametrize("path", ["tensor", "warp"])
+@pytest.mark.parametrize("path", ["tensor", "warp", "latency"])
 def test_duplicate_rows_and_ties(path):
     ct = synth.random_bf16(4000, 128, seed=5)
     ct[1000] = ct[17]
@@ -280,6 +280,11 @@ LATENCY_CASES = [
     ("bf16", 30001, 768, 32, 4, 10, 20),
     ("bf16", 5000, 256, 7, 3, 50, 60),
     ("bf16", 2000, 128, 20, 5, 64, 80),
+    # register-set widths 4, 8, 12 and 16 at their upper ends
+    ("bf16", 50000, 512, 24, 6, 3, 8),
+    ("bf16", 3000, 64, 9, 3, 8, 16),
+    ("bf16", 20000, 128, 16, 4, 12, 24),
+    ("bf16", 40003, 256, 32, 8, 16, 30),
     ("e4m3", 6000, 1024, 32, 1, 10, 100),
     ("e4m3", 7001, 80, 5, 2, 7, 20),
     ("e4m3", 20000, 512, 17, 3, 30, 40),
