@@ -81,6 +81,9 @@ __global__ void __launch_bounds__(kThreads, 1)
     }
     constexpr uint32_t kIdesc = idesc_bf16_f32(128, BN);
 
+    // A kernel launched as this one's programmatic dependent may start now:
+    // it waits for this grid's results itself (griddepcontrol.wait).
+    grid_dep_launch();
     if (threadIdx.x == 0) {
         for (int s = 0; s < kStages; ++s) {
             mbar_init(smem_addr(&sh->full[s]), 1);

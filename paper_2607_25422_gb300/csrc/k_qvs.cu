@@ -39,6 +39,18 @@ __global__ void __launch_bounds__(kLogThreads) k_qvs_logits(const QvsParams p) {
     __shared__ float cpart[kLogThreads / 32];
     const int b = blockIdx.y;
     const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+    // The tokens are inputs of the call, not results of the GEMM before this
+    // kernel: while that GEMM still runs (this kernel is its programmatic
+    // dependent), pull this warp's token rows into L2, one 128-byte line per
+    // lane and step.
+    {
+        const int lines = p.d / 64;  // 128-byte lines per token row
+        const int ws = gridDim.x * (kLogThreads / 32);
+        for (int i = blockIdx.x * (kLogThreads / 32) + warp; i < p.L; i += ws) {
+            const char *row = reinterpret_cast<const char *>(p.tokens) + ((int64_t)b * p.L + i) * p.d * 2;
+            for (int l = lane; l < lines; l += 32) asm volatile("prefetch.global.L2 [%0];" ::"l"(row + l * 128) : "memory");
+        }
+    }
     grid_dep_wait();
     // u = W_v^T f_q / sqrt(d_k) (the GEMM's partial slabs) + w_b; c = <f_q, b_v> / sqrt(d_k)
     const int64_t slab = (int64_t)p.B * p.d;

@@ -42,7 +42,7 @@ constexpr uint32_t kSkvIdesc = idesc_bf16_f32(128, kSkvHidden);
 constexpr uint64_t kDrainTimeoutNs = 1000000000ull;  // 1 s for copies in flight
 
 struct SkvShared {
-    uint64_t full[kSkvStages];   // A built (128 arrivals) and B landed (tx bytes)
+    uint64_t full[kSkvStages];   // A built (one arrival per builder warp) and B landed (tx bytes)
     uint64_t empty[kSkvStages];  // stage consumed (tcgen05.commit)
     uint64_t tfull;              // accumulator complete
     uint32_t tmem_base;
@@ -87,7 +87,7 @@ __global__ void __launch_bounds__(kSkvThreads, 1)
 
     if (threadIdx.x == 0) {
         for (int s = 0; s < kSkvStages; ++s) {
-            mbar_init(smem_addr(&sh->full[s]), 32 * kSkvBuilders + 1);
+            mbar_init(smem_addr(&sh->full[s]), kSkvBuilders + 1);  // one arrival per builder warp + the TMA
             mbar_init(smem_addr(&sh->empty[s]), 1);
         }
         mbar_init(smem_addr(&sh->tfull), 1);
@@ -223,15 +223,20 @@ __global__ void __launch_bounds__(kSkvThreads, 1)
             for (int b = 0; b < 3; ++b) {
                 const int u = 3 * c + b, s = u % kSkvStages;
                 const uint32_t ph = (uint32_t)(u / kSkvStages) & 1u;
-                if (!mbar_wait(smem_addr(&sh->empty[s]), ph ^ 1u, p.timeout_ns)) {
+                // warp-uniform: every lane waits (bounded), then the warp votes
+                if (!__all_sync(0xffffffffu, mbar_wait(smem_addr(&sh->empty[s]), ph ^ 1u, p.timeout_ns))) {
                     ok = false;
                     break;
                 }
                 const uint32_t base = smem_addr(sA + s * kSkvStageA) + r * 128;
 #pragma unroll
                 for (int jj = 0; jj < 4; ++jj) sts128(base + (uint32_t)(((4 * half + jj) ^ sw) << 4), f[b][jj]);
+                // each writer makes its stores visible to the tensor core's
+                // (async) proxy, then one arrival per warp: 257 arrivals on
+                // one barrier per slice were serialised
                 fence_proxy_async_smem();
-                mbar_arrive(smem_addr(&sh->full[s]));
+                __syncwarp();
+                if (lane == 0) mbar_arrive(smem_addr(&sh->full[s]));
             }
             if (!ok) break;
         }
