@@ -682,6 +682,23 @@ def main():
     ms_ev_local, kernels = run_timed(True)
     ms = max_over_ranks(ms_local, world)
     ms_ev = max_over_ranks(ms_ev_local, world)
+    plain_ms = None
+    if args.skv:
+        # the same batch without the gate, timed the same way in this process:
+        # the gate's cost in the step with its launches overlapped
+        def plain():
+            skip.skip_retrieve(c, reg_d, off_d, spec.k_region, spec.K, out_ids, out_sc, stream)
+        for _ in range(args.warmup):
+            plain()
+        torch.cuda.synchronize()
+        e0 = torch.cuda.Event(enable_timing=True)
+        e1 = torch.cuda.Event(enable_timing=True)
+        e0.record(stream)
+        for _ in range(args.steps):
+            plain()
+        e1.record(stream)
+        torch.cuda.synchronize()
+        plain_ms = max_over_ranks(e0.elapsed_time(e1), world)
 
     # ---- end to end through the host-buffer entry point
     reg_h = regions.pin_memory()
@@ -793,6 +810,8 @@ def main():
         mlp = kernels.get("skv_mlp", {"ms": float("nan"), "launches": 1})
         mlp_ms = mlp["ms"] / max(1, mlp["launches"])
         line["skv"] = {"gate_ms_per_step": skv_ms, "mlp_kernel_ms": mlp_ms,
+                       "step_ms_without_gate": plain_ms / args.steps,
+                       "gate_step_delta_ms": (ms - plain_ms) / args.steps,
                        "mlp_algorithmic_flops": 2.0 * P * 3 * spec.d * H,
                        "mlp_tflops": 2.0 * P * 3 * spec.d * H / (mlp_ms / 1e3) / 1e12,
                        "gate_share_of_step": skv_ms / (ms / args.steps), "algorithmic_flops": skv_flops}

@@ -10,8 +10,11 @@
 //                rows and qbar: per 64-column chunk of d, three K-slices
 //                e | bf16(e * qbar) | bf16(|e - qbar|) in the 128-byte
 //                swizzled layout TMA would produce, one slice per stage of a
-//                six-stage ring; the B operand is the matching W1 column
-//                block, loaded by TMA.  tcgen05.mma
+//                four-stage ring; the B operand is the matching W1 column
+//                block, loaded by TMA into an eight-stage ring of its own.
+//                Launched as the programmatic dependent of the c_q GEMM: it
+//                gathers and multiplies while the GEMM runs and waits for c_q
+//                only in its epilogue.  tcgen05.mma
 //                (kind::f16, M = N = 128) accumulates in TMEM; the epilogue
 //                adds c_q, applies ReLU and the w2 dot for its 128 units and
 //                writes one partial logit per slot and hidden block.
@@ -30,11 +33,14 @@ namespace {
 
 constexpr int kSkvRows = 128;                       // passage slots per CTA (TMEM lanes)
 constexpr int kSkvSlice = kSkvRows * 128;           // one [128 x 64] bf16 K-slice, bytes
-// A stage is one K-slice: of A (e, e*qbar or |e - qbar| of one 64-column
-// chunk of d) and of B (the matching W1 column block for 128 units).
+// A stage holds one K-slice of A (e, e*qbar or |e - qbar| of one 64-column
+// chunk of d) or of B (the matching W1 column block for 128 units).  The two
+// rings are separate: B, whose TMA copy from L2 takes microseconds, runs
+// eight slices ahead; A, built from rows the builders already hold, four.
 constexpr int kSkvStageA = kSkvSlice;
 constexpr int kSkvStageB = kSkvSlice;
-constexpr int kSkvStages = 6;
+constexpr int kSkvStagesA = 4;
+constexpr int kSkvStagesB = 8;
 constexpr int kSkvBuilders = 8;                     // two builder warps per TMEM lane quadrant
 constexpr int kSkvThreads = 64 + 32 * kSkvBuilders;  // TMA warp, MMA warp, builders (4 of them: epilogue)
 constexpr int kSkvAhead = 3;                         // chunks of corpus row in flight per builder thread
@@ -42,8 +48,10 @@ constexpr uint32_t kSkvIdesc = idesc_bf16_f32(128, kSkvHidden);
 constexpr uint64_t kDrainTimeoutNs = 1000000000ull;  // 1 s for copies in flight
 
 struct SkvShared {
-    uint64_t full[kSkvStages];   // A built (one arrival per builder warp) and B landed (tx bytes)
-    uint64_t empty[kSkvStages];  // stage consumed (tcgen05.commit)
+    uint64_t fullA[kSkvStagesA];   // A built (one arrival per builder warp)
+    uint64_t emptyA[kSkvStagesA];  // A stage consumed (tcgen05.commit)
+    uint64_t fullB[kSkvStagesB];   // B landed (tx bytes)
+    uint64_t emptyB[kSkvStagesB];  // B stage consumed (tcgen05.commit)
     uint64_t tfull;              // accumulator complete
     uint32_t tmem_base;
 };
@@ -78,17 +86,21 @@ __global__ void __launch_bounds__(kSkvThreads, 1)
     extern __shared__ __align__(1024) uint8_t smem_raw[];
     uint8_t *smem = reinterpret_cast<uint8_t *>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
     uint8_t *sA = smem;
-    uint8_t *sB = smem + kSkvStages * kSkvStageA;
-    SkvShared *sh = reinterpret_cast<SkvShared *>(sB + kSkvStages * kSkvStageB);
+    uint8_t *sB = smem + kSkvStagesA * kSkvStageA;
+    SkvShared *sh = reinterpret_cast<SkvShared *>(sB + kSkvStagesB * kSkvStageB);
     const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
     const int64_t m0 = (int64_t)blockIdx.x * kSkvRows;
     const int n0 = blockIdx.y * kSkvHidden;
     const int nc = p.d / 64;
 
     if (threadIdx.x == 0) {
-        for (int s = 0; s < kSkvStages; ++s) {
-            mbar_init(smem_addr(&sh->full[s]), kSkvBuilders + 1);  // one arrival per builder warp + the TMA
-            mbar_init(smem_addr(&sh->empty[s]), 1);
+        for (int s = 0; s < kSkvStagesA; ++s) {
+            mbar_init(smem_addr(&sh->fullA[s]), kSkvBuilders);  // one arrival per builder warp
+            mbar_init(smem_addr(&sh->emptyA[s]), 1);
+        }
+        for (int s = 0; s < kSkvStagesB; ++s) {
+            mbar_init(smem_addr(&sh->fullB[s]), 1);
+            mbar_init(smem_addr(&sh->emptyB[s]), 1);
         }
         mbar_init(smem_addr(&sh->tfull), 1);
         mbar_fence_init();
@@ -109,23 +121,23 @@ __global__ void __launch_bounds__(kSkvThreads, 1)
             bool ok = true;
             int issued = 0;
             for (int u = 0; u < 3 * nc && ok; ++u) {
-                const int s = u % kSkvStages, c = u / 3, b = u - 3 * c;
-                const uint32_t ph = (uint32_t)(u / kSkvStages) & 1u;
-                if (!mbar_wait(smem_addr(&sh->empty[s]), ph ^ 1u, p.timeout_ns)) {
+                const int s = u % kSkvStagesB, c = u / 3, b = u - 3 * c;
+                const uint32_t ph = (uint32_t)(u / kSkvStagesB) & 1u;
+                if (!mbar_wait(smem_addr(&sh->emptyB[s]), ph ^ 1u, p.timeout_ns)) {
                     ok = false;
                     break;
                 }
-                const uint32_t fb = smem_addr(&sh->full[s]);
+                const uint32_t fb = smem_addr(&sh->fullB[s]);
                 mbar_arrive_expect_tx(fb, kSkvStageB);
                 tma_load_2d(smem_addr(sB + s * kSkvStageB), &tw, fb, (2 + b) * p.d + c * 64, n0);
                 ++issued;
             }
             if (!ok) atomicOr(p.err, kErrTimeout);
             // Copies in flight: wait for the last use of each stage to complete.
-            for (int s = 0; s < kSkvStages; ++s) {
-                const int uses = issued / kSkvStages + (s < issued % kSkvStages ? 1 : 0);
+            for (int s = 0; s < kSkvStagesB; ++s) {
+                const int uses = issued / kSkvStagesB + (s < issued % kSkvStagesB ? 1 : 0);
                 if (uses == 0) continue;
-                if (!mbar_wait(smem_addr(&sh->full[s]), (uint32_t)((uses - 1) & 1), kDrainTimeoutNs))
+                if (!mbar_wait(smem_addr(&sh->fullB[s]), (uint32_t)((uses - 1) & 1), kDrainTimeoutNs))
                     atomicOr(p.err, kErrTimeout);
             }
         }
@@ -134,19 +146,20 @@ __global__ void __launch_bounds__(kSkvThreads, 1)
         if (lane == 0) {
             bool ok = true;
             for (int u = 0; u < 3 * nc && ok; ++u) {
-                const int s = u % kSkvStages;
-                const uint32_t ph = (uint32_t)(u / kSkvStages) & 1u;
-                if (!mbar_wait(smem_addr(&sh->full[s]), ph, p.timeout_ns)) {
+                const int sa = u % kSkvStagesA, sb = u % kSkvStagesB;
+                if (!mbar_wait(smem_addr(&sh->fullA[sa]), (uint32_t)(u / kSkvStagesA) & 1u, p.timeout_ns) ||
+                    !mbar_wait(smem_addr(&sh->fullB[sb]), (uint32_t)(u / kSkvStagesB) & 1u, p.timeout_ns)) {
                     ok = false;
                     break;
                 }
                 tc_fence_after();
-                const uint64_t ad = smem_desc_k128(smem_addr(sA + s * kSkvStageA));
-                const uint64_t bd = smem_desc_k128(smem_addr(sB + s * kSkvStageB));
+                const uint64_t ad = smem_desc_k128(smem_addr(sA + sa * kSkvStageA));
+                const uint64_t bd = smem_desc_k128(smem_addr(sB + sb * kSkvStageB));
 #pragma unroll
                 for (int kk = 0; kk < 4; ++kk)
                     tc_mma_f16(tmem, ad + (uint64_t)(kk * 2), bd + (uint64_t)(kk * 2), kSkvIdesc, (u | kk) != 0);
-                tc_commit(smem_addr(&sh->empty[s]));
+                tc_commit(smem_addr(&sh->emptyA[sa]));
+                tc_commit(smem_addr(&sh->emptyB[sb]));
             }
             if (!ok) atomicOr(p.err, kErrTimeout);
             // Arrives once every MMA issued has completed (also after a timeout).
@@ -221,10 +234,10 @@ __global__ void __launch_bounds__(kSkvThreads, 1)
             const int sw = r & 7;
 #pragma unroll
             for (int b = 0; b < 3; ++b) {
-                const int u = 3 * c + b, s = u % kSkvStages;
-                const uint32_t ph = (uint32_t)(u / kSkvStages) & 1u;
+                const int u = 3 * c + b, s = u % kSkvStagesA;
+                const uint32_t ph = (uint32_t)(u / kSkvStagesA) & 1u;
                 // warp-uniform: every lane waits (bounded), then the warp votes
-                if (!__all_sync(0xffffffffu, mbar_wait(smem_addr(&sh->empty[s]), ph ^ 1u, p.timeout_ns))) {
+                if (!__all_sync(0xffffffffu, mbar_wait(smem_addr(&sh->emptyA[s]), ph ^ 1u, p.timeout_ns))) {
                     ok = false;
                     break;
                 }
@@ -236,7 +249,7 @@ __global__ void __launch_bounds__(kSkvThreads, 1)
                 // one barrier per slice were serialised
                 fence_proxy_async_smem();
                 __syncwarp();
-                if (lane == 0) mbar_arrive(smem_addr(&sh->full[s]));
+                if (lane == 0) mbar_arrive(smem_addr(&sh->fullA[s]));
             }
             if (!ok) break;
         }
@@ -246,9 +259,13 @@ __global__ void __launch_bounds__(kSkvThreads, 1)
             const bool done = mbar_wait(smem_addr(&sh->tfull), 0, p.timeout_ns);
             if (!done) atomicOr(p.err, kErrTimeout);
             tc_fence_after();
+            // c_q comes from the GEMM launched just before this kernel (whose
+            // programmatic dependent it is): wait for that grid here only.
+            grid_dep_wait();
             // c_q of the tile's questions for this CTA's units, the GEMM's
             // K-split slabs summed once, staged in the A ring (free: every
-            // MMA that read it has completed).  cqs[(q - q0) * 128 + n].
+            // MMA that read it has completed; 64 KB holds 128 questions).
+            // cqs[(q - q0) * 128 + n].
             float *cqs = reinterpret_cast<float *>(sA);
             const int q0 = (int)(m0 / p.K);
             const int64_t last = (m0 + kSkvRows < p.P ? m0 + kSkvRows : p.P) - 1;
@@ -304,6 +321,7 @@ __global__ void __launch_bounds__(kSelThreads) k_skv_select(const SkvParams p) {
     const int K = p.K;
     int Kp = 1;
     while (Kp < K) Kp <<= 1;
+    grid_dep_wait();  // the partial logits of the MLP kernel before this one
     if (threadIdx.x == 0) nonempty = 0, ngated = 0;
     __syncthreads();
     const int nb = p.H / kSkvHidden;
@@ -369,7 +387,24 @@ __global__ void __launch_bounds__(kSelThreads) k_skv_select(const SkvParams p) {
 }  // namespace
 
 size_t skv_mlp_smem_bytes() {
-    return 1024 + (size_t)kSkvStages * (kSkvStageA + kSkvStageB) + sizeof(SkvShared);
+    return 1024 + (size_t)kSkvStagesA * kSkvStageA + (size_t)kSkvStagesB * kSkvStageB + sizeof(SkvShared);
+}
+
+// Launch as the programmatic dependent of the previous kernel in the stream.
+template <typename... Args>
+cudaError_t launch_dependent(void (*kern)(Args...), dim3 grid, int threads, size_t smem, cudaStream_t s,
+                             Args... args) {
+    cudaLaunchConfig_t cfg = {};
+    cfg.gridDim = grid;
+    cfg.blockDim = dim3((unsigned)threads);
+    cfg.dynamicSmemBytes = smem;
+    cfg.stream = s;
+    cudaLaunchAttribute attr[1];
+    attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+    attr[0].val.programmaticStreamSerializationAllowed = 1;
+    cfg.attrs = attr;
+    cfg.numAttrs = 1;
+    return cudaLaunchKernelEx(&cfg, kern, args...);
 }
 
 cudaError_t launch_skv_mlp(const CUtensorMap &tw, const SkvParams &p, cudaStream_t s) {
@@ -378,14 +413,12 @@ cudaError_t launch_skv_mlp(const CUtensorMap &tw, const SkvParams &p, cudaStream
     cudaError_t e = cudaFuncSetAttribute(k_skv_mlp, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
     if (e != cudaSuccess) return e;
     dim3 grid((unsigned)((p.P + kSkvRows - 1) / kSkvRows), (unsigned)(p.H / kSkvHidden));
-    k_skv_mlp<<<grid, kSkvThreads, smem, s>>>(tw, p);
-    return cudaGetLastError();
+    return launch_dependent(k_skv_mlp, grid, kSkvThreads, smem, s, tw, p);
 }
 
 cudaError_t launch_skv_select(const SkvParams &p, cudaStream_t s) {
     if (p.Q == 0) return cudaSuccess;
-    k_skv_select<<<p.Q, kSelThreads, 0, s>>>(p);
-    return cudaGetLastError();
+    return launch_dependent(k_skv_select, dim3((unsigned)p.Q), kSelThreads, 0, s, p);
 }
 
 }  // namespace skipk
