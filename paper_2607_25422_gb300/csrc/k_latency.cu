@@ -542,12 +542,18 @@ __global__ void __launch_bounds__(kThreads, 1)
 }
 
 // Splits each bf16 query row into three e4m3 parts with power-of-two scales
-// (rows r, 32 + r, 64 + r of the 96-row operand; the other rows stay zero).
-// One block per query row.
+// (rows r, 32 + r, 64 + r of the 96-row operand).  One block per row slot
+// r < 32: the slots past the batch's R rows write zero parts, so that the
+// operand needs no clearing.
 __global__ void __launch_bounds__(256) k_split_queries(const uint16_t *__restrict__ regions, int R, int d,
                                                        uint8_t *__restrict__ parts, float *__restrict__ qscale) {
     __shared__ float red[8];
     const int r = blockIdx.x;
+    if (r >= R) {
+        for (int j = threadIdx.x; j < d; j += blockDim.x)
+            for (int part = 0; part < 3; ++part) parts[(size_t)(part * 32 + r) * d + j] = 0;
+        return;
+    }
     const uint16_t *q = regions + (size_t)r * d;
     auto block_max = [&](float v) {
         for (int o = 16; o; o >>= 1) v = fmaxf(v, __shfl_xor_sync(0xffffffffu, v, o));
@@ -613,7 +619,7 @@ bool lat_pick_layout(bool fp8, int R, int d, int k, int max_smem, int *Npad, int
 
 cudaError_t launch_split_queries(const uint16_t *regions, int R, int d, uint8_t *parts, float *qscale,
                                  cudaStream_t s) {
-    k_split_queries<<<R, 256, 0, s>>>(regions, R, d, parts, qscale);
+    k_split_queries<<<kLatMaxR, 256, 0, s>>>(regions, R, d, parts, qscale);
     return cudaGetLastError();
 }
 

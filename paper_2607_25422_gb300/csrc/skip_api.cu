@@ -321,7 +321,6 @@ skip_status_t run_regions(skip_corpus *c, const uint16_t *regions, int R, int k,
         if (cudaMemsetAsync(tau, 0, tau_bytes, s) != cudaSuccess) return SKIP_ECUDA;
         CUtensorMap ta, tb;
         if (e4m3) {
-            if (cudaMemsetAsync(parts, 0, parts_bytes, s) != cudaSuccess) return SKIP_ECUDA;
             record(c, s, "split_queries");
             cudaError_t e = launch_split_queries(regions, R, c->d, parts, qscale, s);
             if (e != cudaSuccess) return cuda_status(e);

@@ -107,7 +107,7 @@ struct LatParams {
     uint64_t timeout_ns;
 };
 bool lat_pick_layout(bool fp8, int R, int d, int k, int max_smem, int *Npad, int *slices, int *stages);
-// e4m3 query parts: parts [96 x d] bytes (zeroed by the caller), qscale [3][R].
+// e4m3 query parts: parts [96 x d] bytes (all 96 rows written: rows of slots past R are zero), qscale [3][R].
 cudaError_t launch_split_queries(const uint16_t *regions, int R, int d, uint8_t *parts, float *qscale,
                                  cudaStream_t s);
 cudaError_t launch_latency(bool fp8, const CUtensorMap &ta, const CUtensorMap &tb, const LatParams &p, int grid,
