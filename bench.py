@@ -30,6 +30,7 @@ import argparse
 import hashlib
 import json
 import os
+import platform
 import statistics
 import subprocess
 import sys
@@ -197,6 +198,45 @@ def host_corpus(corpus, scale):
     return corpus.cpu().numpy(), scale.cpu().numpy()
 
 
+def cpu_model():
+    """The host CPU's model name (x86: 'model name'; Arm: implementer and
+    part numbers), for the baseline's record."""
+    try:
+        with open("/proc/cpuinfo") as f:
+            info = f.read()
+    except OSError:
+        return platform.machine()
+    for key in ("model name", "Model name"):
+        for line in info.splitlines():
+            if line.startswith(key):
+                return line.split(":", 1)[1].strip()
+    fields = {}
+    for line in info.splitlines():
+        if ":" in line:
+            k, v = line.split(":", 1)
+            fields.setdefault(k.strip(), v.strip())
+    parts = {"0xd0c": "Neoverse N1", "0xd40": "Neoverse V1", "0xd49": "Neoverse N2", "0xd4f": "Neoverse V2"}
+    part = fields.get("CPU part", "?")
+    return "%s %s (CPU implementer %s, part %s)" % (platform.machine(), parts.get(part, ""),
+                                                   fields.get("CPU implementer", "?"), part)
+
+
+def dedup_rate(skip, c, reg_d, offsets, k):
+    """Share of the pooled region-list entries of a question that repeat an
+    id already in the pool, over the batch (the paper reports 40-60% on real
+    questions): one untimed skip_retrieve_regions call."""
+    rid, _ = skip.skip_retrieve_regions(c, reg_d, k)
+    rid = rid.cpu()
+    off = offsets.numpy()
+    pooled = dup = 0
+    for q in range(off.size - 1):
+        ids = rid[off[q]:off[q + 1]].reshape(-1)
+        ids = ids[ids >= 0]
+        pooled += ids.numel()
+        dup += ids.numel() - torch.unique(ids).numel()
+    return dup / max(1, pooled)
+
+
 def cpu_baseline(spec, corpus_np, scale_np, regions, offsets, questions):
     """The oracle on a bounded sample of the batch over the full corpus.
     Ragged batches: a question with the fewest and one with the most regions
@@ -223,7 +263,7 @@ def cpu_baseline(spec, corpus_np, scale_np, regions, offsets, questions):
     per_region = dt / max(1, len(rows))
     batch_s = per_region * int(off_all[-1])
     return {"value": (counts.size / batch_s) if not spec.fixed_regions else len(qs) / dt, "unit": "queries/s",
-            "cores": nthreads, "kind": "oracle",
+            "cores": nthreads, "kind": "oracle", "cpu": cpu_model(),
             "sample": "%s (%d regions) over the full %d-row corpus, fp64, %d OpenMP threads, %.1f s; %s" % (
                 how, len(rows), spec.N, nthreads, dt,
                 "scaled per region to the batch's %d regions (extrapolated)" % int(off_all[-1])
@@ -271,7 +311,7 @@ def run_reference(args, spec):
             "higher_is_better": True, "scaling": "weak", "vs_baseline": None, "dtype": "f64",
             "data": "synthetic", "config": workload_config(spec, int(offsets[-1]), 1),
             "cpu_baseline": {"value": value, "unit": "queries/s", "cores": nthreads, "kind": "oracle",
-                             "sample": sample},
+                             "cpu": cpu_model(), "sample": sample},
             "e2e": {"value": value, "unit": "queries/s", "h2d_bytes_per_step": 0, "d2h_bytes_per_step": 0}}
     print(json.dumps(line), flush=True)
 
@@ -794,6 +834,7 @@ def main():
         "gpu_launches": int(sum(v["launches"] for v in kernels.values())),
         "kernels": kernels,
         "plan": plan,
+        "dedup_rate": None if args.ivfpq else dedup_rate(skip, c, reg_d, offsets, spec.k_region),
     }
     if args.ivfpq:
         line.update(ivfpq_report(args, spec, skip, c, ix, cent, reg_d, off_d, kernels, build_s, peaks, ms))
