@@ -197,6 +197,60 @@ __global__ void __launch_bounds__(kQThreads)
     }
 }
 
+// Both merges in one launch, for batches whose questions' pooled region
+// lists fit in shared memory (R k <= kQCap): one block per question; its
+// warps merge the question's region rows (k-way over the G partition
+// lists, as k_merge_lists) straight into the block's pool, then the block
+// deduplicates and ranks the pool as k_question_merge does.  One launch
+// and one hand-off fewer for the small batches.
+template <int LPL>
+__global__ void __launch_bounds__(kQThreads)
+    k_merge_regions_questions(const uint64_t *__restrict__ lists, int G, int64_t g_stride, int k,
+                              const int32_t *__restrict__ offsets, int R, int K, int64_t *__restrict__ out_ids,
+                              float *__restrict__ out_scores, int *__restrict__ err) {
+    extern __shared__ uint64_t qsmem[];
+    grid_dep_wait();
+    grid_dep_launch();
+    uint64_t *pool = qsmem;            // [kQCap] id-major keys
+    uint64_t *ranked = qsmem + kQCap;  // [kQCap] ranking keys, negated for the ascending sort
+    __shared__ int s_kept;
+    const int q = blockIdx.x;
+    const int warp = threadIdx.x >> 5, nwarps = blockDim.x >> 5;
+    const int o0 = offsets[q], o1 = offsets[q + 1];
+    const int r0 = min(max(o0, 0), R);
+    const int r1 = min(max(o1, r0), R);
+    if ((r0 != o0 || r1 != o1) && threadIdx.x == 0) atomicOr(err, kErrConfig);
+    const int nreg = r1 - r0, n = nreg * k;  // n <= R k <= kQCap (checked at launch)
+    for (int j = warp; j < nreg; j += nwarps)
+        warp_merge_topk<LPL>(lists + (int64_t)(r0 + j) * k, g_stride, G, k, k,
+                             [&](int i, uint64_t key) { pool[j * k + i] = id_major(key); });
+    const int n2 = pow2_at_least(n > 1 ? n : 1);
+    for (int i = n + threadIdx.x; i < n2; i += blockDim.x) pool[i] = kNone;
+    if (threadIdx.x == 0) s_kept = 0;
+    block_bitonic_sort_asc(pool, n2);  // starts with a block barrier
+    // First entry of every id run = that id with its maximum score.
+    for (int i = threadIdx.x; i < n; i += blockDim.x) {
+        const uint64_t v = pool[i];
+        if (v == kNone) continue;
+        if (i > 0 && (pool[i - 1] >> 32) == (v >> 32)) continue;
+        const int at = atomicAdd(&s_kept, 1);
+        ranked[at] = ~rank_of_id_major(v);
+    }
+    __syncthreads();
+    const int m = s_kept;
+    const int m2 = pow2_at_least(m > 1 ? m : 1);
+    for (int i = m + threadIdx.x; i < m2; i += blockDim.x) ranked[i] = kNone;
+    block_bitonic_sort_asc(ranked, m2);
+    const int nrun = min(m, K);
+    for (int i = threadIdx.x; i < K; i += blockDim.x) {
+        int64_t id = -1;
+        float sc = -__int_as_float(0x7f800000);
+        if (i < nrun) key_decode(~ranked[i], id, sc);
+        out_ids[(int64_t)q * K + i] = id;
+        out_scores[(int64_t)q * K + i] = sc;
+    }
+}
+
 }  // namespace
 
 
@@ -238,6 +292,30 @@ cudaError_t launch_merge_lists(const uint64_t *lists, int G, int64_t g_stride, i
 }
 
 int question_merge_capacity() { return kQCap; }
+
+cudaError_t launch_merge_regions_questions(const uint64_t *lists, int G, int64_t g_stride, int R, int k,
+                                           const int32_t *offsets, int Q, int K, int64_t *out_ids,
+                                           float *out_scores, int *err, cudaStream_t s, bool pdl) {
+    if (Q <= 0) return cudaSuccess;
+    if ((int64_t)R * k > kQCap || K > kQCap || G > 512) return cudaErrorInvalidValue;
+    const int smem = 2 * kQCap * (int)sizeof(uint64_t);
+    auto kern = G <= 32 ? k_merge_regions_questions<1> : G <= 64 ? k_merge_regions_questions<2>
+              : G <= 128 ? k_merge_regions_questions<4> : G <= 256 ? k_merge_regions_questions<8>
+                         : k_merge_regions_questions<16>;
+    cudaError_t e = cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, smem);
+    if (e != cudaSuccess) return e;
+    cudaLaunchConfig_t cfg = {};
+    cfg.gridDim = dim3((unsigned)Q, 1, 1);
+    cfg.blockDim = dim3(kQThreads, 1, 1);
+    cfg.dynamicSmemBytes = smem;
+    cfg.stream = s;
+    cudaLaunchAttribute attr[1];
+    attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+    attr[0].val.programmaticStreamSerializationAllowed = 1;
+    cfg.attrs = attr;
+    cfg.numAttrs = pdl ? 1 : 0;
+    return cudaLaunchKernelEx(&cfg, kern, lists, G, g_stride, k, offsets, R, K, out_ids, out_scores, err);
+}
 
 cudaError_t launch_question_merge(const uint64_t *reg_keys, int k, const int32_t *offsets, int Q,
                                   int R, int K, int64_t *out_ids, float *out_scores, int *err,

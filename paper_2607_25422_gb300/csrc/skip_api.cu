@@ -278,9 +278,19 @@ skip_status_t check_common(skip_corpus *c, const void *regions, int32_t R_total,
 // skip_retrieve and skip_retrieve_regions.
 // When keys_out is non-null the keys go to the head of the workspace (the
 // first ws_extra bytes) and *keys_out receives their address.
+// The question merge that run_regions may do itself (small batches: one
+// launch for both merges); `done` tells the caller whether it did.
+struct QuestionMerge {
+    const int32_t *offsets;
+    int Q, K;
+    int64_t *out_ids;
+    float *out_scores;
+    bool done = false;
+};
+
 skip_status_t run_regions(skip_corpus *c, const uint16_t *regions, int R, int k, uint64_t **keys_out,
                           int64_t *reg_ids, float *reg_scores, cudaStream_t s, Plan &pl,
-                          size_t ws_extra) {
+                          size_t ws_extra, QuestionMerge *qm = nullptr) {
     uint64_t *reg_keys = nullptr;
     const bool e4m3 = c->dtype == SKIP_E4M3;
     const int ctas = c->grid > 0 ? c->grid : c->sm_count;
@@ -351,6 +361,19 @@ skip_status_t run_regions(skip_corpus *c, const uint16_t *regions, int R, int k,
         cudaError_t e = launch_latency(e4m3, ta, tb, p, pl.grid, s);
         if (e != cudaSuccess) return cuda_status(e);
         ++pl.launches;
+        // One block per question merges all its region rows: only while the
+        // questions average at most 8 regions (one question of 32 regions,
+        // merged by one block, took 28 us against 23 us for the two launches).
+        if (qm && qm->Q > 0 && R <= 8 * qm->Q && (int64_t)R * k <= question_merge_capacity() &&
+            qm->K <= question_merge_capacity() && pl.G <= 512) {
+            record(c, s, "merge_regions_questions");
+            e = launch_merge_regions_questions(lists, pl.G, (int64_t)R * k, R, k, qm->offsets, qm->Q, qm->K,
+                                               qm->out_ids, qm->out_scores, c->err, s, true);
+            if (e != cudaSuccess) return cuda_status(e);
+            ++pl.launches;
+            qm->done = true;
+            return SKIP_OK;
+        }
         record(c, s, "merge_lists");
         e = launch_merge_lists(lists, pl.G, (int64_t)R * k, R, k, reg_keys, reg_ids, reg_scores, s, true);
         if (e != cudaSuccess) return cuda_status(e);
@@ -657,16 +680,22 @@ skip_status_t retrieve_impl(skip_corpus *c, const void *regions, const int32_t *
     const size_t keys_bytes = align_up((size_t)std::max(R_total, 1) * k_region * sizeof(uint64_t), 256);
     uint64_t *reg_keys = nullptr;
     skip_status_t st;
+    QuestionMerge qm;
+    qm.offsets = region_offsets;
+    qm.Q = Q;
+    qm.K = K;
+    qm.out_ids = out_ids;
+    qm.out_scores = out_scores;
     if (R_total > 0) {
         st = run_regions(c, reinterpret_cast<const uint16_t *>(regions), R_total, k_region, &reg_keys,
-                         nullptr, nullptr, s, pl, keys_bytes);
+                         nullptr, nullptr, s, pl, keys_bytes, &qm);
         if (st) return st;
     } else {
         st = ensure_ws(c, keys_bytes);
         if (st) return st;
         reg_keys = reinterpret_cast<uint64_t *>(c->ws);
     }
-    if (Q > 0) {
+    if (Q > 0 && !qm.done) {
         record(c, s, "question_merge");
         cudaError_t e = launch_question_merge(reg_keys, k_region, region_offsets, Q, R_total, K, out_ids,
                                               out_scores, c->err, s, R_total > 0);

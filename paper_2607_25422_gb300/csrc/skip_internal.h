@@ -140,6 +140,13 @@ cudaError_t launch_gemm2_bf16_f32(const CUtensorMap &ta, const CUtensorMap &tb, 
 // decoded ids/scores).  pdl (here and below): launched as the programmatic
 // dependent of the kernel just before it in the stream (the merge waits for
 // it before reading, and lets the next kernel launch early).
+int question_merge_capacity();
+// Both merges in one launch (small batches): per question, the k-way merge
+// of each of its region rows' G lists, then dedup / rank / cut to K.
+// Requires R k <= question_merge_capacity(), K <= the same, G <= 512.
+cudaError_t launch_merge_regions_questions(const uint64_t *lists, int G, int64_t g_stride, int R, int k,
+                                           const int32_t *offsets, int Q, int K, int64_t *out_ids,
+                                           float *out_scores, int *err, cudaStream_t s, bool pdl);
 cudaError_t launch_merge_lists(const uint64_t *lists, int G, int64_t g_stride, int R, int k,
                                uint64_t *reg_keys, int64_t *reg_ids, float *reg_scores,
                                cudaStream_t s, bool pdl = false);
