@@ -5,8 +5,8 @@
 //                for all questions at once, on the tensor cores (k_gemm.cu).
 //  k_skv_mlp     per 128 passage slots x 128 hidden units: the passage part
 //                of layer 1 on the tensor cores.  The A operand is built in
-//                shared memory by eight warps (two per slot row, each with
-//                three chunks of its row in flight) from the gathered corpus
+//                shared memory by sixteen warps (four threads per slot row,
+//                each with three chunks of its row in flight) from the gathered corpus
 //                rows and qbar: per 64-column chunk of d, three K-slices
 //                e | bf16(e * qbar) | bf16(|e - qbar|) in the 128-byte
 //                swizzled layout TMA would produce, one slice per stage of a
@@ -41,7 +41,9 @@ constexpr int kSkvStageA = kSkvSlice;
 constexpr int kSkvStageB = kSkvSlice;
 constexpr int kSkvStagesA = 4;
 constexpr int kSkvStagesB = 8;
-constexpr int kSkvBuilders = 8;                     // two builder warps per TMEM lane quadrant
+constexpr int kSkvBuilders = 16;                    // four builder warps per TMEM lane quadrant
+constexpr int kSkvParts = kSkvBuilders / 4;          // builder threads per slot row
+constexpr int kSkvWords = 8 / kSkvParts;             // 16-byte words of a 64-column chunk per thread
 constexpr int kSkvThreads = 64 + 32 * kSkvBuilders;  // TMA warp, MMA warp, builders (4 of them: epilogue)
 constexpr int kSkvAhead = 3;                         // chunks of corpus row in flight per builder thread
 constexpr uint32_t kSkvIdesc = idesc_bf16_f32(128, kSkvHidden);
@@ -167,11 +169,13 @@ __global__ void __launch_bounds__(kSkvThreads, 1)
         }
     } else {
         // ------------------------------------------------ builders, then epilogue
-        // Builder warps w and w + 4 share a TMEM lane quadrant: each thread
-        // owns one slot row and half of every 64-column chunk (16-byte words
-        // 4 h .. 4 h + 3), and keeps the next kSkvAhead chunks of its corpus
-        // row and qbar in flight in registers.
-        const int bw = warp - 2, half = bw >> 2;
+        // Builder warps w, w + 4, w + 8 and w + 12 share a TMEM lane
+        // quadrant: each thread owns one slot row and a quarter of every
+        // 64-column chunk (16-byte words kSkvWords part ...), and keeps the
+        // next kSkvAhead chunks of its corpus row and qbar in flight in
+        // registers.  (Four threads a row instead of two: the builds set the
+        // kernel's pace, the MMAs take a tenth of it.)
+        const int bw = warp - 2, part = bw >> 2;
         const int r = (warp & 3) * 32 + lane;  // TMEM lane = slot row in the tile
         const int64_t slot = m0 + r;
         int64_t id = -1;
@@ -180,27 +184,28 @@ __global__ void __launch_bounds__(kSkvThreads, 1)
             id = p.ids[slot];
             q = (int)(slot / p.K);
             if (id >= p.N) {
-                if (half == 0) atomicOr(p.err, kErrConfig);
+                if (part == 0) atomicOr(p.err, kErrConfig);
                 id = -1;
             }
         }
-        const uint4 *erow = reinterpret_cast<const uint4 *>(p.rows + (id < 0 ? 0 : id) * (int64_t)p.d) + 4 * half;
-        const uint4 *qrow = reinterpret_cast<const uint4 *>(p.qbar + (int64_t)q * p.d) + 4 * half;
+        const uint4 *erow =
+            reinterpret_cast<const uint4 *>(p.rows + (id < 0 ? 0 : id) * (int64_t)p.d) + kSkvWords * part;
+        const uint4 *qrow = reinterpret_cast<const uint4 *>(p.qbar + (int64_t)q * p.d) + kSkvWords * part;
         const uint4 zero = make_uint4(0, 0, 0, 0);
-        uint4 eb[kSkvAhead][4], qb[kSkvAhead][4];
+        uint4 eb[kSkvAhead][kSkvWords], qb[kSkvAhead][kSkvWords];
 #pragma unroll
         for (int a = 0; a < kSkvAhead; ++a)
 #pragma unroll
-            for (int j = 0; j < 4; ++j) {
+            for (int j = 0; j < kSkvWords; ++j) {
                 const bool ld = id >= 0 && a < nc;
                 eb[a][j] = ld ? __ldg(erow + a * 8 + j) : zero;
                 qb[a][j] = ld ? __ldg(qrow + a * 8 + j) : zero;
             }
         bool ok = true;
         for (int c = 0; c < nc; ++c) {
-            uint4 e[4], qv[4];
+            uint4 e[kSkvWords], qv[kSkvWords];
 #pragma unroll
-            for (int j = 0; j < 4; ++j) {
+            for (int j = 0; j < kSkvWords; ++j) {
                 e[j] = eb[0][j];
                 qv[j] = qb[0][j];
             }
@@ -208,7 +213,7 @@ __global__ void __launch_bounds__(kSkvThreads, 1)
 #pragma unroll
             for (int a = 0; a + 1 < kSkvAhead; ++a)
 #pragma unroll
-                for (int j = 0; j < 4; ++j) {
+                for (int j = 0; j < kSkvWords; ++j) {
                     eb[a][j] = eb[a + 1][j];
                     qb[a][j] = qb[a + 1][j];
                 }
@@ -216,14 +221,14 @@ __global__ void __launch_bounds__(kSkvThreads, 1)
                 const int cn = c + kSkvAhead;
                 const bool ld = id >= 0 && cn < nc;
 #pragma unroll
-                for (int j = 0; j < 4; ++j) {
+                for (int j = 0; j < kSkvWords; ++j) {
                     eb[kSkvAhead - 1][j] = ld ? __ldg(erow + cn * 8 + j) : zero;
                     qb[kSkvAhead - 1][j] = ld ? __ldg(qrow + cn * 8 + j) : zero;
                 }
             }
-            uint4 f[3][4];  // the chunk's three K-slices of this thread's half row
+            uint4 f[3][kSkvWords];  // the chunk's three K-slices of this thread's part of the row
 #pragma unroll
-            for (int jj = 0; jj < 4; ++jj) {
+            for (int jj = 0; jj < kSkvWords; ++jj) {
                 f[0][jj] = e[jj];
                 features2(e[jj].x, qv[jj].x, f[1][jj].x, f[2][jj].x);
                 features2(e[jj].y, qv[jj].y, f[1][jj].y, f[2][jj].y);
@@ -243,7 +248,8 @@ __global__ void __launch_bounds__(kSkvThreads, 1)
                 }
                 const uint32_t base = smem_addr(sA + s * kSkvStageA) + r * 128;
 #pragma unroll
-                for (int jj = 0; jj < 4; ++jj) sts128(base + (uint32_t)(((4 * half + jj) ^ sw) << 4), f[b][jj]);
+                for (int jj = 0; jj < kSkvWords; ++jj)
+                    sts128(base + (uint32_t)(((kSkvWords * part + jj) ^ sw) << 4), f[b][jj]);
                 // each writer makes its stores visible to the tensor core's
                 // (async) proxy, then one arrival per warp: 257 arrivals on
                 // one barrier per slice were serialised
@@ -255,7 +261,7 @@ __global__ void __launch_bounds__(kSkvThreads, 1)
         }
         if (!ok) atomicOr(p.err, kErrTimeout);
         // Epilogue: h = acc + c_q, ReLU, dot with w2 over this CTA's units.
-        if (half == 0) {
+        if (part == 0) {
             const bool done = mbar_wait(smem_addr(&sh->tfull), 0, p.timeout_ns);
             if (!done) atomicOr(p.err, kErrTimeout);
             tc_fence_after();
@@ -282,8 +288,10 @@ __global__ void __launch_bounds__(kSkvThreads, 1)
             asm volatile("bar.sync 1, %0;" ::"r"(kSkvRows) : "memory");  // the four epilogue warps
             if (done) {
                 const uint32_t lane_addr = (uint32_t)((warp & 3) * 32) << 16;
-                // rows past the last slot (q = 0) read question q0's entries and write nothing
-                const float *cq = cqs + (slot < p.P ? q - q0 : 0) * kSkvHidden;
+                // rows past the last slot (q = 0) read question q0's entries and write
+                // nothing; the index is clamped to the staged questions in any case
+                const int qq = slot < p.P ? q - q0 : 0;
+                const float *cq = cqs + (qq < 0 ? 0 : qq >= nq ? (nq > 0 ? nq - 1 : 0) : qq) * kSkvHidden;
                 const float *w2 = p.w2 + n0;
                 float part = 0.f;
 #pragma unroll 1
