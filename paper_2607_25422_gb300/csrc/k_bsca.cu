@@ -238,6 +238,7 @@ __global__ void __launch_bounds__(kSelThreads) k_bsca_select(const BscaParams p)
     __shared__ uint32_t wsum[kSelThreads / 32];
     __shared__ int s_bin, s_rank, s_cnt, s_found;
     __shared__ float s_tau;
+    grid_dep_wait();  // the cosines and histograms of k_bsca_cos
     const int q = blockIdx.x;
     const int i0 = p.vis_offsets[q], P = p.vis_offsets[q + 1] - i0;
     const int R = p.chunk_offsets[q + 1] - p.chunk_offsets[q];
@@ -344,6 +345,7 @@ constexpr int kAttSlots = 2;
 constexpr int kAttGroup = 4;  // neighbours whose rows are read together
 
 __global__ void __launch_bounds__(32 * kAttWarps) k_bsca_attend(const BscaParams p, int S) {
+    grid_dep_wait();  // the thresholds (and, through k_bsca_select, the cosines)
     const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
     const int q = blockIdx.x / S, sl = blockIdx.x - q * S;
     const int i0 = p.vis_offsets[q], P = p.vis_offsets[q + 1] - i0;
@@ -542,6 +544,24 @@ __global__ void __launch_bounds__(32 * kAttWarps) k_bsca_attend(const BscaParams
 
 }  // namespace
 
+// Launch as the programmatic dependent of the previous kernel in the stream
+// (its launch overlaps that kernel's tail; it waits for its results).
+template <typename... Args>
+cudaError_t launch_dependent(void (*kern)(Args...), dim3 grid, int threads, size_t smem, cudaStream_t s,
+                             Args... args) {
+    cudaLaunchConfig_t cfg = {};
+    cfg.gridDim = grid;
+    cfg.blockDim = dim3((unsigned)threads);
+    cfg.dynamicSmemBytes = smem;
+    cfg.stream = s;
+    cudaLaunchAttribute attr[1];
+    attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+    attr[0].val.programmaticStreamSerializationAllowed = 1;
+    cfg.attrs = attr;
+    cfg.numAttrs = 1;
+    return cudaLaunchKernelEx(&cfg, kern, args...);
+}
+
 cudaError_t launch_bsca(const BscaParams &p, cudaStream_t s) {
     if (p.Q == 0) return cudaSuccess;
     // slices per question from the mean tokens per question: about 32 tokens
@@ -557,15 +577,13 @@ cudaError_t launch_bsca(const BscaParams &p, cudaStream_t s) {
     const size_t smem2 = (size_t)kBscaMaxPairs * sizeof(float);
     e = cudaFuncSetAttribute(k_bsca_select, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem2);
     if (e != cudaSuccess) return e;
-    k_bsca_select<<<(unsigned)p.Q, kSelThreads, smem2, s>>>(p);
-    if ((e = cudaGetLastError()) != cudaSuccess) {
+    if ((e = launch_dependent(k_bsca_select, dim3((unsigned)p.Q), kSelThreads, smem2, s, p)) != cudaSuccess) {
         // the select clears the histograms; without it they must be cleared here
         cudaMemsetAsync(p.hist, 0, (size_t)p.Q * kBscaBins * sizeof(uint32_t), s);
         return e;
     }
     if (p.Nv == 0) return e;
-    k_bsca_attend<<<(unsigned)(p.Q * S3), 32 * kAttWarps, 0, s>>>(p, S3);
-    return cudaGetLastError();
+    return launch_dependent(k_bsca_attend, dim3((unsigned)(p.Q * S3)), 32 * kAttWarps, (size_t)0, s, p, S3);
 }
 
 }  // namespace skipk
