@@ -722,23 +722,32 @@ def main():
     ms_ev_local, kernels = run_timed(True)
     ms = max_over_ranks(ms_local, world)
     ms_ev = max_over_ranks(ms_ev_local, world)
-    plain_ms = None
+    gate_delta_ms = None
     if args.skv:
-        # the same batch without the gate, timed the same way in this process:
-        # the gate's cost in the step with its launches overlapped
+        # the gate's cost in the step with its launches overlapped: the same
+        # batch with and without the gate, in alternating blocks of steps (so
+        # that clock drift under the power cap falls on both alike)
         def plain():
             skip.skip_retrieve(c, reg_d, off_d, spec.k_region, spec.K, out_ids, out_sc, stream)
         for _ in range(args.warmup):
             plain()
         torch.cuda.synchronize()
-        e0 = torch.cuda.Event(enable_timing=True)
-        e1 = torch.cuda.Event(enable_timing=True)
-        e0.record(stream)
-        for _ in range(args.steps):
-            plain()
-        e1.record(stream)
-        torch.cuda.synchronize()
-        plain_ms = max_over_ranks(e0.elapsed_time(e1), world)
+        t_plain = t_gate = 0.0
+        for fn_is_gate in [False, True] * 5:
+            fn = step if fn_is_gate else plain
+            e0 = torch.cuda.Event(enable_timing=True)
+            e1 = torch.cuda.Event(enable_timing=True)
+            e0.record(stream)
+            for _ in range(max(1, args.steps // 5)):
+                fn()
+            e1.record(stream)
+            torch.cuda.synchronize()
+            if fn_is_gate:
+                t_gate += e0.elapsed_time(e1)
+            else:
+                t_plain += e0.elapsed_time(e1)
+        n_each = 5 * max(1, args.steps // 5)
+        gate_delta_ms = max_over_ranks((t_gate - t_plain) / n_each, world)
 
     # ---- end to end through the host-buffer entry point
     reg_h = regions.pin_memory()
@@ -851,8 +860,7 @@ def main():
         mlp = kernels.get("skv_mlp", {"ms": float("nan"), "launches": 1})
         mlp_ms = mlp["ms"] / max(1, mlp["launches"])
         line["skv"] = {"gate_ms_per_step": skv_ms, "mlp_kernel_ms": mlp_ms,
-                       "step_ms_without_gate": plain_ms / args.steps,
-                       "gate_step_delta_ms": (ms - plain_ms) / args.steps,
+                       "gate_step_delta_ms": gate_delta_ms,
                        "mlp_algorithmic_flops": 2.0 * P * 3 * spec.d * H,
                        "mlp_tflops": 2.0 * P * 3 * spec.d * H / (mlp_ms / 1e3) / 1e12,
                        "gate_share_of_step": skv_ms / (ms / args.steps), "algorithmic_flops": skv_flops}

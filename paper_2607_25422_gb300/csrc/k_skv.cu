@@ -3,21 +3,19 @@
 //
 //  (k_gemm)      per question: c_q = b1 + W1[:, qbar] qbar + W1[:, vbar] vbar
 //                for all questions at once, on the tensor cores (k_gemm.cu).
+//  k_skv_features per passage slot: F = [e | bf16(e * qbar) | bf16(|e - qbar|)]
+//                (3d bf16 in the column order of W1's passage blocks), from
+//                the gathered corpus row and qbar; zeros for an empty slot.
+//                Runs while the c_q GEMM runs (programmatic dependent).
 //  k_skv_mlp     per 128 passage slots x 128 hidden units: the passage part
-//                of layer 1 on the tensor cores.  The A operand is built in
-//                shared memory by sixteen warps (four threads per slot row,
-//                each with three chunks of its row in flight) from the gathered corpus
-//                rows and qbar: per 64-column chunk of d, three K-slices
-//                e | bf16(e * qbar) | bf16(|e - qbar|) in the 128-byte
-//                swizzled layout TMA would produce, one slice per stage of a
-//                four-stage ring; the B operand is the matching W1 column
-//                block, loaded by TMA into an eight-stage ring of its own.
-//                Launched as the programmatic dependent of the c_q GEMM: it
-//                gathers and multiplies while the GEMM runs and waits for c_q
-//                only in its epilogue.  tcgen05.mma
-//                (kind::f16, M = N = 128) accumulates in TMEM; the epilogue
-//                adds c_q, applies ReLU and the w2 dot for its 128 units and
-//                writes one partial logit per slot and hidden block.
+//                of layer 1 on the tensor cores, both operands by TMA (the
+//                feature rows and the matching W1 column blocks) into a
+//                six-stage ring; tcgen05.mma (kind::f16, M = N = 128)
+//                accumulates in TMEM; the epilogue adds c_q, applies ReLU
+//                and the w2 dot for its 128 units and writes one partial
+//                logit per slot and hidden block.  (Building the features in
+//                shared memory inside this kernel instead, once per hidden
+//                block, made the builders and their hand-offs set the pace.)
 //  k_skv_select  per question: logit = b2 + sum of the partial logits,
 //                nu = sigmoid(logit), gate nu >= tau, then the first
 //                ceil(rho |K| - 1e-3) by (nu desc, id asc) (bitonic sort).
@@ -33,40 +31,22 @@ namespace {
 
 constexpr int kSkvRows = 128;                       // passage slots per CTA (TMEM lanes)
 constexpr int kSkvSlice = kSkvRows * 128;           // one [128 x 64] bf16 K-slice, bytes
-// A stage holds one K-slice of A (e, e*qbar or |e - qbar| of one 64-column
-// chunk of d) or of B (the matching W1 column block for 128 units).  The two
-// rings are separate: B, whose TMA copy from L2 takes microseconds, runs
-// eight slices ahead; A, built from rows the builders already hold, four.
+// A stage holds one K-slice of A (64 feature columns of 128 slots) and of B
+// (the matching W1 column block for 128 units), both copied by TMA.
 constexpr int kSkvStageA = kSkvSlice;
 constexpr int kSkvStageB = kSkvSlice;
-constexpr int kSkvStagesA = 4;
-constexpr int kSkvStagesB = 8;
-constexpr int kSkvBuilders = 16;                    // four builder warps per TMEM lane quadrant
-constexpr int kSkvParts = kSkvBuilders / 4;          // builder threads per slot row
-constexpr int kSkvWords = 8 / kSkvParts;             // 16-byte words of a 64-column chunk per thread
-constexpr int kSkvThreads = 64 + 32 * kSkvBuilders;  // TMA warp, MMA warp, builders (4 of them: epilogue)
-constexpr int kSkvAhead = 3;                         // chunks of corpus row in flight per builder thread
+constexpr int kSkvStages = 6;
+constexpr int kSkvThreads = 192;                     // TMA warp, MMA warp, four epilogue warps
 constexpr uint32_t kSkvIdesc = idesc_bf16_f32(128, kSkvHidden);
 constexpr uint64_t kDrainTimeoutNs = 1000000000ull;  // 1 s for copies in flight
+constexpr int kFeatWarps = 8;                        // slots per feature block
 
 struct SkvShared {
-    uint64_t fullA[kSkvStagesA];   // A built (one arrival per builder warp)
-    uint64_t emptyA[kSkvStagesA];  // A stage consumed (tcgen05.commit)
-    uint64_t fullB[kSkvStagesB];   // B landed (tx bytes)
-    uint64_t emptyB[kSkvStagesB];  // B stage consumed (tcgen05.commit)
+    uint64_t full[kSkvStages];   // A and B slices landed (tx bytes)
+    uint64_t empty[kSkvStages];  // stage consumed (tcgen05.commit)
     uint64_t tfull;              // accumulator complete
     uint32_t tmem_base;
 };
-
-__device__ __forceinline__ void sts128(uint32_t addr, uint4 v) {
-    asm volatile("st.shared.v4.b32 [%0], {%1, %2, %3, %4};" ::"r"(addr), "r"(v.x), "r"(v.y), "r"(v.z),
-                 "r"(v.w)
-                 : "memory");
-}
-
-__device__ __forceinline__ void fence_proxy_async_smem() {
-    asm volatile("fence.proxy.async.shared::cta;" ::: "memory");
-}
 
 // Two bf16 lanes of a 32-bit word -> the two interaction features, rounded
 // to bf16 (ties to even).
@@ -83,31 +63,76 @@ __device__ __forceinline__ void features2(uint32_t e2, uint32_t q2, uint32_t &eq
     ad2 = *reinterpret_cast<const uint32_t *>(&a);
 }
 
+// F[slot] = [e | bf16(e * qbar) | bf16(|e - qbar|)] (3d bf16, the column
+// order of W1's passage blocks), zeros for an empty slot; a warp per slot,
+// 16-byte loads and stores.  Launched as the programmatic dependent of the
+// c_q GEMM: it gathers while the GEMM runs and, before it completes, waits
+// for the GEMM, so that a kernel waiting for this grid also sees c_q.
+__global__ void __launch_bounds__(32 * kFeatWarps) k_skv_features(const SkvParams p, uint16_t *__restrict__ F) {
+    const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+    const int64_t slot = (int64_t)blockIdx.x * kFeatWarps + warp;
+    if (slot < p.P) {
+        int64_t id = p.ids[slot];
+        if (id >= p.N) {
+            if (lane == 0) atomicOr(p.err, kErrConfig);
+            id = -1;
+        }
+        const int q = (int)(slot / p.K);
+        const int nw = p.d / 8;  // 16-byte words of a row
+        const uint4 *erow = reinterpret_cast<const uint4 *>(p.rows + (id < 0 ? 0 : id) * (int64_t)p.d);
+        const uint4 *qrow = reinterpret_cast<const uint4 *>(p.qbar + (int64_t)q * p.d);
+        uint4 *f = reinterpret_cast<uint4 *>(F + slot * 3 * (int64_t)p.d);
+        const uint4 zero = make_uint4(0, 0, 0, 0);
+        for (int w0 = 0; w0 < nw; w0 += 64) {
+            uint4 e[2], qv[2];
+#pragma unroll
+            for (int h = 0; h < 2; ++h) {
+                const int w = w0 + lane + 32 * h;
+                e[h] = (id >= 0 && w < nw) ? __ldg(erow + w) : zero;
+                qv[h] = (id >= 0 && w < nw) ? __ldg(qrow + w) : zero;
+            }
+#pragma unroll
+            for (int h = 0; h < 2; ++h) {
+                const int w = w0 + lane + 32 * h;
+                if (w >= nw) continue;
+                uint4 m, a;
+                features2(e[h].x, qv[h].x, m.x, a.x);
+                features2(e[h].y, qv[h].y, m.y, a.y);
+                features2(e[h].z, qv[h].z, m.z, a.z);
+                features2(e[h].w, qv[h].w, m.w, a.w);
+                f[w] = e[h];
+                f[nw + w] = m;
+                f[2 * nw + w] = a;
+            }
+        }
+    }
+    grid_dep_wait();
+}
+
 __global__ void __launch_bounds__(kSkvThreads, 1)
-    k_skv_mlp(const __grid_constant__ CUtensorMap tw, const SkvParams p) {
+    k_skv_mlp(const __grid_constant__ CUtensorMap tf, const __grid_constant__ CUtensorMap tw, const SkvParams p) {
     extern __shared__ __align__(1024) uint8_t smem_raw[];
     uint8_t *smem = reinterpret_cast<uint8_t *>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
     uint8_t *sA = smem;
-    uint8_t *sB = smem + kSkvStagesA * kSkvStageA;
-    SkvShared *sh = reinterpret_cast<SkvShared *>(sB + kSkvStagesB * kSkvStageB);
+    uint8_t *sB = smem + kSkvStages * kSkvStageA;
+    SkvShared *sh = reinterpret_cast<SkvShared *>(sB + kSkvStages * kSkvStageB);
     const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
     const int64_t m0 = (int64_t)blockIdx.x * kSkvRows;
     const int n0 = blockIdx.y * kSkvHidden;
-    const int nc = p.d / 64;
+    const int nsl = 3 * (p.d / 64);  // K-slices: 3d / 64
 
     if (threadIdx.x == 0) {
-        for (int s = 0; s < kSkvStagesA; ++s) {
-            mbar_init(smem_addr(&sh->fullA[s]), kSkvBuilders);  // one arrival per builder warp
-            mbar_init(smem_addr(&sh->emptyA[s]), 1);
-        }
-        for (int s = 0; s < kSkvStagesB; ++s) {
-            mbar_init(smem_addr(&sh->fullB[s]), 1);
-            mbar_init(smem_addr(&sh->emptyB[s]), 1);
+        for (int s = 0; s < kSkvStages; ++s) {
+            mbar_init(smem_addr(&sh->full[s]), 1);
+            mbar_init(smem_addr(&sh->empty[s]), 1);
         }
         mbar_init(smem_addr(&sh->tfull), 1);
         mbar_fence_init();
     }
-    if (warp == 0 && lane == 0) tma_prefetch_desc(&tw);
+    if (warp == 0 && lane == 0) {
+        tma_prefetch_desc(&tf);
+        tma_prefetch_desc(&tw);
+    }
     if (warp == 1) {
         tmem_alloc(smem_addr(&sh->tmem_base), kSkvHidden);
         tmem_relinquish();
@@ -118,28 +143,31 @@ __global__ void __launch_bounds__(kSkvThreads, 1)
     const uint32_t tmem = sh->tmem_base;
 
     if (warp == 0) {
-        // ------------------------------------------------ TMA: W1 column blocks
+        // ------------------------------------------------ TMA: features and W1 blocks
         if (lane == 0) {
+            // the features (and through them c_q) come from the kernels before this one
+            grid_dep_wait();
             bool ok = true;
             int issued = 0;
-            for (int u = 0; u < 3 * nc && ok; ++u) {
-                const int s = u % kSkvStagesB, c = u / 3, b = u - 3 * c;
-                const uint32_t ph = (uint32_t)(u / kSkvStagesB) & 1u;
-                if (!mbar_wait(smem_addr(&sh->emptyB[s]), ph ^ 1u, p.timeout_ns)) {
+            for (int u = 0; u < nsl && ok; ++u) {
+                const int s = u % kSkvStages;
+                const uint32_t ph = (uint32_t)(u / kSkvStages) & 1u;
+                if (!mbar_wait(smem_addr(&sh->empty[s]), ph ^ 1u, p.timeout_ns)) {
                     ok = false;
                     break;
                 }
-                const uint32_t fb = smem_addr(&sh->fullB[s]);
-                mbar_arrive_expect_tx(fb, kSkvStageB);
-                tma_load_2d(smem_addr(sB + s * kSkvStageB), &tw, fb, (2 + b) * p.d + c * 64, n0);
+                const uint32_t fb = smem_addr(&sh->full[s]);
+                mbar_arrive_expect_tx(fb, kSkvStageA + kSkvStageB);
+                tma_load_2d(smem_addr(sA + s * kSkvStageA), &tf, fb, u * 64, (int)m0);
+                tma_load_2d(smem_addr(sB + s * kSkvStageB), &tw, fb, 2 * p.d + u * 64, n0);
                 ++issued;
             }
             if (!ok) atomicOr(p.err, kErrTimeout);
             // Copies in flight: wait for the last use of each stage to complete.
-            for (int s = 0; s < kSkvStagesB; ++s) {
-                const int uses = issued / kSkvStagesB + (s < issued % kSkvStagesB ? 1 : 0);
+            for (int s = 0; s < kSkvStages; ++s) {
+                const int uses = issued / kSkvStages + (s < issued % kSkvStages ? 1 : 0);
                 if (uses == 0) continue;
-                if (!mbar_wait(smem_addr(&sh->fullB[s]), (uint32_t)((uses - 1) & 1), kDrainTimeoutNs))
+                if (!mbar_wait(smem_addr(&sh->full[s]), (uint32_t)((uses - 1) & 1), kDrainTimeoutNs))
                     atomicOr(p.err, kErrTimeout);
             }
         }
@@ -147,166 +175,71 @@ __global__ void __launch_bounds__(kSkvThreads, 1)
         // ------------------------------------------------ MMA issuer
         if (lane == 0) {
             bool ok = true;
-            for (int u = 0; u < 3 * nc && ok; ++u) {
-                const int sa = u % kSkvStagesA, sb = u % kSkvStagesB;
-                if (!mbar_wait(smem_addr(&sh->fullA[sa]), (uint32_t)(u / kSkvStagesA) & 1u, p.timeout_ns) ||
-                    !mbar_wait(smem_addr(&sh->fullB[sb]), (uint32_t)(u / kSkvStagesB) & 1u, p.timeout_ns)) {
+            for (int u = 0; u < nsl && ok; ++u) {
+                const int s = u % kSkvStages;
+                if (!mbar_wait(smem_addr(&sh->full[s]), (uint32_t)(u / kSkvStages) & 1u, p.timeout_ns)) {
                     ok = false;
                     break;
                 }
                 tc_fence_after();
-                const uint64_t ad = smem_desc_k128(smem_addr(sA + sa * kSkvStageA));
-                const uint64_t bd = smem_desc_k128(smem_addr(sB + sb * kSkvStageB));
+                const uint64_t ad = smem_desc_k128(smem_addr(sA + s * kSkvStageA));
+                const uint64_t bd = smem_desc_k128(smem_addr(sB + s * kSkvStageB));
 #pragma unroll
                 for (int kk = 0; kk < 4; ++kk)
                     tc_mma_f16(tmem, ad + (uint64_t)(kk * 2), bd + (uint64_t)(kk * 2), kSkvIdesc, (u | kk) != 0);
-                tc_commit(smem_addr(&sh->emptyA[sa]));
-                tc_commit(smem_addr(&sh->emptyB[sb]));
+                tc_commit(smem_addr(&sh->empty[s]));
             }
             if (!ok) atomicOr(p.err, kErrTimeout);
             // Arrives once every MMA issued has completed (also after a timeout).
             tc_commit(smem_addr(&sh->tfull));
         }
     } else {
-        // ------------------------------------------------ builders, then epilogue
-        // Builder warps w, w + 4, w + 8 and w + 12 share a TMEM lane
-        // quadrant: each thread owns one slot row and a quarter of every
-        // 64-column chunk (16-byte words kSkvWords part ...), and keeps the
-        // next kSkvAhead chunks of its corpus row and qbar in flight in
-        // registers.  (Four threads a row instead of two: the builds set the
-        // kernel's pace, the MMAs take a tenth of it.)
-        const int bw = warp - 2, part = bw >> 2;
+        // ------------------------------------------------ epilogue (warps 2..5)
+        // Epilogue: h = acc + c_q, ReLU, dot with w2 over this CTA's units.
         const int r = (warp & 3) * 32 + lane;  // TMEM lane = slot row in the tile
         const int64_t slot = m0 + r;
-        int64_t id = -1;
-        int q = 0;
-        if (slot < p.P) {
-            id = p.ids[slot];
-            q = (int)(slot / p.K);
-            if (id >= p.N) {
-                if (part == 0) atomicOr(p.err, kErrConfig);
-                id = -1;
+        const int q = slot < p.P ? (int)(slot / p.K) : 0;
+        const bool done = mbar_wait(smem_addr(&sh->tfull), 0, p.timeout_ns);
+        if (!done) atomicOr(p.err, kErrTimeout);
+        tc_fence_after();
+        grid_dep_wait();
+        // c_q of the tile's questions for this CTA's units, the GEMM's K-split
+        // slabs summed once, staged in the A ring (free: every MMA that read it
+        // has completed; its 96 KB hold 128 questions).  cqs[(q - q0) * 128 + n].
+        float *cqs = reinterpret_cast<float *>(sA);
+        const int q0 = (int)(m0 / p.K);
+        const int64_t last = (m0 + kSkvRows < p.P ? m0 + kSkvRows : p.P) - 1;
+        const int nq = m0 < p.P ? (int)(last / p.K) - q0 + 1 : 0;  // <= 128
+        const int et = (warp & 3) * 32 + lane;                      // 0..127
+        const int64_t slab = (int64_t)p.Q * p.H;
+        if (done)
+            for (int t = et; t < nq * kSkvHidden; t += kSkvRows) {
+                const float *src = p.cq + (int64_t)(q0 + t / kSkvHidden) * p.H + n0 + t % kSkvHidden;
+                float v = 0.f;
+                for (int z = 0; z < p.cq_splits; ++z) v += src[z * slab];
+                cqs[t] = v;
             }
-        }
-        const uint4 *erow =
-            reinterpret_cast<const uint4 *>(p.rows + (id < 0 ? 0 : id) * (int64_t)p.d) + kSkvWords * part;
-        const uint4 *qrow = reinterpret_cast<const uint4 *>(p.qbar + (int64_t)q * p.d) + kSkvWords * part;
-        const uint4 zero = make_uint4(0, 0, 0, 0);
-        uint4 eb[kSkvAhead][kSkvWords], qb[kSkvAhead][kSkvWords];
-#pragma unroll
-        for (int a = 0; a < kSkvAhead; ++a)
-#pragma unroll
-            for (int j = 0; j < kSkvWords; ++j) {
-                const bool ld = id >= 0 && a < nc;
-                eb[a][j] = ld ? __ldg(erow + a * 8 + j) : zero;
-                qb[a][j] = ld ? __ldg(qrow + a * 8 + j) : zero;
-            }
-        bool ok = true;
-        for (int c = 0; c < nc; ++c) {
-            uint4 e[kSkvWords], qv[kSkvWords];
-#pragma unroll
-            for (int j = 0; j < kSkvWords; ++j) {
-                e[j] = eb[0][j];
-                qv[j] = qb[0][j];
-            }
-            // rotate the prefetch ring and issue chunk c + kSkvAhead
-#pragma unroll
-            for (int a = 0; a + 1 < kSkvAhead; ++a)
-#pragma unroll
-                for (int j = 0; j < kSkvWords; ++j) {
-                    eb[a][j] = eb[a + 1][j];
-                    qb[a][j] = qb[a + 1][j];
-                }
-            {
-                const int cn = c + kSkvAhead;
-                const bool ld = id >= 0 && cn < nc;
-#pragma unroll
-                for (int j = 0; j < kSkvWords; ++j) {
-                    eb[kSkvAhead - 1][j] = ld ? __ldg(erow + cn * 8 + j) : zero;
-                    qb[kSkvAhead - 1][j] = ld ? __ldg(qrow + cn * 8 + j) : zero;
-                }
-            }
-            uint4 f[3][kSkvWords];  // the chunk's three K-slices of this thread's part of the row
-#pragma unroll
-            for (int jj = 0; jj < kSkvWords; ++jj) {
-                f[0][jj] = e[jj];
-                features2(e[jj].x, qv[jj].x, f[1][jj].x, f[2][jj].x);
-                features2(e[jj].y, qv[jj].y, f[1][jj].y, f[2][jj].y);
-                features2(e[jj].z, qv[jj].z, f[1][jj].z, f[2][jj].z);
-                features2(e[jj].w, qv[jj].w, f[1][jj].w, f[2][jj].w);
-            }
-            // Row r of each slice: 16-byte chunk j at position j ^ (r & 7).
-            const int sw = r & 7;
-#pragma unroll
-            for (int b = 0; b < 3; ++b) {
-                const int u = 3 * c + b, s = u % kSkvStagesA;
-                const uint32_t ph = (uint32_t)(u / kSkvStagesA) & 1u;
-                // warp-uniform: every lane waits (bounded), then the warp votes
-                if (!__all_sync(0xffffffffu, mbar_wait(smem_addr(&sh->emptyA[s]), ph ^ 1u, p.timeout_ns))) {
-                    ok = false;
-                    break;
-                }
-                const uint32_t base = smem_addr(sA + s * kSkvStageA) + r * 128;
-#pragma unroll
-                for (int jj = 0; jj < kSkvWords; ++jj)
-                    sts128(base + (uint32_t)(((kSkvWords * part + jj) ^ sw) << 4), f[b][jj]);
-                // each writer makes its stores visible to the tensor core's
-                // (async) proxy, then one arrival per warp: 257 arrivals on
-                // one barrier per slice were serialised
-                fence_proxy_async_smem();
-                __syncwarp();
-                if (lane == 0) mbar_arrive(smem_addr(&sh->fullA[s]));
-            }
-            if (!ok) break;
-        }
-        if (!ok) atomicOr(p.err, kErrTimeout);
-        // Epilogue: h = acc + c_q, ReLU, dot with w2 over this CTA's units.
-        if (part == 0) {
-            const bool done = mbar_wait(smem_addr(&sh->tfull), 0, p.timeout_ns);
-            if (!done) atomicOr(p.err, kErrTimeout);
-            tc_fence_after();
-            // c_q comes from the GEMM launched just before this kernel (whose
-            // programmatic dependent it is): wait for that grid here only.
-            grid_dep_wait();
-            // c_q of the tile's questions for this CTA's units, the GEMM's
-            // K-split slabs summed once, staged in the A ring (free: every
-            // MMA that read it has completed; 64 KB holds 128 questions).
-            // cqs[(q - q0) * 128 + n].
-            float *cqs = reinterpret_cast<float *>(sA);
-            const int q0 = (int)(m0 / p.K);
-            const int64_t last = (m0 + kSkvRows < p.P ? m0 + kSkvRows : p.P) - 1;
-            const int nq = m0 < p.P ? (int)(last / p.K) - q0 + 1 : 0;  // <= 128: fits the ring
-            const int et = (warp & 3) * 32 + lane;                      // 0..127
-            const int64_t slab = (int64_t)p.Q * p.H;
-            if (done)
-                for (int t = et; t < nq * kSkvHidden; t += kSkvRows) {
-                    const float *src = p.cq + (int64_t)(q0 + t / kSkvHidden) * p.H + n0 + t % kSkvHidden;
-                    float v = 0.f;
-                    for (int z = 0; z < p.cq_splits; ++z) v += src[z * slab];
-                    cqs[t] = v;
-                }
-            asm volatile("bar.sync 1, %0;" ::"r"(kSkvRows) : "memory");  // the four epilogue warps
-            if (done) {
-                const uint32_t lane_addr = (uint32_t)((warp & 3) * 32) << 16;
-                // rows past the last slot (q = 0) read question q0's entries and write
-                // nothing; the index is clamped to the staged questions in any case
-                const int qq = slot < p.P ? q - q0 : 0;
-                const float *cq = cqs + (qq < 0 ? 0 : qq >= nq ? (nq > 0 ? nq - 1 : 0) : qq) * kSkvHidden;
-                const float *w2 = p.w2 + n0;
-                float part = 0.f;
+        asm volatile("bar.sync 1, %0;" ::"r"(kSkvRows) : "memory");  // the four epilogue warps
+        if (done) {
+            const uint32_t lane_addr = (uint32_t)((warp & 3) * 32) << 16;
+            // rows past the last slot read question q0's entries and write nothing;
+            // the index is clamped to the staged questions in any case
+            const int qq = slot < p.P ? q - q0 : 0;
+            const float *cq = cqs + (qq < 0 ? 0 : qq >= nq ? (nq > 0 ? nq - 1 : 0) : qq) * kSkvHidden;
+            const float *w2 = p.w2 + n0;
+            float part = 0.f;
 #pragma unroll 1
-                for (int c = 0; c < kSkvHidden / 32; ++c) {
-                    uint32_t v[32];
-                    tmem_ld_32x32b_x32(tmem + lane_addr + c * 32, v);
-                    tmem_ld_wait(v);
+            for (int c = 0; c < kSkvHidden / 32; ++c) {
+                uint32_t v[32];
+                tmem_ld_32x32b_x32(tmem + lane_addr + c * 32, v);
+                tmem_ld_wait(v);
 #pragma unroll
-                    for (int i = 0; i < 32; ++i) {
-                        const float h = __uint_as_float(v[i]) + cq[c * 32 + i];
-                        part = fmaf(fmaxf(h, 0.f), __ldg(w2 + c * 32 + i), part);
-                    }
+                for (int i = 0; i < 32; ++i) {
+                    const float h = __uint_as_float(v[i]) + cq[c * 32 + i];
+                    part = fmaf(fmaxf(h, 0.f), __ldg(w2 + c * 32 + i), part);
                 }
-                if (slot < p.P) p.partial[(int64_t)blockIdx.y * p.P + slot] = part;
             }
+            if (slot < p.P) p.partial[(int64_t)blockIdx.y * p.P + slot] = part;
         }
     }
 
@@ -395,7 +328,7 @@ __global__ void __launch_bounds__(kSelThreads) k_skv_select(const SkvParams p) {
 }  // namespace
 
 size_t skv_mlp_smem_bytes() {
-    return 1024 + (size_t)kSkvStagesA * kSkvStageA + (size_t)kSkvStagesB * kSkvStageB + sizeof(SkvShared);
+    return 1024 + (size_t)kSkvStages * (kSkvStageA + kSkvStageB) + sizeof(SkvShared);
 }
 
 // Launch as the programmatic dependent of the previous kernel in the stream.
@@ -415,13 +348,19 @@ cudaError_t launch_dependent(void (*kern)(Args...), dim3 grid, int threads, size
     return cudaLaunchKernelEx(&cfg, kern, args...);
 }
 
-cudaError_t launch_skv_mlp(const CUtensorMap &tw, const SkvParams &p, cudaStream_t s) {
+cudaError_t launch_skv_features(const SkvParams &p, uint16_t *F, cudaStream_t s) {
+    if (p.Q == 0) return cudaSuccess;
+    const unsigned blocks = (unsigned)((p.P + kFeatWarps - 1) / kFeatWarps);
+    return launch_dependent(k_skv_features, dim3(blocks), 32 * kFeatWarps, (size_t)0, s, p, F);
+}
+
+cudaError_t launch_skv_mlp(const CUtensorMap &tf, const CUtensorMap &tw, const SkvParams &p, cudaStream_t s) {
     if (p.Q == 0) return cudaSuccess;
     const size_t smem = skv_mlp_smem_bytes();
     cudaError_t e = cudaFuncSetAttribute(k_skv_mlp, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
     if (e != cudaSuccess) return e;
     dim3 grid((unsigned)((p.P + kSkvRows - 1) / kSkvRows), (unsigned)(p.H / kSkvHidden));
-    return launch_dependent(k_skv_mlp, grid, kSkvThreads, smem, s, tw, p);
+    return launch_dependent(k_skv_mlp, grid, kSkvThreads, smem, s, tf, tw, p);
 }
 
 cudaError_t launch_skv_select(const SkvParams &p, cudaStream_t s) {

@@ -720,9 +720,10 @@ skip_status_t check_skv(skip_corpus *c, int32_t Q, int32_t K, const uint16_t *qb
     return SKIP_OK;
 }
 
-size_t skv_ws_bytes(int Q, int K, int H) {
+size_t skv_ws_bytes(int Q, int K, int H, int d) {
     const size_t P = (size_t)Q * K;
-    return align_up((size_t)kSkvCqSplits * Q * H * 4, 256) + align_up((size_t)(H / kSkvHidden) * P * 4, 256);
+    return align_up((size_t)kSkvCqSplits * Q * H * 4, 256) + align_up((size_t)(H / kSkvHidden) * P * 4, 256) +
+           align_up(P * 3 * (size_t)d * 2, 256);
 }
 
 // The gate on cand_ids; its workspace is the head of gws (skv_ws_bytes).
@@ -752,6 +753,7 @@ skip_status_t skv_impl(skip_corpus *c, const int64_t *cand_ids, int32_t Q, int32
     p.rho = rho;
     p.cq = reinterpret_cast<float *>(c->gws);
     p.partial = reinterpret_cast<float *>((char *)c->gws + align_up((size_t)kSkvCqSplits * Q * H * 4, 256));
+    uint16_t *F = reinterpret_cast<uint16_t *>((char *)p.partial + align_up((size_t)(H / kSkvHidden) * p.P * 4, 256));
     p.out_ids = out_ids;
     p.out_nu = out_nu;
     p.out_count = out_count;
@@ -772,13 +774,18 @@ skip_status_t skv_impl(skip_corpus *c, const int64_t *cand_ids, int32_t Q, int32
     cudaError_t e = launch_gemm2_bf16_f32(ta, tb, &ta2, &tb2, tn, Q, H, c->d, c->d, 1.f, mlp->b1, p.cq, H, c->err,
                                           c->timeout_ns, s, p.cq_splits, (int64_t)Q * H);
     if (e != cudaSuccess) return cuda_status(e);
+    CUtensorMap tf;
+    if (!encode_bf16_rows(&tf, F, p.P, 3 * c->d, 128)) return SKIP_ECUDA;
+    record(c, s, "skv_features");
+    e = launch_skv_features(p, F, s);
+    if (e != cudaSuccess) return cuda_status(e);
     record(c, s, "skv_mlp");
-    e = launch_skv_mlp(tw, p, s);
+    e = launch_skv_mlp(tf, tw, p, s);
     if (e != cudaSuccess) return cuda_status(e);
     record(c, s, "skv_select");
     e = launch_skv_select(p, s);
     if (e != cudaSuccess) return cuda_status(e);
-    pl.launches += 3;
+    pl.launches += 4;
     return SKIP_OK;
 }
 
@@ -1073,7 +1080,7 @@ skip_status_t skip_skv_gate(skip_corpus_t c, const int64_t *cand_ids, int32_t Q,
     if (st) return st;
     if (Q > 0 && !cand_ids) return SKIP_EINVAL;
     cudaStream_t s = reinterpret_cast<cudaStream_t>(stream);
-    st = ensure_buf(c->gws, c->gws_bytes, skv_ws_bytes(Q, K, mlp->hidden), "gate", c->canary);
+    st = ensure_buf(c->gws, c->gws_bytes, skv_ws_bytes(Q, K, mlp->hidden, c->d), "gate", c->canary);
     if (st) return st;
     ++c->call_id;
     Plan pl;
@@ -1094,7 +1101,7 @@ skip_status_t skip_retrieve_skv(skip_corpus_t c, const void *regions, const int3
     if (st) return st;
     cudaStream_t s = reinterpret_cast<cudaStream_t>(stream);
     // gate workspace first, then the merged lists (unless the caller keeps them)
-    const size_t gate = skv_ws_bytes(Q, K, mlp->hidden);
+    const size_t gate = skv_ws_bytes(Q, K, mlp->hidden, c->d);
     const size_t mid = align_up((size_t)Q * K * 8, 256), msc = align_up((size_t)Q * K * 4, 256);
     st = ensure_buf(c->gws, c->gws_bytes, gate + mid + msc, "gate", c->canary);
     if (st) return st;

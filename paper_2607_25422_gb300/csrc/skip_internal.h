@@ -193,11 +193,13 @@ struct SkvParams {
     uint64_t timeout_ns;
 };
 size_t skv_mlp_smem_bytes();
-// The gate in three launches: per-question bias (the library GEMM), the
-// tensor-core layer 1 + ReLU + w2 partial dots, and the sigmoid / gate /
-// selection.
-// tw: tensor map over W1 [H x 5d] bf16, box 64 columns x 128 rows, 128-byte swizzle.
-cudaError_t launch_skv_mlp(const CUtensorMap &tw, const SkvParams &p, cudaStream_t s);
+// The gate in four launches: per-question bias (the library GEMM), the
+// passage features F [P x 3d] bf16, the tensor-core layer 1 + ReLU + w2
+// partial dots, and the sigmoid / gate / selection.
+// tf: tensor map over F [P x 3d], tw: over W1 [H x 5d]; both bf16, box 64
+// columns x 128 rows, 128-byte swizzle.
+cudaError_t launch_skv_features(const SkvParams &p, uint16_t *F, cudaStream_t s);
+cudaError_t launch_skv_mlp(const CUtensorMap &tf, const CUtensorMap &tw, const SkvParams &p, cudaStream_t s);
 cudaError_t launch_skv_select(const SkvParams &p, cudaStream_t s);
 
 // ---- IVF-PQ variant (k_ivfpq.cu) ------------------------------------------
