@@ -34,7 +34,9 @@ namespace {
 constexpr int kLogThreads = 256;
 constexpr int kLogTok = 8;  // tokens per warp in flight
 
-__global__ void __launch_bounds__(kLogThreads) k_qvs_logits(const QvsParams p) {
+// (At most 64 registers a thread, four blocks an SM: with 80 registers only
+// three fit, and 576 blocks took two waves.)
+__global__ void __launch_bounds__(kLogThreads, 4) k_qvs_logits(const QvsParams p) {
     extern __shared__ float us[];  // [d]
     __shared__ float cpart[kLogThreads / 32];
     const int b = blockIdx.y;
@@ -114,7 +116,7 @@ __global__ void __launch_bounds__(kLogThreads) k_qvs_logits(const QvsParams p) {
 }
 
 constexpr int kRankWarps = 8;
-constexpr int kRankTok = 4;  // tokens per warp
+constexpr int kRankTok = 8;  // tokens per warp (576 blocks for 64 images: one wave at five an SM)
 
 __global__ void __launch_bounds__(32 * kRankWarps) k_qvs_rank(const QvsParams p) {
     extern __shared__ uint64_t keys[];  // [L]: (ord(logit), ~index) of every token of the image
