@@ -732,22 +732,25 @@ def main():
         for _ in range(args.warmup):
             plain()
         torch.cuda.synchronize()
-        t_plain = t_gate = 0.0
-        for fn_is_gate in [False, True] * 5:
-            fn = step if fn_is_gate else plain
-            e0 = torch.cuda.Event(enable_timing=True)
-            e1 = torch.cuda.Event(enable_timing=True)
-            e0.record(stream)
-            for _ in range(max(1, args.steps // 5)):
-                fn()
-            e1.record(stream)
-            torch.cuda.synchronize()
-            if fn_is_gate:
-                t_gate += e0.elapsed_time(e1)
-            else:
-                t_plain += e0.elapsed_time(e1)
-        n_each = 5 * max(1, args.steps // 5)
-        gate_delta_ms = max_over_ranks((t_gate - t_plain) / n_each, world)
+        # twelve pairs of blocks, the order within a pair alternating; the
+        # median of the pairs' differences (a 1 ms step under the power cap
+        # wanders by a few us between blocks)
+        per = max(1, args.steps // 5)
+        diffs = []
+        for i in range(12):
+            t = {}
+            for fn_is_gate in ([False, True] if i % 2 == 0 else [True, False]):
+                fn = step if fn_is_gate else plain
+                e0 = torch.cuda.Event(enable_timing=True)
+                e1 = torch.cuda.Event(enable_timing=True)
+                e0.record(stream)
+                for _ in range(per):
+                    fn()
+                e1.record(stream)
+                torch.cuda.synchronize()
+                t[fn_is_gate] = e0.elapsed_time(e1) / per
+            diffs.append(t[True] - t[False])
+        gate_delta_ms = max_over_ranks(float(np.median(diffs)), world)
 
     # ---- end to end through the host-buffer entry point
     reg_h = regions.pin_memory()

@@ -10,6 +10,7 @@
 
 #include <algorithm>
 #include <cmath>
+#include <functional>
 #include <map>
 #include <mutex>
 #include <string>
@@ -129,6 +130,10 @@ struct skip_corpus {
     size_t ev_used = 0;
     int call_id = 0;
     char plan[384] = "{}";
+    // Second stream for work that needs no retrieval result (the SKV gate's
+    // per-question bias), forked from and joined back to the caller's stream.
+    cudaStream_t aux = nullptr;
+    cudaEvent_t ev_fork = nullptr, ev_join = nullptr;
 };
 
 namespace {
@@ -286,6 +291,9 @@ struct QuestionMerge {
     int64_t *out_ids;
     float *out_scores;
     bool done = false;
+    // called once the score kernel is queued (work that needs no retrieval
+    // result and should not compete with that kernel for SMs)
+    std::function<skip_status_t()> after_score;
 };
 
 skip_status_t run_regions(skip_corpus *c, const uint16_t *regions, int R, int k, uint64_t **keys_out,
@@ -361,6 +369,10 @@ skip_status_t run_regions(skip_corpus *c, const uint16_t *regions, int R, int k,
         cudaError_t e = launch_latency(e4m3, ta, tb, p, pl.grid, s);
         if (e != cudaSuccess) return cuda_status(e);
         ++pl.launches;
+        if (qm && qm->after_score) {
+            const skip_status_t hs = qm->after_score();
+            if (hs) return hs;
+        }
         // One block per question merges all its region rows: only while the
         // questions average at most 8 regions (one question of 32 regions,
         // merged by one block, took 28 us against 23 us for the two launches).
@@ -434,6 +446,10 @@ skip_status_t run_regions(skip_corpus *c, const uint16_t *regions, int R, int k,
         cudaError_t e = launch_tc_fp8(tq, traw, p, pl.grid, s);
         if (e != cudaSuccess) return cuda_status(e);
         ++pl.launches;
+        if (qm && qm->after_score) {
+            const skip_status_t hs = qm->after_score();
+            if (hs) return hs;
+        }
         record(c, s, "merge_lists");
         e = launch_merge_lists(lists, pl.G, (int64_t)pl.R_pad * k, R, k, reg_keys, reg_ids, reg_scores, s, true);
         if (e != cudaSuccess) return cuda_status(e);
@@ -608,6 +624,10 @@ skip_status_t run_regions(skip_corpus *c, const uint16_t *regions, int R, int k,
         e = launch_tc(pair, tq, tx, p, pl.grid, s, bound);
         if (e != cudaSuccess) return cuda_status(e);
         ++pl.launches;
+        if (qm && qm->after_score) {
+            const skip_status_t hs = qm->after_score();
+            if (hs) return hs;
+        }
         record(c, s, "merge_lists");
         e = launch_merge_lists(lists, pl.G, (int64_t)pl.R_pad * k, R, k, reg_keys, reg_ids, reg_scores, s, true);
         if (e != cudaSuccess) return cuda_status(e);
@@ -644,6 +664,10 @@ skip_status_t run_regions(skip_corpus *c, const uint16_t *regions, int R, int k,
         if (e != cudaSuccess) return cuda_status(e);
         ++pl.launches;
     }
+    if (qm && qm->after_score) {
+        const skip_status_t hs = qm->after_score();
+        if (hs) return hs;
+    }
     record(c, s, "merge_lists");
     cudaError_t e = launch_merge_lists(lists, pl.G, (int64_t)R * k, R, k, reg_keys, reg_ids, reg_scores, s, true);
     if (e != cudaSuccess) return cuda_status(e);
@@ -676,7 +700,7 @@ skip_status_t check_retrieve(skip_corpus *c, const void *regions, const int32_t 
 // Per-region step, then the per-question merge into out_ids / out_scores.
 skip_status_t retrieve_impl(skip_corpus *c, const void *regions, const int32_t *region_offsets, int32_t Q,
                             int32_t R_total, int32_t k_region, int32_t K, int64_t *out_ids, float *out_scores,
-                            cudaStream_t s, Plan &pl) {
+                            cudaStream_t s, Plan &pl, std::function<skip_status_t()> after_score = nullptr) {
     const size_t keys_bytes = align_up((size_t)std::max(R_total, 1) * k_region * sizeof(uint64_t), 256);
     uint64_t *reg_keys = nullptr;
     skip_status_t st;
@@ -686,6 +710,7 @@ skip_status_t retrieve_impl(skip_corpus *c, const void *regions, const int32_t *
     qm.K = K;
     qm.out_ids = out_ids;
     qm.out_scores = out_scores;
+    qm.after_score = std::move(after_score);
     if (R_total > 0) {
         st = run_regions(c, reinterpret_cast<const uint16_t *>(regions), R_total, k_region, &reg_keys,
                          nullptr, nullptr, s, pl, keys_bytes, &qm);
@@ -720,20 +745,83 @@ skip_status_t check_skv(skip_corpus *c, int32_t Q, int32_t K, const uint16_t *qb
     return SKIP_OK;
 }
 
+// Partial-logit slabs of the MLP: at most H / 32 (128 units a pair, two K
+// parts, two column halves).
 size_t skv_ws_bytes(int Q, int K, int H, int d) {
     const size_t P = (size_t)Q * K;
-    return align_up((size_t)kSkvCqSplits * Q * H * 4, 256) + align_up((size_t)(H / kSkvHidden) * P * 4, 256) +
+    return align_up((size_t)kSkvCqSplits * Q * H * 4, 256) + align_up((size_t)(H / 32) * P * 4, 256) +
            align_up(P * 3 * (size_t)d * 2, 256);
 }
 
-// The gate on cand_ids; its workspace is the head of gws (skv_ws_bytes).
+// The per-question bias c_q = b1 + W1[:, 0:d] qbar + W1[:, d:2d] vbar of every
+// question: one GEMM over the two column blocks of W1, K split over up to
+// kSkvCqSplits CTAs per tile (k_skv_mlp sums the slabs), into the head of
+// gws.  It needs no retrieval result: in skip_retrieve_skv it runs on the
+// handle's second stream, forked from s once the score kernel is queued (so
+// that it overlaps the merge kernels, which leave most SMs idle) and joined
+// back before the gate's first kernel; otherwise (no retrieval, or
+// per-kernel timing on) on s before the gate.
+struct CqLaunch {
+    CUtensorMap ta, tb, ta2, tb2;
+    int tn = 0, Q = 0, H = 0, splits = 1;
+    const float *b1 = nullptr;
+    bool launched = false, forked = false;
+};
+skip_status_t skv_prepare_cq(skip_corpus *c, int32_t Q, const uint16_t *qbar, const uint16_t *vbar,
+                             const skip_skv_mlp_t *mlp, CqLaunch &cl) {
+    if (Q == 0) return SKIP_OK;
+    cl.Q = Q;
+    cl.H = mlp->hidden;
+    cl.b1 = mlp->b1;
+    cl.tn = gemm_tile_n(Q, cl.H, c->sm_count);
+    cl.splits = std::min(kSkvCqSplits, gemm_splits(Q, cl.H, 2 * c->d, cl.tn, c->sm_count));
+    if (!encode_bf16_rows(&cl.ta, qbar, Q, c->d, 128) || !encode_bf16_rows(&cl.ta2, vbar, Q, c->d, 128) ||
+        !encode_bf16_block(&cl.tb, mlp->w1, cl.H, c->d, 5 * (int64_t)c->d, cl.tn) ||
+        !encode_bf16_block(&cl.tb2, mlp->w1 + c->d, cl.H, c->d, 5 * (int64_t)c->d, cl.tn))
+        return SKIP_ECUDA;
+    return SKIP_OK;
+}
+
+// Launches the c_q GEMM: forked onto the handle's second stream after the
+// work queued on s so far, or on s itself.
+skip_status_t skv_launch_cq(skip_corpus *c, CqLaunch &cl, cudaStream_t s, bool fork) {
+    if (cl.Q == 0 || cl.launched) return SKIP_OK;
+    cudaStream_t g = s;
+    if (fork) {
+        if (!c->aux) {
+            if (cudaStreamCreateWithFlags(&c->aux, cudaStreamNonBlocking) != cudaSuccess ||
+                cudaEventCreateWithFlags(&c->ev_fork, cudaEventDisableTiming) != cudaSuccess ||
+                cudaEventCreateWithFlags(&c->ev_join, cudaEventDisableTiming) != cudaSuccess) {
+                cudaGetLastError();
+                return SKIP_ECUDA;
+            }
+        }
+        if (cudaEventRecord(c->ev_fork, s) != cudaSuccess || cudaStreamWaitEvent(c->aux, c->ev_fork, 0) != cudaSuccess)
+            return SKIP_ECUDA;
+        g = c->aux;
+    } else {
+        record(c, s, "skv_qbias");
+    }
+    cudaError_t e = launch_gemm2_bf16_f32(cl.ta, cl.tb, &cl.ta2, &cl.tb2, cl.tn, cl.Q, cl.H, c->d, c->d, 1.f, cl.b1,
+                                          reinterpret_cast<float *>(c->gws), cl.H, c->err, c->timeout_ns, g,
+                                          cl.splits, (int64_t)cl.Q * cl.H);
+    if (e != cudaSuccess) return cuda_status(e);
+    if (fork && cudaEventRecord(c->ev_join, c->aux) != cudaSuccess) return SKIP_ECUDA;
+    cl.launched = true;
+    cl.forked = fork;
+    return SKIP_OK;
+}
+
+// The gate on cand_ids (c_q prepared by skv_prepare_cq, launched here if it
+// has not been); its workspace is the head of gws (skv_ws_bytes).
 skip_status_t skv_impl(skip_corpus *c, const int64_t *cand_ids, int32_t Q, int32_t K, const uint16_t *qbar,
                        const uint16_t *vbar, const skip_skv_mlp_t *mlp, float tau, float rho, int64_t *out_ids,
-                       float *out_nu, int32_t *out_count, float *nu_all, cudaStream_t s, Plan &pl) {
+                       float *out_nu, int32_t *out_count, float *nu_all, CqLaunch &cl, cudaStream_t s,
+                       Plan &pl) {
     if (Q == 0) return SKIP_OK;
+    skip_status_t st = skv_launch_cq(c, cl, s, false);
+    if (st) return st;
     const int H = mlp->hidden;
-    CUtensorMap tw;
-    if (!encode_bf16_rows(&tw, mlp->w1, H, 5 * c->d, 128)) return SKIP_ECUDA;
     SkvParams p;
     p.rows = reinterpret_cast<const uint16_t *>(c->rows);
     p.N = c->N;
@@ -752,35 +840,27 @@ skip_status_t skv_impl(skip_corpus *c, const int64_t *cand_ids, int32_t Q, int32
     p.tau = tau;
     p.rho = rho;
     p.cq = reinterpret_cast<float *>(c->gws);
+    p.cq_splits = cl.splits;
     p.partial = reinterpret_cast<float *>((char *)c->gws + align_up((size_t)kSkvCqSplits * Q * H * 4, 256));
-    uint16_t *F = reinterpret_cast<uint16_t *>((char *)p.partial + align_up((size_t)(H / kSkvHidden) * p.P * 4, 256));
+    uint16_t *F = reinterpret_cast<uint16_t *>((char *)p.partial + align_up((size_t)(H / 32) * p.P * 4, 256));
     p.out_ids = out_ids;
     p.out_nu = out_nu;
     p.out_count = out_count;
     p.nu_all = nu_all;
     p.err = c->err;
     p.timeout_ns = c->timeout_ns;
-    // c_q = b1 + W1[:, 0:d] qbar + W1[:, d:2d] vbar for every question: one
-    // GEMM over the two column blocks of W1, K split over up to
-    // kSkvCqSplits CTAs per tile (k_skv_mlp sums the partial slabs).
-    CUtensorMap ta, tb, ta2, tb2;
-    const int tn = gemm_tile_n(Q, H, c->sm_count);
-    p.cq_splits = std::min(kSkvCqSplits, gemm_splits(Q, H, 2 * c->d, tn, c->sm_count));
-    if (!encode_bf16_rows(&ta, qbar, Q, c->d, 128) || !encode_bf16_rows(&ta2, vbar, Q, c->d, 128) ||
-        !encode_bf16_block(&tb, mlp->w1, H, c->d, 5 * (int64_t)c->d, tn) ||
-        !encode_bf16_block(&tb2, mlp->w1 + c->d, H, c->d, 5 * (int64_t)c->d, tn))
+    int BN = 0, S = 0;
+    skv_mlp_shape(p.P, H, &BN, &S);
+    p.nparts = H / BN * S * 2;
+    CUtensorMap tf, tw;
+    if (!encode_bf16_rows(&tf, F, p.P, 3 * c->d, 128) || !encode_bf16_rows(&tw, mlp->w1, H, 5 * c->d, BN / 2))
         return SKIP_ECUDA;
-    record(c, s, "skv_qbias");
-    cudaError_t e = launch_gemm2_bf16_f32(ta, tb, &ta2, &tb2, tn, Q, H, c->d, c->d, 1.f, mlp->b1, p.cq, H, c->err,
-                                          c->timeout_ns, s, p.cq_splits, (int64_t)Q * H);
-    if (e != cudaSuccess) return cuda_status(e);
-    CUtensorMap tf;
-    if (!encode_bf16_rows(&tf, F, p.P, 3 * c->d, 128)) return SKIP_ECUDA;
+    if (cl.forked && cudaStreamWaitEvent(s, c->ev_join, 0) != cudaSuccess) return SKIP_ECUDA;
     record(c, s, "skv_features");
-    e = launch_skv_features(p, F, s);
+    cudaError_t e = launch_skv_features(p, F, s);
     if (e != cudaSuccess) return cuda_status(e);
     record(c, s, "skv_mlp");
-    e = launch_skv_mlp(tf, tw, p, s);
+    e = launch_skv_mlp(tf, tw, p, BN, S, s);
     if (e != cudaSuccess) return cuda_status(e);
     record(c, s, "skv_select");
     e = launch_skv_select(p, s);
@@ -869,6 +949,9 @@ skip_status_t skip_corpus_free(skip_corpus_t c) {
     cudaFree(c->io);
     cudaFree(c->gws);
     for (cudaEvent_t e : c->ev_pool) cudaEventDestroy(e);
+    if (c->ev_fork) cudaEventDestroy(c->ev_fork);
+    if (c->ev_join) cudaEventDestroy(c->ev_join);
+    if (c->aux) cudaStreamDestroy(c->aux);
     delete c;
     return SKIP_OK;
 }
@@ -1084,7 +1167,11 @@ skip_status_t skip_skv_gate(skip_corpus_t c, const int64_t *cand_ids, int32_t Q,
     if (st) return st;
     ++c->call_id;
     Plan pl;
-    st = skv_impl(c, cand_ids, Q, K, qbar, vbar, mlp, tau_nu, rho_r, out_ids, out_nu, out_count, nu_all, s, pl);
+    CqLaunch cl;
+    st = skv_prepare_cq(c, Q, qbar, vbar, mlp, cl);
+    if (st) return st;
+    st = skv_impl(c, cand_ids, Q, K, qbar, vbar, mlp, tau_nu, rho_r, out_ids, out_nu, out_count, nu_all, cl, s,
+                  pl);
     if (st) return st;
     record(c, s, "end");
     return SKIP_OK;
@@ -1109,9 +1196,14 @@ skip_status_t skip_retrieve_skv(skip_corpus_t c, const void *regions, const int3
     float *mscs = merged_scores ? merged_scores : reinterpret_cast<float *>((char *)c->gws + gate + mid);
     ++c->call_id;
     Plan pl;
-    st = retrieve_impl(c, regions, region_offsets, Q, R_total, k_region, K, mids, mscs, s, pl);
+    CqLaunch cl;
+    st = skv_prepare_cq(c, Q, qbar, vbar, mlp, cl);
     if (st) return st;
-    st = skv_impl(c, mids, Q, K, qbar, vbar, mlp, tau_nu, rho_r, out_ids, out_nu, out_count, nullptr, s, pl);
+    const bool fork = !c->timing;
+    st = retrieve_impl(c, regions, region_offsets, Q, R_total, k_region, K, mids, mscs, s, pl,
+                       [&]() { return fork ? skv_launch_cq(c, cl, s, true) : SKIP_OK; });
+    if (st) return st;
+    st = skv_impl(c, mids, Q, K, qbar, vbar, mlp, tau_nu, rho_r, out_ids, out_nu, out_count, nullptr, cl, s, pl);
     if (st) return st;
     record(c, s, "end");
     write_plan(c, pl, R_total, Q, k_region, K);

@@ -164,7 +164,7 @@ cudaError_t launch_question_merge(const uint64_t *reg_keys, int k, const int32_t
                                   cudaStream_t s, bool pdl = false);
 
 // ---- SKV passage gate (k_skv.cu) ------------------------------------------
-constexpr int kSkvHidden = 128;  // hidden units per CTA of the gate MLP (TMEM columns)
+constexpr int kSkvHidden = 128;  // the gate MLP's hidden width is a multiple of this
 constexpr int kSkvMaxK = 2048;   // candidate slots per question (SKIP_MAX_K)
 struct SkvParams {
     const uint16_t *rows;  // bf16 corpus [N x d]
@@ -184,7 +184,8 @@ struct SkvParams {
     float tau, rho;
     float *cq;             // [cq_splits x Q x H] workspace: partial sums of b1 + W1 qbar-part + W1 vbar-part
     int cq_splits;         // K splits of the c_q GEMM (the slabs are summed in k_skv_mlp)
-    float *partial;        // [H / kSkvHidden][P] workspace: partial logits
+    float *partial;        // [nparts][P] workspace: partial logits
+    int nparts;            // partial-logit slabs: H / BN * S * 2 (skv_mlp_shape)
     int64_t *out_ids;      // [Q x K]
     float *out_nu;         // [Q x K]
     int32_t *out_count;    // [Q]
@@ -193,13 +194,19 @@ struct SkvParams {
     uint64_t timeout_ns;
 };
 size_t skv_mlp_smem_bytes();
+// Tile shape of the gate MLP for P slots and H hidden units: BN hidden units
+// per CTA pair (128 or 256) and S K parts (1 or 2; clusters of 2 S CTAs).
+void skv_mlp_shape(int64_t P, int H, int *BN, int *S);
 // The gate in four launches: per-question bias (the library GEMM), the
 // passage features F [P x 3d] bf16, the tensor-core layer 1 + ReLU + w2
 // partial dots, and the sigmoid / gate / selection.
-// tf: tensor map over F [P x 3d], tw: over W1 [H x 5d]; both bf16, box 64
-// columns x 128 rows, 128-byte swizzle.
+// tf: tensor map over F [P x 3d], box 64 columns x 128 rows; tw: over W1
+// [H x 5d], box 64 columns x BN / 2 rows; both bf16, 128-byte swizzle.
+// The features kernel waits for the grid before it (the candidate ids)
+// before it reads; the MLP reads c_q, which must be complete when it starts.
 cudaError_t launch_skv_features(const SkvParams &p, uint16_t *F, cudaStream_t s);
-cudaError_t launch_skv_mlp(const CUtensorMap &tf, const CUtensorMap &tw, const SkvParams &p, cudaStream_t s);
+cudaError_t launch_skv_mlp(const CUtensorMap &tf, const CUtensorMap &tw, const SkvParams &p, int BN, int S,
+                           cudaStream_t s);
 cudaError_t launch_skv_select(const SkvParams &p, cudaStream_t s);
 
 // ---- IVF-PQ variant (k_ivfpq.cu) ------------------------------------------

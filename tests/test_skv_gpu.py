@@ -151,6 +151,14 @@ CASES = [
     (4000, 1024, 3, 100, 128, (0, 40, 99), 0.6, 0.9),
     (2000, 64, 4, 1, 128, (0, 1), 0.5, 1.0),
     (3000, 256, 2, 2048, 384, (0, 1500), 0.4, 0.3),
+    # enough slots that the MLP runs without the K split (one CTA pair per tile)
+    (6000, 128, 64, 200, 512, (0, 7, 150), 0.5, 0.6),
+    # one slot per question: more questions per tile than the MLP stages c_q for
+    (3000, 128, 300, 1, 256, (0, 1), 0.5, 1.0),
+    (20000, 64, 20000, 1, 512, (0, 1), 0.5, 1.0),
+    # the largest K the selection ranks, and the smallest it sorts
+    (3000, 128, 6, 256, 256, (0, 100, 255), 0.5, 0.6),
+    (3000, 128, 5, 257, 256, (0, 1, 256), 0.5, 0.6),
 ]
 
 
