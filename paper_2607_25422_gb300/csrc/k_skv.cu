@@ -80,6 +80,16 @@ __device__ __forceinline__ void bulk_copy_to_peer(uint32_t dst, uint32_t src, ui
                  : "memory");
 }
 
+__device__ __forceinline__ int ld_acquire_gpu(const int *p) {
+    int v;
+    asm volatile("ld.acquire.gpu.global.b32 %0, [%1];" : "=r"(v) : "l"(p) : "memory");
+    return v;
+}
+
+__device__ __forceinline__ void st_release_gpu(int *p, int v) {
+    asm volatile("st.release.gpu.global.b32 [%0], %1;" ::"l"(p), "r"(v) : "memory");
+}
+
 // Generic-proxy writes to shared memory before an async-proxy read of them.
 __device__ __forceinline__ void fence_proxy_async_smem() {
     asm volatile("fence.proxy.async.shared::cta;" ::: "memory");
@@ -150,13 +160,14 @@ __global__ void __launch_bounds__(32 * kFeatWarps) k_skv_features(const SkvParam
 // nu of slot `slot` (logit = b2 + the partial logits of the grid before)
 // and its key (ordered nu bits << 32 | ~id; 0 when empty or below tau).
 __device__ __forceinline__ uint64_t slot_key(const SkvParams &p, int64_t slot, float &nu, bool &nonempty) {
+    // the id and the partial logits in one round of loads
     int64_t id = p.ids[slot];
+    float logit = p.b2;
+    for (int b = 0; b < p.nparts; ++b) logit += p.partial[(int64_t)b * p.P + slot];
     if (id >= p.N) id = -1;  // flagged by k_skv_features
     nu = -__int_as_float(0x7f800000);
     nonempty = id >= 0;
     if (id < 0) return 0ull;
-    float logit = p.b2;
-    for (int b = 0; b < p.nparts; ++b) logit += p.partial[(int64_t)b * p.P + slot];
     nu = 1.f / (1.f + expf(-logit));
     if (!(nu >= p.tau)) return 0ull;
     return ((uint64_t)(__float_as_uint(nu) | 0x80000000u) << 32) | (uint64_t)(0xFFFFFFFFu - (uint32_t)id);
@@ -398,8 +409,24 @@ __global__ void __launch_bounds__(kSkvThreads, 1)
     if (epi) {
         // While the main loop runs: w2 and c_q (the GEMM's K-split slabs
         // summed once) of this CTA's columns into shared memory,
-        // cqs[(q - q0) * ncol + c].  c_q precedes the grid before this one.
+        // cqs[(q - q0) * ncol + c].  c_q comes from a kernel before this one
+        // in the stream, or (cq_flag) from the GEMM on the other stream,
+        // which raises the flag to cq_epoch once it has completed.
         grid_dep_wait();
+        if (p.cq_flag) {
+            if (et == 0) {
+                const uint64_t t0 = globaltimer_ns();
+                while (ld_acquire_gpu(p.cq_flag) != p.cq_epoch) {
+                    if (globaltimer_ns() - t0 > p.timeout_ns) {
+                        atomicOr(p.err, kErrTimeout);
+                        break;
+                    }
+                    __nanosleep(256);
+                }
+            }
+            asm volatile("bar.sync 1, %0;" ::"r"(32 * kSkvEpiWarps) : "memory");
+            (void)ld_acquire_gpu(p.cq_flag);
+        }
         for (int t = et; t < ncol; t += 32 * kSkvEpiWarps) w2s[t] = p.w2[n0 + c0 + t];
         if (cq_staged)
             for (int t = et; t < nq * ncol; t += 32 * kSkvEpiWarps) {
@@ -447,7 +474,9 @@ __global__ void __launch_bounds__(kSkvThreads, 1)
                               mapa_shared(smem_addr(&sh->recv), peer));
         }
         if (epi) {
-            got = mbar_wait(smem_addr(&sh->recv), 0, p.timeout_ns);
+            // a copy in flight writes into this CTA's shared memory: wait for
+            // it at least as long as for any other copy before giving up
+            got = mbar_wait(smem_addr(&sh->recv), 0, p.timeout_ns > kDrainTimeoutNs ? p.timeout_ns : kDrainTimeoutNs);
             if (!got && r == 0) atomicOr(p.err, kErrTimeout);
         }
     }
@@ -520,6 +549,10 @@ __global__ void __launch_bounds__(kSkvThreads, 1)
 }
 
 }  // namespace
+
+// Raises the c_q flag once the GEMM before this kernel in its stream has
+// completed.
+__global__ void k_skv_cq_ready(int *flag, int epoch) { st_release_gpu(flag, epoch); }
 
 size_t skv_mlp_smem_bytes() {
     return 1024 + (size_t)kSkvRing + 1024 + kSkvEpiBytes;
@@ -613,6 +646,11 @@ cudaError_t launch_skv_mlp(const CUtensorMap &tf, const CUtensorMap &tw, const S
     cfg.attrs = attr;
     cfg.numAttrs = 2;
     return cudaLaunchKernelEx(&cfg, kern, tf, tw, p);
+}
+
+cudaError_t launch_skv_cq_ready(int *flag, int epoch, cudaStream_t s) {
+    k_skv_cq_ready<<<1, 1, 0, s>>>(flag, epoch);
+    return cudaGetLastError();
 }
 
 cudaError_t launch_skv_select(const SkvParams &p, cudaStream_t s) {

@@ -134,6 +134,8 @@ struct skip_corpus {
     // per-question bias), forked from and joined back to the caller's stream.
     cudaStream_t aux = nullptr;
     cudaEvent_t ev_fork = nullptr, ev_join = nullptr;
+    int *cq_flag = nullptr;  // device: epoch of the last completed bias GEMM on aux
+    int cq_epoch = 0;
 };
 
 namespace {
@@ -758,14 +760,18 @@ size_t skv_ws_bytes(int Q, int K, int H, int d) {
 // kSkvCqSplits CTAs per tile (k_skv_mlp sums the slabs), into the head of
 // gws.  It needs no retrieval result: in skip_retrieve_skv it runs on the
 // handle's second stream, forked from s once the score kernel is queued (so
-// that it overlaps the merge kernels, which leave most SMs idle) and joined
-// back before the gate's first kernel; otherwise (no retrieval, or
-// per-kernel timing on) on s before the gate.
+// that it overlaps the merge kernels, which leave most SMs idle); a flag it
+// raises afterwards (a per-call epoch) tells the MLP kernel that c_q is
+// complete, and the second stream is joined back into s after the gate's
+// last kernel, so that no event wait sits between the retrieval and the
+// gate.  Otherwise (no retrieval, or per-kernel timing on) it runs on s
+// before the gate.
 struct CqLaunch {
     CUtensorMap ta, tb, ta2, tb2;
     int tn = 0, Q = 0, H = 0, splits = 1;
     const float *b1 = nullptr;
     bool launched = false, forked = false;
+    int epoch = 0;
 };
 skip_status_t skv_prepare_cq(skip_corpus *c, int32_t Q, const uint16_t *qbar, const uint16_t *vbar,
                              const skip_skv_mlp_t *mlp, CqLaunch &cl) {
@@ -796,6 +802,14 @@ skip_status_t skv_launch_cq(skip_corpus *c, CqLaunch &cl, cudaStream_t s, bool f
                 return SKIP_ECUDA;
             }
         }
+        if (!c->cq_flag) {
+            if (dev_alloc(reinterpret_cast<void **>(&c->cq_flag), 16, "gate") != cudaSuccess) {
+                cudaGetLastError();
+                c->cq_flag = nullptr;
+                return SKIP_ENOMEM;
+            }
+            if (cudaMemsetAsync(c->cq_flag, 0, 16, s) != cudaSuccess) return SKIP_ECUDA;
+        }
         if (cudaEventRecord(c->ev_fork, s) != cudaSuccess || cudaStreamWaitEvent(c->aux, c->ev_fork, 0) != cudaSuccess)
             return SKIP_ECUDA;
         g = c->aux;
@@ -806,7 +820,12 @@ skip_status_t skv_launch_cq(skip_corpus *c, CqLaunch &cl, cudaStream_t s, bool f
                                           reinterpret_cast<float *>(c->gws), cl.H, c->err, c->timeout_ns, g,
                                           cl.splits, (int64_t)cl.Q * cl.H);
     if (e != cudaSuccess) return cuda_status(e);
-    if (fork && cudaEventRecord(c->ev_join, c->aux) != cudaSuccess) return SKIP_ECUDA;
+    if (fork) {
+        c->cq_epoch = c->cq_epoch == 0x7fffffff ? 1 : c->cq_epoch + 1;
+        cl.epoch = c->cq_epoch;
+        if ((e = launch_skv_cq_ready(c->cq_flag, cl.epoch, c->aux)) != cudaSuccess) return cuda_status(e);
+        if (cudaEventRecord(c->ev_join, c->aux) != cudaSuccess) return SKIP_ECUDA;
+    }
     cl.launched = true;
     cl.forked = fork;
     return SKIP_OK;
@@ -841,6 +860,8 @@ skip_status_t skv_impl(skip_corpus *c, const int64_t *cand_ids, int32_t Q, int32
     p.rho = rho;
     p.cq = reinterpret_cast<float *>(c->gws);
     p.cq_splits = cl.splits;
+    p.cq_flag = cl.forked ? c->cq_flag : nullptr;
+    p.cq_epoch = cl.epoch;
     p.partial = reinterpret_cast<float *>((char *)c->gws + align_up((size_t)kSkvCqSplits * Q * H * 4, 256));
     uint16_t *F = reinterpret_cast<uint16_t *>((char *)p.partial + align_up((size_t)(H / 32) * p.P * 4, 256));
     p.out_ids = out_ids;
@@ -855,7 +876,6 @@ skip_status_t skv_impl(skip_corpus *c, const int64_t *cand_ids, int32_t Q, int32
     CUtensorMap tf, tw;
     if (!encode_bf16_rows(&tf, F, p.P, 3 * c->d, 128) || !encode_bf16_rows(&tw, mlp->w1, H, 5 * c->d, BN / 2))
         return SKIP_ECUDA;
-    if (cl.forked && cudaStreamWaitEvent(s, c->ev_join, 0) != cudaSuccess) return SKIP_ECUDA;
     record(c, s, "skv_features");
     cudaError_t e = launch_skv_features(p, F, s);
     if (e != cudaSuccess) return cuda_status(e);
@@ -866,6 +886,8 @@ skip_status_t skv_impl(skip_corpus *c, const int64_t *cand_ids, int32_t Q, int32
     e = launch_skv_select(p, s);
     if (e != cudaSuccess) return cuda_status(e);
     pl.launches += 4;
+    // the second stream joins s again (its GEMM is long done by now)
+    if (cl.forked && cudaStreamWaitEvent(s, c->ev_join, 0) != cudaSuccess) return SKIP_ECUDA;
     return SKIP_OK;
 }
 
@@ -952,6 +974,7 @@ skip_status_t skip_corpus_free(skip_corpus_t c) {
     if (c->ev_fork) cudaEventDestroy(c->ev_fork);
     if (c->ev_join) cudaEventDestroy(c->ev_join);
     if (c->aux) cudaStreamDestroy(c->aux);
+    cudaFree(c->cq_flag);
     delete c;
     return SKIP_OK;
 }

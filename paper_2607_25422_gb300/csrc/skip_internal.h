@@ -184,6 +184,8 @@ struct SkvParams {
     float tau, rho;
     float *cq;             // [cq_splits x Q x H] workspace: partial sums of b1 + W1 qbar-part + W1 vbar-part
     int cq_splits;         // K splits of the c_q GEMM (the slabs are summed in k_skv_mlp)
+    const int *cq_flag;    // null, or raised to cq_epoch when c_q (from another stream) is complete
+    int cq_epoch;
     float *partial;        // [nparts][P] workspace: partial logits
     int nparts;            // partial-logit slabs: H / BN * S * 2 (skv_mlp_shape)
     int64_t *out_ids;      // [Q x K]
@@ -208,6 +210,8 @@ cudaError_t launch_skv_features(const SkvParams &p, uint16_t *F, cudaStream_t s)
 cudaError_t launch_skv_mlp(const CUtensorMap &tf, const CUtensorMap &tw, const SkvParams &p, int BN, int S,
                            cudaStream_t s);
 cudaError_t launch_skv_select(const SkvParams &p, cudaStream_t s);
+// One thread stores `epoch` to *flag (release, GPU scope).
+cudaError_t launch_skv_cq_ready(int *flag, int epoch, cudaStream_t s);
 
 // ---- IVF-PQ variant (k_ivfpq.cu) ------------------------------------------
 constexpr int kIvfMaxDs = 32;   // largest sub-space width d / M

@@ -42,3 +42,43 @@ def test_wait_timeout_reports_and_recovers(mma):
     for r, t in enumerate(checker.region_truths(ids_ext, sc_ext, k)):
         _, probs = checker.check_region(rid[r], rsc[r], t)
         assert not probs, (r, probs)
+
+
+def test_gate_wait_timeout_reports_and_recovers():
+    """The retrieval plus SKV gate with every wait allowed to give up at once
+    (the gate's MLP waits for its flag, its TMA and MMA phases and its
+    partner's half of the sums): SKIP_ETIMEOUT, then a normal call on the
+    same handle whose gate matches the oracle on the call's own merged lists."""
+    from tests.test_skv_gpu import check_gate
+    dev = torch.device("cuda")
+    N, d, Q, R_per, k, K = 20000, 128, 16, 4, 20, 50
+    ct = synth.random_bf16(N, d, seed=93)
+    rt = synth.random_bf16(Q * R_per, d, seed=94)
+    offs = torch.arange(0, Q * R_per + 1, R_per, dtype=torch.int32)
+    qbar = synth.random_bf16(Q, d, seed=95)
+    vbar = synth.random_bf16(Q, d, seed=96)
+    w1, b1, w2, b2 = synth.make_skv_mlp(d, 512, seed=97)
+    t = lambda x: x.to(dev).contiguous()
+    c = skip.skip_corpus_load(ct.to(dev))
+    try:
+        c.set_option(skip.SKIP_OPT_PATH, skip.SKIP_PATH_TENSOR)
+        c.set_option(skip.SKIP_OPT_WAIT_TIMEOUT_NS, 0)
+        args = (c, t(rt), t(offs), k, K, t(qbar), t(vbar), t(w1), t(b1.float()), t(w2.float()), b2)
+        skip.skip_retrieve_skv(*args)
+        assert skip.skip_sync_status(c) == skip.SKIP_ETIMEOUT
+        assert skip.skip_sync_status(c) == skip.SKIP_OK
+        c.set_option(skip.SKIP_OPT_WAIT_TIMEOUT_NS, 2_000_000_000)
+        g_ids, g_nu, g_cnt, m_ids, _ = skip.skip_retrieve_skv(*args, with_merged=True)
+        ids_all = skip.skip_skv_gate(c, m_ids, t(qbar), t(vbar), t(w1), t(b1.float()), t(w2.float()), b2,
+                                     with_nu_all=True)
+        assert skip.skip_sync_status(c) == skip.SKIP_OK
+        for a, b in zip((g_ids, g_nu, g_cnt), ids_all[:3]):
+            assert torch.equal(a, b)
+        gpu = [x.cpu().numpy() for x in ids_all]
+        mids = m_ids.cpu()
+    finally:
+        c.free()
+    b = synth.bf16_bits
+    o = oracle.skv(b(ct), mids.numpy(), b(qbar), b(vbar), b(w1), b1.float().numpy(), w2.float().numpy(), b2,
+                   tau=0.5, rho=0.6)
+    check_gate(gpu, o, mids, 0.5, 0.6)
