@@ -11,13 +11,15 @@
 //                copy of W_v^T [d x d_k] (k_transpose_bf16, once per handle),
 //                K split over up to four CTAs per tile (partial slabs).
 //  k_qvs_logits  u = the slabs' sum + w_b in shared memory, c by all warps;
-//                one warp per eight tokens at a time, 16-byte loads.
+//                one warp per eight tokens, each token's row requested whole
+//                (2 KB at a time, 16-byte loads), two tokens per round.
 //  k_qvs_rank    rank of every token = the number of the image's keys
 //                (logit, ~index) above its own, counted against all the
 //                image's keys in shared memory (many blocks per image, a warp
-//                per four tokens); a token with rank < n is written at its
+//                per eight tokens); a token with rank < n is written at its
 //                rank with its sigmoid score, and (optionally) its row copied
-//                out by the same warp.  The same order as a descending sort.
+//                out: the block's kept rows spread over all its warps, two
+//                rows in flight a warp.  The same order as a descending sort.
 // The logits and rank kernels are programmatic dependents of the kernel
 // before them: they launch while it drains and wait for its results.
 #include <cuda_bf16.h>
@@ -76,32 +78,46 @@ __global__ void __launch_bounds__(kLogThreads, 4) k_qvs_logits(const QvsParams p
 #pragma unroll
     for (int w = 0; w < kLogThreads / 32; ++w) cb += cpart[w];
     cb *= rsqrtf((float)p.dk);
-    // kLogTok tokens per warp at a time: their loads are issued together.
+    // kLogTok tokens per warp; each token's row is requested whole (2 KB at a
+    // time: four 16-byte words a lane), two tokens per round.
     constexpr int kT = kLogTok;
     const int wstep = gridDim.x * (kLogThreads / 32);
+    const float4 *us4 = reinterpret_cast<const float4 *>(us);
+    const uint4 *tok = reinterpret_cast<const uint4 *>(p.tokens);
     for (int i0 = blockIdx.x * (kLogThreads / 32) + warp; i0 < p.L; i0 += kT * wstep) {
         float s[kT];
 #pragma unroll
         for (int t = 0; t < kT; ++t) s[t] = 0.f;
-        for (int w = lane; w < nw; w += 32) {
-            uint4 x[kT];
+        for (int c0 = 0; c0 < nw; c0 += 128) {
 #pragma unroll
-            for (int t = 0; t < kT; ++t) {
-                const int i = i0 + t * wstep;
-                x[t] = i < p.L ? __ldg(reinterpret_cast<const uint4 *>(p.tokens) + ((int64_t)b * p.L + i) * nw + w)
-                               : make_uint4(0, 0, 0, 0);
-            }
-            float uu[8];
+            for (int t0 = 0; t0 < kT; t0 += 2) {
+                uint4 x[2][4];
 #pragma unroll
-            for (int e = 0; e < 8; ++e) uu[e] = us[w * 8 + e];
+                for (int tt = 0; tt < 2; ++tt) {
+                    const int i = i0 + (t0 + tt) * wstep;
 #pragma unroll
-            for (int t = 0; t < kT; ++t) {
-                const uint32_t xv[4] = {x[t].x, x[t].y, x[t].z, x[t].w};
+                    for (int j = 0; j < 4; ++j) {
+                        const int w = c0 + lane + 32 * j;
+                        x[tt][j] = (i < p.L && w < nw) ? __ldg(tok + ((int64_t)b * p.L + i) * nw + w)
+                                                       : make_uint4(0, 0, 0, 0);
+                    }
+                }
 #pragma unroll
-                for (int h = 0; h < 4; ++h) {
-                    const float2 f = __bfloat1622float2(*reinterpret_cast<const __nv_bfloat162 *>(&xv[h]));
-                    s[t] = fmaf(f.x, uu[2 * h], s[t]);
-                    s[t] = fmaf(f.y, uu[2 * h + 1], s[t]);
+                for (int j = 0; j < 4; ++j) {
+                    const int w = c0 + lane + 32 * j;
+                    if (w >= nw) break;
+                    const float4 ua = us4[2 * w], ub = us4[2 * w + 1];
+                    const float uu[8] = {ua.x, ua.y, ua.z, ua.w, ub.x, ub.y, ub.z, ub.w};
+#pragma unroll
+                    for (int tt = 0; tt < 2; ++tt) {
+                        const uint32_t xv[4] = {x[tt][j].x, x[tt][j].y, x[tt][j].z, x[tt][j].w};
+#pragma unroll
+                        for (int h = 0; h < 4; ++h) {
+                            const float2 f = __bfloat1622float2(*reinterpret_cast<const __nv_bfloat162 *>(&xv[h]));
+                            s[t0 + tt] = fmaf(f.x, uu[2 * h], s[t0 + tt]);
+                            s[t0 + tt] = fmaf(f.y, uu[2 * h + 1], s[t0 + tt]);
+                        }
+                    }
                 }
             }
         }
@@ -120,55 +136,72 @@ constexpr int kRankTok = 8;  // tokens per warp (576 blocks for 64 images: one w
 
 __global__ void __launch_bounds__(32 * kRankWarps) k_qvs_rank(const QvsParams p) {
     extern __shared__ uint64_t keys[];  // [L]: (ord(logit), ~index) of every token of the image
+    __shared__ int2 kept[kRankWarps * kRankTok];  // (token, rank) of this block's kept tokens
+    __shared__ int nkept;
     const int b = blockIdx.y;
     const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+    if (threadIdx.x == 0) nkept = 0;
     grid_dep_wait();
     const float *lg = p.logits + (int64_t)b * p.L;
     for (int i = threadIdx.x; i < p.L; i += 32 * kRankWarps)
         keys[i] = ((uint64_t)ord_of_score(lg[i]) << 32) | (uint32_t)(0xFFFFFFFFu - i);
     __syncthreads();
     const int i0 = (blockIdx.x * kRankWarps + warp) * kRankTok;
-    if (i0 >= p.L) return;
-    uint64_t mine[kRankTok];
-    int cnt[kRankTok];
+    if (i0 < p.L) {
+        uint64_t mine[kRankTok];
+        int cnt[kRankTok];
 #pragma unroll
-    for (int t = 0; t < kRankTok; ++t) {
-        mine[t] = i0 + t < p.L ? keys[i0 + t] : ~0ull;  // past L: rank 0 of nothing, never written
-        cnt[t] = 0;
-    }
-    // Keys are distinct (the index is in the low word), so a token's rank is
-    // its position in the descending order.
-    for (int j = lane; j < p.L; j += 32) {
-        const uint64_t kj = keys[j];
-#pragma unroll
-        for (int t = 0; t < kRankTok; ++t) cnt[t] += kj > mine[t] ? 1 : 0;
-    }
-#pragma unroll
-    for (int t = 0; t < kRankTok; ++t) cnt[t] = __reduce_add_sync(0xFFFFFFFFu, cnt[t]);
-    const int nw = p.d / 8;  // 16-byte words per token
-#pragma unroll
-    for (int t = 0; t < kRankTok; ++t) {
-        const int i = i0 + t, r = cnt[t];
-        if (i >= p.L || r >= p.n) continue;  // warp-uniform
-        if (lane == 0) {
-            p.out_idx[(int64_t)b * p.n + r] = i;
-            p.out_score[(int64_t)b * p.n + r] = 1.f / (1.f + expf(-score_of_ord((uint32_t)(mine[t] >> 32))));
+        for (int t = 0; t < kRankTok; ++t) {
+            mine[t] = i0 + t < p.L ? keys[i0 + t] : ~0ull;  // past L: rank 0 of nothing, never written
+            cnt[t] = 0;
         }
-        if (p.out_tokens) {
-            const uint4 *src = reinterpret_cast<const uint4 *>(p.tokens) + ((int64_t)b * p.L + i) * nw;
-            uint4 *dst = reinterpret_cast<uint4 *>(p.out_tokens) + ((int64_t)b * p.n + r) * nw;
-            // four 16-byte words per lane in flight
-            for (int w0 = 0; w0 < nw; w0 += 128) {
-                uint4 x[4];
+        // Keys are distinct (the index is in the low word), so a token's rank
+        // is its position in the descending order.
+        for (int j = lane; j < p.L; j += 32) {
+            const uint64_t kj = keys[j];
 #pragma unroll
-                for (int u = 0; u < 4; ++u) {
-                    const int w = w0 + lane + 32 * u;
-                    if (w < nw) x[u] = __ldg(src + w);
+            for (int t = 0; t < kRankTok; ++t) cnt[t] += kj > mine[t] ? 1 : 0;
+        }
+#pragma unroll
+        for (int t = 0; t < kRankTok; ++t) cnt[t] = __reduce_add_sync(0xFFFFFFFFu, cnt[t]);
+#pragma unroll
+        for (int t = 0; t < kRankTok; ++t) {
+            const int i = i0 + t, r = cnt[t];
+            if (i >= p.L || r >= p.n) continue;  // warp-uniform
+            if (lane == 0) {
+                p.out_idx[(int64_t)b * p.n + r] = i;
+                p.out_score[(int64_t)b * p.n + r] = 1.f / (1.f + expf(-score_of_ord((uint32_t)(mine[t] >> 32))));
+                if (p.out_tokens) kept[atomicAdd(&nkept, 1)] = make_int2(i, r);
+            }
+        }
+    }
+    if (!p.out_tokens) return;
+    __syncthreads();
+    // The kept rows, spread over all the block's warps, two rows in flight a
+    // warp (a row is four 16-byte words a lane at a time).
+    const int nw = p.d / 8;  // 16-byte words per token
+    const uint4 *src0 = reinterpret_cast<const uint4 *>(p.tokens) + (int64_t)b * p.L * nw;
+    uint4 *dst0 = reinterpret_cast<uint4 *>(p.out_tokens) + (int64_t)b * p.n * nw;
+    const int m = nkept;
+    for (int e = 2 * warp; e < m; e += 2 * kRankWarps) {
+        const int2 a = kept[e];
+        const int2 c = e + 1 < m ? kept[e + 1] : make_int2(-1, -1);
+        for (int w0 = 0; w0 < nw; w0 += 128) {
+            uint4 x[2][4];
+#pragma unroll
+            for (int u = 0; u < 4; ++u) {
+                const int w = w0 + lane + 32 * u;
+                if (w < nw) {
+                    x[0][u] = __ldg(src0 + (int64_t)a.x * nw + w);
+                    if (c.x >= 0) x[1][u] = __ldg(src0 + (int64_t)c.x * nw + w);
                 }
+            }
 #pragma unroll
-                for (int u = 0; u < 4; ++u) {
-                    const int w = w0 + lane + 32 * u;
-                    if (w < nw) dst[w] = x[u];
+            for (int u = 0; u < 4; ++u) {
+                const int w = w0 + lane + 32 * u;
+                if (w < nw) {
+                    dst0[(int64_t)a.y * nw + w] = x[0][u];
+                    if (c.x >= 0) dst0[(int64_t)c.y * nw + w] = x[1][u];
                 }
             }
         }
