@@ -194,6 +194,11 @@ __global__ void __launch_bounds__(kThreads, 1)
     tc_fence_after();
     const uint32_t tmem = sh->tmem_base;
     const int items = p.G;
+    // The merge after this kernel may launch now (it waits for the lists
+    // itself), and the next call's thresholds start from zero: this kernel
+    // clears them (the next call's kernel starts after this one completes).
+    grid_dep_launch();
+    if (blockIdx.x == 0 && threadIdx.x < kLatMaxR) p.tau_clear[threadIdx.x] = 0u;
 
     if (warp == 0) {
         // ------------------------------------------------ TMA producer

@@ -136,6 +136,10 @@ struct skip_corpus {
     cudaEvent_t ev_fork = nullptr, ev_join = nullptr;
     int *cq_flag = nullptr;  // device: epoch of the last completed bias GEMM on aux
     int cq_epoch = 0;
+    // Small-batch kernel thresholds, two sets of kLatMaxR: a call uses one
+    // and its kernel clears the other for the next call (no clearing launch).
+    uint32_t *lat_tau = nullptr;
+    int lat_parity = 0;
 };
 
 namespace {
@@ -325,20 +329,26 @@ skip_status_t run_regions(skip_corpus *c, const uint16_t *regions, int R, int k,
         pl.R_pad = R;
         pl.stages = lat_stages;
         pl.list_in_smem = true;
-        const size_t tau_bytes = align_up((size_t)R * sizeof(uint32_t), 256);
         const size_t parts_bytes = e4m3 ? align_up((size_t)96 * c->d, 256) : 0;
         const size_t qs_bytes = e4m3 ? align_up((size_t)3 * R * sizeof(float), 256) : 0;
         const size_t lists_bytes = (size_t)pl.G * R * k * sizeof(uint64_t);
-        skip_status_t st =
-            ensure_ws(c, align_up(ws_extra, 256) + tau_bytes + parts_bytes + qs_bytes + lists_bytes);
+        skip_status_t st = ensure_ws(c, align_up(ws_extra, 256) + parts_bytes + qs_bytes + lists_bytes);
         if (st) return st;
+        if (!c->lat_tau) {
+            if (dev_alloc(reinterpret_cast<void **>(&c->lat_tau), 2 * kLatMaxR * sizeof(uint32_t), "workspace") !=
+                cudaSuccess) {
+                cudaGetLastError();
+                c->lat_tau = nullptr;
+                return SKIP_ENOMEM;
+            }
+            if (cudaMemsetAsync(c->lat_tau, 0, 2 * kLatMaxR * sizeof(uint32_t), s) != cudaSuccess) return SKIP_ECUDA;
+        }
         char *w = (char *)c->ws + align_up(ws_extra, 256);
-        uint32_t *tau = reinterpret_cast<uint32_t *>(w);
-        uint8_t *parts = reinterpret_cast<uint8_t *>(w + tau_bytes);
-        float *qscale = reinterpret_cast<float *>(w + tau_bytes + parts_bytes);
-        uint64_t *lists = reinterpret_cast<uint64_t *>(w + tau_bytes + parts_bytes + qs_bytes);
+        uint32_t *tau = c->lat_tau + c->lat_parity * kLatMaxR;
+        uint8_t *parts = reinterpret_cast<uint8_t *>(w);
+        float *qscale = reinterpret_cast<float *>(w + parts_bytes);
+        uint64_t *lists = reinterpret_cast<uint64_t *>(w + parts_bytes + qs_bytes);
         if (keys_out) *keys_out = reg_keys = reinterpret_cast<uint64_t *>(c->ws);
-        if (cudaMemsetAsync(tau, 0, tau_bytes, s) != cudaSuccess) return SKIP_ECUDA;
         CUtensorMap ta, tb;
         if (e4m3) {
             record(c, s, "split_queries");
@@ -365,11 +375,13 @@ skip_status_t run_regions(skip_corpus *c, const uint16_t *regions, int R, int k,
         p.qscale = qscale;
         p.lists = lists;
         p.tau = tau;
+        p.tau_clear = c->lat_tau + (1 - c->lat_parity) * kLatMaxR;
         p.err = c->err;
         p.timeout_ns = c->timeout_ns;
         record(c, s, e4m3 ? "score_topk_latency_e4m3" : "score_topk_latency");
         cudaError_t e = launch_latency(e4m3, ta, tb, p, pl.grid, s);
         if (e != cudaSuccess) return cuda_status(e);
+        c->lat_parity ^= 1;
         ++pl.launches;
         if (qm && qm->after_score) {
             const skip_status_t hs = qm->after_score();
@@ -975,6 +987,7 @@ skip_status_t skip_corpus_free(skip_corpus_t c) {
     if (c->ev_join) cudaEventDestroy(c->ev_join);
     if (c->aux) cudaStreamDestroy(c->aux);
     cudaFree(c->cq_flag);
+    cudaFree(c->lat_tau);
     delete c;
     return SKIP_OK;
 }

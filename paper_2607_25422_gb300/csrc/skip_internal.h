@@ -102,7 +102,8 @@ struct LatParams {
     const float *corpus_scale;  // [N] (e4m3)
     const float *qscale;        // [3][R] scales of the query parts (e4m3)
     uint64_t *lists;          // [G][R][k]
-    uint32_t *tau;            // [R] shared thresholds, zeroed
+    uint32_t *tau;            // [R] shared thresholds, zero at launch
+    uint32_t *tau_clear;      // [kLatMaxR] the next call's thresholds, cleared by this kernel
     int *err;
     uint64_t timeout_ns;
 };
