@@ -62,11 +62,14 @@ typedef struct {
  *  nu_all     optional (NULL) device fp32 [num_questions x K]: nu of every
  *             input slot (-inf for empty ones).
  * Uses the handle's gate workspace (grown on demand, which synchronises the
- * device once).  Asynchronous on `stream`: the per-question half of the
- * first layer (which needs no candidate) runs on a second stream of the
- * handle, forked from `stream` after the work queued on it so far and
- * joined back before the gate reads it, so the call stays ordered on
- * `stream` as a whole (and can be captured into a CUDA graph).
+ * device once).  Asynchronous on `stream`.  In skip_retrieve_skv the
+ * per-question half of the first layer (which needs no candidate) runs on a
+ * second stream of the handle, forked from `stream` once the retrieval's
+ * score kernel is queued.  A flag in device memory tells the gate's MLP
+ * kernel when that half is ready (a bounded wait), and the second stream is
+ * joined back into `stream` after the gate's last kernel.  The call thus
+ * stays ordered on `stream` as a whole, and can be captured into a CUDA
+ * graph.
  * qbar, vbar and the mlp's w1 must start on 16-byte boundaries.
  * Errors: SKIP_EINVAL (null or misaligned pointers, K < 1 or > SKIP_MAX_K,
  * bad hidden, tau or rho), SKIP_EUNSUPPORTED (e4m3 corpus, d % 64 != 0,

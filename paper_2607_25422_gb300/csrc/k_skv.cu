@@ -4,7 +4,8 @@
 //  (k_gemm)      per question: c_q = b1 + W1[:, qbar] qbar + W1[:, vbar] vbar
 //                for all questions at once, on the tensor cores (k_gemm.cu);
 //                it needs no retrieval result and runs beside it on a second
-//                stream.
+//                stream, after which k_skv_cq_ready raises a per-call flag
+//                that the MLP kernel waits for before it reads c_q.
 //  k_skv_features per passage slot: F = [e | bf16(e * qbar) | bf16(|e - qbar|)]
 //                (3d bf16 in the column order of W1's passage blocks), from
 //                the gathered corpus row and qbar; zeros for an empty slot.
