@@ -270,8 +270,9 @@ __global__ void __launch_bounds__(kSelThreads) k_skv_select(const SkvParams p) {
 // half r & 1 of a CTA pair (its 128 slots, and half of the W1 rows it
 // stages) over the K part r >> 1 of the 3d feature columns (S = 1 or 2).
 // With S = 2 the two K parts' sums are added through distributed shared
-// memory: each CTA stores the column half its partner finishes into the
-// partner's (free) ring and finishes the other half itself.  Each epilogue
+// memory: each CTA stages the column half its partner finishes, sends it
+// by bulk copies into the partner's (free) ring and finishes the other half
+// itself.  Each epilogue
 // warp writes one partial logit per slot over its columns: slab
 // ((hidden block * S + part) * 2 + half of the columns).
 template <int BN, int S>
@@ -308,7 +309,7 @@ __global__ void __launch_bounds__(kSkvThreads, 1)
         mbar_init(smem_addr(&sh->tfull), 1);
         mbar_init(smem_addr(&sh->recv), 1);
         mbar_fence_init();
-        // the partner's half arrives by one bulk copy
+        // the partner's half arrives by kSkvPieces bulk copies, counted in bytes
         if (S == 2) mbar_arrive_expect_tx(smem_addr(&sh->recv), (uint32_t)(kSkvRows * G::kStgStride));
     }
     if (warp == 0 && lane == 0) {
