@@ -15,7 +15,8 @@
 //                feature rows and the matching W1 rows) into a ring of
 //                stages; with few slots the feature columns are split over
 //                two pairs of a cluster of four and the two sums added
-//                through distributed shared memory; the epilogue adds c_q,
+//                through distributed shared memory (bulk copies of 32-column
+//                chunks into a receive area); the epilogue adds c_q,
 //                applies ReLU and the w2 dot over its units and writes one
 //                partial logit per slot.  (Building the features in shared
 //                memory inside this kernel instead, once per hidden block,
@@ -38,39 +39,53 @@ namespace {
 
 constexpr int kSkvRows = 128;                // passage slots per CTA (TMEM lanes); a pair has 256
 constexpr int kSkvSliceA = kSkvRows * 128;   // one [128 x 64] bf16 K-slice of the features, bytes
-constexpr int kSkvRing = 192 * 1024;         // operand ring of one CTA, bytes
+constexpr int kSkvSmemMax = 227 * 1024;      // opt-in shared memory of a CTA, bytes
 constexpr int kSkvMaxStages = 8;
 constexpr int kSkvEpiWarps = 8;             // two per TMEM lane quarter, each on half the columns
 constexpr int kSkvThreads = 64 + 32 * kSkvEpiWarps;  // TMA warp, MMA warp, epilogue warps
 constexpr uint64_t kDrainTimeoutNs = 1000000000ull;  // 1 s for copies in flight
 constexpr int kFeatWarps = 8;                // slots per feature block
 
+// Epilogue operands staged during the main loop, after the ring: w2 of this
+// CTA's columns, then c_q of its questions and columns (when they fit).
+constexpr int kSkvEpiBytes = 17 * 1024;
+constexpr int kSkvCqCap = (kSkvEpiBytes - 256 * 4) / 4;  // c_q floats
+constexpr int kSkvChunk = kSkvRows * 128;                // 32 fp32 sums of 128 rows, bytes
+
 // A CTA pair computes 256 slots x BN hidden units (tcgen05 cta_group::2,
 // M = 256, N = BN): each CTA stages its own 128 feature rows and half of the
 // W1 block (BN / 2 rows) per K-slice, and its TMEM holds its 128 rows x BN.
-template <int BN>
+// With the K split (S = 2) a receive area after the epilogue operands holds
+// the partner's sums for this CTA's column half, in chunks of 32 columns.
+// Shared memory: ring | barriers (1 KB) | w2, c_q | receive area.
+template <int BN, int S>
 struct SkvGeom {
     static constexpr int kB = (BN / 2) * 128;              // this CTA's W1 rows of one K-slice, bytes
     static constexpr int kStage = kSkvSliceA + kB;
-    static constexpr int kStages = kSkvRing / kStage < kSkvMaxStages ? kSkvRing / kStage : kSkvMaxStages;
+    static constexpr int kChunks = BN / 64;                // chunks of 32 columns in a column half
+    static constexpr int kRecv = S == 2 ? kChunks * kSkvChunk : 0;
+    static constexpr int kRingMax = kSkvSmemMax - 2 * 1024 - kSkvEpiBytes - kRecv;
+    static constexpr int kStages = kRingMax / kStage < kSkvMaxStages ? kRingMax / kStage : kSkvMaxStages;
+    static constexpr int kRing = kStages * kStage;
+    static constexpr int kSmem = 1024 + kRing + 1024 + kSkvEpiBytes + kRecv;
     static constexpr uint32_t kIdesc = idesc_bf16_f32(2 * kSkvRows, BN);
-    static constexpr int kStgStride = (BN / 2) * 4 + 16;   // one staged half row of sums, bytes
+    static_assert(kStages >= 4 && kSmem <= kSkvSmemMax, "ring of at least four stages");
+    static_assert(kChunks * kSkvChunk <= kRing, "the outgoing half is staged in the ring");
 };
 
 struct SkvShared {
     uint64_t full[kSkvMaxStages];   // A and B slices of both CTAs landed (MMA CTA; tx bytes)
     uint64_t empty[kSkvMaxStages];  // stage consumed (commit, to both CTAs of the pair)
     uint64_t tfull;                 // accumulator complete (commit, to both CTAs)
-    uint64_t recv;                  // the partner's half of the sums landed (K split; tx bytes)
+    uint64_t recv[4];               // chunk c of the partner's sums landed (K split; tx bytes)
     uint32_t tmem_base;
 };
-
-// Epilogue operands staged during the main loop, after the ring: w2 of this
-// CTA's columns, then c_q of its questions and columns (when they fit).
 static_assert(sizeof(SkvShared) <= 1024, "barriers fit their 1 KB");
-constexpr int kSkvPieces = 8;  // bulk copies of the K-split exchange
-constexpr int kSkvEpiBytes = 33 * 1024;
-constexpr int kSkvCqCap = (kSkvEpiBytes - 256 * 4) / 4;  // c_q floats
+
+// Byte offset of sum (row r, 16-byte group j of 8) within a chunk: rows 128
+// bytes apart, the groups of a row permuted by r mod 8 so that a warp's 32
+// rows hit distinct banks.
+__device__ __forceinline__ int chunk_off(int r, int j) { return r * 128 + ((j ^ (r & 7)) << 4); }
 
 // Bulk copy of `bytes` (a multiple of 16) from this CTA's shared memory to
 // that of a CTA of the cluster, counted in bytes on its barrier `bar`.
@@ -270,20 +285,22 @@ __global__ void __launch_bounds__(kSelThreads) k_skv_select(const SkvParams p) {
 // half r & 1 of a CTA pair (its 128 slots, and half of the W1 rows it
 // stages) over the K part r >> 1 of the 3d feature columns (S = 1 or 2).
 // With S = 2 the two K parts' sums are added through distributed shared
-// memory: each CTA stages the column half its partner finishes, sends it
-// by bulk copies into the partner's (free) ring and finishes the other half
-// itself.  Each epilogue
+// memory: each CTA stages the column half its partner finishes, 32 columns
+// at a time, and sends each chunk by a bulk copy into the partner's receive
+// area as soon as it is staged; it finishes the other half itself, chunk by
+// chunk as the partner's copies land.  Each epilogue
 // warp writes one partial logit per slot over its columns: slab
 // ((hidden block * S + part) * 2 + half of the columns).
 template <int BN, int S>
 __global__ void __launch_bounds__(kSkvThreads, 1)
     k_skv_mlp(const __grid_constant__ CUtensorMap tf, const __grid_constant__ CUtensorMap tw, const SkvParams p) {
-    using G = SkvGeom<BN>;
+    using G = SkvGeom<BN, S>;
     extern __shared__ __align__(1024) uint8_t smem_raw[];
     uint8_t *smem = reinterpret_cast<uint8_t *>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
     uint8_t *sA = smem;
     uint8_t *sB = smem + G::kStages * kSkvSliceA;
-    SkvShared *sh = reinterpret_cast<SkvShared *>(sB + G::kStages * G::kB);
+    SkvShared *sh = reinterpret_cast<SkvShared *>(smem + G::kRing);
+    uint8_t *recv = smem + G::kRing + 1024 + kSkvEpiBytes;  // the partner's sums (S = 2)
     const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
     const uint32_t rank = cluster_rank();
     const int half = (int)(rank & 1u), part = (int)(rank >> 1);
@@ -307,10 +324,11 @@ __global__ void __launch_bounds__(kSkvThreads, 1)
             mbar_init(smem_addr(&sh->empty[s]), 1);
         }
         mbar_init(smem_addr(&sh->tfull), 1);
-        mbar_init(smem_addr(&sh->recv), 1);
+        for (int c = 0; c < G::kChunks; ++c) mbar_init(smem_addr(&sh->recv[c]), 1);
         mbar_fence_init();
-        // the partner's half arrives by kSkvPieces bulk copies, counted in bytes
-        if (S == 2) mbar_arrive_expect_tx(smem_addr(&sh->recv), (uint32_t)(kSkvRows * G::kStgStride));
+        // the partner's half arrives as one bulk copy a chunk, counted in bytes
+        if (S == 2)
+            for (int c = 0; c < G::kChunks; ++c) mbar_arrive_expect_tx(smem_addr(&sh->recv[c]), (uint32_t)kSkvChunk);
     }
     if (warp == 0 && lane == 0) {
         tma_prefetch_desc(&tf);
@@ -442,54 +460,41 @@ __global__ void __launch_bounds__(kSkvThreads, 1)
         if (!done) atomicOr(p.err, kErrTimeout);
         tc_fence_after();
     }
-    // Ring reuse once every MMA that read it has completed: with the K split,
-    // the half of the sums the partner finishes (stg_out) and the half it
-    // sends (stg_in), rows kStgStride bytes apart.
-    uint8_t *stg_out = smem;
-    uint8_t *stg_in = smem + kSkvRows * G::kStgStride;
-    bool got = true;
-    if (S == 2) {
-        if (epi && done) {
-            const int oc = (1 - part) * (BN / 2);
-            uint8_t *row = stg_out + r * G::kStgStride;
+    // With the K split: the half of the sums the partner finishes, staged
+    // chunk by chunk in this CTA's ring (free: its MMAs have completed) by
+    // the four warps of the column half that owns the chunk, and pushed into
+    // the partner's receive area as soon as those four warps are done with it.
+    if (S == 2 && epi) {
+        const int oc = (1 - part) * (BN / 2);
 #pragma unroll 1
-            for (int c = hal * (BN / 128); c < (hal + 1) * (BN / 128); ++c) {
+        for (int c = hal * (G::kChunks / 2); c < (hal + 1) * (G::kChunks / 2); ++c) {
+            if (done) {
                 uint32_t v[32];
                 tmem_ld_32x32b_x32(tmem + lane_addr + (uint32_t)(oc + c * 32), v);
                 tmem_ld_wait(v);
+                uint8_t *ch = smem + c * kSkvChunk;
 #pragma unroll
                 for (int j = 0; j < 8; ++j)
-                    *reinterpret_cast<uint4 *>(row + c * 128 + j * 16) =
+                    *reinterpret_cast<uint4 *>(ch + chunk_off(r, j)) =
                         make_uint4(v[4 * j], v[4 * j + 1], v[4 * j + 2], v[4 * j + 3]);
+                fence_proxy_async_smem();
             }
-            fence_proxy_async_smem();
-        }
-        // every MMA of the cluster has completed (the rings are free) and
-        // every CTA's outgoing half is staged
-        cluster_sync_all();
-        if (warp == 2 && lane < kSkvPieces && done) {
-            // in pieces of kSkvRows / kSkvPieces rows, one per lane
-            const uint32_t peer = rank ^ 2u;
-            const uint32_t off = (uint32_t)(lane * (kSkvRows / kSkvPieces) * G::kStgStride);
-            bulk_copy_to_peer(mapa_shared(smem_addr(stg_in) + off, peer), smem_addr(stg_out) + off,
-                              (uint32_t)((kSkvRows / kSkvPieces) * G::kStgStride),
-                              mapa_shared(smem_addr(&sh->recv), peer));
-        }
-        if (epi) {
-            // a copy in flight writes into this CTA's shared memory: wait for
-            // it at least as long as for any other copy before giving up
-            got = mbar_wait(smem_addr(&sh->recv), 0, p.timeout_ns > kDrainTimeoutNs ? p.timeout_ns : kDrainTimeoutNs);
-            if (!got && r == 0) atomicOr(p.err, kErrTimeout);
+            asm volatile("bar.sync %0, %1;" ::"r"(2 + hal), "r"(kSkvRows) : "memory");  // this half's warps
+            if (sub == 0 && lane == 0 && done) {
+                const uint32_t peer = rank ^ 2u;
+                bulk_copy_to_peer(mapa_shared(smem_addr(recv) + c * kSkvChunk, peer), smem_addr(smem) + c * kSkvChunk,
+                                  (uint32_t)kSkvChunk, mapa_shared(smem_addr(&sh->recv[c]), peer));
+            }
         }
     }
-    if (epi && done && got) {
+    if (epi && done) {
         const int64_t slot = m0 + r;
         // rows past the last slot read the first staged question and write nothing
         const int qq = slot < p.P ? (int)(slot / p.K) - q0 : 0;
         const int qc = qq < 0 ? 0 : qq >= nq ? (nq > 0 ? nq - 1 : 0) : qq;
         const float *cq = cqs + qc * ncol;
         const float *cqg = p.cq + (int64_t)(q0 + qc) * p.H + n0 + c0;
-        const uint8_t *in = stg_in + r * G::kStgStride;
+        bool got = true;
         // four partial sums of the w2 dot (any order is within the bound)
         float a0 = 0.f, a1 = 0.f, a2 = 0.f, a3 = 0.f;
         // the loop in two forms, so that no branch splits its body: c_q
@@ -499,6 +504,16 @@ __global__ void __launch_bounds__(kSkvThreads, 1)
             constexpr bool kStaged = decltype(staged)::value;
 #pragma unroll 1
             for (int c = hal * (ncol / 64); c < (hal + 1) * (ncol / 64); ++c) {
+                if (S == 2) {
+                    // the partner's chunk c: a copy in flight writes into this
+                    // CTA's shared memory, so wait for it at least as long as
+                    // for any other copy before giving up
+                    if (!mbar_wait(smem_addr(&sh->recv[c]), 0,
+                                   p.timeout_ns > kDrainTimeoutNs ? p.timeout_ns : kDrainTimeoutNs)) {
+                        got = false;
+                        break;
+                    }
+                }
                 uint32_t v[32];
                 tmem_ld_32x32b_x32(tmem + lane_addr + (uint32_t)(c0 + c * 32), v);
                 tmem_ld_wait(v);
@@ -510,7 +525,7 @@ __global__ void __launch_bounds__(kSkvThreads, 1)
                     float4 h = make_float4(__uint_as_float(v[4 * g]), __uint_as_float(v[4 * g + 1]),
                                            __uint_as_float(v[4 * g + 2]), __uint_as_float(v[4 * g + 3]));
                     if constexpr (S == 2) {
-                        const float4 o = *reinterpret_cast<const float4 *>(in + col * 4);
+                        const float4 o = *reinterpret_cast<const float4 *>(recv + c * kSkvChunk + chunk_off(r, g));
                         h.x += o.x, h.y += o.y, h.z += o.z, h.w += o.w;
                     }
                     if constexpr (kStaged) {
@@ -534,8 +549,9 @@ __global__ void __launch_bounds__(kSkvThreads, 1)
             run(std::true_type{});
         else
             run(std::false_type{});
+        if (!got && lane == 0) atomicOr(p.err, kErrTimeout);
         const float acc = (a0 + a1) + (a2 + a3);
-        if (slot < p.P) p.partial[(int64_t)((ct * S + part) * 2 + hal) * p.P + slot] = acc;
+        if (got && slot < p.P) p.partial[(int64_t)((ct * S + part) * 2 + hal) * p.P + slot] = acc;
     }
 
     tc_fence_before();
@@ -556,14 +572,15 @@ __global__ void __launch_bounds__(kSkvThreads, 1)
 // completed.
 __global__ void k_skv_cq_ready(int *flag, int epoch) { st_release_gpu(flag, epoch); }
 
-size_t skv_mlp_smem_bytes() {
-    return 1024 + (size_t)kSkvRing + 1024 + kSkvEpiBytes;
+size_t skv_mlp_smem_bytes(int BN, int S) {
+    return BN == 256 ? (S == 2 ? SkvGeom<256, 2>::kSmem : SkvGeom<256, 1>::kSmem)
+                     : (S == 2 ? SkvGeom<128, 2>::kSmem : SkvGeom<128, 1>::kSmem);
 }
 
 template <int BN>
 int skv_max_clusters(int CL) {
     auto kern = k_skv_mlp<BN, 2>;
-    const size_t smem = skv_mlp_smem_bytes();
+    const size_t smem = skv_mlp_smem_bytes(BN, 2);
     if (cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem) != cudaSuccess) {
         cudaGetLastError();
         return 0;
@@ -627,7 +644,7 @@ cudaError_t launch_skv_mlp(const CUtensorMap &tf, const CUtensorMap &tw, const S
     if (p.Q == 0) return cudaSuccess;
     if ((BN != 128 && BN != 256) || (S != 1 && S != 2) || p.H % BN != 0 || p.nparts != p.H / BN * S * 2)
         return cudaErrorInvalidValue;
-    const size_t smem = skv_mlp_smem_bytes();
+    const size_t smem = skv_mlp_smem_bytes(BN, S);
     auto kern = BN == 256 ? (S == 2 ? k_skv_mlp<256, 2> : k_skv_mlp<256, 1>)
                           : (S == 2 ? k_skv_mlp<128, 2> : k_skv_mlp<128, 1>);
     cudaError_t e = cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);

@@ -196,7 +196,7 @@ struct SkvParams {
     int *err;
     uint64_t timeout_ns;
 };
-size_t skv_mlp_smem_bytes();
+size_t skv_mlp_smem_bytes(int BN, int S);  // dynamic shared memory of k_skv_mlp
 // Tile shape of the gate MLP for P slots and H hidden units: BN hidden units
 // per CTA pair (128 or 256) and S K parts (1 or 2; clusters of 2 S CTAs).
 void skv_mlp_shape(int64_t P, int H, int *BN, int *S);
