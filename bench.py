@@ -843,7 +843,10 @@ def main():
                 "entry_point": ("skip_ivfpq_search with pinned host copies in and out" if args.ivfpq else
                                 "skip_retrieve_skv with pinned host copies in and out" if args.skv
                                 else "skip_retrieve_host (pinned host buffers)")},
-        "gpu_launches": int(sum(v["launches"] for v in kernels.values())),
+        # kernels counted in the events pass; without events the SKV gate's
+        # bias GEMM runs on a second stream followed by its one-thread ready
+        # flag kernel, one more launch a step
+        "gpu_launches": int(sum(v["launches"] for v in kernels.values())) + (args.steps if args.skv else 0),
         "kernels": kernels,
         "plan": plan,
         "dedup_rate": None if args.ivfpq else dedup_rate(skip, c, reg_d, offsets, spec.k_region),

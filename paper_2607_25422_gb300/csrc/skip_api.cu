@@ -897,7 +897,7 @@ skip_status_t skv_impl(skip_corpus *c, const int64_t *cand_ids, int32_t Q, int32
     record(c, s, "skv_select");
     e = launch_skv_select(p, s);
     if (e != cudaSuccess) return cuda_status(e);
-    pl.launches += 4;
+    pl.launches += cl.forked ? 5 : 4;  // the GEMM (and its ready flag), features, MLP, selection
     // the second stream joins s again (its GEMM is long done by now)
     if (cl.forked && cudaStreamWaitEvent(s, c->ev_join, 0) != cudaSuccess) return SKIP_ECUDA;
     return SKIP_OK;
